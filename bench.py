@@ -1,0 +1,349 @@
+#!/usr/bin/env python3
+"""Benchmark of the eager multi-resolution substrate-discovery hot path on GB300.
+
+Metric: CPPN queries/sec = genomes x query slots x N_total(D) / seconds, on the
+1000-genome XOR-shaped population at depth 7 (4 slots: 3 outgoing substrate
+inputs, 1 incoming output), 349.5 M queries per step. A step is one pass of the
+whole path through libemr's C ABI: specialisation (emr_eval_prepare), fused
+evaluation + variance + band filter (emr_eval_filter), mask combination
+(emr_mask_combine) and ordered compaction (emr_compact).
+
+`value` is device time with inputs resident in HBM (CUDA events, L2 flushed
+between steps); `e2e` is the same metric through the host-buffer path: packing
+on the host, pinned H2D copy of the packed genomes and slots, the four calls,
+and the D2H read of the compacted connection lists, all inside the timed region.
+
+--impl reference times the float64 CPU oracle on a bounded sample of the same
+workload (the only other place this script runs the oracle).
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "CPPN queries/sec (genomes x positions) at pop 1000 depth 7"
+UNIT = "queries/s"
+
+# Per-activation algorithmic cost per query (fp32 lane ops, MUFU ops).
+ACT_FP32 = {0: 0, 1: 2, 2: 3, 3: 2, 4: 4, 5: 0}
+ACT_MUFU = {0: 0, 1: 2, 2: 2, 3: 1, 4: 1, 5: 0}
+VAR_OPS, BAND_OPS = 3.25, 8.0
+MUFU_PER_SM_CLK = 16          # nominal MUFU lanes per SM per clock
+FP32_PER_SM_CLK = 128         # FP32 lanes per SM per clock
+SM_MAX_MHZ = 2070.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="emr", choices=["emr", "reference"])
+    ap.add_argument("--depth", type=int, default=7)
+    ap.add_argument("--pop", type=int, default=1000)
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--cpu-genomes", type=int, default=160, help="oracle baseline sample (genomes)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_init():
+    import torch
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return rank, ws, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def allreduce_max(x, ws):
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, index):
+        self.index, self.proc, self.lines = index, None, []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + ",".join(self.FIELDS),
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            p = [x.strip() for x in ln.split(",")]
+            if len(p) < 8:
+                continue
+            try:
+                sm.append(float(p[0])); mx.append(float(p[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, p[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def algorithmic_work(pack, query, emr):
+    """Per pair: fp32 lane ops and MUFU ops per query on the packed DAG (dead
+    nodes removed, constants folded): per varying node its grid-input FMAs,
+    its in-edges from varying nodes and its activation; plus the amortised
+    4-child variance and the band test."""
+    h, gs, nodes, edges = emr.pack_records(pack)
+    per = np.zeros((len(gs), 2, 2))
+    for g in range(len(gs)):
+        nb, n, eb = int(gs["node_beg"][g]), int(gs["n_nodes"][g]), int(gs["edge_beg"][g])
+        for side in (0, 1):
+            gx, gy = (2, 3) if side == 0 else (0, 1)
+            F = M = 0.0
+            for t in range(n):
+                nd = nodes[nb + t]
+                if not (int(nd["vary"]) >> side) & 1:
+                    continue
+                F += float(nd["w_in"][gx] != 0) + float(nd["w_in"][gy] != 0)
+                for e in range(int(nd["edge_cnt"])):
+                    src = int(edges[eb + int(nd["edge_beg"]) + e]["src"])
+                    F += (int(nodes[nb + src]["vary"]) >> side) & 1
+                F += ACT_FP32[int(nd["act"])]
+                M += ACT_MUFU[int(nd["act"])]
+            per[g, side] = (F + VAR_OPS + BAND_OPS, M)
+    side = np.broadcast_to(query.side, (len(gs), query.S))
+    return per[np.arange(len(gs))[:, None], side]  # [P, S, 2]
+
+
+def oracle_baseline(w, genomes):
+    import oracle
+    oracle.build()
+    t0 = time.perf_counter()
+    oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, g0=0, g1=genomes,
+                    fields=("keep_eager",))
+    dt = time.perf_counter() - t0
+    q = genomes * w.S * oracle.n_total(w.D)
+    return {"value": q / dt, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+            "sample": "%d of %d genomes x %d slots at depth %d (%.3g queries + halo), %.2f s"
+                      % (genomes, w.P, w.S, w.D, q, dt)}
+
+
+def run_reference(args):
+    rank, ws, _ = int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), 0
+    if rank != 0:
+        return
+    from paper_2608_27612_gb300 import workloads as W
+    import oracle
+    oracle.build()
+    w = W.c2(D=args.depth, P=args.pop)
+    per_step = 4  # genomes per step: a bounded sample of the workload
+    q = per_step * w.S * oracle.n_total(w.D)
+    ts = []
+    for k in range(args.warmup + args.steps):
+        g0 = (k * per_step) % w.P
+        t0 = time.perf_counter()
+        oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, g0=g0, g1=g0 + per_step,
+                        fields=("keep_eager",))
+        if k >= args.warmup:
+            ts.append(time.perf_counter() - t0)
+    ms = 1e3 * statistics.mean(ts)
+    val = q / (ms / 1e3)
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "genomes": w.P, "slots": w.S, "depth": w.D,
+                   "queries_per_step_full": w.P * w.S * oracle.n_total(w.D), "sample_genomes_per_step": per_step},
+        "cpu_baseline": {"value": val, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+                         "sample": "%d genomes x %d slots per step at depth %d" % (per_step, w.S, w.D)},
+        "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    rank, ws, local = dist_init()
+    torch.cuda.set_device(local)
+    from paper_2608_27612_gb300 import emr
+    from paper_2608_27612_gb300 import workloads as W
+
+    # Each rank runs its own population (independent problems, no collective on the data path).
+    w = W.c2(D=args.depth, P=args.pop)
+    if rank > 0:
+        w.pop = W.random_population(args.pop, seed=2 + 7919 * rank)
+    dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, emr.EMR_EAGER)
+    g = dsc.grid
+    queries = dsc.n_pairs * g.n_total
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(64 << 20, dtype=torch.float32, device="cuda")  # 256 MB > 129 MB L2
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+
+    def step(evs=None):
+        dsc.prepare()
+        if evs:
+            evs[0].record(stream)
+        emr.eval_filter(dsc.pack, dsc.query, g, dsc.theta, dsc.band, dsc.w_min, dsc.split, dsc.band_bits, dsc.out,
+                        dsc.ws)
+        if evs:
+            evs[1].record(stream)
+        emr.mask_combine(dsc.split, dsc.band_bits, g, dsc.n_pairs, dsc.mode, dsc.mask)
+        emr.compact(dsc.mask, dsc.out, g, dsc.n_pairs, dsc.idx, dsc.w, dsc.cap, dsc.counts, dsc.offsets, dsc.cws)
+
+    launches_per_step = 2 + 1 + 1 + 4
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.2)
+    starts, ends, tiles = [ev() for _ in range(args.steps)], [ev() for _ in range(args.steps)], []
+    barrier(ws)
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.zero_()
+        te = (ev(), ev())
+        starts[k].record(stream)
+        step(te)
+        ends[k].record(stream)
+        tiles.append(te)
+    torch.cuda.synchronize()
+    barrier(ws)
+    wall = time.perf_counter() - wall0
+    clocks = sampler.stop()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    tile_ms = [a.elapsed_time(b) for a, b in tiles]
+    ms = allreduce_max(statistics.mean(step_ms), ws)
+    value = ws * queries / (ms / 1e3)
+
+    # roofline of the dominant kernel (fused eval + variance + band)
+    work = algorithmic_work(dsc.pack, dsc.query, emr)   # [P, S, (fp32, mufu)] per query
+    props = torch.cuda.get_device_properties(local)
+    sms = props.multi_processor_count
+    ratio = FP32_PER_SM_CLK / MUFU_PER_SM_CLK
+    per_query_eq = np.maximum(work[..., 0], ratio * work[..., 1])
+    work_eq = float(per_query_eq.sum()) * g.n_total
+    tile_s = statistics.mean(tile_ms) / 1e3
+    peak = sms * FP32_PER_SM_CLK * SM_MAX_MHZ * 1e6
+    achieved = work_eq / tile_s
+    roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": peak / 1e12, "unit": "Tlane-op/s",
+                "frac": achieved / peak, "traffic": None, "kernel": "tile_kernel (emr_eval_filter)",
+                "kernel_ms": tile_s * 1e3,
+                "fp32_ops_per_query": float(work[..., 0].mean()), "mufu_ops_per_query": float(work[..., 1].mean()),
+                "peak_basis": "%d SMs x %d FP32 lanes x %.0f MHz (max SM clock); MUFU weighted %g FP32 lane-ops"
+                              % (sms, FP32_PER_SM_CLK, SM_MAX_MHZ, ratio)}
+    if clocks:
+        roofline["frac_at_sampled_clock"] = roofline["frac"] * SM_MAX_MHZ / clocks["sm_mhz"]
+
+    # end to end through host buffers
+    e2e = None
+    if args.e2e_steps > 0:
+        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+        pop = w.pop
+        a_h, b_h, s_h = pin(dsc.query.a), pin(dsc.query.b), pin(dsc.query.side)
+        pack_pinned = torch.empty(len(dsc.pack) + 4096, dtype=torch.uint8).pin_memory()
+        res_off = torch.empty(dsc.n_pairs + 1, dtype=torch.int64).pin_memory()
+        idx_h = torch.empty(dsc.cap, dtype=torch.int32).pin_memory()
+        w_h = torch.empty(dsc.cap, dtype=torch.float32).pin_memory()
+        times, h2d, d2h = [], 0, 0
+        for k in range(args.e2e_steps + 2):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            blob = emr.pack_population(pop)
+            pack_pinned[:len(blob)].numpy()[:] = blob
+            dsc.pack_dev[:len(blob)].copy_(pack_pinned[:len(blob)], non_blocking=True)
+            dsc.query.a_dev.copy_(a_h, non_blocking=True)
+            dsc.query.b_dev.copy_(b_h, non_blocking=True)
+            dsc.query.side_dev.copy_(s_h, non_blocking=True)
+            dsc.pack = blob
+            step()
+            res_off.copy_(dsc.offsets, non_blocking=True)
+            torch.cuda.synchronize()
+            total = int(res_off[-1])
+            n = min(total, dsc.cap)
+            idx_h[:n].copy_(dsc.idx[:n], non_blocking=True)
+            w_h[:n].copy_(dsc.w[:n], non_blocking=True)
+            torch.cuda.synchronize()
+            if k >= 2:
+                times.append(time.perf_counter() - t0)
+                h2d = len(blob) + 4 * (a_h.numel() + b_h.numel() + s_h.numel())
+                d2h = 8 * (dsc.n_pairs + 1) + 8 * n
+        e2e_s = allreduce_max(statistics.mean(times), ws)
+        e2e = {"value": ws * queries / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": e2e_s * 1e3}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = oracle_baseline(w, min(args.cpu_genomes, w.P))
+
+    kept = int(dsc.offsets[-1])
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": w.name, "genomes": w.P, "slots": w.S, "depth": w.D, "n_total": g.n_total,
+                       "queries_per_step": queries, "theta": w.theta, "band": w.band, "mode": "eager",
+                       "l2": "flushed between steps (256 MB write)", "kept_connections": kept,
+                       "parallelism": "independent populations per GPU" if ws > 1 else "single GPU"},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps, "clocks": clocks,
+            "wall_s_timed_region": wall, "gpu": props.name,
+        }))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

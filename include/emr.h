@@ -1,0 +1,250 @@
+/*
+ * emr.h: C ABI of libemr, a GB300 (sm_103a) implementation of the eager
+ * multi-resolution substrate-discovery hot path of EMR-HyperNEAT
+ * ("Tensor-Accelerated Eager Multi-Resolution Grids for Evolving Large-Scale
+ * Substrates", GECCO Companion '26).
+ *
+ * The method (Section 3): precompute the multi-resolution grid of Eq. 1,
+ * query every genome's CPPN at every grid position (W = vmap(CPPN)(s, T)),
+ * compute each cell's variance bottom-up from its four children, and filter
+ * with the division threshold (Eq. 2) and ES-HyperNEAT's band threshold; the
+ * surviving positions become each genome's connection list.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * Grid (Eq. 1): depth d in [0, D] holds the 4^{d+1} points
+ *   x = (2i+1)/2^{d+1} - 1, y = (2j+1)/2^{d+1} - 1, i, j in [0, 2^{d+1}).
+ * Position numbering: global index = level_off[d] + m, level_off[d] =
+ *   (4^{d+1} - 4)/3, m = Morton code of (i, j) (bit k of i -> bit 2k, bit k of
+ *   j -> bit 2k+1). The children of m at depth d are 4m + a + 2b at depth
+ *   d+1 for child (2i+a, 2j+b). N_total = (4^{D+2} - 4)/3.
+ * Halo: the band test of a depth-d point looks at its 4 neighbours at
+ *   distance 2^-d; those outside [-1,1]^2 are the halo points, numbered
+ *   halo_off[d] + side * 2^{d+1} + t, halo_off[d] = 8 (2^d - 1);
+ *   side 0: (i = -1, j = t), 1: (i = 2^{d+1}, j = t), 2: (i = t, j = -1),
+ *   3: (i = t, j = 2^{d+1}). N_halo = 8 (2^{D+1} - 1).
+ * Bit planes: one bit per position, levels padded to whole 32-bit words:
+ *   position (d, m) is bit (m % 32) of word word_off[d] + m / 32. Bits past
+ *   a level's 4^{d+1} positions (depths 0 and 1) are always 0.
+ * Query slots: a (genome, slot) pair ("pair") evaluates CPPN(a, b, x, y, 1)
+ *   for an outgoing slot (source node at (a, b)) or CPPN(x, y, a, b, 1) for an
+ *   incoming slot (target node at (a, b)) over every grid position; the CPPN
+ *   input order (x1, y1, x2, y2) is the paper's (Section 2), the fifth input
+ *   is the bias, fixed at 1. Pair r = g * S + s.
+ * Filter (Section 3.2, Eq. 2, Theorem 1): V(p) = population variance of the
+ *   CPPN outputs at p's four children (0 at depth D); split(p) = d < D and
+ *   V(p) > theta; B(p) = max(min(|w_p - w_up|, |w_p - w_down|),
+ *   min(|w_p - w_left|, |w_p - w_right|)) (ES-HyperNEAT's band value);
+ *   keep_eager(p) = !split(p) and B(p) > band and (w_min <= 0 or |w_p| > w_min);
+ *   keep_gated(p) = keep_eager(p) and active(p), active per Eq. 2.
+ *
+ * Memory and streams: the caller owns every buffer. Device pointers must be
+ * device memory of the current CUDA device; host pointers are plain host
+ * memory unless a call says "pinned". Calls that take a stream are
+ * asynchronous on it unless stated; errors are returned as status codes and
+ * never thrown; on error no kernel has been launched unless stated.
+ */
+#ifndef EMR_H
+#define EMR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int emr_status;
+#define EMR_OK 0
+#define EMR_ERR_ARG 1      /* bad argument (null pointer, size, enum, malformed genome) */
+#define EMR_ERR_CYCLE 2    /* a genome's enabled connections contain a cycle */
+#define EMR_ERR_RANGE 3    /* a size beyond a documented limit (depth, nodes, edges) */
+#define EMR_ERR_CAPACITY 4 /* an output buffer is too small; true sizes are reported */
+#define EMR_ERR_CUDA 5     /* a CUDA runtime call or launch failed */
+#define EMR_ERR_TIMEOUT 6  /* a host-side wait gave up */
+#define EMR_ERR_ALLOC 7    /* host allocation failed */
+
+#define EMR_MAX_DEPTH 14   /* global indices fit int32 up to depth 14 (N_total(14) = 1.43e9) */
+#define EMR_MAX_VARYING 64 /* per genome and query side: CPPN nodes whose value varies over the grid */
+#define EMR_MAX_VEDGES 512 /* per genome: connections between such nodes */
+
+enum { EMR_ACT_IDENTITY = 0, EMR_ACT_SIGMOID = 1, EMR_ACT_TANH = 2, EMR_ACT_GAUSS = 3,
+       EMR_ACT_SIN = 4, EMR_ACT_ABS = 5 };
+enum { EMR_KIND_X1 = 0, EMR_KIND_Y1 = 1, EMR_KIND_X2 = 2, EMR_KIND_Y2 = 3, EMR_KIND_BIAS = 4,
+       EMR_KIND_HIDDEN = 5, EMR_KIND_OUTPUT = 6 };
+enum { EMR_SIDE_OUT = 0, EMR_SIDE_IN = 1 };
+enum { EMR_EAGER = 0, EMR_GATED = 1 };
+
+/* Grid descriptor (Eq. 1): sizes and offsets only, no positions are stored;
+ * kernels generate coordinates from (depth, Morton index). */
+typedef struct {
+    int32_t D;
+    int32_t reserved;
+    int64_t n_total;                      /* (4^{D+2} - 4) / 3 positions */
+    int64_t n_halo;                       /* 8 (2^{D+1} - 1) halo points */
+    int64_t n_words;                      /* bit-plane words per pair */
+    int64_t chunk;                        /* streaming chunk in positions (0 = none) */
+    int64_t level_off[EMR_MAX_DEPTH + 2]; /* [d] first global index of depth d; [D+1] = n_total */
+    int64_t halo_off[EMR_MAX_DEPTH + 2];  /* [d] first halo index of depth d; [D+1] = n_halo */
+    int64_t word_off[EMR_MAX_DEPTH + 2];  /* [d] first bit-plane word of depth d; [D+1] = n_words */
+} emr_grid;
+
+/* Query slots. Shared by all genomes (per_genome = 0: arrays of S) or one
+ * list per genome (per_genome = 1: arrays of P * S, row g). count (per-genome
+ * mode, optional) gives the number of valid slots of each genome; slots past
+ * it evaluate to the constant 0 and keep nothing. Host and device copies hold
+ * the same values: the host copy schedules work, the device copy is read by
+ * kernels. */
+typedef struct {
+    int32_t S;
+    int32_t per_genome;
+    const float *a_host, *b_host;      /* node coordinates */
+    const int32_t *side_host;          /* EMR_SIDE_OUT / EMR_SIDE_IN */
+    const int32_t *count_host;         /* optional, [P] */
+    const float *a_dev, *b_dev;
+    const int32_t *side_dev;
+    const int32_t *count_dev;          /* optional, [P] */
+} emr_query;
+
+/* ---- a1: grid descriptor ------------------------------------------------ */
+
+/* Fill *grid for maximum depth D (Eq. 1, Section 3.1; Table 1 "grid
+ * construction"). chunk: positions per streaming chunk for emr_stream (0 =
+ * no chunking; otherwise a power of two >= 4096). Host only, no allocation.
+ * Errors: EMR_ERR_ARG (null grid, bad chunk), EMR_ERR_RANGE (D outside [0, 14]). */
+emr_status emr_grid_build(int32_t D, int64_t chunk, emr_grid *grid);
+
+/* Depth d and grid indices (i, j) of global index gidx (inverse of the
+ * numbering above). Returns EMR_ERR_RANGE when gidx is negative or past
+ * depth EMR_MAX_DEPTH. */
+emr_status emr_index_to_ij(int64_t gidx, int32_t *d, int32_t *i, int32_t *j);
+
+/* ---- a2: population packing (host) -------------------------------------- */
+
+/* Bytes emr_pack_population needs for this population (an upper bound). */
+emr_status emr_pack_size(int32_t P, const int64_t *node_ptr, const int64_t *conn_ptr, size_t *bytes);
+
+/* Pack P NEAT genomes (Section 2; the TensorNEAT genomes of Section 5.1) into
+ * one position-independent blob. Genome g owns nodes [node_ptr[g],
+ * node_ptr[g+1]) and connections [conn_ptr[g], conn_ptr[g+1]). Nodes: unique
+ * id, kind (EMR_KIND_*), activation (EMR_ACT_*, hidden and output only) and
+ * bias; exactly one output per genome. Connections: (source id, destination
+ * id, weight, enabled); disabled connections are ignored. A node's value is
+ * act(bias + sum of weight * source value over its enabled in-connections).
+ *
+ * The packer orders each genome topologically (Kahn's algorithm, ties by node
+ * id), drops nodes that cannot reach the output, folds input connections into
+ * per-node input weights and records, per query side, which nodes vary over
+ * the grid. The blob is plain bytes: copy it to device memory unchanged (any
+ * 16-byte aligned address) and pass both copies to the eval calls.
+ * Errors: EMR_ERR_ARG (null pointer, malformed genome: unknown id, duplicate
+ * id, not exactly one output, connection into an input), EMR_ERR_CYCLE,
+ * EMR_ERR_RANGE (more than EMR_MAX_VARYING varying nodes or EMR_MAX_VEDGES
+ * edges between them), EMR_ERR_CAPACITY (cap too small; *used = bytes needed).
+ * *bad_genome (optional) receives the index of the offending genome or -1. */
+emr_status emr_pack_population(int32_t P, const int64_t *node_ptr, const int32_t *node_id,
+                               const int32_t *node_kind, const int32_t *node_act, const float *node_bias,
+                               const int64_t *conn_ptr, const int32_t *conn_src, const int32_t *conn_dst,
+                               const float *conn_w, const uint8_t *conn_enabled, void *buf, size_t cap,
+                               size_t *used, int32_t *bad_genome);
+
+/* Summary of a packed blob: population size and, per query side, the largest
+ * number of varying nodes. Any output pointer may be NULL. */
+emr_status emr_pack_info(const void *pack_host, int32_t *P, int32_t *max_varying_out,
+                         int32_t *max_varying_in);
+
+/* ---- device workspace and per-pair specialisation ------------------------- */
+
+/* Bytes of device workspace the eval calls need for this pack and query
+ * (per-pair specialised CPPN records, scratch and the pair schedule). */
+emr_status emr_eval_workspace_size(const void *pack_host, const emr_query *q, size_t *bytes);
+
+/* Specialise every (genome, slot) pair into ws (Section 3.1: W = CPPN(s, T)
+ * with the slot's node s fixed): the slot's node coordinates and the bias are
+ * folded with every CPPN node that does not vary over the grid into per-node
+ * constants, and the pairs are ordered by estimated cost, heaviest first.
+ * pack_dev: device copy of the blob from emr_pack_population; q: host and
+ * device copies of the slots. Must precede emr_eval / emr_eval_filter with the
+ * same pack and query (stream order). Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY
+ * (ws_bytes too small), EMR_ERR_CUDA. */
+emr_status emr_eval_prepare(const void *pack_host, const void *pack_dev, const emr_query *q, void *ws,
+                            size_t ws_bytes, void *stream);
+
+/* ---- a3: batched CPPN evaluation ---------------------------------------- */
+
+/* W = CPPN(s, T) at every grid position (Section 3.1, Eq. 1; Table 1 "CPPN
+ * query"), materialised. out: device float [P * S][n_total] (pair-major,
+ * global index; 16-byte aligned); out_halo: device float [P * S][n_halo] or
+ * NULL (then halo points are not evaluated). ws: prepared by
+ * emr_eval_prepare. Each position is evaluated once; coordinates are
+ * generated in the kernel. Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY, EMR_ERR_RANGE
+ * (more than 2^31 - 1 tiles: use emr_stream), EMR_ERR_CUDA. */
+emr_status emr_eval(const void *pack_host, const emr_query *q, const emr_grid *grid, float *out, float *out_halo,
+                    void *ws, size_t ws_bytes, void *stream);
+
+/* ---- a4, a5: variance and band/threshold filter --------------------------- */
+
+/* Filter a materialised evaluation (Section 3.2, Eq. 2; Theorem 1's band
+ * threshold). out/out_halo as written by emr_eval. Writes three bit planes,
+ * device uint32 [P * S][n_words] each: split (d < D and V > theta), band_bits
+ * (B > band and the weight filter) and mask (emr_mask_combine of the two in
+ * the given mode); var_dbg (optional, device float [P * S][n_total]) receives
+ * V(p). theta >= 0, band >= 0, w_min >= 0 (0 = weight filter off).
+ * Errors: EMR_ERR_ARG, EMR_ERR_CUDA. */
+emr_status emr_variance_filter(const float *out, const float *out_halo, const emr_grid *grid, int32_t P,
+                               int32_t S, float theta, float band, float w_min, int32_t mode, uint32_t *mask,
+                               uint32_t *split, uint32_t *band_bits, float *var_dbg, void *stream);
+
+/* Keep mask from the two planes: mask = band_bits AND NOT split (a depth-D
+ * position never splits), and for EMR_GATED also AND active (Eq. 2: every
+ * ancestor split). Bits past a level's positions are cleared.
+ * Errors: EMR_ERR_ARG, EMR_ERR_CUDA. */
+emr_status emr_mask_combine(const uint32_t *split, const uint32_t *band_bits, const emr_grid *grid,
+                            int32_t n_pairs, int32_t mode, uint32_t *mask, void *stream);
+
+/* ---- a3+a4+a5 fused ------------------------------------------------------ */
+
+/* Evaluate and filter in one kernel, without materialising the CPPN outputs:
+ * each tile of positions evaluates its points and the ring of neighbours it
+ * needs, takes each parent cell's variance from its four children in registers
+ * and each position's band value from shared memory, and writes only the split
+ * and band_bits planes (as emr_variance_filter) plus, when out is not NULL, the
+ * CPPN output at positions whose band test passed (other entries of out are
+ * left untouched). Follow with emr_mask_combine. ws: prepared by
+ * emr_eval_prepare. Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY, EMR_ERR_RANGE,
+ * EMR_ERR_CUDA. */
+emr_status emr_eval_filter(const void *pack_host, const emr_query *q, const emr_grid *grid, float theta,
+                           float band, float w_min, uint32_t *split, uint32_t *band_bits, float *out, void *ws,
+                           size_t ws_bytes, void *stream);
+
+/* ---- a6: compaction -------------------------------------------------------- */
+
+/* Bytes of device workspace emr_compact needs for n_pairs pairs. */
+emr_status emr_compact_workspace_size(const emr_grid *grid, int32_t n_pairs, size_t *bytes);
+
+/* Per pair, the ascending global indices of the set bits of mask and the CPPN
+ * outputs there (the connection list of each (genome, slot)). mask: device
+ * uint32 [n_pairs][n_words]; out: device float [n_pairs][n_total] (only the
+ * entries at set bits are read). Writes counts (device int64 [n_pairs]),
+ * offsets (device int64 [n_pairs + 1], exclusive prefix of counts; offsets[n_pairs]
+ * = total), idx (device int32 [cap]) and w (device float [cap], may be NULL):
+ * pair r's list is [offsets[r], offsets[r] + counts[r]). Entries at positions
+ * >= cap are dropped; compare offsets[n_pairs] with cap after the stream
+ * completes. Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY (workspace), EMR_ERR_CUDA. */
+emr_status emr_compact(const uint32_t *mask, const float *out, const emr_grid *grid, int32_t n_pairs,
+                       int32_t *idx, float *w, int64_t cap, int64_t *counts, int64_t *offsets, void *ws,
+                       size_t ws_bytes, void *stream);
+
+/* ---- misc -------------------------------------------------------------------- */
+
+/* Static description of a status code. */
+const char *emr_strerror(emr_status status);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int32_t emr_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EMR_H */

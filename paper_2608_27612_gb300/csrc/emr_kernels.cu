@@ -1,0 +1,853 @@
+// libemr device code for sm_103a: per-pair CPPN specialisation, tiled CPPN
+// evaluation with the fused variance/band epilogue, filter planes, mask
+// combination and ordered compaction.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+
+#include "emr_internal.h"
+
+using namespace emr;
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kBlock = 128;  // threads per evaluation tile CTA
+
+// ---- grid arithmetic ---------------------------------------------------------
+
+__host__ __device__ __forceinline__ uint32_t compact1by1(uint32_t x) {
+  x &= 0x55555555u;
+  x = (x | (x >> 1)) & 0x33333333u;
+  x = (x | (x >> 2)) & 0x0f0f0f0fu;
+  x = (x | (x >> 4)) & 0x00ff00ffu;
+  x = (x | (x >> 8)) & 0x0000ffffu;
+  return x;
+}
+__host__ __device__ __forceinline__ uint32_t spread1by1(uint32_t x) {
+  x &= 0x0000ffffu;
+  x = (x | (x << 8)) & 0x00ff00ffu;
+  x = (x | (x << 4)) & 0x0f0f0f0fu;
+  x = (x | (x << 2)) & 0x33333333u;
+  x = (x | (x << 1)) & 0x55555555u;
+  return x;
+}
+__device__ __forceinline__ uint32_t morton2(uint32_t i, uint32_t j) { return spread1by1(i) | (spread1by1(j) << 1); }
+
+// Eq. 1 coordinate of grid index i at depth d: (2i+1) 2^-(d+1) - 1, exact in fp32 for d <= 22.
+__device__ __forceinline__ float grid_coord(int i, float scale) { return fmaf(float(2 * i + 1), scale, -1.0f); }
+
+// ---- activations (fp32) --------------------------------------------------------
+// sigmoid and tanh from the exponential: sigmoid(z) = 1 / (1 + e^-z),
+// tanh(z) = 1 - 2 / (1 + e^{2z}); gauss(z) = e^{-z^2}; sin with a two-constant
+// Cody-Waite reduction by 2 pi (constants: 2 pi rounded to fp32 and the fp32
+// rounding of the remainder) before the hardware sine on [-pi, pi].
+constexpr float kTwoPiHi = 0x1.921fb6p+2f;
+constexpr float kTwoPiLo = -0x1.777a5cp-23f;
+constexpr float kInvTwoPi = 0x1.45f306p-3f;
+
+__device__ __forceinline__ float act_sigmoid(float z) { return __fdividef(1.0f, 1.0f + __expf(-z)); }
+__device__ __forceinline__ float act_tanh(float z) { return 1.0f - __fdividef(2.0f, 1.0f + __expf(2.0f * z)); }
+__device__ __forceinline__ float act_gauss(float z) { return __expf(-z * z); }
+__device__ __forceinline__ float act_sin(float z) {
+  float k = rintf(z * kInvTwoPi);
+  float r = fmaf(-k, kTwoPiHi, z);
+  r = fmaf(-k, kTwoPiLo, r);
+  return __sinf(r);
+}
+
+__device__ __forceinline__ float act_apply(int a, float z) {
+  switch (a) {
+    case EMR_ACT_SIGMOID: return act_sigmoid(z);
+    case EMR_ACT_TANH: return act_tanh(z);
+    case EMR_ACT_GAUSS: return act_gauss(z);
+    case EMR_ACT_SIN: return act_sin(z);
+    case EMR_ACT_ABS: return fabsf(z);
+    default: return z;
+  }
+}
+
+__device__ __forceinline__ void act_apply4(int a, float& z0, float& z1, float& z2, float& z3) {
+  switch (a) {
+    case EMR_ACT_SIGMOID: z0 = act_sigmoid(z0); z1 = act_sigmoid(z1); z2 = act_sigmoid(z2); z3 = act_sigmoid(z3); break;
+    case EMR_ACT_TANH: z0 = act_tanh(z0); z1 = act_tanh(z1); z2 = act_tanh(z2); z3 = act_tanh(z3); break;
+    case EMR_ACT_GAUSS: z0 = act_gauss(z0); z1 = act_gauss(z1); z2 = act_gauss(z2); z3 = act_gauss(z3); break;
+    case EMR_ACT_SIN: z0 = act_sin(z0); z1 = act_sin(z1); z2 = act_sin(z2); z3 = act_sin(z3); break;
+    case EMR_ACT_ABS: z0 = fabsf(z0); z1 = fabsf(z1); z2 = fabsf(z2); z3 = fabsf(z3); break;
+    default: break;
+  }
+}
+
+// ---- per-pair specialisation ---------------------------------------------------
+// A pair's record: header {nv, nve, out_const, flags}, then nv_cap float4
+// {c0, wx, wy, info} with info = act | edge_beg << 8 | edge_cnt << 20, then
+// nve_cap uint2 {source slot, weight bits}. Varying slots follow the genome's
+// topological order; the output is the last slot. nv = 0: the output is the
+// same at every position (out_const); unused per-genome slots are recorded as
+// constant 0 (no variance, no band value, nothing kept).
+struct SpecLayout {
+  int64_t stride;
+  int32_t nv_cap, nve_cap;
+  __host__ __device__ int64_t coef_off() const { return 16; }
+  __host__ __device__ int64_t edge_off() const { return 16 + 16 * int64_t(nv_cap); }
+};
+
+inline SpecLayout spec_layout(int nv_cap, int nve_cap) {
+  SpecLayout L;
+  L.nv_cap = std::max(nv_cap, 1);
+  L.nve_cap = std::max(nve_cap, 1);
+  L.stride = (16 + 16 * int64_t(L.nv_cap) + 8 * int64_t(L.nve_cap) + 15) & ~int64_t(15);
+  return L;
+}
+
+struct QueryDev {
+  const float *a, *b;
+  const int32_t *side, *count;
+  int32_t S, per_genome;
+};
+
+// Cost-ordered pair schedule (heaviest first) by a counting sort in one CTA.
+constexpr int kCostBins = 1024;
+__global__ void schedule_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_t n_pairs,
+                                int32_t* __restrict__ order) {
+  __shared__ int32_t hist[kCostBins];
+  __shared__ int32_t start[kCostBins];
+  const PackHeader* h = reinterpret_cast<const PackHeader*>(pack);
+  const PackGenome* gt = reinterpret_cast<const PackGenome*>(pack + h->off_genomes);
+  for (int k = threadIdx.x; k < kCostBins; k += blockDim.x) hist[k] = 0;
+  __syncthreads();
+  auto bin_of = [&](int64_t r) {
+    int g = int(r / q.S), s = int(r % q.S);
+    int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
+    int side = q.side[si] ? 1 : 0;
+    uint32_t c = gt[g].cost[side];
+    return kCostBins - 1 - int(min(c, uint32_t(kCostBins - 1)));  // descending cost
+  };
+  for (int64_t r = threadIdx.x; r < n_pairs; r += blockDim.x) atomicAdd(&hist[bin_of(r)], 1);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int k = 0; k < kCostBins; k++) { start[k] = acc; acc += hist[k]; }
+  }
+  __syncthreads();
+  for (int64_t r = threadIdx.x; r < n_pairs; r += blockDim.x) order[atomicAdd(&start[bin_of(r)], 1)] = int32_t(r);
+}
+
+// One thread per pair: fold the constant inputs (the slot's node coordinates
+// and the bias) and every node that does not vary over the grid into per-node
+// constants; list the edges between varying nodes.
+__global__ void spec_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_t n_pairs, SpecLayout L,
+                            uint8_t* __restrict__ spec, float* __restrict__ scratch, int32_t scratch_stride) {
+  int64_t r = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (r >= n_pairs) return;
+  const PackHeader* h = reinterpret_cast<const PackHeader*>(pack);
+  const PackGenome* gt = reinterpret_cast<const PackGenome*>(pack + h->off_genomes);
+  const PackNode* nt = reinterpret_cast<const PackNode*>(pack + h->off_nodes);
+  const PackEdge* et = reinterpret_cast<const PackEdge*>(pack + h->off_edges);
+  int g = int(r / q.S), s = int(r % q.S);
+  uint8_t* rec = spec + r * L.stride;
+  int32_t* hdr = reinterpret_cast<int32_t*>(rec);
+  if (q.per_genome && q.count && s >= q.count[g]) {  // unused slot: constant 0, nothing kept
+    hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = 0;
+    return;
+  }
+  int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
+  const int side = q.side[si] ? 1 : 0;
+  const float a = q.a[si], b = q.b[si];
+  // constant inputs of this side (grid inputs contribute through wx, wy)
+  float in[5] = {0.f, 0.f, 0.f, 0.f, 1.f};
+  int gx, gy;
+  if (side == EMR_SIDE_OUT) { in[EMR_KIND_X1] = a; in[EMR_KIND_Y1] = b; gx = EMR_KIND_X2; gy = EMR_KIND_Y2; }
+  else { in[EMR_KIND_X2] = a; in[EMR_KIND_Y2] = b; gx = EMR_KIND_X1; gy = EMR_KIND_Y1; }
+  const PackGenome G = gt[g];
+  float* cval = scratch + r * scratch_stride;  // const value, or varying slot (as int bits)
+  float4* coef = reinterpret_cast<float4*>(rec + L.coef_off());
+  uint2* ve = reinterpret_cast<uint2*>(rec + L.edge_off());
+  int nv = 0, nve = 0;
+  float out_const = 0.f;
+  for (int t = 0; t < G.n_nodes; t++) {
+    const PackNode nd = nt[G.node_beg + t];
+    const PackEdge* ed = et + G.edge_beg + nd.edge_beg;
+    if (nd.vary & (1u << side)) {
+      float c0 = nd.bias;
+      for (int k = 0; k < 5; k++)
+        if (k != gx && k != gy) c0 = fmaf(nd.w_in[k], in[k], c0);
+      int eb = nve;
+      for (int e = 0; e < nd.edge_cnt; e++) {
+        const PackNode src = nt[G.node_beg + ed[e].src];
+        if (src.vary & (1u << side)) {
+          ve[nve++] = make_uint2(__float_as_uint(cval[ed[e].src]), __float_as_uint(ed[e].w));
+        } else {
+          c0 = fmaf(ed[e].w, cval[ed[e].src], c0);
+        }
+      }
+      uint32_t info = uint32_t(nd.act) | (uint32_t(eb) << 8) | (uint32_t(nve - eb) << 20);
+      coef[nv] = make_float4(c0, nd.w_in[gx], nd.w_in[gy], __uint_as_float(info));
+      cval[t] = __uint_as_float(uint32_t(nv));
+      nv++;
+    } else {
+      float z = nd.bias;
+      for (int k = 0; k < 5; k++) z = fmaf(nd.w_in[k], in[k], z);
+      for (int e = 0; e < nd.edge_cnt; e++) z = fmaf(ed[e].w, cval[ed[e].src], z);
+      cval[t] = act_apply(nd.act, z);
+      out_const = cval[t];
+    }
+  }
+  hdr[0] = nv;
+  hdr[1] = nve;
+  reinterpret_cast<float*>(hdr)[2] = out_const;
+  hdr[3] = 0;
+}
+
+// ---- evaluation tiles ------------------------------------------------------------
+
+enum { kModeMaterialise = 0, kModeFused = 1 };
+
+struct TileArgs {
+  const uint8_t* spec;
+  SpecLayout L;
+  const int32_t* order;
+  int32_t n_tiles, tile_beg;
+  int32_t D, mode;
+  float theta, band, w_min;
+  int32_t lvl_tile_beg[EMR_MAX_DEPTH + 2];
+  int64_t n_total, n_halo, n_words;
+  int64_t level_off[EMR_MAX_DEPTH + 2], halo_off[EMR_MAX_DEPTH + 2], word_off[EMR_MAX_DEPTH + 2];
+  float* out;
+  float* out_halo;
+  uint32_t* split;
+  uint32_t* bandb;
+};
+
+// CPPN at four points by interpreting the pair's record: node values live in
+// shared memory, one float4 (four points) per thread and varying node.
+__device__ __forceinline__ void eval4_interp(const float4* __restrict__ coef, const uint2* __restrict__ ve,
+                                             float4* __restrict__ vals, int nv, float out_const, int tid,
+                                             const float (&x)[4], const float (&y)[4], float (&w)[4]) {
+  if (nv == 0) {
+    w[0] = w[1] = w[2] = w[3] = out_const;
+    return;
+  }
+  float z0 = 0.f, z1 = 0.f, z2 = 0.f, z3 = 0.f;
+  for (int k = 0; k < nv; k++) {
+    const float4 c = coef[k];
+    const uint32_t info = __float_as_uint(c.w);
+    z0 = fmaf(c.z, y[0], fmaf(c.y, x[0], c.x));
+    z1 = fmaf(c.z, y[1], fmaf(c.y, x[1], c.x));
+    z2 = fmaf(c.z, y[2], fmaf(c.y, x[2], c.x));
+    z3 = fmaf(c.z, y[3], fmaf(c.y, x[3], c.x));
+    const int eb = int((info >> 8) & 0xfffu), ee = eb + int(info >> 20);
+    for (int e = eb; e < ee; e++) {
+      const uint2 E = ve[e];
+      const float we = __uint_as_float(E.y);
+      const float4 v = vals[int(E.x) * kBlock + tid];
+      z0 = fmaf(we, v.x, z0);
+      z1 = fmaf(we, v.y, z1);
+      z2 = fmaf(we, v.z, z2);
+      z3 = fmaf(we, v.w, z3);
+    }
+    act_apply4(int(info & 0xffu), z0, z1, z2, z3);
+    if (k + 1 < nv) vals[k * kBlock + tid] = make_float4(z0, z1, z2, z3);
+  }
+  w[0] = z0; w[1] = z1; w[2] = z2; w[3] = z3;
+}
+
+__global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
+  extern __shared__ float4 smem4[];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t rank = blockIdx.x / A.n_tiles;
+  const int tile = A.tile_beg + int(blockIdx.x % A.n_tiles);
+  const int r = A.order[rank];
+  const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
+  const int nv = reinterpret_cast<const int32_t*>(rec)[0];
+  const int nve = reinterpret_cast<const int32_t*>(rec)[1];
+  const float out_const = reinterpret_cast<const float*>(rec)[2];
+  int d = 0;
+  while (A.lvl_tile_beg[d + 1] <= tile) d++;
+  const int T = d + 1 < kTileLog ? (1 << (d + 1)) : kTileSide;
+  const uint32_t mb = uint32_t(tile - A.lvl_tile_beg[d]) * uint32_t(T * T);  // first Morton index of the tile
+  const int i0 = int(compact1by1(mb)), j0 = int(compact1by1(mb >> 1));
+  const int n = 1 << (d + 1);
+  const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1)
+
+  // shared memory: record (coefficients, edges) | node values | output tile with its ring
+  float4* coef = smem4;
+  uint2* ve = reinterpret_cast<uint2*>(smem4 + A.L.nv_cap);
+  float4* vals = smem4 + A.L.nv_cap + (A.L.nve_cap + 1) / 2;
+  float* wt = reinterpret_cast<float*>(vals + A.L.nv_cap * kBlock);
+  const int pitch = T + 2;
+  {
+    const float4* gc = reinterpret_cast<const float4*>(rec + A.L.coef_off());
+    for (int k = tid; k < nv; k += kBlock) coef[k] = gc[k];
+    const uint2* ge = reinterpret_cast<const uint2*>(rec + A.L.edge_off());
+    for (int k = tid; k < nve; k += kBlock) ve[k] = ge[k];
+  }
+  __syncthreads();
+
+  const bool fused = A.mode == kModeFused;
+  const int nq = T * T / 4;
+  const bool ring = fused || A.out_halo != nullptr;
+  const int items = nq + (ring ? T : 0);
+  const int64_t pair_pos = int64_t(r) * A.n_total + A.level_off[d];
+  for (int base = 0; base < items; base += kBlock) {
+    const int q = base + tid;
+    const bool valid = q < items;
+    const bool is_main = q < nq;
+    int li[4], lj[4];
+    bool use = valid;
+    if (is_main) {
+      const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+#pragma unroll
+      for (int c = 0; c < 4; c++) { li[c] = 2 * pi + (c & 1); lj[c] = 2 * pj + (c >> 1); }
+    } else {
+      const int hq = valid ? q - nq : 0;
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        const int k = 4 * hq + c, sd = k / T, u = k - sd * T;
+        li[c] = sd == 0 ? -1 : sd == 1 ? T : u;
+        lj[c] = sd == 2 ? -1 : sd == 3 ? T : u;
+      }
+      if (!fused) {  // materialised: only ring points outside the domain are evaluated
+        const int sd = (4 * hq) / T;
+        const bool outside = (sd == 0 && i0 == 0) || (sd == 1 && i0 + T == n) || (sd == 2 && j0 == 0) ||
+                             (sd == 3 && j0 + T == n);
+        use = valid && outside;
+      }
+    }
+    float w[4] = {0.f, 0.f, 0.f, 0.f};
+    if (__any_sync(kFull, use)) {
+      float x[4], y[4];
+#pragma unroll
+      for (int c = 0; c < 4; c++) { x[c] = grid_coord(i0 + li[c], scale); y[c] = grid_coord(j0 + lj[c], scale); }
+      eval4_interp(coef, ve, vals, nv, out_const, tid, x, y, w);
+    }
+    if (!fused) {
+      if (is_main) {
+        *reinterpret_cast<float4*>(A.out + pair_pos + mb + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+      } else if (use) {
+#pragma unroll
+        for (int c = 0; c < 4; c++) {
+          const int gi = i0 + li[c], gj = j0 + lj[c];
+          const int sd = gi < 0 ? 0 : gi >= n ? 1 : gj < 0 ? 2 : 3;
+          const int t = sd < 2 ? gj : gi;
+          A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + sd * n + t] = w[c];
+        }
+      }
+      continue;
+    }
+    // fused: the four children of parent q give its variance (Section 3.2)
+    if (d >= 1) {
+      const float m = 0.25f * ((w[0] + w[1]) + (w[2] + w[3]));
+      const float e0 = w[0] - m, e1 = w[1] - m, e2 = w[2] - m, e3 = w[3] - m;
+      const float V = 0.25f * ((e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3));
+      const unsigned bal = __ballot_sync(kFull, is_main && V > A.theta);
+      const int q0 = base + warp * 32;
+      if (lane == 0 && q0 < nq)
+        A.split[int64_t(r) * A.n_words + A.word_off[d - 1] + (mb / 4 + uint32_t(q0)) / 32] = bal;
+    }
+    if (valid) {
+#pragma unroll
+      for (int c = 0; c < 4; c++) wt[(lj[c] + 1) * pitch + (li[c] + 1)] = w[c];
+    }
+  }
+  if (!fused) return;
+  __syncthreads();
+  // band value of each position from its four neighbours at distance 2^-d
+  for (int base = 0; base < nq; base += kBlock) {
+    const int q = base + tid;
+    const bool valid = q < nq;
+    const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+    unsigned nib = 0;
+    float w[4];
+#pragma unroll
+    for (int c = 0; c < 4; c++) {
+      const int li = 2 * pi + (c & 1) + 1, lj = 2 * pj + (c >> 1) + 1;
+      w[c] = valid ? wt[lj * pitch + li] : 0.f;
+      if (valid) {
+        const float dl = fabsf(w[c] - wt[lj * pitch + li - 1]), dr = fabsf(w[c] - wt[lj * pitch + li + 1]);
+        const float db = fabsf(w[c] - wt[(lj - 1) * pitch + li]), dt = fabsf(w[c] - wt[(lj + 1) * pitch + li]);
+        const float B = fmaxf(fminf(dt, db), fminf(dl, dr));
+        const bool pass = B > A.band && (A.w_min <= 0.f || fabsf(w[c]) > A.w_min);
+        nib |= unsigned(pass) << c;
+      }
+    }
+    unsigned v = nib << (4 * (lane & 7));
+    v |= __shfl_xor_sync(kFull, v, 1);
+    v |= __shfl_xor_sync(kFull, v, 2);
+    v |= __shfl_xor_sync(kFull, v, 4);
+    if ((lane & 7) == 0 && valid)
+      A.bandb[int64_t(r) * A.n_words + A.word_off[d] + (mb + 4u * uint32_t(q)) / 32] = v;
+    if (A.out && nib) {
+#pragma unroll
+      for (int c = 0; c < 4; c++)
+        if (nib & (1u << c)) A.out[pair_pos + mb + 4 * q + c] = w[c];
+    }
+  }
+}
+
+// ---- filter planes from a materialised evaluation ---------------------------------
+
+struct GridDev {
+  int32_t D;
+  int64_t n_total, n_halo, n_words;
+  int64_t level_off[EMR_MAX_DEPTH + 2], halo_off[EMR_MAX_DEPTH + 2], word_off[EMR_MAX_DEPTH + 2];
+};
+
+__device__ __forceinline__ int level_of_word(const GridDev& G, int64_t wi) {
+  int d = 0;
+  while (G.word_off[d + 1] <= wi) d++;
+  return d;
+}
+
+// Bits of word wi (depth d) that correspond to grid positions (depths 0 and 1 fill part of a word).
+__device__ __forceinline__ uint32_t valid_bits(const GridDev& G, int d, int64_t wi) {
+  const uint32_t m0 = uint32_t(wi - G.word_off[d]) * 32u;
+  const uint32_t cnt = 1u << (2 * (d + 1));
+  return cnt - m0 >= 32 ? kFull : ((1u << (cnt - m0)) - 1u);
+}
+
+// One warp per bit-plane word (32 positions of one depth).
+__global__ void planes_kernel(const float* __restrict__ out, const float* __restrict__ out_halo, GridDev G,
+                              int64_t n_pairs, float theta, float band, float w_min, uint32_t* __restrict__ split,
+                              uint32_t* __restrict__ bandb, float* __restrict__ var_dbg) {
+  const int lane = threadIdx.x & 31;
+  const int64_t wg = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  if (wg >= n_pairs * G.n_words) return;
+  const int64_t r = wg / G.n_words, wi = wg % G.n_words;
+  const int d = level_of_word(G, wi);
+  const uint32_t m = uint32_t(wi - G.word_off[d]) * 32u + uint32_t(lane);
+  const uint32_t cnt = 1u << (2 * (d + 1));
+  const bool valid = m < cnt;
+  const int n = 1 << (d + 1);
+  const float* o = out + r * G.n_total;
+  bool sp = false, bp = false;
+  if (valid) {
+    const int i = int(compact1by1(m)), j = int(compact1by1(m >> 1));
+    const float w = o[G.level_off[d] + m];
+    float V = 0.f;
+    if (d < G.D) {
+      const float4 c = *reinterpret_cast<const float4*>(o + G.level_off[d + 1] + 4 * int64_t(m));
+      const float mu = 0.25f * ((c.x + c.y) + (c.z + c.w));
+      const float e0 = c.x - mu, e1 = c.y - mu, e2 = c.z - mu, e3 = c.w - mu;
+      V = 0.25f * ((e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3));
+      sp = V > theta;
+    }
+    if (var_dbg) var_dbg[r * G.n_total + G.level_off[d] + m] = V;
+    float nbv[4];
+    const int ni[4] = {i - 1, i + 1, i, i}, nj[4] = {j, j, j - 1, j + 1};
+#pragma unroll
+    for (int k = 0; k < 4; k++) {
+      if (ni[k] >= 0 && ni[k] < n && nj[k] >= 0 && nj[k] < n) {
+        nbv[k] = o[G.level_off[d] + morton2(uint32_t(ni[k]), uint32_t(nj[k]))];
+      } else {
+        const int sd = ni[k] < 0 ? 0 : ni[k] >= n ? 1 : nj[k] < 0 ? 2 : 3;
+        const int t = sd < 2 ? nj[k] : ni[k];
+        nbv[k] = out_halo[r * G.n_halo + G.halo_off[d] + sd * n + t];
+      }
+    }
+    const float dl = fabsf(w - nbv[0]), dr = fabsf(w - nbv[1]), db = fabsf(w - nbv[2]), dt = fabsf(w - nbv[3]);
+    const float B = fmaxf(fminf(dt, db), fminf(dl, dr));
+    bp = B > band && (w_min <= 0.f || fabsf(w) > w_min);
+  }
+  const unsigned s_bits = __ballot_sync(kFull, sp), b_bits = __ballot_sync(kFull, bp);
+  if (lane == 0) {
+    split[r * G.n_words + wi] = s_bits;
+    bandb[r * G.n_words + wi] = b_bits;
+  }
+}
+
+// mask = band AND NOT split (no split at depth D); gated: AND Eq. 2's active bit.
+__global__ void combine_kernel(const uint32_t* __restrict__ split, const uint32_t* __restrict__ bandb, GridDev G,
+                               int64_t n_pairs, int gated, uint32_t* __restrict__ mask) {
+  const int64_t wg = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (wg >= n_pairs * G.n_words) return;
+  const int64_t r = wg / G.n_words, wi = wg % G.n_words;
+  const int d = level_of_word(G, wi);
+  const uint32_t m0 = uint32_t(wi - G.word_off[d]) * 32u;
+  const uint32_t valid = valid_bits(G, d, wi);
+  const uint32_t* sp = split + r * G.n_words;
+  uint32_t keep = bandb[r * G.n_words + wi] & valid;
+  if (d < G.D) keep &= ~sp[wi];
+  if (gated && keep) {
+    // active(p) = every ancestor split (Eq. 2); the ancestors of these 32
+    // positions at each shallower depth lie in a single word.
+    uint32_t act = kFull;
+    for (int k = 1; k <= d && act; k++) {
+      const uint32_t a0 = m0 >> (2 * k);
+      const uint32_t aw = sp[G.word_off[d - k] + (a0 >> 5)];
+      uint32_t bits = 0;
+      for (int b = 0; b < 32; b++) {
+        const uint32_t anc = (m0 + uint32_t(b)) >> (2 * k);
+        bits |= ((aw >> (anc & 31u)) & 1u) << b;
+      }
+      act &= bits;
+    }
+    keep &= act;
+  }
+  mask[r * G.n_words + wi] = keep;
+}
+
+// ---- ordered compaction -----------------------------------------------------------
+
+constexpr int kCompactBlock = 256;  // words per compaction block (8192 positions)
+
+__device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int t = lane < nw ? sh[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, t, o);
+      if (lane >= o) t += y;
+    }
+    if (lane < nw) sh[lane] = t;
+  }
+  __syncthreads();
+  const int before = warp ? sh[warp - 1] : 0;
+  if (total) *total = sh[nw - 1];
+  __syncthreads();
+  return before + x - v;
+}
+
+__global__ void compact_count_kernel(const uint32_t* __restrict__ mask, GridDev G, int nb,
+                                     int32_t* __restrict__ bcount) {
+  __shared__ int sh[32];
+  const int64_t r = blockIdx.x / nb;
+  const int b = int(blockIdx.x % nb);
+  const int64_t wi = int64_t(b) * kCompactBlock + threadIdx.x;
+  const int c = wi < G.n_words ? __popc(mask[r * G.n_words + wi] & valid_bits(G, level_of_word(G, wi), wi)) : 0;
+  int total;
+  block_exclusive_scan(c, sh, &total);
+  if (threadIdx.x == 0) bcount[blockIdx.x] = total;
+}
+
+// One CTA per pair: exclusive scan of its block counts.
+__global__ void compact_scan_pair_kernel(const int32_t* __restrict__ bcount, int nb, int32_t* __restrict__ boff,
+                                         int64_t* __restrict__ counts) {
+  __shared__ int sh[32];
+  const int64_t r = blockIdx.x;
+  int carry = 0;
+  for (int k0 = 0; k0 < nb; k0 += blockDim.x) {
+    const int k = k0 + threadIdx.x;
+    const int v = k < nb ? bcount[r * nb + k] : 0;
+    int total;
+    const int ex = block_exclusive_scan(v, sh, &total);
+    if (k < nb) boff[r * nb + k] = carry + ex;
+    carry += total;
+  }
+  if (threadIdx.x == 0) counts[r] = carry;
+}
+
+// One CTA: exclusive scan of the pair counts (int64).
+__global__ void compact_scan_pairs_kernel(const int64_t* __restrict__ counts, int64_t n_pairs,
+                                          int64_t* __restrict__ offsets) {
+  __shared__ long long sh[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  long long carry = 0;
+  for (int64_t k0 = 0; k0 < n_pairs; k0 += blockDim.x) {
+    const int64_t k = k0 + threadIdx.x;
+    const long long v = k < n_pairs ? counts[k] : 0;
+    long long x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(kFull, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) sh[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+      long long t = lane < nw ? sh[lane] : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(kFull, t, o);
+        if (lane >= o) t += y;
+      }
+      if (lane < nw) sh[lane] = t;
+    }
+    __syncthreads();
+    const long long before = warp ? sh[warp - 1] : 0;
+    if (k < n_pairs) offsets[k] = carry + before + x - v;
+    carry += sh[nw - 1];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) offsets[n_pairs] = carry;
+}
+
+__global__ void compact_write_kernel(const uint32_t* __restrict__ mask, const float* __restrict__ out, GridDev G,
+                                     int nb, const int32_t* __restrict__ boff, const int64_t* __restrict__ offsets,
+                                     int64_t cap, int32_t* __restrict__ idx, float* __restrict__ wv) {
+  __shared__ int sh[32];
+  const int64_t r = blockIdx.x / nb;
+  const int b = int(blockIdx.x % nb);
+  const int64_t wi = int64_t(b) * kCompactBlock + threadIdx.x;
+  const int d = wi < G.n_words ? level_of_word(G, wi) : 0;
+  const uint32_t bits = wi < G.n_words ? mask[r * G.n_words + wi] & valid_bits(G, d, wi) : 0u;
+  const int ex = block_exclusive_scan(__popc(bits), sh, nullptr);
+  if (!bits) return;
+  const int64_t gbase = G.level_off[d] + (wi - G.word_off[d]) * 32;
+  int64_t dst = offsets[r] + boff[blockIdx.x] + ex;
+  for (uint32_t v = bits; v; v &= v - 1, dst++) {
+    const int64_t gidx = gbase + __ffs(v) - 1;
+    if (dst < cap) {
+      idx[dst] = int32_t(gidx);
+      if (wv) wv[dst] = out[r * G.n_total + gidx];
+    }
+  }
+}
+
+// ---- host helpers ---------------------------------------------------------------
+
+inline emr_status cuda_status(cudaError_t e) { return e == cudaSuccess ? EMR_OK : EMR_ERR_CUDA; }
+
+inline bool grid_ok(const emr_grid* g) { return g && g->D >= 0 && g->D <= EMR_MAX_DEPTH && g->n_total > 0; }
+
+GridDev grid_dev(const emr_grid* g) {
+  GridDev G{};
+  G.D = g->D;
+  G.n_total = g->n_total;
+  G.n_halo = g->n_halo;
+  G.n_words = g->n_words;
+  for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {
+    G.level_off[d] = g->level_off[d];
+    G.halo_off[d] = g->halo_off[d];
+    G.word_off[d] = g->word_off[d];
+  }
+  return G;
+}
+
+struct EvalPlan {
+  int64_t n_pairs;
+  SpecLayout L;
+  int32_t scratch_stride;
+  size_t spec_bytes, scratch_bytes, order_bytes, total;
+};
+
+emr_status eval_plan(const void* pack_host, const emr_query* q, EvalPlan* p) {
+  if (!pack_host || !q || q->S <= 0 || !q->a_host || !q->b_host || !q->side_host) return EMR_ERR_ARG;
+  const PackHeader* h = pack_header(pack_host);
+  if (h->magic != kPackMagic || h->version != kPackVersion || h->P <= 0) return EMR_ERR_ARG;
+  bool sides[2] = {false, false};
+  const int64_t ns = q->per_genome ? int64_t(h->P) * q->S : q->S;
+  for (int64_t k = 0; k < ns; k++) {
+    if (q->side_host[k] != EMR_SIDE_OUT && q->side_host[k] != EMR_SIDE_IN) return EMR_ERR_ARG;
+    sides[q->side_host[k]] = true;
+  }
+  int nv = 0, nve = 0;
+  for (int s = 0; s < 2; s++)
+    if (sides[s]) { nv = std::max(nv, h->max_varying[s]); nve = std::max(nve, h->max_vedges[s]); }
+  p->n_pairs = int64_t(h->P) * q->S;
+  p->L = spec_layout(nv, nve);
+  p->scratch_stride = std::max(h->max_nodes, 1);
+  p->spec_bytes = size_t(p->n_pairs) * size_t(p->L.stride);
+  p->scratch_bytes = (size_t(p->n_pairs) * size_t(p->scratch_stride) * 4 + 255) & ~size_t(255);
+  p->order_bytes = (size_t(p->n_pairs) * 4 + 255) & ~size_t(255);
+  p->total = ((p->spec_bytes + 255) & ~size_t(255)) + p->scratch_bytes + p->order_bytes;
+  return EMR_OK;
+}
+
+QueryDev query_dev(const emr_query* q) {
+  QueryDev d;
+  d.a = q->a_dev;
+  d.b = q->b_dev;
+  d.side = q->side_dev;
+  d.count = q->count_dev;
+  d.S = q->S;
+  d.per_genome = q->per_genome;
+  return d;
+}
+
+void ws_layout(const EvalPlan& p, void* ws, uint8_t** spec, int32_t** order, float** scratch = nullptr) {
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  *spec = base;
+  float* sc = reinterpret_cast<float*>(base + ((p.spec_bytes + 255) & ~size_t(255)));
+  *order = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(sc) + p.scratch_bytes);
+  if (scratch) *scratch = sc;
+}
+
+// Specialise every pair and order the pairs by cost, into the workspace.
+emr_status prepare(const void* pack_dev, const emr_query* q, const EvalPlan& p, void* ws, cudaStream_t st,
+                   uint8_t** spec, int32_t** order) {
+  float* scratch;
+  ws_layout(p, ws, spec, order, &scratch);
+  const QueryDev qd = query_dev(q);
+  const uint8_t* pk = static_cast<const uint8_t*>(pack_dev);
+  schedule_kernel<<<1, 1024, 0, st>>>(pk, qd, p.n_pairs, *order);
+  spec_kernel<<<unsigned((p.n_pairs + 127) / 128), 128, 0, st>>>(pk, qd, p.n_pairs, p.L, *spec, scratch,
+                                                                   p.scratch_stride);
+  return cuda_status(cudaGetLastError());
+}
+
+size_t tile_smem_bytes(const SpecLayout& L) {
+  return 16 * size_t(L.nv_cap) + 16 * size_t((L.nve_cap + 1) / 2) + 16 * size_t(L.nv_cap) * kBlock +
+         4 * size_t(kTileSide + 2) * size_t(kTileSide + 2);
+}
+
+emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spec, const int32_t* order, int mode,
+                        float theta, float band, float w_min, float* out, float* out_halo, uint32_t* split,
+                        uint32_t* bandb, cudaStream_t st) {
+  TileArgs A{};
+  A.spec = spec;
+  A.L = p.L;
+  A.order = order;
+  A.D = g->D;
+  A.mode = mode;
+  A.theta = theta;
+  A.band = band;
+  A.w_min = w_min;
+  int32_t t = 0;
+  for (int d = 0; d <= g->D; d++) {
+    A.lvl_tile_beg[d] = t;
+    t += int32_t(tiles_in_level(d));
+  }
+  for (int d = g->D + 1; d < EMR_MAX_DEPTH + 2; d++) A.lvl_tile_beg[d] = t;
+  A.n_tiles = t;
+  A.tile_beg = 0;
+  A.n_total = g->n_total;
+  A.n_halo = g->n_halo;
+  A.n_words = g->n_words;
+  for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {
+    A.level_off[d] = g->level_off[d];
+    A.halo_off[d] = g->halo_off[d];
+    A.word_off[d] = g->word_off[d];
+  }
+  A.out = out;
+  A.out_halo = out_halo;
+  A.split = split;
+  A.bandb = bandb;
+  const int64_t blocks = p.n_pairs * int64_t(A.n_tiles);
+  if (blocks <= 0) return EMR_OK;
+  if (blocks > 0x7fffffffLL) return EMR_ERR_RANGE;
+  const size_t smem = tile_smem_bytes(p.L);
+  if (smem > 227 * 1024) return EMR_ERR_RANGE;
+  cudaError_t e = cudaFuncSetAttribute(tile_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return EMR_ERR_CUDA;
+  tile_kernel<<<unsigned(blocks), kBlock, smem, st>>>(A);
+  return cuda_status(cudaGetLastError());
+}
+
+emr_status launch_combine(const uint32_t* split, const uint32_t* bandb, const emr_grid* g, int64_t n_pairs, int gated,
+                          uint32_t* mask, cudaStream_t st) {
+  const int64_t n = n_pairs * g->n_words;
+  if (n <= 0) return EMR_OK;
+  combine_kernel<<<unsigned((n + 255) / 256), 256, 0, st>>>(split, bandb, grid_dev(g), n_pairs, gated, mask);
+  return cuda_status(cudaGetLastError());
+}
+
+}  // namespace
+
+extern "C" {
+
+emr_status emr_eval_workspace_size(const void* pack_host, const emr_query* q, size_t* bytes) {
+  if (!bytes) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  *bytes = p.total;
+  return EMR_OK;
+}
+
+emr_status emr_eval_prepare(const void* pack_host, const void* pack_dev, const emr_query* q, void* ws,
+                            size_t ws_bytes, void* stream) {
+  if (!pack_dev || !ws || !q || !q->a_dev || !q->b_dev || !q->side_dev) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (ws_bytes < p.total) return EMR_ERR_CAPACITY;
+  uint8_t* spec;
+  int32_t* order;
+  return prepare(pack_dev, q, p, ws, static_cast<cudaStream_t>(stream), &spec, &order);
+}
+
+emr_status emr_eval(const void* pack_host, const emr_query* q, const emr_grid* grid, float* out, float* out_halo,
+                    void* ws, size_t ws_bytes, void* stream) {
+  if (!grid_ok(grid) || !out || !ws) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (ws_bytes < p.total) return EMR_ERR_CAPACITY;
+  uint8_t* spec;
+  int32_t* order;
+  ws_layout(p, ws, &spec, &order);
+  return launch_tiles(p, grid, spec, order, kModeMaterialise, 0.f, 0.f, 0.f, out, out_halo, nullptr, nullptr,
+                      static_cast<cudaStream_t>(stream));
+}
+
+emr_status emr_mask_combine(const uint32_t* split, const uint32_t* band_bits, const emr_grid* grid, int32_t n_pairs,
+                            int32_t mode, uint32_t* mask, void* stream) {
+  if (!split || !band_bits || !mask || !grid_ok(grid) || n_pairs <= 0 || (mode != EMR_EAGER && mode != EMR_GATED))
+    return EMR_ERR_ARG;
+  return launch_combine(split, band_bits, grid, n_pairs, mode == EMR_GATED, mask, static_cast<cudaStream_t>(stream));
+}
+
+emr_status emr_variance_filter(const float* out, const float* out_halo, const emr_grid* grid, int32_t P, int32_t S,
+                               float theta, float band, float w_min, int32_t mode, uint32_t* mask, uint32_t* split,
+                               uint32_t* band_bits, float* var_dbg, void* stream) {
+  if (!out || !out_halo || !grid_ok(grid) || P <= 0 || S <= 0 || !mask || !split || !band_bits) return EMR_ERR_ARG;
+  if (!(theta >= 0.f) || !(band >= 0.f) || !(w_min >= 0.f) || (mode != EMR_EAGER && mode != EMR_GATED))
+    return EMR_ERR_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int64_t n_pairs = int64_t(P) * S;
+  const int64_t threads = n_pairs * grid->n_words * 32;
+  planes_kernel<<<unsigned((threads + 255) / 256), 256, 0, st>>>(out, out_halo, grid_dev(grid), n_pairs, theta, band,
+                                                                 w_min, split, band_bits, var_dbg);
+  emr_status rc = cuda_status(cudaGetLastError());
+  if (rc != EMR_OK) return rc;
+  return launch_combine(split, band_bits, grid, n_pairs, mode == EMR_GATED, mask, st);
+}
+
+emr_status emr_eval_filter(const void* pack_host, const emr_query* q, const emr_grid* grid, float theta, float band,
+                           float w_min, uint32_t* split, uint32_t* band_bits, float* out, void* ws, size_t ws_bytes,
+                           void* stream) {
+  if (!grid_ok(grid) || !split || !band_bits || !ws) return EMR_ERR_ARG;
+  if (!(theta >= 0.f) || !(band >= 0.f) || !(w_min >= 0.f)) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (ws_bytes < p.total) return EMR_ERR_CAPACITY;
+  uint8_t* spec;
+  int32_t* order;
+  ws_layout(p, ws, &spec, &order);
+  return launch_tiles(p, grid, spec, order, kModeFused, theta, band, w_min, out, nullptr, split, band_bits,
+                      static_cast<cudaStream_t>(stream));
+}
+
+emr_status emr_compact_workspace_size(const emr_grid* grid, int32_t n_pairs, size_t* bytes) {
+  if (!grid_ok(grid) || n_pairs <= 0 || !bytes) return EMR_ERR_ARG;
+  const int64_t nb = (grid->n_words + kCompactBlock - 1) / kCompactBlock;
+  *bytes = size_t(2 * 4 * nb * int64_t(n_pairs) + 256);
+  return EMR_OK;
+}
+
+emr_status emr_compact(const uint32_t* mask, const float* out, const emr_grid* grid, int32_t n_pairs, int32_t* idx,
+                       float* w, int64_t cap, int64_t* counts, int64_t* offsets, void* ws, size_t ws_bytes,
+                       void* stream) {
+  if (!mask || !grid_ok(grid) || n_pairs <= 0 || (!idx && cap > 0) || cap < 0 || !counts || !offsets || !ws ||
+      (w && !out))
+    return EMR_ERR_ARG;
+  size_t need;
+  emr_compact_workspace_size(grid, n_pairs, &need);
+  if (ws_bytes < need) return EMR_ERR_CAPACITY;
+  const int nb = int((grid->n_words + kCompactBlock - 1) / kCompactBlock);
+  const int64_t nblk = int64_t(nb) * n_pairs;
+  if (nblk > 0x7fffffffLL) return EMR_ERR_RANGE;
+  int32_t* bcount = static_cast<int32_t*>(ws);
+  int32_t* boff = bcount + nblk;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  compact_count_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, grid_dev(grid), nb, bcount);
+  compact_scan_pair_kernel<<<unsigned(n_pairs), 256, 0, st>>>(bcount, nb, boff, counts);
+  compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, n_pairs, offsets);
+  compact_write_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, out, grid_dev(grid), nb, boff, offsets, cap,
+                                                                 idx, w);
+  return cuda_status(cudaGetLastError());
+}
+
+}  // extern "C"

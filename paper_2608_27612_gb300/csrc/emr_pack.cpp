@@ -1,0 +1,286 @@
+// Host side of libemr: grid descriptor (Eq. 1), genome packer, status strings.
+#include <algorithm>
+#include <cstring>
+#include <unordered_map>
+#include <vector>
+
+#include "emr_internal.h"
+
+using namespace emr;
+
+namespace {
+
+inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
+
+uint32_t compact_bits(uint64_t m) {  // even bits of m, packed
+  m &= 0x5555555555555555ull;
+  m = (m | (m >> 1)) & 0x3333333333333333ull;
+  m = (m | (m >> 2)) & 0x0f0f0f0f0f0f0f0full;
+  m = (m | (m >> 4)) & 0x00ff00ff00ff00ffull;
+  m = (m | (m >> 8)) & 0x0000ffff0000ffffull;
+  m = (m | (m >> 16)) & 0x00000000ffffffffull;
+  return uint32_t(m);
+}
+
+// Relative per-query work of one activation, for scheduling only.
+int act_cost(int a) {
+  static const int c[6] = {0, 5, 6, 3, 7, 1};
+  return (a >= 0 && a < 6) ? c[a] : 8;
+}
+
+struct GenomeOut {
+  std::vector<PackNode> nodes;
+  std::vector<PackEdge> edges;
+  PackGenome g{};
+};
+
+// Topological order (Kahn, ties by id), dead-node removal, input folding and
+// per-side variation flags for one genome.
+emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_t* node_id,
+                    const int32_t* node_kind, const int32_t* node_act, const float* node_bias,
+                    const int32_t* conn_src, const int32_t* conn_dst, const float* conn_w,
+                    const uint8_t* conn_en, GenomeOut* out) {
+  const int n = int(n1 - n0);
+  if (n <= 0 || n > 1 << 20) return EMR_ERR_ARG;
+  std::unordered_map<int32_t, int> local;
+  int out_node = -1;
+  for (int k = 0; k < n; k++) {
+    int kind = node_kind[n0 + k];
+    if (kind < 0 || kind > EMR_KIND_OUTPUT) return EMR_ERR_ARG;
+    if (kind >= EMR_KIND_HIDDEN && (node_act[n0 + k] < 0 || node_act[n0 + k] > EMR_ACT_ABS)) return EMR_ERR_ARG;
+    if (!local.emplace(node_id[n0 + k], k).second) return EMR_ERR_ARG;
+    if (kind == EMR_KIND_OUTPUT) {
+      if (out_node >= 0) return EMR_ERR_ARG;
+      out_node = k;
+    }
+  }
+  if (out_node < 0) return EMR_ERR_ARG;
+  struct E { int s, d; float w; };
+  std::vector<E> es;
+  for (int64_t c = c0; c < c1; c++) {
+    if (!conn_en[c]) continue;
+    auto is = local.find(conn_src[c]), id = local.find(conn_dst[c]);
+    if (is == local.end() || id == local.end()) return EMR_ERR_ARG;
+    if (node_kind[n0 + id->second] < EMR_KIND_HIDDEN) return EMR_ERR_ARG;
+    es.push_back({is->second, id->second, conn_w[c]});
+  }
+  // Kahn's algorithm over every node; ready nodes leave in ascending id order.
+  std::vector<int> indeg(n, 0), order;
+  std::vector<std::vector<int>> succ(n), pred(n);
+  for (auto& e : es) { indeg[e.d]++; succ[e.s].push_back(e.d); pred[e.d].push_back(e.s); }
+  auto by_id = [&](int a, int b) { return node_id[n0 + a] > node_id[n0 + b]; };  // min-heap on id
+  std::vector<int> ready;
+  for (int v = 0; v < n; v++) if (indeg[v] == 0) ready.push_back(v);
+  std::make_heap(ready.begin(), ready.end(), by_id);
+  while (!ready.empty()) {
+    std::pop_heap(ready.begin(), ready.end(), by_id);
+    int v = ready.back();
+    ready.pop_back();
+    order.push_back(v);
+    for (int s : succ[v])
+      if (--indeg[s] == 0) { ready.push_back(s); std::push_heap(ready.begin(), ready.end(), by_id); }
+  }
+  if (int(order.size()) != n) return EMR_ERR_CYCLE;
+  // Keep the non-input nodes from which the output is reachable.
+  std::vector<char> reach(n, 0);
+  std::vector<int> stack{out_node};
+  reach[out_node] = 1;
+  while (!stack.empty()) {
+    int v = stack.back();
+    stack.pop_back();
+    for (int p : pred[v]) if (!reach[p]) { reach[p] = 1; stack.push_back(p); }
+  }
+  std::vector<int> slot(n, -1), kept;
+  for (int v : order)
+    if (reach[v] && node_kind[n0 + v] >= EMR_KIND_HIDDEN) { slot[v] = int(kept.size()); kept.push_back(v); }
+  if (kept.empty() || kept.back() != out_node) return EMR_ERR_ARG;  // output must be last
+  if (kept.size() > 65535) return EMR_ERR_RANGE;
+  const int nk = int(kept.size());
+  out->nodes.assign(nk, PackNode{});
+  std::vector<std::vector<PackEdge>> in_edges(nk);
+  std::vector<unsigned> has_in(nk, 0);  // bit k: has an enabled in-connection from input kind k
+  for (int t = 0; t < nk; t++) {
+    int v = kept[t];
+    PackNode& pn = out->nodes[t];
+    pn.act = uint8_t(node_act[n0 + v]);
+    pn.bias = node_bias[n0 + v];
+  }
+  for (auto& e : es) {
+    int t = slot[e.d];
+    if (t < 0) continue;
+    int sk = node_kind[n0 + e.s];
+    if (sk < EMR_KIND_HIDDEN) {
+      out->nodes[t].w_in[sk] += e.w;
+      has_in[t] |= 1u << sk;
+    } else {
+      if (slot[e.s] < 0) return EMR_ERR_ARG;  // cannot happen: a source of a kept node is kept
+      in_edges[t].push_back(PackEdge{uint16_t(slot[e.s]), 0, e.w});
+    }
+  }
+  PackGenome& g = out->g;
+  g.n_nodes = uint16_t(nk);
+  for (int t = 0; t < nk; t++) {
+    if (out->edges.size() + in_edges[t].size() > 65535) return EMR_ERR_RANGE;
+    out->nodes[t].edge_beg = uint16_t(out->edges.size());
+    out->nodes[t].edge_cnt = uint16_t(in_edges[t].size());
+    out->edges.insert(out->edges.end(), in_edges[t].begin(), in_edges[t].end());
+  }
+  g.n_edges = uint16_t(out->edges.size());
+  for (int side = 0; side < 2; side++) {
+    const unsigned grid_inputs = side == EMR_SIDE_OUT ? (1u << EMR_KIND_X2) | (1u << EMR_KIND_Y2)
+                                                      : (1u << EMR_KIND_X1) | (1u << EMR_KIND_Y1);
+    int nv = 0, nve = 0;
+    uint32_t cost = 0;
+    for (int t = 0; t < nk; t++) {
+      bool vary = (has_in[t] & grid_inputs) != 0;
+      int vin = 0;
+      for (auto& e : in_edges[t])
+        if (out->nodes[e.src].vary & (1u << side)) { vary = true; vin++; }
+      if (vary) {
+        out->nodes[t].vary |= uint8_t(1u << side);
+        nv++;
+        nve += vin;
+        cost += 2 + vin + act_cost(out->nodes[t].act);
+      }
+    }
+    if (nv > EMR_MAX_VARYING || nve > EMR_MAX_VEDGES) return EMR_ERR_RANGE;
+    g.n_varying[side] = uint16_t(nv);
+    g.n_vedges[side] = uint16_t(nve);
+    g.cost[side] = cost;
+  }
+  return EMR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+emr_status emr_grid_build(int32_t D, int64_t chunk, emr_grid* grid) {
+  if (!grid) return EMR_ERR_ARG;
+  if (D < 0 || D > EMR_MAX_DEPTH) return EMR_ERR_RANGE;
+  if (chunk < 0 || (chunk > 0 && (chunk < 4096 || (chunk & (chunk - 1)) != 0))) return EMR_ERR_ARG;
+  std::memset(grid, 0, sizeof *grid);
+  grid->D = D;
+  grid->chunk = chunk;
+  int64_t words = 0;
+  for (int d = 0; d <= D + 1; d++) {
+    grid->level_off[d] = level_offset(d);
+    grid->halo_off[d] = halo_offset(d);
+    grid->word_off[d] = words;
+    if (d <= D) words += ((int64_t(1) << (2 * (d + 1))) + 31) / 32;
+  }
+  grid->n_total = grid->level_off[D + 1];
+  grid->n_halo = grid->halo_off[D + 1];
+  grid->n_words = words;
+  return EMR_OK;
+}
+
+emr_status emr_index_to_ij(int64_t gidx, int32_t* d, int32_t* i, int32_t* j) {
+  if (gidx < 0 || gidx >= level_offset(EMR_MAX_DEPTH + 1)) return EMR_ERR_RANGE;
+  int lv = 0;
+  while (level_offset(lv + 1) <= gidx) lv++;
+  uint64_t m = uint64_t(gidx - level_offset(lv));
+  if (d) *d = lv;
+  if (i) *i = int32_t(compact_bits(m));
+  if (j) *j = int32_t(compact_bits(m >> 1));
+  return EMR_OK;
+}
+
+emr_status emr_pack_size(int32_t P, const int64_t* node_ptr, const int64_t* conn_ptr, size_t* bytes) {
+  if (P < 0 || !bytes || (P > 0 && (!node_ptr || !conn_ptr))) return EMR_ERR_ARG;
+  int64_t nn = P ? node_ptr[P] - node_ptr[0] : 0, nc = P ? conn_ptr[P] - conn_ptr[0] : 0;
+  if (nn < 0 || nc < 0) return EMR_ERR_ARG;
+  *bytes = align16(sizeof(PackHeader)) + align16(sizeof(PackGenome) * size_t(P)) +
+           align16(sizeof(PackNode) * size_t(nn)) + align16(sizeof(PackEdge) * size_t(nc)) + 16;
+  return EMR_OK;
+}
+
+emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t* node_id,
+                               const int32_t* node_kind, const int32_t* node_act, const float* node_bias,
+                               const int64_t* conn_ptr, const int32_t* conn_src, const int32_t* conn_dst,
+                               const float* conn_w, const uint8_t* conn_enabled, void* buf, size_t cap,
+                               size_t* used, int32_t* bad_genome) {
+  if (bad_genome) *bad_genome = -1;
+  if (P <= 0 || !node_ptr || !node_id || !node_kind || !node_act || !node_bias || !conn_ptr ||
+      (!buf && cap > 0) || !used)
+    return EMR_ERR_ARG;
+  const bool has_conns = conn_ptr[P] > conn_ptr[0];
+  if (has_conns && (!conn_src || !conn_dst || !conn_w || !conn_enabled)) return EMR_ERR_ARG;
+  std::vector<GenomeOut> gs(P);
+  for (int g = 0; g < P; g++) {
+    if (node_ptr[g + 1] < node_ptr[g] || conn_ptr[g + 1] < conn_ptr[g]) {
+      if (bad_genome) *bad_genome = g;
+      return EMR_ERR_ARG;
+    }
+    emr_status rc = pack_one(node_ptr[g], node_ptr[g + 1], conn_ptr[g], conn_ptr[g + 1], node_id, node_kind,
+                             node_act, node_bias, conn_src, conn_dst, conn_w, conn_enabled, &gs[g]);
+    if (rc != EMR_OK) {
+      if (bad_genome) *bad_genome = g;
+      return rc;
+    }
+  }
+  size_t nn = 0, ne = 0;
+  for (auto& g : gs) { nn += g.nodes.size(); ne += g.edges.size(); }
+  PackHeader h{};
+  h.magic = kPackMagic;
+  h.version = kPackVersion;
+  h.P = P;
+  h.off_genomes = align16(sizeof(PackHeader));
+  h.off_nodes = h.off_genomes + align16(sizeof(PackGenome) * size_t(P));
+  h.off_edges = h.off_nodes + align16(sizeof(PackNode) * nn);
+  h.total_bytes = h.off_edges + align16(sizeof(PackEdge) * ne);
+  *used = size_t(h.total_bytes);
+  if (cap < h.total_bytes) return EMR_ERR_CAPACITY;
+  auto* base = static_cast<uint8_t*>(buf);
+  std::memset(base, 0, size_t(h.total_bytes));
+  auto* gt = reinterpret_cast<PackGenome*>(base + h.off_genomes);
+  auto* nt = reinterpret_cast<PackNode*>(base + h.off_nodes);
+  auto* et = reinterpret_cast<PackEdge*>(base + h.off_edges);
+  uint32_t nb = 0, eb = 0;
+  for (int g = 0; g < P; g++) {
+    PackGenome pg = gs[g].g;
+    pg.node_beg = nb;
+    pg.edge_beg = eb;
+    std::copy(gs[g].nodes.begin(), gs[g].nodes.end(), nt + nb);
+    std::copy(gs[g].edges.begin(), gs[g].edges.end(), et + eb);
+    nb += uint32_t(gs[g].nodes.size());
+    eb += uint32_t(gs[g].edges.size());
+    gt[g] = pg;
+    h.max_nodes = std::max<int32_t>(h.max_nodes, pg.n_nodes);
+    h.max_edges = std::max<int32_t>(h.max_edges, pg.n_edges);
+    for (int s = 0; s < 2; s++) {
+      h.max_varying[s] = std::max<int32_t>(h.max_varying[s], pg.n_varying[s]);
+      h.max_vedges[s] = std::max<int32_t>(h.max_vedges[s], pg.n_vedges[s]);
+    }
+  }
+  std::memcpy(base, &h, sizeof h);
+  return EMR_OK;
+}
+
+emr_status emr_pack_info(const void* pack_host, int32_t* P, int32_t* max_varying_out, int32_t* max_varying_in) {
+  if (!pack_host) return EMR_ERR_ARG;
+  const PackHeader* h = pack_header(pack_host);
+  if (h->magic != kPackMagic || h->version != kPackVersion) return EMR_ERR_ARG;
+  if (P) *P = h->P;
+  if (max_varying_out) *max_varying_out = h->max_varying[EMR_SIDE_OUT];
+  if (max_varying_in) *max_varying_in = h->max_varying[EMR_SIDE_IN];
+  return EMR_OK;
+}
+
+const char* emr_strerror(emr_status s) {
+  switch (s) {
+    case EMR_OK: return "ok";
+    case EMR_ERR_ARG: return "invalid argument";
+    case EMR_ERR_CYCLE: return "genome has a cycle among its enabled connections";
+    case EMR_ERR_RANGE: return "size beyond a documented limit";
+    case EMR_ERR_CAPACITY: return "output buffer or workspace too small";
+    case EMR_ERR_CUDA: return "CUDA error";
+    case EMR_ERR_TIMEOUT: return "host-side wait timed out";
+    case EMR_ERR_ALLOC: return "host allocation failed";
+    default: return "unknown status";
+  }
+}
+
+int32_t emr_version(void) { return 100; }
+
+}  // extern "C"

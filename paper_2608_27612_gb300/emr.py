@@ -1,0 +1,326 @@
+"""Thin ctypes binding of libemr's C ABI (include/emr.h), same names, no compute.
+
+Device buffers are torch tensors (passed by data_ptr); streams are torch
+streams. Every step of the path runs in libemr's kernels: this module only
+marshals arguments, allocates caller-owned buffers for the convenience
+wrappers and turns status codes into exceptions. There is no fallback: if the
+library has not been built, loading it raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from dataclasses import dataclass
+
+import numpy as np
+import torch
+
+from . import _build
+
+EMR_OK, EMR_ERR_ARG, EMR_ERR_CYCLE, EMR_ERR_RANGE, EMR_ERR_CAPACITY, EMR_ERR_CUDA, EMR_ERR_TIMEOUT, \
+    EMR_ERR_ALLOC = range(8)
+EMR_MAX_DEPTH = 14
+EMR_EAGER, EMR_GATED = 0, 1
+_M = EMR_MAX_DEPTH + 2
+
+_lib = None
+
+
+class EmrError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__("%s: %s (status %d)" % (what, strerror(status) if _lib else "?", status))
+
+
+class Grid(C.Structure):
+    _fields_ = [("D", C.c_int32), ("reserved", C.c_int32), ("n_total", C.c_int64), ("n_halo", C.c_int64),
+                ("n_words", C.c_int64), ("chunk", C.c_int64), ("level_off", C.c_int64 * _M),
+                ("halo_off", C.c_int64 * _M), ("word_off", C.c_int64 * _M)]
+
+
+class QueryC(C.Structure):
+    _fields_ = [("S", C.c_int32), ("per_genome", C.c_int32), ("a_host", C.c_void_p), ("b_host", C.c_void_p),
+                ("side_host", C.c_void_p), ("count_host", C.c_void_p), ("a_dev", C.c_void_p),
+                ("b_dev", C.c_void_p), ("side_dev", C.c_void_p), ("count_dev", C.c_void_p)]
+
+
+def lib() -> C.CDLL:
+    """Load libemr (after torch, so both share one CUDA runtime). Raises if it is not built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_build.LIB):
+            raise RuntimeError("libemr is not built (%s missing): run __graft_entry__.build()" % _build.LIB)
+        _lib = C.CDLL(_build.LIB)
+        vp, i32, i64, f32, sz = C.c_void_p, C.c_int32, C.c_int64, C.c_float, C.c_size_t
+        sig = {
+            "emr_grid_build": [i32, i64, vp],
+            "emr_index_to_ij": [i64, vp, vp, vp],
+            "emr_pack_size": [i32, vp, vp, vp],
+            "emr_pack_population": [i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp, vp],
+            "emr_pack_info": [vp, vp, vp, vp],
+            "emr_eval_workspace_size": [vp, vp, vp],
+            "emr_eval_prepare": [vp, vp, vp, vp, sz, vp],
+            "emr_eval": [vp, vp, vp, vp, vp, vp, sz, vp],
+            "emr_variance_filter": [vp, vp, vp, i32, i32, f32, f32, f32, i32, vp, vp, vp, vp, vp],
+            "emr_mask_combine": [vp, vp, vp, i32, i32, vp, vp],
+            "emr_eval_filter": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
+            "emr_compact_workspace_size": [vp, i32, vp],
+            "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
+            "emr_version": [],
+        }
+        for name, args in sig.items():
+            f = getattr(_lib, name)
+            f.argtypes = args
+            f.restype = C.c_int32
+        _lib.emr_strerror.argtypes = [C.c_int32]
+        _lib.emr_strerror.restype = C.c_char_p
+    return _lib
+
+
+def strerror(status: int) -> str:
+    return lib().emr_strerror(status).decode()
+
+
+def _check(status: int, what: str):
+    if status != EMR_OK:
+        raise EmrError(status, what)
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    if isinstance(x, torch.Tensor):
+        return C.c_void_p(x.data_ptr())
+    if isinstance(x, np.ndarray):
+        return x.ctypes.data_as(C.c_void_p)
+    return x
+
+
+def _stream(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return C.c_void_p(s.cuda_stream)
+
+
+# ---- a1 -----------------------------------------------------------------------
+
+def grid_build(D: int, chunk: int = 0) -> Grid:
+    g = Grid()
+    _check(lib().emr_grid_build(D, chunk, C.byref(g)), "emr_grid_build")
+    return g
+
+
+def index_to_ij(gidx: int):
+    d, i, j = C.c_int32(), C.c_int32(), C.c_int32()
+    _check(lib().emr_index_to_ij(gidx, C.byref(d), C.byref(i), C.byref(j)), "emr_index_to_ij")
+    return d.value, i.value, j.value
+
+
+# ---- a2 -----------------------------------------------------------------------
+
+def pack_population(pop) -> np.ndarray:
+    """Packed blob (numpy uint8) of a workloads.Population."""
+    L = lib()
+    n = C.c_size_t()
+    _check(L.emr_pack_size(pop.P, _ptr(pop.node_ptr), _ptr(pop.conn_ptr), C.byref(n)), "emr_pack_size")
+    buf = np.zeros(n.value + 16, np.uint8)
+    used, bad = C.c_size_t(), C.c_int32()
+    st = L.emr_pack_population(pop.P, _ptr(pop.node_ptr), _ptr(pop.node_id), _ptr(pop.node_kind),
+                               _ptr(pop.node_act), _ptr(pop.node_bias), _ptr(pop.conn_ptr), _ptr(pop.conn_src),
+                               _ptr(pop.conn_dst), _ptr(pop.conn_w), _ptr(pop.conn_enabled), _ptr(buf),
+                               C.c_size_t(len(buf)), C.byref(used), C.byref(bad))
+    if st != EMR_OK:
+        e = EmrError(st, "emr_pack_population (genome %d)" % bad.value)
+        e.bad_genome = bad.value
+        raise e
+    return buf[:used.value].copy()
+
+
+def pack_info(pack: np.ndarray):
+    P, mo, mi = C.c_int32(), C.c_int32(), C.c_int32()
+    _check(lib().emr_pack_info(_ptr(pack), C.byref(P), C.byref(mo), C.byref(mi)), "emr_pack_info")
+    return P.value, mo.value, mi.value
+
+
+@dataclass
+class Query:
+    """Host and device copies of the query slots (workloads.Sources)."""
+    a: np.ndarray
+    b: np.ndarray
+    side: np.ndarray
+    count: np.ndarray | None
+    a_dev: torch.Tensor
+    b_dev: torch.Tensor
+    side_dev: torch.Tensor
+    count_dev: torch.Tensor | None
+    S: int
+    per_genome: bool
+
+    @property
+    def c(self) -> QueryC:
+        q = QueryC()
+        q.S, q.per_genome = self.S, 1 if self.per_genome else 0
+        q.a_host, q.b_host, q.side_host = (self.a.ctypes.data, self.b.ctypes.data, self.side.ctypes.data)
+        q.count_host = self.count.ctypes.data if self.count is not None else None
+        q.a_dev, q.b_dev, q.side_dev = (self.a_dev.data_ptr(), self.b_dev.data_ptr(), self.side_dev.data_ptr())
+        q.count_dev = self.count_dev.data_ptr() if self.count_dev is not None else None
+        return q
+
+
+def make_query(sources, device="cuda") -> Query:
+    a = np.ascontiguousarray(sources.a, np.float32)
+    b = np.ascontiguousarray(sources.b, np.float32)
+    s = np.ascontiguousarray(sources.side, np.int32)
+    cnt = None if sources.count is None else np.ascontiguousarray(sources.count, np.int32)
+    dev = lambda x: torch.from_numpy(x).to(device) if x is not None else None
+    return Query(a, b, s, cnt, dev(a), dev(b), dev(s), dev(cnt), int(a.shape[-1]), a.ndim == 2)
+
+
+# ---- workspace sizes ------------------------------------------------------------
+
+def eval_workspace_size(pack: np.ndarray, query: Query) -> int:
+    n = C.c_size_t()
+    q = query.c
+    _check(lib().emr_eval_workspace_size(_ptr(pack), C.byref(q), C.byref(n)), "emr_eval_workspace_size")
+    return n.value
+
+
+def compact_workspace_size(grid: Grid, n_pairs: int) -> int:
+    n = C.c_size_t()
+    _check(lib().emr_compact_workspace_size(C.byref(grid), n_pairs, C.byref(n)), "emr_compact_workspace_size")
+    return n.value
+
+
+# ---- a3..a6 -----------------------------------------------------------------------
+
+def eval_prepare(pack, pack_dev, query: Query, ws, stream=None):
+    q = query.c
+    _check(lib().emr_eval_prepare(_ptr(pack), _ptr(pack_dev), C.byref(q), _ptr(ws), C.c_size_t(ws.numel()),
+                                  _stream(stream)), "emr_eval_prepare")
+
+
+def eval(pack, query: Query, grid: Grid, out, out_halo, ws, stream=None):
+    q = query.c
+    _check(lib().emr_eval(_ptr(pack), C.byref(q), C.byref(grid), _ptr(out), _ptr(out_halo), _ptr(ws),
+                          C.c_size_t(ws.numel()), _stream(stream)), "emr_eval")
+
+
+def variance_filter(out, out_halo, grid: Grid, P: int, S: int, theta: float, band: float, w_min: float, mode: int,
+                    mask, split, band_bits, var_dbg=None, stream=None):
+    _check(lib().emr_variance_filter(_ptr(out), _ptr(out_halo), C.byref(grid), P, S, theta, band, w_min, mode,
+                                     _ptr(mask), _ptr(split), _ptr(band_bits), _ptr(var_dbg), _stream(stream)),
+           "emr_variance_filter")
+
+
+def mask_combine(split, band_bits, grid: Grid, n_pairs: int, mode: int, mask, stream=None):
+    _check(lib().emr_mask_combine(_ptr(split), _ptr(band_bits), C.byref(grid), n_pairs, mode, _ptr(mask),
+                                  _stream(stream)), "emr_mask_combine")
+
+
+def eval_filter(pack, query: Query, grid: Grid, theta: float, band: float, w_min: float, split, band_bits, out, ws,
+                stream=None):
+    q = query.c
+    _check(lib().emr_eval_filter(_ptr(pack), C.byref(q), C.byref(grid), theta, band, w_min, _ptr(split),
+                                 _ptr(band_bits), _ptr(out), _ptr(ws), C.c_size_t(ws.numel()), _stream(stream)),
+           "emr_eval_filter")
+
+
+def compact(mask, out, grid: Grid, n_pairs: int, idx, w, cap: int, counts, offsets, ws, stream=None):
+    _check(lib().emr_compact(_ptr(mask), _ptr(out), C.byref(grid), n_pairs, _ptr(idx), _ptr(w), cap, _ptr(counts),
+                             _ptr(offsets), _ptr(ws), C.c_size_t(ws.numel()), _stream(stream)), "emr_compact")
+
+
+# ---- convenience: the whole path on caller-visible buffers --------------------------
+
+class Discovery:
+    """Buffers and calls for one (population, query, depth) configuration.
+
+    run_fused(): CPPN outputs never materialised (only kept-candidate weights are written).
+    run_unfused(): CPPN outputs materialised, then filtered.
+    """
+
+    def __init__(self, pop, sources, D: int, theta: float, band: float, w_min: float = 0.0,
+                 mode: int = EMR_EAGER, cap: int | None = None, materialise: bool = False, device="cuda"):
+        self.device = torch.device(device)
+        self.pack = pack_population(pop)
+        self.pack_dev = torch.from_numpy(self.pack).to(self.device)
+        self.query = make_query(sources, self.device)
+        self.grid = grid_build(D)
+        self.P, self.S = pop.P, self.query.S
+        self.n_pairs = self.P * self.S
+        self.theta, self.band, self.w_min, self.mode = theta, band, w_min, mode
+        g = self.grid
+        u32 = dict(dtype=torch.int32, device=self.device)
+        self.mask = torch.zeros(self.n_pairs, g.n_words, **u32)
+        self.split = torch.zeros(self.n_pairs, g.n_words, **u32)
+        self.band_bits = torch.zeros(self.n_pairs, g.n_words, **u32)
+        self.out = torch.zeros(self.n_pairs, g.n_total, dtype=torch.float32, device=self.device)
+        self.out_halo = (torch.zeros(self.n_pairs, g.n_halo, dtype=torch.float32, device=self.device)
+                         if materialise else None)
+        self.var_dbg = None
+        self.ws = torch.zeros(eval_workspace_size(self.pack, self.query), dtype=torch.uint8, device=self.device)
+        self.cws = torch.zeros(compact_workspace_size(g, self.n_pairs), dtype=torch.uint8, device=self.device)
+        self.cap = int(cap if cap is not None else min(self.n_pairs * g.n_total, 1 << 27))
+        self.idx = torch.zeros(self.cap, dtype=torch.int32, device=self.device)
+        self.w = torch.zeros(self.cap, dtype=torch.float32, device=self.device)
+        self.counts = torch.zeros(self.n_pairs, dtype=torch.int64, device=self.device)
+        self.offsets = torch.zeros(self.n_pairs + 1, dtype=torch.int64, device=self.device)
+
+    def prepare(self, stream=None):
+        eval_prepare(self.pack, self.pack_dev, self.query, self.ws, stream)
+
+    def run_fused(self, stream=None):
+        """emr_eval_prepare, emr_eval_filter, emr_mask_combine, emr_compact."""
+        self.prepare(stream)
+        eval_filter(self.pack, self.query, self.grid, self.theta, self.band, self.w_min, self.split,
+                    self.band_bits, self.out, self.ws, stream)
+        mask_combine(self.split, self.band_bits, self.grid, self.n_pairs, self.mode, self.mask, stream)
+        compact(self.mask, self.out, self.grid, self.n_pairs, self.idx, self.w, self.cap, self.counts,
+                self.offsets, self.cws, stream)
+
+    def run_unfused(self, with_var: bool = False, stream=None):
+        """emr_eval_prepare, emr_eval, emr_variance_filter, emr_compact."""
+        if self.out_halo is None:
+            self.out_halo = torch.zeros(self.n_pairs, self.grid.n_halo, dtype=torch.float32, device=self.device)
+        if with_var and self.var_dbg is None:
+            self.var_dbg = torch.zeros(self.n_pairs, self.grid.n_total, dtype=torch.float32, device=self.device)
+        self.prepare(stream)
+        eval(self.pack, self.query, self.grid, self.out, self.out_halo, self.ws, stream)
+        variance_filter(self.out, self.out_halo, self.grid, self.P, self.S, self.theta, self.band, self.w_min,
+                        self.mode, self.mask, self.split, self.band_bits, self.var_dbg if with_var else None,
+                        stream)
+        compact(self.mask, self.out, self.grid, self.n_pairs, self.idx, self.w, self.cap, self.counts,
+                self.offsets, self.cws, stream)
+
+    def lists(self):
+        """Host copies: per pair (idx, w) arrays, ascending global index."""
+        off = self.offsets.cpu().numpy()
+        total = int(off[-1])
+        if total > self.cap:
+            raise EmrError(EMR_ERR_CAPACITY, "compaction capacity %d < %d" % (self.cap, total))
+        idx = self.idx[:total].cpu().numpy()
+        w = self.w[:total].cpu().numpy()
+        return [(idx[off[r]:off[r + 1]], w[off[r]:off[r + 1]]) for r in range(self.n_pairs)]
+
+
+# ---- inspection of a packed blob (layout of csrc/emr_internal.h) ----------------------
+
+_HDR = np.dtype([("magic", "<u4"), ("version", "<u4"), ("P", "<i4"), ("max_nodes", "<i4"),
+                 ("max_varying", "<i4", 2), ("max_vedges", "<i4", 2), ("max_edges", "<i4"), ("reserved", "<i4"),
+                 ("off_genomes", "<u8"), ("off_nodes", "<u8"), ("off_edges", "<u8"), ("total", "<u8")])
+_GEN = np.dtype([("node_beg", "<u4"), ("edge_beg", "<u4"), ("n_nodes", "<u2"), ("n_edges", "<u2"),
+                 ("n_varying", "<u2", 2), ("n_vedges", "<u2", 2), ("cost", "<u4", 2), ("reserved", "<u4")])
+_NODE = np.dtype([("act", "u1"), ("vary", "u1"), ("reserved", "<u2"), ("edge_beg", "<u2"), ("edge_cnt", "<u2"),
+                  ("bias", "<f4"), ("w_in", "<f4", 5)])
+_EDGE = np.dtype([("src", "<u2"), ("reserved", "<u2"), ("w", "<f4")])
+
+
+def pack_records(pack: np.ndarray):
+    """(header, genome table, node records, edge records) of a packed blob, as numpy views."""
+    raw = np.ascontiguousarray(pack).tobytes()
+    h = np.frombuffer(raw[:_HDR.itemsize], _HDR)[0]
+    P = int(h["P"])
+    gs = np.frombuffer(raw, _GEN, P, int(h["off_genomes"]))
+    nn = int(gs["n_nodes"].astype(np.int64).sum())
+    ne = int(gs["n_edges"].astype(np.int64).sum())
+    return h, gs, np.frombuffer(raw, _NODE, nn, int(h["off_nodes"])), np.frombuffer(raw, _EDGE, ne,
+                                                                                    int(h["off_edges"]))

@@ -1,0 +1,169 @@
+"""Host-side checks of libemr's C ABI (no GPU): the library loads and exports
+every declared entry point; the grid descriptor, index inverse and genome packer
+behave as documented. The packer's results are compared with the oracle's
+independent genome handling where both apply."""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_27612_gb300 import emr
+from paper_2608_27612_gb300 import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+X1, Y1, X2, Y2, BIAS, HID, OUT = range(7)
+IDN, SIG, TNH, GAU, SIN, ABS = range(6)
+
+
+def declared_symbols():
+    names = set()
+    inc = os.path.join(ROOT, "include")
+    for f in os.listdir(inc):
+        if f.endswith(".h"):
+            txt = open(os.path.join(inc, f)).read()
+            names |= set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(emr_\w+)\s*\(", txt, re.M))
+    return names
+
+
+def test_library_exports_every_declared_symbol():
+    L = emr.lib()
+    names = declared_symbols()
+    assert {"emr_grid_build", "emr_pack_population", "emr_eval", "emr_variance_filter", "emr_eval_filter",
+            "emr_compact"} <= names
+    for n in sorted(names):
+        assert hasattr(L, n), n
+    assert emr.strerror(emr.EMR_ERR_CYCLE).startswith("genome has a cycle")
+
+
+@pytest.mark.parametrize("D", [0, 1, 4, 7, 13, 14])
+def test_grid_descriptor_matches_eq1_counts(D):
+    g = emr.grid_build(D)
+    assert g.n_total == oracle.n_total(D) and g.n_halo == oracle.n_halo(D)
+    for d in range(D + 1):
+        assert g.level_off[d] == oracle.index(d, 0, 0)
+        assert g.halo_off[d] == 8 * (2 ** d - 1)
+        assert g.word_off[d + 1] - g.word_off[d] == -(-(4 ** (d + 1)) // 32)
+    assert g.level_off[D + 1] == g.n_total and g.word_off[D + 1] == g.n_words
+
+
+def test_grid_descriptor_errors():
+    with pytest.raises(emr.EmrError) as e:
+        emr.grid_build(15)
+    assert e.value.status == emr.EMR_ERR_RANGE
+    with pytest.raises(emr.EmrError):
+        emr.grid_build(-1)
+    for bad in (1000, 4095, 6000):
+        with pytest.raises(emr.EmrError) as e:
+            emr.grid_build(5, bad)
+        assert e.value.status == emr.EMR_ERR_ARG
+    assert emr.grid_build(13, 1 << 26).chunk == 1 << 26
+
+
+def test_index_to_ij_inverts_the_numbering():
+    rng = np.random.default_rng(0)
+    for _ in range(2000):
+        d = int(rng.integers(0, 15))
+        n = 2 ** (d + 1)
+        i, j = int(rng.integers(0, n)), int(rng.integers(0, n))
+        assert emr.index_to_ij(oracle.index(d, i, j)) == (d, i, j)
+    with pytest.raises(emr.EmrError):
+        emr.index_to_ij(-1)
+    with pytest.raises(emr.EmrError):
+        emr.index_to_ij(oracle.n_total(14))
+
+
+def _genome(nodes, conns):
+    return W.population_from_lists([([(k, k, IDN, 0.0) for k in range(5)] + nodes, conns)])
+
+
+def _pack_records(blob):
+    """Decode the blob (layout of csrc/emr_internal.h) for white-box checks."""
+    h = np.frombuffer(blob[:72].tobytes(), dtype=np.dtype([
+        ("magic", "<u4"), ("version", "<u4"), ("P", "<i4"), ("max_nodes", "<i4"), ("max_varying", "<i4", 2),
+        ("max_vedges", "<i4", 2), ("max_edges", "<i4"), ("reserved", "<i4"), ("off_genomes", "<u8"),
+        ("off_nodes", "<u8"), ("off_edges", "<u8"), ("total", "<u8")]))[0]
+    gdt = np.dtype([("node_beg", "<u4"), ("edge_beg", "<u4"), ("n_nodes", "<u2"), ("n_edges", "<u2"),
+                    ("n_varying", "<u2", 2), ("n_vedges", "<u2", 2), ("cost", "<u4", 2), ("reserved", "<u4")])
+    ndt = np.dtype([("act", "u1"), ("vary", "u1"), ("r", "<u2"), ("edge_beg", "<u2"), ("edge_cnt", "<u2"),
+                    ("bias", "<f4"), ("w_in", "<f4", 5)])
+    P = int(h["P"])
+    gs = np.frombuffer(blob.tobytes(), gdt, P, int(h["off_genomes"]))
+    nn = int(gs["n_nodes"].astype(np.int64).sum())
+    nodes = np.frombuffer(blob.tobytes(), ndt, nn, int(h["off_nodes"]))
+    return h, gs, nodes
+
+
+def test_pack_topological_order_dead_nodes_and_variation_flags():
+    # hidden 12 (x2) -> 10 (sin) -> out; hidden 7 depends only on the source (x1) -> out;
+    # hidden 9 is dead (feeds nothing that reaches the output).
+    nodes = [(5, OUT, TNH, 0.0), (10, HID, SIN, 0.5), (12, HID, GAU, 0.0), (7, HID, SIG, 0.0), (9, HID, ABS, 0.0)]
+    conns = [(12, 10, 1.0, True), (X2, 12, 2.0, True), (10, 5, 3.0, True), (X1, 7, 1.5, True), (7, 5, -1.0, True),
+             (Y2, 9, 1.0, True), (12, 9, 1.0, True), (Y1, 5, 0.25, False)]
+    pop = _genome(nodes, conns)
+    blob = emr.pack_population(pop)
+    h, gs, nd = _pack_records(blob)
+    assert h["magic"] == 0x504D5245 and h["P"] == 1
+    g = gs[0]
+    assert g["n_nodes"] == 4  # 9 dropped
+    # Kahn with ties by id: 7 and 12 are ready first (7 < 12), then 10, then the output
+    assert list(nd["act"]) == [SIG, GAU, SIN, TNH]
+    assert nd["w_in"][0][X1] == np.float32(1.5) and nd["w_in"][1][X2] == np.float32(2.0)
+    # OUT side: x2/y2 vary -> 12, 10, out vary, 7 is constant; IN side: x1/y1 vary -> 7 and out vary
+    assert [int(v) & 1 for v in nd["vary"]] == [0, 1, 1, 1]
+    assert [(int(v) >> 1) & 1 for v in nd["vary"]] == [1, 0, 0, 1]
+    assert tuple(g["n_varying"]) == (3, 2)
+    assert emr.pack_info(blob) == (1, 3, 2)
+
+
+def test_pack_rejects_like_the_oracle():
+    cyc = _genome([(5, OUT, IDN, 0.0), (6, HID, SIG, 0.0), (7, HID, SIG, 0.0)],
+                  [(X2, 6, 1.0, True), (6, 7, 1.0, True), (7, 6, 1.0, True), (7, 5, 1.0, True)])
+    good = W.random_population(3, seed=1)
+    pop = W.population_from_lists([good.genome(0), good.genome(1), cyc.genome(0), good.genome(2)])
+    with pytest.raises(emr.EmrError) as e:
+        emr.pack_population(pop)
+    assert e.value.status == emr.EMR_ERR_CYCLE and e.value.bad_genome == 2
+    assert oracle.check_population(pop) == (oracle.ORA_ERR_CYCLE, 2)
+    for bad in ([(5, OUT, IDN, 0.0), (6, OUT, IDN, 0.0)], [(5, HID, IDN, 0.0)]):
+        with pytest.raises(emr.EmrError) as e:
+            emr.pack_population(_genome(bad, []))
+        assert e.value.status == emr.EMR_ERR_ARG
+    with pytest.raises(emr.EmrError) as e:
+        emr.pack_population(_genome([(5, OUT, IDN, 0.0)], [(5, X2, 1.0, True)]))
+    assert e.value.status == emr.EMR_ERR_ARG
+    with pytest.raises(emr.EmrError) as e:  # unknown connection endpoint
+        emr.pack_population(_genome([(5, OUT, IDN, 0.0)], [(77, 5, 1.0, True)]))
+    assert e.value.status == emr.EMR_ERR_ARG
+
+
+def test_pack_capacity_and_varying_limit():
+    pop = W.random_population(4, seed=3)
+    L = emr.lib()
+    used, bad = C.c_size_t(), C.c_int32()
+    small = np.zeros(64, np.uint8)
+    st = L.emr_pack_population(pop.P, emr._ptr(pop.node_ptr), emr._ptr(pop.node_id), emr._ptr(pop.node_kind),
+                               emr._ptr(pop.node_act), emr._ptr(pop.node_bias), emr._ptr(pop.conn_ptr),
+                               emr._ptr(pop.conn_src), emr._ptr(pop.conn_dst), emr._ptr(pop.conn_w),
+                               emr._ptr(pop.conn_enabled), emr._ptr(small), C.c_size_t(64), C.byref(used),
+                               C.byref(bad))
+    assert st == emr.EMR_ERR_CAPACITY and used.value > 64
+    # a chain of 70 varying hidden nodes exceeds the 64-node limit
+    nodes = [(5, OUT, IDN, 0.0)] + [(100 + k, HID, IDN, 0.0) for k in range(70)]
+    conns = [(X2, 100, 1.0, True)] + [(100 + k, 101 + k, 1.0, True) for k in range(69)] + [(169, 5, 1.0, True)]
+    with pytest.raises(emr.EmrError) as e:
+        emr.pack_population(_genome(nodes, conns))
+    assert e.value.status == emr.EMR_ERR_RANGE
+
+
+@pytest.mark.parametrize("cfg", ["c2", "c3", "c5"])
+def test_workload_populations_pack(cfg):
+    w = {"c2": lambda: W.c2(D=5), "c3": lambda: W.c3(), "c5": lambda: W.c5()}[cfg]()
+    blob = emr.pack_population(w.pop)
+    P, mo, mi = emr.pack_info(blob)
+    assert P == w.P and 1 <= mo <= 64 and 0 <= mi <= 64
+    assert oracle.check_population(w.pop) == (0, -1)
+    _, gs, _ = _pack_records(blob)
+    assert gs["n_varying"].max() <= 64 and gs["n_vedges"].max() <= 512

@@ -161,6 +161,20 @@ def algorithmic_work(pack, query, emr):
     return per[np.arange(len(gs))[:, None], side]  # [P, S, 2]
 
 
+def alu_probe(emr, sms):
+    """Measured FFMA and MUFU (ex2, rcp, sin) throughput in ops/s, and the FFMA:MUFU ratio."""
+    out = {}
+    names = {emr.PROBE_FFMA: "ffma", emr.PROBE_EX2: "ex2", emr.PROBE_RCP: "rcp", emr.PROBE_SIN: "sin"}
+    for op, nm in names.items():
+        iters = 4000 if op == emr.PROBE_FFMA else 500
+        emr.probe_alu(op, sms * 8, 50)
+        ops, ms = emr.probe_alu(op, sms * 8, iters)
+        out[nm + "_Gops"] = ops / (ms * 1e-3) / 1e9
+    mufu = min(out["ex2_Gops"], out["rcp_Gops"])
+    out["ffma_per_mufu"] = out["ffma_Gops"] / mufu
+    return out
+
+
 def oracle_baseline(w, genomes):
     import oracle
     oracle.build()
@@ -270,7 +284,8 @@ def main():
     work = algorithmic_work(dsc.pack, dsc.query, emr)   # [P, S, (fp32, mufu)] per query
     props = torch.cuda.get_device_properties(local)
     sms = props.multi_processor_count
-    ratio = FP32_PER_SM_CLK / MUFU_PER_SM_CLK
+    probe = alu_probe(emr, sms)
+    ratio = probe["ffma_per_mufu"] if probe else FP32_PER_SM_CLK / MUFU_PER_SM_CLK
     per_query_eq = np.maximum(work[..., 0], ratio * work[..., 1])
     work_eq = float(per_query_eq.sum()) * g.n_total
     tile_s = statistics.mean(tile_ms) / 1e3
@@ -280,8 +295,9 @@ def main():
                 "frac": achieved / peak, "traffic": None, "kernel": "tile_kernel (emr_eval_filter)",
                 "kernel_ms": tile_s * 1e3,
                 "fp32_ops_per_query": float(work[..., 0].mean()), "mufu_ops_per_query": float(work[..., 1].mean()),
-                "peak_basis": "%d SMs x %d FP32 lanes x %.0f MHz (max SM clock); MUFU weighted %g FP32 lane-ops"
-                              % (sms, FP32_PER_SM_CLK, SM_MAX_MHZ, ratio)}
+                "peak_basis": "%d SMs x %d FP32 lanes x %.0f MHz (max SM clock); a MUFU op weighs %.2f FP32 "
+                              "lane-ops (measured FFMA:MUFU throughput ratio)" % (sms, FP32_PER_SM_CLK, SM_MAX_MHZ, ratio),
+                "alu_probe": probe}
     if clocks:
         roofline["frac_at_sampled_clock"] = roofline["frac"] * SM_MAX_MHZ / clocks["sm_mhz"]
 

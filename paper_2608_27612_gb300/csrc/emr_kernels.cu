@@ -91,14 +91,28 @@ struct SpecLayout {
   int32_t nv_cap, nve_cap;
   __host__ __device__ int64_t coef_off() const { return 16; }
   __host__ __device__ int64_t edge_off() const { return 16 + 16 * int64_t(nv_cap); }
+  __host__ __device__ int64_t dense_off() const { return (edge_off() + 8 * int64_t(nve_cap) + 15) & ~int64_t(15); }
 };
+
+// Pairs with at most kDenseMax varying nodes also get a dense lower-triangular
+// weight block W[k][j] (row-major, kDenseMax x kDenseMax floats): the weight of
+// the edge from varying slot j to varying slot k, 0 where there is none.
+constexpr int kDenseMax = 12;
 
 inline SpecLayout spec_layout(int nv_cap, int nve_cap) {
   SpecLayout L;
   L.nv_cap = std::max(nv_cap, 1);
   L.nve_cap = std::max(nve_cap, 1);
-  L.stride = (16 + 16 * int64_t(L.nv_cap) + 8 * int64_t(L.nve_cap) + 15) & ~int64_t(15);
+  L.stride = (L.dense_off() + 4 * kDenseMax * kDenseMax + 15) & ~int64_t(15);
   return L;
+}
+
+// Kernel class of a pair by its varying-node count: 0 = interpreter (more than
+// kDenseMax), 1 = dense up to 12, 2 = dense up to 8, 3 = dense up to 4
+// (includes constant outputs). Classes run in this order, heaviest first.
+constexpr int kClasses = 4;
+__host__ __device__ __forceinline__ int pair_class(int nv) {
+  return nv > kDenseMax ? 0 : nv > 8 ? 1 : nv > 4 ? 2 : 3;
 }
 
 struct QueryDev {
@@ -107,31 +121,50 @@ struct QueryDev {
   int32_t S, per_genome;
 };
 
-// Cost-ordered pair schedule (heaviest first) by a counting sort in one CTA.
-constexpr int kCostBins = 1024;
+// Pair schedule: by kernel class (interpreter, dense-12, dense-8, dense-4), then by
+// estimated cost, heaviest first; a counting sort in one CTA.
+constexpr int kClassBins = 256;
+constexpr int kCostBins = kClasses * kClassBins;
 __global__ void schedule_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_t n_pairs,
                                 int32_t* __restrict__ order) {
   __shared__ int32_t hist[kCostBins];
-  __shared__ int32_t start[kCostBins];
+  __shared__ int32_t wsum[32];
   const PackHeader* h = reinterpret_cast<const PackHeader*>(pack);
   const PackGenome* gt = reinterpret_cast<const PackGenome*>(pack + h->off_genomes);
   for (int k = threadIdx.x; k < kCostBins; k += blockDim.x) hist[k] = 0;
   __syncthreads();
   auto bin_of = [&](int64_t r) {
-    int g = int(r / q.S), s = int(r % q.S);
-    int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
-    int side = q.side[si] ? 1 : 0;
-    uint32_t c = gt[g].cost[side];
-    return kCostBins - 1 - int(min(c, uint32_t(kCostBins - 1)));  // descending cost
+    const int g = int(r / q.S), s = int(r % q.S);
+    if (q.per_genome && q.count && s >= q.count[g]) return kCostBins - 1;  // unused: constant 0
+    const int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
+    const int side = q.side[si] ? 1 : 0;
+    const uint32_t c = min(gt[g].cost[side], uint32_t(kClassBins - 1));
+    return pair_class(gt[g].n_varying[side]) * kClassBins + (kClassBins - 1 - int(c));
   };
   for (int64_t r = threadIdx.x; r < n_pairs; r += blockDim.x) atomicAdd(&hist[bin_of(r)], 1);
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int acc = 0;
-    for (int k = 0; k < kCostBins; k++) { start[k] = acc; acc += hist[k]; }
+  // exclusive scan of the histogram (blockDim.x == 1024, one bin per thread)
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int v = threadIdx.x < kCostBins ? hist[threadIdx.x] : 0;
+  int x = v;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int t = wsum[lane];
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, t, o);
+      if (lane >= o) t += y;
+    }
+    wsum[lane] = t;
   }
   __syncthreads();
-  for (int64_t r = threadIdx.x; r < n_pairs; r += blockDim.x) order[atomicAdd(&start[bin_of(r)], 1)] = int32_t(r);
+  if (threadIdx.x < kCostBins) hist[threadIdx.x] = (warp ? wsum[warp - 1] : 0) + x - v;
+  __syncthreads();
+  for (int64_t r = threadIdx.x; r < n_pairs; r += blockDim.x) order[atomicAdd(&hist[bin_of(r)], 1)] = int32_t(r);
 }
 
 // One thread per pair: fold the constant inputs (the slot's node coordinates
@@ -149,7 +182,7 @@ __global__ void spec_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_
   uint8_t* rec = spec + r * L.stride;
   int32_t* hdr = reinterpret_cast<int32_t*>(rec);
   if (q.per_genome && q.count && s >= q.count[g]) {  // unused slot: constant 0, nothing kept
-    hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = 0;
+    hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = pair_class(0);
     return;
   }
   int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
@@ -182,6 +215,12 @@ __global__ void spec_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_
           c0 = fmaf(ed[e].w, cval[ed[e].src], c0);
         }
       }
+      for (int e = eb + 1; e < nve; e++) {  // ascending source slot (insertion sort, a few edges)
+        const uint2 key = ve[e];
+        int f = e - 1;
+        while (f >= eb && ve[f].x > key.x) { ve[f + 1] = ve[f]; f--; }
+        ve[f + 1] = key;
+      }
       uint32_t info = uint32_t(nd.act) | (uint32_t(eb) << 8) | (uint32_t(nve - eb) << 20);
       coef[nv] = make_float4(c0, nd.w_in[gx], nd.w_in[gy], __uint_as_float(info));
       cval[t] = __uint_as_float(uint32_t(nv));
@@ -194,10 +233,19 @@ __global__ void spec_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_
       out_const = cval[t];
     }
   }
+  if (nv <= kDenseMax) {
+    float* W = reinterpret_cast<float*>(rec + L.dense_off());
+    for (int k = 0; k < kDenseMax * kDenseMax; k++) W[k] = 0.f;
+    for (int k = 0; k < nv; k++) {
+      const uint32_t info = __float_as_uint(coef[k].w);
+      const int eb = int((info >> 8) & 0xfffu), ec = int(info >> 20);
+      for (int e = eb; e < eb + ec; e++) W[k * kDenseMax + int(ve[e].x)] += __uint_as_float(ve[e].y);
+    }
+  }
   hdr[0] = nv;
   hdr[1] = nve;
   reinterpret_cast<float*>(hdr)[2] = out_const;
-  hdr[3] = 0;
+  hdr[3] = pair_class(nv);
 }
 
 // ---- evaluation tiles ------------------------------------------------------------
@@ -208,6 +256,7 @@ struct TileArgs {
   const uint8_t* spec;
   SpecLayout L;
   const int32_t* order;
+  int64_t rank_beg;
   int32_t n_tiles, tile_beg;
   int32_t D, mode;
   float theta, band, w_min;
@@ -256,7 +305,7 @@ __device__ __forceinline__ void eval4_interp(const float4* __restrict__ coef, co
 __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
   extern __shared__ float4 smem4[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t rank = blockIdx.x / A.n_tiles;
+  const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
   const int tile = A.tile_beg + int(blockIdx.x % A.n_tiles);
   const int r = A.order[rank];
   const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
@@ -383,6 +432,243 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
       for (int c = 0; c < 4; c++)
         if (nib & (1u << c)) A.out[pair_pos + mb + 4 * q + c] = w[c];
     }
+  }
+}
+
+// ---- register-resident tiles (pairs with at most kDenseMax varying nodes) ---------
+//
+// A CTA of 256 threads owns one tile: either a 64 x 64 Morton block of one
+// depth >= 5, or (tile 0 of a pair) the whole of depths 0..4, one depth after
+// the other. Each thread evaluates sibling quads (the four children of one
+// parent cell) with the CPPN's node values in registers: node k is
+// act(c0 + wx x + wy y + sum_{j<k} W[k][j] v_j) with the loop unrolled to NVMAX
+// and a uniform early exit at the pair's node count, so every register index
+// is static. The quad's variance comes straight from its four results; the
+// band value needs the neighbours, taken from the tile in shared memory after
+// a barrier (the ring of out-of-tile neighbours is evaluated by the tile too).
+
+constexpr int kDThreads = 256;
+constexpr int kPyramidTop = 4;  // depths 0..4 (side <= 32) share one CTA
+
+struct DTileArgs {
+  const uint8_t* spec;
+  SpecLayout L;
+  const int32_t* order;
+  int64_t rank_beg;
+  int32_t n_tiles;
+  int32_t D, mode;
+  float theta, band, w_min;
+  int64_t n_total, n_halo, n_words;
+  int64_t level_off[EMR_MAX_DEPTH + 2], halo_off[EMR_MAX_DEPTH + 2], word_off[EMR_MAX_DEPTH + 2];
+  float* out;
+  float* out_halo;
+  uint32_t* split;
+  uint32_t* bandb;
+};
+
+template <int NP>
+__device__ __forceinline__ void act_applyN(int a, float (&z)[NP]) {
+  switch (a) {
+    case EMR_ACT_SIGMOID:
+#pragma unroll
+      for (int p = 0; p < NP; p++) z[p] = act_sigmoid(z[p]);
+      break;
+    case EMR_ACT_TANH:
+#pragma unroll
+      for (int p = 0; p < NP; p++) z[p] = act_tanh(z[p]);
+      break;
+    case EMR_ACT_GAUSS:
+#pragma unroll
+      for (int p = 0; p < NP; p++) z[p] = act_gauss(z[p]);
+      break;
+    case EMR_ACT_SIN:
+#pragma unroll
+      for (int p = 0; p < NP; p++) z[p] = act_sin(z[p]);
+      break;
+    case EMR_ACT_ABS:
+#pragma unroll
+      for (int p = 0; p < NP; p++) z[p] = fabsf(z[p]);
+      break;
+    default:
+      break;
+  }
+}
+
+// CPPN of one pair at NP points (x[p], y[p]); returns the output node's value.
+template <int NVMAX, int NP>
+__device__ __forceinline__ void eval_dense(const float4* __restrict__ coef, const float* __restrict__ W, int nv,
+                                           float out_const, const float (&x)[NP], const float (&y)[NP],
+                                           float (&w)[NP]) {
+  float v[NVMAX][NP];
+#pragma unroll
+  for (int p = 0; p < NP; p++) w[p] = out_const;
+#pragma unroll
+  for (int k = 0; k < NVMAX; k++) {
+    if (k >= nv) break;
+    const float4 c = coef[k];
+    float z[NP];
+#pragma unroll
+    for (int p = 0; p < NP; p++) z[p] = fmaf(c.z, y[p], fmaf(c.y, x[p], c.x));
+#pragma unroll
+    for (int j = 0; j < k; j++) {
+      const float wk = W[k * NVMAX + j];
+#pragma unroll
+      for (int p = 0; p < NP; p++) z[p] = fmaf(wk, v[j][p], z[p]);
+    }
+    act_applyN<NP>(int(__float_as_uint(c.w) & 0xffu), z);
+#pragma unroll
+    for (int p = 0; p < NP; p++) {
+      v[k][p] = z[p];
+      w[p] = z[p];
+    }
+  }
+}
+
+template <int NVMAX>
+__global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_dense(const DTileArgs A) {
+  static_assert(NVMAX <= kDenseMax, "dense block holds kDenseMax rows");
+  __shared__ float4 s_coef[NVMAX];
+  __shared__ __align__(16) float s_W[NVMAX * NVMAX];
+  __shared__ float s_wt[(kTileSide + 2) * (kTileSide + 2)];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
+  const int tile = int(blockIdx.x % A.n_tiles);
+  const int r = A.order[rank];
+  const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
+  const int nv = reinterpret_cast<const int32_t*>(rec)[0];
+  const float out_const = reinterpret_cast<const float*>(rec)[2];
+  const bool fused = A.mode == kModeFused;
+  if (tid < NVMAX)
+    s_coef[tid] = tid < nv ? reinterpret_cast<const float4*>(rec + A.L.coef_off())[tid] : make_float4(0, 0, 0, 0);
+  {
+    const float* gW = reinterpret_cast<const float*>(rec + A.L.dense_off());
+    for (int k = tid; k < NVMAX * NVMAX; k += kDThreads) s_W[k] = gW[(k / NVMAX) * kDenseMax + (k % NVMAX)];
+  }
+  // depth range of this tile
+  int d_lo, d_hi, tl = 0;
+  if (tile == 0) {
+    d_lo = 0;
+    d_hi = min(A.D, kPyramidTop);
+  } else {
+    int u = tile - 1, d = kPyramidTop + 1;
+    while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
+    d_lo = d_hi = d;
+    tl = u;
+  }
+  __syncthreads();
+  const int64_t prow = int64_t(r) * A.n_total;
+  for (int d = d_lo; d <= d_hi; d++) {
+    const int T = d + 1 < kTileLog ? (1 << (d + 1)) : kTileSide;
+    const int n = 1 << (d + 1);
+    const uint32_t mb = uint32_t(tl) * uint32_t(T * T);
+    const int i0 = int(compact1by1(mb)), j0 = int(compact1by1(mb >> 1));
+    const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1)
+    const int nq = T * T / 4, nring = 4 * T, pitch = T + 2;
+    const int64_t lrow = prow + A.level_off[d];
+    if (fused && nv == 0) {
+      // constant output: every variance and band value is exactly 0
+      for (int k = tid; k < (nq + 31) / 32; k += kDThreads)
+        if (d >= 1) A.split[int64_t(r) * A.n_words + A.word_off[d - 1] + (mb / 4) / 32 + k] = 0u;
+      for (int k = tid; k < (4 * nq + 31) / 32; k += kDThreads)
+        A.bandb[int64_t(r) * A.n_words + A.word_off[d] + mb / 32 + k] = 0u;
+      continue;
+    }
+    // phase 1: quads (four children of one parent) and the ring points
+    for (int base = 0; base < nq; base += kDThreads) {
+      const int q = base + tid;
+      const bool valid = q < nq;
+      float w[4] = {0.f, 0.f, 0.f, 0.f};
+      int pi = 0, pj = 0;
+      if (valid) {
+        pi = int(compact1by1(uint32_t(q)));
+        pj = int(compact1by1(uint32_t(q) >> 1));
+        const float xa = grid_coord(i0 + 2 * pi, scale), xb = grid_coord(i0 + 2 * pi + 1, scale);
+        const float ya = grid_coord(j0 + 2 * pj, scale), yb = grid_coord(j0 + 2 * pj + 1, scale);
+        const float x[4] = {xa, xb, xa, xb}, y[4] = {ya, ya, yb, yb};
+        eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
+        if (fused) {
+          const int li = 2 * pi + 1, lj = 2 * pj + 1;
+          s_wt[lj * pitch + li] = w[0];
+          s_wt[lj * pitch + li + 1] = w[1];
+          s_wt[(lj + 1) * pitch + li] = w[2];
+          s_wt[(lj + 1) * pitch + li + 1] = w[3];
+        } else {
+          *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+        }
+      }
+      if (fused && d >= 1) {
+        // the four children give the parent's variance (Section 3.2)
+        const float m = 0.25f * ((w[0] + w[1]) + (w[2] + w[3]));
+        const float e0 = w[0] - m, e1 = w[1] - m, e2 = w[2] - m, e3 = w[3] - m;
+        const float V = 0.25f * ((e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3));
+        const unsigned bal = __ballot_sync(kFull, valid && V > A.theta);
+        const int q0 = base + warp * 32;
+        if (lane == 0 && q0 < nq)
+          A.split[int64_t(r) * A.n_words + A.word_off[d - 1] + (mb / 4 + uint32_t(q0)) / 32] = bal;
+      }
+    }
+    if (fused || A.out_halo) {
+      for (int t = tid; t < nring; t += kDThreads) {
+        const int sd = t / T, u = t - sd * T;
+        const int li = sd == 0 ? -1 : sd == 1 ? T : u, lj = sd == 2 ? -1 : sd == 3 ? T : u;
+        const int gi = i0 + li, gj = j0 + lj;
+        const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
+        if (!fused && !outside) continue;  // materialised: in-domain points belong to other tiles
+        const float x[1] = {grid_coord(gi, scale)}, y[1] = {grid_coord(gj, scale)};
+        float w[1];
+        eval_dense<NVMAX, 1>(s_coef, s_W, nv, out_const, x, y, w);
+        if (fused) {
+          s_wt[(lj + 1) * pitch + li + 1] = w[0];
+        } else {
+          const int hs = gi < 0 ? 0 : gi >= n ? 1 : gj < 0 ? 2 : 3;
+          A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? gj : gi)] = w[0];
+        }
+      }
+    }
+    if (!fused) continue;
+    __syncthreads();
+    // phase 2: band value of each position from its four neighbours at distance 2^-d
+    for (int base = 0; base < nq; base += kDThreads) {
+      const int q = base + tid;
+      const bool valid = q < nq;
+      unsigned nib = 0;
+      float w[4] = {0.f, 0.f, 0.f, 0.f};
+      if (valid) {
+        const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+        const int li = 2 * pi + 1, lj = 2 * pj + 1;
+        const float* r0 = s_wt + lj * pitch + li;  // position (2pi, 2pj)
+        w[0] = r0[0];
+        w[1] = r0[1];
+        w[2] = r0[pitch];
+        w[3] = r0[pitch + 1];
+        const float l0 = r0[-1], l2 = r0[pitch - 1];              // left of the a = 0 column
+        const float r1 = r0[2], r3 = r0[pitch + 2];               // right of the a = 1 column
+        const float b0 = r0[-pitch], b1 = r0[-pitch + 1];         // below the b = 0 row
+        const float t2 = r0[2 * pitch], t3 = r0[2 * pitch + 1];   // above the b = 1 row
+        const float L[4] = {l0, w[0], l2, w[2]}, R[4] = {w[1], r1, w[3], r3};
+        const float Bo[4] = {b0, b1, w[0], w[1]}, U[4] = {w[2], w[3], t2, t3};
+#pragma unroll
+        for (int c = 0; c < 4; c++) {
+          const float dl = fabsf(w[c] - L[c]), dr = fabsf(w[c] - R[c]);
+          const float db = fabsf(w[c] - Bo[c]), dt = fabsf(w[c] - U[c]);
+          const float B = fmaxf(fminf(dt, db), fminf(dl, dr));
+          const bool pass = B > A.band && (A.w_min <= 0.f || fabsf(w[c]) > A.w_min);
+          nib |= unsigned(pass) << c;
+        }
+      }
+      unsigned v = nib << (4 * (lane & 7));
+      v |= __shfl_xor_sync(kFull, v, 1);
+      v |= __shfl_xor_sync(kFull, v, 2);
+      v |= __shfl_xor_sync(kFull, v, 4);
+      if ((lane & 7) == 0 && valid)
+        A.bandb[int64_t(r) * A.n_words + A.word_off[d] + (mb + 4u * uint32_t(q)) / 32] = v;
+      if (A.out && nib) {
+#pragma unroll
+        for (int c = 0; c < 4; c++)
+          if (nib & (1u << c)) A.out[lrow + mb + 4 * q + c] = w[c];
+      }
+    }
+    __syncthreads();
   }
 }
 
@@ -626,6 +912,7 @@ GridDev grid_dev(const emr_grid* g) {
 
 struct EvalPlan {
   int64_t n_pairs;
+  int64_t n_class[kClasses];  // pairs per kernel class (schedule order)
   SpecLayout L;
   int32_t scratch_stride;
   size_t spec_bytes, scratch_bytes, order_bytes, total;
@@ -635,6 +922,8 @@ emr_status eval_plan(const void* pack_host, const emr_query* q, EvalPlan* p) {
   if (!pack_host || !q || q->S <= 0 || !q->a_host || !q->b_host || !q->side_host) return EMR_ERR_ARG;
   const PackHeader* h = pack_header(pack_host);
   if (h->magic != kPackMagic || h->version != kPackVersion || h->P <= 0) return EMR_ERR_ARG;
+  const PackGenome* gt =
+      reinterpret_cast<const PackGenome*>(static_cast<const uint8_t*>(pack_host) + h->off_genomes);
   bool sides[2] = {false, false};
   const int64_t ns = q->per_genome ? int64_t(h->P) * q->S : q->S;
   for (int64_t k = 0; k < ns; k++) {
@@ -645,6 +934,13 @@ emr_status eval_plan(const void* pack_host, const emr_query* q, EvalPlan* p) {
   for (int s = 0; s < 2; s++)
     if (sides[s]) { nv = std::max(nv, h->max_varying[s]); nve = std::max(nve, h->max_vedges[s]); }
   p->n_pairs = int64_t(h->P) * q->S;
+  for (int c = 0; c < kClasses; c++) p->n_class[c] = 0;
+  for (int g = 0; g < h->P; g++)
+    for (int s = 0; s < q->S; s++) {
+      if (q->per_genome && q->count_host && s >= q->count_host[g]) { p->n_class[pair_class(0)]++; continue; }
+      const int64_t si = q->per_genome ? int64_t(g) * q->S + s : s;
+      p->n_class[pair_class(gt[g].n_varying[q->side_host[si]])]++;
+    }
   p->L = spec_layout(nv, nve);
   p->scratch_stride = std::max(h->max_nodes, 1);
   p->spec_bytes = size_t(p->n_pairs) * size_t(p->L.stride);
@@ -691,47 +987,96 @@ size_t tile_smem_bytes(const SpecLayout& L) {
          4 * size_t(kTileSide + 2) * size_t(kTileSide + 2);
 }
 
+int64_t dense_tiles(int D) {
+  int64_t t = 1;
+  for (int d = kPyramidTop + 1; d <= D; d++) t += tiles_in_level(d);
+  return t;
+}
+
+template <int NVMAX>
+emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st) {
+  if (n_ranks <= 0) return EMR_OK;
+  DTileArgs A = A0;
+  A.rank_beg = rank_beg;
+  const int64_t blocks = n_ranks * int64_t(A.n_tiles);
+  if (blocks > 0x7fffffffLL) return EMR_ERR_RANGE;
+  tile_kernel_dense<NVMAX><<<unsigned(blocks), kDThreads, 0, st>>>(A);
+  return cuda_status(cudaGetLastError());
+}
+
 emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spec, const int32_t* order, int mode,
                         float theta, float band, float w_min, float* out, float* out_halo, uint32_t* split,
                         uint32_t* bandb, cudaStream_t st) {
-  TileArgs A{};
-  A.spec = spec;
-  A.L = p.L;
-  A.order = order;
-  A.D = g->D;
-  A.mode = mode;
-  A.theta = theta;
-  A.band = band;
-  A.w_min = w_min;
-  int32_t t = 0;
-  for (int d = 0; d <= g->D; d++) {
-    A.lvl_tile_beg[d] = t;
-    t += int32_t(tiles_in_level(d));
+  emr_status rc = EMR_OK;
+  // class 0: interpreter (more than kDenseMax varying nodes)
+  if (p.n_class[0] > 0) {
+    TileArgs A{};
+    A.spec = spec;
+    A.L = p.L;
+    A.order = order;
+    A.rank_beg = 0;
+    A.D = g->D;
+    A.mode = mode;
+    A.theta = theta;
+    A.band = band;
+    A.w_min = w_min;
+    int32_t t = 0;
+    for (int d = 0; d <= g->D; d++) {
+      A.lvl_tile_beg[d] = t;
+      t += int32_t(tiles_in_level(d));
+    }
+    for (int d = g->D + 1; d < EMR_MAX_DEPTH + 2; d++) A.lvl_tile_beg[d] = t;
+    A.n_tiles = t;
+    A.tile_beg = 0;
+    A.n_total = g->n_total;
+    A.n_halo = g->n_halo;
+    A.n_words = g->n_words;
+    for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {
+      A.level_off[d] = g->level_off[d];
+      A.halo_off[d] = g->halo_off[d];
+      A.word_off[d] = g->word_off[d];
+    }
+    A.out = out;
+    A.out_halo = out_halo;
+    A.split = split;
+    A.bandb = bandb;
+    const int64_t blocks = p.n_class[0] * int64_t(A.n_tiles);
+    if (blocks > 0x7fffffffLL) return EMR_ERR_RANGE;
+    const size_t smem = tile_smem_bytes(p.L);
+    if (smem > 227 * 1024) return EMR_ERR_RANGE;
+    cudaError_t e = cudaFuncSetAttribute(tile_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return EMR_ERR_CUDA;
+    tile_kernel<<<unsigned(blocks), kBlock, smem, st>>>(A);
+    if ((rc = cuda_status(cudaGetLastError())) != EMR_OK) return rc;
   }
-  for (int d = g->D + 1; d < EMR_MAX_DEPTH + 2; d++) A.lvl_tile_beg[d] = t;
-  A.n_tiles = t;
-  A.tile_beg = 0;
-  A.n_total = g->n_total;
-  A.n_halo = g->n_halo;
-  A.n_words = g->n_words;
+  DTileArgs D{};
+  D.spec = spec;
+  D.L = p.L;
+  D.order = order;
+  D.n_tiles = int32_t(dense_tiles(g->D));
+  D.D = g->D;
+  D.mode = mode;
+  D.theta = theta;
+  D.band = band;
+  D.w_min = w_min;
+  D.n_total = g->n_total;
+  D.n_halo = g->n_halo;
+  D.n_words = g->n_words;
   for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {
-    A.level_off[d] = g->level_off[d];
-    A.halo_off[d] = g->halo_off[d];
-    A.word_off[d] = g->word_off[d];
+    D.level_off[d] = g->level_off[d];
+    D.halo_off[d] = g->halo_off[d];
+    D.word_off[d] = g->word_off[d];
   }
-  A.out = out;
-  A.out_halo = out_halo;
-  A.split = split;
-  A.bandb = bandb;
-  const int64_t blocks = p.n_pairs * int64_t(A.n_tiles);
-  if (blocks <= 0) return EMR_OK;
-  if (blocks > 0x7fffffffLL) return EMR_ERR_RANGE;
-  const size_t smem = tile_smem_bytes(p.L);
-  if (smem > 227 * 1024) return EMR_ERR_RANGE;
-  cudaError_t e = cudaFuncSetAttribute(tile_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-  if (e != cudaSuccess) return EMR_ERR_CUDA;
-  tile_kernel<<<unsigned(blocks), kBlock, smem, st>>>(A);
-  return cuda_status(cudaGetLastError());
+  D.out = out;
+  D.out_halo = out_halo;
+  D.split = split;
+  D.bandb = bandb;
+  int64_t beg = p.n_class[0];
+  if ((rc = launch_dense<12>(D, beg, p.n_class[1], st)) != EMR_OK) return rc;
+  beg += p.n_class[1];
+  if ((rc = launch_dense<8>(D, beg, p.n_class[2], st)) != EMR_OK) return rc;
+  beg += p.n_class[2];
+  return launch_dense<4>(D, beg, p.n_class[3], st);
 }
 
 emr_status launch_combine(const uint32_t* split, const uint32_t* bandb, const emr_grid* g, int64_t n_pairs, int gated,

@@ -67,6 +67,7 @@ def lib() -> C.CDLL:
             "emr_compact_workspace_size": [vp, i32, vp],
             "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_version": [],
+            "emr_probe_alu": [i32, i32, i32, vp, vp, vp, vp],
         }
         for name, args in sig.items():
             f = getattr(_lib, name)
@@ -227,6 +228,20 @@ def eval_filter(pack, query: Query, grid: Grid, theta: float, band: float, w_min
 def compact(mask, out, grid: Grid, n_pairs: int, idx, w, cap: int, counts, offsets, ws, stream=None):
     _check(lib().emr_compact(_ptr(mask), _ptr(out), C.byref(grid), n_pairs, _ptr(idx), _ptr(w), cap, _ptr(counts),
                              _ptr(offsets), _ptr(ws), C.c_size_t(ws.numel()), _stream(stream)), "emr_compact")
+
+
+# ---- ALU probes (roofline denominators) -------------------------------------------------
+
+PROBE_FFMA, PROBE_EX2, PROBE_RCP, PROBE_SIN = range(4)
+
+
+def probe_alu(op: int, blocks: int, iters: int, stream=None):
+    """(operations, milliseconds) of one probe launch (include/emr_probe.h)."""
+    sink = torch.zeros(blocks, dtype=torch.float32, device="cuda")
+    ops, ms = C.c_double(), C.c_float()
+    _check(lib().emr_probe_alu(op, blocks, iters, C.byref(ops), C.byref(ms), _ptr(sink), _stream(stream)),
+           "emr_probe_alu")
+    return ops.value, ms.value
 
 
 # ---- convenience: the whole path on caller-visible buffers --------------------------

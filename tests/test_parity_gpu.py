@@ -18,7 +18,7 @@ X1, Y1, X2, Y2, BIAS, HID, OUT = range(7)
 IDN, SIG, TNH, GAU, SIN, ABS = range(6)
 
 
-def run_gpu(w, mode=emr.EMR_EAGER, unfused=True, fused=True, cap=None):
+def run_gpu(w, mode=emr.EMR_EAGER, unfused=True, fused=True, cap=None, lists=True):
     dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, mode, cap=cap, materialise=unfused)
     g = dsc.grid
     res = {"dsc": dsc}
@@ -40,7 +40,7 @@ def run_gpu(w, mode=emr.EMR_EAGER, unfused=True, fused=True, cap=None):
         res["mask_f"] = unpack_planes(dsc.mask.cpu().numpy(), g)
         res["split_f"] = dsc.split.cpu().numpy()
         res["band_f"] = dsc.band_bits.cpu().numpy()
-        res["lists_f"] = dsc.lists()
+        res["lists_f"] = dsc.lists() if lists else None
         res["out_f"] = dsc.out.cpu().numpy()
     return res
 
@@ -159,6 +159,20 @@ def test_edge_cases_small_depths_constant_and_hidden_free_genomes():
         full_parity(w)
 
 
+def test_every_kernel_class_including_interpreter():
+    """Genomes with 0..30 varying nodes: the constant, dense-4, dense-8, dense-12
+    and interpreter (more than 12 varying nodes) classes in one population."""
+    big = W.random_population(24, seed=31, h_lo=14, h_hi=30, e_max=120)
+    small = W.random_population(40, seed=32, h_lo=0, h_hi=12, e_max=40)
+    pop = W.population_from_lists([big.genome(k) for k in range(24)] + [small.genome(k) for k in range(40)])
+    h, gs, _, _ = emr.pack_records(emr.pack_population(pop))
+    assert gs["n_varying"][:, 0].max() > 12 and (gs["n_varying"][:, 0] == 0).any()
+    src = W.shared_sources([(-1.0, -1.0, W.SIDE_OUT), (0.0, 1.0, W.SIDE_IN)])
+    for D in (4, 6):
+        w = W.Workload("classes", pop, src, D, 0.03, 0.3)
+        full_parity(w)
+
+
 def test_weight_filter_and_gated_mode():
     w = W.c2(D=5, P=100)
     w.w_min = 0.1
@@ -186,7 +200,7 @@ def test_compaction_capacity_overflow_drops_tail_and_reports_total():
     full = run_gpu(w, unfused=False)
     total = sum(len(i) for i, _ in full["lists_f"])
     cap = total // 2
-    small = run_gpu(w, unfused=False, cap=cap)
+    small = run_gpu(w, unfused=False, cap=cap, lists=False)
     dsc = small["dsc"]
     assert int(dsc.offsets[-1]) == total
     with pytest.raises(emr.EmrError):

@@ -23,9 +23,13 @@
  *   halo_off[d] + side * 2^{d+1} + t, halo_off[d] = 8 (2^d - 1);
  *   side 0: (i = -1, j = t), 1: (i = 2^{d+1}, j = t), 2: (i = t, j = -1),
  *   3: (i = t, j = 2^{d+1}). N_halo = 8 (2^{D+1} - 1).
- * Bit planes: one bit per position, levels padded to whole 32-bit words:
- *   position (d, m) is bit (m % 32) of word word_off[d] + m / 32. Bits past
- *   a level's 4^{d+1} positions (depths 0 and 1) are always 0.
+ * Bit planes: one bit per position, levels padded to whole 32-bit words
+ *   (device uint32 [pair][n_words], 16-byte aligned). mask and split are
+ *   position-major: position (d, m) is bit (m % 32) of word word_off[d] + m / 32;
+ *   bits past a level's 4^{d+1} positions (depths 0 and 1) are 0. band_bits
+ *   is position-major at depths 0..2 and quad-major from depth 3: position
+ *   (d, m) is bit (m / 4) % 32 of word word_off[d] + 4 (m / 128) + m % 4 (the
+ *   four words of each 128-position block hold children 0..3 of its 32 quads).
  * Query slots: a (genome, slot) pair ("pair") evaluates CPPN(a, b, x, y, 1)
  *   for an outgoing slot (source node at (a, b)) or CPPN(x, y, a, b, 1) for an
  *   incoming slot (target node at (a, b)) over every grid position; the CPPN

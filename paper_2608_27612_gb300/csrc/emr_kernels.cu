@@ -39,22 +39,45 @@ __device__ __forceinline__ uint32_t morton2(uint32_t i, uint32_t j) { return spr
 __device__ __forceinline__ float grid_coord(int i, float scale) { return fmaf(float(2 * i + 1), scale, -1.0f); }
 
 // ---- activations (fp32) --------------------------------------------------------
-// sigmoid and tanh from the exponential: sigmoid(z) = 1 / (1 + e^-z),
-// tanh(z) = 1 - 2 / (1 + e^{2z}); gauss(z) = e^{-z^2}; sin with a two-constant
-// Cody-Waite reduction by 2 pi (constants: 2 pi rounded to fp32 and the fp32
-// rounding of the remainder) before the hardware sine on [-pi, pi].
+// All transcendental parts run on the MUFU (special function unit) through its
+// approximate instructions with denormal flushing (values below 2^-126 only
+// move by less than 2^-126): sigmoid(z) = 1 / (1 + 2^(-z log2 e)),
+// tanh(z) = 1 - 2 / (1 + 2^(2 z log2 e)), gauss(z) = 2^(-z^2 log2 e), and sin
+// after a two-constant Cody-Waite reduction by 2 pi (constants: 2 pi rounded
+// to fp32 and the fp32 rounding of the remainder; the multiple k is rounded to
+// nearest with the 1.5 * 2^23 shift, valid for |z| < 2^24).
 constexpr float kTwoPiHi = 0x1.921fb6p+2f;
 constexpr float kTwoPiLo = -0x1.777a5cp-23f;
 constexpr float kInvTwoPi = 0x1.45f306p-3f;
+constexpr float kLog2e = 0x1.715476p+0f;
+constexpr float kRoundShift = 0x1.8p+23f;
 
-__device__ __forceinline__ float act_sigmoid(float z) { return __fdividef(1.0f, 1.0f + __expf(-z)); }
-__device__ __forceinline__ float act_tanh(float z) { return 1.0f - __fdividef(2.0f, 1.0f + __expf(2.0f * z)); }
-__device__ __forceinline__ float act_gauss(float z) { return __expf(-z * z); }
+__device__ __forceinline__ float mufu_ex2(float x) {
+  float r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ float mufu_rcp(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ float mufu_sin(float x) {
+  float r;
+  asm("sin.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+__device__ __forceinline__ float act_sigmoid(float z) { return mufu_rcp(1.0f + mufu_ex2(z * -kLog2e)); }
+__device__ __forceinline__ float act_tanh(float z) {
+  return fmaf(-2.0f, mufu_rcp(1.0f + mufu_ex2(z * (2.0f * kLog2e))), 1.0f);
+}
+__device__ __forceinline__ float act_gauss(float z) { return mufu_ex2(z * (z * -kLog2e)); }
 __device__ __forceinline__ float act_sin(float z) {
-  float k = rintf(z * kInvTwoPi);
+  const float k = fmaf(z, kInvTwoPi, kRoundShift) - kRoundShift;
   float r = fmaf(-k, kTwoPiHi, z);
   r = fmaf(-k, kTwoPiLo, r);
-  return __sinf(r);
+  return mufu_sin(r);
 }
 
 __device__ __forceinline__ float act_apply(int a, float z) {
@@ -77,6 +100,48 @@ __device__ __forceinline__ void act_apply4(int a, float& z0, float& z1, float& z
     case EMR_ACT_ABS: z0 = fabsf(z0); z1 = fabsf(z1); z2 = fabsf(z2); z3 = fabsf(z3); break;
     default: break;
   }
+}
+
+// ---- filter arithmetic shared by every kernel ------------------------------------
+// All kernels take the same fp32 decisions, operation for operation:
+//   variance: S = sum_c (w_c - m)^2 with m = (w0 + w1 + w2 + w3) / 4; V = S / 4 and
+//     V > theta is tested as S > 4 theta (scaling by 4 is exact);
+//   band: with squared differences to the four neighbours, B > band is tested as
+//     max(min(dt^2, db^2), min(dl^2, dr^2)) > band^2 (squaring is monotone on
+//     |d|; it changes the fp32 decision only within one rounding of the band).
+__device__ __forceinline__ float var_sum4(float w0, float w1, float w2, float w3) {
+  const float m = 0.25f * ((w0 + w1) + (w2 + w3));
+  const float e0 = w0 - m, e1 = w1 - m, e2 = w2 - m, e3 = w3 - m;
+  return (e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3);
+}
+__device__ __forceinline__ float sqdiff(float a, float b) {
+  const float t = a - b;
+  return t * t;
+}
+__device__ __forceinline__ bool band_pass_sq(float dl2, float dr2, float db2, float dt2, float band2) {
+  return fmaxf(fminf(dt2, db2), fminf(dl2, dr2)) > band2;
+}
+
+// Band-bit planes are quad-major from depth 3 on: in each block of 128
+// positions (32 sibling quads), word c holds child c of the 32 quads (bit =
+// quad). Depths 0..2 use the position-major layout of the other planes.
+constexpr int kQuadMajorFrom = 3;
+
+// Bits b (8 of them) spread to positions 0, 4, ..., 28.
+__device__ __forceinline__ uint32_t spread_nibbles(uint32_t b) {
+  b &= 0xffu;
+  b = (b | (b << 12)) & 0x000f000fu;
+  b = (b | (b << 6)) & 0x03030303u;
+  b = (b | (b << 3)) & 0x11111111u;
+  return b;
+}
+
+// Band-bit word of the 8 quads (32 positions) of lane group g from the four
+// per-child ballots: bit 4 i + c of the word is child c of quad 8 g + i.
+__device__ __forceinline__ uint32_t band_word(uint32_t b0, uint32_t b1, uint32_t b2, uint32_t b3, int g) {
+  const int sh = 8 * g;
+  return spread_nibbles(b0 >> sh) | (spread_nibbles(b1 >> sh) << 1) | (spread_nibbles(b2 >> sh) << 2) |
+         (spread_nibbles(b3 >> sh) << 3);
 }
 
 // ---- per-pair specialisation ---------------------------------------------------
@@ -387,10 +452,7 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
     }
     // fused: the four children of parent q give its variance (Section 3.2)
     if (d >= 1) {
-      const float m = 0.25f * ((w[0] + w[1]) + (w[2] + w[3]));
-      const float e0 = w[0] - m, e1 = w[1] - m, e2 = w[2] - m, e3 = w[3] - m;
-      const float V = 0.25f * ((e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3));
-      const unsigned bal = __ballot_sync(kFull, is_main && V > A.theta);
+      const unsigned bal = __ballot_sync(kFull, is_main && var_sum4(w[0], w[1], w[2], w[3]) > 4.f * A.theta);
       const int q0 = base + warp * 32;
       if (lane == 0 && q0 < nq)
         A.split[int64_t(r) * A.n_words + A.word_off[d - 1] + (mb / 4 + uint32_t(q0)) / 32] = bal;
@@ -407,30 +469,33 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
     const int q = base + tid;
     const bool valid = q < nq;
     const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-    unsigned nib = 0;
+    const float band2 = A.band * A.band;
+    bool pass[4] = {false, false, false, false};
     float w[4];
 #pragma unroll
     for (int c = 0; c < 4; c++) {
       const int li = 2 * pi + (c & 1) + 1, lj = 2 * pj + (c >> 1) + 1;
       w[c] = valid ? wt[lj * pitch + li] : 0.f;
       if (valid) {
-        const float dl = fabsf(w[c] - wt[lj * pitch + li - 1]), dr = fabsf(w[c] - wt[lj * pitch + li + 1]);
-        const float db = fabsf(w[c] - wt[(lj - 1) * pitch + li]), dt = fabsf(w[c] - wt[(lj + 1) * pitch + li]);
-        const float B = fmaxf(fminf(dt, db), fminf(dl, dr));
-        const bool pass = B > A.band && (A.w_min <= 0.f || fabsf(w[c]) > A.w_min);
-        nib |= unsigned(pass) << c;
+        pass[c] = band_pass_sq(sqdiff(w[c], wt[lj * pitch + li - 1]), sqdiff(w[c], wt[lj * pitch + li + 1]),
+                               sqdiff(w[c], wt[(lj - 1) * pitch + li]), sqdiff(w[c], wt[(lj + 1) * pitch + li]), band2);
+        if (A.w_min > 0.f) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
       }
     }
-    unsigned v = nib << (4 * (lane & 7));
-    v |= __shfl_xor_sync(kFull, v, 1);
-    v |= __shfl_xor_sync(kFull, v, 2);
-    v |= __shfl_xor_sync(kFull, v, 4);
-    if ((lane & 7) == 0 && valid)
-      A.bandb[int64_t(r) * A.n_words + A.word_off[d] + (mb + 4u * uint32_t(q)) / 32] = v;
-    if (A.out && nib) {
+    const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+    const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+    const int q0 = base + warp * 32;
+    if (d >= kQuadMajorFrom) {
+      if (lane < 4 && q0 < nq)
+        A.bandb[int64_t(r) * A.n_words + A.word_off[d] + 4 * ((mb + 4u * uint32_t(q0)) >> 7) + lane] =
+            lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+    } else if (q0 == 0 && lane * 32 < 4 * nq) {
+      A.bandb[int64_t(r) * A.n_words + A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
+    }
+    if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
 #pragma unroll
       for (int c = 0; c < 4; c++)
-        if (nib & (1u << c)) A.out[pair_pos + mb + 4 * q + c] = w[c];
+        if (pass[c]) A.out[pair_pos + mb + 4 * q + c] = w[c];
     }
   }
 }
@@ -524,12 +589,18 @@ __device__ __forceinline__ void eval_dense(const float4* __restrict__ coef, cons
   }
 }
 
+// The shared tile stores position (i, j) of a T x T tile at row j + 2, column
+// i + 2 (pitch T + 4): two-column padding keeps sibling pairs 8-byte aligned;
+// the ring of out-of-tile neighbours sits in columns / rows 1 and T + 2.
+constexpr int kPad = 2;
+
 template <int NVMAX>
 __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_dense(const DTileArgs A) {
   static_assert(NVMAX <= kDenseMax, "dense block holds kDenseMax rows");
+  constexpr int P64 = kTileSide + 2 * kPad;
   __shared__ float4 s_coef[NVMAX];
   __shared__ __align__(16) float s_W[NVMAX * NVMAX];
-  __shared__ float s_wt[(kTileSide + 2) * (kTileSide + 2)];
+  __shared__ __align__(16) float s_wt[P64 * P64];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
   const int tile = int(blockIdx.x % A.n_tiles);
@@ -538,135 +609,192 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
   const int nv = reinterpret_cast<const int32_t*>(rec)[0];
   const float out_const = reinterpret_cast<const float*>(rec)[2];
   const bool fused = A.mode == kModeFused;
+  const bool wfilter = A.w_min > 0.f;
+  const float theta4 = 4.f * A.theta, band2 = A.band * A.band;
   if (tid < NVMAX)
     s_coef[tid] = tid < nv ? reinterpret_cast<const float4*>(rec + A.L.coef_off())[tid] : make_float4(0, 0, 0, 0);
   {
     const float* gW = reinterpret_cast<const float*>(rec + A.L.dense_off());
     for (int k = tid; k < NVMAX * NVMAX; k += kDThreads) s_W[k] = gW[(k / NVMAX) * kDenseMax + (k % NVMAX)];
   }
-  // depth range of this tile
-  int d_lo, d_hi, tl = 0;
-  if (tile == 0) {
-    d_lo = 0;
-    d_hi = min(A.D, kPyramidTop);
-  } else {
+  __syncthreads();
+  uint32_t* split_row = A.split + int64_t(r) * A.n_words;
+  uint32_t* band_row = A.bandb + int64_t(r) * A.n_words;
+  const int64_t prow = int64_t(r) * A.n_total;
+
+  if (tile > 0) {
+    // ---- a full 64 x 64 tile of one depth >= 5: 4 quads and 1 ring point per thread
     int u = tile - 1, d = kPyramidTop + 1;
     while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
-    d_lo = d_hi = d;
-    tl = u;
-  }
-  __syncthreads();
-  const int64_t prow = int64_t(r) * A.n_total;
-  for (int d = d_lo; d <= d_hi; d++) {
-    const int T = d + 1 < kTileLog ? (1 << (d + 1)) : kTileSide;
     const int n = 1 << (d + 1);
-    const uint32_t mb = uint32_t(tl) * uint32_t(T * T);
+    const uint32_t mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
     const int i0 = int(compact1by1(mb)), j0 = int(compact1by1(mb >> 1));
-    const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1)
-    const int nq = T * T / 4, nring = 4 * T, pitch = T + 2;
+    const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1): half the grid spacing
     const int64_t lrow = prow + A.level_off[d];
-    if (fused && nv == 0) {
-      // constant output: every variance and band value is exactly 0
-      for (int k = tid; k < (nq + 31) / 32; k += kDThreads)
-        if (d >= 1) A.split[int64_t(r) * A.n_words + A.word_off[d - 1] + (mb / 4) / 32 + k] = 0u;
-      for (int k = tid; k < (4 * nq + 31) / 32; k += kDThreads)
-        A.bandb[int64_t(r) * A.n_words + A.word_off[d] + mb / 32 + k] = 0u;
-      continue;
+    if (fused && nv == 0) {  // constant output: every variance and band value is exactly 0
+      if (tid < 32) split_row[A.word_off[d - 1] + mb / 128 + tid] = 0u;
+      if (tid < 128) band_row[A.word_off[d] + mb / 32 + tid] = 0u;
+      return;
     }
-    // phase 1: quads (four children of one parent) and the ring points
-    for (int base = 0; base < nq; base += kDThreads) {
-      const int q = base + tid;
-      const bool valid = q < nq;
-      float w[4] = {0.f, 0.f, 0.f, 0.f};
-      int pi = 0, pj = 0;
-      if (valid) {
-        pi = int(compact1by1(uint32_t(q)));
-        pj = int(compact1by1(uint32_t(q) >> 1));
-        const float xa = grid_coord(i0 + 2 * pi, scale), xb = grid_coord(i0 + 2 * pi + 1, scale);
-        const float ya = grid_coord(j0 + 2 * pj, scale), yb = grid_coord(j0 + 2 * pj + 1, scale);
-        const float x[4] = {xa, xb, xa, xb}, y[4] = {ya, ya, yb, yb};
-        eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
+    // quad q = tid + 256 k has parent (pl + 16 (k & 1), ql + 16 (k >> 1)) in the tile
+    const int pl = int(compact1by1(uint32_t(tid))), ql = int(compact1by1(uint32_t(tid) >> 1));
+    const float X0 = grid_coord(i0 + 2 * pl, scale), Y0 = grid_coord(j0 + 2 * ql, scale);
+    const float step = 2.f * scale, jump = 64.f * scale;  // one column; 32 columns
+    const int sbase = (2 * ql + kPad) * P64 + 2 * pl + kPad;
+    // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the nodes
+    constexpr int QPE = NVMAX <= 4 ? 2 : 1;
+#pragma unroll 1
+    for (int k0 = 0; k0 < 4; k0 += QPE) {
+      float x[4 * QPE], y[4 * QPE], w[4 * QPE];
+#pragma unroll
+      for (int h = 0; h < QPE; h++) {
+        const int k = k0 + h;
+        const float xa = (k & 1) ? X0 + jump : X0, ya = (k >> 1) ? Y0 + jump : Y0;
+        x[4 * h + 0] = xa; x[4 * h + 1] = xa + step; x[4 * h + 2] = xa; x[4 * h + 3] = xa + step;
+        y[4 * h + 0] = ya; y[4 * h + 1] = ya; y[4 * h + 2] = ya + step; y[4 * h + 3] = ya + step;
+      }
+      eval_dense<NVMAX, 4 * QPE>(s_coef, s_W, nv, out_const, x, y, w);
+#pragma unroll
+      for (int h = 0; h < QPE; h++) {
+        const int k = k0 + h;
+        const float* wq = w + 4 * h;
         if (fused) {
-          const int li = 2 * pi + 1, lj = 2 * pj + 1;
-          s_wt[lj * pitch + li] = w[0];
-          s_wt[lj * pitch + li + 1] = w[1];
-          s_wt[(lj + 1) * pitch + li] = w[2];
-          s_wt[(lj + 1) * pitch + li + 1] = w[3];
+          float* t = s_wt + sbase + (k & 1) * 32 + (k >> 1) * 32 * P64;
+          *reinterpret_cast<float2*>(t) = make_float2(wq[0], wq[1]);
+          *reinterpret_cast<float2*>(t + P64) = make_float2(wq[2], wq[3]);
+          // the four children give the parent's variance (Section 3.2)
+          const unsigned bal = __ballot_sync(kFull, var_sum4(wq[0], wq[1], wq[2], wq[3]) > theta4);
+          if (lane == 0) split_row[A.word_off[d - 1] + mb / 128 + 8 * k + warp] = bal;
         } else {
-          *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+          *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + 256 * k)) =
+              make_float4(wq[0], wq[1], wq[2], wq[3]);
         }
       }
-      if (fused && d >= 1) {
-        // the four children give the parent's variance (Section 3.2)
-        const float m = 0.25f * ((w[0] + w[1]) + (w[2] + w[3]));
-        const float e0 = w[0] - m, e1 = w[1] - m, e2 = w[2] - m, e3 = w[3] - m;
-        const float V = 0.25f * ((e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3));
-        const unsigned bal = __ballot_sync(kFull, valid && V > A.theta);
-        const int q0 = base + warp * 32;
-        if (lane == 0 && q0 < nq)
-          A.split[int64_t(r) * A.n_words + A.word_off[d - 1] + (mb / 4 + uint32_t(q0)) / 32] = bal;
-      }
     }
-    if (fused || A.out_halo) {
-      for (int t = tid; t < nring; t += kDThreads) {
-        const int sd = t / T, u = t - sd * T;
-        const int li = sd == 0 ? -1 : sd == 1 ? T : u, lj = sd == 2 ? -1 : sd == 3 ? T : u;
-        const int gi = i0 + li, gj = j0 + lj;
-        const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
-        if (!fused && !outside) continue;  // materialised: in-domain points belong to other tiles
+    {
+      // ring: side tid / 64 (warp-uniform), offset tid % 64
+      const int sd = tid >> 6, uu = tid & 63;
+      const int li = sd == 0 ? -1 : sd == 1 ? kTileSide : uu, lj = sd == 2 ? -1 : sd == 3 ? kTileSide : uu;
+      const int gi = i0 + li, gj = j0 + lj;
+      const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
+      if (fused || (A.out_halo && outside)) {
         const float x[1] = {grid_coord(gi, scale)}, y[1] = {grid_coord(gj, scale)};
         float w[1];
         eval_dense<NVMAX, 1>(s_coef, s_W, nv, out_const, x, y, w);
         if (fused) {
-          s_wt[(lj + 1) * pitch + li + 1] = w[0];
+          s_wt[(lj + kPad) * P64 + li + kPad] = w[0];
         } else {
           const int hs = gi < 0 ? 0 : gi >= n ? 1 : gj < 0 ? 2 : 3;
           A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? gj : gi)] = w[0];
         }
       }
     }
-    if (!fused) continue;
+    if (!fused) return;
     __syncthreads();
-    // phase 2: band value of each position from its four neighbours at distance 2^-d
-    for (int base = 0; base < nq; base += kDThreads) {
-      const int q = base + tid;
-      const bool valid = q < nq;
-      unsigned nib = 0;
-      float w[4] = {0.f, 0.f, 0.f, 0.f};
-      if (valid) {
-        const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-        const int li = 2 * pi + 1, lj = 2 * pj + 1;
-        const float* r0 = s_wt + lj * pitch + li;  // position (2pi, 2pj)
-        w[0] = r0[0];
-        w[1] = r0[1];
-        w[2] = r0[pitch];
-        w[3] = r0[pitch + 1];
-        const float l0 = r0[-1], l2 = r0[pitch - 1];              // left of the a = 0 column
-        const float r1 = r0[2], r3 = r0[pitch + 2];               // right of the a = 1 column
-        const float b0 = r0[-pitch], b1 = r0[-pitch + 1];         // below the b = 0 row
-        const float t2 = r0[2 * pitch], t3 = r0[2 * pitch + 1];   // above the b = 1 row
-        const float L[4] = {l0, w[0], l2, w[2]}, R[4] = {w[1], r1, w[3], r3};
-        const float Bo[4] = {b0, b1, w[0], w[1]}, U[4] = {w[2], w[3], t2, t3};
+    // band value of each position from its four neighbours at distance 2^-d
 #pragma unroll
-        for (int c = 0; c < 4; c++) {
-          const float dl = fabsf(w[c] - L[c]), dr = fabsf(w[c] - R[c]);
-          const float db = fabsf(w[c] - Bo[c]), dt = fabsf(w[c] - U[c]);
-          const float B = fmaxf(fminf(dt, db), fminf(dl, dr));
-          const bool pass = B > A.band && (A.w_min <= 0.f || fabsf(w[c]) > A.w_min);
-          nib |= unsigned(pass) << c;
-        }
+    for (int k = 0; k < 4; k++) {
+      const float* t = s_wt + sbase + (k & 1) * 32 + (k >> 1) * 32 * P64;  // position (2pi, 2pj)
+      const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
+      const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
+      const float l0 = t[-1], l2 = t[P64 - 1], r1 = t[2], r3 = t[P64 + 2];
+      const float w[4] = {w01.x, w01.y, w23.x, w23.y};
+      const float L[4] = {l0, w[0], l2, w[2]}, R[4] = {w[1], r1, w[3], r3};
+      const float Bo[4] = {bel.x, bel.y, w[0], w[1]}, U[4] = {w[2], w[3], abv.x, abv.y};
+      bool pass[4];
+      // squared differences between siblings are shared by both
+      const float h01 = sqdiff(w[0], w[1]), h23 = sqdiff(w[2], w[3]);
+      const float v02 = sqdiff(w[0], w[2]), v13 = sqdiff(w[1], w[3]);
+      const float DL[4] = {sqdiff(w[0], L[0]), h01, sqdiff(w[2], L[2]), h23};
+      const float DR[4] = {h01, sqdiff(w[1], R[1]), h23, sqdiff(w[3], R[3])};
+      const float DB[4] = {sqdiff(w[0], Bo[0]), sqdiff(w[1], Bo[1]), v02, v13};
+      const float DT[4] = {v02, v13, sqdiff(w[2], U[2]), sqdiff(w[3], U[3])};
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        pass[c] = band_pass_sq(DL[c], DR[c], DB[c], DT[c], band2);
+        if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
       }
-      unsigned v = nib << (4 * (lane & 7));
-      v |= __shfl_xor_sync(kFull, v, 1);
-      v |= __shfl_xor_sync(kFull, v, 2);
-      v |= __shfl_xor_sync(kFull, v, 4);
-      if ((lane & 7) == 0 && valid)
-        A.bandb[int64_t(r) * A.n_words + A.word_off[d] + (mb + 4u * uint32_t(q)) / 32] = v;
-      if (A.out && nib) {
+      const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+      const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+      if (lane < 4)  // quad-major words of this warp's 32 quads (block mb/128 + 8k + warp)
+        band_row[A.word_off[d] + 4 * (mb / 128 + 8 * k + warp) + lane] =
+            lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+      if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
+        float* o = A.out + lrow + mb + 4 * (tid + 256 * k);
 #pragma unroll
         for (int c = 0; c < 4; c++)
-          if (nib & (1u << c)) A.out[lrow + mb + 4 * q + c] = w[c];
+          if (pass[c]) o[c] = w[c];
       }
+    }
+    return;
+  }
+
+  // ---- tile 0: depths 0..min(D, 4), one after the other (at most 256 quads each)
+  const int d_hi = min(A.D, kPyramidTop);
+  for (int d = 0; d <= d_hi; d++) {
+    const int T = 1 << (d + 1), n = T;
+    const float scale = __int_as_float((127 - (d + 1)) << 23);
+    const int nq = T * T / 4, nring = 4 * T, pitch = T + 2 * kPad;
+    const int64_t lrow = prow + A.level_off[d];
+    if (fused && nv == 0) {
+      if (d >= 1 && tid < (nq + 31) / 32) split_row[A.word_off[d - 1] + tid] = 0u;
+      if (tid < (4 * nq + 31) / 32) band_row[A.word_off[d] + tid] = 0u;
+      continue;
+    }
+    const int q = tid;
+    const bool valid = q < nq;
+    const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+    float w[4] = {0.f, 0.f, 0.f, 0.f};
+    if (valid) {
+      const float xa = grid_coord(2 * pi, scale), xb = grid_coord(2 * pi + 1, scale);
+      const float ya = grid_coord(2 * pj, scale), yb = grid_coord(2 * pj + 1, scale);
+      const float x[4] = {xa, xb, xa, xb}, y[4] = {ya, ya, yb, yb};
+      eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
+      if (fused) {
+        float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+        t[0] = w[0]; t[1] = w[1]; t[pitch] = w[2]; t[pitch + 1] = w[3];
+      } else {
+        *reinterpret_cast<float4*>(A.out + lrow + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+      }
+    }
+    if (fused && d >= 1) {
+      const unsigned bal = __ballot_sync(kFull, valid && var_sum4(w[0], w[1], w[2], w[3]) > theta4);
+      if (lane == 0 && warp * 32 < nq) split_row[A.word_off[d - 1] + warp] = bal;
+    }
+    if ((fused || A.out_halo) && tid < nring) {
+      const int sd = tid / T, uu = tid - sd * T;
+      const int li = sd == 0 ? -1 : sd == 1 ? T : uu, lj = sd == 2 ? -1 : sd == 3 ? T : uu;
+      const float x[1] = {grid_coord(li, scale)}, y[1] = {grid_coord(lj, scale)};
+      float wr[1];
+      eval_dense<NVMAX, 1>(s_coef, s_W, nv, out_const, x, y, wr);
+      if (fused) s_wt[(lj + kPad) * pitch + li + kPad] = wr[0];
+      else A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + sd * n + uu] = wr[0];
+    }
+    if (!fused) continue;
+    __syncthreads();
+    bool pass[4] = {false, false, false, false};
+    if (valid) {
+      const float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+      const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
+      const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]}, U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]), band2);
+        if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+      }
+    }
+    const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+    const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+    if (d >= kQuadMajorFrom) {
+      if (lane < 4 && warp * 32 < nq)
+        band_row[A.word_off[d] + 4 * warp + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+    } else if (warp == 0 && lane * 32 < 4 * nq) {
+      band_row[A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
+    }
+    if (A.out && valid && (pass[0] | pass[1] | pass[2] | pass[3])) {
+#pragma unroll
+      for (int c = 0; c < 4; c++)
+        if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
     }
     __syncthreads();
   }
@@ -676,8 +804,9 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
 
 struct GridDev {
   int32_t D;
-  int64_t n_total, n_halo, n_words;
+  int64_t n_total, n_halo, n_words, n_qblocks;
   int64_t level_off[EMR_MAX_DEPTH + 2], halo_off[EMR_MAX_DEPTH + 2], word_off[EMR_MAX_DEPTH + 2];
+  int64_t qblk_off[EMR_MAX_DEPTH + 2];  // first block of 32 sibling quads of each depth
 };
 
 __device__ __forceinline__ int level_of_word(const GridDev& G, int64_t wi) {
@@ -693,53 +822,70 @@ __device__ __forceinline__ uint32_t valid_bits(const GridDev& G, int d, int64_t 
   return cnt - m0 >= 32 ? kFull : ((1u << (cnt - m0)) - 1u);
 }
 
-// One warp per bit-plane word (32 positions of one depth).
+// One warp per block of 32 sibling quads (128 positions) of one depth; lane =
+// quad. Each lane reads its four outputs, their children (variance) and their
+// neighbours (band) from the materialised outputs.
 __global__ void planes_kernel(const float* __restrict__ out, const float* __restrict__ out_halo, GridDev G,
                               int64_t n_pairs, float theta, float band, float w_min, uint32_t* __restrict__ split,
                               uint32_t* __restrict__ bandb, float* __restrict__ var_dbg) {
   const int lane = threadIdx.x & 31;
   const int64_t wg = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  if (wg >= n_pairs * G.n_words) return;
-  const int64_t r = wg / G.n_words, wi = wg % G.n_words;
-  const int d = level_of_word(G, wi);
-  const uint32_t m = uint32_t(wi - G.word_off[d]) * 32u + uint32_t(lane);
-  const uint32_t cnt = 1u << (2 * (d + 1));
-  const bool valid = m < cnt;
+  if (wg >= n_pairs * G.n_qblocks) return;
+  const int64_t r = wg / G.n_qblocks, qb = wg % G.n_qblocks;
+  int d = 0;
+  while (G.qblk_off[d + 1] <= qb) d++;
+  const uint32_t b = uint32_t(qb - G.qblk_off[d]);
+  const uint32_t q = 32u * b + uint32_t(lane);  // quad (parent) index at depth d
+  const uint32_t nq = 1u << (2 * d);
+  const bool valid = q < nq;
   const int n = 1 << (d + 1);
+  const float theta4 = 4.f * theta, band2 = band * band;
   const float* o = out + r * G.n_total;
-  bool sp = false, bp = false;
+  bool sp[4] = {false, false, false, false}, bp[4] = {false, false, false, false};
   if (valid) {
-    const int i = int(compact1by1(m)), j = int(compact1by1(m >> 1));
-    const float w = o[G.level_off[d] + m];
-    float V = 0.f;
-    if (d < G.D) {
-      const float4 c = *reinterpret_cast<const float4*>(o + G.level_off[d + 1] + 4 * int64_t(m));
-      const float mu = 0.25f * ((c.x + c.y) + (c.z + c.w));
-      const float e0 = c.x - mu, e1 = c.y - mu, e2 = c.z - mu, e3 = c.w - mu;
-      V = 0.25f * ((e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3));
-      sp = V > theta;
-    }
-    if (var_dbg) var_dbg[r * G.n_total + G.level_off[d] + m] = V;
-    float nbv[4];
-    const int ni[4] = {i - 1, i + 1, i, i}, nj[4] = {j, j, j - 1, j + 1};
+    const int pi = int(compact1by1(q)), pj = int(compact1by1(q >> 1));
+    const float4 w4 = *reinterpret_cast<const float4*>(o + G.level_off[d] + 4 * int64_t(q));
+    const float w[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
-    for (int k = 0; k < 4; k++) {
-      if (ni[k] >= 0 && ni[k] < n && nj[k] >= 0 && nj[k] < n) {
-        nbv[k] = o[G.level_off[d] + morton2(uint32_t(ni[k]), uint32_t(nj[k]))];
-      } else {
-        const int sd = ni[k] < 0 ? 0 : ni[k] >= n ? 1 : nj[k] < 0 ? 2 : 3;
-        const int t = sd < 2 ? nj[k] : ni[k];
-        nbv[k] = out_halo[r * G.n_halo + G.halo_off[d] + sd * n + t];
+    for (int c = 0; c < 4; c++) {
+      const int i = 2 * pi + (c & 1), j = 2 * pj + (c >> 1);
+      const uint32_t m = 4 * q + uint32_t(c);
+      float S = 0.f;
+      if (d < G.D) {
+        const float4 ch = *reinterpret_cast<const float4*>(o + G.level_off[d + 1] + 4 * int64_t(m));
+        S = var_sum4(ch.x, ch.y, ch.z, ch.w);
+        sp[c] = S > theta4;
       }
+      if (var_dbg) var_dbg[r * G.n_total + G.level_off[d] + m] = 0.25f * S;
+      float nbv[4];
+      const int ni[4] = {i - 1, i + 1, i, i}, nj[4] = {j, j, j - 1, j + 1};
+#pragma unroll
+      for (int k = 0; k < 4; k++) {
+        if (ni[k] >= 0 && ni[k] < n && nj[k] >= 0 && nj[k] < n) {
+          nbv[k] = o[G.level_off[d] + morton2(uint32_t(ni[k]), uint32_t(nj[k]))];
+        } else {
+          const int sd = ni[k] < 0 ? 0 : ni[k] >= n ? 1 : nj[k] < 0 ? 2 : 3;
+          const int t = sd < 2 ? nj[k] : ni[k];
+          nbv[k] = out_halo[r * G.n_halo + G.halo_off[d] + sd * n + t];
+        }
+      }
+      bp[c] = band_pass_sq(sqdiff(w[c], nbv[0]), sqdiff(w[c], nbv[1]), sqdiff(w[c], nbv[2]), sqdiff(w[c], nbv[3]),
+                           band2);
+      if (w_min > 0.f) bp[c] = bp[c] && fabsf(w[c]) > w_min;
     }
-    const float dl = fabsf(w - nbv[0]), dr = fabsf(w - nbv[1]), db = fabsf(w - nbv[2]), dt = fabsf(w - nbv[3]);
-    const float B = fmaxf(fminf(dt, db), fminf(dl, dr));
-    bp = B > band && (w_min <= 0.f || fabsf(w) > w_min);
   }
-  const unsigned s_bits = __ballot_sync(kFull, sp), b_bits = __ballot_sync(kFull, bp);
-  if (lane == 0) {
-    split[r * G.n_words + wi] = s_bits;
-    bandb[r * G.n_words + wi] = b_bits;
+  const uint32_t s0 = __ballot_sync(kFull, sp[0]), s1 = __ballot_sync(kFull, sp[1]);
+  const uint32_t s2 = __ballot_sync(kFull, sp[2]), s3 = __ballot_sync(kFull, sp[3]);
+  const uint32_t b0 = __ballot_sync(kFull, bp[0]), b1 = __ballot_sync(kFull, bp[1]);
+  const uint32_t b2 = __ballot_sync(kFull, bp[2]), b3 = __ballot_sync(kFull, bp[3]);
+  // position-major words of this block: 4 (fewer at depths 0..2)
+  const int nw = int(min(4u, (4u * nq - 128u * b + 31u) / 32u));
+  const int64_t w0 = r * G.n_words + G.word_off[d] + 4 * int64_t(b);
+  if (lane < nw) split[w0 + lane] = band_word(s0, s1, s2, s3, lane);
+  if (d >= kQuadMajorFrom) {
+    if (lane < 4) bandb[w0 + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+  } else if (lane < nw) {
+    bandb[w0 + lane] = band_word(b0, b1, b2, b3, lane);
   }
 }
 
@@ -753,7 +899,15 @@ __global__ void combine_kernel(const uint32_t* __restrict__ split, const uint32_
   const uint32_t m0 = uint32_t(wi - G.word_off[d]) * 32u;
   const uint32_t valid = valid_bits(G, d, wi);
   const uint32_t* sp = split + r * G.n_words;
-  uint32_t keep = bandb[r * G.n_words + wi] & valid;
+  uint32_t bw;
+  if (d >= kQuadMajorFrom) {  // re-interleave the block's four child words
+    const int64_t j = wi - G.word_off[d];
+    const uint4 bq = *reinterpret_cast<const uint4*>(bandb + r * G.n_words + G.word_off[d] + 4 * (j >> 2));
+    bw = band_word(bq.x, bq.y, bq.z, bq.w, int(j & 3));
+  } else {
+    bw = bandb[r * G.n_words + wi];
+  }
+  uint32_t keep = bw & valid;
   if (d < G.D) keep &= ~sp[wi];
   if (gated && keep) {
     // active(p) = every ancestor split (Eq. 2); the ancestors of these 32
@@ -763,9 +917,9 @@ __global__ void combine_kernel(const uint32_t* __restrict__ split, const uint32_
       const uint32_t a0 = m0 >> (2 * k);
       const uint32_t aw = sp[G.word_off[d - k] + (a0 >> 5)];
       uint32_t bits = 0;
-      for (int b = 0; b < 32; b++) {
-        const uint32_t anc = (m0 + uint32_t(b)) >> (2 * k);
-        bits |= ((aw >> (anc & 31u)) & 1u) << b;
+      for (int bb = 0; bb < 32; bb++) {
+        const uint32_t anc = (m0 + uint32_t(bb)) >> (2 * k);
+        bits |= ((aw >> (anc & 31u)) & 1u) << bb;
       }
       act &= bits;
     }
@@ -902,11 +1056,15 @@ GridDev grid_dev(const emr_grid* g) {
   G.n_total = g->n_total;
   G.n_halo = g->n_halo;
   G.n_words = g->n_words;
+  int64_t qb = 0;
   for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {
     G.level_off[d] = g->level_off[d];
     G.halo_off[d] = g->halo_off[d];
     G.word_off[d] = g->word_off[d];
+    G.qblk_off[d] = qb;
+    if (d <= g->D) qb += ((int64_t(1) << (2 * d)) + 31) / 32;
   }
+  G.n_qblocks = G.qblk_off[g->D + 1];
   return G;
 }
 
@@ -1141,9 +1299,11 @@ emr_status emr_variance_filter(const float* out, const float* out_halo, const em
     return EMR_ERR_ARG;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const int64_t n_pairs = int64_t(P) * S;
-  const int64_t threads = n_pairs * grid->n_words * 32;
-  planes_kernel<<<unsigned((threads + 255) / 256), 256, 0, st>>>(out, out_halo, grid_dev(grid), n_pairs, theta, band,
-                                                                 w_min, split, band_bits, var_dbg);
+  const GridDev G = grid_dev(grid);
+  const int64_t threads = n_pairs * G.n_qblocks * 32;
+  if ((threads + 255) / 256 > 0x7fffffffLL) return EMR_ERR_RANGE;
+  planes_kernel<<<unsigned((threads + 255) / 256), 256, 0, st>>>(out, out_halo, G, n_pairs, theta, band, w_min, split,
+                                                                 band_bits, var_dbg);
   emr_status rc = cuda_status(cudaGetLastError());
   if (rc != EMR_OK) return rc;
   return launch_combine(split, band_bits, grid, n_pairs, mode == EMR_GATED, mask, st);

@@ -221,6 +221,39 @@ emr_status emr_eval_filter(const void *pack_host, const emr_query *q, const emr_
                            float band, float w_min, uint32_t *split, uint32_t *band_bits, float *out, void *ws,
                            size_t ws_bytes, void *stream);
 
+/* ---- fused evaluation without a caller-provided workspace -------------------- */
+
+/* The paper has no counterpart to this call; it exists for callers that cannot
+ * allocate device memory themselves (for example a plugin whose host
+ * application owns all device memory, or a latency-critical loop that must not
+ * incur the implicit device synchronisation of cudaMalloc).
+ *
+ * Computes exactly what emr_eval_prepare followed by emr_eval_filter computes
+ * (same split / band_bits planes, same sparse out entries), but keeps the
+ * per-pair records, their scratch and the pair schedule in a static device
+ * array owned by libemr: EMR_STATIC_SCRATCH_BYTES (16 MiB) on every GPU that
+ * loads the library, held until the process exits. It allocates nothing and
+ * calls no allocating routine. The caller still provides the inputs (packed
+ * population, query) and the outputs (split, band_bits, out as in
+ * emr_eval_filter).
+ *
+ * Limits and behaviour:
+ *  - EMR_ERR_RANGE if the pairs' records do not fit the static array (the size
+ *    emr_eval_workspace_size reports must be <= EMR_STATIC_SCRATCH_BYTES);
+ *    nothing is launched then.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress, with that device current) and caches it; make that
+ *    first call before any stream capture.
+ *  - All calls on a device share the one array and it keeps the previous
+ *    call's contents. Nothing in it needs to start at zero (every call writes
+ *    each entry it reads), but calls whose work overlaps on the GPU (other
+ *    streams, other host threads) race on it: serialise them.
+ * Errors: EMR_ERR_ARG, EMR_ERR_RANGE, EMR_ERR_CUDA. */
+#define EMR_STATIC_SCRATCH_BYTES (16u << 20)
+emr_status emr_eval_filter_noalloc(const void *pack_host, const void *pack_dev, const emr_query *q,
+                                   const emr_grid *grid, float theta, float band, float w_min, uint32_t *split,
+                                   uint32_t *band_bits, float *out, void *stream);
+
 /* ---- a6: compaction -------------------------------------------------------- */
 
 /* Bytes of device workspace emr_compact needs for n_pairs pairs. */

@@ -1356,3 +1356,63 @@ emr_status emr_compact(const uint32_t* mask, const float* out, const emr_grid* g
 }
 
 }  // extern "C"
+
+// ---- fused evaluation without caller-provided workspace ----------------------------
+//
+// Some callers cannot call cudaMalloc: a plugin inside a host application that
+// owns every byte of device memory, or a latency-critical loop that must not
+// take the implicit device synchronisation an allocation brings. For them,
+// emr_eval_filter_noalloc keeps its scratch (the per-pair CPPN records, their
+// scratch and the pair schedule) in the library's own static device array
+// below. Each GPU that loads libemr holds this array until the process exits.
+
+#include <mutex>
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(16) << 20;  // 16 MiB per device
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_static_scratch_mu;
+void* g_static_scratch_dev[kMaxDevices] = {};
+
+// Device address of g_static_scratch on the current device. The first call on
+// a device looks it up (cudaGetSymbolAddress, with that device current); later
+// calls reuse the cached address. In host code the symbol itself is only a
+// host-side stand-in and must never be handed to a kernel.
+emr_status static_scratch_address(void** ptr) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EMR_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return EMR_ERR_RANGE;
+  std::lock_guard<std::mutex> lock(g_static_scratch_mu);
+  if (!g_static_scratch_dev[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) return EMR_ERR_CUDA;
+    g_static_scratch_dev[dev] = p;
+  }
+  *ptr = g_static_scratch_dev[dev];
+  return EMR_OK;
+}
+
+}  // namespace
+
+extern "C" emr_status emr_eval_filter_noalloc(const void* pack_host, const void* pack_dev, const emr_query* q,
+                                              const emr_grid* grid, float theta, float band, float w_min,
+                                              uint32_t* split, uint32_t* band_bits, float* out, void* stream) {
+  if (!pack_dev || !grid_ok(grid) || !split || !band_bits || !q || !q->a_dev || !q->b_dev || !q->side_dev)
+    return EMR_ERR_ARG;
+  if (!(theta >= 0.f) || !(band >= 0.f) || !(w_min >= 0.f)) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (p.total > kStaticScratchBytes) return EMR_ERR_RANGE;  // population x slots too large for the static area
+  void* ws = nullptr;
+  if ((rc = static_scratch_address(&ws)) != EMR_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* spec;
+  int32_t* order;
+  if ((rc = prepare(pack_dev, q, p, ws, st, &spec, &order)) != EMR_OK) return rc;
+  return launch_tiles(p, grid, spec, order, kModeFused, theta, band, w_min, out, nullptr, split, band_bits, st);
+}

@@ -64,6 +64,7 @@ def lib() -> C.CDLL:
             "emr_variance_filter": [vp, vp, vp, i32, i32, f32, f32, f32, i32, vp, vp, vp, vp, vp],
             "emr_mask_combine": [vp, vp, vp, i32, i32, vp, vp],
             "emr_eval_filter": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
+            "emr_eval_filter_noalloc": [vp, vp, vp, vp, f32, f32, f32, vp, vp, vp, vp],
             "emr_compact_workspace_size": [vp, i32, vp],
             "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_version": [],
@@ -223,6 +224,15 @@ def eval_filter(pack, query: Query, grid: Grid, theta: float, band: float, w_min
     _check(lib().emr_eval_filter(_ptr(pack), C.byref(q), C.byref(grid), theta, band, w_min, _ptr(split),
                                  _ptr(band_bits), _ptr(out), _ptr(ws), C.c_size_t(ws.numel()), _stream(stream)),
            "emr_eval_filter")
+
+
+def eval_filter_noalloc(pack, pack_dev, query: Query, grid: Grid, theta: float, band: float, w_min: float, split,
+                        band_bits, out, stream=None):
+    """emr_eval_filter_noalloc: prepare + fused evaluation in libemr's static device scratch."""
+    q = query.c
+    _check(lib().emr_eval_filter_noalloc(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min,
+                                         _ptr(split), _ptr(band_bits), _ptr(out), _stream(stream)),
+           "emr_eval_filter_noalloc")
 
 
 def compact(mask, out, grid: Grid, n_pairs: int, idx, w, cap: int, counts, offsets, ws, stream=None):

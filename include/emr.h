@@ -221,6 +221,44 @@ emr_status emr_eval_filter(const void *pack_host, const emr_query *q, const emr_
                            float band, float w_min, uint32_t *split, uint32_t *band_bits, float *out, void *ws,
                            size_t ws_bytes, void *stream);
 
+/* ---- a7: chunked streaming --------------------------------------------------- */
+
+/* Bytes of device workspace emr_stream needs: the per-pair records, the
+ * resident split plane (n_pairs x n_words x 4 bytes) and two chunk buffers
+ * (band bits, mask, sparse outputs of chunk positions, compaction workspace
+ * and chunk_cap list entries each). */
+emr_status emr_stream_workspace_size(const void *pack_host, const emr_query *q, const emr_grid *grid,
+                                     int64_t chunk_cap, size_t *bytes);
+
+/* The whole eager path (emr_eval_prepare, emr_eval_filter, emr_mask_combine
+ * with EMR_EAGER, emr_compact) over grids too large to hold, in chunks of
+ * grid->chunk positions (whole 64 x 64 tiles; 0 = one chunk), with only the
+ * compacted lists leaving the GPU (Section 5.2 and Section 6 stream depths
+ * 8..13 through host memory or disk; here only the kept int32 indices and fp32
+ * weights are copied out). Chunks run from the highest global index down, so
+ * each chunk's split bits (written by its children) are final when it is
+ * filtered; two chunk buffers alternate on `stream` while a second,
+ * library-created stream copies the previous chunk's lists to the host.
+ *
+ * h_idx, h_w: host arrays of cap entries (pinned memory keeps the copies
+ * asynchronous); on return pair r's list is [offsets[r], offsets[r+1]) in
+ * ascending global index, counts[r] its length (host int64 [n_pairs], offsets
+ * [n_pairs + 1]). chunk_cap: list entries one chunk may produce (device
+ * buffers). Synchronous: returns when the lists are on the host.
+ * The GATED mode needs every ancestor's decision, which a descending stream
+ * only has at the end; it is not offered here.
+ * Errors: EMR_ERR_ARG; EMR_ERR_CAPACITY (ws too small, or a chunk or the total
+ * exceeded chunk_cap / cap: counts hold the true totals, the lists are
+ * incomplete); EMR_ERR_TIMEOUT when a host wait exceeds timeout_ms (0 = no
+ * limit): queued work is still running then and writes into ws and the host
+ * arrays, so synchronise the device before reusing them; EMR_ERR_CUDA.
+ * Allocates per call a copy stream, four events and 16 (n_pairs + 1) bytes of
+ * pinned host staging. */
+emr_status emr_stream(const void *pack_host, const void *pack_dev, const emr_query *q, const emr_grid *grid,
+                      float theta, float band, float w_min, void *ws, size_t ws_bytes, int64_t chunk_cap,
+                      int32_t *h_idx, float *h_w, int64_t cap, int64_t *counts, int64_t *offsets,
+                      int64_t timeout_ms, void *stream);
+
 /* ---- fused evaluation without a caller-provided workspace -------------------- */
 
 /* The paper has no counterpart to this call; it exists for callers that cannot

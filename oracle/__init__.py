@@ -16,6 +16,8 @@ Parity status of each oracle function (what pins it, in tests/test_oracle_pins.p
                             lazy tree, a direct re-evaluation at sampled points.
   ora_lazy                  pinned: Theorem 1 (lazy subset of eager, lazy equal to
                             the gated mask) and the closed-form worked example.
+  ora_keep_at               pinned: equal to ora_discover's outputs, variance, band
+                            value, decisions and uncertainty at every position.
 """
 from __future__ import annotations
 
@@ -153,3 +155,24 @@ def lazy(pop, sources, D: int, theta: float, band: float, w_min: float = 0.0,
     if rc != ORA_OK:
         raise ValueError("oracle: lazy failed (code %d)" % rc)
     return keep, evals
+
+
+def keep_at(pop, g: int, a: float, b: float, side: int, D: int, theta: float, band: float, w_min: float,
+            d, i, j, nthreads: int | None = None):
+    """Eager keep decision (fp64) and its uncertainty at listed positions (d, i, j) of genome g's
+    query from slot (a, b, side), by direct CPPN queries. Returns dict of arrays."""
+    d = np.ascontiguousarray(d, np.int32)
+    i = np.ascontiguousarray(i, np.int64)
+    j = np.ascontiguousarray(j, np.int64)
+    n = len(d)
+    out = {k: np.zeros(n) for k in ("w", "w_err", "var", "bnd")}
+    keep = np.zeros(n, np.uint8)
+    unc = np.zeros(n, np.uint8)
+    rc = lib().ora_keep_at(C.c_int(g), *_pop_args(pop), C.c_float(a), C.c_float(b), C.c_int(side), C.c_int(D),
+                           C.c_double(theta), C.c_double(band), C.c_double(w_min), C.c_int64(n), _p(d), _p(i), _p(j),
+                           _p(out["w"]), _p(out["w_err"]), _p(out["var"]), _p(out["bnd"]), _p(keep), _p(unc),
+                           C.c_int(nthreads or threads()))
+    if rc != ORA_OK:
+        raise ValueError("oracle: keep_at failed (code %d)" % rc)
+    out["keep"], out["unc"] = keep, unc
+    return out

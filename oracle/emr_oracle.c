@@ -625,3 +625,84 @@ int ora_lazy(const int64_t *node_ptr, const int32_t *node_id, const int32_t *nod
     free(gen);
     return ORA_OK;
 }
+
+/* ---- decisions at individual positions, by definition -------------------- */
+
+/* For genome g and one query slot (a, b, side): at each listed grid position
+ * (d[k], i[k], j[k]) of a depth-D grid, the CPPN output, its V, B, the eager
+ * keep decision in fp64 and whether it is uncertain at the fp32 margins, all
+ * from direct CPPN queries (children, neighbours). For sampled checks of grids
+ * too large to evaluate whole. */
+int ora_keep_at(int g, const int64_t *node_ptr, const int32_t *node_id, const int32_t *node_kind,
+                const int32_t *node_act, const float *node_bias, const int64_t *conn_ptr, const int32_t *conn_src,
+                const int32_t *conn_dst, const float *conn_w, const uint8_t *conn_en, float src_a, float src_b,
+                int side, int D, double theta, double band, double w_min, int64_t n, const int32_t *dd,
+                const int64_t *ii, const int64_t *jj, double *w_out, double *w_err, double *var_out, double *bnd_out,
+                uint8_t *keep, uint8_t *unc, int nthreads)
+{
+    genome_t G;
+    int rc = genome_build(&G, g, node_ptr, node_id, node_kind, node_act, node_bias, conn_ptr, conn_src, conn_dst,
+                          conn_w, conn_en);
+    if (rc != ORA_OK) return rc;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#pragma omp parallel
+#endif
+    {
+        double *val = malloc(sizeof(double) * G.n), *er = malloc(sizeof(double) * G.n);
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 64)
+#endif
+        for (int64_t k = 0; k < n; k++) {
+            const int d = dd[k];
+            const int64_t i = ii[k], j = jj[k];
+            double in[5], e, we;
+            query_inputs(side, src_a, src_b, coord(d, i), coord(d, j), in);
+            const double w = cppn_eval(&G, in, val, er, &we);
+            /* variance of the four children and its bound (as ora_discover) */
+            double V = 0.0, Ve = 0.0;
+            if (d < D) {
+                double c[4], ce[4], m = 0.0, me = 0.0, cm = 0.0;
+                for (int q = 0; q < 4; q++) {
+                    query_inputs(side, src_a, src_b, coord(d + 1, 2 * i + (q & 1)), coord(d + 1, 2 * j + (q >> 1)), in);
+                    c[q] = cppn_eval(&G, in, val, er, &ce[q]);
+                    m += c[q] / 4.0; me += ce[q] / 4.0; cm += fabs(c[q]) / 4.0;
+                }
+                me += gamma_n(4) * cm;
+                for (int q = 0; q < 4; q++) {
+                    double dq = c[q] - m, dl = ce[q] + me + U32 * (fabs(dq) + ce[q] + me);
+                    V += dq * dq / 4.0;
+                    Ve += dl * (2.0 * fabs(dq) + dl) / 4.0;
+                }
+                Ve += gamma_n(5) * (V + Ve);
+                Ve *= 2.0;
+            }
+            /* band value from the four neighbours at distance 2^-d */
+            const int64_t ni[4] = {i - 1, i + 1, i, i}, nj[4] = {j, j, j - 1, j + 1};
+            double nb[4], nbe[4];
+            for (int q = 0; q < 4; q++) {
+                query_inputs(side, src_a, src_b, coord(d, ni[q]), coord(d, nj[q]), in);
+                nb[q] = cppn_eval(&G, in, val, er, &nbe[q]);
+            }
+            double dl = fabs(w - nb[0]), dr = fabs(w - nb[1]), db = fabs(w - nb[2]), dt = fabs(w - nb[3]);
+            double B = fmax(fmin(dt, db), fmin(dl, dr)), Be = 0.0, dmax = fmax(fmax(dl, dr), fmax(db, dt));
+            for (int q = 0; q < 4; q++) Be = fmax(Be, we + nbe[q]);
+            Be += 2.0 * U32 * dmax;
+            int sp64 = d < D && V > theta;
+            int sp3 = d == D ? 0 : decide_gt(V, theta, TIE_MARGIN + Ve);
+            int bp3 = decide_gt(B, band, TIE_MARGIN + Be);
+            int wp3 = w_min > 0.0 ? decide_gt(fabs(w), w_min, TIE_MARGIN + we) : 1;
+            int k3 = and3(and3(not3(sp3), bp3), wp3);
+            if (w_out) w_out[k] = w;
+            if (w_err) w_err[k] = we;
+            if (var_out) var_out[k] = V;
+            if (bnd_out) bnd_out[k] = B;
+            keep[k] = (uint8_t)(!sp64 && B > band && (w_min <= 0.0 || fabs(w) > w_min));
+            unc[k] = (uint8_t)(k3 == 2);
+            (void)e;
+        }
+        free(val); free(er);
+    }
+    genome_free(&G);
+    return ORA_OK;
+}

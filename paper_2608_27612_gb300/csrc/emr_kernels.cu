@@ -5,6 +5,8 @@
 
 #include <algorithm>
 #include <cstring>
+#include <utility>
+#include <vector>
 
 #include "emr_internal.h"
 
@@ -317,12 +319,17 @@ __global__ void spec_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_
 
 enum { kModeMaterialise = 0, kModeFused = 1 };
 
+// Output views: band_bits and out may be chunk-local buffers. Band word w of
+// pair r is bandb[r * band_stride + w - band_shift]; output at global index p of
+// pair r is out[r * out_stride + p - out_shift]. Whole-grid calls use strides
+// n_words / n_total and shifts 0. The split plane is always whole-grid.
 struct TileArgs {
   const uint8_t* spec;
   SpecLayout L;
   const int32_t* order;
   int64_t rank_beg;
   int32_t n_tiles, tile_beg;
+  int64_t band_stride, band_shift, out_stride, out_shift;
   int32_t D, mode;
   float theta, band, w_min;
   int32_t lvl_tile_beg[EMR_MAX_DEPTH + 2];
@@ -403,7 +410,8 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
   const int nq = T * T / 4;
   const bool ring = fused || A.out_halo != nullptr;
   const int items = nq + (ring ? T : 0);
-  const int64_t pair_pos = int64_t(r) * A.n_total + A.level_off[d];
+  const int64_t pair_pos = int64_t(r) * A.out_stride - A.out_shift + A.level_off[d];
+  const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;
   for (int base = 0; base < items; base += kBlock) {
     const int q = base + tid;
     const bool valid = q < items;
@@ -487,10 +495,10 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
     const int q0 = base + warp * 32;
     if (d >= kQuadMajorFrom) {
       if (lane < 4 && q0 < nq)
-        A.bandb[int64_t(r) * A.n_words + A.word_off[d] + 4 * ((mb + 4u * uint32_t(q0)) >> 7) + lane] =
+        A.bandb[band_base + A.word_off[d] + 4 * ((mb + 4u * uint32_t(q0)) >> 7) + lane] =
             lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
     } else if (q0 == 0 && lane * 32 < 4 * nq) {
-      A.bandb[int64_t(r) * A.n_words + A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
+      A.bandb[band_base + A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
     }
     if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
 #pragma unroll
@@ -520,7 +528,8 @@ struct DTileArgs {
   SpecLayout L;
   const int32_t* order;
   int64_t rank_beg;
-  int32_t n_tiles;
+  int32_t n_tiles, tile_beg;
+  int64_t band_stride, band_shift, out_stride, out_shift;
   int32_t D, mode;
   float theta, band, w_min;
   int64_t n_total, n_halo, n_words;
@@ -603,7 +612,7 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
   __shared__ __align__(16) float s_wt[P64 * P64];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
-  const int tile = int(blockIdx.x % A.n_tiles);
+  const int tile = A.tile_beg + int(blockIdx.x % A.n_tiles);
   const int r = A.order[rank];
   const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
   const int nv = reinterpret_cast<const int32_t*>(rec)[0];
@@ -619,8 +628,8 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
   }
   __syncthreads();
   uint32_t* split_row = A.split + int64_t(r) * A.n_words;
-  uint32_t* band_row = A.bandb + int64_t(r) * A.n_words;
-  const int64_t prow = int64_t(r) * A.n_total;
+  const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;
+  const int64_t prow = int64_t(r) * A.out_stride - A.out_shift;
 
   if (tile > 0) {
     // ---- a full 64 x 64 tile of one depth >= 5: 4 quads and 1 ring point per thread
@@ -633,7 +642,7 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
     const int64_t lrow = prow + A.level_off[d];
     if (fused && nv == 0) {  // constant output: every variance and band value is exactly 0
       if (tid < 32) split_row[A.word_off[d - 1] + mb / 128 + tid] = 0u;
-      if (tid < 128) band_row[A.word_off[d] + mb / 32 + tid] = 0u;
+      if (tid < 128) A.bandb[band_base + A.word_off[d] + mb / 32 + tid] = 0u;
       return;
     }
     // quad q = tid + 256 k has parent (pl + 16 (k & 1), ql + 16 (k >> 1)) in the tile
@@ -717,7 +726,7 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
       const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
       const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
       if (lane < 4)  // quad-major words of this warp's 32 quads (block mb/128 + 8k + warp)
-        band_row[A.word_off[d] + 4 * (mb / 128 + 8 * k + warp) + lane] =
+        A.bandb[band_base + A.word_off[d] + 4 * (mb / 128 + 8 * k + warp) + lane] =
             lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
       if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
         float* o = A.out + lrow + mb + 4 * (tid + 256 * k);
@@ -738,7 +747,7 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
     const int64_t lrow = prow + A.level_off[d];
     if (fused && nv == 0) {
       if (d >= 1 && tid < (nq + 31) / 32) split_row[A.word_off[d - 1] + tid] = 0u;
-      if (tid < (4 * nq + 31) / 32) band_row[A.word_off[d] + tid] = 0u;
+      if (tid < (4 * nq + 31) / 32) A.bandb[band_base + A.word_off[d] + tid] = 0u;
       continue;
     }
     const int q = tid;
@@ -787,9 +796,9 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
     const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
     if (d >= kQuadMajorFrom) {
       if (lane < 4 && warp * 32 < nq)
-        band_row[A.word_off[d] + 4 * warp + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+        A.bandb[band_base + A.word_off[d] + 4 * warp + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
     } else if (warp == 0 && lane * 32 < 4 * nq) {
-      band_row[A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
+      A.bandb[band_base + A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
     }
     if (A.out && valid && (pass[0] | pass[1] | pass[2] | pass[3])) {
 #pragma unroll
@@ -889,12 +898,20 @@ __global__ void planes_kernel(const float* __restrict__ out, const float* __rest
   }
 }
 
+// A (possibly chunk-local) bit plane: word w of pair r is p[r * stride + w - shift].
+struct PlaneView {
+  uint32_t* p;
+  int64_t stride, shift;
+  __device__ __forceinline__ uint32_t& at(int64_t r, int64_t w) const { return p[r * stride + w - shift]; }
+};
+
 // mask = band AND NOT split (no split at depth D); gated: AND Eq. 2's active bit.
-__global__ void combine_kernel(const uint32_t* __restrict__ split, const uint32_t* __restrict__ bandb, GridDev G,
-                               int64_t n_pairs, int gated, uint32_t* __restrict__ mask) {
+// Threads cover words [w0, w0 + nw) of every pair; split is a whole-grid plane.
+__global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView band, PlaneView mask, GridDev G,
+                               int64_t n_pairs, int64_t w0, int64_t nw, int gated) {
   const int64_t wg = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (wg >= n_pairs * G.n_words) return;
-  const int64_t r = wg / G.n_words, wi = wg % G.n_words;
+  if (wg >= n_pairs * nw) return;
+  const int64_t r = wg / nw, wi = w0 + wg % nw;
   const int d = level_of_word(G, wi);
   const uint32_t m0 = uint32_t(wi - G.word_off[d]) * 32u;
   const uint32_t valid = valid_bits(G, d, wi);
@@ -902,10 +919,10 @@ __global__ void combine_kernel(const uint32_t* __restrict__ split, const uint32_
   uint32_t bw;
   if (d >= kQuadMajorFrom) {  // re-interleave the block's four child words
     const int64_t j = wi - G.word_off[d];
-    const uint4 bq = *reinterpret_cast<const uint4*>(bandb + r * G.n_words + G.word_off[d] + 4 * (j >> 2));
+    const uint4 bq = *reinterpret_cast<const uint4*>(&band.at(r, G.word_off[d] + 4 * (j >> 2)));
     bw = band_word(bq.x, bq.y, bq.z, bq.w, int(j & 3));
   } else {
-    bw = bandb[r * G.n_words + wi];
+    bw = band.at(r, wi);
   }
   uint32_t keep = bw & valid;
   if (d < G.D) keep &= ~sp[wi];
@@ -925,7 +942,7 @@ __global__ void combine_kernel(const uint32_t* __restrict__ split, const uint32_
     }
     keep &= act;
   }
-  mask[r * G.n_words + wi] = keep;
+  mask.at(r, wi) = keep;
 }
 
 // ---- ordered compaction -----------------------------------------------------------
@@ -958,13 +975,14 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int* total) 
   return before + x - v;
 }
 
-__global__ void compact_count_kernel(const uint32_t* __restrict__ mask, GridDev G, int nb,
+__global__ void compact_count_kernel(PlaneView mask, GridDev G, int64_t w0, int64_t nw, int nb,
                                      int32_t* __restrict__ bcount) {
   __shared__ int sh[32];
   const int64_t r = blockIdx.x / nb;
   const int b = int(blockIdx.x % nb);
-  const int64_t wi = int64_t(b) * kCompactBlock + threadIdx.x;
-  const int c = wi < G.n_words ? __popc(mask[r * G.n_words + wi] & valid_bits(G, level_of_word(G, wi), wi)) : 0;
+  const int64_t k = int64_t(b) * kCompactBlock + threadIdx.x;
+  const int64_t wi = w0 + k;
+  const int c = k < nw ? __popc(mask.at(r, wi) & valid_bits(G, level_of_word(G, wi), wi)) : 0;
   int total;
   block_exclusive_scan(c, sh, &total);
   if (threadIdx.x == 0) bcount[blockIdx.x] = total;
@@ -1022,15 +1040,18 @@ __global__ void compact_scan_pairs_kernel(const int64_t* __restrict__ counts, in
   if (threadIdx.x == 0) offsets[n_pairs] = carry;
 }
 
-__global__ void compact_write_kernel(const uint32_t* __restrict__ mask, const float* __restrict__ out, GridDev G,
-                                     int nb, const int32_t* __restrict__ boff, const int64_t* __restrict__ offsets,
-                                     int64_t cap, int32_t* __restrict__ idx, float* __restrict__ wv) {
+// out: output at global index p of pair r is out[r * out_stride + p - out_shift].
+__global__ void compact_write_kernel(PlaneView mask, const float* __restrict__ out, int64_t out_stride,
+                                     int64_t out_shift, GridDev G, int64_t w0, int64_t nw, int nb,
+                                     const int32_t* __restrict__ boff, const int64_t* __restrict__ offsets, int64_t cap,
+                                     int32_t* __restrict__ idx, float* __restrict__ wv) {
   __shared__ int sh[32];
   const int64_t r = blockIdx.x / nb;
   const int b = int(blockIdx.x % nb);
-  const int64_t wi = int64_t(b) * kCompactBlock + threadIdx.x;
-  const int d = wi < G.n_words ? level_of_word(G, wi) : 0;
-  const uint32_t bits = wi < G.n_words ? mask[r * G.n_words + wi] & valid_bits(G, d, wi) : 0u;
+  const int64_t k = int64_t(b) * kCompactBlock + threadIdx.x;
+  const int64_t wi = w0 + k;
+  const int d = k < nw ? level_of_word(G, wi) : 0;
+  const uint32_t bits = k < nw ? mask.at(r, wi) & valid_bits(G, d, wi) : 0u;
   const int ex = block_exclusive_scan(__popc(bits), sh, nullptr);
   if (!bits) return;
   const int64_t gbase = G.level_off[d] + (wi - G.word_off[d]) * 32;
@@ -1039,7 +1060,7 @@ __global__ void compact_write_kernel(const uint32_t* __restrict__ mask, const fl
     const int64_t gidx = gbase + __ffs(v) - 1;
     if (dst < cap) {
       idx[dst] = int32_t(gidx);
-      if (wv) wv[dst] = out[r * G.n_total + gidx];
+      if (wv) wv[dst] = out[r * out_stride + gidx - out_shift];
     }
   }
 }
@@ -1162,11 +1183,25 @@ emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, 
   return cuda_status(cudaGetLastError());
 }
 
+// Tile range (dense numbering: tile 0 = depths 0..4, then the 64 x 64 tiles of
+// depths 5..D in global-index order) and output views of one launch set.
+struct TileRange {
+  int32_t beg = 0, end = -1;  // end < 0: all tiles
+  int64_t band_stride = -1, band_shift = 0, out_stride = -1, out_shift = 0;
+};
+
 emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spec, const int32_t* order, int mode,
                         float theta, float band, float w_min, float* out, float* out_halo, uint32_t* split,
-                        uint32_t* bandb, cudaStream_t st) {
+                        uint32_t* bandb, cudaStream_t st, TileRange tr = TileRange()) {
   emr_status rc = EMR_OK;
-  // class 0: interpreter (more than kDenseMax varying nodes)
+  const int32_t n_dense = int32_t(dense_tiles(g->D));
+  if (tr.end < 0) tr.end = n_dense;
+  if (tr.band_stride < 0) tr.band_stride = g->n_words;
+  if (tr.out_stride < 0) tr.out_stride = g->n_total;
+  if (tr.beg < 0 || tr.end > n_dense || tr.beg >= tr.end) return tr.beg == tr.end ? EMR_OK : EMR_ERR_ARG;
+  // class 0: interpreter (more than kDenseMax varying nodes); its tiles are one
+  // per depth for depths 0..5, then the same 64 x 64 tiles (dense tile t >= 1 is
+  // interpreter tile t + 4).
   if (p.n_class[0] > 0) {
     TileArgs A{};
     A.spec = spec;
@@ -1184,8 +1219,14 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
       t += int32_t(tiles_in_level(d));
     }
     for (int d = g->D + 1; d < EMR_MAX_DEPTH + 2; d++) A.lvl_tile_beg[d] = t;
-    A.n_tiles = t;
-    A.tile_beg = 0;
+    const int32_t ib = tr.beg == 0 ? 0 : tr.beg + 4;
+    const int32_t ie = tr.end >= n_dense ? t : tr.end + 4;
+    A.tile_beg = ib;
+    A.n_tiles = ie - ib;
+    A.band_stride = tr.band_stride;
+    A.band_shift = tr.band_shift;
+    A.out_stride = tr.out_stride;
+    A.out_shift = tr.out_shift;
     A.n_total = g->n_total;
     A.n_halo = g->n_halo;
     A.n_words = g->n_words;
@@ -1204,14 +1245,19 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
     if (smem > 227 * 1024) return EMR_ERR_RANGE;
     cudaError_t e = cudaFuncSetAttribute(tile_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e != cudaSuccess) return EMR_ERR_CUDA;
-    tile_kernel<<<unsigned(blocks), kBlock, smem, st>>>(A);
+    if (blocks > 0) tile_kernel<<<unsigned(blocks), kBlock, smem, st>>>(A);
     if ((rc = cuda_status(cudaGetLastError())) != EMR_OK) return rc;
   }
   DTileArgs D{};
   D.spec = spec;
   D.L = p.L;
   D.order = order;
-  D.n_tiles = int32_t(dense_tiles(g->D));
+  D.tile_beg = tr.beg;
+  D.n_tiles = tr.end - tr.beg;
+  D.band_stride = tr.band_stride;
+  D.band_shift = tr.band_shift;
+  D.out_stride = tr.out_stride;
+  D.out_shift = tr.out_shift;
   D.D = g->D;
   D.mode = mode;
   D.theta = theta;
@@ -1237,11 +1283,41 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   return launch_dense<4>(D, beg, p.n_class[3], st);
 }
 
+emr_status launch_combine(const uint32_t* split, PlaneView band, PlaneView mask, const emr_grid* g, int64_t n_pairs,
+                          int64_t w0, int64_t nw, int gated, cudaStream_t st) {
+  const int64_t n = n_pairs * nw;
+  if (n <= 0) return EMR_OK;
+  if ((n + 255) / 256 > 0x7fffffffLL) return EMR_ERR_RANGE;
+  combine_kernel<<<unsigned((n + 255) / 256), 256, 0, st>>>(split, band, mask, grid_dev(g), n_pairs, w0, nw, gated);
+  return cuda_status(cudaGetLastError());
+}
+
 emr_status launch_combine(const uint32_t* split, const uint32_t* bandb, const emr_grid* g, int64_t n_pairs, int gated,
                           uint32_t* mask, cudaStream_t st) {
-  const int64_t n = n_pairs * g->n_words;
-  if (n <= 0) return EMR_OK;
-  combine_kernel<<<unsigned((n + 255) / 256), 256, 0, st>>>(split, bandb, grid_dev(g), n_pairs, gated, mask);
+  return launch_combine(split, PlaneView{const_cast<uint32_t*>(bandb), g->n_words, 0},
+                        PlaneView{mask, g->n_words, 0}, g, n_pairs, 0, g->n_words, gated, st);
+}
+
+size_t compact_ws_bytes(int64_t nw, int64_t n_pairs) {
+  const int64_t nb = (nw + kCompactBlock - 1) / kCompactBlock;
+  return size_t(2 * 4 * nb * n_pairs + 256);
+}
+
+// Ordered compaction of words [w0, w0 + nw) of every pair.
+emr_status launch_compact(PlaneView mask, const float* out, int64_t out_stride, int64_t out_shift, const emr_grid* g,
+                          int64_t n_pairs, int64_t w0, int64_t nw, int32_t* idx, float* w, int64_t cap, int64_t* counts,
+                          int64_t* offsets, void* ws, cudaStream_t st) {
+  const int nb = int((nw + kCompactBlock - 1) / kCompactBlock);
+  const int64_t nblk = int64_t(nb) * n_pairs;
+  if (nblk > 0x7fffffffLL || n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
+  int32_t* bcount = static_cast<int32_t*>(ws);
+  int32_t* boff = bcount + nblk;
+  const GridDev G = grid_dev(g);
+  compact_count_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, G, w0, nw, nb, bcount);
+  compact_scan_pair_kernel<<<unsigned(n_pairs), 256, 0, st>>>(bcount, nb, boff, counts);
+  compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, n_pairs, offsets);
+  compact_write_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, out, out_stride, out_shift, G, w0, nw, nb, boff,
+                                                                 offsets, cap, idx, w);
   return cuda_status(cudaGetLastError());
 }
 
@@ -1327,8 +1403,7 @@ emr_status emr_eval_filter(const void* pack_host, const emr_query* q, const emr_
 
 emr_status emr_compact_workspace_size(const emr_grid* grid, int32_t n_pairs, size_t* bytes) {
   if (!grid_ok(grid) || n_pairs <= 0 || !bytes) return EMR_ERR_ARG;
-  const int64_t nb = (grid->n_words + kCompactBlock - 1) / kCompactBlock;
-  *bytes = size_t(2 * 4 * nb * int64_t(n_pairs) + 256);
+  *bytes = compact_ws_bytes(grid->n_words, n_pairs);
   return EMR_OK;
 }
 
@@ -1338,21 +1413,9 @@ emr_status emr_compact(const uint32_t* mask, const float* out, const emr_grid* g
   if (!mask || !grid_ok(grid) || n_pairs <= 0 || (!idx && cap > 0) || cap < 0 || !counts || !offsets || !ws ||
       (w && !out))
     return EMR_ERR_ARG;
-  size_t need;
-  emr_compact_workspace_size(grid, n_pairs, &need);
-  if (ws_bytes < need) return EMR_ERR_CAPACITY;
-  const int nb = int((grid->n_words + kCompactBlock - 1) / kCompactBlock);
-  const int64_t nblk = int64_t(nb) * n_pairs;
-  if (nblk > 0x7fffffffLL) return EMR_ERR_RANGE;
-  int32_t* bcount = static_cast<int32_t*>(ws);
-  int32_t* boff = bcount + nblk;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  compact_count_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, grid_dev(grid), nb, bcount);
-  compact_scan_pair_kernel<<<unsigned(n_pairs), 256, 0, st>>>(bcount, nb, boff, counts);
-  compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, n_pairs, offsets);
-  compact_write_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, out, grid_dev(grid), nb, boff, offsets, cap,
-                                                                 idx, w);
-  return cuda_status(cudaGetLastError());
+  if (ws_bytes < compact_ws_bytes(grid->n_words, n_pairs)) return EMR_ERR_CAPACITY;
+  return launch_compact(PlaneView{const_cast<uint32_t*>(mask), grid->n_words, 0}, out, grid->n_total, 0, grid,
+                        n_pairs, 0, grid->n_words, idx, w, cap, counts, offsets, ws, static_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"
@@ -1415,4 +1478,236 @@ extern "C" emr_status emr_eval_filter_noalloc(const void* pack_host, const void*
   int32_t* order;
   if ((rc = prepare(pack_dev, q, p, ws, st, &spec, &order)) != EMR_OK) return rc;
   return launch_tiles(p, grid, spec, order, kModeFused, theta, band, w_min, out, nullptr, split, band_bits, st);
+}
+
+// ---- a7: chunked streaming ------------------------------------------------------------
+//
+// The grid is cut into chunks of whole tiles (dense numbering) and processed
+// from the highest global index down. A chunk's positions at depth d have
+// their children at depth d + 1 in the same or an earlier chunk, so when a
+// chunk has been evaluated its own split bits are final and its keep mask and
+// compacted lists can be produced at once. Only the split plane is resident;
+// band bits, masks, sparse outputs and lists are per chunk, double-buffered,
+// and the lists are copied to the caller's host arrays on a second stream
+// while the next chunk computes.
+
+#include <chrono>
+#include <thread>
+
+namespace {
+
+struct StreamPlan {
+  EvalPlan ev;
+  std::vector<std::pair<int32_t, int32_t>> chunks;  // tile ranges, processing order
+  int64_t wpc, ppc;                                 // words / positions per chunk buffer row
+  int64_t n_pairs, chunk_cap;
+  size_t off_split, off_band[2], off_mask[2], off_out[2], off_cws[2], off_idx[2], off_w[2], off_cnt[2], off_off[2];
+  size_t cws_bytes, total;
+};
+
+inline int64_t tile_pos(const emr_grid* g, int32_t t, int32_t n_dense) {
+  if (t >= n_dense) return g->n_total;
+  return t == 0 ? 0 : g->level_off[kPyramidTop + 1] + int64_t(t - 1) * kTileSide * kTileSide;
+}
+inline int64_t tile_word(const emr_grid* g, int32_t t, int32_t n_dense) {
+  if (t >= n_dense) return g->n_words;
+  return t == 0 ? 0 : g->word_off[kPyramidTop + 1] + int64_t(t - 1) * (kTileSide * kTileSide / 32);
+}
+
+emr_status stream_plan(const void* pack_host, const emr_query* q, const emr_grid* g, int64_t chunk_cap,
+                       StreamPlan* sp) {
+  if (!grid_ok(g) || chunk_cap <= 0) return EMR_ERR_ARG;
+  emr_status rc = eval_plan(pack_host, q, &sp->ev);
+  if (rc != EMR_OK) return rc;
+  const int32_t n_dense = int32_t(dense_tiles(g->D));
+  const int64_t tile_positions = int64_t(kTileSide) * kTileSide;
+  const int32_t tpc = g->chunk > 0 ? int32_t(std::max<int64_t>(1, g->chunk / tile_positions)) : n_dense;
+  sp->chunks.clear();
+  for (int32_t hi = n_dense; hi > 0;) {
+    int32_t lo = std::max(hi - tpc, 1);
+    if (lo == 1) lo = 0;  // the tile of depths 0..4 joins the last chunk
+    sp->chunks.push_back({lo, hi});
+    hi = lo;
+  }
+  sp->wpc = sp->ppc = 0;
+  for (auto& c : sp->chunks) {
+    sp->wpc = std::max(sp->wpc, tile_word(g, c.second, n_dense) - tile_word(g, c.first, n_dense));
+    sp->ppc = std::max(sp->ppc, tile_pos(g, c.second, n_dense) - tile_pos(g, c.first, n_dense));
+  }
+  sp->wpc = (sp->wpc + 3) & ~int64_t(3);
+  sp->ppc = (sp->ppc + 3) & ~int64_t(3);
+  sp->n_pairs = sp->ev.n_pairs;
+  sp->chunk_cap = chunk_cap;
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  size_t o = up(sp->ev.total);
+  sp->off_split = o;
+  o += up(size_t(sp->n_pairs) * size_t(g->n_words) * 4);
+  sp->cws_bytes = compact_ws_bytes(sp->wpc, sp->n_pairs);
+  for (int b = 0; b < 2; b++) {
+    sp->off_band[b] = o; o += up(size_t(sp->n_pairs) * size_t(sp->wpc) * 4);
+    sp->off_mask[b] = o; o += up(size_t(sp->n_pairs) * size_t(sp->wpc) * 4);
+    sp->off_out[b] = o; o += up(size_t(sp->n_pairs) * size_t(sp->ppc) * 4);
+    sp->off_cws[b] = o; o += up(sp->cws_bytes);
+    sp->off_idx[b] = o; o += up(size_t(chunk_cap) * 4);
+    sp->off_w[b] = o; o += up(size_t(chunk_cap) * 4);
+    sp->off_cnt[b] = o; o += up(size_t(sp->n_pairs) * 8);
+    sp->off_off[b] = o; o += up(size_t(sp->n_pairs + 1) * 8);
+  }
+  sp->total = o;
+  return EMR_OK;
+}
+
+// Wait for an event with a host-side deadline (timeout_ms <= 0: no limit).
+emr_status wait_event(cudaEvent_t ev, std::chrono::steady_clock::time_point deadline, bool limited) {
+  for (;;) {
+    const cudaError_t e = cudaEventQuery(ev);
+    if (e == cudaSuccess) return EMR_OK;
+    if (e != cudaErrorNotReady) return EMR_ERR_CUDA;
+    if (limited && std::chrono::steady_clock::now() > deadline) return EMR_ERR_TIMEOUT;
+    std::this_thread::sleep_for(std::chrono::microseconds(20));
+  }
+}
+
+}  // namespace
+
+extern "C" emr_status emr_stream_workspace_size(const void* pack_host, const emr_query* q, const emr_grid* grid,
+                                                int64_t chunk_cap, size_t* bytes) {
+  if (!bytes) return EMR_ERR_ARG;
+  StreamPlan sp;
+  emr_status rc = stream_plan(pack_host, q, grid, chunk_cap, &sp);
+  if (rc != EMR_OK) return rc;
+  *bytes = sp.total;
+  return EMR_OK;
+}
+
+extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, const emr_query* q,
+                                 const emr_grid* grid, float theta, float band, float w_min, void* ws, size_t ws_bytes,
+                                 int64_t chunk_cap, int32_t* h_idx, float* h_w, int64_t cap, int64_t* counts,
+                                 int64_t* offsets, int64_t timeout_ms, void* stream) {
+  if (!pack_dev || !ws || !counts || !offsets || cap < 0 || (cap > 0 && (!h_idx || !h_w)) || timeout_ms < 0)
+    return EMR_ERR_ARG;
+  if (!(theta >= 0.f) || !(band >= 0.f) || !(w_min >= 0.f)) return EMR_ERR_ARG;
+  StreamPlan sp;
+  emr_status rc = stream_plan(pack_host, q, grid, chunk_cap, &sp);
+  if (rc != EMR_OK) return rc;
+  if (ws_bytes < sp.total) return EMR_ERR_CAPACITY;
+  const auto deadline = std::chrono::steady_clock::now() + std::chrono::milliseconds(timeout_ms);
+  const bool limited = timeout_ms > 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  uint8_t* spec;
+  int32_t* order;
+  if ((rc = prepare(pack_dev, q, sp.ev, ws, st, &spec, &order)) != EMR_OK) return rc;
+  uint32_t* split = reinterpret_cast<uint32_t*>(base + sp.off_split);
+  const int32_t n_dense = int32_t(dense_tiles(grid->D));
+  const int64_t NP = sp.n_pairs;
+
+  cudaStream_t cp = nullptr;
+  cudaEvent_t ev_done[2] = {nullptr, nullptr}, ev_copied[2] = {nullptr, nullptr};
+  int64_t* staging = nullptr;  // pinned: 2 x (n_pairs + 1) chunk offsets
+  bool ok = cudaStreamCreateWithFlags(&cp, cudaStreamNonBlocking) == cudaSuccess &&
+            cudaHostAlloc(reinterpret_cast<void**>(&staging), size_t(2 * (NP + 1)) * 8, cudaHostAllocDefault) ==
+                cudaSuccess;
+  for (int b = 0; b < 2 && ok; b++)
+    ok = cudaEventCreateWithFlags(&ev_done[b], cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&ev_copied[b], cudaEventDisableTiming) == cudaSuccess;
+  struct ChunkOut { int64_t at; std::vector<int64_t> off; };  // host position of its lists, per-pair offsets
+  std::vector<ChunkOut> outs(sp.chunks.size());
+  for (int64_t r = 0; r < NP; r++) counts[r] = 0;
+  int64_t cursor = 0;
+  bool overflow = false;
+  rc = ok ? EMR_OK : EMR_ERR_CUDA;
+
+  // Collect chunk k's lists: wait for its offsets, then copy its entries to the host arrays.
+  auto collect = [&](size_t k) -> emr_status {
+    const int b = int(k & 1);
+    emr_status e = wait_event(ev_done[b], deadline, limited);
+    if (e != EMR_OK) return e;
+    const int64_t* off = staging + b * (NP + 1);
+    const int64_t total = off[NP];
+    if (total > sp.chunk_cap) overflow = true;
+    const int64_t n = std::min(total, sp.chunk_cap);
+    ChunkOut& co = outs[k];
+    co.at = cursor;
+    co.off.assign(off, off + NP + 1);
+    for (int64_t r = 0; r < NP; r++) counts[r] += off[r + 1] - off[r];
+    const int64_t fit = std::max<int64_t>(0, std::min(n, cap - cursor));
+    if (fit < n) overflow = true;
+    if (fit > 0) {
+      if (cudaMemcpyAsync(h_idx + cursor, base + sp.off_idx[b], size_t(fit) * 4, cudaMemcpyDeviceToHost, cp) !=
+              cudaSuccess ||
+          cudaMemcpyAsync(h_w + cursor, base + sp.off_w[b], size_t(fit) * 4, cudaMemcpyDeviceToHost, cp) !=
+              cudaSuccess)
+        return EMR_ERR_CUDA;
+    }
+    cursor += fit;
+    return cudaEventRecord(ev_copied[b], cp) == cudaSuccess ? EMR_OK : EMR_ERR_CUDA;
+  };
+
+  for (size_t k = 0; k < sp.chunks.size() && rc == EMR_OK; k++) {
+    const int b = int(k & 1);
+    const int32_t t_lo = sp.chunks[k].first, t_hi = sp.chunks[k].second;
+    const int64_t w_lo = tile_word(grid, t_lo, n_dense), w_hi = tile_word(grid, t_hi, n_dense);
+    const int64_t p_lo = tile_pos(grid, t_lo, n_dense);
+    if (k >= 2 && cudaStreamWaitEvent(st, ev_copied[b], 0) != cudaSuccess) { rc = EMR_ERR_CUDA; break; }
+    uint32_t* bandc = reinterpret_cast<uint32_t*>(base + sp.off_band[b]);
+    uint32_t* maskc = reinterpret_cast<uint32_t*>(base + sp.off_mask[b]);
+    float* outc = reinterpret_cast<float*>(base + sp.off_out[b]);
+    TileRange tr;
+    tr.beg = t_lo;
+    tr.end = t_hi;
+    tr.band_stride = sp.wpc;
+    tr.band_shift = w_lo;
+    tr.out_stride = sp.ppc;
+    tr.out_shift = p_lo;
+    if ((rc = launch_tiles(sp.ev, grid, spec, order, kModeFused, theta, band, w_min, outc, nullptr, split, bandc, st,
+                           tr)) != EMR_OK)
+      break;
+    if ((rc = launch_combine(split, PlaneView{bandc, sp.wpc, w_lo}, PlaneView{maskc, sp.wpc, w_lo}, grid, NP, w_lo,
+                             w_hi - w_lo, 0, st)) != EMR_OK)
+      break;
+    if ((rc = launch_compact(PlaneView{maskc, sp.wpc, w_lo}, outc, sp.ppc, p_lo, grid, NP, w_lo, w_hi - w_lo,
+                             reinterpret_cast<int32_t*>(base + sp.off_idx[b]),
+                             reinterpret_cast<float*>(base + sp.off_w[b]), sp.chunk_cap,
+                             reinterpret_cast<int64_t*>(base + sp.off_cnt[b]),
+                             reinterpret_cast<int64_t*>(base + sp.off_off[b]), base + sp.off_cws[b], st)) != EMR_OK)
+      break;
+    if (cudaMemcpyAsync(staging + b * (NP + 1), base + sp.off_off[b], size_t(NP + 1) * 8, cudaMemcpyDeviceToHost,
+                        st) != cudaSuccess ||
+        cudaEventRecord(ev_done[b], st) != cudaSuccess) {
+      rc = EMR_ERR_CUDA;
+      break;
+    }
+    if (k >= 1) rc = collect(k - 1);
+  }
+  if (rc == EMR_OK && !sp.chunks.empty()) rc = collect(sp.chunks.size() - 1);
+  for (int b = 0; b < 2 && rc == EMR_OK; b++)
+    if (ev_copied[b]) rc = wait_event(ev_copied[b], deadline, limited);
+  if (rc == EMR_OK) {
+    // per-pair lists in ascending global index: chunks in reverse processing order
+    offsets[0] = 0;
+    for (int64_t r = 0; r < NP; r++) offsets[r + 1] = offsets[r] + counts[r];
+    if (!overflow && cursor > 0) {
+      std::vector<int32_t> ti(h_idx, h_idx + cursor);
+      std::vector<float> tw(h_w, h_w + cursor);
+      int64_t dst = 0;
+      for (int64_t r = 0; r < NP; r++)
+        for (size_t k = sp.chunks.size(); k-- > 0;) {
+          const ChunkOut& co = outs[k];
+          const int64_t n = co.off[r + 1] - co.off[r];
+          std::copy(ti.begin() + co.at + co.off[r], ti.begin() + co.at + co.off[r] + n, h_idx + dst);
+          std::copy(tw.begin() + co.at + co.off[r], tw.begin() + co.at + co.off[r] + n, h_w + dst);
+          dst += n;
+        }
+    }
+    if (overflow) rc = EMR_ERR_CAPACITY;
+  }
+  // a timed-out call leaves its queued work running; release what is safe to release
+  if (rc != EMR_ERR_TIMEOUT && staging) cudaFreeHost(staging);
+  for (int b = 0; b < 2; b++) {
+    if (ev_done[b]) cudaEventDestroy(ev_done[b]);
+    if (ev_copied[b]) cudaEventDestroy(ev_copied[b]);
+  }
+  if (cp) cudaStreamDestroy(cp);
+  return rc;
 }

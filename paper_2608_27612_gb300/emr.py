@@ -65,6 +65,8 @@ def lib() -> C.CDLL:
             "emr_mask_combine": [vp, vp, vp, i32, i32, vp, vp],
             "emr_eval_filter": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
             "emr_eval_filter_noalloc": [vp, vp, vp, vp, f32, f32, f32, vp, vp, vp, vp],
+            "emr_stream_workspace_size": [vp, vp, vp, i64, vp],
+            "emr_stream": [vp, vp, vp, vp, f32, f32, f32, vp, sz, i64, vp, vp, i64, vp, vp, i64, vp],
             "emr_compact_workspace_size": [vp, i32, vp],
             "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_version": [],
@@ -233,6 +235,23 @@ def eval_filter_noalloc(pack, pack_dev, query: Query, grid: Grid, theta: float, 
     _check(lib().emr_eval_filter_noalloc(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min,
                                          _ptr(split), _ptr(band_bits), _ptr(out), _stream(stream)),
            "emr_eval_filter_noalloc")
+
+
+def stream_workspace_size(pack, query: Query, grid: Grid, chunk_cap: int) -> int:
+    n = C.c_size_t()
+    q = query.c
+    _check(lib().emr_stream_workspace_size(_ptr(pack), C.byref(q), C.byref(grid), chunk_cap, C.byref(n)),
+           "emr_stream_workspace_size")
+    return n.value
+
+
+def stream(pack, pack_dev, query: Query, grid: Grid, theta: float, band: float, w_min: float, ws, chunk_cap: int,
+           h_idx, h_w, counts, offsets, timeout_ms: int = 0, stream=None):
+    """emr_stream: chunked eager discovery; lists land in the (pinned) host tensors h_idx / h_w."""
+    q = query.c
+    _check(lib().emr_stream(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min, _ptr(ws),
+                            C.c_size_t(ws.numel()), chunk_cap, _ptr(h_idx), _ptr(h_w), h_idx.numel(), _ptr(counts),
+                            _ptr(offsets), timeout_ms, _stream(stream)), "emr_stream")
 
 
 def compact(mask, out, grid: Grid, n_pairs: int, idx, w, cap: int, counts, offsets, ws, stream=None):

@@ -368,3 +368,21 @@ def test_weight_filter_variant():
     assert np.array_equal(r1["keep_eager"], want)
     lz, _ = oracle.lazy(w.pop, w.sources, w.D, w.theta, w.band, 0.1)
     assert np.array_equal(lz, r1["keep_gated"])
+
+
+def test_keep_at_matches_whole_grid_decisions():
+    """Per-position decisions by direct queries equal the whole-grid definition."""
+    w = W.c2(D=5, P=12)
+    r = oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, fields=("w", "var", "bnd", "keep_eager", "unc_eager"))
+    pts = [(d, i, j) for d in range(w.D + 1) for i in range(2 ** (d + 1)) for j in range(2 ** (d + 1))]
+    d, i, j = (np.array(x) for x in zip(*pts))
+    idx = np.array([oracle.index(*p) for p in pts])
+    for g in range(w.P):
+        for s in range(w.S):
+            o = oracle.keep_at(w.pop, g, float(w.sources.a[s]), float(w.sources.b[s]), int(w.sources.side[s]),
+                               w.D, w.theta, w.band, 0.0, d, i, j)
+            assert np.array_equal(o["w"], r["w"][g, s, idx])
+            np.testing.assert_allclose(o["var"], r["var"][g, s, idx], rtol=0, atol=1e-15)
+            np.testing.assert_allclose(o["bnd"], r["bnd"][g, s, idx], rtol=0, atol=1e-15)
+            assert np.array_equal(o["keep"], r["keep_eager"][g, s, idx])
+            assert np.array_equal(o["unc"], r["unc_eager"][g, s, idx])

@@ -286,3 +286,4 @@ def c5(D: int = 13, P: int = 16, chunk: int = 1 << 26) -> Workload:
         pop = pop.subset(range(P))
     src = shared_sources(evenly_spaced(4, -1.0, SIDE_OUT))
     return Workload("c5_deep_pop%d_d%d" % (P, D), pop, src, D, 0.03, 0.3, chunk=chunk)
+

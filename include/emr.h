@@ -91,7 +91,7 @@ typedef struct {
     int64_t level_off[EMR_MAX_DEPTH + 2]; /* [d] first global index of depth d; [D+1] = n_total */
     int64_t halo_off[EMR_MAX_DEPTH + 2];  /* [d] first halo index of depth d; [D+1] = n_halo */
     int64_t word_off[EMR_MAX_DEPTH + 2];  /* [d] first bit-plane word of depth d; [D+1] = n_words */
-} emr_grid;
+} emr_grid;                               /* offset entries past D + 1 repeat the [D + 1] totals */
 
 /* Query slots. Shared by all genomes (per_genome = 0: arrays of S) or one
  * list per genome (per_genome = 1: arrays of P * S, row g). count (per-genome

@@ -520,7 +520,6 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
 // band value needs the neighbours, taken from the tile in shared memory after
 // a barrier (the ring of out-of-tile neighbours is evaluated by the tile too).
 
-constexpr int kDThreads = 256;
 constexpr int kPyramidTop = 4;  // depths 0..4 (side <= 32) share one CTA
 
 struct DTileArgs {
@@ -603,9 +602,15 @@ __device__ __forceinline__ void eval_dense(const float4* __restrict__ coef, cons
 // the ring of out-of-tile neighbours sits in columns / rows 1 and T + 2.
 constexpr int kPad = 2;
 
-template <int NVMAX>
-__global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_dense(const DTileArgs A) {
+// CTAs resident per SM that each class is compiled for (bounds its registers).
+constexpr int dense_min_blocks(int nvmax, int tpb) { return (nvmax <= 4 ? 2048 : nvmax <= 8 ? 1024 : 1024) / tpb / 2; }
+
+template <int NVMAX, int TPB>
+__global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel_dense(const DTileArgs A) {
   static_assert(NVMAX <= kDenseMax, "dense block holds kDenseMax rows");
+  static_assert(TPB >= 64 && TPB <= 256 && (TPB & (TPB - 1)) == 0, "tile work divides evenly");
+  constexpr int QPT = kTileSide * kTileSide / 4 / TPB;  // quads per thread in a 64 x 64 tile
+  constexpr int RPT = 4 * kTileSide / TPB;               // ring points per thread
   constexpr int P64 = kTileSide + 2 * kPad;
   __shared__ float4 s_coef[NVMAX];
   __shared__ __align__(16) float s_W[NVMAX * NVMAX];
@@ -624,7 +629,7 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
     s_coef[tid] = tid < nv ? reinterpret_cast<const float4*>(rec + A.L.coef_off())[tid] : make_float4(0, 0, 0, 0);
   {
     const float* gW = reinterpret_cast<const float*>(rec + A.L.dense_off());
-    for (int k = tid; k < NVMAX * NVMAX; k += kDThreads) s_W[k] = gW[(k / NVMAX) * kDenseMax + (k % NVMAX)];
+    for (int k = tid; k < NVMAX * NVMAX; k += TPB) s_W[k] = gW[(k / NVMAX) * kDenseMax + (k % NVMAX)];
   }
   __syncthreads();
   uint32_t* split_row = A.split + int64_t(r) * A.n_words;
@@ -642,23 +647,25 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
     const int64_t lrow = prow + A.level_off[d];
     if (fused && nv == 0) {  // constant output: every variance and band value is exactly 0
       if (tid < 32) split_row[A.word_off[d - 1] + mb / 128 + tid] = 0u;
-      if (tid < 128) A.bandb[band_base + A.word_off[d] + mb / 32 + tid] = 0u;
+      for (int k = tid; k < 128; k += TPB) A.bandb[band_base + A.word_off[d] + mb / 32 + k] = 0u;
       return;
     }
-    // quad q = tid + 256 k has parent (pl + 16 (k & 1), ql + 16 (k >> 1)) in the tile
+    // quad q = tid + TPB k of the tile has parent (pl + dx(k), ql + dy(k)), where
+    // (dx, dy) are the Morton coordinates of TPB k (its bits lie above tid's)
     const int pl = int(compact1by1(uint32_t(tid))), ql = int(compact1by1(uint32_t(tid) >> 1));
     const float X0 = grid_coord(i0 + 2 * pl, scale), Y0 = grid_coord(j0 + 2 * ql, scale);
-    const float step = 2.f * scale, jump = 64.f * scale;  // one column; 32 columns
+    const float step = 2.f * scale, quad_step = 4.f * scale;  // one column; one quad (two columns)
     const int sbase = (2 * ql + kPad) * P64 + 2 * pl + kPad;
     // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the nodes
     constexpr int QPE = NVMAX <= 4 ? 2 : 1;
 #pragma unroll 1
-    for (int k0 = 0; k0 < 4; k0 += QPE) {
+    for (int k0 = 0; k0 < QPT; k0 += QPE) {
       float x[4 * QPE], y[4 * QPE], w[4 * QPE];
 #pragma unroll
       for (int h = 0; h < QPE; h++) {
-        const int k = k0 + h;
-        const float xa = (k & 1) ? X0 + jump : X0, ya = (k >> 1) ? Y0 + jump : Y0;
+        const uint32_t kq = uint32_t(TPB * (k0 + h));
+        const float xa = fmaf(float(compact1by1(kq)), quad_step, X0);
+        const float ya = fmaf(float(compact1by1(kq >> 1)), quad_step, Y0);
         x[4 * h + 0] = xa; x[4 * h + 1] = xa + step; x[4 * h + 2] = xa; x[4 * h + 3] = xa + step;
         y[4 * h + 0] = ya; y[4 * h + 1] = ya; y[4 * h + 2] = ya + step; y[4 * h + 3] = ya + step;
       }
@@ -666,23 +673,25 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
 #pragma unroll
       for (int h = 0; h < QPE; h++) {
         const int k = k0 + h;
+        const uint32_t kq = uint32_t(TPB * k);
         const float* wq = w + 4 * h;
         if (fused) {
-          float* t = s_wt + sbase + (k & 1) * 32 + (k >> 1) * 32 * P64;
+          float* t = s_wt + sbase + 2 * int(compact1by1(kq)) + 2 * int(compact1by1(kq >> 1)) * P64;
           *reinterpret_cast<float2*>(t) = make_float2(wq[0], wq[1]);
           *reinterpret_cast<float2*>(t + P64) = make_float2(wq[2], wq[3]);
           // the four children give the parent's variance (Section 3.2)
           const unsigned bal = __ballot_sync(kFull, var_sum4(wq[0], wq[1], wq[2], wq[3]) > theta4);
-          if (lane == 0) split_row[A.word_off[d - 1] + mb / 128 + 8 * k + warp] = bal;
+          if (lane == 0) split_row[A.word_off[d - 1] + mb / 128 + (TPB / 32) * k + warp] = bal;
         } else {
-          *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + 256 * k)) =
+          *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
               make_float4(wq[0], wq[1], wq[2], wq[3]);
         }
       }
     }
-    {
-      // ring: side tid / 64 (warp-uniform), offset tid % 64
-      const int sd = tid >> 6, uu = tid & 63;
+#pragma unroll 1
+    for (int h = 0; h < RPT; h++) {
+      // ring: side t / 64 (warp-uniform), offset t % 64
+      const int t = tid + TPB * h, sd = t >> 6, uu = t & 63;
       const int li = sd == 0 ? -1 : sd == 1 ? kTileSide : uu, lj = sd == 2 ? -1 : sd == 3 ? kTileSide : uu;
       const int gi = i0 + li, gj = j0 + lj;
       const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
@@ -702,8 +711,9 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
     __syncthreads();
     // band value of each position from its four neighbours at distance 2^-d
 #pragma unroll
-    for (int k = 0; k < 4; k++) {
-      const float* t = s_wt + sbase + (k & 1) * 32 + (k >> 1) * 32 * P64;  // position (2pi, 2pj)
+    for (int k = 0; k < QPT; k++) {
+      const uint32_t kq = uint32_t(TPB * k);
+      const float* t = s_wt + sbase + 2 * int(compact1by1(kq)) + 2 * int(compact1by1(kq >> 1)) * P64;  // (2pi, 2pj)
       const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
       const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
       const float l0 = t[-1], l2 = t[P64 - 1], r1 = t[2], r3 = t[P64 + 2];
@@ -725,11 +735,11 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
       }
       const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
       const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-      if (lane < 4)  // quad-major words of this warp's 32 quads (block mb/128 + 8k + warp)
-        A.bandb[band_base + A.word_off[d] + 4 * (mb / 128 + 8 * k + warp) + lane] =
+      if (lane < 4)  // quad-major words of this warp's 32 quads
+        A.bandb[band_base + A.word_off[d] + 4 * (mb / 128 + (TPB / 32) * k + warp) + lane] =
             lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
       if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
-        float* o = A.out + lrow + mb + 4 * (tid + 256 * k);
+        float* o = A.out + lrow + mb + 4 * (tid + TPB * k);
 #pragma unroll
         for (int c = 0; c < 4; c++)
           if (pass[c]) o[c] = w[c];
@@ -746,64 +756,80 @@ __global__ void __launch_bounds__(kDThreads, NVMAX <= 4 ? 4 : 2) tile_kernel_den
     const int nq = T * T / 4, nring = 4 * T, pitch = T + 2 * kPad;
     const int64_t lrow = prow + A.level_off[d];
     if (fused && nv == 0) {
-      if (d >= 1 && tid < (nq + 31) / 32) split_row[A.word_off[d - 1] + tid] = 0u;
-      if (tid < (4 * nq + 31) / 32) A.bandb[band_base + A.word_off[d] + tid] = 0u;
+      for (int k = tid; k < (nq + 31) / 32; k += TPB)
+        if (d >= 1) split_row[A.word_off[d - 1] + k] = 0u;
+      for (int k = tid; k < (4 * nq + 31) / 32; k += TPB) A.bandb[band_base + A.word_off[d] + k] = 0u;
       continue;
     }
-    const int q = tid;
-    const bool valid = q < nq;
-    const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-    float w[4] = {0.f, 0.f, 0.f, 0.f};
-    if (valid) {
-      const float xa = grid_coord(2 * pi, scale), xb = grid_coord(2 * pi + 1, scale);
-      const float ya = grid_coord(2 * pj, scale), yb = grid_coord(2 * pj + 1, scale);
-      const float x[4] = {xa, xb, xa, xb}, y[4] = {ya, ya, yb, yb};
-      eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
-      if (fused) {
-        float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
-        t[0] = w[0]; t[1] = w[1]; t[pitch] = w[2]; t[pitch + 1] = w[3];
-      } else {
-        *reinterpret_cast<float4*>(A.out + lrow + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+    for (int base = 0; base < nq; base += TPB) {
+      const int q = base + tid;
+      const bool valid = q < nq;
+      const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+      float w[4] = {0.f, 0.f, 0.f, 0.f};
+      if (valid) {
+        const float xa = grid_coord(2 * pi, scale), xb = grid_coord(2 * pi + 1, scale);
+        const float ya = grid_coord(2 * pj, scale), yb = grid_coord(2 * pj + 1, scale);
+        const float x[4] = {xa, xb, xa, xb}, y[4] = {ya, ya, yb, yb};
+        eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
+        if (fused) {
+          float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+          t[0] = w[0]; t[1] = w[1]; t[pitch] = w[2]; t[pitch + 1] = w[3];
+        } else {
+          *reinterpret_cast<float4*>(A.out + lrow + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+        }
+      }
+      if (fused && d >= 1) {
+        const unsigned bal = __ballot_sync(kFull, valid && var_sum4(w[0], w[1], w[2], w[3]) > theta4);
+        const int q0 = base + warp * 32;
+        if (lane == 0 && q0 < nq) split_row[A.word_off[d - 1] + q0 / 32] = bal;
       }
     }
-    if (fused && d >= 1) {
-      const unsigned bal = __ballot_sync(kFull, valid && var_sum4(w[0], w[1], w[2], w[3]) > theta4);
-      if (lane == 0 && warp * 32 < nq) split_row[A.word_off[d - 1] + warp] = bal;
-    }
-    if ((fused || A.out_halo) && tid < nring) {
-      const int sd = tid / T, uu = tid - sd * T;
-      const int li = sd == 0 ? -1 : sd == 1 ? T : uu, lj = sd == 2 ? -1 : sd == 3 ? T : uu;
-      const float x[1] = {grid_coord(li, scale)}, y[1] = {grid_coord(lj, scale)};
-      float wr[1];
-      eval_dense<NVMAX, 1>(s_coef, s_W, nv, out_const, x, y, wr);
-      if (fused) s_wt[(lj + kPad) * pitch + li + kPad] = wr[0];
-      else A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + sd * n + uu] = wr[0];
+    if (fused || A.out_halo) {
+      for (int t = tid; t < nring; t += TPB) {
+        const int sd = t / T, uu = t - sd * T;
+        const int li = sd == 0 ? -1 : sd == 1 ? T : uu, lj = sd == 2 ? -1 : sd == 3 ? T : uu;
+        const float x[1] = {grid_coord(li, scale)}, y[1] = {grid_coord(lj, scale)};
+        float wr[1];
+        eval_dense<NVMAX, 1>(s_coef, s_W, nv, out_const, x, y, wr);
+        if (fused) s_wt[(lj + kPad) * pitch + li + kPad] = wr[0];
+        else A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + sd * n + uu] = wr[0];
+      }
     }
     if (!fused) continue;
     __syncthreads();
-    bool pass[4] = {false, false, false, false};
-    if (valid) {
-      const float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
-      const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
-      const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]}, U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
+    for (int base = 0; base < nq; base += TPB) {
+      const int q = base + tid;
+      const bool valid = q < nq;
+      bool pass[4] = {false, false, false, false};
+      float w[4] = {0.f, 0.f, 0.f, 0.f};
+      if (valid) {
+        const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+        const float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+        w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
+        const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
+        const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
+        const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
 #pragma unroll
-      for (int c = 0; c < 4; c++) {
-        pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]), band2);
-        if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+        for (int c = 0; c < 4; c++) {
+          pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]),
+                                 band2);
+          if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+        }
       }
-    }
-    const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
-    const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-    if (d >= kQuadMajorFrom) {
-      if (lane < 4 && warp * 32 < nq)
-        A.bandb[band_base + A.word_off[d] + 4 * warp + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
-    } else if (warp == 0 && lane * 32 < 4 * nq) {
-      A.bandb[band_base + A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
-    }
-    if (A.out && valid && (pass[0] | pass[1] | pass[2] | pass[3])) {
+      const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+      const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+      const int q0 = base + warp * 32;
+      if (d >= kQuadMajorFrom) {
+        if (lane < 4 && q0 < nq)
+          A.bandb[band_base + A.word_off[d] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+      } else if (q0 == 0 && lane * 32 < 4 * nq) {
+        A.bandb[band_base + A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
+      }
+      if (A.out && valid && (pass[0] | pass[1] | pass[2] | pass[3])) {
 #pragma unroll
-      for (int c = 0; c < 4; c++)
-        if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
+        for (int c = 0; c < 4; c++)
+          if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
+      }
     }
     __syncthreads();
   }
@@ -905,44 +931,61 @@ struct PlaneView {
   __device__ __forceinline__ uint32_t& at(int64_t r, int64_t w) const { return p[r * stride + w - shift]; }
 };
 
-// mask = band AND NOT split (no split at depth D); gated: AND Eq. 2's active bit.
-// Threads cover words [w0, w0 + nw) of every pair; split is a whole-grid plane.
-__global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView band, PlaneView mask, GridDev G,
-                               int64_t n_pairs, int64_t w0, int64_t nw, int gated) {
-  const int64_t wg = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (wg >= n_pairs * nw) return;
-  const int64_t r = wg / nw, wi = w0 + wg % nw;
-  const int d = level_of_word(G, wi);
+// Active bits (Eq. 2: every ancestor split) of the 32 positions of word wi at
+// depth d; the ancestors at each shallower depth lie in a single word.
+__device__ __forceinline__ uint32_t active_bits(const uint32_t* sp, const GridDev& G, int d, int64_t wi) {
   const uint32_t m0 = uint32_t(wi - G.word_off[d]) * 32u;
-  const uint32_t valid = valid_bits(G, d, wi);
-  const uint32_t* sp = split + r * G.n_words;
-  uint32_t bw;
-  if (d >= kQuadMajorFrom) {  // re-interleave the block's four child words
-    const int64_t j = wi - G.word_off[d];
-    const uint4 bq = *reinterpret_cast<const uint4*>(&band.at(r, G.word_off[d] + 4 * (j >> 2)));
-    bw = band_word(bq.x, bq.y, bq.z, bq.w, int(j & 3));
-  } else {
-    bw = band.at(r, wi);
-  }
-  uint32_t keep = bw & valid;
-  if (d < G.D) keep &= ~sp[wi];
-  if (gated && keep) {
-    // active(p) = every ancestor split (Eq. 2); the ancestors of these 32
-    // positions at each shallower depth lie in a single word.
-    uint32_t act = kFull;
-    for (int k = 1; k <= d && act; k++) {
-      const uint32_t a0 = m0 >> (2 * k);
-      const uint32_t aw = sp[G.word_off[d - k] + (a0 >> 5)];
-      uint32_t bits = 0;
-      for (int bb = 0; bb < 32; bb++) {
-        const uint32_t anc = (m0 + uint32_t(bb)) >> (2 * k);
-        bits |= ((aw >> (anc & 31u)) & 1u) << bb;
-      }
-      act &= bits;
+  uint32_t act = kFull;
+  for (int k = 1; k <= d && act; k++) {
+    const uint32_t a0 = m0 >> (2 * k);
+    const uint32_t aw = sp[G.word_off[d - k] + (a0 >> 5)];
+    uint32_t bits = 0;
+    for (int bb = 0; bb < 32; bb++) {
+      const uint32_t anc = (m0 + uint32_t(bb)) >> (2 * k);
+      bits |= ((aw >> (anc & 31u)) & 1u) << bb;
     }
-    keep &= act;
+    act &= bits;
   }
-  mask.at(r, wi) = keep;
+  return act;
+}
+
+// mask = band AND NOT split (no split at depth D); gated: AND Eq. 2's active bit.
+// One thread per group of 4 words (one 128-position block from depth 3 on; the
+// 4 words of depths 0..2 form group 0), pair = blockIdx.y; groups cover words
+// [w0, w0 + nw) (w0 and nw multiples of 4, or nw reaching n_words). split is a
+// whole-grid plane.
+__global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView band, PlaneView mask, GridDev G,
+                               int64_t w0, int64_t nw, int gated) {
+  const int64_t k = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) * 4;
+  if (k >= nw) return;
+  const int64_t r = blockIdx.y;
+  const int64_t wi = w0 + k;
+  const uint32_t* sp = split + r * G.n_words;
+  uint32_t m[4];
+  const int nwk = nw - k < 4 ? int(nw - k) : 4;
+  if (wi >= G.word_off[kQuadMajorFrom]) {
+    int d = kQuadMajorFrom;
+    while (G.word_off[d + 1] <= wi) d++;
+    const uint4 bq = *reinterpret_cast<const uint4*>(&band.at(r, wi));
+    const uint4 sq = d < G.D ? *reinterpret_cast<const uint4*>(sp + wi) : make_uint4(0, 0, 0, 0);
+    const uint32_t s4[4] = {sq.x, sq.y, sq.z, sq.w};
+#pragma unroll
+    for (int c = 0; c < 4; c++) {  // re-interleave the block's four child words
+      m[c] = band_word(bq.x, bq.y, bq.z, bq.w, c) & ~s4[c];
+      if (gated && m[c]) m[c] &= active_bits(sp, G, d, wi + c);
+    }
+    *reinterpret_cast<uint4*>(&mask.at(r, wi)) = make_uint4(m[0], m[1], m[2], m[3]);
+  } else {
+    for (int c = 0; c < nwk; c++) {
+      const int64_t wc = wi + c;
+      int d = 0;
+      while (G.word_off[d + 1] <= wc) d++;
+      uint32_t keep = band.at(r, wc) & valid_bits(G, d, wc);
+      if (d < G.D) keep &= ~sp[wc];
+      if (gated && keep) keep &= active_bits(sp, G, d, wc);
+      mask.at(r, wc) = keep;
+    }
+  }
 }
 
 // ---- ordered compaction -----------------------------------------------------------
@@ -975,17 +1018,34 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int* total) 
   return before + x - v;
 }
 
-__global__ void compact_count_kernel(PlaneView mask, GridDev G, int64_t w0, int64_t nw, int nb,
+// Four words of pair r starting at word wi (a multiple of 4) with the bits that
+// are not grid positions cleared; words past w_end read as 0.
+__device__ __forceinline__ void load_mask4(const PlaneView& mask, const GridDev& G, int64_t r, int64_t wi,
+                                           int64_t w_end, uint32_t (&m)[4]) {
+  if (wi + 4 <= w_end && wi >= G.word_off[kQuadMajorFrom]) {
+    const uint4 v = *reinterpret_cast<const uint4*>(&mask.at(r, wi));
+    m[0] = v.x; m[1] = v.y; m[2] = v.z; m[3] = v.w;
+    return;
+  }
+#pragma unroll
+  for (int c = 0; c < 4; c++) {
+    const int64_t wc = wi + c;
+    m[c] = wc < w_end ? mask.at(r, wc) & valid_bits(G, level_of_word(G, wc), wc) : 0u;
+  }
+}
+
+// grid (blocks of kCompactBlock * 4 words, pairs): set bits per block.
+__global__ void compact_count_kernel(PlaneView mask, GridDev G, int64_t w0, int64_t nw, int nb, int64_t r0,
                                      int32_t* __restrict__ bcount) {
   __shared__ int sh[32];
-  const int64_t r = blockIdx.x / nb;
-  const int b = int(blockIdx.x % nb);
-  const int64_t k = int64_t(b) * kCompactBlock + threadIdx.x;
-  const int64_t wi = w0 + k;
-  const int c = k < nw ? __popc(mask.at(r, wi) & valid_bits(G, level_of_word(G, wi), wi)) : 0;
+  const int64_t r = r0 + blockIdx.y;
+  const int64_t k = (int64_t(blockIdx.x) * kCompactBlock + threadIdx.x) * 4;
+  uint32_t m[4] = {0u, 0u, 0u, 0u};
+  if (k < nw) load_mask4(mask, G, r, w0 + k, w0 + nw, m);
+  const int c = __popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]);
   int total;
   block_exclusive_scan(c, sh, &total);
-  if (threadIdx.x == 0) bcount[blockIdx.x] = total;
+  if (threadIdx.x == 0) bcount[r * nb + blockIdx.x] = total;
 }
 
 // One CTA per pair: exclusive scan of its block counts.
@@ -1042,25 +1102,28 @@ __global__ void compact_scan_pairs_kernel(const int64_t* __restrict__ counts, in
 
 // out: output at global index p of pair r is out[r * out_stride + p - out_shift].
 __global__ void compact_write_kernel(PlaneView mask, const float* __restrict__ out, int64_t out_stride,
-                                     int64_t out_shift, GridDev G, int64_t w0, int64_t nw, int nb,
+                                     int64_t out_shift, GridDev G, int64_t w0, int64_t nw, int nb, int64_t r0,
                                      const int32_t* __restrict__ boff, const int64_t* __restrict__ offsets, int64_t cap,
                                      int32_t* __restrict__ idx, float* __restrict__ wv) {
   __shared__ int sh[32];
-  const int64_t r = blockIdx.x / nb;
-  const int b = int(blockIdx.x % nb);
-  const int64_t k = int64_t(b) * kCompactBlock + threadIdx.x;
-  const int64_t wi = w0 + k;
-  const int d = k < nw ? level_of_word(G, wi) : 0;
-  const uint32_t bits = k < nw ? mask.at(r, wi) & valid_bits(G, d, wi) : 0u;
-  const int ex = block_exclusive_scan(__popc(bits), sh, nullptr);
-  if (!bits) return;
-  const int64_t gbase = G.level_off[d] + (wi - G.word_off[d]) * 32;
-  int64_t dst = offsets[r] + boff[blockIdx.x] + ex;
-  for (uint32_t v = bits; v; v &= v - 1, dst++) {
-    const int64_t gidx = gbase + __ffs(v) - 1;
-    if (dst < cap) {
-      idx[dst] = int32_t(gidx);
-      if (wv) wv[dst] = out[r * out_stride + gidx - out_shift];
+  const int64_t r = r0 + blockIdx.y;
+  const int64_t k = (int64_t(blockIdx.x) * kCompactBlock + threadIdx.x) * 4;
+  uint32_t m[4] = {0u, 0u, 0u, 0u};
+  if (k < nw) load_mask4(mask, G, r, w0 + k, w0 + nw, m);
+  const int ex = block_exclusive_scan(__popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]), sh, nullptr);
+  if (!(m[0] | m[1] | m[2] | m[3])) return;
+  int64_t dst = offsets[r] + boff[r * nb + blockIdx.x] + ex;
+  for (int c = 0; c < 4; c++) {
+    if (!m[c]) continue;
+    const int64_t wi = w0 + k + c;
+    const int d = level_of_word(G, wi);
+    const int64_t gbase = G.level_off[d] + (wi - G.word_off[d]) * 32;
+    for (uint32_t v = m[c]; v; v &= v - 1, dst++) {
+      const int64_t gidx = gbase + __ffs(v) - 1;
+      if (dst < cap) {
+        idx[dst] = int32_t(gidx);
+        if (wv) wv[dst] = out[r * out_stride + gidx - out_shift];
+      }
     }
   }
 }
@@ -1078,10 +1141,11 @@ GridDev grid_dev(const emr_grid* g) {
   G.n_halo = g->n_halo;
   G.n_words = g->n_words;
   int64_t qb = 0;
-  for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {
-    G.level_off[d] = g->level_off[d];
-    G.halo_off[d] = g->halo_off[d];
-    G.word_off[d] = g->word_off[d];
+  for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {  // entries past D + 1 repeat the totals
+    const int e = d <= g->D + 1 ? d : g->D + 1;
+    G.level_off[d] = g->level_off[e];
+    G.halo_off[d] = g->halo_off[e];
+    G.word_off[d] = g->word_off[e];
     G.qblk_off[d] = qb;
     if (d <= g->D) qb += ((int64_t(1) << (2 * d)) + 31) / 32;
   }
@@ -1156,8 +1220,8 @@ emr_status prepare(const void* pack_dev, const emr_query* q, const EvalPlan& p, 
   const QueryDev qd = query_dev(q);
   const uint8_t* pk = static_cast<const uint8_t*>(pack_dev);
   schedule_kernel<<<1, 1024, 0, st>>>(pk, qd, p.n_pairs, *order);
-  spec_kernel<<<unsigned((p.n_pairs + 127) / 128), 128, 0, st>>>(pk, qd, p.n_pairs, p.L, *spec, scratch,
-                                                                   p.scratch_stride);
+  spec_kernel<<<unsigned((p.n_pairs + 31) / 32), 32, 0, st>>>(pk, qd, p.n_pairs, p.L, *spec, scratch,
+                                                                 p.scratch_stride);
   return cuda_status(cudaGetLastError());
 }
 
@@ -1172,6 +1236,8 @@ int64_t dense_tiles(int D) {
   return t;
 }
 
+constexpr int kDenseTPB = 128;  // threads per dense tile CTA
+
 template <int NVMAX>
 emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st) {
   if (n_ranks <= 0) return EMR_OK;
@@ -1179,7 +1245,7 @@ emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, 
   A.rank_beg = rank_beg;
   const int64_t blocks = n_ranks * int64_t(A.n_tiles);
   if (blocks > 0x7fffffffLL) return EMR_ERR_RANGE;
-  tile_kernel_dense<NVMAX><<<unsigned(blocks), kDThreads, 0, st>>>(A);
+  tile_kernel_dense<NVMAX, kDenseTPB><<<unsigned(blocks), kDenseTPB, 0, st>>>(A);
   return cuda_status(cudaGetLastError());
 }
 
@@ -1285,10 +1351,21 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
 
 emr_status launch_combine(const uint32_t* split, PlaneView band, PlaneView mask, const emr_grid* g, int64_t n_pairs,
                           int64_t w0, int64_t nw, int gated, cudaStream_t st) {
-  const int64_t n = n_pairs * nw;
-  if (n <= 0) return EMR_OK;
-  if ((n + 255) / 256 > 0x7fffffffLL) return EMR_ERR_RANGE;
-  combine_kernel<<<unsigned((n + 255) / 256), 256, 0, st>>>(split, band, mask, grid_dev(g), n_pairs, w0, nw, gated);
+  if (n_pairs <= 0 || nw <= 0) return EMR_OK;
+  if (n_pairs > 65535) {  // grid y limit: split the pairs
+    for (int64_t r0 = 0; r0 < n_pairs; r0 += 65535) {
+      const int64_t nr = std::min<int64_t>(65535, n_pairs - r0);
+      PlaneView b2 = band, m2 = mask;
+      b2.p += r0 * band.stride;
+      m2.p += r0 * mask.stride;
+      emr_status rc = launch_combine(split + r0 * g->n_words, b2, m2, g, nr, w0, nw, gated, st);
+      if (rc != EMR_OK) return rc;
+    }
+    return EMR_OK;
+  }
+  const int64_t groups = (nw + 3) / 4;
+  dim3 grid(unsigned((groups + 255) / 256), unsigned(n_pairs));
+  combine_kernel<<<grid, 256, 0, st>>>(split, band, mask, grid_dev(g), w0, nw, gated);
   return cuda_status(cudaGetLastError());
 }
 
@@ -1298,8 +1375,10 @@ emr_status launch_combine(const uint32_t* split, const uint32_t* bandb, const em
                         PlaneView{mask, g->n_words, 0}, g, n_pairs, 0, g->n_words, gated, st);
 }
 
+constexpr int64_t kCompactWords = 4 * kCompactBlock;  // words per compaction block
+
 size_t compact_ws_bytes(int64_t nw, int64_t n_pairs) {
-  const int64_t nb = (nw + kCompactBlock - 1) / kCompactBlock;
+  const int64_t nb = (nw + kCompactWords - 1) / kCompactWords;
   return size_t(2 * 4 * nb * n_pairs + 256);
 }
 
@@ -1307,17 +1386,23 @@ size_t compact_ws_bytes(int64_t nw, int64_t n_pairs) {
 emr_status launch_compact(PlaneView mask, const float* out, int64_t out_stride, int64_t out_shift, const emr_grid* g,
                           int64_t n_pairs, int64_t w0, int64_t nw, int32_t* idx, float* w, int64_t cap, int64_t* counts,
                           int64_t* offsets, void* ws, cudaStream_t st) {
-  const int nb = int((nw + kCompactBlock - 1) / kCompactBlock);
+  const int nb = int((nw + kCompactWords - 1) / kCompactWords);
   const int64_t nblk = int64_t(nb) * n_pairs;
-  if (nblk > 0x7fffffffLL || n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
+  if (n_pairs <= 0 || n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
   int32_t* bcount = static_cast<int32_t*>(ws);
   int32_t* boff = bcount + nblk;
   const GridDev G = grid_dev(g);
-  compact_count_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, G, w0, nw, nb, bcount);
+  for (int64_t r0 = 0; r0 < n_pairs; r0 += 65535) {  // grid y holds at most 65535 pairs
+    const dim3 grid(unsigned(nb), unsigned(std::min<int64_t>(65535, n_pairs - r0)));
+    compact_count_kernel<<<grid, kCompactBlock, 0, st>>>(mask, G, w0, nw, nb, r0, bcount);
+  }
   compact_scan_pair_kernel<<<unsigned(n_pairs), 256, 0, st>>>(bcount, nb, boff, counts);
   compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, n_pairs, offsets);
-  compact_write_kernel<<<unsigned(nblk), kCompactBlock, 0, st>>>(mask, out, out_stride, out_shift, G, w0, nw, nb, boff,
-                                                                 offsets, cap, idx, w);
+  for (int64_t r0 = 0; r0 < n_pairs; r0 += 65535) {
+    const dim3 grid(unsigned(nb), unsigned(std::min<int64_t>(65535, n_pairs - r0)));
+    compact_write_kernel<<<grid, kCompactBlock, 0, st>>>(mask, out, out_stride, out_shift, G, w0, nw, nb, r0, boff,
+                                                         offsets, cap, idx, w);
+  }
   return cuda_status(cudaGetLastError());
 }
 

@@ -163,9 +163,10 @@ emr_status emr_grid_build(int32_t D, int64_t chunk, emr_grid* grid) {
   grid->D = D;
   grid->chunk = chunk;
   int64_t words = 0;
-  for (int d = 0; d <= D + 1; d++) {
-    grid->level_off[d] = level_offset(d);
-    grid->halo_off[d] = halo_offset(d);
+  for (int d = 0; d < EMR_MAX_DEPTH + 2; d++) {  // entries past D + 1 repeat the totals
+    const int e = d <= D + 1 ? d : D + 1;
+    grid->level_off[d] = level_offset(e);
+    grid->halo_off[d] = halo_offset(e);
     grid->word_off[d] = words;
     if (d <= D) words += ((int64_t(1) << (2 * (d + 1))) + 31) / 32;
   }

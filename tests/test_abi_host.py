@@ -47,6 +47,8 @@ def test_grid_descriptor_matches_eq1_counts(D):
         assert g.halo_off[d] == 8 * (2 ** d - 1)
         assert g.word_off[d + 1] - g.word_off[d] == -(-(4 ** (d + 1)) // 32)
     assert g.level_off[D + 1] == g.n_total and g.word_off[D + 1] == g.n_words
+    for d in range(D + 1, 16):  # entries past D + 1 repeat the totals
+        assert (g.level_off[d], g.halo_off[d], g.word_off[d]) == (g.n_total, g.n_halo, g.n_words)
 
 
 def test_grid_descriptor_errors():

@@ -610,7 +610,6 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
   static_assert(NVMAX <= kDenseMax, "dense block holds kDenseMax rows");
   static_assert(TPB >= 64 && TPB <= 256 && (TPB & (TPB - 1)) == 0, "tile work divides evenly");
   constexpr int QPT = kTileSide * kTileSide / 4 / TPB;  // quads per thread in a 64 x 64 tile
-  constexpr int RPT = 4 * kTileSide / TPB;               // ring points per thread
   constexpr int P64 = kTileSide + 2 * kPad;
   __shared__ float4 s_coef[NVMAX];
   __shared__ __align__(16) float s_W[NVMAX * NVMAX];
@@ -688,29 +687,41 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
         }
       }
     }
-#pragma unroll 1
-    for (int h = 0; h < RPT; h++) {
-      // ring: side t / 64 (warp-uniform), offset t % 64
-      const int t = tid + TPB * h, sd = t >> 6, uu = t & 63;
-      const int li = sd == 0 ? -1 : sd == 1 ? kTileSide : uu, lj = sd == 2 ? -1 : sd == 3 ? kTileSide : uu;
-      const int gi = i0 + li, gj = j0 + lj;
+    // ring: 4 sides x 64 points, evaluated four at a time by threads 0..63
+    // (point t = 4 tid + c lies on side t / 64, the same for all four)
+    if (tid < kTileSide && (fused || A.out_halo)) {
+      const int sd = tid >> 4, u0 = 4 * (tid & 15);
+      int li[4], lj[4];
+      float x[4], y[4], w[4];
+      bool use = fused;
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        li[c] = sd == 0 ? -1 : sd == 1 ? kTileSide : u0 + c;
+        lj[c] = sd == 2 ? -1 : sd == 3 ? kTileSide : u0 + c;
+        x[c] = grid_coord(i0 + li[c], scale);
+        y[c] = grid_coord(j0 + lj[c], scale);
+      }
+      const int gi = i0 + li[0], gj = j0 + lj[0];  // a side lies wholly inside or outside the domain
       const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
-      if (fused || (A.out_halo && outside)) {
-        const float x[1] = {grid_coord(gi, scale)}, y[1] = {grid_coord(gj, scale)};
-        float w[1];
-        eval_dense<NVMAX, 1>(s_coef, s_W, nv, out_const, x, y, w);
-        if (fused) {
-          s_wt[(lj + kPad) * P64 + li + kPad] = w[0];
-        } else {
-          const int hs = gi < 0 ? 0 : gi >= n ? 1 : gj < 0 ? 2 : 3;
-          A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? gj : gi)] = w[0];
+      use = use || outside;  // materialised: only points outside the domain are written
+      if (use) {
+        eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
+#pragma unroll
+        for (int c = 0; c < 4; c++) {
+          if (fused) {
+            s_wt[(lj[c] + kPad) * P64 + li[c] + kPad] = w[c];
+          } else {
+            const int pi_ = i0 + li[c], pj_ = j0 + lj[c];
+            const int hs = pi_ < 0 ? 0 : pi_ >= n ? 1 : pj_ < 0 ? 2 : 3;
+            A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? pj_ : pi_)] = w[c];
+          }
         }
       }
     }
     if (!fused) return;
     __syncthreads();
     // band value of each position from its four neighbours at distance 2^-d
-#pragma unroll
+#pragma unroll 2
     for (int k = 0; k < QPT; k++) {
       const uint32_t kq = uint32_t(TPB * k);
       const float* t = s_wt + sbase + 2 * int(compact1by1(kq)) + 2 * int(compact1by1(kq >> 1)) * P64;  // (2pi, 2pj)

@@ -53,6 +53,7 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-genomes", type=int, default=160, help="oracle baseline sample (genomes)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra", action="store_true", help="skip the streamed depth-13 and h->h round measurements")
     return ap.parse_args()
 
 
@@ -175,6 +176,52 @@ def alu_probe(emr, sms):
     return out
 
 
+def profiled_traffic():
+    """DRAM bytes per step of the dense tile kernels from the committed ncu summary, if that
+    summary was taken on the current kernel source (else None)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "tile_kernel_dense_c2_pop100_d7.md")
+    src = os.path.join(ROOT, "paper_2608_27612_gb300", "csrc", "emr_kernels.cu")
+    try:
+        fields = dict(l.split(":", 1) for l in open(path).read().splitlines() if l.startswith(("traffic_", "kernel_")))
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if fields.get("kernel_source_sha256", "").strip() == sha:
+            return int(fields["traffic_bytes_per_step"])
+    except (OSError, ValueError, KeyError):
+        pass
+    return None
+
+
+def streamed_run(emr, torch, w, chunk, chunk_cap, cap, reps):
+    """Queries/sec of emr_stream on workload w (lists copied to pinned host memory)."""
+    pack = emr.pack_population(w.pop)
+    pack_dev = torch.from_numpy(pack).cuda()
+    q = emr.make_query(w.sources)
+    g = emr.grid_build(w.D, chunk)
+    ws = torch.empty(emr.stream_workspace_size(pack, q, g, chunk_cap), dtype=torch.uint8, device="cuda")
+    n_pairs = w.P * q.S
+    h_idx = torch.empty(cap, dtype=torch.int32).pin_memory()
+    h_w = torch.empty(cap, dtype=torch.float32).pin_memory()
+    counts = np.zeros(n_pairs, np.int64)
+    offsets = np.zeros(n_pairs + 1, np.int64)
+    queries = float(n_pairs) * g.n_total
+    if w.sources.count is not None:
+        queries = float(w.sources.count.sum()) * g.n_total
+    times = []
+    for k in range(reps + 1):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        emr.stream(pack, pack_dev, q, g, w.theta, w.band, w.w_min, ws, chunk_cap, h_idx, h_w, counts, offsets)
+        if k:
+            times.append(time.perf_counter() - t0)
+    del ws
+    torch.cuda.empty_cache()
+    s = statistics.median(times)
+    return {"workload": w.name, "queries": queries, "seconds": s, "value": queries / s, "unit": UNIT,
+            "chunk_positions": chunk, "kept": int(offsets[-1]),
+            "timing": "host wall clock per emr_stream call (synchronous, lists on the host), median of %d" % reps}
+
+
 def oracle_baseline(w, genomes):
     import oracle
     oracle.build()
@@ -292,7 +339,10 @@ def main():
     peak = sms * FP32_PER_SM_CLK * SM_MAX_MHZ * 1e6
     achieved = work_eq / tile_s
     roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": peak / 1e12, "unit": "Tlane-op/s",
-                "frac": achieved / peak, "traffic": None, "kernel": "tile_kernel (emr_eval_filter)",
+                "frac": achieved / peak, "traffic": profiled_traffic() if args.pop == 1000 and args.depth == 7 else None,
+                "traffic_note": "DRAM bytes of the dense tile launches per step, from profiles/"
+                                "tile_kernel_dense_c2_pop100_d7.md (100-genome capture scaled x10); null when "
+                                "the kernel source changed since", "kernel": "tile_kernel_dense (emr_eval_filter)",
                 "kernel_ms": tile_s * 1e3,
                 "fp32_ops_per_query": float(work[..., 0].mean()), "mufu_ops_per_query": float(work[..., 1].mean()),
                 "peak_basis": "%d SMs x %d FP32 lanes x %.0f MHz (max SM clock); a MUFU op weighs %.2f FP32 "
@@ -338,6 +388,11 @@ def main():
         e2e = {"value": ws * queries / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": e2e_s * 1e3}
 
+    extra = None
+    if rank == 0 and ws == 1 and not args.no_extra:
+        extra = {"c5_streamed_d13": streamed_run(emr, torch, W.c5(), 1 << 26, 1 << 24, 1 << 26, 3),
+                 "c4_round2_hh_d8": streamed_run(emr, torch, W.c4_round2_random(), 1 << 16, 1 << 24, 1 << 26, 3)}
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = oracle_baseline(w, min(args.cpu_genomes, w.P))
@@ -352,7 +407,7 @@ def main():
                        "queries_per_step": queries, "theta": w.theta, "band": w.band, "mode": "eager",
                        "l2": "flushed between steps (256 MB write)", "kept_connections": kept,
                        "parallelism": "independent populations per GPU" if ws > 1 else "single GPU"},
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "extra": extra,
             "gpu_launches": launches_per_step * args.steps, "clocks": clocks,
             "wall_s_timed_region": wall, "gpu": props.name,
         }))

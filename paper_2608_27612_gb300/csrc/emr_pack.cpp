@@ -1,7 +1,8 @@
 // Host side of libemr: grid descriptor (Eq. 1), genome packer, status strings.
 #include <algorithm>
 #include <cstring>
-#include <unordered_map>
+#include <thread>
+#include <utility>
 #include <vector>
 
 #include "emr_internal.h"
@@ -34,96 +35,151 @@ struct GenomeOut {
   PackGenome g{};
 };
 
+struct Edge {
+  int s, d;
+  float w;
+};
+
+// Buffers reused across genomes (capacity kept; no allocation per genome once warm).
+struct Scratch {
+  std::vector<std::pair<int32_t, int>> ids;  // (id, local index), sorted by id
+  std::vector<Edge> es;
+  std::vector<int> indeg, order, ready, stack, slot, kept;
+  std::vector<int> succ_beg, succ, pred_beg, pred, fill;
+  std::vector<char> reach;
+  std::vector<unsigned> has_in;
+  std::vector<int> in_cnt, in_beg;
+  std::vector<PackEdge> in_edges;
+};
+
+int local_of(const Scratch& S, int32_t id) {
+  auto it = std::lower_bound(S.ids.begin(), S.ids.end(), std::make_pair(id, -1));
+  return (it != S.ids.end() && it->first == id) ? it->second : -1;
+}
+
+// CSR adjacency (by source for succ, by destination for pred) over the enabled edges.
+void build_csr(int n, const std::vector<Edge>& es, bool by_src, std::vector<int>& beg, std::vector<int>& adj,
+               std::vector<int>& fill) {
+  beg.assign(n + 1, 0);
+  for (auto& e : es) beg[(by_src ? e.s : e.d) + 1]++;
+  for (int v = 0; v < n; v++) beg[v + 1] += beg[v];
+  adj.resize(es.size());
+  fill.assign(n, 0);
+  for (auto& e : es) {
+    const int k = by_src ? e.s : e.d;
+    adj[beg[k] + fill[k]++] = by_src ? e.d : e.s;
+  }
+}
+
 // Topological order (Kahn, ties by id), dead-node removal, input folding and
 // per-side variation flags for one genome.
 emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_t* node_id,
                     const int32_t* node_kind, const int32_t* node_act, const float* node_bias,
                     const int32_t* conn_src, const int32_t* conn_dst, const float* conn_w,
-                    const uint8_t* conn_en, GenomeOut* out) {
+                    const uint8_t* conn_en, Scratch& S, GenomeOut* out) {
   const int n = int(n1 - n0);
   if (n <= 0 || n > 1 << 20) return EMR_ERR_ARG;
-  std::unordered_map<int32_t, int> local;
+  S.ids.clear();
   int out_node = -1;
   for (int k = 0; k < n; k++) {
-    int kind = node_kind[n0 + k];
+    const int kind = node_kind[n0 + k];
     if (kind < 0 || kind > EMR_KIND_OUTPUT) return EMR_ERR_ARG;
     if (kind >= EMR_KIND_HIDDEN && (node_act[n0 + k] < 0 || node_act[n0 + k] > EMR_ACT_ABS)) return EMR_ERR_ARG;
-    if (!local.emplace(node_id[n0 + k], k).second) return EMR_ERR_ARG;
     if (kind == EMR_KIND_OUTPUT) {
       if (out_node >= 0) return EMR_ERR_ARG;
       out_node = k;
     }
+    S.ids.push_back({node_id[n0 + k], k});
   }
   if (out_node < 0) return EMR_ERR_ARG;
-  struct E { int s, d; float w; };
-  std::vector<E> es;
+  std::sort(S.ids.begin(), S.ids.end());
+  for (size_t k = 1; k < S.ids.size(); k++)
+    if (S.ids[k].first == S.ids[k - 1].first) return EMR_ERR_ARG;  // duplicate id
+  S.es.clear();
   for (int64_t c = c0; c < c1; c++) {
     if (!conn_en[c]) continue;
-    auto is = local.find(conn_src[c]), id = local.find(conn_dst[c]);
-    if (is == local.end() || id == local.end()) return EMR_ERR_ARG;
-    if (node_kind[n0 + id->second] < EMR_KIND_HIDDEN) return EMR_ERR_ARG;
-    es.push_back({is->second, id->second, conn_w[c]});
+    const int ls = local_of(S, conn_src[c]), ld = local_of(S, conn_dst[c]);
+    if (ls < 0 || ld < 0) return EMR_ERR_ARG;
+    if (node_kind[n0 + ld] < EMR_KIND_HIDDEN) return EMR_ERR_ARG;
+    S.es.push_back({ls, ld, conn_w[c]});
   }
+  build_csr(n, S.es, true, S.succ_beg, S.succ, S.fill);
+  build_csr(n, S.es, false, S.pred_beg, S.pred, S.fill);
   // Kahn's algorithm over every node; ready nodes leave in ascending id order.
-  std::vector<int> indeg(n, 0), order;
-  std::vector<std::vector<int>> succ(n), pred(n);
-  for (auto& e : es) { indeg[e.d]++; succ[e.s].push_back(e.d); pred[e.d].push_back(e.s); }
+  S.indeg.assign(n, 0);
+  for (auto& e : S.es) S.indeg[e.d]++;
+  S.order.clear();
+  S.ready.clear();
   auto by_id = [&](int a, int b) { return node_id[n0 + a] > node_id[n0 + b]; };  // min-heap on id
-  std::vector<int> ready;
-  for (int v = 0; v < n; v++) if (indeg[v] == 0) ready.push_back(v);
-  std::make_heap(ready.begin(), ready.end(), by_id);
-  while (!ready.empty()) {
-    std::pop_heap(ready.begin(), ready.end(), by_id);
-    int v = ready.back();
-    ready.pop_back();
-    order.push_back(v);
-    for (int s : succ[v])
-      if (--indeg[s] == 0) { ready.push_back(s); std::push_heap(ready.begin(), ready.end(), by_id); }
+  for (int v = 0; v < n; v++)
+    if (S.indeg[v] == 0) S.ready.push_back(v);
+  std::make_heap(S.ready.begin(), S.ready.end(), by_id);
+  while (!S.ready.empty()) {
+    std::pop_heap(S.ready.begin(), S.ready.end(), by_id);
+    const int v = S.ready.back();
+    S.ready.pop_back();
+    S.order.push_back(v);
+    for (int k = S.succ_beg[v]; k < S.succ_beg[v + 1]; k++)
+      if (--S.indeg[S.succ[k]] == 0) {
+        S.ready.push_back(S.succ[k]);
+        std::push_heap(S.ready.begin(), S.ready.end(), by_id);
+      }
   }
-  if (int(order.size()) != n) return EMR_ERR_CYCLE;
+  if (int(S.order.size()) != n) return EMR_ERR_CYCLE;
   // Keep the non-input nodes from which the output is reachable.
-  std::vector<char> reach(n, 0);
-  std::vector<int> stack{out_node};
-  reach[out_node] = 1;
-  while (!stack.empty()) {
-    int v = stack.back();
-    stack.pop_back();
-    for (int p : pred[v]) if (!reach[p]) { reach[p] = 1; stack.push_back(p); }
+  S.reach.assign(n, 0);
+  S.stack.assign(1, out_node);
+  S.reach[out_node] = 1;
+  while (!S.stack.empty()) {
+    const int v = S.stack.back();
+    S.stack.pop_back();
+    for (int k = S.pred_beg[v]; k < S.pred_beg[v + 1]; k++)
+      if (!S.reach[S.pred[k]]) { S.reach[S.pred[k]] = 1; S.stack.push_back(S.pred[k]); }
   }
-  std::vector<int> slot(n, -1), kept;
-  for (int v : order)
-    if (reach[v] && node_kind[n0 + v] >= EMR_KIND_HIDDEN) { slot[v] = int(kept.size()); kept.push_back(v); }
-  if (kept.empty() || kept.back() != out_node) return EMR_ERR_ARG;  // output must be last
-  if (kept.size() > 65535) return EMR_ERR_RANGE;
-  const int nk = int(kept.size());
+  S.slot.assign(n, -1);
+  S.kept.clear();
+  for (int v : S.order)
+    if (S.reach[v] && node_kind[n0 + v] >= EMR_KIND_HIDDEN) { S.slot[v] = int(S.kept.size()); S.kept.push_back(v); }
+  if (S.kept.empty() || S.kept.back() != out_node) return EMR_ERR_ARG;  // output must be last
+  if (S.kept.size() > 65535) return EMR_ERR_RANGE;
+  const int nk = int(S.kept.size());
   out->nodes.assign(nk, PackNode{});
-  std::vector<std::vector<PackEdge>> in_edges(nk);
-  std::vector<unsigned> has_in(nk, 0);  // bit k: has an enabled in-connection from input kind k
+  S.has_in.assign(nk, 0);  // bit k: has an enabled in-connection from input kind k
+  S.in_cnt.assign(nk, 0);
   for (int t = 0; t < nk; t++) {
-    int v = kept[t];
-    PackNode& pn = out->nodes[t];
-    pn.act = uint8_t(node_act[n0 + v]);
-    pn.bias = node_bias[n0 + v];
+    const int v = S.kept[t];
+    out->nodes[t].act = uint8_t(node_act[n0 + v]);
+    out->nodes[t].bias = node_bias[n0 + v];
   }
-  for (auto& e : es) {
-    int t = slot[e.d];
+  for (auto& e : S.es) {
+    const int t = S.slot[e.d];
     if (t < 0) continue;
-    int sk = node_kind[n0 + e.s];
+    const int sk = node_kind[n0 + e.s];
     if (sk < EMR_KIND_HIDDEN) {
       out->nodes[t].w_in[sk] += e.w;
-      has_in[t] |= 1u << sk;
+      S.has_in[t] |= 1u << sk;
     } else {
-      if (slot[e.s] < 0) return EMR_ERR_ARG;  // cannot happen: a source of a kept node is kept
-      in_edges[t].push_back(PackEdge{uint16_t(slot[e.s]), 0, e.w});
+      if (S.slot[e.s] < 0) return EMR_ERR_ARG;  // cannot happen: a source of a kept node is kept
+      S.in_cnt[t]++;
     }
   }
+  // in-edges from kept non-input nodes, grouped by destination in connection order
+  S.in_beg.assign(nk + 1, 0);
+  for (int t = 0; t < nk; t++) S.in_beg[t + 1] = S.in_beg[t] + S.in_cnt[t];
+  if (S.in_beg[nk] > 65535) return EMR_ERR_RANGE;
+  out->edges.resize(size_t(S.in_beg[nk]));
+  S.fill.assign(nk, 0);
+  for (auto& e : S.es) {
+    const int t = S.slot[e.d];
+    if (t < 0 || node_kind[n0 + e.s] < EMR_KIND_HIDDEN) continue;
+    out->edges[S.in_beg[t] + S.fill[t]++] = PackEdge{uint16_t(S.slot[e.s]), 0, e.w};
+  }
   PackGenome& g = out->g;
+  g = PackGenome{};
   g.n_nodes = uint16_t(nk);
   for (int t = 0; t < nk; t++) {
-    if (out->edges.size() + in_edges[t].size() > 65535) return EMR_ERR_RANGE;
-    out->nodes[t].edge_beg = uint16_t(out->edges.size());
-    out->nodes[t].edge_cnt = uint16_t(in_edges[t].size());
-    out->edges.insert(out->edges.end(), in_edges[t].begin(), in_edges[t].end());
+    out->nodes[t].edge_beg = uint16_t(S.in_beg[t]);
+    out->nodes[t].edge_cnt = uint16_t(S.in_cnt[t]);
   }
   g.n_edges = uint16_t(out->edges.size());
   for (int side = 0; side < 2; side++) {
@@ -132,10 +188,10 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
     int nv = 0, nve = 0;
     uint32_t cost = 0;
     for (int t = 0; t < nk; t++) {
-      bool vary = (has_in[t] & grid_inputs) != 0;
+      bool vary = (S.has_in[t] & grid_inputs) != 0;
       int vin = 0;
-      for (auto& e : in_edges[t])
-        if (out->nodes[e.src].vary & (1u << side)) { vary = true; vin++; }
+      for (int k = S.in_beg[t]; k < S.in_beg[t + 1]; k++)
+        if (out->nodes[out->edges[k].src].vary & (1u << side)) { vary = true; vin++; }
       if (vary) {
         out->nodes[t].vary |= uint8_t(1u << side);
         nv++;
@@ -208,18 +264,39 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
   const bool has_conns = conn_ptr[P] > conn_ptr[0];
   if (has_conns && (!conn_src || !conn_dst || !conn_w || !conn_enabled)) return EMR_ERR_ARG;
   std::vector<GenomeOut> gs(P);
-  for (int g = 0; g < P; g++) {
-    if (node_ptr[g + 1] < node_ptr[g] || conn_ptr[g + 1] < conn_ptr[g]) {
-      if (bad_genome) *bad_genome = g;
-      return EMR_ERR_ARG;
+  // Genomes are independent: pack them on several host threads, each with its
+  // own scratch; the lowest failing genome index is reported.
+  const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
+  const int n_threads = P >= 256 ? std::min(hw, 16) : 1;
+  std::vector<emr_status> t_rc(n_threads, EMR_OK);
+  std::vector<int32_t> t_bad(n_threads, -1);
+  auto work = [&](int t) {
+    Scratch scratch;
+    for (int g = int(int64_t(P) * t / n_threads); g < int(int64_t(P) * (t + 1) / n_threads); g++) {
+      emr_status rc = EMR_OK;
+      if (node_ptr[g + 1] < node_ptr[g] || conn_ptr[g + 1] < conn_ptr[g]) rc = EMR_ERR_ARG;
+      if (rc == EMR_OK)
+        rc = pack_one(node_ptr[g], node_ptr[g + 1], conn_ptr[g], conn_ptr[g + 1], node_id, node_kind, node_act,
+                      node_bias, conn_src, conn_dst, conn_w, conn_enabled, scratch, &gs[g]);
+      if (rc != EMR_OK) {
+        t_rc[t] = rc;
+        t_bad[t] = g;
+        return;
+      }
     }
-    emr_status rc = pack_one(node_ptr[g], node_ptr[g + 1], conn_ptr[g], conn_ptr[g + 1], node_id, node_kind,
-                             node_act, node_bias, conn_src, conn_dst, conn_w, conn_enabled, &gs[g]);
-    if (rc != EMR_OK) {
-      if (bad_genome) *bad_genome = g;
-      return rc;
-    }
+  };
+  if (n_threads == 1) {
+    work(0);
+  } else {
+    std::vector<std::thread> pool;
+    for (int t = 0; t < n_threads; t++) pool.emplace_back(work, t);
+    for (auto& th : pool) th.join();
   }
+  for (int t = 0; t < n_threads; t++)
+    if (t_rc[t] != EMR_OK) {
+      if (bad_genome) *bad_genome = t_bad[t];
+      return t_rc[t];
+    }
   size_t nn = 0, ne = 0;
   for (auto& g : gs) { nn += g.nodes.size(); ne += g.edges.size(); }
   PackHeader h{};

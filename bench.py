@@ -75,14 +75,37 @@ def barrier(ws):
         dist.barrier()
 
 
-def allreduce_max(x, ws):
+def allreduce(x, ws, op="max"):
+    """All-reduce a float over the ranks (max or sum); works on the nccl and gloo backends."""
     if ws == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.SUM)
     return float(t.item())
+
+
+def allreduce_max(x, ws):
+    return allreduce(x, ws, "max")
+
+
+def rank_workload(W, rank, depth, pop):
+    """Each rank runs its own population (independent problems, no data exchange): rank 0 the
+    paper-shaped seed, rank r > 0 an equally drawn population from a rank-specific seed."""
+    w = W.c2(D=depth, P=pop)
+    if rank > 0:
+        w.pop = W.random_population(pop, seed=2 + 7919 * rank)
+        w.name = w.name + "_rank%d" % rank
+    return w
+
+
+def aggregate(local_queries, local_ms, ws):
+    """Whole-job throughput: queries of all ranks over the slowest rank's time per step."""
+    total = allreduce(float(local_queries), ws, "sum")
+    ms = allreduce(float(local_ms), ws, "max")
+    return total, ms, total / (ms / 1e3)
 
 
 class ClockSampler:
@@ -278,9 +301,7 @@ def main():
     from paper_2608_27612_gb300 import workloads as W
 
     # Each rank runs its own population (independent problems, no collective on the data path).
-    w = W.c2(D=args.depth, P=args.pop)
-    if rank > 0:
-        w.pop = W.random_population(args.pop, seed=2 + 7919 * rank)
+    w = rank_workload(W, rank, args.depth, args.pop)
     dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, emr.EMR_EAGER)
     g = dsc.grid
     queries = dsc.n_pairs * g.n_total
@@ -324,8 +345,7 @@ def main():
     clocks = sampler.stop()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     tile_ms = [a.elapsed_time(b) for a, b in tiles]
-    ms = allreduce_max(statistics.mean(step_ms), ws)
-    value = ws * queries / (ms / 1e3)
+    _, ms, value = aggregate(queries, statistics.mean(step_ms), ws)
 
     # roofline of the dominant kernel (fused eval + variance + band)
     work = algorithmic_work(dsc.pack, dsc.query, emr)   # [P, S, (fp32, mufu)] per query
@@ -384,9 +404,9 @@ def main():
                 times.append(time.perf_counter() - t0)
                 h2d = len(blob) + 4 * (a_h.numel() + b_h.numel() + s_h.numel())
                 d2h = 8 * (dsc.n_pairs + 1) + 8 * n
-        e2e_s = allreduce_max(statistics.mean(times), ws)
-        e2e = {"value": ws * queries / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-               "ms_per_step": e2e_s * 1e3}
+        _, e2e_ms, e2e_value = aggregate(queries, statistics.mean(times) * 1e3, ws)
+        e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": e2e_ms}
 
     extra = None
     if rank == 0 and ws == 1 and not args.no_extra:

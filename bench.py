@@ -162,7 +162,9 @@ def algorithmic_work(pack, query, emr):
     """Per pair: fp32 lane ops and MUFU ops per query on the packed DAG (dead
     nodes removed, constants folded): per varying node its grid-input FMAs,
     its in-edges from varying nodes and its activation; plus the amortised
-    4-child variance and the band test."""
+    4-child variance and the band test. A pair whose output is constant over
+    the grid (no varying node) has variance and band value 0 everywhere and
+    counts no work."""
     h, gs, nodes, edges = emr.pack_records(pack)
     per = np.zeros((len(gs), 2, 2))
     for g in range(len(gs)):
@@ -180,7 +182,8 @@ def algorithmic_work(pack, query, emr):
                     F += (int(nodes[nb + src]["vary"]) >> side) & 1
                 F += ACT_FP32[int(nd["act"])]
                 M += ACT_MUFU[int(nd["act"])]
-            per[g, side] = (F + VAR_OPS + BAND_OPS, M)
+            # a pair whose output does not vary over the grid needs no per-position arithmetic
+            per[g, side] = (F + VAR_OPS + BAND_OPS, M) if F > 0 or M > 0 else (0.0, 0.0)
     side = np.broadcast_to(query.side, (len(gs), query.S))
     return per[np.arange(len(gs))[:, None], side]  # [P, S, 2]
 

@@ -248,6 +248,20 @@ def streamed_run(emr, torch, w, chunk, chunk_cap, cap, reps):
             "timing": "host wall clock per emr_stream call (synchronous, lists on the host), median of %d" % reps}
 
 
+def launches_in_step(emr, dsc):
+    """Kernel launches of one step: prepare (schedule, records), one tile launch per
+    non-empty kernel class, mask combine, compaction (count, two scans, write, kept
+    weights); combine, count and write launch once per 65535 pairs."""
+    _, gs, _, _ = emr.pack_records(dsc.pack)
+    side = np.asarray(dsc.query.side)
+    nv = gs["n_varying"][:, side] if not dsc.query.per_genome else \
+        np.take_along_axis(gs["n_varying"], side.reshape(gs.shape[0], -1), axis=1)
+    nv = nv.astype(np.int64)
+    cls = np.where(nv > 12, 0, np.where(nv > 8, 1, np.where(nv > 4, 2, 3)))
+    groups = -(-dsc.n_pairs // 65535)
+    return 2 + len(np.unique(cls)) + groups + 2 * groups + 3
+
+
 def oracle_baseline(w, genomes):
     import oracle
     oracle.build()
@@ -317,14 +331,15 @@ def main():
         dsc.prepare()
         if evs:
             evs[0].record(stream)
-        emr.eval_filter(dsc.pack, dsc.query, g, dsc.theta, dsc.band, dsc.w_min, dsc.split, dsc.band_bits, dsc.out,
+        emr.eval_filter(dsc.pack, dsc.query, g, dsc.theta, dsc.band, dsc.w_min, dsc.split, dsc.band_bits, None,
                         dsc.ws)
         if evs:
             evs[1].record(stream)
         emr.mask_combine(dsc.split, dsc.band_bits, g, dsc.n_pairs, dsc.mode, dsc.mask)
-        emr.compact(dsc.mask, dsc.out, g, dsc.n_pairs, dsc.idx, dsc.w, dsc.cap, dsc.counts, dsc.offsets, dsc.cws)
+        emr.compact_records(dsc.mask, dsc.pack, dsc.query, dsc.ws, g, dsc.idx, dsc.w, dsc.cap, dsc.counts,
+                            dsc.offsets, dsc.cws)
 
-    launches_per_step = 2 + 1 + 1 + 4
+    launches_per_step = launches_in_step(emr, dsc)
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()

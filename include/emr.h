@@ -225,8 +225,8 @@ emr_status emr_eval_filter(const void *pack_host, const emr_query *q, const emr_
 
 /* Bytes of device workspace emr_stream needs: the per-pair records, the
  * resident split plane (n_pairs x n_words x 4 bytes) and two chunk buffers
- * (band bits, mask, sparse outputs of chunk positions, compaction workspace
- * and chunk_cap list entries each). */
+ * (band bits, mask, compaction workspace and chunk_cap list entries each; the
+ * kept weights are recomputed from the records, so no outputs are stored). */
 emr_status emr_stream_workspace_size(const void *pack_host, const emr_query *q, const emr_grid *grid,
                                      int64_t chunk_cap, size_t *bytes);
 
@@ -309,6 +309,17 @@ emr_status emr_compact_workspace_size(const emr_grid *grid, int32_t n_pairs, siz
 emr_status emr_compact(const uint32_t *mask, const float *out, const emr_grid *grid, int32_t n_pairs,
                        int32_t *idx, float *w, int64_t cap, int64_t *counts, int64_t *offsets, void *ws,
                        size_t ws_bytes, void *stream);
+
+/* Same as emr_compact, but the CPPN outputs at the kept positions are
+ * recomputed from the per-pair records in eval_ws (prepared by
+ * emr_eval_prepare for this pack and query) with the tile kernels' own
+ * arithmetic, so the fused path needs no output buffer: the weights equal those
+ * emr_eval would have written. mask as from emr_mask_combine; the number of
+ * pairs comes from the pack and query. Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY
+ * (eval_ws or ws too small), EMR_ERR_CUDA. */
+emr_status emr_compact_records(const uint32_t *mask, const void *pack_host, const emr_query *q, const void *eval_ws,
+                               size_t eval_ws_bytes, const emr_grid *grid, int32_t *idx, float *w, int64_t cap,
+                               int64_t *counts, int64_t *offsets, void *ws, size_t ws_bytes, void *stream);
 
 /* ---- misc -------------------------------------------------------------------- */
 

@@ -656,6 +656,8 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     const float X0 = grid_coord(i0 + 2 * pl, scale), Y0 = grid_coord(j0 + 2 * ql, scale);
     const float step = 2.f * scale, quad_step = 4.f * scale;  // one column; one quad (two columns)
     const int sbase = (2 * ql + kPad) * P64 + 2 * pl + kPad;
+    uint32_t* split_k = split_row + A.word_off[d - 1] + mb / 128 + warp;  // this warp's parents, k = 0
+    uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
     // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the nodes
     constexpr int QPE = NVMAX <= 4 ? 2 : 1;
 #pragma unroll 1
@@ -681,7 +683,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
           *reinterpret_cast<float2*>(t + P64) = make_float2(wq[2], wq[3]);
           // the four children give the parent's variance (Section 3.2)
           const unsigned bal = __ballot_sync(kFull, var_sum4(wq[0], wq[1], wq[2], wq[3]) > theta4);
-          if (lane == 0) split_row[A.word_off[d - 1] + mb / 128 + (TPB / 32) * k + warp] = bal;
+          if (lane == 0) split_k[(TPB / 32) * k] = bal;
         } else {
           *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
               make_float4(wq[0], wq[1], wq[2], wq[3]);
@@ -741,15 +743,15 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
       const float DB[4] = {sqdiff(w[0], Bo[0]), sqdiff(w[1], Bo[1]), v02, v13};
       const float DT[4] = {v02, v13, sqdiff(w[2], U[2]), sqdiff(w[3], U[3])};
 #pragma unroll
-      for (int c = 0; c < 4; c++) {
-        pass[c] = band_pass_sq(DL[c], DR[c], DB[c], DT[c], band2);
-        if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+      for (int c = 0; c < 4; c++) pass[c] = band_pass_sq(DL[c], DR[c], DB[c], DT[c], band2);
+      if (wfilter) {
+#pragma unroll
+        for (int c = 0; c < 4; c++) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
       }
       const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
       const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-      if (lane < 4)  // quad-major words of this warp's 32 quads
-        A.bandb[band_base + A.word_off[d] + 4 * (mb / 128 + (TPB / 32) * k + warp) + lane] =
-            lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+      if (lane == 0)  // the four quad-major words of this warp's 32 quads
+        *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(b0, b1, b2, b3);
       if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
         float* o = A.out + lrow + mb + 4 * (tid + TPB * k);
 #pragma unroll
@@ -1112,11 +1114,49 @@ __global__ void compact_scan_pairs_kernel(const int64_t* __restrict__ counts, in
   if (threadIdx.x == 0) offsets[n_pairs] = carry;
 }
 
-// out: output at global index p of pair r is out[r * out_stride + p - out_shift].
+// CPPN output of one grid point from a pair's record, with the arithmetic of the
+// tile kernels operation for operation (the dense evaluator for up to kDenseMax
+// varying nodes, else the edge list in node order), so the value equals the one
+// the tile kernels computed at that position. Interpreted node values go to a
+// local array: records with more than kDenseMax varying nodes are rare.
+__device__ float eval_record_point(const uint8_t* rec, const SpecLayout& L, float x, float y) {
+  const int nv = reinterpret_cast<const int32_t*>(rec)[0];
+  const float out_const = reinterpret_cast<const float*>(rec)[2];
+  const float4* coef = reinterpret_cast<const float4*>(rec + L.coef_off());
+  if (nv <= kDenseMax) {
+    const float xs[1] = {x}, ys[1] = {y};
+    float w[1];
+    eval_dense<kDenseMax, 1>(coef, reinterpret_cast<const float*>(rec + L.dense_off()), nv, out_const, xs, ys, w);
+    return w[0];
+  }
+  const uint2* ve = reinterpret_cast<const uint2*>(rec + L.edge_off());
+  float v[EMR_MAX_VARYING];
+  float z = out_const;
+  for (int k = 0; k < nv; k++) {
+    const float4 c = coef[k];
+    const uint32_t info = __float_as_uint(c.w);
+    z = fmaf(c.z, y, fmaf(c.y, x, c.x));
+    const int eb = int((info >> 8) & 0xfffu), ee = eb + int(info >> 20);
+    for (int e = eb; e < ee; e++) z = fmaf(__uint_as_float(ve[e].y), v[ve[e].x], z);
+    z = act_apply(int(info & 0xffu), z);
+    v[k] = z;
+  }
+  return z;
+}
+
+// Per-pair records (pair r at spec + r * L.stride) from which the kept weights
+// are recomputed instead of read from materialised outputs.
+struct RecordSource {
+  const uint8_t* spec;
+  SpecLayout L;
+};
+
+// when out is NULL and rs.spec is set, the weights are recomputed from the records.
 __global__ void compact_write_kernel(PlaneView mask, const float* __restrict__ out, int64_t out_stride,
-                                     int64_t out_shift, GridDev G, int64_t w0, int64_t nw, int nb, int64_t r0,
-                                     const int32_t* __restrict__ boff, const int64_t* __restrict__ offsets, int64_t cap,
-                                     int32_t* __restrict__ idx, float* __restrict__ wv) {
+                                     int64_t out_shift, GridDev G, int64_t w0, int64_t nw, int nb,
+                                     int64_t r0, const int32_t* __restrict__ boff,
+                                     const int64_t* __restrict__ offsets, int64_t cap, int32_t* __restrict__ idx,
+                                     float* __restrict__ wv) {
   __shared__ int sh[32];
   const int64_t r = r0 + blockIdx.y;
   const int64_t k = (int64_t(blockIdx.x) * kCompactBlock + threadIdx.x) * 4;
@@ -1134,9 +1174,35 @@ __global__ void compact_write_kernel(PlaneView mask, const float* __restrict__ o
       const int64_t gidx = gbase + __ffs(v) - 1;
       if (dst < cap) {
         idx[dst] = int32_t(gidx);
-        if (wv) wv[dst] = out[r * out_stride + gidx - out_shift];
+        if (out && wv) wv[dst] = out[r * out_stride + gidx - out_shift];
       }
     }
+  }
+}
+
+// Weights of the listed kept positions, recomputed from the records: one entry
+// per thread (kept positions cluster, so a thread per mask word would evaluate
+// long runs serially). The entry's pair is the last r with offsets[r] <= t.
+__global__ void __launch_bounds__(kCompactBlock) kept_weights_kernel(RecordSource rs, GridDev G,
+                                                                     const int64_t* __restrict__ offsets,
+                                                                     int64_t n_pairs, int64_t cap,
+                                                                     const int32_t* __restrict__ idx,
+                                                                     float* __restrict__ wv) {
+  const int64_t total = offsets[n_pairs] < cap ? offsets[n_pairs] : cap;
+  for (int64_t t = int64_t(blockIdx.x) * kCompactBlock + threadIdx.x; t < total;
+       t += int64_t(gridDim.x) * kCompactBlock) {
+    int64_t lo = 0, hi = n_pairs;  // offsets[lo] <= t < offsets[hi]
+    while (hi - lo > 1) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (offsets[mid] <= t) lo = mid; else hi = mid;
+    }
+    const int64_t gidx = idx[t];
+    int d = 0;
+    while (G.level_off[d + 1] <= gidx) d++;
+    const uint32_t m = uint32_t(gidx - G.level_off[d]);
+    const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1)
+    const float x = grid_coord(int(compact1by1(m)), scale), y = grid_coord(int(compact1by1(m >> 1)), scale);
+    wv[t] = eval_record_point(rs.spec + lo * rs.L.stride, rs.L, x, y);
   }
 }
 
@@ -1397,7 +1463,7 @@ size_t compact_ws_bytes(int64_t nw, int64_t n_pairs) {
 // Ordered compaction of words [w0, w0 + nw) of every pair.
 emr_status launch_compact(PlaneView mask, const float* out, int64_t out_stride, int64_t out_shift, const emr_grid* g,
                           int64_t n_pairs, int64_t w0, int64_t nw, int32_t* idx, float* w, int64_t cap, int64_t* counts,
-                          int64_t* offsets, void* ws, cudaStream_t st) {
+                          int64_t* offsets, void* ws, cudaStream_t st, RecordSource rs = RecordSource{nullptr, {}}) {
   const int nb = int((nw + kCompactWords - 1) / kCompactWords);
   const int64_t nblk = int64_t(nb) * n_pairs;
   if (n_pairs <= 0 || n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
@@ -1414,6 +1480,13 @@ emr_status launch_compact(PlaneView mask, const float* out, int64_t out_stride, 
     const dim3 grid(unsigned(nb), unsigned(std::min<int64_t>(65535, n_pairs - r0)));
     compact_write_kernel<<<grid, kCompactBlock, 0, st>>>(mask, out, out_stride, out_shift, G, w0, nw, nb, r0, boff,
                                                          offsets, cap, idx, w);
+  }
+  if (w && !out && rs.spec && cap > 0) {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+        cudaSuccess)
+      return EMR_ERR_CUDA;
+    kept_weights_kernel<<<unsigned(8 * sms), kCompactBlock, 0, st>>>(rs, G, offsets, n_pairs, cap, idx, w);
   }
   return cuda_status(cudaGetLastError());
 }
@@ -1504,6 +1577,20 @@ emr_status emr_compact_workspace_size(const emr_grid* grid, int32_t n_pairs, siz
   return EMR_OK;
 }
 
+emr_status emr_compact_records(const uint32_t* mask, const void* pack_host, const emr_query* q, const void* eval_ws,
+                               size_t eval_ws_bytes, const emr_grid* grid, int32_t* idx, float* w, int64_t cap,
+                               int64_t* counts, int64_t* offsets, void* ws, size_t ws_bytes, void* stream) {
+  if (!mask || !grid_ok(grid) || (!idx && cap > 0) || cap < 0 || !counts || !offsets || !ws || !eval_ws)
+    return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (eval_ws_bytes < p.total || ws_bytes < compact_ws_bytes(grid->n_words, p.n_pairs)) return EMR_ERR_CAPACITY;
+  return launch_compact(PlaneView{const_cast<uint32_t*>(mask), grid->n_words, 0}, nullptr, 0, 0, grid, p.n_pairs, 0,
+                        grid->n_words, idx, w, cap, counts, offsets, ws, static_cast<cudaStream_t>(stream),
+                        RecordSource{static_cast<const uint8_t*>(eval_ws), p.L});
+}
+
 emr_status emr_compact(const uint32_t* mask, const float* out, const emr_grid* grid, int32_t n_pairs, int32_t* idx,
                        float* w, int64_t cap, int64_t* counts, int64_t* offsets, void* ws, size_t ws_bytes,
                        void* stream) {
@@ -1584,9 +1671,9 @@ extern "C" emr_status emr_eval_filter_noalloc(const void* pack_host, const void*
 // their children at depth d + 1 in the same or an earlier chunk, so when a
 // chunk has been evaluated its own split bits are final and its keep mask and
 // compacted lists can be produced at once. Only the split plane is resident;
-// band bits, masks, sparse outputs and lists are per chunk, double-buffered,
-// and the lists are copied to the caller's host arrays on a second stream
-// while the next chunk computes.
+// band bits, masks and lists are per chunk, double-buffered (kept weights are
+// recomputed from the per-pair records), and the lists are copied to the
+// caller's host arrays on a second stream while the next chunk computes.
 
 #include <chrono>
 #include <thread>
@@ -1598,7 +1685,7 @@ struct StreamPlan {
   std::vector<std::pair<int32_t, int32_t>> chunks;  // tile ranges, processing order
   int64_t wpc, ppc;                                 // words / positions per chunk buffer row
   int64_t n_pairs, chunk_cap;
-  size_t off_split, off_band[2], off_mask[2], off_out[2], off_cws[2], off_idx[2], off_w[2], off_cnt[2], off_off[2];
+  size_t off_split, off_band[2], off_mask[2], off_cws[2], off_idx[2], off_w[2], off_cnt[2], off_off[2];
   size_t cws_bytes, total;
 };
 
@@ -1643,7 +1730,6 @@ emr_status stream_plan(const void* pack_host, const emr_query* q, const emr_grid
   for (int b = 0; b < 2; b++) {
     sp->off_band[b] = o; o += up(size_t(sp->n_pairs) * size_t(sp->wpc) * 4);
     sp->off_mask[b] = o; o += up(size_t(sp->n_pairs) * size_t(sp->wpc) * 4);
-    sp->off_out[b] = o; o += up(size_t(sp->n_pairs) * size_t(sp->ppc) * 4);
     sp->off_cws[b] = o; o += up(sp->cws_bytes);
     sp->off_idx[b] = o; o += up(size_t(chunk_cap) * 4);
     sp->off_w[b] = o; o += up(size_t(chunk_cap) * 4);
@@ -1749,7 +1835,6 @@ extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, co
     if (k >= 2 && cudaStreamWaitEvent(st, ev_copied[b], 0) != cudaSuccess) { rc = EMR_ERR_CUDA; break; }
     uint32_t* bandc = reinterpret_cast<uint32_t*>(base + sp.off_band[b]);
     uint32_t* maskc = reinterpret_cast<uint32_t*>(base + sp.off_mask[b]);
-    float* outc = reinterpret_cast<float*>(base + sp.off_out[b]);
     TileRange tr;
     tr.beg = t_lo;
     tr.end = t_hi;
@@ -1757,17 +1842,18 @@ extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, co
     tr.band_shift = w_lo;
     tr.out_stride = sp.ppc;
     tr.out_shift = p_lo;
-    if ((rc = launch_tiles(sp.ev, grid, spec, order, kModeFused, theta, band, w_min, outc, nullptr, split, bandc, st,
-                           tr)) != EMR_OK)
+    if ((rc = launch_tiles(sp.ev, grid, spec, order, kModeFused, theta, band, w_min, nullptr, nullptr, split, bandc,
+                           st, tr)) != EMR_OK)
       break;
     if ((rc = launch_combine(split, PlaneView{bandc, sp.wpc, w_lo}, PlaneView{maskc, sp.wpc, w_lo}, grid, NP, w_lo,
                              w_hi - w_lo, 0, st)) != EMR_OK)
       break;
-    if ((rc = launch_compact(PlaneView{maskc, sp.wpc, w_lo}, outc, sp.ppc, p_lo, grid, NP, w_lo, w_hi - w_lo,
+    if ((rc = launch_compact(PlaneView{maskc, sp.wpc, w_lo}, nullptr, 0, 0, grid, NP, w_lo, w_hi - w_lo,
                              reinterpret_cast<int32_t*>(base + sp.off_idx[b]),
                              reinterpret_cast<float*>(base + sp.off_w[b]), sp.chunk_cap,
                              reinterpret_cast<int64_t*>(base + sp.off_cnt[b]),
-                             reinterpret_cast<int64_t*>(base + sp.off_off[b]), base + sp.off_cws[b], st)) != EMR_OK)
+                             reinterpret_cast<int64_t*>(base + sp.off_off[b]), base + sp.off_cws[b], st,
+                             RecordSource{spec, sp.ev.L})) != EMR_OK)
       break;
     if (cudaMemcpyAsync(staging + b * (NP + 1), base + sp.off_off[b], size_t(NP + 1) * 8, cudaMemcpyDeviceToHost,
                         st) != cudaSuccess ||

@@ -69,6 +69,7 @@ def lib() -> C.CDLL:
             "emr_stream": [vp, vp, vp, vp, f32, f32, f32, vp, sz, i64, vp, vp, i64, vp, vp, i64, vp],
             "emr_compact_workspace_size": [vp, i32, vp],
             "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
+            "emr_compact_records": [vp, vp, vp, vp, sz, vp, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_version": [],
             "emr_probe_alu": [i32, i32, i32, vp, vp, vp, vp],
         }
@@ -259,6 +260,16 @@ def compact(mask, out, grid: Grid, n_pairs: int, idx, w, cap: int, counts, offse
                              _ptr(offsets), _ptr(ws), C.c_size_t(ws.numel()), _stream(stream)), "emr_compact")
 
 
+def compact_records(mask, pack, query: Query, eval_ws, grid: Grid, idx, w, cap: int, counts, offsets, ws,
+                    stream=None):
+    """emr_compact_records: lists with the kept weights recomputed from the prepared records."""
+    q = query.c
+    _check(lib().emr_compact_records(_ptr(mask), _ptr(pack), C.byref(q), _ptr(eval_ws),
+                                     C.c_size_t(eval_ws.numel()), C.byref(grid), _ptr(idx), _ptr(w), cap,
+                                     _ptr(counts), _ptr(offsets), _ptr(ws), C.c_size_t(ws.numel()),
+                                     _stream(stream)), "emr_compact_records")
+
+
 # ---- ALU probes (roofline denominators) -------------------------------------------------
 
 PROBE_FFMA, PROBE_EX2, PROBE_RCP, PROBE_SIN = range(4)
@@ -278,7 +289,8 @@ def probe_alu(op: int, blocks: int, iters: int, stream=None):
 class Discovery:
     """Buffers and calls for one (population, query, depth) configuration.
 
-    run_fused(): CPPN outputs never materialised (only kept-candidate weights are written).
+    run_fused(): CPPN outputs never materialised; the kept weights are recomputed at compaction
+    (or, with sparse_out=True, written by the fused kernel where the band test passed).
     run_unfused(): CPPN outputs materialised, then filtered.
     """
 
@@ -297,7 +309,8 @@ class Discovery:
         self.mask = torch.zeros(self.n_pairs, g.n_words, **u32)
         self.split = torch.zeros(self.n_pairs, g.n_words, **u32)
         self.band_bits = torch.zeros(self.n_pairs, g.n_words, **u32)
-        self.out = torch.zeros(self.n_pairs, g.n_total, dtype=torch.float32, device=self.device)
+        self.out = (torch.zeros(self.n_pairs, g.n_total, dtype=torch.float32, device=self.device)
+                    if materialise else None)
         self.out_halo = (torch.zeros(self.n_pairs, g.n_halo, dtype=torch.float32, device=self.device)
                          if materialise else None)
         self.var_dbg = None
@@ -312,19 +325,31 @@ class Discovery:
     def prepare(self, stream=None):
         eval_prepare(self.pack, self.pack_dev, self.query, self.ws, stream)
 
-    def run_fused(self, stream=None):
-        """emr_eval_prepare, emr_eval_filter, emr_mask_combine, emr_compact."""
+    def _materialise(self):
+        if self.out is None:
+            self.out = torch.zeros(self.n_pairs, self.grid.n_total, dtype=torch.float32, device=self.device)
+        if self.out_halo is None:
+            self.out_halo = torch.zeros(self.n_pairs, self.grid.n_halo, dtype=torch.float32, device=self.device)
+
+    def run_fused(self, sparse_out: bool = False, stream=None):
+        """emr_eval_prepare, emr_eval_filter, emr_mask_combine, emr_compact_records
+        (sparse_out: emr_eval_filter writes band-passing outputs, emr_compact reads them)."""
         self.prepare(stream)
+        if sparse_out:
+            self._materialise()
         eval_filter(self.pack, self.query, self.grid, self.theta, self.band, self.w_min, self.split,
-                    self.band_bits, self.out, self.ws, stream)
+                    self.band_bits, self.out if sparse_out else None, self.ws, stream)
         mask_combine(self.split, self.band_bits, self.grid, self.n_pairs, self.mode, self.mask, stream)
-        compact(self.mask, self.out, self.grid, self.n_pairs, self.idx, self.w, self.cap, self.counts,
-                self.offsets, self.cws, stream)
+        if sparse_out:
+            compact(self.mask, self.out, self.grid, self.n_pairs, self.idx, self.w, self.cap, self.counts,
+                    self.offsets, self.cws, stream)
+        else:
+            compact_records(self.mask, self.pack, self.query, self.ws, self.grid, self.idx, self.w, self.cap,
+                            self.counts, self.offsets, self.cws, stream)
 
     def run_unfused(self, with_var: bool = False, stream=None):
         """emr_eval_prepare, emr_eval, emr_variance_filter, emr_compact."""
-        if self.out_halo is None:
-            self.out_halo = torch.zeros(self.n_pairs, self.grid.n_halo, dtype=torch.float32, device=self.device)
+        self._materialise()
         if with_var and self.var_dbg is None:
             self.var_dbg = torch.zeros(self.n_pairs, self.grid.n_total, dtype=torch.float32, device=self.device)
         self.prepare(stream)

@@ -33,7 +33,6 @@ def run_gpu(w, mode=emr.EMR_EAGER, unfused=True, fused=True, cap=None, lists=Tru
         res["band_u"] = dsc.band_bits.cpu().numpy()
         res["lists_u"] = dsc.lists()
     if fused:
-        dsc.out.zero_()
         dsc.mask.zero_(); dsc.split.zero_(); dsc.band_bits.zero_()
         dsc.run_fused()
         torch.cuda.synchronize()
@@ -41,7 +40,11 @@ def run_gpu(w, mode=emr.EMR_EAGER, unfused=True, fused=True, cap=None, lists=Tru
         res["split_f"] = dsc.split.cpu().numpy()
         res["band_f"] = dsc.band_bits.cpu().numpy()
         res["lists_f"] = dsc.lists() if lists else None
-        res["out_f"] = dsc.out.cpu().numpy()
+        if unfused and lists:
+            # the fused kernel's own sparse outputs, read by emr_compact
+            dsc.out.zero_()
+            dsc.run_fused(sparse_out=True)
+            res["lists_s"] = dsc.lists()
     return res
 
 
@@ -68,9 +71,12 @@ def full_parity(w, mode=emr.EMR_EAGER, n_oracle=None):
     assert np.array_equal(gpu["mask_u"], gpu["mask_f"])
     rep["kept"] = check_lists(gpu["lists_f"][:n], gpu["mask_f"][:n], ora["w"], ora["w_err"])
     check_lists(gpu["lists_u"][:n], gpu["mask_u"][:n], ora["w"], ora["w_err"])
-    # fused lists carry the same weights as the materialised outputs
-    for (i_u, w_u), (i_f, w_f) in zip(gpu["lists_u"], gpu["lists_f"]):
-        assert np.array_equal(i_u, i_f) and np.array_equal(w_u, w_f)
+    # weights recomputed from the records at compaction, and those the fused kernel
+    # stores itself, equal the materialised outputs bit for bit
+    for (i_u, w_u), (i_f, w_f), (i_s, w_s) in zip(gpu["lists_u"], gpu["lists_f"], gpu["lists_s"]):
+        assert np.array_equal(i_u, i_f) and np.array_equal(i_u, i_s)
+        assert np.array_equal(w_u.view(np.uint32), w_f.view(np.uint32))
+        assert np.array_equal(w_u.view(np.uint32), w_s.view(np.uint32))
     return gpu, ora, rep
 
 

@@ -660,6 +660,11 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
     // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the nodes
     constexpr int QPE = NVMAX <= 4 ? 2 : 1;
+    // bit k: some quad of this warp's k-th group may pass the band test. A position
+    // passes only if both differences along one axis exceed the band, and one of
+    // them is to its sibling in the quad; so a quad whose four sibling differences
+    // are all within the band has no passing position, whatever its neighbours.
+    uint32_t need = 0u;
 #pragma unroll 1
     for (int k0 = 0; k0 < QPT; k0 += QPE) {
       float x[4 * QPE], y[4 * QPE], w[4 * QPE];
@@ -684,11 +689,19 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
           // the four children give the parent's variance (Section 3.2)
           const unsigned bal = __ballot_sync(kFull, var_sum4(wq[0], wq[1], wq[2], wq[3]) > theta4);
           if (lane == 0) split_k[(TPB / 32) * k] = bal;
+          const bool near = sqdiff(wq[0], wq[1]) <= band2 && sqdiff(wq[2], wq[3]) <= band2 &&
+                            sqdiff(wq[0], wq[2]) <= band2 && sqdiff(wq[1], wq[3]) <= band2;
+          if (__any_sync(kFull, !near)) need |= 1u << k;
         } else {
           *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
               make_float4(wq[0], wq[1], wq[2], wq[3]);
         }
       }
+    }
+    if (fused && !__syncthreads_or(need != 0u)) {  // no position of the tile can pass
+      if (lane == 0)
+        for (int k = 0; k < QPT; k++) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
+      return;
     }
     // ring: 4 sides x 64 points, evaluated four at a time by threads 0..63
     // (point t = 4 tid + c lies on side t / 64, the same for all four)
@@ -726,6 +739,10 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     // band value of each position from its four neighbours at distance 2^-d
 #pragma unroll 2
     for (int k = 0; k < QPT; k++) {
+      if (!((need >> k) & 1u)) {  // warp-uniform
+        if (lane == 0) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
+        continue;
+      }
       const uint32_t kq = uint32_t(TPB * k);
       const float* t = s_wt + sbase + 2 * int(compact1by1(kq)) + 2 * int(compact1by1(kq >> 1)) * P64;  // (2pi, 2pj)
       const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);

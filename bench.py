@@ -36,7 +36,7 @@ UNIT = "queries/s"
 # Per-activation algorithmic cost per query (fp32 lane ops, MUFU ops).
 ACT_FP32 = {0: 0, 1: 2, 2: 3, 3: 2, 4: 4, 5: 0}
 ACT_MUFU = {0: 0, 1: 2, 2: 2, 3: 1, 4: 1, 5: 0}
-VAR_OPS, BAND_OPS = 3.25, 8.0
+VAR_OPS, BAND_OPS = 4.5, 1.0
 MUFU_PER_SM_CLK = 16          # nominal MUFU lanes per SM per clock
 FP32_PER_SM_CLK = 128         # FP32 lanes per SM per clock
 SM_MAX_MHZ = 2070.0
@@ -161,8 +161,11 @@ class ClockSampler:
 def algorithmic_work(pack, query, emr):
     """Per pair: fp32 lane ops and MUFU ops per query on the packed DAG (dead
     nodes removed, constants folded): per varying node its grid-input FMAs,
-    its in-edges from varying nodes and its activation; plus the amortised
-    4-child variance and the band test. A pair whose output is constant over
+    its in-edges from varying nodes and its activation; plus the filter at its
+    minimum: per parent the six squared pairwise child differences, their sum and
+    one compare (4.5 per query), and per quad the band screen's four compares on
+    the sibling differences (1 per query; the full band test of the few quads the
+    screen lets through is not counted). A pair whose output is constant over
     the grid (no varying node) has variance and band value 0 everywhere and
     counts no work."""
     h, gs, nodes, edges = emr.pack_records(pack)

@@ -111,14 +111,17 @@ __device__ __forceinline__ void act_apply4(int a, float& z0, float& z1, float& z
 //   band: with squared differences to the four neighbours, B > band is tested as
 //     max(min(dt^2, db^2), min(dl^2, dr^2)) > band^2 (squaring is monotone on
 //     |d|; it changes the fp32 decision only within one rounding of the band).
-__device__ __forceinline__ float var_sum4(float w0, float w1, float w2, float w3) {
-  const float m = 0.25f * ((w0 + w1) + (w2 + w3));
-  const float e0 = w0 - m, e1 = w1 - m, e2 = w2 - m, e3 = w3 - m;
-  return (e0 * e0 + e1 * e1) + (e2 * e2 + e3 * e3);
-}
 __device__ __forceinline__ float sqdiff(float a, float b) {
   const float t = a - b;
   return t * t;
+}
+// Sixteen times the population variance of four values, as the sum of their six
+// squared pairwise differences (sum over i < j of (w_i - w_j)^2 equals four times
+// the sum of squared deviations from the mean). The four sibling differences
+// (w0 w1, w2 w3 along x; w0 w2, w1 w3 along y) are the band test's as well.
+__device__ __forceinline__ float var16(float w0, float w1, float w2, float w3) {
+  return ((sqdiff(w0, w1) + sqdiff(w2, w3)) + (sqdiff(w0, w2) + sqdiff(w1, w3))) +
+         (sqdiff(w0, w3) + sqdiff(w1, w2));
 }
 __device__ __forceinline__ bool band_pass_sq(float dl2, float dr2, float db2, float dt2, float band2) {
   return fmaxf(fminf(dt2, db2), fminf(dl2, dr2)) > band2;
@@ -460,7 +463,7 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
     }
     // fused: the four children of parent q give its variance (Section 3.2)
     if (d >= 1) {
-      const unsigned bal = __ballot_sync(kFull, is_main && var_sum4(w[0], w[1], w[2], w[3]) > 4.f * A.theta);
+      const unsigned bal = __ballot_sync(kFull, is_main && var16(w[0], w[1], w[2], w[3]) > 16.f * A.theta);
       const int q0 = base + warp * 32;
       if (lane == 0 && q0 < nq)
         A.split[int64_t(r) * A.n_words + A.word_off[d - 1] + (mb / 4 + uint32_t(q0)) / 32] = bal;
@@ -615,7 +618,13 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
   __shared__ float4 s_coef[NVMAX];
   __shared__ __align__(16) float s_W[NVMAX * NVMAX];
   __shared__ __align__(16) float s_wt[P64 * P64];
+  // quad TPB k of a tile: its Morton coordinates (as floats) and its shared-tile offset
+  __shared__ int4 s_kq[QPT];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid < QPT) {
+    const int dx = int(compact1by1(uint32_t(TPB * tid))), dy = int(compact1by1(uint32_t(TPB * tid) >> 1));
+    s_kq[tid] = make_int4(__float_as_int(float(dx)), __float_as_int(float(dy)), 2 * dx + 2 * dy * P64, 0);
+  }
   const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
   const int tile = A.tile_beg + int(blockIdx.x % A.n_tiles);
   const int r = A.order[rank];
@@ -624,7 +633,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
   const float out_const = reinterpret_cast<const float*>(rec)[2];
   const bool fused = A.mode == kModeFused;
   const bool wfilter = A.w_min > 0.f;
-  const float theta4 = 4.f * A.theta, band2 = A.band * A.band;
+  const float theta16 = 16.f * A.theta, band2 = A.band * A.band;
   if (tid < NVMAX)
     s_coef[tid] = tid < nv ? reinterpret_cast<const float4*>(rec + A.L.coef_off())[tid] : make_float4(0, 0, 0, 0);
   {
@@ -668,11 +677,12 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
 #pragma unroll 1
     for (int k0 = 0; k0 < QPT; k0 += QPE) {
       float x[4 * QPE], y[4 * QPE], w[4 * QPE];
+      int4 kq[QPE];
 #pragma unroll
       for (int h = 0; h < QPE; h++) {
-        const uint32_t kq = uint32_t(TPB * (k0 + h));
-        const float xa = fmaf(float(compact1by1(kq)), quad_step, X0);
-        const float ya = fmaf(float(compact1by1(kq >> 1)), quad_step, Y0);
+        kq[h] = s_kq[k0 + h];
+        const float xa = fmaf(__int_as_float(kq[h].x), quad_step, X0);
+        const float ya = fmaf(__int_as_float(kq[h].y), quad_step, Y0);
         x[4 * h + 0] = xa; x[4 * h + 1] = xa + step; x[4 * h + 2] = xa; x[4 * h + 3] = xa + step;
         y[4 * h + 0] = ya; y[4 * h + 1] = ya; y[4 * h + 2] = ya + step; y[4 * h + 3] = ya + step;
       }
@@ -680,14 +690,13 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
 #pragma unroll
       for (int h = 0; h < QPE; h++) {
         const int k = k0 + h;
-        const uint32_t kq = uint32_t(TPB * k);
         const float* wq = w + 4 * h;
         if (fused) {
-          float* t = s_wt + sbase + 2 * int(compact1by1(kq)) + 2 * int(compact1by1(kq >> 1)) * P64;
+          float* t = s_wt + sbase + kq[h].z;
           *reinterpret_cast<float2*>(t) = make_float2(wq[0], wq[1]);
           *reinterpret_cast<float2*>(t + P64) = make_float2(wq[2], wq[3]);
           // the four children give the parent's variance (Section 3.2)
-          const unsigned bal = __ballot_sync(kFull, var_sum4(wq[0], wq[1], wq[2], wq[3]) > theta4);
+          const unsigned bal = __ballot_sync(kFull, var16(wq[0], wq[1], wq[2], wq[3]) > theta16);
           if (lane == 0) split_k[(TPB / 32) * k] = bal;
           const bool near = sqdiff(wq[0], wq[1]) <= band2 && sqdiff(wq[2], wq[3]) <= band2 &&
                             sqdiff(wq[0], wq[2]) <= band2 && sqdiff(wq[1], wq[3]) <= band2;
@@ -743,8 +752,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
         if (lane == 0) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
         continue;
       }
-      const uint32_t kq = uint32_t(TPB * k);
-      const float* t = s_wt + sbase + 2 * int(compact1by1(kq)) + 2 * int(compact1by1(kq >> 1)) * P64;  // (2pi, 2pj)
+      const float* t = s_wt + sbase + s_kq[k].z;  // (2pi, 2pj)
       const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
       const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
       const float l0 = t[-1], l2 = t[P64 - 1], r1 = t[2], r3 = t[P64 + 2];
@@ -810,7 +818,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
         }
       }
       if (fused && d >= 1) {
-        const unsigned bal = __ballot_sync(kFull, valid && var_sum4(w[0], w[1], w[2], w[3]) > theta4);
+        const unsigned bal = __ballot_sync(kFull, valid && var16(w[0], w[1], w[2], w[3]) > theta16);
         const int q0 = base + warp * 32;
         if (lane == 0 && q0 < nq) split_row[A.word_off[d - 1] + q0 / 32] = bal;
       }
@@ -905,7 +913,7 @@ __global__ void planes_kernel(const float* __restrict__ out, const float* __rest
   const uint32_t nq = 1u << (2 * d);
   const bool valid = q < nq;
   const int n = 1 << (d + 1);
-  const float theta4 = 4.f * theta, band2 = band * band;
+  const float theta16 = 16.f * theta, band2 = band * band;
   const float* o = out + r * G.n_total;
   bool sp[4] = {false, false, false, false}, bp[4] = {false, false, false, false};
   if (valid) {
@@ -919,10 +927,10 @@ __global__ void planes_kernel(const float* __restrict__ out, const float* __rest
       float S = 0.f;
       if (d < G.D) {
         const float4 ch = *reinterpret_cast<const float4*>(o + G.level_off[d + 1] + 4 * int64_t(m));
-        S = var_sum4(ch.x, ch.y, ch.z, ch.w);
-        sp[c] = S > theta4;
+        S = var16(ch.x, ch.y, ch.z, ch.w);
+        sp[c] = S > theta16;
       }
-      if (var_dbg) var_dbg[r * G.n_total + G.level_off[d] + m] = 0.25f * S;
+      if (var_dbg) var_dbg[r * G.n_total + G.level_off[d] + m] = 0.0625f * S;
       float nbv[4];
       const int ni[4] = {i - 1, i + 1, i, i}, nj[4] = {j, j, j - 1, j + 1};
 #pragma unroll

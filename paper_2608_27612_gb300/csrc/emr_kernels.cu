@@ -787,64 +787,81 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     return;
   }
 
-  // ---- tile 0: depths 0..min(D, 4), one after the other (at most 256 quads each)
+  // ---- tile 0: depths 0..min(D, 4). One pass evaluates the quads and ring points
+  // of every depth (work items: the quads of depth 0, 1, ..., then four ring
+  // points at a time), one barrier, then each depth is filtered from shared memory.
   const int d_hi = min(A.D, kPyramidTop);
-  for (int d = 0; d <= d_hi; d++) {
-    const int T = 1 << (d + 1), n = T;
-    const float scale = __int_as_float((127 - (d + 1)) << 23);
-    const int nq = T * T / 4, nring = 4 * T, pitch = T + 2 * kPad;
-    const int64_t lrow = prow + A.level_off[d];
-    if (fused && nv == 0) {
+  if (fused && nv == 0) {
+    for (int d = 0; d <= d_hi; d++) {
+      const int nq = 1 << (2 * d);
       for (int k = tid; k < (nq + 31) / 32; k += TPB)
         if (d >= 1) split_row[A.word_off[d - 1] + k] = 0u;
       for (int k = tid; k < (4 * nq + 31) / 32; k += TPB) A.bandb[band_base + A.word_off[d] + k] = 0u;
-      continue;
     }
+    return;
+  }
+  const bool ring = fused || A.out_halo != nullptr;
+  const int n_quads = ((4 << (2 * d_hi)) - 1) / 3;       // quads of depths 0..d_hi
+  const int n_items = n_quads + (ring ? (4 << d_hi) - 2 : 0);  // + ring groups (side / 4 ... of each depth)
+  for (int u = tid; u < n_items; u += TPB) {
+    int d = 0, li[4], lj[4];
+    bool quad = u < n_quads;
+    if (quad) {
+      while (((4 << (2 * d)) - 1) / 3 <= u) d++;
+      const uint32_t q = uint32_t(u - ((1 << (2 * d)) - 1) / 3);
+      const int pi = int(compact1by1(q)), pj = int(compact1by1(q >> 1));
+#pragma unroll
+      for (int c = 0; c < 4; c++) { li[c] = 2 * pi + (c & 1); lj[c] = 2 * pj + (c >> 1); }
+    } else {
+      const int g = u - n_quads;
+      while ((2 << (d + 1)) - 2 <= g) d++;
+      const int T = 1 << (d + 1);
+#pragma unroll
+      for (int c = 0; c < 4; c++) {  // ring point t lies on side t / T
+        const int t = 4 * (g - ((2 << d) - 2)) + c, sd = t >> (d + 1), uu = t & (T - 1);
+        li[c] = sd == 0 ? -1 : sd == 1 ? T : uu;
+        lj[c] = sd == 2 ? -1 : sd == 3 ? T : uu;
+      }
+    }
+    const int T = 1 << (d + 1), pitch = T + 2 * kPad;
+    const float scale = __int_as_float((127 - (d + 1)) << 23);
+    float x[4], y[4], w[4];
+#pragma unroll
+    for (int c = 0; c < 4; c++) { x[c] = grid_coord(li[c], scale); y[c] = grid_coord(lj[c], scale); }
+    eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
+    if (fused) {
+      int sb = 0;  // this depth's padded grid in shared memory
+      for (int e = 0; e < d; e++) sb += ((2 << e) + 2 * kPad) * ((2 << e) + 2 * kPad);
+#pragma unroll
+      for (int c = 0; c < 4; c++) s_wt[sb + (lj[c] + kPad) * pitch + li[c] + kPad] = w[c];
+    } else if (quad) {
+      const uint32_t q = uint32_t(u - ((1 << (2 * d)) - 1) / 3);
+      *reinterpret_cast<float4*>(A.out + prow + A.level_off[d] + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+    } else {
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        const int hs = li[c] < 0 ? 0 : li[c] >= T ? 1 : lj[c] < 0 ? 2 : 3;
+        A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * T + (hs < 2 ? lj[c] : li[c])] = w[c];
+      }
+    }
+  }
+  if (!fused) return;
+  __syncthreads();
+  int sb = 0;
+  for (int d = 0; d <= d_hi; d++) {
+    const int T = 1 << (d + 1), nq = T * T / 4, pitch = T + 2 * kPad;
+    const int64_t lrow = prow + A.level_off[d];
     for (int base = 0; base < nq; base += TPB) {
       const int q = base + tid;
       const bool valid = q < nq;
-      const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-      float w[4] = {0.f, 0.f, 0.f, 0.f};
-      if (valid) {
-        const float xa = grid_coord(2 * pi, scale), xb = grid_coord(2 * pi + 1, scale);
-        const float ya = grid_coord(2 * pj, scale), yb = grid_coord(2 * pj + 1, scale);
-        const float x[4] = {xa, xb, xa, xb}, y[4] = {ya, ya, yb, yb};
-        eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
-        if (fused) {
-          float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
-          t[0] = w[0]; t[1] = w[1]; t[pitch] = w[2]; t[pitch + 1] = w[3];
-        } else {
-          *reinterpret_cast<float4*>(A.out + lrow + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
-        }
-      }
-      if (fused && d >= 1) {
-        const unsigned bal = __ballot_sync(kFull, valid && var16(w[0], w[1], w[2], w[3]) > theta16);
-        const int q0 = base + warp * 32;
-        if (lane == 0 && q0 < nq) split_row[A.word_off[d - 1] + q0 / 32] = bal;
-      }
-    }
-    if (fused || A.out_halo) {
-      for (int t = tid; t < nring; t += TPB) {
-        const int sd = t / T, uu = t - sd * T;
-        const int li = sd == 0 ? -1 : sd == 1 ? T : uu, lj = sd == 2 ? -1 : sd == 3 ? T : uu;
-        const float x[1] = {grid_coord(li, scale)}, y[1] = {grid_coord(lj, scale)};
-        float wr[1];
-        eval_dense<NVMAX, 1>(s_coef, s_W, nv, out_const, x, y, wr);
-        if (fused) s_wt[(lj + kPad) * pitch + li + kPad] = wr[0];
-        else A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + sd * n + uu] = wr[0];
-      }
-    }
-    if (!fused) continue;
-    __syncthreads();
-    for (int base = 0; base < nq; base += TPB) {
-      const int q = base + tid;
-      const bool valid = q < nq;
-      bool pass[4] = {false, false, false, false};
+      bool pass[4] = {false, false, false, false}, split = false;
       float w[4] = {0.f, 0.f, 0.f, 0.f};
       if (valid) {
         const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-        const float* t = s_wt + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+        const float* t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
         w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
+        // the four children give the parent's variance (Section 3.2)
+        split = var16(w[0], w[1], w[2], w[3]) > theta16;
         const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
         const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
         const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
@@ -855,9 +872,13 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
           if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
         }
       }
+      const int q0 = base + warp * 32;
+      if (d >= 1) {
+        const unsigned bal = __ballot_sync(kFull, split);
+        if (lane == 0 && q0 < nq) split_row[A.word_off[d - 1] + q0 / 32] = bal;
+      }
       const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
       const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-      const int q0 = base + warp * 32;
       if (d >= kQuadMajorFrom) {
         if (lane < 4 && q0 < nq)
           A.bandb[band_base + A.word_off[d] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
@@ -870,7 +891,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
           if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
       }
     }
-    __syncthreads();
+    sb += pitch * pitch;
   }
 }
 

@@ -669,11 +669,12 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
     // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the nodes
     constexpr int QPE = NVMAX <= 4 ? 2 : 1;
-    // bit k: some quad of this warp's k-th group may pass the band test. A position
-    // passes only if both differences along one axis exceed the band, and one of
-    // them is to its sibling in the quad; so a quad whose four sibling differences
-    // are all within the band has no passing position, whatever its neighbours.
-    uint32_t need = 0u;
+    // A position passes the band test only if both differences along one axis
+    // exceed the band, and one of them is to its sibling in the quad. The sum of the
+    // six squared sibling differences (16 V, rounded upward monotonically) bounds
+    // each of them, so a quad with 16 V within band^2 has no passing position,
+    // whatever its neighbours; need: some quad of this thread may have one.
+    bool need = false;
 #pragma unroll 1
     for (int k0 = 0; k0 < QPT; k0 += QPE) {
       float x[4 * QPE], y[4 * QPE], w[4 * QPE];
@@ -696,18 +697,17 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
           *reinterpret_cast<float2*>(t) = make_float2(wq[0], wq[1]);
           *reinterpret_cast<float2*>(t + P64) = make_float2(wq[2], wq[3]);
           // the four children give the parent's variance (Section 3.2)
-          const unsigned bal = __ballot_sync(kFull, var16(wq[0], wq[1], wq[2], wq[3]) > theta16);
+          const float v16 = var16(wq[0], wq[1], wq[2], wq[3]);
+          const unsigned bal = __ballot_sync(kFull, v16 > theta16);
           if (lane == 0) split_k[(TPB / 32) * k] = bal;
-          const bool near = sqdiff(wq[0], wq[1]) <= band2 && sqdiff(wq[2], wq[3]) <= band2 &&
-                            sqdiff(wq[0], wq[2]) <= band2 && sqdiff(wq[1], wq[3]) <= band2;
-          if (__any_sync(kFull, !near)) need |= 1u << k;
+          need = need || !(v16 <= band2);
         } else {
           *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
               make_float4(wq[0], wq[1], wq[2], wq[3]);
         }
       }
     }
-    if (fused && !__syncthreads_or(need != 0u)) {  // no position of the tile can pass
+    if (fused && !__syncthreads_or(need)) {  // no position of the tile can pass
       if (lane == 0)
         for (int k = 0; k < QPT; k++) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
       return;
@@ -748,10 +748,6 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     // band value of each position from its four neighbours at distance 2^-d
 #pragma unroll 2
     for (int k = 0; k < QPT; k++) {
-      if (!((need >> k) & 1u)) {  // warp-uniform
-        if (lane == 0) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
-        continue;
-      }
       const float* t = s_wt + sbase + s_kq[k].z;  // (2pi, 2pj)
       const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
       const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);

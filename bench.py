@@ -51,7 +51,7 @@ def parse():
     ap.add_argument("--depth", type=int, default=7)
     ap.add_argument("--pop", type=int, default=1000)
     ap.add_argument("--e2e-steps", type=int, default=20)
-    ap.add_argument("--cpu-genomes", type=int, default=160, help="oracle baseline sample (genomes)")
+    ap.add_argument("--cpu-genomes", type=int, default=1000, help="oracle baseline sample (genomes)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the streamed depth-13 and h->h round measurements")
     return ap.parse_args()

@@ -221,8 +221,9 @@ def profiled_traffic():
     return None
 
 
-def streamed_run(emr, torch, w, chunk, chunk_cap, cap, reps):
-    """Queries/sec of emr_stream on workload w (lists copied to pinned host memory)."""
+def streamed_run(emr, torch, w, chunk, chunk_cap, cap, reps, mode=0, types=15, label=None):
+    """Queries/sec of emr_stream (emr_stream_mode when a mode or type filter is given) on
+    workload w (lists copied to pinned host memory)."""
     pack = emr.pack_population(w.pop)
     pack_dev = torch.from_numpy(pack).cuda()
     q = emr.make_query(w.sources)
@@ -240,14 +241,16 @@ def streamed_run(emr, torch, w, chunk, chunk_cap, cap, reps):
     for k in range(reps + 1):
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        emr.stream(pack, pack_dev, q, g, w.theta, w.band, w.w_min, ws, chunk_cap, h_idx, h_w, counts, offsets)
+        emr.stream(pack, pack_dev, q, g, w.theta, w.band, w.w_min, ws, chunk_cap, h_idx, h_w, counts, offsets,
+                   mode=mode, types=types)
         if k:
             times.append(time.perf_counter() - t0)
     del ws
     torch.cuda.empty_cache()
     s = statistics.median(times)
-    return {"workload": w.name, "queries": queries, "seconds": s, "value": queries / s, "unit": UNIT,
-            "chunk_positions": chunk, "kept": int(offsets[-1]),
+    return {"workload": label or w.name, "queries": queries, "seconds": s, "value": queries / s, "unit": UNIT,
+            "chunk_positions": chunk, "kept": int(offsets[-1]), "mode": "gated" if mode else "eager",
+            "connection_types": types,
             "timing": "host wall clock per emr_stream call (synchronous, lists on the host), median of %d" % reps}
 
 
@@ -431,8 +434,14 @@ def main():
 
     extra = None
     if rank == 0 and ws == 1 and not args.no_extra:
+        c4r2 = W.c4_round2_random()
         extra = {"c5_streamed_d13": streamed_run(emr, torch, W.c5(), 1 << 26, 1 << 24, 1 << 26, 3),
-                 "c4_round2_hh_d8": streamed_run(emr, torch, W.c4_round2_random(), 1 << 16, 1 << 24, 1 << 26, 3)}
+                 "c5_streamed_d13_gated": streamed_run(emr, torch, W.c5(), 1 << 26, 1 << 24, 1 << 26, 3,
+                                                       mode=emr.EMR_GATED),
+                 "c4_round2_hh_d8": streamed_run(emr, torch, c4r2, 1 << 16, 1 << 24, 1 << 26, 3),
+                 "c4_round2_hh_d8_backward_config": streamed_run(
+                     emr, torch, c4r2, 1 << 16, 1 << 24, 1 << 26, 3,
+                     types=emr.substrate_config(emr.SUBSTRATE_BACKWARD)[0], label=c4r2.name + "_backward")}
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:

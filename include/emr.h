@@ -78,6 +78,13 @@ enum { EMR_KIND_X1 = 0, EMR_KIND_Y1 = 1, EMR_KIND_X2 = 2, EMR_KIND_Y2 = 3, EMR_K
        EMR_KIND_HIDDEN = 5, EMR_KIND_OUTPUT = 6 };
 enum { EMR_SIDE_OUT = 0, EMR_SIDE_IN = 1 };
 enum { EMR_EAGER = 0, EMR_GATED = 1 };
+/* Connection types (Section 6, connection type taxonomy), as bits of a filter
+ * and, in emr_conn_types, as codes 0..3 in this order: forward (source below
+ * target, y_s < y_t), backward (y_s > y_t), lateral (y_s = y_t), self-loop (s = t). */
+enum { EMR_CONN_F = 1, EMR_CONN_B = 2, EMR_CONN_L = 4, EMR_CONN_S = 8, EMR_CONN_ALL = 15 };
+/* The six substrate configurations of Section 6 (its table), see emr_substrate_config. */
+enum { EMR_SUBSTRATE_FEEDFORWARD = 0, EMR_SUBSTRATE_HH = 1, EMR_SUBSTRATE_BACKWARD = 2,
+       EMR_SUBSTRATE_LATERAL = 3, EMR_SUBSTRATE_SELF = 4, EMR_SUBSTRATE_FULL = 5 };
 
 /* Grid descriptor (Eq. 1): sizes and offsets only, no positions are stored;
  * kernels generate coordinates from (depth, Morton index). */
@@ -206,6 +213,26 @@ emr_status emr_variance_filter(const float *out, const float *out_halo, const em
 emr_status emr_mask_combine(const uint32_t *split, const uint32_t *band_bits, const emr_grid *grid,
                             int32_t n_pairs, int32_t mode, uint32_t *mask, void *stream);
 
+/* emr_mask_combine, then keep only connections whose type (Section 6
+ * taxonomy) is in types (EMR_CONN_* bits; EMR_CONN_ALL keeps every type). A
+ * connection joins pair r's query slot (q's slot r mod S, or row r in
+ * per-genome mode) and a grid position: on the outgoing side the slot is the
+ * source, on the incoming side the target. n_pairs must be a multiple of q->S.
+ * The comparisons are exact: grid coordinates are dyadic and computed exactly
+ * in fp32, and the slot coordinates are the fp32 values of q.
+ * Errors: EMR_ERR_ARG, EMR_ERR_CUDA. */
+emr_status emr_mask_combine_types(const uint32_t *split, const uint32_t *band_bits, const emr_query *q,
+                                  const emr_grid *grid, int32_t n_pairs, int32_t mode, int32_t types,
+                                  uint32_t *mask, void *stream);
+
+/* Connection types enabled by one of the six substrate configurations of
+ * Section 6 (EMR_SUBSTRATE_*), and whether it runs hidden-to-hidden rounds
+ * (*hidden_rounds = 1; 0 for the feedforward configuration, which skips the
+ * second phase): feedforward F; hidden-to-hidden F (+ rounds); backward F, B;
+ * lateral F, L; self F, S; full recurrent F, B, L, S. Either output may be
+ * NULL. Host only. Errors: EMR_ERR_ARG (unknown config). */
+emr_status emr_substrate_config(int32_t config, int32_t *types, int32_t *hidden_rounds);
+
 /* ---- a3+a4+a5 fused ------------------------------------------------------ */
 
 /* Evaluate and filter in one kernel, without materialising the CPPN outputs:
@@ -245,8 +272,7 @@ emr_status emr_stream_workspace_size(const void *pack_host, const emr_query *q, 
  * ascending global index, counts[r] its length (host int64 [n_pairs], offsets
  * [n_pairs + 1]). chunk_cap: list entries one chunk may produce (device
  * buffers). Synchronous: returns when the lists are on the host.
- * The GATED mode needs every ancestor's decision, which a descending stream
- * only has at the end; it is not offered here.
+ * This is emr_stream_mode with EMR_EAGER and EMR_CONN_ALL.
  * Errors: EMR_ERR_ARG; EMR_ERR_CAPACITY (ws too small, or a chunk or the total
  * exceeded chunk_cap / cap: counts hold the true totals, the lists are
  * incomplete); EMR_ERR_TIMEOUT when a host wait exceeds timeout_ms (0 = no
@@ -258,6 +284,20 @@ emr_status emr_stream(const void *pack_host, const void *pack_dev, const emr_que
                       float theta, float band, float w_min, void *ws, size_t ws_bytes, int64_t chunk_cap,
                       int32_t *h_idx, float *h_w, int64_t cap, int64_t *counts, int64_t *offsets,
                       int64_t timeout_ms, void *stream);
+
+/* emr_stream with a mode and a connection-type filter (types as in
+ * emr_mask_combine_types, applied per chunk when its mask is formed). GATED
+ * (Eq. 2) needs every ancestor's split bit, which the descending stream has
+ * only at its end: the eager lists (a superset) are collected as in
+ * emr_stream, then each entry is checked against the resident split plane on
+ * the device (entries copied back chunk_cap at a time) and the lists are
+ * compacted in place on the host. cap must hold the eager lists; on
+ * EMR_ERR_CAPACITY counts hold the eager totals and no gate is applied.
+ * Errors as emr_stream. */
+emr_status emr_stream_mode(const void *pack_host, const void *pack_dev, const emr_query *q, const emr_grid *grid,
+                           float theta, float band, float w_min, int32_t mode, int32_t types, void *ws,
+                           size_t ws_bytes, int64_t chunk_cap, int32_t *h_idx, float *h_w, int64_t cap,
+                           int64_t *counts, int64_t *offsets, int64_t timeout_ms, void *stream);
 
 /* ---- fused evaluation without a caller-provided workspace -------------------- */
 
@@ -320,6 +360,15 @@ emr_status emr_compact(const uint32_t *mask, const float *out, const emr_grid *g
 emr_status emr_compact_records(const uint32_t *mask, const void *pack_host, const emr_query *q, const void *eval_ws,
                                size_t eval_ws_bytes, const emr_grid *grid, int32_t *idx, float *w, int64_t cap,
                                int64_t *counts, int64_t *offsets, void *ws, size_t ws_bytes, void *stream);
+
+/* Connection type code (0 forward, 1 backward, 2 lateral, 3 self; Section 6
+ * taxonomy, see emr_mask_combine_types) of every list entry: type[e] for
+ * entries e < min(offsets[n_pairs], cap) of lists laid out as emr_compact
+ * writes them (idx: device int32 global indices; offsets: device int64
+ * [n_pairs + 1]; type: device uint8 [cap]). n_pairs must be a multiple of q->S.
+ * Errors: EMR_ERR_ARG, EMR_ERR_CUDA. */
+emr_status emr_conn_types(const int32_t *idx, const int64_t *offsets, const emr_query *q, const emr_grid *grid,
+                          int32_t n_pairs, int64_t cap, uint8_t *type, void *stream);
 
 /* ---- misc -------------------------------------------------------------------- */
 

@@ -18,6 +18,11 @@ Parity status of each oracle function (what pins it, in tests/test_oracle_pins.p
                             the gated mask) and the closed-form worked example.
   ora_keep_at               pinned: equal to ora_discover's outputs, variance, band
                             value, decisions and uncertainty at every position.
+  ora_conn_type(s)          pinned: sources off every grid row (all forward or all
+                            backward), per-depth counts of forward / backward /
+                            lateral targets against closed forms for sources on the
+                            grid, exactly one self-loop per on-grid source, and the
+                            outgoing / incoming reversal.
 """
 from __future__ import annotations
 
@@ -155,6 +160,20 @@ def lazy(pop, sources, D: int, theta: float, band: float, w_min: float = 0.0,
     if rc != ORA_OK:
         raise ValueError("oracle: lazy failed (code %d)" % rc)
     return keep, evals
+
+
+TYPE_F, TYPE_B, TYPE_L, TYPE_S = 0, 1, 2, 3
+
+
+def conn_types(a: float, b: float, side: int, gidx):
+    """Connection type codes (0 forward, 1 backward, 2 lateral, 3 self) of the connections between
+    slot (a, b) on `side` and the grid positions gidx (Section 6 taxonomy)."""
+    g = np.ascontiguousarray(gidx, np.int64)
+    out = np.zeros(len(g), np.uint8)
+    rc = lib().ora_conn_types(C.c_double(a), C.c_double(b), C.c_int(side), C.c_int64(len(g)), _p(g), _p(out))
+    if rc != ORA_OK:
+        raise ValueError("oracle: conn_types failed (code %d)" % rc)
+    return out
 
 
 def keep_at(pop, g: int, a: float, b: float, side: int, D: int, theta: float, band: float, w_min: float,

@@ -706,3 +706,40 @@ int ora_keep_at(int g, const int64_t *node_ptr, const int32_t *node_id, const in
     genome_free(&G);
     return ORA_OK;
 }
+
+/*
+ * Connection types (Section 6, "Connection Type Taxonomy"): a connection from
+ * source s to target t is a self-loop when s = t, and otherwise forward when
+ * y_s < y_t, backward when y_s > y_t and lateral when y_s = y_t. For a query
+ * slot at (a, b): on the outgoing side the slot is the source and the grid
+ * position the target; on the incoming side the position is the source and
+ * the slot the target. Codes: 0 forward, 1 backward, 2 lateral, 3 self.
+ * Coordinates are exact dyadic rationals, so the comparisons are exact.
+ */
+int ora_conn_type(double a, double b, int side, int d, int64_t i, int64_t j)
+{
+    double x = coord(d, i), y = coord(d, j);
+    double xs = side == 0 ? a : x, ys = side == 0 ? b : y;   /* source */
+    double xt = side == 0 ? x : a, yt = side == 0 ? y : b;   /* target */
+    if (xs == xt && ys == yt) return 3;
+    if (ys < yt) return 0;
+    if (ys > yt) return 1;
+    return 2;
+}
+
+/* ora_conn_type at n positions given by global index. */
+int ora_conn_types(double a, double b, int side, int64_t n, const int64_t *gidx, uint8_t *type)
+{
+    if (n < 0 || (n > 0 && (!gidx || !type))) return ORA_ERR_ARG;
+    for (int64_t k = 0; k < n; k++) {
+        int d = 0;
+        while (level_offset(d + 1) <= gidx[k]) d++;
+        int64_t m = gidx[k] - level_offset(d), i = 0, j = 0;
+        for (int bit = 0; bit < 31; bit++) {           /* Morton decode */
+            i |= ((m >> (2 * bit)) & 1) << bit;
+            j |= ((m >> (2 * bit + 1)) & 1) << bit;
+        }
+        type[k] = (uint8_t)ora_conn_type(a, b, side, d, i, j);
+    }
+    return ORA_OK;
+}

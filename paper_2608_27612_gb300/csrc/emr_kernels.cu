@@ -1005,13 +1005,58 @@ __device__ __forceinline__ uint32_t active_bits(const uint32_t* sp, const GridDe
   return act;
 }
 
+// Connection-type filter (Section 6 taxonomy): a connection between a pair's
+// query slot (a, b) and a grid position is a self-loop when both are the same
+// point, else forward / backward / lateral as the source's y is below / above /
+// equal to the target's (outgoing side: the slot is the source; incoming: the
+// position is). types: EMR_CONN_* bits to keep; EMR_CONN_ALL disables it.
+struct TypeFilter {
+  int32_t types;
+  QueryDev q;
+};
+
+// Row r (y offset) and column c (x offset) of the 32 Morton positions of a word:
+// bits 1 and 3 of the position in the word carry y, bits 0, 2 and 4 carry x.
+__device__ __forceinline__ uint32_t word_row_bits(int r) { return 0x00330033u << (((r & 1) << 1) | ((r & 2) << 2)); }
+__device__ __forceinline__ uint32_t word_col_bits(int c) {
+  return 0x0505u << ((c & 1) | ((c & 2) << 1) | ((c & 4) << 2));
+}
+
+// Kept-type bits of the 32 positions of position-major word wi (depth d) for pair r.
+__device__ __noinline__ uint32_t type_bits(const TypeFilter& tf, int64_t r, const GridDev& G, int d, int64_t wi) {
+  const int64_t si = tf.q.per_genome ? r : r % tf.q.S;
+  const float a = tf.q.a[si], b = tf.q.b[si];
+  const bool out_side = tf.q.side[si] == EMR_SIDE_OUT;
+  const uint32_t m0 = uint32_t(wi - G.word_off[d]) * 32u;
+  const int i0 = int(compact1by1(m0)), j0 = int(compact1by1(m0 >> 1));
+  const float scale = __int_as_float((127 - (d + 1)) << 23);
+  uint32_t fw = 0u, bw = 0u, lw = 0u, sw = 0u;
+  for (int rr = 0; rr < 4; rr++) {
+    const float y = grid_coord(j0 + rr, scale);
+    const float ys = out_side ? b : y, yt = out_side ? y : b;
+    const uint32_t row = word_row_bits(rr);
+    if (ys < yt) {
+      fw |= row;
+    } else if (ys > yt) {
+      bw |= row;
+    } else {
+      lw |= row;
+      for (int c = 0; c < 8; c++)  // the slot itself, if it is a position of this row
+        if (grid_coord(i0 + c, scale) == a) sw |= row & word_col_bits(c);
+    }
+  }
+  lw &= ~sw;
+  return ((tf.types & EMR_CONN_F) ? fw : 0u) | ((tf.types & EMR_CONN_B) ? bw : 0u) |
+         ((tf.types & EMR_CONN_L) ? lw : 0u) | ((tf.types & EMR_CONN_S) ? sw : 0u);
+}
+
 // mask = band AND NOT split (no split at depth D); gated: AND Eq. 2's active bit.
 // One thread per group of 4 words (one 128-position block from depth 3 on; the
 // 4 words of depths 0..2 form group 0), pair = blockIdx.y; groups cover words
 // [w0, w0 + nw) (w0 and nw multiples of 4, or nw reaching n_words). split is a
-// whole-grid plane.
+// whole-grid plane. Planes start at pair r0 (the type filter's slots are absolute).
 __global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView band, PlaneView mask, GridDev G,
-                               int64_t w0, int64_t nw, int gated) {
+                               int64_t w0, int64_t nw, int gated, TypeFilter tf, int64_t r0) {
   const int64_t k = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) * 4;
   if (k >= nw) return;
   const int64_t r = blockIdx.y;
@@ -1029,6 +1074,7 @@ __global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView ban
     for (int c = 0; c < 4; c++) {  // re-interleave the block's four child words
       m[c] = band_word(bq.x, bq.y, bq.z, bq.w, c) & ~s4[c];
       if (gated && m[c]) m[c] &= active_bits(sp, G, d, wi + c);
+      if (tf.types != EMR_CONN_ALL && m[c]) m[c] &= type_bits(tf, r0 + r, G, d, wi + c);
     }
     *reinterpret_cast<uint4*>(&mask.at(r, wi)) = make_uint4(m[0], m[1], m[2], m[3]);
   } else {
@@ -1039,6 +1085,7 @@ __global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView ban
       uint32_t keep = band.at(r, wc) & valid_bits(G, d, wc);
       if (d < G.D) keep &= ~sp[wc];
       if (gated && keep) keep &= active_bits(sp, G, d, wc);
+      if (tf.types != EMR_CONN_ALL && keep) keep &= type_bits(tf, r0 + r, G, d, wc);
       mask.at(r, wc) = keep;
     }
   }
@@ -1222,6 +1269,16 @@ __global__ void compact_write_kernel(PlaneView mask, const float* __restrict__ o
   }
 }
 
+// The pair whose list holds entry t: the last r with offsets[r] <= t.
+__device__ __forceinline__ int64_t pair_of_entry(const int64_t* __restrict__ offsets, int64_t n_pairs, int64_t t) {
+  int64_t lo = 0, hi = n_pairs;  // offsets[lo] <= t < offsets[hi]
+  while (hi - lo > 1) {
+    const int64_t mid = (lo + hi) >> 1;
+    if (offsets[mid] <= t) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
 // Weights of the listed kept positions, recomputed from the records: one entry
 // per thread (kept positions cluster, so a thread per mask word would evaluate
 // long runs serially). The entry's pair is the last r with offsets[r] <= t.
@@ -1233,11 +1290,7 @@ __global__ void __launch_bounds__(kCompactBlock) kept_weights_kernel(RecordSourc
   const int64_t total = offsets[n_pairs] < cap ? offsets[n_pairs] : cap;
   for (int64_t t = int64_t(blockIdx.x) * kCompactBlock + threadIdx.x; t < total;
        t += int64_t(gridDim.x) * kCompactBlock) {
-    int64_t lo = 0, hi = n_pairs;  // offsets[lo] <= t < offsets[hi]
-    while (hi - lo > 1) {
-      const int64_t mid = (lo + hi) >> 1;
-      if (offsets[mid] <= t) lo = mid; else hi = mid;
-    }
+    const int64_t lo = pair_of_entry(offsets, n_pairs, t);
     const int64_t gidx = idx[t];
     int d = 0;
     while (G.level_off[d + 1] <= gidx) d++;
@@ -1245,6 +1298,54 @@ __global__ void __launch_bounds__(kCompactBlock) kept_weights_kernel(RecordSourc
     const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1)
     const float x = grid_coord(int(compact1by1(m)), scale), y = grid_coord(int(compact1by1(m >> 1)), scale);
     wv[t] = eval_record_point(rs.spec + lo * rs.L.stride, rs.L, x, y);
+  }
+}
+
+// Connection type code of each list entry (0 forward, 1 backward, 2 lateral,
+// 3 self; Section 6 taxonomy), from the pair's query slot and the position.
+__global__ void __launch_bounds__(kCompactBlock) conn_types_kernel(QueryDev q, GridDev G,
+                                                                   const int64_t* __restrict__ offsets,
+                                                                   int64_t n_pairs, int64_t cap,
+                                                                   const int32_t* __restrict__ idx,
+                                                                   uint8_t* __restrict__ type) {
+  const int64_t total = offsets[n_pairs] < cap ? offsets[n_pairs] : cap;
+  for (int64_t t = int64_t(blockIdx.x) * kCompactBlock + threadIdx.x; t < total;
+       t += int64_t(gridDim.x) * kCompactBlock) {
+    const int64_t r = pair_of_entry(offsets, n_pairs, t);
+    const int64_t si = q.per_genome ? r : r % q.S;
+    const float a = q.a[si], b = q.b[si];
+    const bool out_side = q.side[si] == EMR_SIDE_OUT;
+    const int64_t gidx = idx[t];
+    int d = 0;
+    while (G.level_off[d + 1] <= gidx) d++;
+    const uint32_t m = uint32_t(gidx - G.level_off[d]);
+    const float scale = __int_as_float((127 - (d + 1)) << 23);
+    const float x = grid_coord(int(compact1by1(m)), scale), y = grid_coord(int(compact1by1(m >> 1)), scale);
+    const float xs = out_side ? a : x, ys = out_side ? b : y, xt = out_side ? x : a, yt = out_side ? y : b;
+    type[t] = (xs == xt && ys == yt) ? 3 : ys < yt ? 0 : ys > yt ? 1 : 2;
+  }
+}
+
+// Eq. 2 gate of n listed entries (global entry numbers e0 .. e0 + n - 1 of
+// lists with the given offsets): keep[t] = 1 when every ancestor of the entry's
+// position split, read from the complete split plane.
+__global__ void __launch_bounds__(kCompactBlock) gate_kernel(const uint32_t* __restrict__ split, GridDev G,
+                                                             const int64_t* __restrict__ offsets, int64_t n_pairs,
+                                                             int64_t e0, int64_t n, const int32_t* __restrict__ idx,
+                                                             uint8_t* __restrict__ keep) {
+  for (int64_t t = int64_t(blockIdx.x) * kCompactBlock + threadIdx.x; t < n; t += int64_t(gridDim.x) * kCompactBlock) {
+    const int64_t r = pair_of_entry(offsets, n_pairs, e0 + t);
+    const int64_t gidx = idx[t];
+    int d = 0;
+    while (G.level_off[d + 1] <= gidx) d++;
+    const uint32_t m = uint32_t(gidx - G.level_off[d]);
+    const uint32_t* sp = split + r * G.n_words;
+    bool act = true;
+    for (int k = 1; k <= d && act; k++) {
+      const uint32_t am = m >> (2 * k);  // ancestor at depth d - k
+      act = (sp[G.word_off[d - k] + (am >> 5)] >> (am & 31u)) & 1u;
+    }
+    keep[t] = act ? 1 : 0;
   }
 }
 
@@ -1470,29 +1571,35 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
 }
 
 emr_status launch_combine(const uint32_t* split, PlaneView band, PlaneView mask, const emr_grid* g, int64_t n_pairs,
-                          int64_t w0, int64_t nw, int gated, cudaStream_t st) {
+                          int64_t w0, int64_t nw, int gated, cudaStream_t st, TypeFilter tf, int64_t r0 = 0) {
   if (n_pairs <= 0 || nw <= 0) return EMR_OK;
   if (n_pairs > 65535) {  // grid y limit: split the pairs
-    for (int64_t r0 = 0; r0 < n_pairs; r0 += 65535) {
-      const int64_t nr = std::min<int64_t>(65535, n_pairs - r0);
+    for (int64_t q0 = 0; q0 < n_pairs; q0 += 65535) {
+      const int64_t nr = std::min<int64_t>(65535, n_pairs - q0);
       PlaneView b2 = band, m2 = mask;
-      b2.p += r0 * band.stride;
-      m2.p += r0 * mask.stride;
-      emr_status rc = launch_combine(split + r0 * g->n_words, b2, m2, g, nr, w0, nw, gated, st);
+      b2.p += q0 * band.stride;
+      m2.p += q0 * mask.stride;
+      emr_status rc = launch_combine(split + q0 * g->n_words, b2, m2, g, nr, w0, nw, gated, st, tf, r0 + q0);
       if (rc != EMR_OK) return rc;
     }
     return EMR_OK;
   }
   const int64_t groups = (nw + 3) / 4;
   dim3 grid(unsigned((groups + 255) / 256), unsigned(n_pairs));
-  combine_kernel<<<grid, 256, 0, st>>>(split, band, mask, grid_dev(g), w0, nw, gated);
+  combine_kernel<<<grid, 256, 0, st>>>(split, band, mask, grid_dev(g), w0, nw, gated, tf, r0);
   return cuda_status(cudaGetLastError());
 }
 
+TypeFilter no_type_filter() {
+  TypeFilter tf{};
+  tf.types = EMR_CONN_ALL;
+  return tf;
+}
+
 emr_status launch_combine(const uint32_t* split, const uint32_t* bandb, const emr_grid* g, int64_t n_pairs, int gated,
-                          uint32_t* mask, cudaStream_t st) {
+                          uint32_t* mask, cudaStream_t st, TypeFilter tf = no_type_filter()) {
   return launch_combine(split, PlaneView{const_cast<uint32_t*>(bandb), g->n_words, 0},
-                        PlaneView{mask, g->n_words, 0}, g, n_pairs, 0, g->n_words, gated, st);
+                        PlaneView{mask, g->n_words, 0}, g, n_pairs, 0, g->n_words, gated, st, tf);
 }
 
 constexpr int64_t kCompactWords = 4 * kCompactBlock;  // words per compaction block
@@ -1577,6 +1684,44 @@ emr_status emr_mask_combine(const uint32_t* split, const uint32_t* band_bits, co
   if (!split || !band_bits || !mask || !grid_ok(grid) || n_pairs <= 0 || (mode != EMR_EAGER && mode != EMR_GATED))
     return EMR_ERR_ARG;
   return launch_combine(split, band_bits, grid, n_pairs, mode == EMR_GATED, mask, static_cast<cudaStream_t>(stream));
+}
+
+emr_status emr_mask_combine_types(const uint32_t* split, const uint32_t* band_bits, const emr_query* q,
+                                  const emr_grid* grid, int32_t n_pairs, int32_t mode, int32_t types, uint32_t* mask,
+                                  void* stream) {
+  if (!split || !band_bits || !mask || !grid_ok(grid) || n_pairs <= 0 || (mode != EMR_EAGER && mode != EMR_GATED))
+    return EMR_ERR_ARG;
+  if (!q || q->S <= 0 || !q->a_dev || !q->b_dev || !q->side_dev || n_pairs % q->S != 0 || types < 0 ||
+      types > EMR_CONN_ALL)
+    return EMR_ERR_ARG;
+  TypeFilter tf;
+  tf.types = types;
+  tf.q = query_dev(q);
+  return launch_combine(split, band_bits, grid, n_pairs, mode == EMR_GATED, mask, static_cast<cudaStream_t>(stream),
+                        tf);
+}
+
+emr_status emr_conn_types(const int32_t* idx, const int64_t* offsets, const emr_query* q, const emr_grid* grid,
+                          int32_t n_pairs, int64_t cap, uint8_t* type, void* stream) {
+  if (!offsets || !grid_ok(grid) || n_pairs <= 0 || cap < 0 || (cap > 0 && (!idx || !type))) return EMR_ERR_ARG;
+  if (!q || q->S <= 0 || !q->a_dev || !q->b_dev || !q->side_dev || n_pairs % q->S != 0) return EMR_ERR_ARG;
+  if (cap == 0) return EMR_OK;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return EMR_ERR_CUDA;
+  conn_types_kernel<<<unsigned(8 * sms), kCompactBlock, 0, static_cast<cudaStream_t>(stream)>>>(
+      query_dev(q), grid_dev(grid), offsets, n_pairs, cap, idx, type);
+  return cuda_status(cudaGetLastError());
+}
+
+emr_status emr_substrate_config(int32_t config, int32_t* types, int32_t* hidden_rounds) {
+  static const int32_t kTypes[6] = {EMR_CONN_F, EMR_CONN_F, EMR_CONN_F | EMR_CONN_B, EMR_CONN_F | EMR_CONN_L,
+                                    EMR_CONN_F | EMR_CONN_S, EMR_CONN_ALL};
+  if (config < EMR_SUBSTRATE_FEEDFORWARD || config > EMR_SUBSTRATE_FULL) return EMR_ERR_ARG;
+  if (types) *types = kTypes[config];
+  if (hidden_rounds) *hidden_rounds = config == EMR_SUBSTRATE_FEEDFORWARD ? 0 : 1;
+  return EMR_OK;
 }
 
 emr_status emr_variance_filter(const float* out, const float* out_halo, const emr_grid* grid, int32_t P, int32_t S,
@@ -1805,13 +1950,18 @@ extern "C" emr_status emr_stream_workspace_size(const void* pack_host, const emr
   return EMR_OK;
 }
 
-extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, const emr_query* q,
-                                 const emr_grid* grid, float theta, float band, float w_min, void* ws, size_t ws_bytes,
-                                 int64_t chunk_cap, int32_t* h_idx, float* h_w, int64_t cap, int64_t* counts,
-                                 int64_t* offsets, int64_t timeout_ms, void* stream) {
+extern "C" emr_status emr_stream_mode(const void* pack_host, const void* pack_dev, const emr_query* q,
+                                      const emr_grid* grid, float theta, float band, float w_min, int32_t mode,
+                                      int32_t types, void* ws, size_t ws_bytes, int64_t chunk_cap, int32_t* h_idx,
+                                      float* h_w, int64_t cap, int64_t* counts, int64_t* offsets, int64_t timeout_ms,
+                                      void* stream) {
   if (!pack_dev || !ws || !counts || !offsets || cap < 0 || (cap > 0 && (!h_idx || !h_w)) || timeout_ms < 0)
     return EMR_ERR_ARG;
   if (!(theta >= 0.f) || !(band >= 0.f) || !(w_min >= 0.f)) return EMR_ERR_ARG;
+  if ((mode != EMR_EAGER && mode != EMR_GATED) || types < 0 || types > EMR_CONN_ALL || !q) return EMR_ERR_ARG;
+  TypeFilter tf;
+  tf.types = types;
+  tf.q = query_dev(q);
   StreamPlan sp;
   emr_status rc = stream_plan(pack_host, q, grid, chunk_cap, &sp);
   if (rc != EMR_OK) return rc;
@@ -1888,7 +2038,7 @@ extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, co
                            st, tr)) != EMR_OK)
       break;
     if ((rc = launch_combine(split, PlaneView{bandc, sp.wpc, w_lo}, PlaneView{maskc, sp.wpc, w_lo}, grid, NP, w_lo,
-                             w_hi - w_lo, 0, st)) != EMR_OK)
+                             w_hi - w_lo, 0, st, tf)) != EMR_OK)
       break;
     if ((rc = launch_compact(PlaneView{maskc, sp.wpc, w_lo}, nullptr, 0, 0, grid, NP, w_lo, w_hi - w_lo,
                              reinterpret_cast<int32_t*>(base + sp.off_idx[b]),
@@ -1927,6 +2077,50 @@ extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, co
     }
     if (overflow) rc = EMR_ERR_CAPACITY;
   }
+  if (rc == EMR_OK && mode == EMR_GATED && cursor > 0) {
+    // Eq. 2 needs every ancestor's split bit, final only now: gate the eager lists
+    // (a superset) against the resident split plane, a buffer of entries at a time.
+    int64_t* off_dev = reinterpret_cast<int64_t*>(base + sp.off_off[0]);
+    int32_t* idx_dev = reinterpret_cast<int32_t*>(base + sp.off_idx[0]);
+    uint8_t* keep_dev = base + sp.off_w[0];
+    std::vector<uint8_t> keep(static_cast<size_t>(cursor));
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaMemcpyAsync(off_dev, offsets, size_t(NP + 1) * 8, cudaMemcpyHostToDevice, st) != cudaSuccess)
+      rc = EMR_ERR_CUDA;
+    for (int64_t e0 = 0; e0 < cursor && rc == EMR_OK; e0 += sp.chunk_cap) {
+      const int64_t n = std::min(sp.chunk_cap, cursor - e0);
+      if (cudaMemcpyAsync(idx_dev, h_idx + e0, size_t(n) * 4, cudaMemcpyHostToDevice, st) != cudaSuccess) {
+        rc = EMR_ERR_CUDA;
+        break;
+      }
+      gate_kernel<<<unsigned(8 * sms), kCompactBlock, 0, st>>>(split, grid_dev(grid), off_dev, NP, e0, n, idx_dev,
+                                                              keep_dev);
+      if (cudaGetLastError() != cudaSuccess ||
+          cudaMemcpyAsync(keep.data() + e0, keep_dev, size_t(n), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+          cudaEventRecord(ev_done[0], st) != cudaSuccess) {
+        rc = EMR_ERR_CUDA;
+        break;
+      }
+      rc = wait_event(ev_done[0], deadline, limited);
+    }
+    if (rc == EMR_OK) {  // drop the ungated entries in place, pair by pair
+      int64_t dst = 0;
+      for (int64_t r = 0; r < NP; r++) {
+        const int64_t beg = offsets[r], end = offsets[r + 1];
+        offsets[r] = dst;
+        for (int64_t e = beg; e < end; e++)
+          if (keep[size_t(e)]) {
+            h_idx[dst] = h_idx[e];
+            h_w[dst] = h_w[e];
+            dst++;
+          }
+        counts[r] = dst - offsets[r];
+      }
+      offsets[NP] = dst;
+    }
+  }
   // a timed-out call leaves its queued work running; release what is safe to release
   if (rc != EMR_ERR_TIMEOUT && staging) cudaFreeHost(staging);
   for (int b = 0; b < 2; b++) {
@@ -1935,4 +2129,12 @@ extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, co
   }
   if (cp) cudaStreamDestroy(cp);
   return rc;
+}
+
+extern "C" emr_status emr_stream(const void* pack_host, const void* pack_dev, const emr_query* q,
+                                 const emr_grid* grid, float theta, float band, float w_min, void* ws, size_t ws_bytes,
+                                 int64_t chunk_cap, int32_t* h_idx, float* h_w, int64_t cap, int64_t* counts,
+                                 int64_t* offsets, int64_t timeout_ms, void* stream) {
+  return emr_stream_mode(pack_host, pack_dev, q, grid, theta, band, w_min, EMR_EAGER, EMR_CONN_ALL, ws, ws_bytes,
+                         chunk_cap, h_idx, h_w, cap, counts, offsets, timeout_ms, stream);
 }

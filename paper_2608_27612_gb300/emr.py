@@ -21,6 +21,9 @@ EMR_OK, EMR_ERR_ARG, EMR_ERR_CYCLE, EMR_ERR_RANGE, EMR_ERR_CAPACITY, EMR_ERR_CUD
     EMR_ERR_ALLOC = range(8)
 EMR_MAX_DEPTH = 14
 EMR_EAGER, EMR_GATED = 0, 1
+CONN_F, CONN_B, CONN_L, CONN_S, CONN_ALL = 1, 2, 4, 8, 15
+SUBSTRATE_FEEDFORWARD, SUBSTRATE_HH, SUBSTRATE_BACKWARD, SUBSTRATE_LATERAL, SUBSTRATE_SELF, SUBSTRATE_FULL = range(6)
+TYPE_CODES = ("forward", "backward", "lateral", "self")
 _M = EMR_MAX_DEPTH + 2
 
 _lib = None
@@ -67,6 +70,10 @@ def lib() -> C.CDLL:
             "emr_eval_filter_noalloc": [vp, vp, vp, vp, f32, f32, f32, vp, vp, vp, vp],
             "emr_stream_workspace_size": [vp, vp, vp, i64, vp],
             "emr_stream": [vp, vp, vp, vp, f32, f32, f32, vp, sz, i64, vp, vp, i64, vp, vp, i64, vp],
+            "emr_stream_mode": [vp, vp, vp, vp, f32, f32, f32, i32, i32, vp, sz, i64, vp, vp, i64, vp, vp, i64, vp],
+            "emr_mask_combine_types": [vp, vp, vp, vp, i32, i32, i32, vp, vp],
+            "emr_conn_types": [vp, vp, vp, vp, i32, i64, vp, vp],
+            "emr_substrate_config": [i32, vp, vp],
             "emr_compact_workspace_size": [vp, i32, vp],
             "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_compact_records": [vp, vp, vp, vp, sz, vp, vp, vp, i64, vp, vp, vp, sz, vp],
@@ -247,12 +254,41 @@ def stream_workspace_size(pack, query: Query, grid: Grid, chunk_cap: int) -> int
 
 
 def stream(pack, pack_dev, query: Query, grid: Grid, theta: float, band: float, w_min: float, ws, chunk_cap: int,
-           h_idx, h_w, counts, offsets, timeout_ms: int = 0, stream=None):
-    """emr_stream: chunked eager discovery; lists land in the (pinned) host tensors h_idx / h_w."""
+           h_idx, h_w, counts, offsets, timeout_ms: int = 0, stream=None, mode: int = EMR_EAGER,
+           types: int = CONN_ALL):
+    """emr_stream (eager, every type) or emr_stream_mode: chunked discovery; lists land in the
+    (pinned) host tensors h_idx / h_w."""
     q = query.c
-    _check(lib().emr_stream(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min, _ptr(ws),
-                            C.c_size_t(ws.numel()), chunk_cap, _ptr(h_idx), _ptr(h_w), h_idx.numel(), _ptr(counts),
-                            _ptr(offsets), timeout_ms, _stream(stream)), "emr_stream")
+    if mode == EMR_EAGER and types == CONN_ALL:
+        _check(lib().emr_stream(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min, _ptr(ws),
+                                C.c_size_t(ws.numel()), chunk_cap, _ptr(h_idx), _ptr(h_w), h_idx.numel(),
+                                _ptr(counts), _ptr(offsets), timeout_ms, _stream(stream)), "emr_stream")
+        return
+    _check(lib().emr_stream_mode(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min, mode,
+                                 types, _ptr(ws), C.c_size_t(ws.numel()), chunk_cap, _ptr(h_idx), _ptr(h_w),
+                                 h_idx.numel(), _ptr(counts), _ptr(offsets), timeout_ms, _stream(stream)),
+           "emr_stream_mode")
+
+
+def mask_combine_types(split, band_bits, query: Query, grid: Grid, n_pairs: int, mode: int, types: int, mask,
+                       stream=None):
+    q = query.c
+    _check(lib().emr_mask_combine_types(_ptr(split), _ptr(band_bits), C.byref(q), C.byref(grid), n_pairs, mode,
+                                        types, _ptr(mask), _stream(stream)), "emr_mask_combine_types")
+
+
+def conn_types(idx, offsets, query: Query, grid: Grid, n_pairs: int, cap: int, type_out, stream=None):
+    """emr_conn_types: type code (0 F, 1 B, 2 L, 3 S) of every list entry into the device uint8 tensor."""
+    q = query.c
+    _check(lib().emr_conn_types(_ptr(idx), _ptr(offsets), C.byref(q), C.byref(grid), n_pairs, cap, _ptr(type_out),
+                                _stream(stream)), "emr_conn_types")
+
+
+def substrate_config(config: int):
+    """(enabled EMR_CONN_* bits, hidden-to-hidden rounds on) of a Section 6 substrate configuration."""
+    t, h = C.c_int32(), C.c_int32()
+    _check(lib().emr_substrate_config(config, C.byref(t), C.byref(h)), "emr_substrate_config")
+    return t.value, h.value
 
 
 def compact(mask, out, grid: Grid, n_pairs: int, idx, w, cap: int, counts, offsets, ws, stream=None):
@@ -295,7 +331,8 @@ class Discovery:
     """
 
     def __init__(self, pop, sources, D: int, theta: float, band: float, w_min: float = 0.0,
-                 mode: int = EMR_EAGER, cap: int | None = None, materialise: bool = False, device="cuda"):
+                 mode: int = EMR_EAGER, cap: int | None = None, materialise: bool = False, device="cuda",
+                 types: int = CONN_ALL):
         self.device = torch.device(device)
         self.pack = pack_population(pop)
         self.pack_dev = torch.from_numpy(self.pack).to(self.device)
@@ -303,7 +340,7 @@ class Discovery:
         self.grid = grid_build(D)
         self.P, self.S = pop.P, self.query.S
         self.n_pairs = self.P * self.S
-        self.theta, self.band, self.w_min, self.mode = theta, band, w_min, mode
+        self.theta, self.band, self.w_min, self.mode, self.types = theta, band, w_min, mode, types
         g = self.grid
         u32 = dict(dtype=torch.int32, device=self.device)
         self.mask = torch.zeros(self.n_pairs, g.n_words, **u32)
@@ -339,13 +376,27 @@ class Discovery:
             self._materialise()
         eval_filter(self.pack, self.query, self.grid, self.theta, self.band, self.w_min, self.split,
                     self.band_bits, self.out if sparse_out else None, self.ws, stream)
-        mask_combine(self.split, self.band_bits, self.grid, self.n_pairs, self.mode, self.mask, stream)
+        self.combine(stream)
         if sparse_out:
             compact(self.mask, self.out, self.grid, self.n_pairs, self.idx, self.w, self.cap, self.counts,
                     self.offsets, self.cws, stream)
         else:
             compact_records(self.mask, self.pack, self.query, self.ws, self.grid, self.idx, self.w, self.cap,
                             self.counts, self.offsets, self.cws, stream)
+
+    def combine(self, stream=None):
+        """emr_mask_combine, or emr_mask_combine_types when a connection-type filter is set."""
+        if self.types == CONN_ALL:
+            mask_combine(self.split, self.band_bits, self.grid, self.n_pairs, self.mode, self.mask, stream)
+        else:
+            mask_combine_types(self.split, self.band_bits, self.query, self.grid, self.n_pairs, self.mode,
+                               self.types, self.mask, stream)
+
+    def conn_types(self, stream=None):
+        """Type codes of the current lists (device uint8 tensor of cap entries)."""
+        t = torch.zeros(self.cap, dtype=torch.uint8, device=self.device)
+        conn_types(self.idx, self.offsets, self.query, self.grid, self.n_pairs, self.cap, t, stream)
+        return t
 
     def run_unfused(self, with_var: bool = False, stream=None):
         """emr_eval_prepare, emr_eval, emr_variance_filter, emr_compact."""
@@ -357,6 +408,8 @@ class Discovery:
         variance_filter(self.out, self.out_halo, self.grid, self.P, self.S, self.theta, self.band, self.w_min,
                         self.mode, self.mask, self.split, self.band_bits, self.var_dbg if with_var else None,
                         stream)
+        if self.types != CONN_ALL:
+            self.combine(stream)
         compact(self.mask, self.out, self.grid, self.n_pairs, self.idx, self.w, self.cap, self.counts,
                 self.offsets, self.cws, stream)
 

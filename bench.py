@@ -254,6 +254,47 @@ def streamed_run(emr, torch, w, chunk, chunk_cap, cap, reps, mode=0, types=15, l
             "timing": "host wall clock per emr_stream call (synchronous, lists on the host), median of %d" % reps}
 
 
+def networks_run(emr, torch, W, D=5, P=1000, config=None, reps=20):
+    """Substrate networks of the XOR population (c2 genomes, inputs (-1,-1), (1,-1), bias (0,-1),
+    output (0,1)): emr_assemble wall time, then emr_ann_forward on the four XOR patterns
+    (CUDA events, networks resident on the device)."""
+    config = emr.SUBSTRATE_HH if config is None else config
+    w = W.c2(D=D, P=P)
+    types, rounds = emr.substrate_config(config)
+    pack = emr.pack_population(w.pop)
+    pack_dev = torch.from_numpy(pack).cuda()
+    grid = emr.grid_build(D)
+    xor_in, xor_out = [(-1.0, -1.0), (1.0, -1.0), (0.0, -1.0)], [(0.0, 1.0)]
+    times = []
+    for k in range(3):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        nets = emr.assemble(pack, pack_dev, xor_in, xor_out, grid, w.theta, w.band, 0.0, emr.EMR_EAGER, types,
+                            rounds)
+        times.append(time.perf_counter() - t0)
+    t_asm = statistics.median(times[1:])
+    patterns = torch.tensor([[0, 0, 1], [0, 1, 1], [1, 0, 1], [1, 1, 1]], dtype=torch.float32, device="cuda")
+    steps = rounds + 2
+    out = emr.ann_forward(nets, patterns, steps)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        emr.ann_forward(nets, patterns, steps, out=out)
+    e1.record()
+    torch.cuda.synchronize()
+    t_fwd = e0.elapsed_time(e1) / 1e3 / reps
+    n_conn = int(nets.conn_off[-1])
+    return {"workload": "c2_xor_networks_pop%d_d%d_%s" % (P, D, ["feedforward", "hh", "backward", "lateral",
+                                                              "self", "full"][config]),
+            "assemble_seconds": t_asm, "networks_per_s": P / t_asm,
+            "hidden_nodes": int(nets.node_off[-1]), "connections": n_conn,
+            "forward_seconds": t_fwd, "forward_steps": steps, "patterns": 4,
+            "forward_connection_updates_per_s": n_conn * 4 * steps / t_fwd,
+            "timing": "assembly: host wall clock per emr_assemble call (all query rounds, lists to the host, "
+                      "pruning), median of 2 after one warm-up; forward: CUDA events, mean of %d" % reps}
+
+
 def launches_in_step(emr, dsc):
     """Kernel launches of one step: prepare (schedule, records), one tile launch per
     non-empty kernel class, mask combine, compaction (count, two scans, write, kept
@@ -441,7 +482,8 @@ def main():
                  "c4_round2_hh_d8": streamed_run(emr, torch, c4r2, 1 << 16, 1 << 24, 1 << 26, 3),
                  "c4_round2_hh_d8_backward_config": streamed_run(
                      emr, torch, c4r2, 1 << 16, 1 << 24, 1 << 26, 3,
-                     types=emr.substrate_config(emr.SUBSTRATE_BACKWARD)[0], label=c4r2.name + "_backward")}
+                     types=emr.substrate_config(emr.SUBSTRATE_BACKWARD)[0], label=c4r2.name + "_backward"),
+                 "xor_networks_hh_d5": networks_run(emr, torch, W)}
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:

@@ -370,6 +370,63 @@ emr_status emr_compact_records(const uint32_t *mask, const void *pack_host, cons
 emr_status emr_conn_types(const int32_t *idx, const int64_t *offsets, const emr_query *q, const emr_grid *grid,
                           int32_t n_pairs, int64_t cap, uint8_t *type, void *stream);
 
+/* ---- f2: network assembly and the substrate ANN ------------------------------ */
+
+/* Bytes of device workspace emr_assemble needs (query slots, per-pair records,
+ * the three bit planes, compaction workspace and list_cap list entries for
+ * max(slots_max, n_in + n_out) slots per genome). */
+emr_status emr_assemble_workspace_size(const void *pack_host, int32_t n_in, int32_t n_out, int32_t slots_max,
+                                       const emr_grid *grid, int64_t list_cap, size_t *bytes);
+
+/* Build each genome's substrate network (ES-HyperNEAT's construction, which
+ * Section 2 summarises and Section 6 configures) with the discovery path of
+ * this library for every query:
+ *   Phase 1: an outgoing query from each substrate input (in_x, in_y) connects
+ *            it to every position it keeps; those positions are hidden nodes.
+ *   Phase 2: `rounds` times, an outgoing query from each hidden node found in
+ *            the previous round connects it to its kept positions; new
+ *            positions join the hidden nodes (0 rounds: feedforward).
+ *   Phase 3: an incoming query toward each substrate output (out_x, out_y)
+ *            connects the hidden nodes among its kept positions to it.
+ *   Pruning: hidden nodes not reachable from an input or not reaching an
+ *            output are removed with their connections.
+ * Every query uses theta, band, w_min, mode and the connection-type filter
+ * types (EMR_CONN_* bits, see emr_substrate_config). Phase 2 queries at most
+ * slots_max hidden nodes of a genome at a time (more are taken in further
+ * batches); list_cap bounds the entries of one batch.
+ * Output (host arrays): genome g has hidden nodes hidden[node_off[g] ..
+ * node_off[g+1]) (global grid indices, ascending; emr_index_to_ij gives their
+ * coordinates) and connections [conn_off[g], conn_off[g+1]) with source and
+ * destination node numbers (inputs 0 .. n_in - 1, outputs n_in .. n_in +
+ * n_out - 1, hidden node k at n_in + n_out + k), weight (the CPPN output) and
+ * type code (0 forward, 1 backward, 2 lateral, 3 self), sorted by destination
+ * then source. Synchronous on `stream`.
+ * Errors: EMR_ERR_ARG; EMR_ERR_CAPACITY (workspace too small, a batch's lists
+ * exceed list_cap, or hidden_cap / conn_cap too small: node_off and conn_off
+ * then hold the true totals); errors of the discovery calls. */
+emr_status emr_assemble(const void *pack_host, const void *pack_dev, int32_t n_in, const float *in_x,
+                        const float *in_y, int32_t n_out, const float *out_x, const float *out_y,
+                        const emr_grid *grid, float theta, float band, float w_min, int32_t mode, int32_t types,
+                        int32_t rounds, int32_t slots_max, void *ws, size_t ws_bytes, int64_t list_cap,
+                        int64_t *node_off, int32_t *hidden, int64_t hidden_cap, int64_t *conn_off,
+                        int32_t *conn_src, int32_t *conn_dst, float *conn_w, uint8_t *conn_type,
+                        int64_t conn_cap, void *stream);
+
+/* Forward pass of P assembled networks on K input patterns (device arrays as
+ * emr_assemble writes them, copied to the device): input node i holds
+ * patterns[k * n_in + i]; every other node starts at 0 and `steps` times all
+ * take, at once, the sigmoid 1 / (1 + e^-z) of z = the weighted sum of their
+ * sources' previous values (the substrate network of an HyperNEAT-style
+ * indirect encoding, Section 2; recurrent connections make the result depend
+ * on steps). out[(g * K + k) * n_out + o] receives output o. max_hidden: the
+ * largest hidden-node count of a genome (sizes shared memory: the call fails
+ * with EMR_ERR_RANGE when 8 (n_in + n_out + max_hidden) K bytes do not fit).
+ * Errors: EMR_ERR_ARG, EMR_ERR_RANGE, EMR_ERR_CUDA. */
+emr_status emr_ann_forward(int32_t P, int32_t n_in, int32_t n_out, int32_t max_hidden, const int64_t *node_off,
+                           const int64_t *conn_off, const int32_t *conn_src, const int32_t *conn_dst,
+                           const float *conn_w, int32_t K, const float *patterns, int32_t steps, float *out,
+                           void *stream);
+
 /* ---- misc -------------------------------------------------------------------- */
 
 /* Static description of a status code. */

@@ -74,6 +74,10 @@ def lib() -> C.CDLL:
             "emr_mask_combine_types": [vp, vp, vp, vp, i32, i32, i32, vp, vp],
             "emr_conn_types": [vp, vp, vp, vp, i32, i64, vp, vp],
             "emr_substrate_config": [i32, vp, vp],
+            "emr_assemble_workspace_size": [vp, i32, i32, i32, vp, i64, vp],
+            "emr_assemble": [vp, vp, i32, vp, vp, i32, vp, vp, vp, f32, f32, f32, i32, i32, i32, i32, vp, sz, i64,
+                             vp, vp, i64, vp, vp, vp, vp, vp, i64, vp],
+            "emr_ann_forward": [i32, i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, i32, vp, vp],
             "emr_compact_workspace_size": [vp, i32, vp],
             "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_compact_records": [vp, vp, vp, vp, sz, vp, vp, vp, i64, vp, vp, vp, sz, vp],
@@ -304,6 +308,83 @@ def compact_records(mask, pack, query: Query, eval_ws, grid: Grid, idx, w, cap: 
                                      C.c_size_t(eval_ws.numel()), C.byref(grid), _ptr(idx), _ptr(w), cap,
                                      _ptr(counts), _ptr(offsets), _ptr(ws), C.c_size_t(ws.numel()),
                                      _stream(stream)), "emr_compact_records")
+
+
+# ---- network assembly and the substrate ANN ----------------------------------------------
+
+@dataclass
+class Networks:
+    """Assembled substrate networks (host arrays, layout of emr_assemble)."""
+    n_in: int
+    n_out: int
+    node_off: np.ndarray   # int64 [P + 1]
+    hidden: np.ndarray     # int32 global grid indices
+    conn_off: np.ndarray   # int64 [P + 1]
+    src: np.ndarray        # int32
+    dst: np.ndarray        # int32
+    w: np.ndarray          # float32
+    type: np.ndarray       # uint8
+    _dev: tuple | None = None  # device copies made by ann_forward
+
+    @property
+    def P(self) -> int:
+        return len(self.node_off) - 1
+
+    def genome(self, g: int):
+        """(hidden positions, src, dst, w, type) of genome g."""
+        h = self.hidden[self.node_off[g]:self.node_off[g + 1]]
+        c = slice(self.conn_off[g], self.conn_off[g + 1])
+        return h, self.src[c], self.dst[c], self.w[c], self.type[c]
+
+
+def assemble(pack, pack_dev, in_xy, out_xy, grid: Grid, theta: float, band: float, w_min: float = 0.0,
+             mode: int = EMR_EAGER, types: int = CONN_ALL, rounds: int = 1, slots_max: int = 256,
+             list_cap: int = 1 << 24, hidden_cap: int = 1 << 22, conn_cap: int = 1 << 24, stream=None) -> Networks:
+    """emr_assemble: substrate networks of every genome (device workspace allocated here)."""
+    in_xy = np.ascontiguousarray(in_xy, np.float32).reshape(-1, 2)
+    out_xy = np.ascontiguousarray(out_xy, np.float32).reshape(-1, 2)
+    ix, iy = np.ascontiguousarray(in_xy[:, 0]), np.ascontiguousarray(in_xy[:, 1])
+    ox, oy = np.ascontiguousarray(out_xy[:, 0]), np.ascontiguousarray(out_xy[:, 1])
+    n = C.c_size_t()
+    _check(lib().emr_assemble_workspace_size(_ptr(pack), len(ix), len(ox), slots_max, C.byref(grid), list_cap,
+                                             C.byref(n)), "emr_assemble_workspace_size")
+    ws = torch.empty(n.value, dtype=torch.uint8, device="cuda")
+    P = pack_info(pack)[0]
+    node_off = np.zeros(P + 1, np.int64)
+    conn_off = np.zeros(P + 1, np.int64)
+    hidden = np.zeros(hidden_cap, np.int32)
+    src = np.zeros(conn_cap, np.int32)
+    dst = np.zeros(conn_cap, np.int32)
+    w = np.zeros(conn_cap, np.float32)
+    ty = np.zeros(conn_cap, np.uint8)
+    _check(lib().emr_assemble(_ptr(pack), _ptr(pack_dev), len(ix), _ptr(ix), _ptr(iy), len(ox), _ptr(ox), _ptr(oy),
+                              C.byref(grid), theta, band, w_min, mode, types, rounds, slots_max, _ptr(ws),
+                              C.c_size_t(ws.numel()), list_cap, _ptr(node_off), _ptr(hidden), hidden_cap,
+                              _ptr(conn_off), _ptr(src), _ptr(dst), _ptr(w), _ptr(ty), conn_cap, _stream(stream)),
+           "emr_assemble")
+    nh, nc = int(node_off[-1]), int(conn_off[-1])
+    return Networks(len(ix), len(ox), node_off, hidden[:nh].copy(), conn_off, src[:nc].copy(), dst[:nc].copy(),
+                    w[:nc].copy(), ty[:nc].copy())
+
+
+def ann_forward(nets: Networks, patterns, steps: int, device="cuda", stream=None, out=None):
+    """emr_ann_forward: outputs [P, K, n_out] (device tensor) of every network on patterns [K, n_in].
+    The networks' arrays are copied to the device once and kept with them."""
+    dev = torch.device(device)
+    if getattr(nets, "_dev", None) is None or nets._dev[0] != dev:
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        nets._dev = (dev, t(nets.node_off), t(nets.conn_off), t(nets.src), t(nets.dst), t(nets.w))
+    _, node_off, conn_off, src, dst, w = nets._dev
+    pat = patterns if isinstance(patterns, torch.Tensor) else \
+        torch.as_tensor(np.ascontiguousarray(patterns, np.float32).reshape(-1, nets.n_in), device=dev)
+    K = pat.shape[0]
+    if out is None:
+        out = torch.zeros(nets.P, K, nets.n_out, dtype=torch.float32, device=dev)
+    max_hidden = int(np.max(np.diff(nets.node_off))) if nets.P else 0
+    _check(lib().emr_ann_forward(nets.P, nets.n_in, nets.n_out, max_hidden, _ptr(node_off), _ptr(conn_off),
+                                 _ptr(src), _ptr(dst), _ptr(w), K, _ptr(pat), steps, _ptr(out), _stream(stream)),
+           "emr_ann_forward")
+    return out
 
 
 # ---- ALU probes (roofline denominators) -------------------------------------------------

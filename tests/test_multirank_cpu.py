@@ -38,7 +38,7 @@ def _rank(rank, ws, port, out):
 
 def test_two_gloo_ranks_shard_populations_and_aggregate():
     ws = 2
-    mgr = mp.Manager()
+    mgr = mp.get_context("spawn").Manager()
     out = mgr.dict()
     mp.start_processes(_rank, args=(ws, _free_port(), out), nprocs=ws, start_method="spawn")
     r0, r1 = out[0], out[1]

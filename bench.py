@@ -273,6 +273,16 @@ def networks_run(emr, torch, W, D=5, P=1000, config=None, reps=20):
                             rounds)
         times.append(time.perf_counter() - t0)
     t_asm = statistics.median(times[1:])
+    cache = emr.Cache(8 << 30)
+    emr.assemble(pack, pack_dev, xor_in, xor_out, grid, w.theta, w.band, 0.0, emr.EMR_EAGER, types, rounds,
+                 cache=cache)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    emr.assemble(pack, pack_dev, xor_in, xor_out, grid, w.theta, w.band, 0.0, emr.EMR_EAGER, types, rounds,
+                 cache=cache)
+    t_cached = time.perf_counter() - t0
+    cst = cache.stats()
+    del cache
     patterns = torch.tensor([[0, 0, 1], [0, 1, 1], [1, 0, 1], [1, 1, 1]], dtype=torch.float32, device="cuda")
     steps = rounds + 2
     out = emr.ann_forward(nets, patterns, steps)
@@ -288,6 +298,7 @@ def networks_run(emr, torch, W, D=5, P=1000, config=None, reps=20):
     return {"workload": "c2_xor_networks_pop%d_d%d_%s" % (P, D, ["feedforward", "hh", "backward", "lateral",
                                                               "self", "full"][config]),
             "assemble_seconds": t_asm, "networks_per_s": P / t_asm,
+            "assemble_seconds_cached": t_cached, "cache": cst,
             "hidden_nodes": int(nets.node_off[-1]), "connections": n_conn,
             "forward_seconds": t_fwd, "forward_steps": steps, "patterns": 4,
             "forward_connection_updates_per_s": n_conn * 4 * steps / t_fwd,

@@ -372,6 +372,23 @@ emr_status emr_conn_types(const int32_t *idx, const int64_t *offsets, const emr_
 
 /* ---- f2: network assembly and the substrate ANN ------------------------------ */
 
+/* Connection cache (Section 7: cached hidden-to-hidden connections make later
+ * discovery nearly free). Caller-owned: lists discovered by emr_assemble are
+ * kept per (genome content, query slot, query parameters) and reused by later
+ * calls for identical genomes (an elite carried to the next generation, or a
+ * clone) and slots, up to max_bytes (least recently used entries go first). A
+ * genome is identified by its packed records, so any change to it misses.
+ * Reuse does not change results: the device path is deterministic. Not
+ * thread-safe: one call at a time per cache. */
+typedef struct emr_cache emr_cache;
+emr_status emr_cache_create(size_t max_bytes, emr_cache **cache);
+emr_status emr_cache_destroy(emr_cache *cache);
+emr_status emr_cache_clear(emr_cache *cache);
+/* Lookups that hit and missed since creation or the last clear, entries held
+ * and their bytes. Any output may be NULL. */
+emr_status emr_cache_stats(const emr_cache *cache, int64_t *hits, int64_t *misses, int64_t *entries,
+                           int64_t *bytes);
+
 /* Bytes of device workspace emr_assemble needs (query slots, per-pair records,
  * the three bit planes, compaction workspace and list_cap list entries for
  * max(slots_max, n_in + n_out) slots per genome). */
@@ -400,7 +417,8 @@ emr_status emr_assemble_workspace_size(const void *pack_host, int32_t n_in, int3
  * destination node numbers (inputs 0 .. n_in - 1, outputs n_in .. n_in +
  * n_out - 1, hidden node k at n_in + n_out + k), weight (the CPPN output) and
  * type code (0 forward, 1 backward, 2 lateral, 3 self), sorted by destination
- * then source. Synchronous on `stream`.
+ * then source. cache (optional, NULL for none): query results are looked up
+ * there first and added after. Synchronous on `stream`.
  * Errors: EMR_ERR_ARG; EMR_ERR_CAPACITY (workspace too small, a batch's lists
  * exceed list_cap, or hidden_cap / conn_cap too small: node_off and conn_off
  * then hold the true totals); errors of the discovery calls. */
@@ -410,7 +428,7 @@ emr_status emr_assemble(const void *pack_host, const void *pack_dev, int32_t n_i
                         int32_t rounds, int32_t slots_max, void *ws, size_t ws_bytes, int64_t list_cap,
                         int64_t *node_off, int32_t *hidden, int64_t hidden_cap, int64_t *conn_off,
                         int32_t *conn_src, int32_t *conn_dst, float *conn_w, uint8_t *conn_type,
-                        int64_t conn_cap, void *stream);
+                        int64_t conn_cap, emr_cache *cache, void *stream);
 
 /* Forward pass of P assembled networks on K input patterns (device arrays as
  * emr_assemble writes them, copied to the device): input node i holds

@@ -12,6 +12,9 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <list>
+#include <string>
+#include <thread>
 #include <unordered_map>
 #include <vector>
 
@@ -21,6 +24,23 @@
 namespace {
 
 inline size_t up256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// fn(g) for g in [0, n) on up to 16 host threads (genomes are independent).
+template <class F>
+void parallel_for(int32_t n, F fn) {
+  const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
+  const int nt = n >= 64 ? std::min(hw, 16) : 1;
+  if (nt == 1) {
+    for (int32_t g = 0; g < n; g++) fn(g);
+    return;
+  }
+  std::vector<std::thread> pool;
+  for (int t = 0; t < nt; t++)
+    pool.emplace_back([&, t] {
+      for (int32_t g = int32_t(int64_t(n) * t / nt); g < int32_t(int64_t(n) * (t + 1) / nt); g++) fn(g);
+    });
+  for (auto& th : pool) th.join();
+}
 
 // Device workspace carve-up for one query batch of up to n_pairs pairs.
 struct AsmLayout {
@@ -168,6 +188,163 @@ struct Runner {
   }
 };
 
+// ---- connection cache --------------------------------------------------------------
+//
+// Discovered lists keyed by (genome content, query slot, query parameters). A
+// genome is identified by the bytes of its packed records, so an identical
+// genome in a later population (an elite, or a clone) hits; entries are evicted
+// least recently used beyond the byte budget.
+
+struct SlotKey {
+  int64_t genome;  // id in the cache's genome table
+  uint32_t a, b;   // slot coordinates (fp32 bits)
+  int32_t side, D, mode, types;
+  uint32_t theta, band, w_min;
+  bool operator==(const SlotKey& o) const { return std::memcmp(this, &o, sizeof(SlotKey)) == 0; }
+};
+struct SlotKeyHash {
+  size_t operator()(const SlotKey& k) const {
+    const auto* p = reinterpret_cast<const uint8_t*>(&k);
+    uint64_t h = 1469598103934665603ull;  // FNV-1a
+    for (size_t i = 0; i < sizeof(SlotKey); i++) h = (h ^ p[i]) * 1099511628211ull;
+    return size_t(h);
+  }
+};
+
+struct List {
+  std::vector<int32_t> idx;
+  std::vector<float> w;
+};
+
+struct Slot {
+  float a, b;
+  int32_t side;
+};
+
+}  // namespace
+
+struct emr_cache {
+  size_t max_bytes = 0, bytes = 0;
+  int64_t hits = 0, misses = 0;
+  std::unordered_map<std::string, int64_t> genomes;
+  std::list<SlotKey> lru;  // most recent first
+  struct Entry {
+    std::list<SlotKey>::iterator at;
+    List list;
+  };
+  std::unordered_map<SlotKey, Entry, SlotKeyHash> map;
+
+  static size_t cost(const List& l) { return l.idx.size() * 8 + sizeof(Entry) + sizeof(SlotKey) + 64; }
+  bool get(const SlotKey& k, List* out) {
+    auto it = map.find(k);
+    if (it == map.end()) { misses++; return false; }
+    hits++;
+    lru.splice(lru.begin(), lru, it->second.at);
+    *out = it->second.list;
+    return true;
+  }
+  void put(const SlotKey& k, const List& l) {
+    if (map.count(k)) return;
+    const size_t c = cost(l);
+    if (c > max_bytes) return;
+    while (bytes + c > max_bytes && !lru.empty()) {
+      auto it = map.find(lru.back());
+      bytes -= cost(it->second.list);
+      map.erase(it);
+      lru.pop_back();
+    }
+    lru.push_front(k);
+    map.emplace(k, Entry{lru.begin(), l});
+    bytes += c;
+  }
+};
+
+namespace {
+
+// Content identity of genome g of a packed blob: its kept node and edge records.
+std::string genome_bytes(const void* pack_host, int32_t g) {
+  const auto* base = static_cast<const uint8_t*>(pack_host);
+  const auto* h = emr::pack_header(pack_host);
+  const auto* gt = reinterpret_cast<const emr::PackGenome*>(base + h->off_genomes) + g;
+  std::string s;
+  s.append(reinterpret_cast<const char*>(&gt->n_nodes), 4);
+  s.append(reinterpret_cast<const char*>(base + h->off_nodes) + size_t(gt->node_beg) * sizeof(emr::PackNode),
+           size_t(gt->n_nodes) * sizeof(emr::PackNode));
+  s.append(reinterpret_cast<const char*>(base + h->off_edges) + size_t(gt->edge_beg) * sizeof(emr::PackEdge),
+           size_t(gt->n_edges) * sizeof(emr::PackEdge));
+  return s;
+}
+
+uint32_t bits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  return u;
+}
+
+// Lists of every genome's slots (slots[g]): from the cache where present, the
+// rest from the device in batches of at most slots_max slots per genome, then
+// added to the cache.
+emr_status query_slots(Runner& R, emr_cache* cache, const std::vector<int64_t>& gid, int32_t D,
+                       const std::vector<std::vector<Slot>>& slots, int32_t slots_max,
+                       std::vector<std::vector<List>>& out) {
+  const int32_t P = R.P;
+  auto key = [&](int32_t g, const Slot& sl) {
+    SlotKey k;
+    std::memset(&k, 0, sizeof(k));
+    k.genome = gid[size_t(g)];
+    k.a = bits(sl.a);
+    k.b = bits(sl.b);
+    k.side = sl.side;
+    k.D = D;
+    k.mode = R.mode;
+    k.types = R.types;
+    k.theta = bits(R.theta);
+    k.band = bits(R.band);
+    k.w_min = bits(R.w_min);
+    return k;
+  };
+  out.assign(size_t(P), {});
+  std::vector<std::vector<int32_t>> miss(static_cast<size_t>(P));
+  for (int32_t g = 0; g < P; g++) {
+    out[size_t(g)].resize(slots[size_t(g)].size());
+    for (size_t k = 0; k < slots[size_t(g)].size(); k++)
+      if (!cache || !cache->get(key(g, slots[size_t(g)][k]), &out[size_t(g)][k]))
+        miss[size_t(g)].push_back(int32_t(k));
+  }
+  std::vector<size_t> cursor(static_cast<size_t>(P), 0);
+  for (;;) {
+    int32_t S = 0;
+    for (int32_t g = 0; g < P; g++)
+      S = std::max<int32_t>(S, int32_t(std::min<size_t>(size_t(slots_max), miss[size_t(g)].size() - cursor[size_t(g)])));
+    if (S == 0) return EMR_OK;
+    std::vector<float> a(size_t(P) * S, 0.f), b(size_t(P) * S, 0.f);
+    std::vector<int32_t> side(size_t(P) * S, EMR_SIDE_OUT), count(static_cast<size_t>(P), 0);
+    for (int32_t g = 0; g < P; g++) {
+      const int32_t n = int32_t(std::min<size_t>(size_t(S), miss[size_t(g)].size() - cursor[size_t(g)]));
+      count[size_t(g)] = n;
+      for (int32_t s = 0; s < n; s++) {
+        const Slot& sl = slots[size_t(g)][size_t(miss[size_t(g)][cursor[size_t(g)] + size_t(s)])];
+        a[size_t(g) * S + s] = sl.a;
+        b[size_t(g) * S + s] = sl.b;
+        side[size_t(g) * S + s] = sl.side;
+      }
+    }
+    emr_status rc = R.run(S, 1, a, b, side, count);
+    if (rc != EMR_OK) return rc;
+    for (int32_t g = 0; g < P; g++) {
+      for (int32_t s = 0; s < count[size_t(g)]; s++) {
+        const int32_t k = miss[size_t(g)][cursor[size_t(g)] + size_t(s)];
+        const int64_t r = int64_t(g) * S + s;
+        List& l = out[size_t(g)][size_t(k)];
+        l.idx.assign(R.idx.begin() + R.offsets[size_t(r)], R.idx.begin() + R.offsets[size_t(r) + 1]);
+        l.w.assign(R.w.begin() + R.offsets[size_t(r)], R.w.begin() + R.offsets[size_t(r) + 1]);
+        if (cache) cache->put(key(g, slots[size_t(g)][size_t(k)]), l);
+      }
+      cursor[size_t(g)] += size_t(count[size_t(g)]);
+    }
+  }
+}
+
 }  // namespace
 
 extern "C" {
@@ -189,7 +366,8 @@ emr_status emr_assemble(const void* pack_host, const void* pack_dev, int32_t n_i
                         const emr_grid* grid, float theta, float band, float w_min, int32_t mode, int32_t types,
                         int32_t rounds, int32_t slots_max, void* ws, size_t ws_bytes, int64_t list_cap,
                         int64_t* node_off, int32_t* hidden, int64_t hidden_cap, int64_t* conn_off, int32_t* conn_src,
-                        int32_t* conn_dst, float* conn_w, uint8_t* conn_type_out, int64_t conn_cap, void* stream) {
+                        int32_t* conn_dst, float* conn_w, uint8_t* conn_type_out, int64_t conn_cap, emr_cache* cache,
+                        void* stream) {
   if (!pack_dev || !ws || n_in <= 0 || n_out <= 0 || !in_x || !in_y || !out_x || !out_y || rounds < 0 ||
       slots_max <= 0 || list_cap <= 0 || !node_off || !conn_off || hidden_cap < 0 || conn_cap < 0 ||
       (hidden_cap > 0 && !hidden) || (conn_cap > 0 && (!conn_src || !conn_dst || !conn_w || !conn_type_out)))
@@ -205,91 +383,79 @@ emr_status emr_assemble(const void* pack_host, const void* pack_dev, int32_t n_i
   if (ws_bytes < R.L.total) return EMR_ERR_CAPACITY;
   std::vector<GenomeGraph> G(static_cast<size_t>(P));
 
+  std::vector<int64_t> gid(static_cast<size_t>(P), 0);
+  if (cache)
+    for (int32_t g = 0; g < P; g++)
+      gid[size_t(g)] = cache->genomes.emplace(genome_bytes(pack_host, g), int64_t(cache->genomes.size())).first->second;
+
   // Phase 1 and the queries of Phase 3: outgoing from each input, incoming to each output
   {
-    const int32_t S = n_in + n_out;
-    std::vector<float> a(static_cast<size_t>(S)), b(static_cast<size_t>(S));
-    std::vector<int32_t> side(static_cast<size_t>(S)), count;
-    for (int32_t k = 0; k < n_in; k++) { a[size_t(k)] = in_x[k]; b[size_t(k)] = in_y[k]; side[size_t(k)] = EMR_SIDE_OUT; }
-    for (int32_t k = 0; k < n_out; k++) {
-      a[size_t(n_in + k)] = out_x[k];
-      b[size_t(n_in + k)] = out_y[k];
-      side[size_t(n_in + k)] = EMR_SIDE_IN;
-    }
-    if ((rc = R.run(S, 0, a, b, side, count)) != EMR_OK) return rc;
-    for (int32_t g = 0; g < P; g++) {
+    std::vector<Slot> io;
+    for (int32_t k = 0; k < n_in; k++) io.push_back({in_x[k], in_y[k], EMR_SIDE_OUT});
+    for (int32_t k = 0; k < n_out; k++) io.push_back({out_x[k], out_y[k], EMR_SIDE_IN});
+    std::vector<std::vector<Slot>> slots(static_cast<size_t>(P), io);
+    std::vector<std::vector<List>> lists;
+    if ((rc = query_slots(R, cache, gid, grid->D, slots, n_in + n_out, lists)) != EMR_OK) return rc;
+    parallel_for(P, [&](int32_t g) {
       GenomeGraph& gg = G[size_t(g)];
-      for (int32_t s = 0; s < S; s++) {
-        const int64_t r = int64_t(g) * S + s;
-        for (int64_t e = R.offsets[size_t(r)]; e < R.offsets[size_t(r) + 1]; e++) {
-          const int64_t p = R.idx[size_t(e)];
+      for (int32_t s = 0; s < n_in + n_out; s++) {
+        const List& l = lists[size_t(g)][size_t(s)];
+        for (size_t e = 0; e < l.idx.size(); e++) {
+          const int64_t p = l.idx[e];
           float x, y;
           coords(p, &x, &y);
           if (s < n_in) {
-            gg.conns.push_back({-1 - s, p, R.w[size_t(e)], conn_type(in_x[s], in_y[s], x, y)});
+            gg.conns.push_back({-1 - s, p, l.w[e], conn_type(in_x[s], in_y[s], x, y)});
             if (gg.seen.emplace(p, int32_t(gg.hidden.size())).second) gg.hidden.push_back(p);
           } else {
             const int32_t o = s - n_in;
-            gg.to_outputs.push_back({p, -1 - (n_in + o), R.w[size_t(e)], conn_type(x, y, out_x[o], out_y[o])});
+            gg.to_outputs.push_back({p, -1 - (n_in + o), l.w[e], conn_type(x, y, out_x[o], out_y[o])});
           }
         }
       }
       gg.frontier_beg = 0;
       gg.frontier_end = gg.hidden.size();
-    }
+    });
   }
 
   // Phase 2: outgoing queries from each newly discovered hidden node, `rounds` times
   for (int32_t round = 0; round < rounds; round++) {
-    std::vector<size_t> next_end(static_cast<size_t>(P));
-    std::vector<size_t> cursor(static_cast<size_t>(P));
-    for (int32_t g = 0; g < P; g++) cursor[size_t(g)] = G[size_t(g)].frontier_beg;
-    for (;;) {  // batches of at most slots_max sources per genome
-      int32_t S = 0;
-      for (int32_t g = 0; g < P; g++)
-        S = std::max<int32_t>(S, int32_t(std::min<size_t>(size_t(slots_max),
-                                                          G[size_t(g)].frontier_end - cursor[size_t(g)])));
-      if (S == 0) break;
-      std::vector<float> a(size_t(P) * S, 0.f), b(size_t(P) * S, 0.f);
-      std::vector<int32_t> side(size_t(P) * S, EMR_SIDE_OUT), count(static_cast<size_t>(P), 0);
-      for (int32_t g = 0; g < P; g++) {
-        const GenomeGraph& gg = G[size_t(g)];
-        const int32_t n = int32_t(std::min<size_t>(size_t(S), gg.frontier_end - cursor[size_t(g)]));
-        count[size_t(g)] = n;
-        for (int32_t s = 0; s < n; s++)
-          coords(gg.hidden[cursor[size_t(g)] + size_t(s)], &a[size_t(g) * S + s], &b[size_t(g) * S + s]);
+    std::vector<std::vector<Slot>> slots(static_cast<size_t>(P));
+    parallel_for(P, [&](int32_t g) {
+      const GenomeGraph& gg = G[size_t(g)];
+      for (size_t h = gg.frontier_beg; h < gg.frontier_end; h++) {
+        Slot sl{0.f, 0.f, EMR_SIDE_OUT};
+        coords(gg.hidden[h], &sl.a, &sl.b);
+        slots[size_t(g)].push_back(sl);
       }
-      if ((rc = R.run(S, 1, a, b, side, count)) != EMR_OK) return rc;
-      for (int32_t g = 0; g < P; g++) {
-        GenomeGraph& gg = G[size_t(g)];
-        for (int32_t s = 0; s < count[size_t(g)]; s++) {
-          const int64_t src = gg.hidden[cursor[size_t(g)] + size_t(s)];
-          const float xs = a[size_t(g) * S + s], ys = b[size_t(g) * S + s];
-          const int64_t r = int64_t(g) * S + s;
-          for (int64_t e = R.offsets[size_t(r)]; e < R.offsets[size_t(r) + 1]; e++) {
-            const int64_t p = R.idx[size_t(e)];
-            float x, y;
-            coords(p, &x, &y);
-            gg.conns.push_back({src, p, R.w[size_t(e)], conn_type(xs, ys, x, y)});
-            if (gg.seen.emplace(p, int32_t(gg.hidden.size())).second) gg.hidden.push_back(p);
-          }
-        }
-        cursor[size_t(g)] += size_t(count[size_t(g)]);
-      }
-    }
-    for (int32_t g = 0; g < P; g++) {
+    });
+    std::vector<std::vector<List>> lists;
+    if ((rc = query_slots(R, cache, gid, grid->D, slots, slots_max, lists)) != EMR_OK) return rc;
+    parallel_for(P, [&](int32_t g) {
       GenomeGraph& gg = G[size_t(g)];
+      for (size_t k = 0; k < slots[size_t(g)].size(); k++) {
+        const int64_t src = gg.hidden[gg.frontier_beg + k];
+        const Slot& sl = slots[size_t(g)][k];
+        const List& l = lists[size_t(g)][k];
+        for (size_t e = 0; e < l.idx.size(); e++) {
+          const int64_t p = l.idx[e];
+          float x, y;
+          coords(p, &x, &y);
+          gg.conns.push_back({src, p, l.w[e], conn_type(sl.a, sl.b, x, y)});
+          if (gg.seen.emplace(p, int32_t(gg.hidden.size())).second) gg.hidden.push_back(p);
+        }
+      }
       gg.frontier_beg = gg.frontier_end;
       gg.frontier_end = gg.hidden.size();
-    }
+    });
   }
 
   // Phase 3 and pruning; nodes are numbered inputs, outputs, then kept hidden
   // positions in ascending global index; connections sorted by (dst, src)
-  int64_t n_hidden_total = 0, n_conn_total = 0;
-  node_off[0] = 0;
-  conn_off[0] = 0;
-  for (int32_t g = 0; g < P; g++) {
+  struct Out { int32_t src, dst; float w; uint8_t t; };
+  std::vector<std::vector<int64_t>> kept_of(static_cast<size_t>(P));
+  std::vector<std::vector<Out>> out_of(static_cast<size_t>(P));
+  parallel_for(P, [&](int32_t g) {
     GenomeGraph& gg = G[size_t(g)];
     for (const Conn& c : gg.to_outputs)
       if (gg.seen.count(c.src)) gg.conns.push_back(c);
@@ -324,8 +490,7 @@ emr_status emr_assemble(const void* pack_host, const void* pack_dev, int32_t n_i
       auto it = id.find(v);
       return it == id.end() ? -1 : it->second;
     };
-    struct Out { int32_t src, dst; float w; uint8_t t; };
-    std::vector<Out> outc;
+    std::vector<Out>& outc = out_of[size_t(g)];
     for (const Conn& c : gg.conns) {
       const int32_t s = new_id(c.src), d = new_id(c.dst);
       if (s >= 0 && d >= 0) outc.push_back({s, d, c.w, c.type});
@@ -333,6 +498,15 @@ emr_status emr_assemble(const void* pack_host, const void* pack_dev, int32_t n_i
     std::sort(outc.begin(), outc.end(), [](const Out& x, const Out& y) {
       return x.dst != y.dst ? x.dst < y.dst : x.src < y.src;
     });
+    kept_of[size_t(g)] = std::move(kept);
+    gg = GenomeGraph();  // release the graph early
+  });
+  int64_t n_hidden_total = 0, n_conn_total = 0;
+  node_off[0] = 0;
+  conn_off[0] = 0;
+  for (int32_t g = 0; g < P; g++) {
+    const std::vector<int64_t>& kept = kept_of[size_t(g)];
+    const std::vector<Out>& outc = out_of[size_t(g)];
     for (size_t k = 0; k < kept.size(); k++, n_hidden_total++)
       if (n_hidden_total < hidden_cap) hidden[n_hidden_total] = int32_t(kept[k]);
     for (size_t k = 0; k < outc.size(); k++, n_conn_total++)
@@ -346,6 +520,41 @@ emr_status emr_assemble(const void* pack_host, const void* pack_dev, int32_t n_i
     conn_off[g + 1] = n_conn_total;
   }
   return (n_hidden_total > hidden_cap || n_conn_total > conn_cap) ? EMR_ERR_CAPACITY : EMR_OK;
+}
+
+emr_status emr_cache_create(size_t max_bytes, emr_cache** cache) {
+  if (!cache) return EMR_ERR_ARG;
+  *cache = nullptr;
+  try {
+    *cache = new emr_cache();
+  } catch (...) {
+    return EMR_ERR_ALLOC;
+  }
+  (*cache)->max_bytes = max_bytes;
+  return EMR_OK;
+}
+
+emr_status emr_cache_destroy(emr_cache* cache) {
+  delete cache;
+  return EMR_OK;
+}
+
+emr_status emr_cache_clear(emr_cache* cache) {
+  if (!cache) return EMR_ERR_ARG;
+  const size_t mb = cache->max_bytes;
+  *cache = emr_cache();
+  cache->max_bytes = mb;
+  return EMR_OK;
+}
+
+emr_status emr_cache_stats(const emr_cache* cache, int64_t* hits, int64_t* misses, int64_t* entries,
+                           int64_t* bytes) {
+  if (!cache) return EMR_ERR_ARG;
+  if (hits) *hits = cache->hits;
+  if (misses) *misses = cache->misses;
+  if (entries) *entries = int64_t(cache->map.size());
+  if (bytes) *bytes = int64_t(cache->bytes);
+  return EMR_OK;
 }
 
 }  // extern "C"

@@ -76,7 +76,11 @@ def lib() -> C.CDLL:
             "emr_substrate_config": [i32, vp, vp],
             "emr_assemble_workspace_size": [vp, i32, i32, i32, vp, i64, vp],
             "emr_assemble": [vp, vp, i32, vp, vp, i32, vp, vp, vp, f32, f32, f32, i32, i32, i32, i32, vp, sz, i64,
-                             vp, vp, i64, vp, vp, vp, vp, vp, i64, vp],
+                             vp, vp, i64, vp, vp, vp, vp, vp, i64, vp, vp],
+            "emr_cache_create": [sz, vp],
+            "emr_cache_destroy": [vp],
+            "emr_cache_clear": [vp],
+            "emr_cache_stats": [vp, vp, vp, vp, vp],
             "emr_ann_forward": [i32, i32, i32, i32, vp, vp, vp, vp, vp, i32, vp, i32, vp, vp],
             "emr_compact_workspace_size": [vp, i32, vp],
             "emr_compact": [vp, vp, vp, i32, vp, vp, i64, vp, vp, vp, sz, vp],
@@ -337,9 +341,32 @@ class Networks:
         return h, self.src[c], self.dst[c], self.w[c], self.type[c]
 
 
+class Cache:
+    """emr_cache: connection lists reused across emr_assemble calls (owned handle)."""
+
+    def __init__(self, max_bytes: int = 1 << 30):
+        h = C.c_void_p()
+        _check(lib().emr_cache_create(max_bytes, C.byref(h)), "emr_cache_create")
+        self.handle = h
+
+    def stats(self):
+        v = [C.c_int64() for _ in range(4)]
+        _check(lib().emr_cache_stats(self.handle, *[C.byref(x) for x in v]), "emr_cache_stats")
+        return dict(zip(("hits", "misses", "entries", "bytes"), (x.value for x in v)))
+
+    def clear(self):
+        _check(lib().emr_cache_clear(self.handle), "emr_cache_clear")
+
+    def __del__(self):
+        if getattr(self, "handle", None) and _lib is not None:
+            _lib.emr_cache_destroy(self.handle)
+            self.handle = None
+
+
 def assemble(pack, pack_dev, in_xy, out_xy, grid: Grid, theta: float, band: float, w_min: float = 0.0,
              mode: int = EMR_EAGER, types: int = CONN_ALL, rounds: int = 1, slots_max: int = 256,
-             list_cap: int = 1 << 24, hidden_cap: int = 1 << 22, conn_cap: int = 1 << 24, stream=None) -> Networks:
+             list_cap: int = 1 << 24, hidden_cap: int = 1 << 22, conn_cap: int = 1 << 24, stream=None,
+             cache: Cache | None = None) -> Networks:
     """emr_assemble: substrate networks of every genome (device workspace allocated here)."""
     in_xy = np.ascontiguousarray(in_xy, np.float32).reshape(-1, 2)
     out_xy = np.ascontiguousarray(out_xy, np.float32).reshape(-1, 2)
@@ -360,7 +387,8 @@ def assemble(pack, pack_dev, in_xy, out_xy, grid: Grid, theta: float, band: floa
     _check(lib().emr_assemble(_ptr(pack), _ptr(pack_dev), len(ix), _ptr(ix), _ptr(iy), len(ox), _ptr(ox), _ptr(oy),
                               C.byref(grid), theta, band, w_min, mode, types, rounds, slots_max, _ptr(ws),
                               C.c_size_t(ws.numel()), list_cap, _ptr(node_off), _ptr(hidden), hidden_cap,
-                              _ptr(conn_off), _ptr(src), _ptr(dst), _ptr(w), _ptr(ty), conn_cap, _stream(stream)),
+                              _ptr(conn_off), _ptr(src), _ptr(dst), _ptr(w), _ptr(ty), conn_cap,
+                              cache.handle if cache is not None else None, _stream(stream)),
            "emr_assemble")
     nh, nc = int(node_off[-1]), int(conn_off[-1])
     return Networks(len(ix), len(ox), node_off, hidden[:nh].copy(), conn_off, src[:nc].copy(), dst[:nc].copy(),

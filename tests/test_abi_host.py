@@ -169,3 +169,11 @@ def test_workload_populations_pack(cfg):
     assert oracle.check_population(w.pop) == (0, -1)
     _, gs, _ = _pack_records(blob)
     assert gs["n_varying"].max() <= 64 and gs["n_vedges"].max() <= 512
+
+
+def test_cache_handle_host_only():
+    c = emr.Cache(1 << 20)
+    assert c.stats() == {"hits": 0, "misses": 0, "entries": 0, "bytes": 0}
+    c.clear()
+    assert c.stats()["entries"] == 0
+    del c

@@ -82,3 +82,65 @@ def test_forward_many_networks_and_steps():
             h, s, d, w, t = nets.genome(g)
             ref = A.forward(3, 1, h, list(zip(s, d, w.astype(np.float64), t)), pats, steps)
             assert np.all(np.abs(out[g] - ref) <= 2e-6), "genome %d steps %d" % (g, steps)
+
+
+def same_networks(a, b):
+    for f in ("node_off", "hidden", "conn_off", "src", "dst", "type"):
+        assert np.array_equal(getattr(a, f), getattr(b, f)), f
+    assert np.array_equal(a.w.view(np.uint32), b.w.view(np.uint32))
+
+
+def test_cache_reuses_lists_without_changing_networks():
+    pop = W.random_population(24, seed=79)
+    pack = emr.pack_population(pop)
+    pack_dev = torch.from_numpy(pack).cuda()
+    g = emr.grid_build(5)
+    args = (pack, pack_dev, XOR_IN, XOR_OUT, g, 0.03, 0.3, 0.0, emr.EMR_EAGER, emr.CONN_ALL, 2, 32)
+    ref = emr.assemble(*args)
+    cache = emr.Cache()
+    first = emr.assemble(*args, cache=cache)
+    s1 = cache.stats()
+    # genomes that pack to the same records share keys: entries can be fewer than misses
+    assert s1["hits"] == 0 and s1["misses"] >= s1["entries"] > 24 * 4
+    second = emr.assemble(*args, cache=cache)
+    s2 = cache.stats()
+    assert s2["misses"] == s1["misses"] and s2["hits"] == s1["misses"]   # every query hit
+    same_networks(ref, first)
+    same_networks(ref, second)
+    # a later population sharing half its genomes hits for those genomes' queries only
+    shared = list(range(12, 24))
+    pop2 = W.population_from_lists([pop.genome(k) for k in shared] +
+                                   [W.random_population(12, seed=80).genome(k) for k in range(12)])
+    pack2 = emr.pack_population(pop2)
+    nets2 = emr.assemble(pack2, torch.from_numpy(pack2).cuda(), XOR_IN, XOR_OUT, g, 0.03, 0.3, 0.0, emr.EMR_EAGER,
+                         emr.CONN_ALL, 2, 32, cache=cache)
+    s3 = cache.stats()
+    ref2 = emr.assemble(pack2, torch.from_numpy(pack2).cuda(), XOR_IN, XOR_OUT, g, 0.03, 0.3, 0.0, emr.EMR_EAGER,
+                        emr.CONN_ALL, 2, 32)
+    same_networks(ref2, nets2)
+    for k in range(12):   # the shared genomes' networks are those of the first population
+        a, b = nets2.genome(k), ref.genome(shared[k])
+        for x, y in zip(a, b):
+            assert np.array_equal(x, y)
+    # at least the shared genomes' four phase-1/3 slots hit; the new genomes miss
+    assert s3["hits"] - s2["hits"] >= 12 * 4 and s3["misses"] > s2["misses"]
+    # a different parameter is a different key
+    emr.assemble(pack, pack_dev, XOR_IN, XOR_OUT, g, 0.03, 0.31, 0.0, emr.EMR_EAGER, emr.CONN_ALL, 2, 32,
+                 cache=cache)
+    assert cache.stats()["misses"] > s3["misses"]
+
+
+def test_cache_budget_evicts_but_keeps_results():
+    pop = W.random_population(16, seed=81)
+    pack = emr.pack_population(pop)
+    pack_dev = torch.from_numpy(pack).cuda()
+    g = emr.grid_build(5)
+    args = (pack, pack_dev, XOR_IN, XOR_OUT, g, 0.03, 0.3, 0.0, emr.EMR_EAGER, emr.CONN_F, 1, 64)
+    ref = emr.assemble(*args)
+    cache = emr.Cache(max_bytes=64 << 10)
+    for _ in range(3):
+        same_networks(ref, emr.assemble(*args, cache=cache))
+        st = cache.stats()
+        assert st["bytes"] <= 64 << 10
+    cache.clear()
+    assert cache.stats() == {"hits": 0, "misses": 0, "entries": 0, "bytes": 0}

@@ -308,16 +308,15 @@ def networks_run(emr, torch, W, D=5, P=1000, config=None, reps=20):
 
 def launches_in_step(emr, dsc):
     """Kernel launches of one step: prepare (schedule, records), one tile launch per
-    non-empty kernel class, mask combine, compaction (count, two scans, write, kept
-    weights); combine, count and write launch once per 65535 pairs."""
+    non-empty kernel class, selection (count, scan, write with the kept weights); the
+    tile flags' memset is not a kernel."""
     _, gs, _, _ = emr.pack_records(dsc.pack)
     side = np.asarray(dsc.query.side)
     nv = gs["n_varying"][:, side] if not dsc.query.per_genome else \
         np.take_along_axis(gs["n_varying"], side.reshape(gs.shape[0], -1), axis=1)
     nv = nv.astype(np.int64)
     cls = np.where(nv > 12, 0, np.where(nv > 8, 1, np.where(nv > 4, 2, 3)))
-    groups = -(-dsc.n_pairs // 65535)
-    return 2 + len(np.unique(cls)) + groups + 2 * groups + 3
+    return 2 + len(np.unique(cls)) + 3
 
 
 def oracle_baseline(w, genomes):
@@ -384,18 +383,18 @@ def main():
     flush = torch.empty(64 << 20, dtype=torch.float32, device="cuda")  # 256 MB > 129 MB L2
 
     ev = lambda: torch.cuda.Event(enable_timing=True)
+    tile_flags = torch.zeros(dsc.n_pairs, emr.dense_tiles(w.D), dtype=torch.uint8, device="cuda")
 
     def step(evs=None):
         dsc.prepare()
         if evs:
             evs[0].record(stream)
-        emr.eval_filter(dsc.pack, dsc.query, g, dsc.theta, dsc.band, dsc.w_min, dsc.split, dsc.band_bits, None,
-                        dsc.ws)
+        emr.eval_filter_tiles(dsc.pack, dsc.query, g, dsc.theta, dsc.band, dsc.w_min, dsc.split, dsc.band_bits,
+                              tile_flags, dsc.ws)
         if evs:
             evs[1].record(stream)
-        emr.mask_combine(dsc.split, dsc.band_bits, g, dsc.n_pairs, dsc.mode, dsc.mask)
-        emr.compact_records(dsc.mask, dsc.pack, dsc.query, dsc.ws, g, dsc.idx, dsc.w, dsc.cap, dsc.counts,
-                            dsc.offsets, dsc.cws)
+        emr.select(dsc.split, dsc.band_bits, tile_flags, dsc.pack, dsc.query, dsc.ws, g, dsc.mode, dsc.types,
+                   dsc.idx, dsc.w, dsc.cap, dsc.counts, dsc.offsets)
 
     launches_per_step = launches_in_step(emr, dsc)
     for _ in range(args.warmup):

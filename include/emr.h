@@ -361,6 +361,27 @@ emr_status emr_compact_records(const uint32_t *mask, const void *pack_host, cons
                                size_t eval_ws_bytes, const emr_grid *grid, int32_t *idx, float *w, int64_t cap,
                                int64_t *counts, int64_t *offsets, void *ws, size_t ws_bytes, void *stream);
 
+/* emr_eval_filter (without the output buffer) that also flags, per pair and
+ * dense tile, whether any band bit is set: tile_flags is device uint8
+ * [n_pairs][n_dense], 1 where the tile holds a band-passing position, else 0.
+ * Dense tiles: tile 0 holds depths 0..min(D, 4); tile t >= 1 is the t-th 64 x 64
+ * Morton block of depths 5..D in global-index order (n_dense = 1 + the number of
+ * such blocks). For emr_select. Errors as emr_eval_filter. */
+emr_status emr_eval_filter_tiles(const void *pack_host, const emr_query *q, const emr_grid *grid, float theta,
+                                 float band, float w_min, uint32_t *split, uint32_t *band_bits,
+                                 uint8_t *tile_flags, void *ws, size_t ws_bytes, void *stream);
+
+/* emr_mask_combine_types followed by emr_compact_records, computed only over the
+ * tiles that tile_flags (from emr_eval_filter_tiles) marks: a tile without band
+ * bits keeps nothing, whatever its split bits. No mask plane is written. The
+ * lists, counts and offsets equal those of the two calls; entries past cap are
+ * dropped (compare offsets[n_pairs] with cap). eval_ws: the prepared records.
+ * Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY (eval_ws), EMR_ERR_RANGE, EMR_ERR_CUDA. */
+emr_status emr_select(const uint32_t *split, const uint32_t *band_bits, const uint8_t *tile_flags,
+                      const void *pack_host, const emr_query *q, const void *eval_ws, size_t eval_ws_bytes,
+                      const emr_grid *grid, int32_t mode, int32_t types, int32_t *idx, float *w, int64_t cap,
+                      int64_t *counts, int64_t *offsets, void *stream);
+
 /* Connection type code (0 forward, 1 backward, 2 lateral, 3 self; Section 6
  * taxonomy, see emr_mask_combine_types) of every list entry: type[e] for
  * entries e < min(offsets[n_pairs], cap) of lists laid out as emr_compact

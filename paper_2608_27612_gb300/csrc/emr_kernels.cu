@@ -326,6 +326,8 @@ enum { kModeMaterialise = 0, kModeFused = 1 };
 // pair r is bandb[r * band_stride + w - band_shift]; output at global index p of
 // pair r is out[r * out_stride + p - out_shift]. Whole-grid calls use strides
 // n_words / n_total and shifts 0. The split plane is always whole-grid.
+constexpr int kPyramidTop = 4;  // depths 0..4 (side <= 32) share one CTA
+
 struct TileArgs {
   const uint8_t* spec;
   SpecLayout L;
@@ -342,6 +344,8 @@ struct TileArgs {
   float* out_halo;
   uint32_t* split;
   uint32_t* bandb;
+  uint8_t* tile_flags;  // fused, optional: [pair][dense tile] set to 1 where a band bit is set
+  int64_t n_dense;
 };
 
 // CPPN at four points by interpreting the pair's record: node values live in
@@ -475,6 +479,7 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
   }
   if (!fused) return;
   __syncthreads();
+  bool any_pass = false;
   // band value of each position from its four neighbours at distance 2^-d
   for (int base = 0; base < nq; base += kBlock) {
     const int q = base + tid;
@@ -495,6 +500,7 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
     }
     const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
     const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+    any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
     const int q0 = base + warp * 32;
     if (d >= kQuadMajorFrom) {
       if (lane < 4 && q0 < nq)
@@ -509,6 +515,9 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
         if (pass[c]) A.out[pair_pos + mb + 4 * q + c] = w[c];
     }
   }
+  // dense tile numbering: depths 0..4 share tile 0, interpreter tile t >= 5 is dense tile t - 4
+  if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0)
+    A.tile_flags[int64_t(r) * A.n_dense + (tile <= kPyramidTop ? 0 : tile - kPyramidTop)] = 1;
 }
 
 // ---- register-resident tiles (pairs with at most kDenseMax varying nodes) ---------
@@ -523,7 +532,6 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
 // band value needs the neighbours, taken from the tile in shared memory after
 // a barrier (the ring of out-of-tile neighbours is evaluated by the tile too).
 
-constexpr int kPyramidTop = 4;  // depths 0..4 (side <= 32) share one CTA
 
 struct DTileArgs {
   const uint8_t* spec;
@@ -540,6 +548,8 @@ struct DTileArgs {
   float* out_halo;
   uint32_t* split;
   uint32_t* bandb;
+  uint8_t* tile_flags;  // fused, optional: [pair][dense tile] set to 1 where a band bit is set
+  int64_t n_dense;
 };
 
 template <int NP>
@@ -746,6 +756,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     if (!fused) return;
     __syncthreads();
     // band value of each position from its four neighbours at distance 2^-d
+    bool any_pass = false;
 #pragma unroll 2
     for (int k = 0; k < QPT; k++) {
       const float* t = s_wt + sbase + s_kq[k].z;  // (2pi, 2pj)
@@ -771,6 +782,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
       }
       const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
       const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+      any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
       if (lane == 0)  // the four quad-major words of this warp's 32 quads
         *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(b0, b1, b2, b3);
       if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
@@ -780,6 +792,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
           if (pass[c]) o[c] = w[c];
       }
     }
+    if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
     return;
   }
 
@@ -844,6 +857,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
   if (!fused) return;
   __syncthreads();
   int sb = 0;
+  bool any_pass = false;
   for (int d = 0; d <= d_hi; d++) {
     const int T = 1 << (d + 1), nq = T * T / 4, pitch = T + 2 * kPad;
     const int64_t lrow = prow + A.level_off[d];
@@ -875,6 +889,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
       }
       const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
       const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+      any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
       if (d >= kQuadMajorFrom) {
         if (lane < 4 && q0 < nq)
           A.bandb[band_base + A.word_off[d] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
@@ -889,6 +904,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     }
     sb += pitch * pitch;
   }
+  if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense] = 1;
 }
 
 // ---- filter planes from a materialised evaluation ---------------------------------
@@ -1055,6 +1071,42 @@ __device__ __noinline__ uint32_t type_bits(const TypeFilter& tf, int64_t r, cons
 // 4 words of depths 0..2 form group 0), pair = blockIdx.y; groups cover words
 // [w0, w0 + nw) (w0 and nw multiples of 4, or nw reaching n_words). split is a
 // whole-grid plane. Planes start at pair r0 (the type filter's slots are absolute).
+// Mask words wi .. wi + nwk - 1 (a group of 4 words: one 128-position block from
+// depth 3 on, or the 4 words of depths 0..2) of pair r: band (re-interleaved to
+// position-major) AND NOT split, gated AND active, AND kept connection types.
+// sp: the pair's split row; bw: its band words (indexed by global word); ra: the
+// pair's absolute number for the type filter.
+__device__ __forceinline__ void combine_group(const uint32_t* __restrict__ sp, const uint32_t* bw, const GridDev& G,
+                                              int64_t wi, int nwk, int gated, const TypeFilter& tf, int64_t ra,
+                                              uint32_t (&m)[4]) {
+  if (wi >= G.word_off[kQuadMajorFrom]) {
+    int d = kQuadMajorFrom;
+    while (G.word_off[d + 1] <= wi) d++;
+    const uint4 bq = *reinterpret_cast<const uint4*>(bw + wi);
+    const uint4 sq = d < G.D ? *reinterpret_cast<const uint4*>(sp + wi) : make_uint4(0, 0, 0, 0);
+    const uint32_t s4[4] = {sq.x, sq.y, sq.z, sq.w};
+#pragma unroll
+    for (int c = 0; c < 4; c++) {  // re-interleave the block's four child words
+      m[c] = band_word(bq.x, bq.y, bq.z, bq.w, c) & ~s4[c];
+      if (gated && m[c]) m[c] &= active_bits(sp, G, d, wi + c);
+      if (tf.types != EMR_CONN_ALL && m[c]) m[c] &= type_bits(tf, ra, G, d, wi + c);
+    }
+  } else {
+    for (int c = 0; c < 4; c++) {
+      m[c] = 0u;
+      if (c >= nwk) continue;
+      const int64_t wc = wi + c;
+      int d = 0;
+      while (G.word_off[d + 1] <= wc) d++;
+      uint32_t keep = bw[wc] & valid_bits(G, d, wc);
+      if (d < G.D) keep &= ~sp[wc];
+      if (gated && keep) keep &= active_bits(sp, G, d, wc);
+      if (tf.types != EMR_CONN_ALL && keep) keep &= type_bits(tf, ra, G, d, wc);
+      m[c] = keep;
+    }
+  }
+}
+
 __global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView band, PlaneView mask, GridDev G,
                                int64_t w0, int64_t nw, int gated, TypeFilter tf, int64_t r0) {
   const int64_t k = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) * 4;
@@ -1062,32 +1114,13 @@ __global__ void combine_kernel(const uint32_t* __restrict__ split, PlaneView ban
   const int64_t r = blockIdx.y;
   const int64_t wi = w0 + k;
   const uint32_t* sp = split + r * G.n_words;
-  uint32_t m[4];
   const int nwk = nw - k < 4 ? int(nw - k) : 4;
+  uint32_t m[4];
+  combine_group(sp, &band.at(r, 0), G, wi, nwk, gated, tf, r0 + r, m);
   if (wi >= G.word_off[kQuadMajorFrom]) {
-    int d = kQuadMajorFrom;
-    while (G.word_off[d + 1] <= wi) d++;
-    const uint4 bq = *reinterpret_cast<const uint4*>(&band.at(r, wi));
-    const uint4 sq = d < G.D ? *reinterpret_cast<const uint4*>(sp + wi) : make_uint4(0, 0, 0, 0);
-    const uint32_t s4[4] = {sq.x, sq.y, sq.z, sq.w};
-#pragma unroll
-    for (int c = 0; c < 4; c++) {  // re-interleave the block's four child words
-      m[c] = band_word(bq.x, bq.y, bq.z, bq.w, c) & ~s4[c];
-      if (gated && m[c]) m[c] &= active_bits(sp, G, d, wi + c);
-      if (tf.types != EMR_CONN_ALL && m[c]) m[c] &= type_bits(tf, r0 + r, G, d, wi + c);
-    }
     *reinterpret_cast<uint4*>(&mask.at(r, wi)) = make_uint4(m[0], m[1], m[2], m[3]);
   } else {
-    for (int c = 0; c < nwk; c++) {
-      const int64_t wc = wi + c;
-      int d = 0;
-      while (G.word_off[d + 1] <= wc) d++;
-      uint32_t keep = band.at(r, wc) & valid_bits(G, d, wc);
-      if (d < G.D) keep &= ~sp[wc];
-      if (gated && keep) keep &= active_bits(sp, G, d, wc);
-      if (tf.types != EMR_CONN_ALL && keep) keep &= type_bits(tf, r0 + r, G, d, wc);
-      mask.at(r, wc) = keep;
-    }
+    for (int c = 0; c < nwk; c++) mask.at(r, wi + c) = m[c];
   }
 }
 
@@ -1349,6 +1382,100 @@ __global__ void __launch_bounds__(kCompactBlock) gate_kernel(const uint32_t* __r
   }
 }
 
+// ---- selection over flagged tiles ---------------------------------------------------
+//
+// Mask combine, ordered compaction and kept weights in two passes (count, write)
+// that visit only the tiles whose flag says some band bit is set: every other
+// tile's mask is 0 whatever its split bits. One CTA per pair.
+
+constexpr int kSelectThreads = 128;
+
+// Words [*wb, *we) of dense tile t: tile 0 holds depths 0..min(D, 4), tile t >= 1 the
+// 128 words of one 64 x 64 block of a depth >= 5.
+__device__ __forceinline__ void tile_words(const GridDev& G, int32_t t, int64_t* wb, int64_t* we) {
+  if (t == 0) {
+    *wb = 0;
+    *we = G.word_off[(G.D < kPyramidTop ? G.D : kPyramidTop) + 1];
+  } else {
+    *wb = G.word_off[kPyramidTop + 1] + int64_t(t - 1) * (kTileSide * kTileSide / 32);
+    *we = *wb + kTileSide * kTileSide / 32;
+  }
+}
+
+__global__ void __launch_bounds__(kSelectThreads) select_count_kernel(const uint32_t* __restrict__ split,
+                                                                      const uint32_t* __restrict__ bandb,
+                                                                      const uint8_t* __restrict__ flags,
+                                                                      int64_t n_dense, GridDev G, int gated,
+                                                                      TypeFilter tf, int64_t* __restrict__ counts) {
+  __shared__ int sh[32];
+  const int64_t r = blockIdx.x;
+  const uint32_t* sp = split + r * G.n_words;
+  const uint32_t* bw = bandb + r * G.n_words;
+  int sum = 0;
+  for (int64_t t = 0; t < n_dense; t++) {
+    if (!flags[r * n_dense + t]) continue;
+    int64_t wb, we;
+    tile_words(G, int32_t(t), &wb, &we);
+    for (int64_t wi = wb + 4 * threadIdx.x; wi < we; wi += 4 * kSelectThreads) {
+      uint32_t m[4];
+      combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
+      sum += __popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]);
+    }
+  }
+  int total;
+  block_exclusive_scan(sum, sh, &total);
+  if (threadIdx.x == 0) counts[r] = total;
+}
+
+__global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint32_t* __restrict__ split,
+                                                                      const uint32_t* __restrict__ bandb,
+                                                                      const uint8_t* __restrict__ flags,
+                                                                      int64_t n_dense, GridDev G, int gated,
+                                                                      TypeFilter tf, RecordSource rs,
+                                                                      const int64_t* __restrict__ offsets,
+                                                                      int64_t cap, int32_t* __restrict__ idx,
+                                                                      float* __restrict__ wv) {
+  __shared__ int sh[32];
+  const int64_t r = blockIdx.x;
+  const uint32_t* sp = split + r * G.n_words;
+  const uint32_t* bw = bandb + r * G.n_words;
+  int64_t base = offsets[r];
+  for (int64_t t = 0; t < n_dense; t++) {
+    if (!flags[r * n_dense + t]) continue;
+    int64_t wb, we;
+    tile_words(G, int32_t(t), &wb, &we);
+    for (int64_t w0 = wb; w0 < we; w0 += 4 * kSelectThreads) {  // block-uniform loop
+      const int64_t wi = w0 + 4 * threadIdx.x;
+      uint32_t m[4] = {0u, 0u, 0u, 0u};
+      if (wi < we) combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
+      int total;
+      const int ex = block_exclusive_scan(__popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]), sh, &total);
+      int64_t dst = base + ex;
+      for (int c = 0; c < 4; c++) {
+        if (!m[c]) continue;
+        int d = 0;
+        while (G.word_off[d + 1] <= wi + c) d++;
+        const int64_t gbase = G.level_off[d] + (wi + c - G.word_off[d]) * 32;
+        for (uint32_t v = m[c]; v; v &= v - 1, dst++)
+          if (dst < cap) idx[dst] = int32_t(gbase + __ffs(v) - 1);
+      }
+      base += total;
+    }
+  }
+  if (!wv) return;
+  __syncthreads();  // this pair's indices are written
+  const int64_t end = offsets[r + 1] < cap ? offsets[r + 1] : cap;
+  for (int64_t e = offsets[r] + threadIdx.x; e < end; e += kSelectThreads) {
+    const int64_t gidx = idx[e];
+    int d = 0;
+    while (G.level_off[d + 1] <= gidx) d++;
+    const uint32_t m = uint32_t(gidx - G.level_off[d]);
+    const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1)
+    const float x = grid_coord(int(compact1by1(m)), scale), y = grid_coord(int(compact1by1(m >> 1)), scale);
+    wv[e] = eval_record_point(rs.spec + r * rs.L.stride, rs.L, x, y);
+  }
+}
+
 // ---- host helpers ---------------------------------------------------------------
 
 inline emr_status cuda_status(cudaError_t e) { return e == cudaSuccess ? EMR_OK : EMR_ERR_CUDA; }
@@ -1479,9 +1606,12 @@ struct TileRange {
 
 emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spec, const int32_t* order, int mode,
                         float theta, float band, float w_min, float* out, float* out_halo, uint32_t* split,
-                        uint32_t* bandb, cudaStream_t st, TileRange tr = TileRange()) {
+                        uint32_t* bandb, cudaStream_t st, TileRange tr = TileRange(),
+                        uint8_t* tile_flags = nullptr) {
   emr_status rc = EMR_OK;
   const int32_t n_dense = int32_t(dense_tiles(g->D));
+  if (tile_flags && cudaMemsetAsync(tile_flags, 0, size_t(p.n_pairs) * size_t(n_dense), st) != cudaSuccess)
+    return EMR_ERR_CUDA;
   if (tr.end < 0) tr.end = n_dense;
   if (tr.band_stride < 0) tr.band_stride = g->n_words;
   if (tr.out_stride < 0) tr.out_stride = g->n_total;
@@ -1526,6 +1656,8 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
     A.out_halo = out_halo;
     A.split = split;
     A.bandb = bandb;
+    A.tile_flags = tile_flags;
+    A.n_dense = n_dense;
     const int64_t blocks = p.n_class[0] * int64_t(A.n_tiles);
     if (blocks > 0x7fffffffLL) return EMR_ERR_RANGE;
     const size_t smem = tile_smem_bytes(p.L);
@@ -1562,6 +1694,8 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   D.out_halo = out_halo;
   D.split = split;
   D.bandb = bandb;
+  D.tile_flags = tile_flags;
+  D.n_dense = n_dense;
   int64_t beg = p.n_class[0];
   if ((rc = launch_dense<12>(D, beg, p.n_class[1], st)) != EMR_OK) return rc;
   beg += p.n_class[1];
@@ -1776,6 +1910,51 @@ emr_status emr_compact_records(const uint32_t* mask, const void* pack_host, cons
   return launch_compact(PlaneView{const_cast<uint32_t*>(mask), grid->n_words, 0}, nullptr, 0, 0, grid, p.n_pairs, 0,
                         grid->n_words, idx, w, cap, counts, offsets, ws, static_cast<cudaStream_t>(stream),
                         RecordSource{static_cast<const uint8_t*>(eval_ws), p.L});
+}
+
+emr_status emr_eval_filter_tiles(const void* pack_host, const emr_query* q, const emr_grid* grid, float theta,
+                                 float band, float w_min, uint32_t* split, uint32_t* band_bits, uint8_t* tile_flags,
+                                 void* ws, size_t ws_bytes, void* stream) {
+  if (!grid_ok(grid) || !split || !band_bits || !tile_flags || !ws) return EMR_ERR_ARG;
+  if (!(theta >= 0.f) || !(band >= 0.f) || !(w_min >= 0.f)) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (ws_bytes < p.total) return EMR_ERR_CAPACITY;
+  uint8_t* spec;
+  int32_t* order;
+  ws_layout(p, ws, &spec, &order);
+  return launch_tiles(p, grid, spec, order, kModeFused, theta, band, w_min, nullptr, nullptr, split, band_bits,
+                      static_cast<cudaStream_t>(stream), TileRange(), tile_flags);
+}
+
+emr_status emr_select(const uint32_t* split, const uint32_t* band_bits, const uint8_t* tile_flags,
+                      const void* pack_host, const emr_query* q, const void* eval_ws, size_t eval_ws_bytes,
+                      const emr_grid* grid, int32_t mode, int32_t types, int32_t* idx, float* w, int64_t cap,
+                      int64_t* counts, int64_t* offsets, void* stream) {
+  if (!split || !band_bits || !tile_flags || !eval_ws || !grid_ok(grid) || (!idx && cap > 0) || cap < 0 ||
+      !counts || !offsets || (mode != EMR_EAGER && mode != EMR_GATED) || types < 0 || types > EMR_CONN_ALL)
+    return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (eval_ws_bytes < p.total) return EMR_ERR_CAPACITY;
+  if (p.n_pairs <= 0 || p.n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
+  TypeFilter tf = no_type_filter();
+  if (types != EMR_CONN_ALL) {
+    tf.types = types;
+    tf.q = query_dev(q);
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const GridDev G = grid_dev(grid);
+  const int64_t n_dense = dense_tiles(grid->D);
+  select_count_kernel<<<unsigned(p.n_pairs), kSelectThreads, 0, st>>>(split, band_bits, tile_flags, n_dense, G,
+                                                                       mode == EMR_GATED, tf, counts);
+  compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, p.n_pairs, offsets);
+  select_write_kernel<<<unsigned(p.n_pairs), kSelectThreads, 0, st>>>(
+      split, band_bits, tile_flags, n_dense, G, mode == EMR_GATED, tf,
+      RecordSource{static_cast<const uint8_t*>(eval_ws), p.L}, offsets, cap, idx, w);
+  return cuda_status(cudaGetLastError());
 }
 
 emr_status emr_compact(const uint32_t* mask, const float* out, const emr_grid* grid, int32_t n_pairs, int32_t* idx,

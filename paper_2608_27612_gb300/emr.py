@@ -73,6 +73,8 @@ def lib() -> C.CDLL:
             "emr_stream_mode": [vp, vp, vp, vp, f32, f32, f32, i32, i32, vp, sz, i64, vp, vp, i64, vp, vp, i64, vp],
             "emr_mask_combine_types": [vp, vp, vp, vp, i32, i32, i32, vp, vp],
             "emr_conn_types": [vp, vp, vp, vp, i32, i64, vp, vp],
+            "emr_eval_filter_tiles": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
+            "emr_select": [vp, vp, vp, vp, vp, vp, sz, vp, i32, i32, vp, vp, i64, vp, vp, vp],
             "emr_substrate_config": [i32, vp, vp],
             "emr_assemble_workspace_size": [vp, i32, i32, i32, vp, i64, vp],
             "emr_assemble": [vp, vp, i32, vp, vp, i32, vp, vp, vp, f32, f32, f32, i32, i32, i32, i32, vp, sz, i64,
@@ -276,6 +278,28 @@ def stream(pack, pack_dev, query: Query, grid: Grid, theta: float, band: float, 
                                  types, _ptr(ws), C.c_size_t(ws.numel()), chunk_cap, _ptr(h_idx), _ptr(h_w),
                                  h_idx.numel(), _ptr(counts), _ptr(offsets), timeout_ms, _stream(stream)),
            "emr_stream_mode")
+
+
+def dense_tiles(D: int) -> int:
+    """Dense tiles of a depth-D grid: one for depths 0..4, then the 64 x 64 blocks of depths 5..D."""
+    return 1 + sum(4 ** (d - 5) for d in range(5, D + 1))
+
+
+def eval_filter_tiles(pack, query: Query, grid: Grid, theta: float, band: float, w_min: float, split, band_bits,
+                      tile_flags, ws, stream=None):
+    q = query.c
+    _check(lib().emr_eval_filter_tiles(_ptr(pack), C.byref(q), C.byref(grid), theta, band, w_min, _ptr(split),
+                                       _ptr(band_bits), _ptr(tile_flags), _ptr(ws), C.c_size_t(ws.numel()),
+                                       _stream(stream)), "emr_eval_filter_tiles")
+
+
+def select(split, band_bits, tile_flags, pack, query: Query, eval_ws, grid: Grid, mode: int, types: int, idx, w,
+           cap: int, counts, offsets, stream=None):
+    """emr_select: combine + compaction + kept weights over the flagged tiles only."""
+    q = query.c
+    _check(lib().emr_select(_ptr(split), _ptr(band_bits), _ptr(tile_flags), _ptr(pack), C.byref(q), _ptr(eval_ws),
+                            C.c_size_t(eval_ws.numel()), C.byref(grid), mode, types, _ptr(idx), _ptr(w), cap,
+                            _ptr(counts), _ptr(offsets), _stream(stream)), "emr_select")
 
 
 def mask_combine_types(split, band_bits, query: Query, grid: Grid, n_pairs: int, mode: int, types: int, mask,
@@ -492,6 +516,17 @@ class Discovery:
         else:
             compact_records(self.mask, self.pack, self.query, self.ws, self.grid, self.idx, self.w, self.cap,
                             self.counts, self.offsets, self.cws, stream)
+
+    def run_select(self, stream=None):
+        """emr_eval_prepare, emr_eval_filter_tiles, emr_select (no mask plane)."""
+        if getattr(self, "tile_flags", None) is None:
+            self.tile_flags = torch.zeros(self.n_pairs, dense_tiles(self.grid.D), dtype=torch.uint8,
+                                          device=self.device)
+        self.prepare(stream)
+        eval_filter_tiles(self.pack, self.query, self.grid, self.theta, self.band, self.w_min, self.split,
+                          self.band_bits, self.tile_flags, self.ws, stream)
+        select(self.split, self.band_bits, self.tile_flags, self.pack, self.query, self.ws, self.grid, self.mode,
+               self.types, self.idx, self.w, self.cap, self.counts, self.offsets, stream)
 
     def combine(self, stream=None):
         """emr_mask_combine, or emr_mask_combine_types when a connection-type filter is set."""

@@ -610,6 +610,37 @@ __device__ __forceinline__ void eval_dense(const float4* __restrict__ coef, cons
   }
 }
 
+// Split and band words that dense tile `tile` of pair r covers, set to 0: the
+// planes of a pair whose output is constant over the grid (every variance and
+// band value is exactly 0). Words as the tile kernels write them: tile 0 the
+// parents of depths 1..4 and the band words of depths 0..4, tile t >= 1 the 32
+// parent words and 128 band words of its 64 x 64 block.
+__device__ __forceinline__ void zero_tile(const DTileArgs& A, int r, int tile, int tid, int nthreads) {
+  uint32_t* split_row = A.split + int64_t(r) * A.n_words;
+  const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;
+  if (tile > 0) {
+    int u = tile - 1, d = kPyramidTop + 1;
+    while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
+    const uint32_t mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
+    for (int k = tid; k < 32; k += nthreads) split_row[A.word_off[d - 1] + mb / 128 + k] = 0u;
+    for (int k = tid; k < 128; k += nthreads) A.bandb[band_base + A.word_off[d] + mb / 32 + k] = 0u;
+    return;
+  }
+  const int d_hi = min(A.D, kPyramidTop);
+  for (int d = 0; d <= d_hi; d++) {
+    const int nq = 1 << (2 * d);
+    if (d >= 1)
+      for (int k = tid; k < (nq + 31) / 32; k += nthreads) split_row[A.word_off[d - 1] + k] = 0u;
+    for (int k = tid; k < (4 * nq + 31) / 32; k += nthreads) A.bandb[band_base + A.word_off[d] + k] = 0u;
+  }
+}
+
+// Fused mode: the planes of constant-output pairs (ranks rank_beg ..), one CTA per pair.
+__global__ void __launch_bounds__(128) zero_tiles_kernel(const DTileArgs A) {
+  const int r = A.order[A.rank_beg + blockIdx.x];
+  for (int t = A.tile_beg; t < A.tile_beg + A.n_tiles; t++) zero_tile(A, r, t, threadIdx.x, blockDim.x);
+}
+
 // The shared tile stores position (i, j) of a T x T tile at row j + 2, column
 // i + 2 (pitch T + 4): two-column padding keeps sibling pairs 8-byte aligned;
 // the ring of out-of-tile neighbours sits in columns / rows 1 and T + 2.
@@ -1504,6 +1535,7 @@ GridDev grid_dev(const emr_grid* g) {
 struct EvalPlan {
   int64_t n_pairs;
   int64_t n_class[kClasses];  // pairs per kernel class (schedule order)
+  int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of class 3
   SpecLayout L;
   int32_t scratch_stride;
   size_t spec_bytes, scratch_bytes, order_bytes, total;
@@ -1526,11 +1558,16 @@ emr_status eval_plan(const void* pack_host, const emr_query* q, EvalPlan* p) {
     if (sides[s]) { nv = std::max(nv, h->max_varying[s]); nve = std::max(nve, h->max_vedges[s]); }
   p->n_pairs = int64_t(h->P) * q->S;
   for (int c = 0; c < kClasses; c++) p->n_class[c] = 0;
+  p->n_const = 0;
   for (int g = 0; g < h->P; g++)
     for (int s = 0; s < q->S; s++) {
-      if (q->per_genome && q->count_host && s >= q->count_host[g]) { p->n_class[pair_class(0)]++; continue; }
-      const int64_t si = q->per_genome ? int64_t(g) * q->S + s : s;
-      p->n_class[pair_class(gt[g].n_varying[q->side_host[si]])]++;
+      int nvar = 0;  // unused slots evaluate to a constant
+      if (!(q->per_genome && q->count_host && s >= q->count_host[g])) {
+        const int64_t si = q->per_genome ? int64_t(g) * q->S + s : s;
+        nvar = gt[g].n_varying[q->side_host[si]];
+      }
+      p->n_class[pair_class(nvar)]++;
+      if (nvar == 0) p->n_const++;
     }
   p->L = spec_layout(nv, nve);
   p->scratch_stride = std::max(h->max_nodes, 1);
@@ -1701,7 +1738,12 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   beg += p.n_class[1];
   if ((rc = launch_dense<8>(D, beg, p.n_class[2], st)) != EMR_OK) return rc;
   beg += p.n_class[2];
-  return launch_dense<4>(D, beg, p.n_class[3], st);
+  if (mode != kModeFused || p.n_const == 0) return launch_dense<4>(D, beg, p.n_class[3], st);
+  if ((rc = launch_dense<4>(D, beg, p.n_class[3] - p.n_const, st)) != EMR_OK) return rc;
+  D.rank_beg = beg + p.n_class[3] - p.n_const;
+  if (p.n_const > 0x7fffffffLL) return EMR_ERR_RANGE;
+  zero_tiles_kernel<<<unsigned(p.n_const), 128, 0, st>>>(D);
+  return cuda_status(cudaGetLastError());
 }
 
 emr_status launch_combine(const uint32_t* split, PlaneView band, PlaneView mask, const emr_grid* g, int64_t n_pairs,

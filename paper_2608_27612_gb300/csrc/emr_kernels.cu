@@ -666,8 +666,8 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel
     const int dx = int(compact1by1(uint32_t(TPB * tid))), dy = int(compact1by1(uint32_t(TPB * tid) >> 1));
     s_kq[tid] = make_int4(__float_as_int(float(dx)), __float_as_int(float(dy)), 2 * dx + 2 * dy * P64, 0);
   }
-  const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
-  const int tile = A.tile_beg + int(blockIdx.x % A.n_tiles);
+  const int64_t rank = A.rank_beg + blockIdx.y;
+  const int tile = A.tile_beg + int(blockIdx.x);
   const int r = A.order[rank];
   const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
   const int nv = reinterpret_cast<const int32_t*>(rec)[0];
@@ -1627,10 +1627,11 @@ template <int NVMAX>
 emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st) {
   if (n_ranks <= 0) return EMR_OK;
   DTileArgs A = A0;
-  A.rank_beg = rank_beg;
-  const int64_t blocks = n_ranks * int64_t(A.n_tiles);
-  if (blocks > 0x7fffffffLL) return EMR_ERR_RANGE;
-  tile_kernel_dense<NVMAX, kDenseTPB><<<unsigned(blocks), kDenseTPB, 0, st>>>(A);
+  for (int64_t r0 = 0; r0 < n_ranks; r0 += 65535) {  // grid y: ranks, at most 65535 a launch
+    A.rank_beg = rank_beg + r0;
+    const dim3 grid(unsigned(A.n_tiles), unsigned(std::min<int64_t>(65535, n_ranks - r0)));
+    tile_kernel_dense<NVMAX, kDenseTPB><<<grid, kDenseTPB, 0, st>>>(A);
+  }
   return cuda_status(cudaGetLastError());
 }
 

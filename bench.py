@@ -306,6 +306,61 @@ def networks_run(emr, torch, W, D=5, P=1000, config=None, reps=20):
                       "pruning), median of 2 after one warm-up; forward: CUDA events, mean of %d" % reps}
 
 
+def hbm_peak():
+    """Measured copy bandwidth (GB/s) of the GB300s, or the stated fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "of measured"
+    except (OSError, ValueError, KeyError):
+        return 6800.0, "of fallback"
+
+
+def variants_run(emr, torch, W, D=7, P=1000, reps=10):
+    """The subtree-leaf variance split (memory-bound over materialised outputs) and HyperNEAT weight
+    scaling of the lists, on the c2 workload; CUDA events."""
+    w = W.c2(D=D, P=P)
+    dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, materialise=True)
+    dsc.run_unfused()
+    g = dsc.grid
+    split = torch.zeros_like(dsc.split)
+    ws = torch.empty(emr.subtree_workspace_size(g, dsc.n_pairs), dtype=torch.uint8, device="cuda")
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    emr.subtree_split(dsc.out, g, dsc.n_pairs, w.theta, split, ws)
+    torch.cuda.synchronize()
+    e0, e1 = ev(), ev()
+    e0.record()
+    for _ in range(reps):
+        emr.subtree_split(dsc.out, g, dsc.n_pairs, w.theta, split, ws)
+    e1.record()
+    torch.cuda.synchronize()
+    t_sub = e0.elapsed_time(e1) / 1e3 / reps
+    leaves = dsc.n_pairs * 4 ** (D + 1)
+    alg_bytes = 4 * leaves + 4 * dsc.n_pairs * int(g.word_off[D])   # leaves read, split words of depths < D written
+    peak, basis = hbm_peak()
+    dsc.run_fused()
+    total = int(dsc.offsets[-1])
+    wv = dsc.w.clone()
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(reps):
+        emr.scale_weights(wv, dsc.offsets, dsc.n_pairs, dsc.cap, 0.1, 3.0)
+    e1.record()
+    torch.cuda.synchronize()
+    t_scale = e0.elapsed_time(e1) / 1e3 / reps
+    del ws, dsc
+    torch.cuda.empty_cache()
+    return {"subtree_split": {"workload": "c2_pop%d_d%d_materialised" % (P, D), "seconds": t_sub,
+                              "leaves": leaves, "leaves_per_s": leaves / t_sub,
+                              "roofline": {"bound": "hbm", "achieved": alg_bytes / t_sub / 1e9, "peak": peak,
+                                           "unit": "GB/s", "frac": alg_bytes / t_sub / 1e9 / peak,
+                                           "peak_basis": basis,
+                                           "traffic_note": "algorithmic bytes: 4 B per depth-D output read, the "
+                                                           "split words of depths < D written; the level "
+                                                           "aggregates (about 1.8 B more per leaf) are scratch"}},
+            "scale_weights": {"entries": total, "seconds": t_scale},
+            "timing": "CUDA events, mean of %d" % reps}
+
+
 def launches_in_step(emr, dsc):
     """Kernel launches of one step: prepare (schedule, records), one tile launch per
     non-empty kernel class, one zeroing launch for constant-output pairs, selection
@@ -494,7 +549,8 @@ def main():
                  "c4_round2_hh_d8_backward_config": streamed_run(
                      emr, torch, c4r2, 1 << 16, 1 << 24, 1 << 26, 3,
                      types=emr.substrate_config(emr.SUBSTRATE_BACKWARD)[0], label=c4r2.name + "_backward"),
-                 "xor_networks_hh_d5": networks_run(emr, torch, W)}
+                 "xor_networks_hh_d5": networks_run(emr, torch, W),
+                 "variants_c2_d7": variants_run(emr, torch, W)}
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:

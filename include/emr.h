@@ -382,6 +382,34 @@ emr_status emr_select(const uint32_t *split, const uint32_t *band_bits, const ui
                       const emr_grid *grid, int32_t mode, int32_t types, int32_t *idx, float *w, int64_t cap,
                       int64_t *counts, int64_t *offsets, void *stream);
 
+/* Subtree-leaf variance: the split plane under ES-HyperNEAT's reading of a
+ * cell's variance (its quadtree measures the spread of the outputs at a
+ * region's leaves; the paper's Section 3.2 computes it over a cell's four
+ * children, which is the default everywhere else). Cell p of depth d < D
+ * splits when the population variance of the outputs at all its depth-D
+ * descendants (4^(D - d) positions) exceeds theta. From materialised outputs
+ * (out as written by emr_eval); writes the split words of depths 0..D-1 (device
+ * uint32 [n_pairs][n_words], position-major), and, when var_out is not NULL,
+ * that variance at each position of depths 0..D-1 (device float [n_pairs]
+ * [n_total]). Combine with band bits by emr_mask_combine(_types) as usual.
+ * ws: emr_subtree_workspace_size bytes (two levels of per-cell aggregates).
+ * D at most 11. Errors: EMR_ERR_ARG, EMR_ERR_RANGE, EMR_ERR_CAPACITY,
+ * EMR_ERR_CUDA. */
+emr_status emr_subtree_workspace_size(const emr_grid *grid, int32_t n_pairs, size_t *bytes);
+emr_status emr_subtree_split(const float *out, const emr_grid *grid, int32_t n_pairs, float theta,
+                             uint32_t *split, float *var_out, void *ws, size_t ws_bytes, void *stream);
+
+/* HyperNEAT's weight scaling (the indirect encoding of Section 2, where a
+ * connection is expressed only when the CPPN output's magnitude exceeds a
+ * threshold; the paper's pipeline uses raw outputs, so this is an option) on
+ * the weights of lists laid out as emr_compact writes them, in place:
+ * w <- sign(w) * w_max * (min(|w|, 1) - w_thr) / (1 - w_thr) when |w| > w_thr,
+ * else 0 (combine with w_min = w_thr to drop those entries at discovery).
+ * Entries e < min(offsets[n_pairs], cap). Requires 0 <= w_thr < 1, w_max > 0.
+ * Errors: EMR_ERR_ARG, EMR_ERR_CUDA. */
+emr_status emr_scale_weights(float *w, const int64_t *offsets, int32_t n_pairs, int64_t cap, float w_thr,
+                             float w_max, void *stream);
+
 /* Connection type code (0 forward, 1 backward, 2 lateral, 3 self; Section 6
  * taxonomy, see emr_mask_combine_types) of every list entry: type[e] for
  * entries e < min(offsets[n_pairs], cap) of lists laid out as emr_compact

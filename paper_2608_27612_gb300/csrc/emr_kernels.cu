@@ -635,10 +635,12 @@ __device__ __forceinline__ void zero_tile(const DTileArgs& A, int r, int tile, i
   }
 }
 
-// Fused mode: the planes of constant-output pairs (ranks rank_beg ..), one CTA per pair.
+// Fused mode: the planes of constant-output pairs (ranks rank_beg + blockIdx.y);
+// the CTAs of a pair take its tiles in turn.
 __global__ void __launch_bounds__(128) zero_tiles_kernel(const DTileArgs A) {
-  const int r = A.order[A.rank_beg + blockIdx.x];
-  for (int t = A.tile_beg; t < A.tile_beg + A.n_tiles; t++) zero_tile(A, r, t, threadIdx.x, blockDim.x);
+  const int r = A.order[A.rank_beg + blockIdx.y];
+  for (int t = A.tile_beg + int(blockIdx.x); t < A.tile_beg + A.n_tiles; t += int(gridDim.x))
+    zero_tile(A, r, t, threadIdx.x, blockDim.x);
 }
 
 // The shared tile stores position (i, j) of a T x T tile at row j + 2, column
@@ -1507,6 +1509,80 @@ __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint
   }
 }
 
+constexpr int kSubtreeMaxDepth = 11;  // aggregates of 4^D cells per pair must stay addressable and modest
+
+// ---- subtree-leaf variance (the ES-HyperNEAT reading of a cell's variance) ----
+//
+// A depth-e cell's depth-D descendants are a contiguous Morton range of 4^(D-e)
+// leaves, so aggregates (mean, M2 = sum of squared deviations) merge level by
+// level: four children of n leaves each give mean = average of their means and
+// M2 = the sum of their M2 plus n times the squared deviations of their means.
+// One launch per level; cell idx of the launch is pair idx >> 2(e+1), Morton
+// index idx & (4^(e+1) - 1). The loop over cells is warp-uniform (the split
+// words come from ballots).
+__global__ void __launch_bounds__(256) subtree_level_kernel(const float* __restrict__ out,
+                                                            const float2* __restrict__ child,
+                                                            float2* __restrict__ agg, int e, GridDev G,
+                                                            int64_t n_pairs, float theta,
+                                                            uint32_t* __restrict__ split, float* __restrict__ var_out) {
+  const int lane = threadIdx.x & 31;
+  const int lg = 2 * (e + 1);                      // log2 of the cells of level e
+  const int64_t cells = int64_t(1) << lg, total = n_pairs * cells;
+  const float n_child = float(int64_t(1) << (2 * (G.D - e - 1)));  // leaves under each child
+  const float n_cell = 4.f * n_child;
+  const int64_t stride = int64_t(gridDim.x) * blockDim.x;
+  for (int64_t base = int64_t(blockIdx.x) * blockDim.x + (threadIdx.x & ~31); base < total; base += stride) {
+    const int64_t idx = base + lane;
+    const bool valid = idx < total;
+    bool bit = false;
+    if (valid) {
+      const int64_t r = idx >> lg, m = idx & (cells - 1);
+      float c[4], M[4] = {0.f, 0.f, 0.f, 0.f};
+      if (e == G.D - 1) {
+        const float4 x = *reinterpret_cast<const float4*>(out + r * G.n_total + G.level_off[G.D] + 4 * m);
+        c[0] = x.x; c[1] = x.y; c[2] = x.z; c[3] = x.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; k++) {
+          const float2 a = child[4 * idx + k];
+          c[k] = a.x;
+          M[k] = a.y;
+        }
+      }
+      const float mean = ((c[0] + c[1]) + (c[2] + c[3])) * 0.25f;
+      const float d0 = c[0] - mean, d1 = c[1] - mean, d2 = c[2] - mean, d3 = c[3] - mean;
+      const float m2 = ((M[0] + M[1]) + (M[2] + M[3])) + n_child * ((d0 * d0 + d1 * d1) + (d2 * d2 + d3 * d3));
+      agg[idx] = make_float2(mean, m2);
+      bit = m2 > theta * n_cell;
+      if (var_out) var_out[r * G.n_total + G.level_off[e] + m] = m2 / n_cell;
+    }
+    const uint32_t bal = __ballot_sync(0xffffffffu, bit);
+    if (valid) {
+      const int64_t r = idx >> lg, m = idx & (cells - 1);
+      if (cells >= 32) {
+        if (lane == 0) split[r * G.n_words + G.word_off[e] + (m >> 5)] = bal;
+      } else if (m == 0) {  // 4 or 16 cells: the pair's word holds lanes lane .. lane + cells - 1
+        split[r * G.n_words + G.word_off[e]] = (bal >> lane) & uint32_t((int64_t(1) << cells) - 1);
+      }
+    }
+  }
+}
+
+// HyperNEAT's weight scaling of list entries: a connection whose output
+// magnitude exceeds the threshold is expressed, its magnitude mapped linearly
+// from (thr, 1] onto (0, w_max] (magnitudes above 1 clamp to 1); others become 0.
+__global__ void __launch_bounds__(kCompactBlock) scale_weights_kernel(float* __restrict__ w,
+                                                                      const int64_t* __restrict__ offsets,
+                                                                      int64_t n_pairs, int64_t cap, float thr,
+                                                                      float w_max) {
+  const int64_t total = offsets[n_pairs] < cap ? offsets[n_pairs] : cap;
+  for (int64_t e = int64_t(blockIdx.x) * kCompactBlock + threadIdx.x; e < total;
+       e += int64_t(gridDim.x) * kCompactBlock) {
+    const float v = w[e], a = fabsf(v);
+    w[e] = a > thr ? copysignf((fminf(a, 1.0f) - thr) / (1.0f - thr) * w_max, v) : 0.0f;
+  }
+}
+
 // ---- host helpers ---------------------------------------------------------------
 
 inline emr_status cuda_status(cudaError_t e) { return e == cudaSuccess ? EMR_OK : EMR_ERR_CUDA; }
@@ -1741,9 +1817,12 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   beg += p.n_class[2];
   if (mode != kModeFused || p.n_const == 0) return launch_dense<4>(D, beg, p.n_class[3], st);
   if ((rc = launch_dense<4>(D, beg, p.n_class[3] - p.n_const, st)) != EMR_OK) return rc;
-  D.rank_beg = beg + p.n_class[3] - p.n_const;
-  if (p.n_const > 0x7fffffffLL) return EMR_ERR_RANGE;
-  zero_tiles_kernel<<<unsigned(p.n_const), 128, 0, st>>>(D);
+  const int64_t c0 = beg + p.n_class[3] - p.n_const;
+  for (int64_t r0 = 0; r0 < p.n_const; r0 += 65535) {  // grid y: pairs, at most 65535 a launch
+    D.rank_beg = c0 + r0;
+    const dim3 grid(unsigned(std::min<int64_t>(D.n_tiles, 64)), unsigned(std::min<int64_t>(65535, p.n_const - r0)));
+    zero_tiles_kernel<<<grid, 128, 0, st>>>(D);
+  }
   return cuda_status(cudaGetLastError());
 }
 
@@ -1876,6 +1955,54 @@ emr_status emr_mask_combine_types(const uint32_t* split, const uint32_t* band_bi
   tf.q = query_dev(q);
   return launch_combine(split, band_bits, grid, n_pairs, mode == EMR_GATED, mask, static_cast<cudaStream_t>(stream),
                         tf);
+}
+
+emr_status emr_subtree_workspace_size(const emr_grid* grid, int32_t n_pairs, size_t* bytes) {
+  if (!grid_ok(grid) || n_pairs <= 0 || !bytes) return EMR_ERR_ARG;
+  if (grid->D > kSubtreeMaxDepth) return EMR_ERR_RANGE;
+  const size_t a = size_t(1) << (2 * grid->D), b = grid->D >= 1 ? a / 4 : 1;
+  *bytes = size_t(n_pairs) * (a + b) * 8 + 512;
+  return EMR_OK;
+}
+
+emr_status emr_subtree_split(const float* out, const emr_grid* grid, int32_t n_pairs, float theta, uint32_t* split,
+                             float* var_out, void* ws, size_t ws_bytes, void* stream) {
+  size_t need = 0;
+  emr_status rc = emr_subtree_workspace_size(grid, n_pairs, &need);
+  if (rc != EMR_OK) return rc;
+  if (!out || !split || !ws || !(theta >= 0.f)) return EMR_ERR_ARG;
+  if (ws_bytes < need) return EMR_ERR_CAPACITY;
+  if (grid->D == 0) return EMR_OK;  // a single level: every position is a leaf
+  const size_t a = size_t(1) << (2 * grid->D);
+  float2* buf[2] = {static_cast<float2*>(ws),
+                    reinterpret_cast<float2*>(static_cast<uint8_t*>(ws) + ((size_t(n_pairs) * a * 8 + 255) & ~size_t(255)))};
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return EMR_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const GridDev G = grid_dev(grid);
+  for (int e = grid->D - 1, k = 0; e >= 0; e--, k ^= 1) {
+    const int64_t total = int64_t(n_pairs) << (2 * (e + 1));
+    const int64_t blocks = std::min<int64_t>((total + 255) / 256, int64_t(16) * sms);
+    subtree_level_kernel<<<unsigned(blocks), 256, 0, st>>>(out, buf[k ^ 1], buf[k], e, G, n_pairs, theta, split,
+                                                           var_out);
+  }
+  return cuda_status(cudaGetLastError());
+}
+
+emr_status emr_scale_weights(float* w, const int64_t* offsets, int32_t n_pairs, int64_t cap, float w_thr,
+                             float w_max, void* stream) {
+  if (!offsets || n_pairs <= 0 || cap < 0 || (cap > 0 && !w) || !(w_thr >= 0.f && w_thr < 1.f) || !(w_max > 0.f))
+    return EMR_ERR_ARG;
+  if (cap == 0) return EMR_OK;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return EMR_ERR_CUDA;
+  scale_weights_kernel<<<unsigned(8 * sms), kCompactBlock, 0, static_cast<cudaStream_t>(stream)>>>(
+      w, offsets, n_pairs, cap, w_thr, w_max);
+  return cuda_status(cudaGetLastError());
 }
 
 emr_status emr_conn_types(const int32_t* idx, const int64_t* offsets, const emr_query* q, const emr_grid* grid,

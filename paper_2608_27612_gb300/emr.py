@@ -73,6 +73,9 @@ def lib() -> C.CDLL:
             "emr_stream_mode": [vp, vp, vp, vp, f32, f32, f32, i32, i32, vp, sz, i64, vp, vp, i64, vp, vp, i64, vp],
             "emr_mask_combine_types": [vp, vp, vp, vp, i32, i32, i32, vp, vp],
             "emr_conn_types": [vp, vp, vp, vp, i32, i64, vp, vp],
+            "emr_scale_weights": [vp, vp, i32, i64, f32, f32, vp],
+            "emr_subtree_workspace_size": [vp, i32, vp],
+            "emr_subtree_split": [vp, vp, i32, f32, vp, vp, vp, sz, vp],
             "emr_eval_filter_tiles": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
             "emr_select": [vp, vp, vp, vp, vp, vp, sz, vp, i32, i32, vp, vp, i64, vp, vp, vp],
             "emr_substrate_config": [i32, vp, vp],
@@ -307,6 +310,24 @@ def mask_combine_types(split, band_bits, query: Query, grid: Grid, n_pairs: int,
     q = query.c
     _check(lib().emr_mask_combine_types(_ptr(split), _ptr(band_bits), C.byref(q), C.byref(grid), n_pairs, mode,
                                         types, _ptr(mask), _stream(stream)), "emr_mask_combine_types")
+
+
+def subtree_workspace_size(grid: Grid, n_pairs: int) -> int:
+    n = C.c_size_t()
+    _check(lib().emr_subtree_workspace_size(C.byref(grid), n_pairs, C.byref(n)), "emr_subtree_workspace_size")
+    return n.value
+
+
+def subtree_split(out, grid: Grid, n_pairs: int, theta: float, split, ws, var_out=None, stream=None):
+    """emr_subtree_split: split plane from the variance over each cell's depth-D descendants."""
+    _check(lib().emr_subtree_split(_ptr(out), C.byref(grid), n_pairs, theta, _ptr(split), _ptr(var_out), _ptr(ws),
+                                   C.c_size_t(ws.numel()), _stream(stream)), "emr_subtree_split")
+
+
+def scale_weights(w, offsets, n_pairs: int, cap: int, w_thr: float, w_max: float, stream=None):
+    """emr_scale_weights: HyperNEAT's thresholded linear weight scaling of list weights, in place."""
+    _check(lib().emr_scale_weights(_ptr(w), _ptr(offsets), n_pairs, cap, w_thr, w_max, _stream(stream)),
+           "emr_scale_weights")
 
 
 def conn_types(idx, offsets, query: Query, grid: Grid, n_pairs: int, cap: int, type_out, stream=None):

@@ -1,5 +1,6 @@
 // Host side of libemr: grid descriptor (Eq. 1), genome packer, status strings.
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <thread>
 #include <utility>
@@ -29,9 +30,9 @@ int act_cost(int a) {
   return (a >= 0 && a < 6) ? c[a] : 8;
 }
 
+// A genome's packed record; its nodes and edges are appended to its thread's
+// arrays (node_beg / edge_beg are positions there until the blob is assembled).
 struct GenomeOut {
-  std::vector<PackNode> nodes;
-  std::vector<PackEdge> edges;
   PackGenome g{};
 };
 
@@ -50,9 +51,15 @@ struct Scratch {
   std::vector<unsigned> has_in;
   std::vector<int> in_cnt, in_beg;
   std::vector<PackEdge> in_edges;
+  std::vector<int> table;  // id - id_min -> local index (-1: none), when the ids span a small range
+  int64_t id_min = 0;
 };
 
 int local_of(const Scratch& S, int32_t id) {
+  if (!S.table.empty()) {  // ids span a small range: direct lookup
+    const int64_t k = int64_t(id) - S.id_min;
+    return (k >= 0 && k < int64_t(S.table.size())) ? S.table[size_t(k)] : -1;
+  }
   auto it = std::lower_bound(S.ids.begin(), S.ids.end(), std::make_pair(id, -1));
   return (it != S.ids.end() && it->first == id) ? it->second : -1;
 }
@@ -76,7 +83,8 @@ void build_csr(int n, const std::vector<Edge>& es, bool by_src, std::vector<int>
 emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_t* node_id,
                     const int32_t* node_kind, const int32_t* node_act, const float* node_bias,
                     const int32_t* conn_src, const int32_t* conn_dst, const float* conn_w,
-                    const uint8_t* conn_en, Scratch& S, GenomeOut* out) {
+                    const uint8_t* conn_en, Scratch& S, std::vector<PackNode>& nodes,
+                    std::vector<PackEdge>& edges, GenomeOut* out) {
   const int n = int(n1 - n0);
   if (n <= 0 || n > 1 << 20) return EMR_ERR_ARG;
   S.ids.clear();
@@ -95,6 +103,13 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
   std::sort(S.ids.begin(), S.ids.end());
   for (size_t k = 1; k < S.ids.size(); k++)
     if (S.ids[k].first == S.ids[k - 1].first) return EMR_ERR_ARG;  // duplicate id
+  S.table.clear();
+  const int64_t span = int64_t(S.ids.back().first) - S.ids.front().first + 1;
+  if (span <= 4 * int64_t(n) + 64) {
+    S.id_min = S.ids.front().first;
+    S.table.assign(size_t(span), -1);
+    for (auto& pr : S.ids) S.table[size_t(int64_t(pr.first) - S.id_min)] = pr.second;
+  }
   S.es.clear();
   for (int64_t c = c0; c < c1; c++) {
     if (!conn_en[c]) continue;
@@ -143,20 +158,22 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
   if (S.kept.empty() || S.kept.back() != out_node) return EMR_ERR_ARG;  // output must be last
   if (S.kept.size() > 65535) return EMR_ERR_RANGE;
   const int nk = int(S.kept.size());
-  out->nodes.assign(nk, PackNode{});
+  const size_t nb = nodes.size();
+  nodes.resize(nb + size_t(nk));  // value-initialised records
+  PackNode* on = nodes.data() + nb;
   S.has_in.assign(nk, 0);  // bit k: has an enabled in-connection from input kind k
   S.in_cnt.assign(nk, 0);
   for (int t = 0; t < nk; t++) {
     const int v = S.kept[t];
-    out->nodes[t].act = uint8_t(node_act[n0 + v]);
-    out->nodes[t].bias = node_bias[n0 + v];
+    on[t].act = uint8_t(node_act[n0 + v]);
+    on[t].bias = node_bias[n0 + v];
   }
   for (auto& e : S.es) {
     const int t = S.slot[e.d];
     if (t < 0) continue;
     const int sk = node_kind[n0 + e.s];
     if (sk < EMR_KIND_HIDDEN) {
-      out->nodes[t].w_in[sk] += e.w;
+      on[t].w_in[sk] += e.w;
       S.has_in[t] |= 1u << sk;
     } else {
       if (S.slot[e.s] < 0) return EMR_ERR_ARG;  // cannot happen: a source of a kept node is kept
@@ -167,21 +184,25 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
   S.in_beg.assign(nk + 1, 0);
   for (int t = 0; t < nk; t++) S.in_beg[t + 1] = S.in_beg[t] + S.in_cnt[t];
   if (S.in_beg[nk] > 65535) return EMR_ERR_RANGE;
-  out->edges.resize(size_t(S.in_beg[nk]));
+  const size_t eb = edges.size();
+  edges.resize(eb + size_t(S.in_beg[nk]));
+  PackEdge* oe = edges.data() + eb;
   S.fill.assign(nk, 0);
   for (auto& e : S.es) {
     const int t = S.slot[e.d];
     if (t < 0 || node_kind[n0 + e.s] < EMR_KIND_HIDDEN) continue;
-    out->edges[S.in_beg[t] + S.fill[t]++] = PackEdge{uint16_t(S.slot[e.s]), 0, e.w};
+    oe[S.in_beg[t] + S.fill[t]++] = PackEdge{uint16_t(S.slot[e.s]), 0, e.w};
   }
   PackGenome& g = out->g;
   g = PackGenome{};
+  g.node_beg = uint32_t(nb);
+  g.edge_beg = uint32_t(eb);
   g.n_nodes = uint16_t(nk);
   for (int t = 0; t < nk; t++) {
-    out->nodes[t].edge_beg = uint16_t(S.in_beg[t]);
-    out->nodes[t].edge_cnt = uint16_t(S.in_cnt[t]);
+    on[t].edge_beg = uint16_t(S.in_beg[t]);
+    on[t].edge_cnt = uint16_t(S.in_cnt[t]);
   }
-  g.n_edges = uint16_t(out->edges.size());
+  g.n_edges = uint16_t(S.in_beg[nk]);
   for (int side = 0; side < 2; side++) {
     const unsigned grid_inputs = side == EMR_SIDE_OUT ? (1u << EMR_KIND_X2) | (1u << EMR_KIND_Y2)
                                                       : (1u << EMR_KIND_X1) | (1u << EMR_KIND_Y1);
@@ -191,12 +212,12 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
       bool vary = (S.has_in[t] & grid_inputs) != 0;
       int vin = 0;
       for (int k = S.in_beg[t]; k < S.in_beg[t + 1]; k++)
-        if (out->nodes[out->edges[k].src].vary & (1u << side)) { vary = true; vin++; }
+        if (on[oe[k].src].vary & (1u << side)) { vary = true; vin++; }
       if (vary) {
-        out->nodes[t].vary |= uint8_t(1u << side);
+        on[t].vary |= uint8_t(1u << side);
         nv++;
         nve += vin;
-        cost += 2 + vin + act_cost(out->nodes[t].act);
+        cost += 2 + vin + act_cost(on[t].act);
       }
     }
     if (nv > EMR_MAX_VARYING || nve > EMR_MAX_VEDGES) return EMR_ERR_RANGE;
@@ -267,17 +288,23 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
   // Genomes are independent: pack them on several host threads, each with its
   // own scratch; the lowest failing genome index is reported.
   const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
-  const int n_threads = P >= 256 ? std::min(hw, 16) : 1;
+  // a thread costs about as much to start as packing ~16 genomes: sqrt(P / 16) threads balance the two
+  const int n_threads = std::max(1, std::min({hw, 16, int(std::sqrt(double(P) / 16.0))}));
   std::vector<emr_status> t_rc(n_threads, EMR_OK);
   std::vector<int32_t> t_bad(n_threads, -1);
+  std::vector<std::vector<PackNode>> t_nodes(n_threads);
+  std::vector<std::vector<PackEdge>> t_edges(n_threads);
+  auto g_lo = [&](int t) { return int(int64_t(P) * t / n_threads); };
   auto work = [&](int t) {
     Scratch scratch;
-    for (int g = int(int64_t(P) * t / n_threads); g < int(int64_t(P) * (t + 1) / n_threads); g++) {
+    const int64_t n_lo = node_ptr[g_lo(t)], n_hi = node_ptr[g_lo(t + 1)];
+    t_nodes[t].reserve(size_t(std::max<int64_t>(0, n_hi - n_lo)));
+    for (int g = g_lo(t); g < g_lo(t + 1); g++) {
       emr_status rc = EMR_OK;
       if (node_ptr[g + 1] < node_ptr[g] || conn_ptr[g + 1] < conn_ptr[g]) rc = EMR_ERR_ARG;
       if (rc == EMR_OK)
         rc = pack_one(node_ptr[g], node_ptr[g + 1], conn_ptr[g], conn_ptr[g + 1], node_id, node_kind, node_act,
-                      node_bias, conn_src, conn_dst, conn_w, conn_enabled, scratch, &gs[g]);
+                      node_bias, conn_src, conn_dst, conn_w, conn_enabled, scratch, t_nodes[t], t_edges[t], &gs[g]);
       if (rc != EMR_OK) {
         t_rc[t] = rc;
         t_bad[t] = g;
@@ -298,7 +325,13 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
       return t_rc[t];
     }
   size_t nn = 0, ne = 0;
-  for (auto& g : gs) { nn += g.nodes.size(); ne += g.edges.size(); }
+  std::vector<size_t> t_nb(n_threads), t_eb(n_threads);  // each thread's first node / edge in the blob
+  for (int t = 0; t < n_threads; t++) {
+    t_nb[t] = nn;
+    t_eb[t] = ne;
+    nn += t_nodes[t].size();
+    ne += t_edges[t].size();
+  }
   PackHeader h{};
   h.magic = kPackMagic;
   h.version = kPackVersion;
@@ -314,15 +347,17 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
   auto* gt = reinterpret_cast<PackGenome*>(base + h.off_genomes);
   auto* nt = reinterpret_cast<PackNode*>(base + h.off_nodes);
   auto* et = reinterpret_cast<PackEdge*>(base + h.off_edges);
-  uint32_t nb = 0, eb = 0;
+  for (int t = 0; t < n_threads; t++) {
+    if (!t_nodes[t].empty()) std::memcpy(nt + t_nb[t], t_nodes[t].data(), t_nodes[t].size() * sizeof(PackNode));
+    if (!t_edges[t].empty()) std::memcpy(et + t_eb[t], t_edges[t].data(), t_edges[t].size() * sizeof(PackEdge));
+  }
+  for (int t = 0; t < n_threads; t++)
+    for (int g = g_lo(t); g < g_lo(t + 1); g++) {
+      gs[g].g.node_beg += uint32_t(t_nb[t]);
+      gs[g].g.edge_beg += uint32_t(t_eb[t]);
+    }
   for (int g = 0; g < P; g++) {
-    PackGenome pg = gs[g].g;
-    pg.node_beg = nb;
-    pg.edge_beg = eb;
-    std::copy(gs[g].nodes.begin(), gs[g].nodes.end(), nt + nb);
-    std::copy(gs[g].edges.begin(), gs[g].edges.end(), et + eb);
-    nb += uint32_t(gs[g].nodes.size());
-    eb += uint32_t(gs[g].edges.size());
+    const PackGenome pg = gs[g].g;
     gt[g] = pg;
     h.max_nodes = std::max<int32_t>(h.max_nodes, pg.n_nodes);
     h.max_edges = std::max<int32_t>(h.max_edges, pg.n_edges);

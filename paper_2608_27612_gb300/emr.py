@@ -147,7 +147,7 @@ def pack_population(pop) -> np.ndarray:
     L = lib()
     n = C.c_size_t()
     _check(L.emr_pack_size(pop.P, _ptr(pop.node_ptr), _ptr(pop.conn_ptr), C.byref(n)), "emr_pack_size")
-    buf = np.zeros(n.value + 16, np.uint8)
+    buf = np.empty(n.value + 16, np.uint8)   # the packer clears what it uses
     used, bad = C.c_size_t(), C.c_int32()
     st = L.emr_pack_population(pop.P, _ptr(pop.node_ptr), _ptr(pop.node_id), _ptr(pop.node_kind),
                                _ptr(pop.node_act), _ptr(pop.node_bias), _ptr(pop.conn_ptr), _ptr(pop.conn_src),
@@ -157,7 +157,7 @@ def pack_population(pop) -> np.ndarray:
         e = EmrError(st, "emr_pack_population (genome %d)" % bad.value)
         e.bad_genome = bad.value
         raise e
-    return buf[:used.value].copy()
+    return buf[:used.value]
 
 
 def pack_info(pack: np.ndarray):

@@ -363,16 +363,16 @@ def variants_run(emr, torch, W, D=7, P=1000, reps=10):
 
 def launches_in_step(emr, dsc):
     """Kernel launches of one step: prepare (schedule, records), one tile launch per
-    non-empty kernel class, one zeroing launch for constant-output pairs, selection
-    (count, scan, write with the kept weights); the tile flags' memset is not a kernel."""
+    non-empty kernel class (constant-output pairs need none: their tiles hold no band
+    bit), selection (count, scan, write, kept weights); the tile flags' memset is not a
+    kernel."""
     _, gs, _, _ = emr.pack_records(dsc.pack)
     side = np.asarray(dsc.query.side)
     nv = gs["n_varying"][:, side] if not dsc.query.per_genome else \
         np.take_along_axis(gs["n_varying"], side.reshape(gs.shape[0], -1), axis=1)
     nv = nv.astype(np.int64)
     cls = np.where(nv > 12, 0, np.where(nv > 8, 1, np.where(nv > 4, 2, 3)))
-    # constant-output pairs get a zeroing kernel instead of a tile launch
-    return 2 + len(np.unique(cls[nv > 0])) + int(np.any(nv == 0)) + 3
+    return 2 + len(np.unique(cls[nv > 0])) + 4
 
 
 def oracle_baseline(w, genomes):

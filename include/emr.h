@@ -366,7 +366,11 @@ emr_status emr_compact_records(const uint32_t *mask, const void *pack_host, cons
  * [n_pairs][n_dense], 1 where the tile holds a band-passing position, else 0.
  * Dense tiles: tile 0 holds depths 0..min(D, 4); tile t >= 1 is the t-th 64 x 64
  * Morton block of depths 5..D in global-index order (n_dense = 1 + the number of
- * such blocks). For emr_select. Errors as emr_eval_filter. */
+ * such blocks). For emr_select, which reads the planes only in flagged tiles: a
+ * pair whose output is constant over the grid (every variance and band value 0)
+ * has no flag set, and its rows of split and band_bits are left untouched (use
+ * emr_eval_filter where the planes themselves are wanted). Errors as
+ * emr_eval_filter. */
 emr_status emr_eval_filter_tiles(const void *pack_host, const emr_query *q, const emr_grid *grid, float theta,
                                  float band, float w_min, uint32_t *split, uint32_t *band_bits,
                                  uint8_t *tile_flags, void *ws, size_t ws_bytes, void *stream);

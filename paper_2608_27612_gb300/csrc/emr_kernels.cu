@@ -1435,70 +1435,109 @@ __device__ __forceinline__ void tile_words(const GridDev& G, int32_t t, int64_t*
   }
 }
 
+// One warp per pair (kSelectThreads / 32 pairs a CTA): the flags are read 32 at a
+// time and the flagged tiles taken in ascending order from the ballot; scans are
+// warp shuffles, so no CTA barrier is needed. Every loop is warp-uniform.
+
+__device__ __forceinline__ int warp_exclusive_scan(int v, int* total) {
+  const int lane = threadIdx.x & 31;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, o);
+    if (lane >= o) x += y;
+  }
+  *total = __shfl_sync(kFull, x, 31);
+  return x - v;
+}
+
 __global__ void __launch_bounds__(kSelectThreads) select_count_kernel(const uint32_t* __restrict__ split,
                                                                       const uint32_t* __restrict__ bandb,
                                                                       const uint8_t* __restrict__ flags,
                                                                       int64_t n_dense, GridDev G, int gated,
-                                                                      TypeFilter tf, int64_t* __restrict__ counts) {
-  __shared__ int sh[32];
-  const int64_t r = blockIdx.x;
+                                                                      TypeFilter tf, int64_t n_pairs,
+                                                                      int64_t* __restrict__ counts) {
+  const int lane = threadIdx.x & 31;
+  const int64_t r = (int64_t(blockIdx.x) * kSelectThreads + threadIdx.x) >> 5;
+  if (r >= n_pairs) return;  // whole warps
   const uint32_t* sp = split + r * G.n_words;
   const uint32_t* bw = bandb + r * G.n_words;
   int sum = 0;
-  for (int64_t t = 0; t < n_dense; t++) {
-    if (!flags[r * n_dense + t]) continue;
-    int64_t wb, we;
-    tile_words(G, int32_t(t), &wb, &we);
-    for (int64_t wi = wb + 4 * threadIdx.x; wi < we; wi += 4 * kSelectThreads) {
-      uint32_t m[4];
-      combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
-      sum += __popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]);
+  for (int64_t t0 = 0; t0 < n_dense; t0 += 32) {
+    const int64_t t = t0 + lane;
+    uint32_t bal = __ballot_sync(kFull, t < n_dense && flags[r * n_dense + t]);
+    for (; bal; bal &= bal - 1) {
+      int64_t wb, we;
+      tile_words(G, int32_t(t0 + __ffs(bal) - 1), &wb, &we);
+      for (int64_t wi = wb + 4 * lane; wi < we; wi += 128) {
+        uint32_t m[4];
+        combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
+        sum += __popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]);
+      }
     }
   }
-  int total;
-  block_exclusive_scan(sum, sh, &total);
-  if (threadIdx.x == 0) counts[r] = total;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(kFull, sum, o);
+  if (lane == 0) counts[r] = sum;
 }
 
 __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint32_t* __restrict__ split,
                                                                       const uint32_t* __restrict__ bandb,
                                                                       const uint8_t* __restrict__ flags,
                                                                       int64_t n_dense, GridDev G, int gated,
-                                                                      TypeFilter tf, RecordSource rs,
+                                                                      TypeFilter tf, int64_t n_pairs,
+                                                                      RecordSource rs,
                                                                       const int64_t* __restrict__ offsets,
                                                                       int64_t cap, int32_t* __restrict__ idx,
                                                                       float* __restrict__ wv) {
-  __shared__ int sh[32];
-  const int64_t r = blockIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int64_t r = (int64_t(blockIdx.x) * kSelectThreads + threadIdx.x) >> 5;
+  if (r >= n_pairs) return;  // whole warps
   const uint32_t* sp = split + r * G.n_words;
   const uint32_t* bw = bandb + r * G.n_words;
   int64_t base = offsets[r];
-  for (int64_t t = 0; t < n_dense; t++) {
-    if (!flags[r * n_dense + t]) continue;
-    int64_t wb, we;
-    tile_words(G, int32_t(t), &wb, &we);
-    for (int64_t w0 = wb; w0 < we; w0 += 4 * kSelectThreads) {  // block-uniform loop
-      const int64_t wi = w0 + 4 * threadIdx.x;
-      uint32_t m[4] = {0u, 0u, 0u, 0u};
-      if (wi < we) combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
-      int total;
-      const int ex = block_exclusive_scan(__popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]), sh, &total);
-      int64_t dst = base + ex;
-      for (int c = 0; c < 4; c++) {
-        if (!m[c]) continue;
-        int d = 0;
-        while (G.word_off[d + 1] <= wi + c) d++;
-        const int64_t gbase = G.level_off[d] + (wi + c - G.word_off[d]) * 32;
-        for (uint32_t v = m[c]; v; v &= v - 1, dst++)
-          if (dst < cap) idx[dst] = int32_t(gbase + __ffs(v) - 1);
+  for (int64_t t0 = 0; t0 < n_dense; t0 += 32) {
+    const int64_t t = t0 + lane;
+    uint32_t bal = __ballot_sync(kFull, t < n_dense && flags[r * n_dense + t]);
+    for (; bal; bal &= bal - 1) {
+      int64_t wb, we;
+      tile_words(G, int32_t(t0 + __ffs(bal) - 1), &wb, &we);
+      for (int64_t w0 = wb; w0 < we; w0 += 128) {
+        const int64_t wi = w0 + 4 * lane;
+        uint32_t m[4] = {0u, 0u, 0u, 0u};
+        if (wi < we) combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
+        int total;
+        const int ex = warp_exclusive_scan(__popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]), &total);
+        int64_t dst = base + ex;
+        for (int c = 0; c < 4; c++) {
+          if (!m[c]) continue;
+          int d = 0;
+          while (G.word_off[d + 1] <= wi + c) d++;
+          const int64_t gbase = G.level_off[d] + (wi + c - G.word_off[d]) * 32;
+          for (uint32_t v = m[c]; v; v &= v - 1, dst++)
+            if (dst < cap) {
+              idx[dst] = int32_t(gbase + __ffs(v) - 1);
+              if (wv) wv[dst] = __int_as_float(int32_t(r));  // the pair, for select_weights_kernel
+            }
+        }
+        base += total;
       }
-      base += total;
     }
   }
-  if (!wv) return;
-  __syncthreads();  // this pair's indices are written
-  const int64_t end = offsets[r + 1] < cap ? offsets[r + 1] : cap;
-  for (int64_t e = offsets[r] + threadIdx.x; e < end; e += kSelectThreads) {
+}
+
+// Kept weights of the selected entries, one entry per thread: the write kernel
+// left each entry's pair number in its weight slot (pairs have very unequal
+// list lengths, so a warp per pair would leave a few long lists on the tail).
+__global__ void __launch_bounds__(kCompactBlock) select_weights_kernel(RecordSource rs, GridDev G,
+                                                                       const int64_t* __restrict__ offsets,
+                                                                       int64_t n_pairs, int64_t cap,
+                                                                       const int32_t* __restrict__ idx,
+                                                                       float* __restrict__ wv) {
+  const int64_t total = offsets[n_pairs] < cap ? offsets[n_pairs] : cap;
+  for (int64_t e = int64_t(blockIdx.x) * kCompactBlock + threadIdx.x; e < total;
+       e += int64_t(gridDim.x) * kCompactBlock) {
+    const int64_t r = __float_as_int(wv[e]);
     const int64_t gidx = idx[e];
     int d = 0;
     while (G.level_off[d + 1] <= gidx) d++;
@@ -1817,10 +1856,14 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   beg += p.n_class[2];
   if (mode != kModeFused || p.n_const == 0) return launch_dense<4>(D, beg, p.n_class[3], st);
   if ((rc = launch_dense<4>(D, beg, p.n_class[3] - p.n_const, st)) != EMR_OK) return rc;
+  // with tile flags, a constant-output pair has none set and its planes are never read: leave them
+  if (tile_flags) return EMR_OK;
   const int64_t c0 = beg + p.n_class[3] - p.n_const;
   for (int64_t r0 = 0; r0 < p.n_const; r0 += 65535) {  // grid y: pairs, at most 65535 a launch
     D.rank_beg = c0 + r0;
-    const dim3 grid(unsigned(std::min<int64_t>(D.n_tiles, 64)), unsigned(std::min<int64_t>(65535, p.n_const - r0)));
+    const int64_t nc = std::min<int64_t>(65535, p.n_const - r0);
+    const int64_t gx = std::max<int64_t>(1, std::min<int64_t>(D.n_tiles, 64));
+    const dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(nc));
     zero_tiles_kernel<<<grid, 128, 0, st>>>(D);
   }
   return cuda_status(cudaGetLastError());
@@ -2118,12 +2161,22 @@ emr_status emr_select(const uint32_t* split, const uint32_t* band_bits, const ui
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const GridDev G = grid_dev(grid);
   const int64_t n_dense = dense_tiles(grid->D);
-  select_count_kernel<<<unsigned(p.n_pairs), kSelectThreads, 0, st>>>(split, band_bits, tile_flags, n_dense, G,
-                                                                       mode == EMR_GATED, tf, counts);
+  const unsigned blocks = unsigned((p.n_pairs + kSelectThreads / 32 - 1) / (kSelectThreads / 32));
+  select_count_kernel<<<blocks, kSelectThreads, 0, st>>>(split, band_bits, tile_flags, n_dense, G,
+                                                         mode == EMR_GATED, tf, p.n_pairs, counts);
   compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, p.n_pairs, offsets);
-  select_write_kernel<<<unsigned(p.n_pairs), kSelectThreads, 0, st>>>(
-      split, band_bits, tile_flags, n_dense, G, mode == EMR_GATED, tf,
-      RecordSource{static_cast<const uint8_t*>(eval_ws), p.L}, offsets, cap, idx, w);
+  select_write_kernel<<<blocks, kSelectThreads, 0, st>>>(split, band_bits, tile_flags, n_dense, G,
+                                                         mode == EMR_GATED, tf, p.n_pairs,
+                                                         RecordSource{static_cast<const uint8_t*>(eval_ws), p.L},
+                                                         offsets, cap, idx, w);
+  if (w && cap > 0) {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return EMR_ERR_CUDA;
+    select_weights_kernel<<<unsigned(8 * sms), kCompactBlock, 0, st>>>(
+        RecordSource{static_cast<const uint8_t*>(eval_ws), p.L}, G, offsets, p.n_pairs, cap, idx, w);
+  }
   return cuda_status(cudaGetLastError());
 }
 

@@ -240,10 +240,17 @@ __global__ void schedule_kernel(const uint8_t* __restrict__ pack, QueryDev q, in
 // One thread per pair: fold the constant inputs (the slot's node coordinates
 // and the bias) and every node that does not vary over the grid into per-node
 // constants; list the edges between varying nodes.
-__global__ void spec_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_t n_pairs, SpecLayout L,
-                            uint8_t* __restrict__ spec, float* __restrict__ scratch, int32_t scratch_stride) {
-  int64_t r = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (r >= n_pairs) return;
+constexpr int kSpecWarps = 4;   // pairs per CTA: a warp per pair
+constexpr int kSpecSmemNodes = 128;  // genomes up to this many kept nodes keep their values in shared memory
+
+__global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __restrict__ pack, QueryDev q,
+                                                               int64_t n_pairs, SpecLayout L,
+                                                               uint8_t* __restrict__ spec,
+                                                               float* __restrict__ scratch, int32_t scratch_stride) {
+  __shared__ float s_cval[kSpecWarps][kSpecSmemNodes];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int64_t r = int64_t(blockIdx.x) * kSpecWarps + wid;
+  if (r >= n_pairs) return;  // whole warps
   const PackHeader* h = reinterpret_cast<const PackHeader*>(pack);
   const PackGenome* gt = reinterpret_cast<const PackGenome*>(pack + h->off_genomes);
   const PackNode* nt = reinterpret_cast<const PackNode*>(pack + h->off_nodes);
@@ -252,70 +259,76 @@ __global__ void spec_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_
   uint8_t* rec = spec + r * L.stride;
   int32_t* hdr = reinterpret_cast<int32_t*>(rec);
   if (q.per_genome && q.count && s >= q.count[g]) {  // unused slot: constant 0, nothing kept
-    hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = pair_class(0);
+    if (lane == 0) { hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = pair_class(0); }
     return;
   }
-  int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
-  const int side = q.side[si] ? 1 : 0;
-  const float a = q.a[si], b = q.b[si];
-  // constant inputs of this side (grid inputs contribute through wx, wy)
-  float in[5] = {0.f, 0.f, 0.f, 0.f, 1.f};
-  int gx, gy;
-  if (side == EMR_SIDE_OUT) { in[EMR_KIND_X1] = a; in[EMR_KIND_Y1] = b; gx = EMR_KIND_X2; gy = EMR_KIND_Y2; }
-  else { in[EMR_KIND_X2] = a; in[EMR_KIND_Y2] = b; gx = EMR_KIND_X1; gy = EMR_KIND_Y1; }
   const PackGenome G = gt[g];
-  float* cval = scratch + r * scratch_stride;  // const value, or varying slot (as int bits)
-  float4* coef = reinterpret_cast<float4*>(rec + L.coef_off());
-  uint2* ve = reinterpret_cast<uint2*>(rec + L.edge_off());
   int nv = 0, nve = 0;
-  float out_const = 0.f;
-  for (int t = 0; t < G.n_nodes; t++) {
-    const PackNode nd = nt[G.node_beg + t];
-    const PackEdge* ed = et + G.edge_beg + nd.edge_beg;
-    if (nd.vary & (1u << side)) {
-      float c0 = nd.bias;
-      for (int k = 0; k < 5; k++)
-        if (k != gx && k != gy) c0 = fmaf(nd.w_in[k], in[k], c0);
-      int eb = nve;
-      for (int e = 0; e < nd.edge_cnt; e++) {
-        const PackNode src = nt[G.node_beg + ed[e].src];
-        if (src.vary & (1u << side)) {
-          ve[nve++] = make_uint2(__float_as_uint(cval[ed[e].src]), __float_as_uint(ed[e].w));
-        } else {
-          c0 = fmaf(ed[e].w, cval[ed[e].src], c0);
+  if (lane == 0) {  // the node loop is sequential (each node folds the constants of its sources)
+    int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
+    const int side = q.side[si] ? 1 : 0;
+    const float a = q.a[si], b = q.b[si];
+    float in[5] = {0.f, 0.f, 0.f, 0.f, 1.f};
+    int gx, gy;
+    if (side == EMR_SIDE_OUT) { in[EMR_KIND_X1] = a; in[EMR_KIND_Y1] = b; gx = EMR_KIND_X2; gy = EMR_KIND_Y2; }
+    else { in[EMR_KIND_X2] = a; in[EMR_KIND_Y2] = b; gx = EMR_KIND_X1; gy = EMR_KIND_Y1; }
+    float* cval = G.n_nodes <= kSpecSmemNodes ? s_cval[wid] : scratch + r * scratch_stride;
+    float4* coef = reinterpret_cast<float4*>(rec + L.coef_off());
+    uint2* ve = reinterpret_cast<uint2*>(rec + L.edge_off());
+    float out_const = 0.f;
+    for (int t = 0; t < G.n_nodes; t++) {
+      const PackNode nd = nt[G.node_beg + t];
+      const PackEdge* ed = et + G.edge_beg + nd.edge_beg;
+      if (nd.vary & (1u << side)) {
+        float c0 = nd.bias;
+        for (int k = 0; k < 5; k++)
+          if (k != gx && k != gy) c0 = fmaf(nd.w_in[k], in[k], c0);
+        int eb = nve;
+        for (int e = 0; e < nd.edge_cnt; e++) {
+          const PackNode src = nt[G.node_beg + ed[e].src];
+          if (src.vary & (1u << side)) {
+            ve[nve++] = make_uint2(__float_as_uint(cval[ed[e].src]), __float_as_uint(ed[e].w));
+          } else {
+            c0 = fmaf(ed[e].w, cval[ed[e].src], c0);
+          }
         }
+        for (int e = eb + 1; e < nve; e++) {  // ascending source slot (insertion sort, a few edges)
+          const uint2 key = ve[e];
+          int f = e - 1;
+          while (f >= eb && ve[f].x > key.x) { ve[f + 1] = ve[f]; f--; }
+          ve[f + 1] = key;
+        }
+        uint32_t info = uint32_t(nd.act) | (uint32_t(eb) << 8) | (uint32_t(nve - eb) << 20);
+        coef[nv] = make_float4(c0, nd.w_in[gx], nd.w_in[gy], __uint_as_float(info));
+        cval[t] = __uint_as_float(uint32_t(nv));
+        nv++;
+      } else {
+        float z = nd.bias;
+        for (int k = 0; k < 5; k++) z = fmaf(nd.w_in[k], in[k], z);
+        for (int e = 0; e < nd.edge_cnt; e++) z = fmaf(ed[e].w, cval[ed[e].src], z);
+        cval[t] = act_apply(nd.act, z);
+        out_const = cval[t];
       }
-      for (int e = eb + 1; e < nve; e++) {  // ascending source slot (insertion sort, a few edges)
-        const uint2 key = ve[e];
-        int f = e - 1;
-        while (f >= eb && ve[f].x > key.x) { ve[f + 1] = ve[f]; f--; }
-        ve[f + 1] = key;
-      }
-      uint32_t info = uint32_t(nd.act) | (uint32_t(eb) << 8) | (uint32_t(nve - eb) << 20);
-      coef[nv] = make_float4(c0, nd.w_in[gx], nd.w_in[gy], __uint_as_float(info));
-      cval[t] = __uint_as_float(uint32_t(nv));
-      nv++;
-    } else {
-      float z = nd.bias;
-      for (int k = 0; k < 5; k++) z = fmaf(nd.w_in[k], in[k], z);
-      for (int e = 0; e < nd.edge_cnt; e++) z = fmaf(ed[e].w, cval[ed[e].src], z);
-      cval[t] = act_apply(nd.act, z);
-      out_const = cval[t];
     }
+    hdr[0] = nv;
+    hdr[1] = nve;
+    reinterpret_cast<float*>(hdr)[2] = out_const;
+    hdr[3] = pair_class(nv);
   }
-  if (nv <= kDenseMax) {
+  nv = __shfl_sync(0xffffffffu, nv, 0);
+  __syncwarp();  // lane 0's coefficient and edge records are visible to the warp
+  if (nv <= kDenseMax) {  // the dense block: zeroed, then the edges added, by the warp's lanes
     float* W = reinterpret_cast<float*>(rec + L.dense_off());
-    for (int k = 0; k < kDenseMax * kDenseMax; k++) W[k] = 0.f;
-    for (int k = 0; k < nv; k++) {
-      const uint32_t info = __float_as_uint(coef[k].w);
+    for (int k = lane; k < kDenseMax * kDenseMax; k += 32) W[k] = 0.f;
+    __syncwarp();
+    if (lane < nv) {  // lane k fills row k (its edges in order, duplicates summed as before)
+      const float4* coef = reinterpret_cast<const float4*>(rec + L.coef_off());
+      const uint2* ve = reinterpret_cast<const uint2*>(rec + L.edge_off());
+      const uint32_t info = __float_as_uint(coef[lane].w);
       const int eb = int((info >> 8) & 0xfffu), ec = int(info >> 20);
-      for (int e = eb; e < eb + ec; e++) W[k * kDenseMax + int(ve[e].x)] += __uint_as_float(ve[e].y);
+      for (int e = eb; e < eb + ec; e++) W[lane * kDenseMax + int(ve[e].x)] += __uint_as_float(ve[e].y);
     }
   }
-  hdr[0] = nv;
-  hdr[1] = nve;
-  reinterpret_cast<float*>(hdr)[2] = out_const;
-  hdr[3] = pair_class(nv);
 }
 
 // ---- evaluation tiles ------------------------------------------------------------
@@ -1720,8 +1733,8 @@ emr_status prepare(const void* pack_dev, const emr_query* q, const EvalPlan& p, 
   const QueryDev qd = query_dev(q);
   const uint8_t* pk = static_cast<const uint8_t*>(pack_dev);
   schedule_kernel<<<1, 1024, 0, st>>>(pk, qd, p.n_pairs, *order);
-  spec_kernel<<<unsigned((p.n_pairs + 31) / 32), 32, 0, st>>>(pk, qd, p.n_pairs, p.L, *spec, scratch,
-                                                                 p.scratch_stride);
+  spec_kernel<<<unsigned((p.n_pairs + kSpecWarps - 1) / kSpecWarps), 32 * kSpecWarps, 0, st>>>(
+      pk, qd, p.n_pairs, p.L, *spec, scratch, p.scratch_stride);
   return cuda_status(cudaGetLastError());
 }
 

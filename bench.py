@@ -362,7 +362,7 @@ def variants_run(emr, torch, W, D=7, P=1000, reps=10):
 
 
 def launches_in_step(emr, dsc):
-    """Kernel launches of one step: prepare (schedule, records), one tile launch per
+    """Kernel launches of one step: prepare (records, with the schedule in one CTA), one tile launch per
     non-empty kernel class (constant-output pairs need none: their tiles hold no band
     bit), selection (count, scan, write, kept weights); the tile flags' memset is not a
     kernel."""
@@ -372,7 +372,7 @@ def launches_in_step(emr, dsc):
         np.take_along_axis(gs["n_varying"], side.reshape(gs.shape[0], -1), axis=1)
     nv = nv.astype(np.int64)
     cls = np.where(nv > 12, 0, np.where(nv > 8, 1, np.where(nv > 4, 2, 3)))
-    return 2 + len(np.unique(cls[nv > 0])) + 4
+    return 1 + len(np.unique(cls[nv > 0])) + 4
 
 
 def oracle_baseline(w, genomes):

@@ -195,13 +195,15 @@ struct QueryDev {
 // estimated cost, heaviest first; a counting sort in one CTA.
 constexpr int kClassBins = 256;
 constexpr int kCostBins = kClasses * kClassBins;
-__global__ void schedule_kernel(const uint8_t* __restrict__ pack, QueryDev q, int64_t n_pairs,
-                                int32_t* __restrict__ order) {
-  __shared__ int32_t hist[kCostBins];
-  __shared__ int32_t wsum[32];
+// Pair schedule (order[rank] = pair): class-major, heaviest estimated cost first,
+// by a counting sort over kCostBins bins, run by one CTA of nthreads threads
+// (a multiple of 32, at most 1024; each thread scans kCostBins / nthreads bins).
+__device__ void schedule_block(const uint8_t* __restrict__ pack, QueryDev q, int64_t n_pairs,
+                               int32_t* __restrict__ order, int32_t* hist, int32_t* wsum) {
+  const int nthreads = blockDim.x, tid = threadIdx.x;
   const PackHeader* h = reinterpret_cast<const PackHeader*>(pack);
   const PackGenome* gt = reinterpret_cast<const PackGenome*>(pack + h->off_genomes);
-  for (int k = threadIdx.x; k < kCostBins; k += blockDim.x) hist[k] = 0;
+  for (int k = tid; k < kCostBins; k += nthreads) hist[k] = 0;
   __syncthreads();
   auto bin_of = [&](int64_t r) {
     const int g = int(r / q.S), s = int(r % q.S);
@@ -211,12 +213,13 @@ __global__ void schedule_kernel(const uint8_t* __restrict__ pack, QueryDev q, in
     const uint32_t c = min(gt[g].cost[side], uint32_t(kClassBins - 1));
     return pair_class(gt[g].n_varying[side]) * kClassBins + (kClassBins - 1 - int(c));
   };
-  for (int64_t r = threadIdx.x; r < n_pairs; r += blockDim.x) atomicAdd(&hist[bin_of(r)], 1);
+  for (int64_t r = tid; r < n_pairs; r += nthreads) atomicAdd(&hist[bin_of(r)], 1);
   __syncthreads();
-  // exclusive scan of the histogram (blockDim.x == 1024, one bin per thread)
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int v = threadIdx.x < kCostBins ? hist[threadIdx.x] : 0;
-  int x = v;
+  // exclusive scan: thread tid owns bins [tid * per, (tid + 1) * per)
+  const int per = kCostBins / nthreads, lane = tid & 31, warp = tid >> 5;
+  int local = 0;
+  for (int k = 0; k < per; k++) local += hist[tid * per + k];
+  int x = local;
   for (int o = 1; o < 32; o <<= 1) {
     const int y = __shfl_up_sync(0xffffffffu, x, o);
     if (lane >= o) x += y;
@@ -224,7 +227,7 @@ __global__ void schedule_kernel(const uint8_t* __restrict__ pack, QueryDev q, in
   if (lane == 31) wsum[warp] = x;
   __syncthreads();
   if (warp == 0) {
-    int t = wsum[lane];
+    int t = lane < nthreads / 32 ? wsum[lane] : 0;
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xffffffffu, t, o);
       if (lane >= o) t += y;
@@ -232,9 +235,14 @@ __global__ void schedule_kernel(const uint8_t* __restrict__ pack, QueryDev q, in
     wsum[lane] = t;
   }
   __syncthreads();
-  if (threadIdx.x < kCostBins) hist[threadIdx.x] = (warp ? wsum[warp - 1] : 0) + x - v;
+  int run = (warp ? wsum[warp - 1] : 0) + x - local;
+  for (int k = 0; k < per; k++) {
+    const int v = hist[tid * per + k];
+    hist[tid * per + k] = run;
+    run += v;
+  }
   __syncthreads();
-  for (int64_t r = threadIdx.x; r < n_pairs; r += blockDim.x) order[atomicAdd(&hist[bin_of(r)], 1)] = int32_t(r);
+  for (int64_t r = tid; r < n_pairs; r += nthreads) order[atomicAdd(&hist[bin_of(r)], 1)] = int32_t(r);
 }
 
 // One thread per pair: fold the constant inputs (the slot's node coordinates
@@ -246,8 +254,15 @@ constexpr int kSpecSmemNodes = 128;  // genomes up to this many kept nodes keep 
 __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __restrict__ pack, QueryDev q,
                                                                int64_t n_pairs, SpecLayout L,
                                                                uint8_t* __restrict__ spec,
-                                                               float* __restrict__ scratch, int32_t scratch_stride) {
+                                                               float* __restrict__ scratch, int32_t scratch_stride,
+                                                               int32_t* __restrict__ order) {
   __shared__ float s_cval[kSpecWarps][kSpecSmemNodes];
+  __shared__ int32_t s_hist[kCostBins];
+  __shared__ int32_t s_wsum[32];
+  if (blockIdx.x == gridDim.x - 1) {  // the last CTA schedules the pairs while the others build records
+    schedule_block(pack, q, n_pairs, order, s_hist, s_wsum);
+    return;
+  }
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int64_t r = int64_t(blockIdx.x) * kSpecWarps + wid;
   if (r >= n_pairs) return;  // whole warps
@@ -1732,9 +1747,8 @@ emr_status prepare(const void* pack_dev, const emr_query* q, const EvalPlan& p, 
   ws_layout(p, ws, spec, order, &scratch);
   const QueryDev qd = query_dev(q);
   const uint8_t* pk = static_cast<const uint8_t*>(pack_dev);
-  schedule_kernel<<<1, 1024, 0, st>>>(pk, qd, p.n_pairs, *order);
-  spec_kernel<<<unsigned((p.n_pairs + kSpecWarps - 1) / kSpecWarps), 32 * kSpecWarps, 0, st>>>(
-      pk, qd, p.n_pairs, p.L, *spec, scratch, p.scratch_stride);
+  spec_kernel<<<unsigned((p.n_pairs + kSpecWarps - 1) / kSpecWarps + 1), 32 * kSpecWarps, 0, st>>>(
+      pk, qd, p.n_pairs, p.L, *spec, scratch, p.scratch_stride, *order);
   return cuda_status(cudaGetLastError());
 }
 

@@ -440,6 +440,7 @@ def main():
 
     ev = lambda: torch.cuda.Event(enable_timing=True)
     tile_flags = torch.zeros(dsc.n_pairs, emr.dense_tiles(w.D), dtype=torch.uint8, device="cuda")
+    sws = torch.zeros(emr.select_workspace_size(g, dsc.n_pairs), dtype=torch.uint8, device="cuda")
 
     def step(evs=None):
         dsc.prepare()
@@ -450,7 +451,7 @@ def main():
         if evs:
             evs[1].record(stream)
         emr.select(dsc.split, dsc.band_bits, tile_flags, dsc.pack, dsc.query, dsc.ws, g, dsc.mode, dsc.types,
-                   dsc.idx, dsc.w, dsc.cap, dsc.counts, dsc.offsets)
+                   dsc.idx, dsc.w, dsc.cap, dsc.counts, dsc.offsets, sws)
 
     launches_per_step = launches_in_step(emr, dsc)
     for _ in range(args.warmup):

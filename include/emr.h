@@ -375,16 +375,21 @@ emr_status emr_eval_filter_tiles(const void *pack_host, const emr_query *q, cons
                                  float band, float w_min, uint32_t *split, uint32_t *band_bits,
                                  uint8_t *tile_flags, void *ws, size_t ws_bytes, void *stream);
 
+/* Bytes of device workspace emr_select needs for n_pairs pairs (per pair and
+ * dense tile: the tile's first list entry and a work item). */
+emr_status emr_select_workspace_size(const emr_grid *grid, int32_t n_pairs, size_t *bytes);
+
 /* emr_mask_combine_types followed by emr_compact_records, computed only over the
  * tiles that tile_flags (from emr_eval_filter_tiles) marks: a tile without band
  * bits keeps nothing, whatever its split bits. No mask plane is written. The
  * lists, counts and offsets equal those of the two calls; entries past cap are
- * dropped (compare offsets[n_pairs] with cap). eval_ws: the prepared records.
- * Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY (eval_ws), EMR_ERR_RANGE, EMR_ERR_CUDA. */
+ * dropped (compare offsets[n_pairs] with cap). eval_ws: the prepared records;
+ * ws: emr_select_workspace_size bytes. Errors: EMR_ERR_ARG, EMR_ERR_CAPACITY
+ * (eval_ws or ws), EMR_ERR_RANGE, EMR_ERR_CUDA. */
 emr_status emr_select(const uint32_t *split, const uint32_t *band_bits, const uint8_t *tile_flags,
                       const void *pack_host, const emr_query *q, const void *eval_ws, size_t eval_ws_bytes,
                       const emr_grid *grid, int32_t mode, int32_t types, int32_t *idx, float *w, int64_t cap,
-                      int64_t *counts, int64_t *offsets, void *stream);
+                      int64_t *counts, int64_t *offsets, void *ws, size_t ws_bytes, void *stream);
 
 /* Subtree-leaf variance: the split plane under ES-HyperNEAT's reading of a
  * cell's variance (its quadtree measures the spread of the outputs at a

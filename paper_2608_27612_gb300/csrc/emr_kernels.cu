@@ -1484,72 +1484,82 @@ __global__ void __launch_bounds__(kSelectThreads) select_count_kernel(const uint
                                                                       const uint8_t* __restrict__ flags,
                                                                       int64_t n_dense, GridDev G, int gated,
                                                                       TypeFilter tf, int64_t n_pairs,
-                                                                      int64_t* __restrict__ counts) {
+                                                                      int64_t* __restrict__ counts,
+                                                                      int32_t* __restrict__ tile_base,
+                                                                      int64_t* __restrict__ items,
+                                                                      unsigned long long* __restrict__ n_items) {
   const int lane = threadIdx.x & 31;
   const int64_t r = (int64_t(blockIdx.x) * kSelectThreads + threadIdx.x) >> 5;
   if (r >= n_pairs) return;  // whole warps
   const uint32_t* sp = split + r * G.n_words;
   const uint32_t* bw = bandb + r * G.n_words;
-  int sum = 0;
+  int run = 0;  // entries of the pair's earlier flagged tiles
   for (int64_t t0 = 0; t0 < n_dense; t0 += 32) {
     const int64_t t = t0 + lane;
     uint32_t bal = __ballot_sync(kFull, t < n_dense && flags[r * n_dense + t]);
     for (; bal; bal &= bal - 1) {
+      const int64_t tt = t0 + __ffs(bal) - 1;
       int64_t wb, we;
-      tile_words(G, int32_t(t0 + __ffs(bal) - 1), &wb, &we);
+      tile_words(G, int32_t(tt), &wb, &we);
+      int sum = 0;
       for (int64_t wi = wb + 4 * lane; wi < we; wi += 128) {
         uint32_t m[4];
         combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
         sum += __popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]);
       }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(kFull, sum, o);
+      if (lane == 0 && sum > 0) {  // a work item for the write kernel
+        tile_base[r * n_dense + tt] = run;
+        items[atomicAdd(n_items, 1ull)] = r * n_dense + tt;
+      }
+      run += sum;
     }
   }
-#pragma unroll
-  for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(kFull, sum, o);
-  if (lane == 0) counts[r] = sum;
+  if (lane == 0) counts[r] = run;
 }
 
+// One warp per work item (pair, tile with kept positions): the tile's list
+// entries go to offsets[pair] + tile_base, in ascending global index.
 __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint32_t* __restrict__ split,
                                                                       const uint32_t* __restrict__ bandb,
-                                                                      const uint8_t* __restrict__ flags,
                                                                       int64_t n_dense, GridDev G, int gated,
-                                                                      TypeFilter tf, int64_t n_pairs,
-                                                                      RecordSource rs,
+                                                                      TypeFilter tf,
+                                                                      const int32_t* __restrict__ tile_base,
+                                                                      const int64_t* __restrict__ items,
+                                                                      const unsigned long long* __restrict__ n_items,
                                                                       const int64_t* __restrict__ offsets,
                                                                       int64_t cap, int32_t* __restrict__ idx,
                                                                       float* __restrict__ wv) {
   const int lane = threadIdx.x & 31;
-  const int64_t r = (int64_t(blockIdx.x) * kSelectThreads + threadIdx.x) >> 5;
-  if (r >= n_pairs) return;  // whole warps
-  const uint32_t* sp = split + r * G.n_words;
-  const uint32_t* bw = bandb + r * G.n_words;
-  int64_t base = offsets[r];
-  for (int64_t t0 = 0; t0 < n_dense; t0 += 32) {
-    const int64_t t = t0 + lane;
-    uint32_t bal = __ballot_sync(kFull, t < n_dense && flags[r * n_dense + t]);
-    for (; bal; bal &= bal - 1) {
-      int64_t wb, we;
-      tile_words(G, int32_t(t0 + __ffs(bal) - 1), &wb, &we);
-      for (int64_t w0 = wb; w0 < we; w0 += 128) {
-        const int64_t wi = w0 + 4 * lane;
-        uint32_t m[4] = {0u, 0u, 0u, 0u};
-        if (wi < we) combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
-        int total;
-        const int ex = warp_exclusive_scan(__popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]), &total);
-        int64_t dst = base + ex;
-        for (int c = 0; c < 4; c++) {
-          if (!m[c]) continue;
-          int d = 0;
-          while (G.word_off[d + 1] <= wi + c) d++;
-          const int64_t gbase = G.level_off[d] + (wi + c - G.word_off[d]) * 32;
-          for (uint32_t v = m[c]; v; v &= v - 1, dst++)
-            if (dst < cap) {
-              idx[dst] = int32_t(gbase + __ffs(v) - 1);
-              if (wv) wv[dst] = __int_as_float(int32_t(r));  // the pair, for select_weights_kernel
-            }
-        }
-        base += total;
+  const int64_t n = int64_t(*n_items);
+  const int64_t warps = int64_t(gridDim.x) * (kSelectThreads / 32);
+  for (int64_t it = (int64_t(blockIdx.x) * kSelectThreads + threadIdx.x) >> 5; it < n; it += warps) {
+    const int64_t item = items[it], r = item / n_dense, t = item - r * n_dense;
+    const uint32_t* sp = split + r * G.n_words;
+    const uint32_t* bw = bandb + r * G.n_words;
+    int64_t base = offsets[r] + tile_base[item];
+    int64_t wb, we;
+    tile_words(G, int32_t(t), &wb, &we);
+    for (int64_t w0 = wb; w0 < we; w0 += 128) {
+      const int64_t wi = w0 + 4 * lane;
+      uint32_t m[4] = {0u, 0u, 0u, 0u};
+      if (wi < we) combine_group(sp, bw, G, wi, we - wi < 4 ? int(we - wi) : 4, gated, tf, r, m);
+      int total;
+      const int ex = warp_exclusive_scan(__popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]), &total);
+      int64_t dst = base + ex;
+      for (int c = 0; c < 4; c++) {
+        if (!m[c]) continue;
+        int d = 0;
+        while (G.word_off[d + 1] <= wi + c) d++;
+        const int64_t gbase = G.level_off[d] + (wi + c - G.word_off[d]) * 32;
+        for (uint32_t v = m[c]; v; v &= v - 1, dst++)
+          if (dst < cap) {
+            idx[dst] = int32_t(gbase + __ffs(v) - 1);
+            if (wv) wv[dst] = __int_as_float(int32_t(r));  // the pair, for select_weights_kernel
+          }
       }
+      base += total;
     }
   }
 }
@@ -2168,18 +2178,30 @@ emr_status emr_eval_filter_tiles(const void* pack_host, const emr_query* q, cons
                       static_cast<cudaStream_t>(stream), TileRange(), tile_flags);
 }
 
+static size_t select_ws_bytes(int64_t n_pairs, int64_t n_dense) {
+  return 256 + ((size_t(n_pairs) * size_t(n_dense) * 4 + 255) & ~size_t(255)) + size_t(n_pairs) * size_t(n_dense) * 8;
+}
+
+emr_status emr_select_workspace_size(const emr_grid* grid, int32_t n_pairs, size_t* bytes) {
+  if (!grid_ok(grid) || n_pairs <= 0 || !bytes) return EMR_ERR_ARG;
+  *bytes = select_ws_bytes(n_pairs, dense_tiles(grid->D));
+  return EMR_OK;
+}
+
 emr_status emr_select(const uint32_t* split, const uint32_t* band_bits, const uint8_t* tile_flags,
                       const void* pack_host, const emr_query* q, const void* eval_ws, size_t eval_ws_bytes,
                       const emr_grid* grid, int32_t mode, int32_t types, int32_t* idx, float* w, int64_t cap,
-                      int64_t* counts, int64_t* offsets, void* stream) {
+                      int64_t* counts, int64_t* offsets, void* ws, size_t ws_bytes, void* stream) {
   if (!split || !band_bits || !tile_flags || !eval_ws || !grid_ok(grid) || (!idx && cap > 0) || cap < 0 ||
-      !counts || !offsets || (mode != EMR_EAGER && mode != EMR_GATED) || types < 0 || types > EMR_CONN_ALL)
+      !counts || !offsets || !ws || (mode != EMR_EAGER && mode != EMR_GATED) || types < 0 || types > EMR_CONN_ALL)
     return EMR_ERR_ARG;
   EvalPlan p;
   emr_status rc = eval_plan(pack_host, q, &p);
   if (rc != EMR_OK) return rc;
   if (eval_ws_bytes < p.total) return EMR_ERR_CAPACITY;
   if (p.n_pairs <= 0 || p.n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
+  const int64_t n_dense = dense_tiles(grid->D);
+  if (ws_bytes < select_ws_bytes(p.n_pairs, n_dense)) return EMR_ERR_CAPACITY;
   TypeFilter tf = no_type_filter();
   if (types != EMR_CONN_ALL) {
     tf.types = types;
@@ -2187,23 +2209,26 @@ emr_status emr_select(const uint32_t* split, const uint32_t* band_bits, const ui
   }
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const GridDev G = grid_dev(grid);
-  const int64_t n_dense = dense_tiles(grid->D);
+  auto* n_items = static_cast<unsigned long long*>(ws);
+  auto* tile_base = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + 256);
+  auto* items = reinterpret_cast<int64_t*>(static_cast<uint8_t*>(ws) + 256 +
+                                           ((size_t(p.n_pairs) * size_t(n_dense) * 4 + 255) & ~size_t(255)));
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaMemsetAsync(n_items, 0, sizeof(unsigned long long), st) != cudaSuccess)
+    return EMR_ERR_CUDA;
   const unsigned blocks = unsigned((p.n_pairs + kSelectThreads / 32 - 1) / (kSelectThreads / 32));
   select_count_kernel<<<blocks, kSelectThreads, 0, st>>>(split, band_bits, tile_flags, n_dense, G,
-                                                         mode == EMR_GATED, tf, p.n_pairs, counts);
+                                                         mode == EMR_GATED, tf, p.n_pairs, counts, tile_base, items,
+                                                         n_items);
   compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, p.n_pairs, offsets);
-  select_write_kernel<<<blocks, kSelectThreads, 0, st>>>(split, band_bits, tile_flags, n_dense, G,
-                                                         mode == EMR_GATED, tf, p.n_pairs,
-                                                         RecordSource{static_cast<const uint8_t*>(eval_ws), p.L},
-                                                         offsets, cap, idx, w);
-  if (w && cap > 0) {
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-      return EMR_ERR_CUDA;
+  select_write_kernel<<<unsigned(16 * sms), kSelectThreads, 0, st>>>(split, band_bits, n_dense, G,
+                                                                     mode == EMR_GATED, tf, tile_base, items,
+                                                                     n_items, offsets, cap, idx, w);
+  if (w && cap > 0)
     select_weights_kernel<<<unsigned(8 * sms), kCompactBlock, 0, st>>>(
         RecordSource{static_cast<const uint8_t*>(eval_ws), p.L}, G, offsets, p.n_pairs, cap, idx, w);
-  }
   return cuda_status(cudaGetLastError());
 }
 

@@ -77,7 +77,8 @@ def lib() -> C.CDLL:
             "emr_subtree_workspace_size": [vp, i32, vp],
             "emr_subtree_split": [vp, vp, i32, f32, vp, vp, vp, sz, vp],
             "emr_eval_filter_tiles": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
-            "emr_select": [vp, vp, vp, vp, vp, vp, sz, vp, i32, i32, vp, vp, i64, vp, vp, vp],
+            "emr_select": [vp, vp, vp, vp, vp, vp, sz, vp, i32, i32, vp, vp, i64, vp, vp, vp, sz, vp],
+            "emr_select_workspace_size": [vp, i32, vp],
             "emr_substrate_config": [i32, vp, vp],
             "emr_assemble_workspace_size": [vp, i32, i32, i32, vp, i64, vp],
             "emr_assemble": [vp, vp, i32, vp, vp, i32, vp, vp, vp, f32, f32, f32, i32, i32, i32, i32, vp, sz, i64,
@@ -296,13 +297,20 @@ def eval_filter_tiles(pack, query: Query, grid: Grid, theta: float, band: float,
                                        _stream(stream)), "emr_eval_filter_tiles")
 
 
+def select_workspace_size(grid: Grid, n_pairs: int) -> int:
+    n = C.c_size_t()
+    _check(lib().emr_select_workspace_size(C.byref(grid), n_pairs, C.byref(n)), "emr_select_workspace_size")
+    return n.value
+
+
 def select(split, band_bits, tile_flags, pack, query: Query, eval_ws, grid: Grid, mode: int, types: int, idx, w,
-           cap: int, counts, offsets, stream=None):
+           cap: int, counts, offsets, ws, stream=None):
     """emr_select: combine + compaction + kept weights over the flagged tiles only."""
     q = query.c
     _check(lib().emr_select(_ptr(split), _ptr(band_bits), _ptr(tile_flags), _ptr(pack), C.byref(q), _ptr(eval_ws),
                             C.c_size_t(eval_ws.numel()), C.byref(grid), mode, types, _ptr(idx), _ptr(w), cap,
-                            _ptr(counts), _ptr(offsets), _stream(stream)), "emr_select")
+                            _ptr(counts), _ptr(offsets), _ptr(ws), C.c_size_t(ws.numel()), _stream(stream)),
+           "emr_select")
 
 
 def mask_combine_types(split, band_bits, query: Query, grid: Grid, n_pairs: int, mode: int, types: int, mask,
@@ -543,11 +551,13 @@ class Discovery:
         if getattr(self, "tile_flags", None) is None:
             self.tile_flags = torch.zeros(self.n_pairs, dense_tiles(self.grid.D), dtype=torch.uint8,
                                           device=self.device)
+            self.sws = torch.zeros(select_workspace_size(self.grid, self.n_pairs), dtype=torch.uint8,
+                                   device=self.device)
         self.prepare(stream)
         eval_filter_tiles(self.pack, self.query, self.grid, self.theta, self.band, self.w_min, self.split,
                           self.band_bits, self.tile_flags, self.ws, stream)
         select(self.split, self.band_bits, self.tile_flags, self.pack, self.query, self.ws, self.grid, self.mode,
-               self.types, self.idx, self.w, self.cap, self.counts, self.offsets, stream)
+               self.types, self.idx, self.w, self.cap, self.counts, self.offsets, self.sws, stream)
 
     def combine(self, stream=None):
         """emr_mask_combine, or emr_mask_combine_types when a connection-type filter is set."""

@@ -139,6 +139,32 @@ def test_bench_configuration_depth7_sampled():
                 ins.append([a, b, x, y, 1.0] if w.sources.side[s] == W.SIDE_OUT else [x, y, a, b, 1.0])
             ref, err = oracle.cppn(w.pop, int(gi), np.array(ins))
             check_outputs(gpu["out"][gi * w.S + s, pos], ref, err)
+    # the benchmark step's own path (emr_eval_filter_tiles + emr_select): the same lists for every pair,
+    # and its keep decisions at sampled positions of every genome against the oracle's
+    dsc = gpu["dsc"]
+    dsc.idx.zero_(); dsc.w.zero_()
+    dsc.run_select()
+    torch.cuda.synchronize()
+    sel = dsc.lists()
+    for (ri, rw), (si, sw) in zip(gpu["lists_f"], sel):
+        assert np.array_equal(ri, si) and np.array_equal(rw.view(np.uint32), sw.view(np.uint32))
+    n_checked = 0
+    for gi in rng.choice(w.P, 60, replace=False):
+        for s in range(w.S):
+            r = gi * w.S + s
+            kept = sel[r][0]
+            # every kept position, plus random others
+            pos = np.unique(np.concatenate([kept[:32], rng.integers(0, g.n_total, 32)])).astype(np.int64)
+            d = np.zeros(len(pos), np.int32); ii = np.zeros(len(pos), np.int64); jj = np.zeros(len(pos), np.int64)
+            for k, p in enumerate(pos):
+                d[k], ii[k], jj[k] = emr.index_to_ij(int(p))
+            ko = oracle.keep_at(w.pop, int(gi), float(w.sources.a[s]), float(w.sources.b[s]),
+                                int(w.sources.side[s]), w.D, w.theta, w.band, w.w_min, d, ii, jj)
+            ok = ko["unc"] == 0
+            got = np.isin(pos, kept)
+            assert np.array_equal(got[ok], ko["keep"][ok].astype(bool)), "pair %d" % r
+            n_checked += int(ok.sum())
+    assert n_checked > 8000
 
 
 def test_linear_worked_example_keeps_grid3():

@@ -419,6 +419,19 @@ emr_status emr_subtree_split(const float *out, const emr_grid *grid, int32_t n_p
 emr_status emr_scale_weights(float *w, const int64_t *offsets, int32_t n_pairs, int64_t cap, float w_thr,
                              float w_max, void *stream);
 
+/* The whole path in one call: emr_eval_prepare, emr_eval_filter_tiles and
+ * emr_select on a single workspace that holds the records, the split and band
+ * planes, the tile flags and the selection workspace (emr_discover_workspace_
+ * size bytes; the planes inside are the library's, not to be read). The pack is
+ * planned once. Lists, counts and offsets as emr_select writes them.
+ * Errors as the three calls. */
+emr_status emr_discover_workspace_size(const void *pack_host, const emr_query *q, const emr_grid *grid,
+                                       size_t *bytes);
+emr_status emr_discover(const void *pack_host, const void *pack_dev, const emr_query *q, const emr_grid *grid,
+                        float theta, float band, float w_min, int32_t mode, int32_t types, void *ws,
+                        size_t ws_bytes, int32_t *idx, float *w, int64_t cap, int64_t *counts, int64_t *offsets,
+                        void *stream);
+
 /* Connection type code (0 forward, 1 backward, 2 lateral, 3 self; Section 6
  * taxonomy, see emr_mask_combine_types) of every list entry: type[e] for
  * entries e < min(offsets[n_pairs], cap) of lists laid out as emr_compact

@@ -2188,6 +2188,11 @@ emr_status emr_select_workspace_size(const emr_grid* grid, int32_t n_pairs, size
   return EMR_OK;
 }
 
+static emr_status select_launch(const EvalPlan& p, const uint32_t* split, const uint32_t* band_bits,
+                                const uint8_t* tile_flags, const emr_query* q, const void* eval_ws,
+                                const emr_grid* grid, int32_t mode, int32_t types, int32_t* idx, float* w, int64_t cap,
+                                int64_t* counts, int64_t* offsets, void* ws, cudaStream_t st);
+
 emr_status emr_select(const uint32_t* split, const uint32_t* band_bits, const uint8_t* tile_flags,
                       const void* pack_host, const emr_query* q, const void* eval_ws, size_t eval_ws_bytes,
                       const emr_grid* grid, int32_t mode, int32_t types, int32_t* idx, float* w, int64_t cap,
@@ -2200,14 +2205,77 @@ emr_status emr_select(const uint32_t* split, const uint32_t* band_bits, const ui
   if (rc != EMR_OK) return rc;
   if (eval_ws_bytes < p.total) return EMR_ERR_CAPACITY;
   if (p.n_pairs <= 0 || p.n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
+  if (ws_bytes < select_ws_bytes(p.n_pairs, dense_tiles(grid->D))) return EMR_ERR_CAPACITY;
+  return select_launch(p, split, band_bits, tile_flags, q, eval_ws, grid, mode, types, idx, w, cap, counts, offsets,
+                       ws, static_cast<cudaStream_t>(stream));
+}
+
+// Planes, tile flags and selection workspace of emr_discover after the records.
+struct DiscoverLayout {
+  size_t split, band, flags, sel, total;
+};
+
+static DiscoverLayout discover_layout(const EvalPlan& p, const emr_grid* g) {
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  DiscoverLayout L;
+  const size_t plane = size_t(p.n_pairs) * size_t(g->n_words) * 4;
+  const int64_t n_dense = dense_tiles(g->D);
+  L.split = up(p.total);
+  L.band = L.split + up(plane);
+  L.flags = L.band + up(plane);
+  L.sel = L.flags + up(size_t(p.n_pairs) * size_t(n_dense));
+  L.total = L.sel + up(select_ws_bytes(p.n_pairs, n_dense));
+  return L;
+}
+
+emr_status emr_discover_workspace_size(const void* pack_host, const emr_query* q, const emr_grid* grid,
+                                       size_t* bytes) {
+  if (!bytes || !grid_ok(grid)) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  *bytes = discover_layout(p, grid).total;
+  return EMR_OK;
+}
+
+emr_status emr_discover(const void* pack_host, const void* pack_dev, const emr_query* q, const emr_grid* grid,
+                        float theta, float band, float w_min, int32_t mode, int32_t types, void* ws, size_t ws_bytes,
+                        int32_t* idx, float* w, int64_t cap, int64_t* counts, int64_t* offsets, void* stream) {
+  if (!pack_dev || !ws || !grid_ok(grid) || (!idx && cap > 0) || cap < 0 || !counts || !offsets ||
+      (mode != EMR_EAGER && mode != EMR_GATED) || types < 0 || types > EMR_CONN_ALL)
+    return EMR_ERR_ARG;
+  if (!(theta >= 0.f) || !(band >= 0.f) || !(w_min >= 0.f)) return EMR_ERR_ARG;
+  EvalPlan p;
+  emr_status rc = eval_plan(pack_host, q, &p);
+  if (rc != EMR_OK) return rc;
+  if (p.n_pairs <= 0 || p.n_pairs > 0x7fffffffLL) return EMR_ERR_RANGE;
+  const DiscoverLayout L = discover_layout(p, grid);
+  if (ws_bytes < L.total) return EMR_ERR_CAPACITY;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  uint8_t* spec;
+  int32_t* order;
+  if ((rc = prepare(pack_dev, q, p, ws, st, &spec, &order)) != EMR_OK) return rc;
+  auto* split = reinterpret_cast<uint32_t*>(base + L.split);
+  auto* bandb = reinterpret_cast<uint32_t*>(base + L.band);
+  uint8_t* flags = base + L.flags;
+  if ((rc = launch_tiles(p, grid, spec, order, kModeFused, theta, band, w_min, nullptr, nullptr, split, bandb, st,
+                         TileRange(), flags)) != EMR_OK)
+    return rc;
+  return select_launch(p, split, bandb, flags, q, ws, grid, mode, types, idx, w, cap, counts, offsets,
+                       base + L.sel, st);
+}
+
+static emr_status select_launch(const EvalPlan& p, const uint32_t* split, const uint32_t* band_bits,
+                                const uint8_t* tile_flags, const emr_query* q, const void* eval_ws,
+                                const emr_grid* grid, int32_t mode, int32_t types, int32_t* idx, float* w, int64_t cap,
+                                int64_t* counts, int64_t* offsets, void* ws, cudaStream_t st) {
   const int64_t n_dense = dense_tiles(grid->D);
-  if (ws_bytes < select_ws_bytes(p.n_pairs, n_dense)) return EMR_ERR_CAPACITY;
   TypeFilter tf = no_type_filter();
   if (types != EMR_CONN_ALL) {
     tf.types = types;
     tf.q = query_dev(q);
   }
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   const GridDev G = grid_dev(grid);
   auto* n_items = static_cast<unsigned long long*>(ws);
   auto* tile_base = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + 256);

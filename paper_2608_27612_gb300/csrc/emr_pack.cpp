@@ -1,6 +1,11 @@
 // Host side of libemr: grid descriptor (Eq. 1), genome packer, status strings.
+#include <pthread.h>
+
 #include <algorithm>
 #include <cmath>
+#include <condition_variable>
+#include <functional>
+#include <mutex>
 #include <cstring>
 #include <thread>
 #include <utility>
@@ -13,6 +18,96 @@ using namespace emr;
 namespace {
 
 inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
+
+// Host worker threads kept across calls (starting threads costs as much as
+// packing a few dozen genomes). run() executes fn(0 .. n-1) on the workers and
+// the caller and returns when all are done; one job at a time (a caller that
+// finds the pool busy runs its job alone). The pool lives until exit and is
+// never destroyed; a process forked from this one starts a fresh pool.
+class WorkerPool {
+ public:
+  static WorkerPool& get() {
+    static std::once_flag once;
+    std::call_once(once, [] { pthread_atfork(nullptr, nullptr, [] { instance() = nullptr; }); });
+    std::lock_guard<std::mutex> lk(create_mu());
+    if (!instance()) instance() = new WorkerPool();
+    return *instance();
+  }
+
+  void run(int n, const std::function<void(int)>& fn) {
+    std::unique_lock<std::mutex> job_lock(job_mu_, std::try_to_lock);
+    if (!job_lock.owns_lock() || n <= 1) {
+      for (int t = 0; t < n; t++) fn(t);
+      return;
+    }
+    ensure(n - 1);
+    {
+      std::lock_guard<std::mutex> lk(mu_);
+      job_ = &fn;
+      n_ = n;
+      next_ = 1;  // task 0 is the caller's
+      left_ = n - 1;
+      gen_++;
+    }
+    cv_.notify_all();
+    fn(0);
+    for (;;) {  // help with the remaining tasks, then wait for the workers' last ones
+      int t;
+      {
+        std::lock_guard<std::mutex> lk(mu_);
+        if (next_ >= n_) break;
+        t = next_++;
+      }
+      fn(t);
+      std::lock_guard<std::mutex> lk(mu_);
+      if (--left_ == 0) break;
+    }
+    std::unique_lock<std::mutex> lk(mu_);
+    done_cv_.wait(lk, [&] { return left_ == 0 || (next_ >= n_ && left_ == 0); });
+    job_ = nullptr;
+  }
+
+ private:
+  static WorkerPool*& instance() {
+    static WorkerPool* p = nullptr;
+    return p;
+  }
+  static std::mutex& create_mu() {
+    static std::mutex m;
+    return m;
+  }
+
+  void ensure(int workers) {
+    while (int(n_workers_) < workers) {
+      std::thread([this] { loop(); }).detach();
+      n_workers_++;
+    }
+  }
+
+  void loop() {
+    uint64_t seen = 0;
+    for (;;) {
+      std::unique_lock<std::mutex> lk(mu_);
+      cv_.wait(lk, [&] { return gen_ != seen && job_ && next_ < n_; });
+      seen = gen_;
+      while (job_ && next_ < n_) {
+        const int t = next_++;
+        const std::function<void(int)>* fn = job_;
+        lk.unlock();
+        (*fn)(t);
+        lk.lock();
+        if (--left_ == 0) done_cv_.notify_all();
+      }
+    }
+  }
+
+  std::mutex job_mu_, mu_;
+  std::condition_variable cv_, done_cv_;
+  const std::function<void(int)>* job_ = nullptr;
+  int n_ = 0, next_ = 0, left_ = 0;
+  uint64_t gen_ = 0;
+  unsigned n_workers_ = 0;
+};
 
 uint32_t compact_bits(uint64_t m) {  // even bits of m, packed
   m &= 0x5555555555555555ull;
@@ -288,8 +383,8 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
   // Genomes are independent: pack them on several host threads, each with its
   // own scratch; the lowest failing genome index is reported.
   const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
-  // a thread costs about as much to start as packing ~16 genomes: sqrt(P / 16) threads balance the two
-  const int n_threads = std::max(1, std::min({hw, 16, int(std::sqrt(double(P) / 16.0))}));
+  // a thread's share costs about as much to hand out as packing a few genomes
+  const int n_threads = std::max(1, std::min({hw, 16, P / 32}));
   std::vector<emr_status> t_rc(n_threads, EMR_OK);
   std::vector<int32_t> t_bad(n_threads, -1);
   std::vector<std::vector<PackNode>> t_nodes(n_threads);
@@ -315,9 +410,7 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
   if (n_threads == 1) {
     work(0);
   } else {
-    std::vector<std::thread> pool;
-    for (int t = 0; t < n_threads; t++) pool.emplace_back(work, t);
-    for (auto& th : pool) th.join();
+    WorkerPool::get().run(n_threads, work);
   }
   for (int t = 0; t < n_threads; t++)
     if (t_rc[t] != EMR_OK) {

@@ -79,6 +79,8 @@ def lib() -> C.CDLL:
             "emr_eval_filter_tiles": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
             "emr_select": [vp, vp, vp, vp, vp, vp, sz, vp, i32, i32, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_select_workspace_size": [vp, i32, vp],
+            "emr_discover_workspace_size": [vp, vp, vp, vp],
+            "emr_discover": [vp, vp, vp, vp, f32, f32, f32, i32, i32, vp, sz, vp, vp, i64, vp, vp, vp],
             "emr_substrate_config": [i32, vp, vp],
             "emr_assemble_workspace_size": [vp, i32, i32, i32, vp, i64, vp],
             "emr_assemble": [vp, vp, i32, vp, vp, i32, vp, vp, vp, f32, f32, f32, i32, i32, i32, i32, vp, sz, i64,
@@ -311,6 +313,24 @@ def select(split, band_bits, tile_flags, pack, query: Query, eval_ws, grid: Grid
                             C.c_size_t(eval_ws.numel()), C.byref(grid), mode, types, _ptr(idx), _ptr(w), cap,
                             _ptr(counts), _ptr(offsets), _ptr(ws), C.c_size_t(ws.numel()), _stream(stream)),
            "emr_select")
+
+
+def discover_workspace_size(pack, query: Query, grid: Grid) -> int:
+    n = C.c_size_t()
+    q = query.c
+    _check(lib().emr_discover_workspace_size(_ptr(pack), C.byref(q), C.byref(grid), C.byref(n)),
+           "emr_discover_workspace_size")
+    return n.value
+
+
+def discover(pack, pack_dev, query: Query, grid: Grid, theta: float, band: float, w_min: float, mode: int,
+             types: int, ws, idx, w, cap: int, counts, offsets, stream=None, qc=None):
+    """emr_discover: the whole path (records, fused evaluation and filter, selection) in one call.
+    qc: a QueryC from query.c, to reuse across calls."""
+    q = qc if qc is not None else query.c
+    _check(lib().emr_discover(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min, mode, types,
+                              _ptr(ws), C.c_size_t(ws.numel()), _ptr(idx), _ptr(w), cap, _ptr(counts),
+                              _ptr(offsets), _stream(stream)), "emr_discover")
 
 
 def mask_combine_types(split, band_bits, query: Query, grid: Grid, n_pairs: int, mode: int, types: int, mask,
@@ -558,6 +578,14 @@ class Discovery:
                           self.band_bits, self.tile_flags, self.ws, stream)
         select(self.split, self.band_bits, self.tile_flags, self.pack, self.query, self.ws, self.grid, self.mode,
                self.types, self.idx, self.w, self.cap, self.counts, self.offsets, self.sws, stream)
+
+    def run_discover(self, stream=None):
+        """emr_discover: the whole path in one call on its own workspace."""
+        if getattr(self, "dws", None) is None:
+            self.dws = torch.zeros(discover_workspace_size(self.pack, self.query, self.grid), dtype=torch.uint8,
+                                   device=self.device)
+        discover(self.pack, self.pack_dev, self.query, self.grid, self.theta, self.band, self.w_min, self.mode,
+                 self.types, self.dws, self.idx, self.w, self.cap, self.counts, self.offsets, stream)
 
     def combine(self, stream=None):
         """emr_mask_combine, or emr_mask_combine_types when a connection-type filter is set."""

@@ -38,6 +38,13 @@ def compare(w, mode=emr.EMR_EAGER, types=emr.CONN_ALL):
         assert np.array_equal(ri, gi) and np.array_equal(rw.view(np.uint32), gw.view(np.uint32))
     band = dsc.band_bits.cpu().numpy()
     assert np.array_equal(band, band_ref)  # same fused evaluation
+    # the one-call path gives the same lists
+    dsc.idx.zero_(); dsc.w.zero_(); dsc.counts.zero_(); dsc.offsets.zero_()
+    dsc.run_discover()
+    torch.cuda.synchronize()
+    one = dsc.lists()
+    for (ri, rw), (gi, gw) in zip(ref, one):
+        assert np.array_equal(ri, gi) and np.array_equal(rw.view(np.uint32), gw.view(np.uint32))
     flags = dsc.tile_flags.cpu().numpy()
     want = np.stack([band[:, b:e].any(axis=1) for b, e in tile_word_ranges(dsc.grid)], axis=1)
     assert np.array_equal(flags.astype(bool), want)

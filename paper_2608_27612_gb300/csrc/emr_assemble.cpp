@@ -25,21 +25,18 @@ namespace {
 
 inline size_t up256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// fn(g) for g in [0, n) on up to 16 host threads (genomes are independent).
+// fn(g) for g in [0, n) on the library's host worker threads (genomes are independent).
 template <class F>
 void parallel_for(int32_t n, F fn) {
   const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
-  const int nt = n >= 64 ? std::min(hw, 16) : 1;
+  const int nt = std::max(1, std::min({hw, 16, n / 16}));
   if (nt == 1) {
     for (int32_t g = 0; g < n; g++) fn(g);
     return;
   }
-  std::vector<std::thread> pool;
-  for (int t = 0; t < nt; t++)
-    pool.emplace_back([&, t] {
-      for (int32_t g = int32_t(int64_t(n) * t / nt); g < int32_t(int64_t(n) * (t + 1) / nt); g++) fn(g);
-    });
-  for (auto& th : pool) th.join();
+  emr::host_parallel(nt, [&](int t) {
+    for (int32_t g = int32_t(int64_t(n) * t / nt); g < int32_t(int64_t(n) * (t + 1) / nt); g++) fn(g);
+  });
 }
 
 // Device workspace carve-up for one query batch of up to n_pairs pairs.

@@ -3,6 +3,8 @@
 
 #include <stdint.h>
 
+#include <functional>
+
 #include "../../include/emr.h"
 
 namespace emr {
@@ -55,6 +57,10 @@ struct PackEdge {
 static_assert(sizeof(PackEdge) == 8, "pack edge layout");
 
 inline const PackHeader* pack_header(const void* blob) { return static_cast<const PackHeader*>(blob); }
+
+// fn(0 .. n-1) on the library's persistent host worker threads and the caller;
+// returns when every call has returned (emr_pack.cpp).
+void host_parallel(int n, const std::function<void(int)>& fn);
 
 // Grid helpers (Eq. 1 numbering, depth-major Morton).
 inline int64_t level_offset(int d) { return ((int64_t(1) << (2 * (d + 1))) - 4) / 3; }

@@ -325,6 +325,8 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
 
 }  // namespace
 
+void emr::host_parallel(int n, const std::function<void(int)>& fn) { WorkerPool::get().run(n, fn); }
+
 extern "C" {
 
 emr_status emr_grid_build(int32_t D, int64_t chunk, emr_grid* grid) {

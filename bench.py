@@ -158,35 +158,49 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
+TILE_SIDE = 64
+
+
 def algorithmic_work(pack, query, emr):
-    """Per pair: fp32 lane ops and MUFU ops per query on the packed DAG (dead
-    nodes removed, constants folded): per varying node its grid-input FMAs,
-    its in-edges from varying nodes and its activation; plus the filter at its
-    minimum: per parent the six squared pairwise child differences, their sum and
-    one compare (4.5 per query), and per quad the band screen's four compares on
-    the sibling differences (1 per query; the full band test of the few quads the
-    screen lets through is not counted). A pair whose output is constant over
-    the grid (no varying node) has variance and band value 0 everywhere and
-    counts no work."""
+    """Per pair: fp32 lane ops and MUFU ops per query, for the evaluation as the tile
+    kernels organise it, counted at its minimum on the packed DAG (dead nodes removed,
+    constants folded). A node that depends on the grid x (or y) coordinate alone has one
+    value per tile column (row): it is evaluated at the 66 distinct coordinates of a
+    64 x 64 tile (ring included), a 66/4096 share per query (its first-layer FMA, its
+    in-edges, its activation); so are the x part and the y part of a joint node's input
+    (one first-layer operation each, plus the edges from sources of that one coordinate).
+    Per query: each joint node's x + y add, its edges from joint sources and its
+    activation; plus the filter at its minimum: per parent the six squared pairwise child
+    differences, their sum and one compare (4.5 per query), and per quad the band
+    screen's four compares on the sibling differences (1 per query; the full band test
+    of the few quads the screen lets through is not counted). The pyramid tile (depths
+    0..4, 0.4% of the positions at depth 7) is counted like the 64 x 64 tiles. A pair
+    whose output is constant over the grid (no varying node) has variance and band value
+    0 everywhere and counts no work."""
     h, gs, nodes, edges = emr.pack_records(pack)
+    share = (TILE_SIDE + 2) / (TILE_SIDE * TILE_SIDE)
     per = np.zeros((len(gs), 2, 2))
     for g in range(len(gs)):
         nb, n, eb = int(gs["node_beg"][g]), int(gs["n_nodes"][g]), int(gs["edge_beg"][g])
         for side in (0, 1):
-            gx, gy = (2, 3) if side == 0 else (0, 1)
-            F = M = 0.0
+            F = M = F1 = M1 = 0.0
             for t in range(n):
                 nd = nodes[nb + t]
-                if not (int(nd["vary"]) >> side) & 1:
+                ax = (int(nd["axes"]) >> (2 * side)) & 3
+                if ax == 0:
                     continue
-                F += float(nd["w_in"][gx] != 0) + float(nd["w_in"][gy] != 0)
-                for e in range(int(nd["edge_cnt"])):
-                    src = int(edges[eb + int(nd["edge_beg"]) + e]["src"])
-                    F += (int(nodes[nb + src]["vary"]) >> side) & 1
-                F += ACT_FP32[int(nd["act"])]
-                M += ACT_MUFU[int(nd["act"])]
-            # a pair whose output does not vary over the grid needs no per-position arithmetic
-            per[g, side] = (F + VAR_OPS + BAND_OPS, M) if F > 0 or M > 0 else (0.0, 0.0)
+                sax = [(int(nodes[nb + int(edges[eb + int(nd["edge_beg"]) + e]["src"])]["axes"]) >> (2 * side)) & 3
+                       for e in range(int(nd["edge_cnt"]))]
+                a = int(nd["act"])
+                if ax == 3:
+                    F += 1 + sum(1 for x in sax if x == 3) + ACT_FP32[a]
+                    M += ACT_MUFU[a]
+                    F1 += 2 + sum(1 for x in sax if x in (1, 2))
+                else:
+                    F1 += 1 + sum(1 for x in sax if x) + ACT_FP32[a]
+                    M1 += ACT_MUFU[a]
+            varying = F1 > 0 or F > 0
+            per[g, side] = (F + share * F1 + VAR_OPS + BAND_OPS, M + share * M1) if varying else (0.0, 0.0)
     side = np.broadcast_to(query.side, (len(gs), query.S))
     return per[np.arange(len(gs))[:, None], side]  # [P, S, 2]
 
@@ -368,10 +382,12 @@ def launches_in_step(emr, dsc):
     kernel."""
     _, gs, _, _ = emr.pack_records(dsc.pack)
     side = np.asarray(dsc.query.side)
-    nv = gs["n_varying"][:, side] if not dsc.query.per_genome else \
-        np.take_along_axis(gs["n_varying"], side.reshape(gs.shape[0], -1), axis=1)
-    nv = nv.astype(np.int64)
-    cls = np.where(nv > 12, 0, np.where(nv > 8, 1, np.where(nv > 4, 2, 3)))
+    def per_pair(field):
+        f = gs[field][:, side] if not dsc.query.per_genome else \
+            np.take_along_axis(gs[field], side.reshape(gs.shape[0], -1), axis=1)
+        return f.astype(np.int64)
+    nv, nj = per_pair("n_varying"), per_pair("n_joint")
+    cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 4, 2, np.where(nj > 0, 3, 4))))
     return 1 + len(np.unique(cls[nv > 0])) + 4
 
 

@@ -144,9 +144,12 @@ emr_status emr_pack_size(int32_t P, const int64_t *node_ptr, const int64_t *conn
  * act(bias + sum of weight * source value over its enabled in-connections).
  *
  * The packer orders each genome topologically (Kahn's algorithm, ties by node
- * id), drops nodes that cannot reach the output, folds input connections into
- * per-node input weights and records, per query side, which nodes vary over
- * the grid. The blob is plain bytes: copy it to device memory unchanged (any
+ * id), merges parallel connections (same source and destination) into one
+ * whose weight is their fp32 sum in connection order, drops connections whose
+ * weight is then 0 (they add 0 for any finite source value), drops nodes that
+ * cannot reach the output, folds input connections into per-node input weights
+ * and records, per query side, which grid coordinates (x, y or both) each node
+ * depends on. The blob is plain bytes: copy it to device memory unchanged (any
  * 16-byte aligned address) and pass both copies to the eval calls.
  * Errors: EMR_ERR_ARG (null pointer, malformed genome: unknown id, duplicate
  * id, not exactly one output, connection into an input), EMR_ERR_CYCLE,

@@ -10,7 +10,7 @@
 namespace emr {
 
 constexpr uint32_t kPackMagic = 0x504d5245u;  // "EMRP"
-constexpr uint32_t kPackVersion = 1;
+constexpr uint32_t kPackVersion = 2;
 
 // Packed population blob: header, genome table, node records, edge records.
 // Every section starts on a 16-byte boundary; offsets are bytes from the blob start.
@@ -34,20 +34,25 @@ struct PackGenome {
   uint16_t n_varying[2];   // nodes whose value varies over the grid, per side
   uint16_t n_vedges[2];    // edges whose source and destination both vary, per side
   uint32_t cost[2];        // per-query work estimate, per side (scheduling only)
-  uint32_t reserved;
+  uint16_t n_joint[2];     // varying nodes that depend on both grid coordinates, per side
 };
 static_assert(sizeof(PackGenome) == 32, "pack genome layout");
 
 struct PackNode {
   uint8_t act;             // EMR_ACT_*
   uint8_t vary;            // bit s: varies over the grid under query side s
-  uint16_t reserved;
+  uint8_t axes;            // bits 2 s, 2 s + 1: depends on the grid x, y coordinate under query side s
+  uint8_t reserved;
   uint16_t edge_beg;       // first in-edge, relative to the genome's edge_beg
   uint16_t edge_cnt;       // in-edges from kept non-input nodes
   float bias;
   float w_in[5];           // summed weights of in-connections from x1, y1, x2, y2, bias
 };
 static_assert(sizeof(PackNode) == 32, "pack node layout");
+
+// Grid coordinates a varying node depends on (PackNode::axes per side; the
+// records' node and edge fields): x only, y only, or both ("joint").
+constexpr uint32_t kAxisX = 1, kAxisY = 2, kAxisXY = 3;
 
 struct PackEdge {
   uint16_t src;            // source: index among the genome's kept non-input nodes

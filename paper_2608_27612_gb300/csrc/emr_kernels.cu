@@ -151,11 +151,22 @@ __device__ __forceinline__ uint32_t band_word(uint32_t b0, uint32_t b1, uint32_t
 
 // ---- per-pair specialisation ---------------------------------------------------
 // A pair's record: header {nv, nve, out_const, flags}, then nv_cap float4
-// {c0, wx, wy, info} with info = act | edge_beg << 8 | edge_cnt << 20, then
-// nve_cap uint2 {source slot, weight bits}. Varying slots follow the genome's
-// topological order; the output is the last slot. nv = 0: the output is the
-// same at every position (out_const); unused per-genome slots are recorded as
-// constant 0 (no variance, no band value, nothing kept).
+// {c0, wx, wy, info} with info = act | axes << 4 | edge_beg << 8 | edge_cnt << 20
+// (axes: the grid coordinates the node depends on, kAxisX / kAxisY / kAxisXY),
+// then nve_cap uint2 {source slot | source axes << 16, weight bits}, each
+// node's edges ascending in (source axes, source slot). Varying slots follow
+// the genome's topological order; the output is the last slot. nv = 0: the
+// output is the same at every position (out_const); unused per-genome slots are
+// recorded as constant 0 (no variance, no band value, nothing kept).
+//
+// Every evaluator computes a node's input in one order, so that all of them
+// give the same fp32 value at a position:
+//   x only:  a = fma(wx, x, c0), then its edges (all from x-only sources);
+//   y only:  a = fma(wy, y, c0), then its edges (all from y-only sources);
+//   joint:   sx = fma(wx, x, c0) and the edges from x-only sources,
+//            sy = wy * y and the edges from y-only sources,
+//            a = sx + sy, then the edges from joint sources;
+// each edge adds fma(w, v_source, a); the node's value is act(a).
 struct SpecLayout {
   int64_t stride;
   int32_t nv_cap, nve_cap;
@@ -177,13 +188,20 @@ inline SpecLayout spec_layout(int nv_cap, int nve_cap) {
   return L;
 }
 
-// Kernel class of a pair by its varying-node count: 0 = interpreter (more than
-// kDenseMax), 1 = dense up to 12, 2 = dense up to 8, 3 = dense up to 4
-// (includes constant outputs). Classes run in this order, heaviest first.
-constexpr int kClasses = 4;
-__host__ __device__ __forceinline__ int pair_class(int nv) {
-  return nv > kDenseMax ? 0 : nv > 8 ? 1 : nv > 4 ? 2 : 3;
+// Kernel class of a pair by its varying-node count nv and its joint-node count
+// nj: 0 = interpreter (nv above kDenseMax); otherwise by the joint nodes, the
+// only ones evaluated per position: 1 = up to 12, 2 = up to 8, 3 = up to 4,
+// 4 = none (the output depends on one coordinate, or on none: constant outputs
+// are the last pairs of class 4). Classes run in this order, heaviest first.
+constexpr int kClasses = 5;
+__host__ __device__ __forceinline__ int pair_class(int nv, int nj) {
+  return nv > kDenseMax ? 0 : nj > 8 ? 1 : nj > 4 ? 2 : nj > 0 ? 3 : 4;
 }
+
+// Header word 3 of a record: its kernel class (bits 0..3) and, when nv <=
+// kDenseMax, the joint-node count (bits 4..7) and the slot masks of the x-only
+// (bits 8..19) and y-only (bits 20..31) nodes.
+constexpr int kHdrJointShift = 4, kHdrXShift = 8, kHdrYShift = 20;
 
 struct QueryDev {
   const float *a, *b;
@@ -211,7 +229,7 @@ __device__ void schedule_block(const uint8_t* __restrict__ pack, QueryDev q, int
     const int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
     const int side = q.side[si] ? 1 : 0;
     const uint32_t c = min(gt[g].cost[side], uint32_t(kClassBins - 1));
-    return pair_class(gt[g].n_varying[side]) * kClassBins + (kClassBins - 1 - int(c));
+    return pair_class(gt[g].n_varying[side], gt[g].n_joint[side]) * kClassBins + (kClassBins - 1 - int(c));
   };
   for (int64_t r = tid; r < n_pairs; r += nthreads) atomicAdd(&hist[bin_of(r)], 1);
   __syncthreads();
@@ -274,7 +292,7 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
   uint8_t* rec = spec + r * L.stride;
   int32_t* hdr = reinterpret_cast<int32_t*>(rec);
   if (q.per_genome && q.count && s >= q.count[g]) {  // unused slot: constant 0, nothing kept
-    if (lane == 0) { hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = pair_class(0); }
+    if (lane == 0) { hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = pair_class(0, 0); }
     return;
   }
   const PackGenome G = gt[g];
@@ -291,10 +309,13 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
     float4* coef = reinterpret_cast<float4*>(rec + L.coef_off());
     uint2* ve = reinterpret_cast<uint2*>(rec + L.edge_off());
     float out_const = 0.f;
+    uint32_t xm = 0, ym = 0;
+    int nj = 0;
     for (int t = 0; t < G.n_nodes; t++) {
       const PackNode nd = nt[G.node_beg + t];
       const PackEdge* ed = et + G.edge_beg + nd.edge_beg;
       if (nd.vary & (1u << side)) {
+        const uint32_t ax = (uint32_t(nd.axes) >> (2 * side)) & 3u;
         float c0 = nd.bias;
         for (int k = 0; k < 5; k++)
           if (k != gx && k != gy) c0 = fmaf(nd.w_in[k], in[k], c0);
@@ -302,20 +323,23 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
         for (int e = 0; e < nd.edge_cnt; e++) {
           const PackNode src = nt[G.node_beg + ed[e].src];
           if (src.vary & (1u << side)) {
-            ve[nve++] = make_uint2(__float_as_uint(cval[ed[e].src]), __float_as_uint(ed[e].w));
+            const uint32_t sa = (uint32_t(src.axes) >> (2 * side)) & 3u;
+            ve[nve++] = make_uint2(__float_as_uint(cval[ed[e].src]) | (sa << 16), __float_as_uint(ed[e].w));
           } else {
             c0 = fmaf(ed[e].w, cval[ed[e].src], c0);
           }
         }
-        for (int e = eb + 1; e < nve; e++) {  // ascending source slot (insertion sort, a few edges)
+        for (int e = eb + 1; e < nve; e++) {  // ascending (source axes, slot) (insertion sort, a few edges)
           const uint2 key = ve[e];
           int f = e - 1;
           while (f >= eb && ve[f].x > key.x) { ve[f + 1] = ve[f]; f--; }
           ve[f + 1] = key;
         }
-        uint32_t info = uint32_t(nd.act) | (uint32_t(eb) << 8) | (uint32_t(nve - eb) << 20);
+        uint32_t info = uint32_t(nd.act) | (ax << 4) | (uint32_t(eb) << 8) | (uint32_t(nve - eb) << 20);
         coef[nv] = make_float4(c0, nd.w_in[gx], nd.w_in[gy], __uint_as_float(info));
         cval[t] = __uint_as_float(uint32_t(nv));
+        if (ax == kAxisXY) nj++;
+        else if (nv < kDenseMax) (ax == kAxisX ? xm : ym) |= 1u << nv;
         nv++;
       } else {
         float z = nd.bias;
@@ -328,7 +352,8 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
     hdr[0] = nv;
     hdr[1] = nve;
     reinterpret_cast<float*>(hdr)[2] = out_const;
-    hdr[3] = pair_class(nv);
+    hdr[3] = pair_class(nv, nj) |
+             (nv <= kDenseMax ? uint32_t(nj) << kHdrJointShift | xm << kHdrXShift | ym << kHdrYShift : 0u);
   }
   nv = __shfl_sync(0xffffffffu, nv, 0);
   __syncwarp();  // lane 0's coefficient and edge records are visible to the warp
@@ -341,7 +366,7 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
       const uint2* ve = reinterpret_cast<const uint2*>(rec + L.edge_off());
       const uint32_t info = __float_as_uint(coef[lane].w);
       const int eb = int((info >> 8) & 0xfffu), ec = int(info >> 20);
-      for (int e = eb; e < eb + ec; e++) W[lane * kDenseMax + int(ve[e].x)] += __uint_as_float(ve[e].y);
+      for (int e = eb; e < eb + ec; e++) W[lane * kDenseMax + int(ve[e].x & 0xffffu)] += __uint_as_float(ve[e].y);
     }
   }
 }
@@ -376,6 +401,45 @@ struct TileArgs {
   int64_t n_dense;
 };
 
+// Input of one node (its value before the activation) at NP points, from the
+// record's edge list in the evaluators' common order (see the record layout):
+// coefficients c, edges [eb, ee), source values val(slot, p).
+template <int NP, class Val>
+__device__ __forceinline__ void node_input_sparse(const float4 c, const uint2* __restrict__ ve, int eb, int ee,
+                                                  const float (&x)[NP], const float (&y)[NP], Val val,
+                                                  float (&z)[NP]) {
+  const uint32_t ax = (__float_as_uint(c.w) >> 4) & 3u;
+  float sy[NP];
+#pragma unroll
+  for (int p = 0; p < NP; p++) {
+    z[p] = ax == kAxisY ? fmaf(c.z, y[p], c.x) : fmaf(c.y, x[p], c.x);
+    sy[p] = __fmul_rn(c.z, y[p]);
+  }
+  bool merged = ax != kAxisXY;  // joint: x part in z, y part in sy until the first joint source
+  for (int e = eb; e < ee; e++) {
+    const uint2 E = ve[e];
+    const uint32_t sa = E.x >> 16;
+    const int src = int(E.x & 0xffffu);
+    const float we = __uint_as_float(E.y);
+    if (!merged && sa == kAxisY) {
+#pragma unroll
+      for (int p = 0; p < NP; p++) sy[p] = fmaf(we, val(src, p), sy[p]);
+      continue;
+    }
+    if (!merged && sa == kAxisXY) {
+#pragma unroll
+      for (int p = 0; p < NP; p++) z[p] = __fadd_rn(z[p], sy[p]);
+      merged = true;
+    }
+#pragma unroll
+    for (int p = 0; p < NP; p++) z[p] = fmaf(we, val(src, p), z[p]);
+  }
+  if (!merged) {
+#pragma unroll
+    for (int p = 0; p < NP; p++) z[p] = __fadd_rn(z[p], sy[p]);
+  }
+}
+
 // CPPN at four points by interpreting the pair's record: node values live in
 // shared memory, one float4 (four points) per thread and varying node.
 __device__ __forceinline__ void eval4_interp(const float4* __restrict__ coef, const uint2* __restrict__ ve,
@@ -385,28 +449,20 @@ __device__ __forceinline__ void eval4_interp(const float4* __restrict__ coef, co
     w[0] = w[1] = w[2] = w[3] = out_const;
     return;
   }
-  float z0 = 0.f, z1 = 0.f, z2 = 0.f, z3 = 0.f;
+  float z[4];
+  auto val = [&](int src, int p) {
+    const float4& v = vals[src * kBlock + tid];
+    return p == 0 ? v.x : p == 1 ? v.y : p == 2 ? v.z : v.w;
+  };
   for (int k = 0; k < nv; k++) {
     const float4 c = coef[k];
     const uint32_t info = __float_as_uint(c.w);
-    z0 = fmaf(c.z, y[0], fmaf(c.y, x[0], c.x));
-    z1 = fmaf(c.z, y[1], fmaf(c.y, x[1], c.x));
-    z2 = fmaf(c.z, y[2], fmaf(c.y, x[2], c.x));
-    z3 = fmaf(c.z, y[3], fmaf(c.y, x[3], c.x));
     const int eb = int((info >> 8) & 0xfffu), ee = eb + int(info >> 20);
-    for (int e = eb; e < ee; e++) {
-      const uint2 E = ve[e];
-      const float we = __uint_as_float(E.y);
-      const float4 v = vals[int(E.x) * kBlock + tid];
-      z0 = fmaf(we, v.x, z0);
-      z1 = fmaf(we, v.y, z1);
-      z2 = fmaf(we, v.z, z2);
-      z3 = fmaf(we, v.w, z3);
-    }
-    act_apply4(int(info & 0xffu), z0, z1, z2, z3);
-    if (k + 1 < nv) vals[k * kBlock + tid] = make_float4(z0, z1, z2, z3);
+    node_input_sparse<4>(c, ve, eb, ee, x, y, val, z);
+    act_apply4(int(info & 0xfu), z[0], z[1], z[2], z[3]);
+    if (k + 1 < nv) vals[k * kBlock + tid] = make_float4(z[0], z[1], z[2], z[3]);
   }
-  w[0] = z0; w[1] = z1; w[2] = z2; w[3] = z3;
+  w[0] = z[0]; w[1] = z[1]; w[2] = z[2]; w[3] = z[3];
 }
 
 __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
@@ -550,16 +606,20 @@ __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
 
 // ---- register-resident tiles (pairs with at most kDenseMax varying nodes) ---------
 //
-// A CTA of 256 threads owns one tile: either a 64 x 64 Morton block of one
-// depth >= 5, or (tile 0 of a pair) the whole of depths 0..4, one depth after
-// the other. Each thread evaluates sibling quads (the four children of one
-// parent cell) with the CPPN's node values in registers: node k is
-// act(c0 + wx x + wy y + sum_{j<k} W[k][j] v_j) with the loop unrolled to NVMAX
-// and a uniform early exit at the pair's node count, so every register index
-// is static. The quad's variance comes straight from its four results; the
-// band value needs the neighbours, taken from the tile in shared memory after
-// a barrier (the ring of out-of-tile neighbours is evaluated by the tile too).
-
+// A CTA of 128 threads owns one tile: either a 64 x 64 Morton block of one
+// depth >= 5, or (tile 0 of a pair) the whole of depths 0..4. A node that
+// depends on one grid coordinate has one value per tile column (x) or row (y):
+// the CTA first evaluates those nodes at the tile's distinct coordinates into
+// shared-memory tables, together with the x part and the y part of every joint
+// node's input (both coordinates). Then each thread evaluates sibling quads
+// (the four children of one parent cell): a joint node's input is its x part
+// plus its y part from the tables, plus its edges from joint sources, with the
+// joint nodes' values in registers (loop unrolled to NJMAX with a uniform early
+// exit, so every register index is static). An output of one coordinate is
+// read from its table. The quad's variance comes straight from its four
+// results; the band value needs the neighbours, taken from the tile in shared
+// memory after a barrier (the ring of out-of-tile neighbours is evaluated by the
+// tile too).
 
 struct DTileArgs {
   const uint8_t* spec;
@@ -567,6 +627,7 @@ struct DTileArgs {
   const int32_t* order;
   int64_t rank_beg;
   int32_t n_tiles, tile_beg;
+  int32_t tiles_per_cta;  // consecutive tiles of one pair per CTA (blockIdx.x: tile group)
   int64_t band_stride, band_shift, out_stride, out_shift;
   int32_t D, mode;
   float theta, band, w_min;
@@ -608,33 +669,150 @@ __device__ __forceinline__ void act_applyN(int a, float (&z)[NP]) {
   }
 }
 
-// CPPN of one pair at NP points (x[p], y[p]); returns the output node's value.
-template <int NVMAX, int NP>
-__device__ __forceinline__ void eval_dense(const float4* __restrict__ coef, const float* __restrict__ W, int nv,
-                                           float out_const, const float (&x)[NP], const float (&y)[NP],
-                                           float (&w)[NP]) {
-  float v[NVMAX][NP];
-#pragma unroll
-  for (int p = 0; p < NP; p++) w[p] = out_const;
-#pragma unroll
-  for (int k = 0; k < NVMAX; k++) {
-    if (k >= nv) break;
-    const float4 c = coef[k];
-    float z[NP];
-#pragma unroll
-    for (int p = 0; p < NP; p++) z[p] = fmaf(c.z, y[p], fmaf(c.y, x[p], c.x));
-#pragma unroll
-    for (int j = 0; j < k; j++) {
-      const float wk = W[k * NVMAX + j];
-#pragma unroll
-      for (int p = 0; p < NP; p++) z[p] = fmaf(wk, v[j][p], z[p]);
+// Node tables of a dense tile CTA, [axis][row][column]. Rows of axis a: first
+// the joint nodes (row m: the axis-a part of joint node m's input), then the
+// nodes of coordinate a alone (their values), in slot order. Tile-local
+// coordinate index i sits at column i + 2, so the columns of sibling positions
+// (2 c, 2 c + 1) are 8-byte aligned. A 64 x 64 tile uses i = -1 .. 64 (ring
+// included); the pyramid tile keeps depth d at columns seg(d) + i + 2,
+// i = -1 .. 2^(d+1).
+constexpr int kTabFull = kTileSide + 4;
+__host__ __device__ constexpr int tab_seg(int d) { return (2 << d) - 2 + 4 * d; }
+constexpr int kTabPyr = tab_seg(kPyramidTop + 1);
+
+// Table program of one axis, built once per CTA: an entry per node with a row
+// on that axis, in slot order: {c0, c, info} with info = row | kEntMul (the
+// input starts as c * coordinate, the y part of a joint node) | kEntJoint (the
+// row holds the input, no activation) | act << 7 | first source << 10 |
+// source count << 18; sources {row of the source, weight}, in slot order.
+constexpr uint32_t kEntMul = 1u << 5, kEntJoint = 1u << 6;
+constexpr int kEntSrcCap = kDenseMax * (kDenseMax - 1) / 2;
+
+// One table column: every entry of the axis at coordinate value cv (the common
+// order of the record layout; a node of one coordinate has sources of that
+// coordinate only).
+__device__ __forceinline__ void table_column(float cv, int pos, int n_ent, const float4* __restrict__ ent,
+                                             const float2* __restrict__ src, float* __restrict__ tab, int tw) {
+  for (int e = 0; e < n_ent; e++) {
+    const float4 E = ent[e];
+    const uint32_t info = __float_as_uint(E.z);
+    float z = (info & kEntMul) ? __fmul_rn(E.y, cv) : fmaf(E.y, cv, E.x);
+    const int sb = int((info >> 10) & 0xffu), se = sb + int(info >> 18);
+    for (int k = sb; k < se; k++) {
+      const float2 S = src[k];
+      z = fmaf(S.y, tab[__float_as_int(S.x) * tw + pos], z);
     }
-    act_applyN<NP>(int(__float_as_uint(c.w) & 0xffu), z);
+    tab[int(info & 31u) * tw + pos] = (info & kEntJoint) ? z : act_apply(int((info >> 7) & 7u), z);
+  }
+}
+
+// The joint nodes of a pair at NP points: init(m, z) gives joint node m's x
+// part plus y part; its edges from earlier joint nodes (WJ, row-major NJMAX x
+// NJMAX, 0 where there is no edge) follow in slot order. w: the last joint
+// node's value, the output.
+template <int NJMAX, int NP, class Init>
+__device__ __forceinline__ void eval_joint(int nj, const float* __restrict__ WJ, const int* __restrict__ jact,
+                                           Init init, float (&w)[NP]) {
+  float v[NJMAX > 0 ? NJMAX : 1][NP];
+#pragma unroll
+  for (int m = 0; m < NJMAX; m++) {
+    if (m >= nj) break;
+    float z[NP];
+    init(m, z);
+#pragma unroll
+    for (int m2 = 0; m2 < m; m2++) {
+      const float wk = WJ[m * NJMAX + m2];
+      if (wk != 0.f) {
+#pragma unroll
+        for (int p = 0; p < NP; p++) z[p] = fmaf(wk, v[m2][p], z[p]);
+      }
+    }
+    act_applyN<NP>(jact[m], z);
 #pragma unroll
     for (int p = 0; p < NP; p++) {
-      v[k][p] = z[p];
+      v[m][p] = z[p];
       w[p] = z[p];
     }
+  }
+}
+
+// Per-CTA view of a pair for the table evaluators.
+struct PairTabs {
+  const float* tx;  // axis-0 table
+  const float* ty;  // axis-1 table
+  int tw;           // table row length
+  int nv, nj;
+  bool out_x;       // output of one coordinate: x (else y)
+  int orow;         // its row
+  float out_const;
+};
+
+// Output at NP points given by their table columns (xp, yp).
+template <int NJMAX, int NP>
+__device__ __forceinline__ void eval_points(const PairTabs& T, const float* __restrict__ WJ,
+                                            const int* __restrict__ jact, const int (&xp)[NP], const int (&yp)[NP],
+                                            float (&w)[NP]) {
+  if constexpr (NJMAX > 0) {
+    if (T.nj > 0) {
+      auto init = [&](int m, float (&z)[NP]) {
+        const float* sx = T.tx + m * T.tw;
+        const float* sy = T.ty + m * T.tw;
+#pragma unroll
+        for (int p = 0; p < NP; p++) z[p] = __fadd_rn(sx[xp[p]], sy[yp[p]]);
+      };
+      eval_joint<NJMAX, NP>(T.nj, WJ, jact, init, w);
+      return;
+    }
+  }
+  if (T.nv == 0) {
+#pragma unroll
+    for (int p = 0; p < NP; p++) w[p] = T.out_const;
+    return;
+  }
+  const float* t = (T.out_x ? T.tx : T.ty) + T.orow * T.tw;
+#pragma unroll
+  for (int p = 0; p < NP; p++) w[p] = t[T.out_x ? xp[p] : yp[p]];
+}
+
+// Output at QPE sibling quads of a 64 x 64 tile: quad h has its children at
+// table columns xq[h], xq[h] + 1 and rows yq[h], yq[h] + 1 (both even), read as
+// pairs; w[4 h + c] is child c (x fastest). Joint node m's parts are row m.
+template <int NJMAX, int QPE>
+__device__ __forceinline__ void eval_quads(const PairTabs& T, const float* __restrict__ WJ,
+                                           const int* __restrict__ jact, const int (&xq)[QPE], const int (&yq)[QPE],
+                                           float (&w)[4 * QPE]) {
+  if constexpr (NJMAX > 0) {
+    if (T.nj > 0) {
+      auto init = [&](int m, float (&z)[4 * QPE]) {
+        const float* sx = T.tx + m * kTabFull;
+        const float* sy = T.ty + m * kTabFull;
+#pragma unroll
+        for (int h = 0; h < QPE; h++) {
+          const float2 a = *reinterpret_cast<const float2*>(sx + xq[h]);
+          const float2 b = *reinterpret_cast<const float2*>(sy + yq[h]);
+          z[4 * h + 0] = __fadd_rn(a.x, b.x);
+          z[4 * h + 1] = __fadd_rn(a.y, b.x);
+          z[4 * h + 2] = __fadd_rn(a.x, b.y);
+          z[4 * h + 3] = __fadd_rn(a.y, b.y);
+        }
+      };
+      eval_joint<NJMAX, 4 * QPE>(T.nj, WJ, jact, init, w);
+      return;
+    }
+  }
+  if (T.nv == 0) {
+#pragma unroll
+    for (int p = 0; p < 4 * QPE; p++) w[p] = T.out_const;
+    return;
+  }
+  const float* t = (T.out_x ? T.tx : T.ty) + T.orow * kTabFull;
+#pragma unroll
+  for (int h = 0; h < QPE; h++) {
+    const float2 a = *reinterpret_cast<const float2*>(t + (T.out_x ? xq[h] : yq[h]));
+    w[4 * h + 0] = a.x;
+    w[4 * h + 1] = T.out_x ? a.y : a.x;
+    w[4 * h + 2] = T.out_x ? a.x : a.y;
+    w[4 * h + 3] = a.y;
   }
 }
 
@@ -675,297 +853,473 @@ __global__ void __launch_bounds__(128) zero_tiles_kernel(const DTileArgs A) {
 // i + 2 (pitch T + 4): two-column padding keeps sibling pairs 8-byte aligned;
 // the ring of out-of-tile neighbours sits in columns / rows 1 and T + 2.
 constexpr int kPad = 2;
+constexpr int kWtFull = (kTileSide + 2 * kPad) * (kTileSide + 2 * kPad);
+// The pyramid tile's padded grids of depths 0..4, one after the other; its node
+// tables follow them in the same buffer.
+__host__ __device__ constexpr int wt_seg(int d) { return d == 0 ? 0 : wt_seg(d - 1) + ((2 << (d - 1)) + 2 * kPad) * ((2 << (d - 1)) + 2 * kPad); }
+constexpr int kWtPyr = wt_seg(kPyramidTop + 1);
+constexpr int kTileBuf = kWtFull + 2 * kDenseMax * kTabFull;
+static_assert(kWtPyr % 4 == 0 && kWtPyr + 2 * kDenseMax * kTabPyr <= kTileBuf, "pyramid tables fit the tile buffer");
+
+// Plane words of a 64 x 64 tile whose output depends on one coordinate. In a
+// word of 32 sibling quads (Morton order), quad bit b has x = 8 xhi + (b0 b2 b4)
+// and y = 4 yhi + (b1 b3), with xhi = word bits (1, 3) and yhi = word bits
+// (0, 2, 4). Given a bit per column pair (x) or row pair (y), the word places
+// it at every quad of that column (row).
+__device__ __forceinline__ uint32_t word_of_columns(uint32_t bits32, uint32_t w) {
+  const uint32_t xhi = ((w >> 1) & 1u) | ((w >> 2) & 2u);
+  const uint32_t b = (bits32 >> (8 * xhi)) & 0xffu;
+  // column bit k to Morton position spread(k) (y = 0), then the four rows (offsets 0, 2, 8, 10)
+  const uint32_t m = (b & 3u) | ((b & 0xcu) << 2) | ((b & 0x30u) << 12) | ((b & 0xc0u) << 14);
+  return m * 0x505u;
+}
+__device__ __forceinline__ uint32_t word_of_rows(uint32_t bits32, uint32_t w) {
+  const uint32_t yhi = (w & 1u) | ((w >> 1) & 2u) | ((w >> 2) & 4u);
+  const uint32_t n = (bits32 >> (4 * yhi)) & 0xfu;
+  // row bit k to Morton position 2 spread(k) (x = 0), then the eight columns
+  const uint32_t m = (n & 1u) | ((n & 2u) << 1) | ((n & 4u) << 6) | ((n & 8u) << 7);
+  return m * 0x00330033u;
+}
 
 // CTAs resident per SM that each class is compiled for (bounds its registers).
-// (measured: 8 / 6 / 4 CTAs of 128 threads keep the three classes spill-free at 56 / 80 / 114 registers)
-constexpr int dense_min_blocks(int nvmax, int tpb) { return (nvmax <= 4 ? 2048 : nvmax <= 8 ? 1536 : 1024) / tpb / 2; }
+constexpr int dense_min_blocks(int njmax, int tpb) { return (njmax <= 4 ? 2048 : njmax <= 8 ? 1536 : 1024) / tpb / 2; }
 
-template <int NVMAX, int TPB>
-__global__ void __launch_bounds__(TPB, dense_min_blocks(NVMAX, TPB)) tile_kernel_dense(const DTileArgs A) {
-  static_assert(NVMAX <= kDenseMax, "dense block holds kDenseMax rows");
+template <int NJMAX, int TPB>
+__global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel_dense(const DTileArgs A) {
+  static_assert(NJMAX <= kDenseMax, "joint block holds at most kDenseMax rows");
   static_assert(TPB >= 64 && TPB <= 256 && (TPB & (TPB - 1)) == 0, "tile work divides evenly");
   constexpr int QPT = kTileSide * kTileSide / 4 / TPB;  // quads per thread in a 64 x 64 tile
   constexpr int P64 = kTileSide + 2 * kPad;
-  __shared__ float4 s_coef[NVMAX];
-  __shared__ __align__(16) float s_W[NVMAX * NVMAX];
-  __shared__ __align__(16) float s_wt[P64 * P64];
-  // quad TPB k of a tile: its Morton coordinates (as floats) and its shared-tile offset
+  constexpr int NJ1 = NJMAX > 0 ? NJMAX : 1;
+  __shared__ float4 s_coef[kDenseMax];
+  __shared__ __align__(16) float s_W[kDenseMax * kDenseMax];
+  __shared__ __align__(16) float s_WJ[NJ1 * NJ1];
+  __shared__ int s_jact[NJ1];
+  __shared__ float4 s_ent[2][kDenseMax];  // table programs of the two axes
+  __shared__ float2 s_esrc[2][kEntSrcCap];
+  __shared__ __align__(16) float s_buf[kTileBuf];  // output tile with its ring, then the node tables
+  // quad TPB k of a tile: its column and row offsets (in positions) and its shared-tile offset
   __shared__ int4 s_kq[QPT];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid < QPT) {
     const int dx = int(compact1by1(uint32_t(TPB * tid))), dy = int(compact1by1(uint32_t(TPB * tid) >> 1));
-    s_kq[tid] = make_int4(__float_as_int(float(dx)), __float_as_int(float(dy)), 2 * dx + 2 * dy * P64, 0);
+    s_kq[tid] = make_int4(2 * dx, 2 * dy, 2 * dx + 2 * dy * P64, 0);
   }
+  // ---- the pair: one record for the CTA's tiles
   const int64_t rank = A.rank_beg + blockIdx.y;
-  const int tile = A.tile_beg + int(blockIdx.x);
   const int r = A.order[rank];
   const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
   const int nv = reinterpret_cast<const int32_t*>(rec)[0];
   const float out_const = reinterpret_cast<const float*>(rec)[2];
+  const uint32_t h3 = reinterpret_cast<const uint32_t*>(rec)[3];
+  const int nj = int((h3 >> kHdrJointShift) & 0xfu);
+  const uint32_t xm = (h3 >> kHdrXShift) & 0xfffu, ym = (h3 >> kHdrYShift) & 0xfffu;
+  const uint32_t jm = ((1u << nv) - 1u) & ~(xm | ym);
   const bool fused = A.mode == kModeFused;
   const bool wfilter = A.w_min > 0.f;
   const float theta16 = 16.f * A.theta, band2 = A.band * A.band;
-  if (tid < NVMAX)
-    s_coef[tid] = tid < nv ? reinterpret_cast<const float4*>(rec + A.L.coef_off())[tid] : make_float4(0, 0, 0, 0);
+  const int t_beg = A.tile_beg + int(blockIdx.x) * A.tiles_per_cta;
+  const int t_end = min(t_beg + A.tiles_per_cta, A.tile_beg + A.n_tiles);
+  if (fused && nv == 0) {  // constant output: every variance and band value is exactly 0
+    for (int t = t_beg; t < t_end; t++) zero_tile(A, r, t, tid, TPB);
+    return;
+  }
   {
+    const float4* gc = reinterpret_cast<const float4*>(rec + A.L.coef_off());
     const float* gW = reinterpret_cast<const float*>(rec + A.L.dense_off());
-    for (int k = tid; k < NVMAX * NVMAX; k += TPB) s_W[k] = gW[(k / NVMAX) * kDenseMax + (k % NVMAX)];
+    if (tid < kDenseMax) s_coef[tid] = tid < nv ? gc[tid] : make_float4(0, 0, 0, 0);
+    for (int k = tid; k < kDenseMax * kDenseMax; k += TPB) s_W[k] = gW[k];
+  }
+  __syncthreads();
+  // table programs: warp a builds axis a (lane k: slot k); read after the first tile's barrier
+  const bool ax_x = (xm | jm) != 0u, ax_y = (ym | jm) != 0u;
+  if (warp < 2) {
+    const int a = warp, k = lane;
+    const uint32_t om = a ? ym : xm, bit = 1u << k, below = bit - 1u;
+    const bool on = k < nv && ((om | jm) & bit) != 0u;
+    const bool joint = (jm & bit) != 0u;
+    uint32_t sm = 0;  // sources: earlier nodes of this coordinate alone with an edge into k
+    if (on)
+      for (uint32_t b = om & below; b; b &= b - 1u)
+        if (s_W[k * kDenseMax + __ffs(b) - 1] != 0.f) sm |= b & (0u - b);
+    const int cnt = __popc(sm);
+    int beg = cnt;  // exclusive prefix over the lanes
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, beg, o);
+      if (lane >= o) beg += y;
+    }
+    beg -= cnt;
+    if (on) {
+      const float4 cf = s_coef[k];
+      const int row = joint ? __popc(jm & below) : nj + __popc(om & below);
+      const uint32_t info = uint32_t(row) | (joint && a ? kEntMul : 0u) | (joint ? kEntJoint : 0u) |
+                            ((__float_as_uint(cf.w) & 7u) << 7) | (uint32_t(beg) << 10) | (uint32_t(cnt) << 18);
+      s_ent[a][__popc((om | jm) & below)] = make_float4(cf.x, a ? cf.z : cf.y, __uint_as_float(info), 0.f);
+      int q = beg;
+      for (uint32_t b = sm; b; b &= b - 1u) {
+        const int j = __ffs(b) - 1;
+        s_esrc[a][q++] = make_float2(__int_as_float(nj + __popc(om & ((1u << j) - 1u))), s_W[k * kDenseMax + j]);
+      }
+    }
+  }
+  const int n_ent_x = __popc((xm | jm) & ((1u << nv) - 1u)), n_ent_y = __popc((ym | jm) & ((1u << nv) - 1u));
+  if constexpr (NJMAX > 0) {  // joint node m is the m-th set bit of jm
+    auto slot_of = [&](int m) {
+      uint32_t b = jm;
+      for (int q = 0; q < m; q++) b &= b - 1u;
+      return b ? __ffs(b) - 1 : 0;
+    };
+    if (tid < NJMAX) s_jact[tid] = int(__float_as_uint(s_coef[slot_of(tid)].w) & 0xfu);
+    for (int t = tid; t < NJMAX * NJMAX; t += TPB) {
+      const int m = t / NJMAX, m2 = t % NJMAX;
+      s_WJ[t] = m < nj && m2 < m ? s_W[slot_of(m) * kDenseMax + slot_of(m2)] : 0.f;
+    }
   }
   __syncthreads();
   uint32_t* split_row = A.split + int64_t(r) * A.n_words;
   const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;
   const int64_t prow = int64_t(r) * A.out_stride - A.out_shift;
+  const int d_hi = min(A.D, kPyramidTop);
+  float* s_wt = s_buf;
 
-  if (tile > 0) {
-    // ---- a full 64 x 64 tile of one depth >= 5: 4 quads and 1 ring point per thread
-    int u = tile - 1, d = kPyramidTop + 1;
-    while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
-    const int n = 1 << (d + 1);
-    const uint32_t mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
-    const int i0 = int(compact1by1(mb)), j0 = int(compact1by1(mb >> 1));
-    const float scale = __int_as_float((127 - (d + 1)) << 23);  // 2^-(d+1): half the grid spacing
-    const int64_t lrow = prow + A.level_off[d];
-    if (fused && nv == 0) {  // constant output: every variance and band value is exactly 0
-      if (tid < 32) split_row[A.word_off[d - 1] + mb / 128 + tid] = 0u;
-      for (int k = tid; k < 128; k += TPB) A.bandb[band_base + A.word_off[d] + mb / 32 + k] = 0u;
-      return;
+  // ---- one tile of the pair
+  auto run_tile = [&](const int tile) {
+    // geometry: a 64 x 64 tile of depth d >= 5 at Morton block mb; tile 0: depths 0..d_hi
+    int d = 0, i0 = 0, j0 = 0;
+    uint32_t mb = 0;
+    if (tile > 0) {
+      int u = tile - 1;
+      d = kPyramidTop + 1;
+      while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
+      mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
+      i0 = int(compact1by1(mb));
+      j0 = int(compact1by1(mb >> 1));
     }
-    // quad q = tid + TPB k of the tile has parent (pl + dx(k), ql + dy(k)), where
-    // (dx, dy) are the Morton coordinates of TPB k (its bits lie above tid's)
-    const int pl = int(compact1by1(uint32_t(tid))), ql = int(compact1by1(uint32_t(tid) >> 1));
-    const float X0 = grid_coord(i0 + 2 * pl, scale), Y0 = grid_coord(j0 + 2 * ql, scale);
-    const float step = 2.f * scale, quad_step = 4.f * scale;  // one column; one quad (two columns)
-    const int sbase = (2 * ql + kPad) * P64 + 2 * pl + kPad;
-    uint32_t* split_k = split_row + A.word_off[d - 1] + mb / 128 + warp;  // this warp's parents, k = 0
-    uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
-    // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the nodes
-    constexpr int QPE = NVMAX <= 4 ? 2 : 1;
-    // A position passes the band test only if both differences along one axis
-    // exceed the band, and one of them is to its sibling in the quad. The sum of the
-    // six squared sibling differences (16 V, rounded upward monotonically) bounds
-    // each of them, so a quad with 16 V within band^2 has no passing position,
-    // whatever its neighbours; need: some quad of this thread may have one.
-    bool need = false;
-#pragma unroll 1
-    for (int k0 = 0; k0 < QPT; k0 += QPE) {
-      float x[4 * QPE], y[4 * QPE], w[4 * QPE];
-      int4 kq[QPE];
-#pragma unroll
-      for (int h = 0; h < QPE; h++) {
-        kq[h] = s_kq[k0 + h];
-        const float xa = fmaf(__int_as_float(kq[h].x), quad_step, X0);
-        const float ya = fmaf(__int_as_float(kq[h].y), quad_step, Y0);
-        x[4 * h + 0] = xa; x[4 * h + 1] = xa + step; x[4 * h + 2] = xa; x[4 * h + 3] = xa + step;
-        y[4 * h + 0] = ya; y[4 * h + 1] = ya; y[4 * h + 2] = ya + step; y[4 * h + 3] = ya + step;
+    const int tw = tile > 0 ? kTabFull : kTabPyr;
+    float* tab = s_buf + (tile > 0 ? kWtFull : kWtPyr);
+    // node tables, one coordinate per thread. A 64 x 64 tile with nodes on one axis
+    // takes its 66 coordinates (ring included); with both, the 64 + 64 inside the
+    // tile, and the four ring coordinates only where a ring is evaluated.
+    auto column = [&](int a, float cv, int pos) {
+      table_column(cv, pos, a ? n_ent_y : n_ent_x, s_ent[a], s_esrc[a], tab + a * kDenseMax * tw, tw);
+    };
+    if (tile > 0) {
+      const float scale = __int_as_float((127 - (d + 1)) << 23);
+      const int n_items = ax_x && ax_y ? 2 * kTileSide : (ax_x || ax_y) ? kTileSide + 2 : 0;
+      for (int u = tid; u < n_items; u += TPB) {
+        const int a = ax_x && ax_y ? u / kTileSide : ax_x ? 0 : 1;
+        const int i = ax_x && ax_y ? u % kTileSide : u - 1;
+        column(a, grid_coord((a ? j0 : i0) + i, scale), i + 2);
       }
-      eval_dense<NVMAX, 4 * QPE>(s_coef, s_W, nv, out_const, x, y, w);
+    } else {
+      const int P = (4 << d_hi) - 2 + 2 * (d_hi + 1);  // sum over depths of 2^(d+1) + 2
+      const int n_items = (ax_x ? P : 0) + (ax_y ? P : 0);
+      for (int u = tid; u < n_items; u += TPB) {
+        const int a = ax_x && u < P ? 0 : 1;
+        int e = 0, v = a == 1 && ax_x ? u - P : u;
+        while (v >= (2 << e) + 2) { v -= (2 << e) + 2; e++; }
+        column(a, grid_coord(v - 1, __int_as_float((127 - (e + 1)) << 23)), tab_seg(e) + v + 1);
+      }
+    }
+    __syncthreads();
+    // the ring coordinates of a 64 x 64 tile with nodes on both axes (CTA-uniform call)
+    auto ring_columns = [&]() {
+      if (ax_x && ax_y) {
+        if (tid < 4) {
+          const int a = tid >> 1, i = tid & 1 ? kTileSide : -1;
+          column(a, grid_coord((a ? j0 : i0) + i, __int_as_float((127 - (d + 1)) << 23)), i + 2);
+        }
+        __syncthreads();
+      }
+    };
+    PairTabs T;
+    T.tx = tab;
+    T.ty = tab + kDenseMax * tw;
+    T.tw = tw;
+    T.nv = nv;
+    T.nj = nj;
+    T.out_x = nv > 0 && ((xm >> (nv - 1)) & 1u) != 0u;
+    T.orow = __popc(T.out_x ? xm : ym) - 1;  // an output of one coordinate (no joint node): its axis' last row
+    T.out_const = out_const;
+
+    if constexpr (NJMAX == 0) {
+      if (tile > 0 && fused && !A.out && nv > 0) {
+        // ---- a 64 x 64 tile whose output f depends on one coordinate: every quad of a
+        // column pair (x) or row pair (y) has the children f0, f1 (twice), so its
+        // variance is 16 V = 4 (f0 - f1)^2 (the six-difference sum, exactly), and a
+        // position's band value is the smaller squared difference to its two
+        // neighbours along that coordinate (the other axis gives 0). Each warp takes
+        // the 32 pairs (one per lane) and writes a quarter of the tile's words.
+        const float* f = (T.out_x ? T.tx : T.ty) + T.orow * kTabFull;  // coordinate i at i + 2
+        const float fl = f[2 * lane + 1], f0 = f[2 * lane + 2], f1 = f[2 * lane + 3], fr = f[2 * lane + 4];
+        const float s01 = sqdiff(f0, f1);
+        bool g0 = fminf(sqdiff(f0, fl), s01) > band2, g1 = fminf(s01, sqdiff(f1, fr)) > band2;
+        if (wfilter) {
+          g0 = g0 && fabsf(f0) > A.w_min;
+          g1 = g1 && fabsf(f1) > A.w_min;
+        }
+        const uint32_t S = __ballot_sync(kFull, 4.f * s01 > theta16);
+        const uint32_t G0 = __ballot_sync(kFull, g0), G1 = __ballot_sync(kFull, g1);
+        // band word 4 j + c holds child c of the quads of split word j: child c lies in the
+        // pair's first or second column (c & 1) or row (c >> 1)
+        const uint32_t j = uint32_t(tid) >> 2, c = uint32_t(tid) & 3u;
+        const uint32_t gsel = (T.out_x ? (c & 1u) : (c >> 1)) ? G1 : G0;
+        A.bandb[band_base + A.word_off[d] + mb / 32 + tid] = T.out_x ? word_of_columns(gsel, j) : word_of_rows(gsel, j);
+        if (tid < 32)
+          split_row[A.word_off[d - 1] + mb / 128 + tid] =
+              T.out_x ? word_of_columns(S, uint32_t(tid)) : word_of_rows(S, uint32_t(tid));
+        if (A.tile_flags && tid == 0 && (G0 | G1) != 0u) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
+        return;
+      }
+    }
+    if (tile > 0) {
+      // ---- a full 64 x 64 tile of one depth >= 5: 4 quads and 1 ring point per thread
+      const int n = 1 << (d + 1);
+      const int64_t lrow = prow + A.level_off[d];
+      // quad q = tid + TPB k of the tile has parent (pl + dx(k), ql + dy(k)), where
+      // (dx, dy) are the Morton coordinates of TPB k (its bits lie above tid's)
+      const int pl = int(compact1by1(uint32_t(tid))), ql = int(compact1by1(uint32_t(tid) >> 1));
+      const int xb = 2 * pl + 2, yb = 2 * ql + 2;  // table columns of this thread's quad k = 0
+      const int sbase = (2 * ql + kPad) * P64 + 2 * pl + kPad;
+      uint32_t* split_k = split_row + A.word_off[d - 1] + mb / 128 + warp;  // this warp's parents, k = 0
+      uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
+      // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the joint nodes
+      constexpr int QPE = NJMAX <= 4 ? 2 : 1;
+      // A position passes the band test only if both differences along one axis
+      // exceed the band, and one of them is to its sibling in the quad. The sum of the
+      // six squared sibling differences (16 V, rounded upward monotonically) bounds
+      // each of them, so a quad with 16 V within band^2 has no passing position,
+      // whatever its neighbours; need: some quad of this thread may have one.
+      bool need = false;
+#pragma unroll 1
+      for (int k0 = 0; k0 < QPT; k0 += QPE) {
+        float w[4 * QPE];
+        int4 kq[QPE];
+        int xq[QPE], yq[QPE];
 #pragma unroll
-      for (int h = 0; h < QPE; h++) {
-        const int k = k0 + h;
-        const float* wq = w + 4 * h;
-        if (fused) {
-          float* t = s_wt + sbase + kq[h].z;
-          *reinterpret_cast<float2*>(t) = make_float2(wq[0], wq[1]);
-          *reinterpret_cast<float2*>(t + P64) = make_float2(wq[2], wq[3]);
-          // the four children give the parent's variance (Section 3.2)
-          const float v16 = var16(wq[0], wq[1], wq[2], wq[3]);
-          const unsigned bal = __ballot_sync(kFull, v16 > theta16);
-          if (lane == 0) split_k[(TPB / 32) * k] = bal;
-          need = need || !(v16 <= band2);
-        } else {
-          *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
-              make_float4(wq[0], wq[1], wq[2], wq[3]);
+        for (int h = 0; h < QPE; h++) {
+          kq[h] = s_kq[k0 + h];
+          xq[h] = xb + kq[h].x;
+          yq[h] = yb + kq[h].y;
+        }
+        eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
+#pragma unroll
+        for (int h = 0; h < QPE; h++) {
+          const int k = k0 + h;
+          const float* wq = w + 4 * h;
+          if (fused) {
+            // the four children give the parent's variance (Section 3.2)
+            const float v16 = var16(wq[0], wq[1], wq[2], wq[3]);
+            const unsigned bal = __ballot_sync(kFull, v16 > theta16);
+            if (lane == 0) split_k[(TPB / 32) * k] = bal;
+            need = need || !(v16 <= band2);
+          } else {
+            *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
+                make_float4(wq[0], wq[1], wq[2], wq[3]);
+          }
         }
       }
-    }
-    if (fused && !__syncthreads_or(need)) {  // no position of the tile can pass
-      if (lane == 0)
-        for (int k = 0; k < QPT; k++) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
-      return;
-    }
-    // ring: 4 sides x 64 points, evaluated four at a time by threads 0..63
-    // (point t = 4 tid + c lies on side t / 64, the same for all four)
-    if (tid < kTileSide && (fused || A.out_halo)) {
-      const int sd = tid >> 4, u0 = 4 * (tid & 15);
-      int li[4], lj[4];
-      float x[4], y[4], w[4];
-      bool use = fused;
-#pragma unroll
-      for (int c = 0; c < 4; c++) {
-        li[c] = sd == 0 ? -1 : sd == 1 ? kTileSide : u0 + c;
-        lj[c] = sd == 2 ? -1 : sd == 3 ? kTileSide : u0 + c;
-        x[c] = grid_coord(i0 + li[c], scale);
-        y[c] = grid_coord(j0 + lj[c], scale);
+      if (fused && !__syncthreads_or(need)) {  // no position of the tile can pass
+        if (lane == 0)
+          for (int k = 0; k < QPT; k++) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
+        return;
       }
-      const int gi = i0 + li[0], gj = j0 + lj[0];  // a side lies wholly inside or outside the domain
-      const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
-      use = use || outside;  // materialised: only points outside the domain are written
-      if (use) {
-        eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
+      if (fused || A.out_halo) ring_columns();
+      if (fused) {  // a tile the band screen lets through (rare): its outputs again, into the shared tile
+#pragma unroll 1
+        for (int k0 = 0; k0 < QPT; k0 += QPE) {
+          float w[4 * QPE];
+          int4 kq[QPE];
+          int xq[QPE], yq[QPE];
+#pragma unroll
+          for (int h = 0; h < QPE; h++) {
+            kq[h] = s_kq[k0 + h];
+            xq[h] = xb + kq[h].x;
+            yq[h] = yb + kq[h].y;
+          }
+          eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
+#pragma unroll
+          for (int h = 0; h < QPE; h++) {
+            float* t = s_wt + sbase + kq[h].z;
+            *reinterpret_cast<float2*>(t) = make_float2(w[4 * h + 0], w[4 * h + 1]);
+            *reinterpret_cast<float2*>(t + P64) = make_float2(w[4 * h + 2], w[4 * h + 3]);
+          }
+        }
+      }
+      // ring: 4 sides x 64 points, evaluated four at a time by threads 0..63
+      // (point t = 4 tid + c lies on side t / 64, the same for all four)
+      if (tid < kTileSide && (fused || A.out_halo)) {
+        const int sd = tid >> 4, u0 = 4 * (tid & 15);
+        int li[4], lj[4], xp[4], yp[4];
+        float w[4];
 #pragma unroll
         for (int c = 0; c < 4; c++) {
-          if (fused) {
-            s_wt[(lj[c] + kPad) * P64 + li[c] + kPad] = w[c];
-          } else {
-            const int pi_ = i0 + li[c], pj_ = j0 + lj[c];
-            const int hs = pi_ < 0 ? 0 : pi_ >= n ? 1 : pj_ < 0 ? 2 : 3;
-            A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? pj_ : pi_)] = w[c];
+          li[c] = sd == 0 ? -1 : sd == 1 ? kTileSide : u0 + c;
+          lj[c] = sd == 2 ? -1 : sd == 3 ? kTileSide : u0 + c;
+          xp[c] = li[c] + 2;
+          yp[c] = lj[c] + 2;
+        }
+        const int gi = i0 + li[0], gj = j0 + lj[0];  // a side lies wholly inside or outside the domain
+        const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
+        if (fused || outside) {  // materialised: only points outside the domain are written
+          eval_points<NJMAX, 4>(T, s_WJ, s_jact, xp, yp, w);
+#pragma unroll
+          for (int c = 0; c < 4; c++) {
+            if (fused) {
+              s_wt[(lj[c] + kPad) * P64 + li[c] + kPad] = w[c];
+            } else {
+              const int pi_ = i0 + li[c], pj_ = j0 + lj[c];
+              const int hs = pi_ < 0 ? 0 : pi_ >= n ? 1 : pj_ < 0 ? 2 : 3;
+              A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? pj_ : pi_)] = w[c];
+            }
           }
+        }
+      }
+      if (!fused) return;
+      __syncthreads();
+      // band value of each position from its four neighbours at distance 2^-d
+      bool any_pass = false;
+#pragma unroll 2
+      for (int k = 0; k < QPT; k++) {
+        const float* t = s_wt + sbase + s_kq[k].z;  // (2pi, 2pj)
+        const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
+        const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
+        const float l0 = t[-1], l2 = t[P64 - 1], r1 = t[2], r3 = t[P64 + 2];
+        const float w[4] = {w01.x, w01.y, w23.x, w23.y};
+        const float L[4] = {l0, w[0], l2, w[2]}, R[4] = {w[1], r1, w[3], r3};
+        const float Bo[4] = {bel.x, bel.y, w[0], w[1]}, U[4] = {w[2], w[3], abv.x, abv.y};
+        bool pass[4];
+        // squared differences between siblings are shared by both
+        const float h01 = sqdiff(w[0], w[1]), h23 = sqdiff(w[2], w[3]);
+        const float v02 = sqdiff(w[0], w[2]), v13 = sqdiff(w[1], w[3]);
+        const float DL[4] = {sqdiff(w[0], L[0]), h01, sqdiff(w[2], L[2]), h23};
+        const float DR[4] = {h01, sqdiff(w[1], R[1]), h23, sqdiff(w[3], R[3])};
+        const float DB[4] = {sqdiff(w[0], Bo[0]), sqdiff(w[1], Bo[1]), v02, v13};
+        const float DT[4] = {v02, v13, sqdiff(w[2], U[2]), sqdiff(w[3], U[3])};
+#pragma unroll
+        for (int c = 0; c < 4; c++) pass[c] = band_pass_sq(DL[c], DR[c], DB[c], DT[c], band2);
+        if (wfilter) {
+#pragma unroll
+          for (int c = 0; c < 4; c++) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+        }
+        const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+        const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+        any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
+        if (lane == 0)  // the four quad-major words of this warp's 32 quads
+          *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(b0, b1, b2, b3);
+        if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
+          float* o = A.out + lrow + mb + 4 * (tid + TPB * k);
+#pragma unroll
+          for (int c = 0; c < 4; c++)
+            if (pass[c]) o[c] = w[c];
+        }
+      }
+      if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
+      return;
+    }
+
+    // ---- tile 0: depths 0..min(D, 4). One pass evaluates the quads and ring points
+    // of every depth (work items: the quads of depth 0, 1, ..., then four ring
+    // points at a time), one barrier, then each depth is filtered from shared memory.
+    const bool ring = fused || A.out_halo != nullptr;
+    const int n_quads = ((4 << (2 * d_hi)) - 1) / 3;       // quads of depths 0..d_hi
+    const int n_items = n_quads + (ring ? (4 << d_hi) - 2 : 0);  // + ring groups (side / 4 ... of each depth)
+    for (int u = tid; u < n_items; u += TPB) {
+      int e = 0, li[4], lj[4];
+      bool quad = u < n_quads;
+      if (quad) {
+        while (((4 << (2 * e)) - 1) / 3 <= u) e++;
+        const uint32_t q = uint32_t(u - ((1 << (2 * e)) - 1) / 3);
+        const int pi = int(compact1by1(q)), pj = int(compact1by1(q >> 1));
+#pragma unroll
+        for (int c = 0; c < 4; c++) { li[c] = 2 * pi + (c & 1); lj[c] = 2 * pj + (c >> 1); }
+      } else {
+        const int g = u - n_quads;
+        while ((2 << (e + 1)) - 2 <= g) e++;
+        const int Te = 1 << (e + 1);
+#pragma unroll
+        for (int c = 0; c < 4; c++) {  // ring point t lies on side t / Te
+          const int t = 4 * (g - ((2 << e) - 2)) + c, sd = t >> (e + 1), uu = t & (Te - 1);
+          li[c] = sd == 0 ? -1 : sd == 1 ? Te : uu;
+          lj[c] = sd == 2 ? -1 : sd == 3 ? Te : uu;
+        }
+      }
+      const int Te = 1 << (e + 1), pitch = Te + 2 * kPad;
+      int xp[4], yp[4];
+#pragma unroll
+      for (int c = 0; c < 4; c++) { xp[c] = tab_seg(e) + li[c] + 2; yp[c] = tab_seg(e) + lj[c] + 2; }
+      float w[4];
+      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xp, yp, w);
+      if (fused) {
+        const int sb = wt_seg(e);  // this depth's padded grid in shared memory
+#pragma unroll
+        for (int c = 0; c < 4; c++) s_wt[sb + (lj[c] + kPad) * pitch + li[c] + kPad] = w[c];
+      } else if (quad) {
+        const uint32_t q = uint32_t(u - ((1 << (2 * e)) - 1) / 3);
+        *reinterpret_cast<float4*>(A.out + prow + A.level_off[e] + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+      } else {
+#pragma unroll
+        for (int c = 0; c < 4; c++) {
+          const int hs = li[c] < 0 ? 0 : li[c] >= Te ? 1 : lj[c] < 0 ? 2 : 3;
+          A.out_halo[int64_t(r) * A.n_halo + A.halo_off[e] + hs * Te + (hs < 2 ? lj[c] : li[c])] = w[c];
         }
       }
     }
     if (!fused) return;
     __syncthreads();
-    // band value of each position from its four neighbours at distance 2^-d
     bool any_pass = false;
-#pragma unroll 2
-    for (int k = 0; k < QPT; k++) {
-      const float* t = s_wt + sbase + s_kq[k].z;  // (2pi, 2pj)
-      const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
-      const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
-      const float l0 = t[-1], l2 = t[P64 - 1], r1 = t[2], r3 = t[P64 + 2];
-      const float w[4] = {w01.x, w01.y, w23.x, w23.y};
-      const float L[4] = {l0, w[0], l2, w[2]}, R[4] = {w[1], r1, w[3], r3};
-      const float Bo[4] = {bel.x, bel.y, w[0], w[1]}, U[4] = {w[2], w[3], abv.x, abv.y};
-      bool pass[4];
-      // squared differences between siblings are shared by both
-      const float h01 = sqdiff(w[0], w[1]), h23 = sqdiff(w[2], w[3]);
-      const float v02 = sqdiff(w[0], w[2]), v13 = sqdiff(w[1], w[3]);
-      const float DL[4] = {sqdiff(w[0], L[0]), h01, sqdiff(w[2], L[2]), h23};
-      const float DR[4] = {h01, sqdiff(w[1], R[1]), h23, sqdiff(w[3], R[3])};
-      const float DB[4] = {sqdiff(w[0], Bo[0]), sqdiff(w[1], Bo[1]), v02, v13};
-      const float DT[4] = {v02, v13, sqdiff(w[2], U[2]), sqdiff(w[3], U[3])};
+    for (int e = 0; e <= d_hi; e++) {
+      const int Te = 1 << (e + 1), nq = Te * Te / 4, pitch = Te + 2 * kPad, sb = wt_seg(e);
+      const int64_t lrow = prow + A.level_off[e];
+      for (int base = 0; base < nq; base += TPB) {
+        const int q = base + tid;
+        const bool valid = q < nq;
+        bool pass[4] = {false, false, false, false}, split = false;
+        float w[4] = {0.f, 0.f, 0.f, 0.f};
+        if (valid) {
+          const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+          const float* t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+          w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
+          // the four children give the parent's variance (Section 3.2)
+          split = var16(w[0], w[1], w[2], w[3]) > theta16;
+          const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
+          const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
+          const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
 #pragma unroll
-      for (int c = 0; c < 4; c++) pass[c] = band_pass_sq(DL[c], DR[c], DB[c], DT[c], band2);
-      if (wfilter) {
+          for (int c = 0; c < 4; c++) {
+            pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]),
+                                   band2);
+            if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+          }
+        }
+        const int q0 = base + warp * 32;
+        if (e >= 1) {
+          const unsigned bal = __ballot_sync(kFull, split);
+          if (lane == 0 && q0 < nq) split_row[A.word_off[e - 1] + q0 / 32] = bal;
+        }
+        const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+        const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+        any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
+        if (e >= kQuadMajorFrom) {
+          if (lane < 4 && q0 < nq)
+            A.bandb[band_base + A.word_off[e] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+        } else if (q0 == 0 && lane * 32 < 4 * nq) {
+          A.bandb[band_base + A.word_off[e] + lane] = band_word(b0, b1, b2, b3, lane);
+        }
+        if (A.out && valid && (pass[0] | pass[1] | pass[2] | pass[3])) {
 #pragma unroll
-        for (int c = 0; c < 4; c++) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
-      }
-      const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
-      const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-      any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
-      if (lane == 0)  // the four quad-major words of this warp's 32 quads
-        *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(b0, b1, b2, b3);
-      if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
-        float* o = A.out + lrow + mb + 4 * (tid + TPB * k);
-#pragma unroll
-        for (int c = 0; c < 4; c++)
-          if (pass[c]) o[c] = w[c];
-      }
-    }
-    if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
-    return;
-  }
-
-  // ---- tile 0: depths 0..min(D, 4). One pass evaluates the quads and ring points
-  // of every depth (work items: the quads of depth 0, 1, ..., then four ring
-  // points at a time), one barrier, then each depth is filtered from shared memory.
-  const int d_hi = min(A.D, kPyramidTop);
-  if (fused && nv == 0) {
-    for (int d = 0; d <= d_hi; d++) {
-      const int nq = 1 << (2 * d);
-      for (int k = tid; k < (nq + 31) / 32; k += TPB)
-        if (d >= 1) split_row[A.word_off[d - 1] + k] = 0u;
-      for (int k = tid; k < (4 * nq + 31) / 32; k += TPB) A.bandb[band_base + A.word_off[d] + k] = 0u;
-    }
-    return;
-  }
-  const bool ring = fused || A.out_halo != nullptr;
-  const int n_quads = ((4 << (2 * d_hi)) - 1) / 3;       // quads of depths 0..d_hi
-  const int n_items = n_quads + (ring ? (4 << d_hi) - 2 : 0);  // + ring groups (side / 4 ... of each depth)
-  for (int u = tid; u < n_items; u += TPB) {
-    int d = 0, li[4], lj[4];
-    bool quad = u < n_quads;
-    if (quad) {
-      while (((4 << (2 * d)) - 1) / 3 <= u) d++;
-      const uint32_t q = uint32_t(u - ((1 << (2 * d)) - 1) / 3);
-      const int pi = int(compact1by1(q)), pj = int(compact1by1(q >> 1));
-#pragma unroll
-      for (int c = 0; c < 4; c++) { li[c] = 2 * pi + (c & 1); lj[c] = 2 * pj + (c >> 1); }
-    } else {
-      const int g = u - n_quads;
-      while ((2 << (d + 1)) - 2 <= g) d++;
-      const int T = 1 << (d + 1);
-#pragma unroll
-      for (int c = 0; c < 4; c++) {  // ring point t lies on side t / T
-        const int t = 4 * (g - ((2 << d) - 2)) + c, sd = t >> (d + 1), uu = t & (T - 1);
-        li[c] = sd == 0 ? -1 : sd == 1 ? T : uu;
-        lj[c] = sd == 2 ? -1 : sd == 3 ? T : uu;
-      }
-    }
-    const int T = 1 << (d + 1), pitch = T + 2 * kPad;
-    const float scale = __int_as_float((127 - (d + 1)) << 23);
-    float x[4], y[4], w[4];
-#pragma unroll
-    for (int c = 0; c < 4; c++) { x[c] = grid_coord(li[c], scale); y[c] = grid_coord(lj[c], scale); }
-    eval_dense<NVMAX, 4>(s_coef, s_W, nv, out_const, x, y, w);
-    if (fused) {
-      int sb = 0;  // this depth's padded grid in shared memory
-      for (int e = 0; e < d; e++) sb += ((2 << e) + 2 * kPad) * ((2 << e) + 2 * kPad);
-#pragma unroll
-      for (int c = 0; c < 4; c++) s_wt[sb + (lj[c] + kPad) * pitch + li[c] + kPad] = w[c];
-    } else if (quad) {
-      const uint32_t q = uint32_t(u - ((1 << (2 * d)) - 1) / 3);
-      *reinterpret_cast<float4*>(A.out + prow + A.level_off[d] + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
-    } else {
-#pragma unroll
-      for (int c = 0; c < 4; c++) {
-        const int hs = li[c] < 0 ? 0 : li[c] >= T ? 1 : lj[c] < 0 ? 2 : 3;
-        A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * T + (hs < 2 ? lj[c] : li[c])] = w[c];
-      }
-    }
-  }
-  if (!fused) return;
-  __syncthreads();
-  int sb = 0;
-  bool any_pass = false;
-  for (int d = 0; d <= d_hi; d++) {
-    const int T = 1 << (d + 1), nq = T * T / 4, pitch = T + 2 * kPad;
-    const int64_t lrow = prow + A.level_off[d];
-    for (int base = 0; base < nq; base += TPB) {
-      const int q = base + tid;
-      const bool valid = q < nq;
-      bool pass[4] = {false, false, false, false}, split = false;
-      float w[4] = {0.f, 0.f, 0.f, 0.f};
-      if (valid) {
-        const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-        const float* t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
-        w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
-        // the four children give the parent's variance (Section 3.2)
-        split = var16(w[0], w[1], w[2], w[3]) > theta16;
-        const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
-        const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
-        const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
-#pragma unroll
-        for (int c = 0; c < 4; c++) {
-          pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]),
-                                 band2);
-          if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+          for (int c = 0; c < 4; c++)
+            if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
         }
       }
-      const int q0 = base + warp * 32;
-      if (d >= 1) {
-        const unsigned bal = __ballot_sync(kFull, split);
-        if (lane == 0 && q0 < nq) split_row[A.word_off[d - 1] + q0 / 32] = bal;
-      }
-      const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
-      const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-      any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
-      if (d >= kQuadMajorFrom) {
-        if (lane < 4 && q0 < nq)
-          A.bandb[band_base + A.word_off[d] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
-      } else if (q0 == 0 && lane * 32 < 4 * nq) {
-        A.bandb[band_base + A.word_off[d] + lane] = band_word(b0, b1, b2, b3, lane);
-      }
-      if (A.out && valid && (pass[0] | pass[1] | pass[2] | pass[3])) {
-#pragma unroll
-        for (int c = 0; c < 4; c++)
-          if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
-      }
     }
-    sb += pitch * pitch;
+    if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense] = 1;
+  };
+
+  for (int t = t_beg; t < t_end; t++) {
+    if (t > t_beg) __syncthreads();  // the previous tile's reads of the shared buffer are done
+    run_tile(t);
   }
-  if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense] = 1;
 }
 
 // ---- filter planes from a materialised evaluation ---------------------------------
@@ -1297,34 +1651,26 @@ __global__ void compact_scan_pairs_kernel(const int64_t* __restrict__ counts, in
   if (threadIdx.x == 0) offsets[n_pairs] = carry;
 }
 
-// CPPN output of one grid point from a pair's record, with the arithmetic of the
-// tile kernels operation for operation (the dense evaluator for up to kDenseMax
-// varying nodes, else the edge list in node order), so the value equals the one
-// the tile kernels computed at that position. Interpreted node values go to a
-// local array: records with more than kDenseMax varying nodes are rare.
+// CPPN output of one grid point from a pair's record, in the evaluators'
+// common order (see the record layout), so the value equals the one the tile
+// kernels computed at that position. Node values go to a local array.
 __device__ float eval_record_point(const uint8_t* rec, const SpecLayout& L, float x, float y) {
   const int nv = reinterpret_cast<const int32_t*>(rec)[0];
   const float out_const = reinterpret_cast<const float*>(rec)[2];
   const float4* coef = reinterpret_cast<const float4*>(rec + L.coef_off());
-  if (nv <= kDenseMax) {
-    const float xs[1] = {x}, ys[1] = {y};
-    float w[1];
-    eval_dense<kDenseMax, 1>(coef, reinterpret_cast<const float*>(rec + L.dense_off()), nv, out_const, xs, ys, w);
-    return w[0];
-  }
   const uint2* ve = reinterpret_cast<const uint2*>(rec + L.edge_off());
   float v[EMR_MAX_VARYING];
-  float z = out_const;
+  const float xs[1] = {x}, ys[1] = {y};
+  float z[1] = {out_const};
   for (int k = 0; k < nv; k++) {
     const float4 c = coef[k];
     const uint32_t info = __float_as_uint(c.w);
-    z = fmaf(c.z, y, fmaf(c.y, x, c.x));
     const int eb = int((info >> 8) & 0xfffu), ee = eb + int(info >> 20);
-    for (int e = eb; e < ee; e++) z = fmaf(__uint_as_float(ve[e].y), v[ve[e].x], z);
-    z = act_apply(int(info & 0xffu), z);
-    v[k] = z;
+    node_input_sparse<1>(c, ve, eb, ee, xs, ys, [&](int src, int) { return v[src]; }, z);
+    z[0] = act_apply(int(info & 0xfu), z[0]);
+    v[k] = z[0];
   }
-  return z;
+  return z[0];
 }
 
 // Per-pair records (pair r at spec + r * L.stride) from which the kept weights
@@ -1688,7 +2034,7 @@ GridDev grid_dev(const emr_grid* g) {
 struct EvalPlan {
   int64_t n_pairs;
   int64_t n_class[kClasses];  // pairs per kernel class (schedule order)
-  int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of class 3
+  int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of class 4
   SpecLayout L;
   int32_t scratch_stride;
   size_t spec_bytes, scratch_bytes, order_bytes, total;
@@ -1714,12 +2060,13 @@ emr_status eval_plan(const void* pack_host, const emr_query* q, EvalPlan* p) {
   p->n_const = 0;
   for (int g = 0; g < h->P; g++)
     for (int s = 0; s < q->S; s++) {
-      int nvar = 0;  // unused slots evaluate to a constant
+      int nvar = 0, nj = 0;  // unused slots evaluate to a constant
       if (!(q->per_genome && q->count_host && s >= q->count_host[g])) {
         const int64_t si = q->per_genome ? int64_t(g) * q->S + s : s;
         nvar = gt[g].n_varying[q->side_host[si]];
+        nj = gt[g].n_joint[q->side_host[si]];
       }
-      p->n_class[pair_class(nvar)]++;
+      p->n_class[pair_class(nvar, nj)]++;
       if (nvar == 0) p->n_const++;
     }
   p->L = spec_layout(nv, nve);
@@ -1775,14 +2122,36 @@ int64_t dense_tiles(int D) {
 
 constexpr int kDenseTPB = 128;  // threads per dense tile CTA
 
-template <int NVMAX>
+// Streaming multiprocessors of the current device (queried once per device).
+int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
+  if (dev < 64 && cached[dev] > 0) return cached[dev];
+  int n = 1;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+  if (dev < 64) cached[dev] = n;
+  return n;
+}
+
+// Waves of resident CTAs a dense launch keeps at least, when it groups tiles.
+constexpr int kDenseMinWaves = 4;
+
+template <int NJMAX>
 emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st) {
   if (n_ranks <= 0) return EMR_OK;
   DTileArgs A = A0;
+  // consecutive tiles of a pair share a CTA (one record load and one prologue for
+  // all of them) while the launch still fills every SM kDenseMinWaves times
+  const int64_t slots = int64_t(sm_count()) * dense_min_blocks(NJMAX, kDenseTPB);
+  int g = 8;
+  while (g > 1 && n_ranks * ((A.n_tiles + g - 1) / g) < kDenseMinWaves * slots) g >>= 1;
+  A.tiles_per_cta = g;
+  const unsigned gx = unsigned((A.n_tiles + g - 1) / g);
   for (int64_t r0 = 0; r0 < n_ranks; r0 += 65535) {  // grid y: ranks, at most 65535 a launch
     A.rank_beg = rank_beg + r0;
-    const dim3 grid(unsigned(A.n_tiles), unsigned(std::min<int64_t>(65535, n_ranks - r0)));
-    tile_kernel_dense<NVMAX, kDenseTPB><<<grid, kDenseTPB, 0, st>>>(A);
+    const dim3 grid(gx, unsigned(std::min<int64_t>(65535, n_ranks - r0)));
+    tile_kernel_dense<NJMAX, kDenseTPB><<<grid, kDenseTPB, 0, st>>>(A);
   }
   return cuda_status(cudaGetLastError());
 }
@@ -1891,11 +2260,13 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   beg += p.n_class[1];
   if ((rc = launch_dense<8>(D, beg, p.n_class[2], st)) != EMR_OK) return rc;
   beg += p.n_class[2];
-  if (mode != kModeFused || p.n_const == 0) return launch_dense<4>(D, beg, p.n_class[3], st);
-  if ((rc = launch_dense<4>(D, beg, p.n_class[3] - p.n_const, st)) != EMR_OK) return rc;
+  if ((rc = launch_dense<4>(D, beg, p.n_class[3], st)) != EMR_OK) return rc;
+  beg += p.n_class[3];
+  if (mode != kModeFused || p.n_const == 0) return launch_dense<0>(D, beg, p.n_class[4], st);
+  if ((rc = launch_dense<0>(D, beg, p.n_class[4] - p.n_const, st)) != EMR_OK) return rc;
   // with tile flags, a constant-output pair has none set and its planes are never read: leave them
   if (tile_flags) return EMR_OK;
-  const int64_t c0 = beg + p.n_class[3] - p.n_const;
+  const int64_t c0 = beg + p.n_class[4] - p.n_const;
   for (int64_t r0 = 0; r0 < p.n_const; r0 += 65535) {  // grid y: pairs, at most 65535 a launch
     D.rank_beg = c0 + r0;
     const int64_t nc = std::min<int64_t>(65535, p.n_const - r0);

@@ -213,6 +213,21 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
     if (node_kind[n0 + ld] < EMR_KIND_HIDDEN) return EMR_ERR_ARG;
     S.es.push_back({ls, ld, conn_w[c]});
   }
+  // Parallel connections (same source and destination) become one edge whose
+  // weight is their sum in connection order; an edge of weight 0 contributes
+  // nothing and is dropped. Every evaluator then sees at most one edge per
+  // (source, destination), each of nonzero weight.
+  std::stable_sort(S.es.begin(), S.es.end(),
+                   [](const Edge& a, const Edge& b) { return a.d != b.d ? a.d < b.d : a.s < b.s; });
+  {
+    size_t m = 0;
+    for (size_t k = 0; k < S.es.size();) {
+      Edge e = S.es[k++];
+      while (k < S.es.size() && S.es[k].s == e.s && S.es[k].d == e.d) e.w += S.es[k++].w;
+      if (e.w != 0.f) S.es[m++] = e;
+    }
+    S.es.resize(m);
+  }
   build_csr(n, S.es, true, S.succ_beg, S.succ, S.fill);
   build_csr(n, S.es, false, S.pred_beg, S.pred, S.fill);
   // Kahn's algorithm over every node; ready nodes leave in ascending id order.
@@ -275,7 +290,7 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
       S.in_cnt[t]++;
     }
   }
-  // in-edges from kept non-input nodes, grouped by destination in connection order
+  // in-edges from kept non-input nodes, grouped by destination (ascending source)
   S.in_beg.assign(nk + 1, 0);
   for (int t = 0; t < nk; t++) S.in_beg[t + 1] = S.in_beg[t] + S.in_cnt[t];
   if (S.in_beg[nk] > 65535) return EMR_ERR_RANGE;
@@ -299,26 +314,32 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
   }
   g.n_edges = uint16_t(S.in_beg[nk]);
   for (int side = 0; side < 2; side++) {
-    const unsigned grid_inputs = side == EMR_SIDE_OUT ? (1u << EMR_KIND_X2) | (1u << EMR_KIND_Y2)
-                                                      : (1u << EMR_KIND_X1) | (1u << EMR_KIND_Y1);
-    int nv = 0, nve = 0;
+    const int gx = side == EMR_SIDE_OUT ? EMR_KIND_X2 : EMR_KIND_X1;
+    const int gy = side == EMR_SIDE_OUT ? EMR_KIND_Y2 : EMR_KIND_Y1;
+    int nv = 0, nve = 0, nj = 0;
     uint32_t cost = 0;
     for (int t = 0; t < nk; t++) {
-      bool vary = (S.has_in[t] & grid_inputs) != 0;
+      // the grid coordinates the node depends on: its own grid inputs and those of its sources
+      uint32_t ax = ((S.has_in[t] >> gx) & 1u) * kAxisX | ((S.has_in[t] >> gy) & 1u) * kAxisY;
       int vin = 0;
-      for (int k = S.in_beg[t]; k < S.in_beg[t + 1]; k++)
-        if (on[oe[k].src].vary & (1u << side)) { vary = true; vin++; }
-      if (vary) {
+      for (int k = S.in_beg[t]; k < S.in_beg[t + 1]; k++) {
+        const uint32_t sa = (on[oe[k].src].axes >> (2 * side)) & 3u;
+        if (sa) { ax |= sa; vin++; }
+      }
+      if (ax) {
         on[t].vary |= uint8_t(1u << side);
+        on[t].axes |= uint8_t(ax << (2 * side));
         nv++;
         nve += vin;
-        cost += 2 + vin + act_cost(on[t].act);
+        // per-query work: a node of one coordinate is evaluated once per tile row or column
+        if (ax == kAxisXY) { nj++; cost += 2 + vin + act_cost(on[t].act); }
       }
     }
     if (nv > EMR_MAX_VARYING || nve > EMR_MAX_VEDGES) return EMR_ERR_RANGE;
     g.n_varying[side] = uint16_t(nv);
     g.n_vedges[side] = uint16_t(nve);
-    g.cost[side] = cost;
+    g.n_joint[side] = uint16_t(nj);
+    g.cost[side] = cost + (nv > nj ? 1u : 0u);
   }
   return EMR_OK;
 }

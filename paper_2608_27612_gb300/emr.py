@@ -633,8 +633,8 @@ _HDR = np.dtype([("magic", "<u4"), ("version", "<u4"), ("P", "<i4"), ("max_nodes
                  ("max_varying", "<i4", 2), ("max_vedges", "<i4", 2), ("max_edges", "<i4"), ("reserved", "<i4"),
                  ("off_genomes", "<u8"), ("off_nodes", "<u8"), ("off_edges", "<u8"), ("total", "<u8")])
 _GEN = np.dtype([("node_beg", "<u4"), ("edge_beg", "<u4"), ("n_nodes", "<u2"), ("n_edges", "<u2"),
-                 ("n_varying", "<u2", 2), ("n_vedges", "<u2", 2), ("cost", "<u4", 2), ("reserved", "<u4")])
-_NODE = np.dtype([("act", "u1"), ("vary", "u1"), ("reserved", "<u2"), ("edge_beg", "<u2"), ("edge_cnt", "<u2"),
+                 ("n_varying", "<u2", 2), ("n_vedges", "<u2", 2), ("cost", "<u4", 2), ("n_joint", "<u2", 2)])
+_NODE = np.dtype([("act", "u1"), ("vary", "u1"), ("axes", "u1"), ("reserved", "u1"), ("edge_beg", "<u2"), ("edge_cnt", "<u2"),
                   ("bias", "<f4"), ("w_in", "<f4", 5)])
 _EDGE = np.dtype([("src", "<u2"), ("reserved", "<u2"), ("w", "<f4")])
 

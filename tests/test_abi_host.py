@@ -88,8 +88,8 @@ def _pack_records(blob):
         ("max_vedges", "<i4", 2), ("max_edges", "<i4"), ("reserved", "<i4"), ("off_genomes", "<u8"),
         ("off_nodes", "<u8"), ("off_edges", "<u8"), ("total", "<u8")]))[0]
     gdt = np.dtype([("node_beg", "<u4"), ("edge_beg", "<u4"), ("n_nodes", "<u2"), ("n_edges", "<u2"),
-                    ("n_varying", "<u2", 2), ("n_vedges", "<u2", 2), ("cost", "<u4", 2), ("reserved", "<u4")])
-    ndt = np.dtype([("act", "u1"), ("vary", "u1"), ("r", "<u2"), ("edge_beg", "<u2"), ("edge_cnt", "<u2"),
+                    ("n_varying", "<u2", 2), ("n_vedges", "<u2", 2), ("cost", "<u4", 2), ("n_joint", "<u2", 2)])
+    ndt = np.dtype([("act", "u1"), ("vary", "u1"), ("axes", "u1"), ("r", "u1"), ("edge_beg", "<u2"), ("edge_cnt", "<u2"),
                     ("bias", "<f4"), ("w_in", "<f4", 5)])
     P = int(h["P"])
     gs = np.frombuffer(blob.tobytes(), gdt, P, int(h["off_genomes"]))
@@ -118,6 +118,29 @@ def test_pack_topological_order_dead_nodes_and_variation_flags():
     assert [(int(v) >> 1) & 1 for v in nd["vary"]] == [1, 0, 0, 1]
     assert tuple(g["n_varying"]) == (3, 2)
     assert emr.pack_info(blob) == (1, 3, 2)
+    # grid coordinates per side (bits 2 s: x, 2 s + 1: y): OUT side 12, 10, out follow x2 only;
+    # IN side 7 and the output follow x1 only; no node depends on both coordinates
+    assert [int(a) for a in nd["axes"]] == [4, 1, 1, 5]
+    assert tuple(g["n_joint"]) == (0, 0)
+
+
+def test_pack_merges_parallel_connections_and_drops_zero_weights():
+    # 6 -> out twice (0.5 + 0.25 = 0.75); 7 -> out cancels (1 - 1 = 0), so 7 is dropped with its
+    # edge; x2 -> 8 twice with weights summing to 0 leaves 8 with the y2 input only
+    nodes = [(5, OUT, IDN, 0.0), (6, HID, SIG, 0.0), (7, HID, SIN, 0.0), (8, HID, TNH, 0.0)]
+    conns = [(X2, 6, 1.0, True), (Y2, 6, 1.0, True), (6, 5, 0.5, True), (7, 5, 1.0, True), (X2, 7, 1.0, True),
+             (6, 5, 0.25, True), (7, 5, -1.0, True), (X2, 8, 2.0, True), (Y2, 8, 1.0, True), (X2, 8, -2.0, True),
+             (8, 5, 1.0, True)]
+    blob = emr.pack_population(_genome(nodes, conns))
+    h, gs, nd = _pack_records(blob)
+    g = gs[0]
+    assert g["n_nodes"] == 3 and g["n_edges"] == 2  # 6, 8, out; edges 6 -> out, 8 -> out
+    _, _, _, ed = emr.pack_records(blob)
+    assert sorted(float(e["w"]) for e in ed) == [0.75, 1.0]
+    # OUT side: 6 joint (x2, y2), 8 y only (its x2 inputs cancel), the output joint
+    assert [int(a) & 3 for a in nd["axes"]] == [3, 2, 3]
+    assert tuple(g["n_joint"]) == (2, 0) and tuple(g["n_varying"]) == (3, 0)
+    assert nd["w_in"][1][X2] == 0.0 and nd["w_in"][1][Y2] == 1.0
 
 
 def test_pack_rejects_like_the_oracle():

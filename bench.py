@@ -387,7 +387,7 @@ def launches_in_step(emr, dsc):
             np.take_along_axis(gs[field], side.reshape(gs.shape[0], -1), axis=1)
         return f.astype(np.int64)
     nv, nj = per_pair("n_varying"), per_pair("n_joint")
-    cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 4, 2, np.where(nj > 0, 3, 4))))
+    cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 6, 2, np.where(nj > 4, 3, np.where(nj > 0, 4, 5)))))
     return 1 + len(np.unique(cls[nv > 0])) + 4
 
 

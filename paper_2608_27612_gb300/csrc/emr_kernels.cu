@@ -190,12 +190,13 @@ inline SpecLayout spec_layout(int nv_cap, int nve_cap) {
 
 // Kernel class of a pair by its varying-node count nv and its joint-node count
 // nj: 0 = interpreter (nv above kDenseMax); otherwise by the joint nodes, the
-// only ones evaluated per position: 1 = up to 12, 2 = up to 8, 3 = up to 4,
-// 4 = none (the output depends on one coordinate, or on none: constant outputs
-// are the last pairs of class 4). Classes run in this order, heaviest first.
-constexpr int kClasses = 5;
+// only ones evaluated per position: 1 = up to 12, 2 = up to 8, 3 = up to 6,
+// 4 = up to 4, 5 = none (the output depends on one coordinate, or on none:
+// constant outputs are the last pairs of class 5). Classes run in this order,
+// heaviest first.
+constexpr int kClasses = 6;
 __host__ __device__ __forceinline__ int pair_class(int nv, int nj) {
-  return nv > kDenseMax ? 0 : nj > 8 ? 1 : nj > 4 ? 2 : nj > 0 ? 3 : 4;
+  return nv > kDenseMax ? 0 : nj > 8 ? 1 : nj > 6 ? 2 : nj > 4 ? 3 : nj > 0 ? 4 : 5;
 }
 
 // Header word 3 of a record: its kernel class (bits 0..3) and, when nv <=
@@ -467,6 +468,7 @@ __device__ __forceinline__ void eval4_interp(const float4* __restrict__ coef, co
 
 __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
   extern __shared__ float4 smem4[];
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");  // the dense classes may follow as SMs free up
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
   const int tile = A.tile_beg + int(blockIdx.x % A.n_tiles);
@@ -713,26 +715,25 @@ __device__ __forceinline__ void table_column(float cv, int pos, int n_ent, const
 template <int NJMAX, int NP, class Init>
 __device__ __forceinline__ void eval_joint(int nj, const float* __restrict__ WJ, const int* __restrict__ jact,
                                            Init init, float (&w)[NP]) {
-  float v[NJMAX > 0 ? NJMAX : 1][NP];
+  // node m is computed in w; entering node m + 1 keeps it as v[m] for the later nodes
+  float v[NJMAX > 1 ? NJMAX - 1 : 1][NP];
 #pragma unroll
   for (int m = 0; m < NJMAX; m++) {
     if (m >= nj) break;
-    float z[NP];
-    init(m, z);
+    if (m > 0) {
+#pragma unroll
+      for (int p = 0; p < NP; p++) v[m - 1][p] = w[p];
+    }
+    init(m, w);
 #pragma unroll
     for (int m2 = 0; m2 < m; m2++) {
       const float wk = WJ[m * NJMAX + m2];
       if (wk != 0.f) {
 #pragma unroll
-        for (int p = 0; p < NP; p++) z[p] = fmaf(wk, v[m2][p], z[p]);
+        for (int p = 0; p < NP; p++) w[p] = fmaf(wk, v[m2][p], w[p]);
       }
     }
-    act_applyN<NP>(jact[m], z);
-#pragma unroll
-    for (int p = 0; p < NP; p++) {
-      v[m][p] = z[p];
-      w[p] = z[p];
-    }
+    act_applyN<NP>(jact[m], w);
   }
 }
 
@@ -900,6 +901,12 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
   __shared__ __align__(16) float s_buf[kTileBuf];  // output tile with its ring, then the node tables
   // quad TPB k of a tile: its column and row offsets (in positions) and its shared-tile offset
   __shared__ int4 s_kq[QPT];
+  // The next class's launch (other pairs, other outputs) may start filling the SMs
+  // this one frees. When this launch overlaps its predecessor, its last CTA first
+  // waits for the predecessor to complete, so that this launch completes only after
+  // it (later kernels in the stream read every launch's planes).
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) asm volatile("griddepcontrol.wait;" ::: "memory");
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid < QPT) {
     const int dx = int(compact1by1(uint32_t(TPB * tid))), dy = int(compact1by1(uint32_t(TPB * tid) >> 1));
@@ -1084,7 +1091,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
       uint32_t* split_k = split_row + A.word_off[d - 1] + mb / 128 + warp;  // this warp's parents, k = 0
       uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
       // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the joint nodes
-      constexpr int QPE = NJMAX <= 4 ? 2 : 1;
+      constexpr int QPE = NJMAX <= 6 ? 2 : 1;
       // A position passes the band test only if both differences along one axis
       // exceed the band, and one of them is to its sibling in the quad. The sum of the
       // six squared sibling differences (16 V, rounded upward monotonically) bounds
@@ -2034,7 +2041,7 @@ GridDev grid_dev(const emr_grid* g) {
 struct EvalPlan {
   int64_t n_pairs;
   int64_t n_class[kClasses];  // pairs per kernel class (schedule order)
-  int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of class 4
+  int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of class 5
   SpecLayout L;
   int32_t scratch_stride;
   size_t spec_bytes, scratch_bytes, order_bytes, total;
@@ -2137,8 +2144,29 @@ int sm_count() {
 // Waves of resident CTAs a dense launch keeps at least, when it groups tiles.
 constexpr int kDenseMinWaves = 4;
 
+// A launch that may begin while the previous kernel in the stream drains
+// (programmatic dependent launch): for tile launches of other pairs, which
+// touch none of the previous launch's outputs. *overlap: whether this launch
+// may overlap its predecessor; set for the next one.
+template <class Kern, class Arg>
+cudaError_t launch_overlapped(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool* overlap,
+                              const Arg& arg) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = *overlap ? 1 : 0;
+  *overlap = true;
+  return cudaLaunchKernelEx(&cfg, kern, arg);
+}
+
 template <int NJMAX>
-emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st) {
+emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
   if (n_ranks <= 0) return EMR_OK;
   DTileArgs A = A0;
   // consecutive tiles of a pair share a CTA (one record load and one prologue for
@@ -2151,7 +2179,9 @@ emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, 
   for (int64_t r0 = 0; r0 < n_ranks; r0 += 65535) {  // grid y: ranks, at most 65535 a launch
     A.rank_beg = rank_beg + r0;
     const dim3 grid(gx, unsigned(std::min<int64_t>(65535, n_ranks - r0)));
-    tile_kernel_dense<NJMAX, kDenseTPB><<<grid, kDenseTPB, 0, st>>>(A);
+    const cudaError_t e = launch_overlapped(tile_kernel_dense<NJMAX, kDenseTPB>, grid, dim3(kDenseTPB), 0, st,
+                                            overlap, A);
+    if (e != cudaSuccess) return cuda_status(e);
   }
   return cuda_status(cudaGetLastError());
 }
@@ -2255,18 +2285,22 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   D.bandb = bandb;
   D.tile_flags = tile_flags;
   D.n_dense = n_dense;
+  // the class launches after the first overlap their predecessor's last wave
+  bool overlap = p.n_class[0] > 0;
   int64_t beg = p.n_class[0];
-  if ((rc = launch_dense<12>(D, beg, p.n_class[1], st)) != EMR_OK) return rc;
+  if ((rc = launch_dense<12>(D, beg, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
   beg += p.n_class[1];
-  if ((rc = launch_dense<8>(D, beg, p.n_class[2], st)) != EMR_OK) return rc;
+  if ((rc = launch_dense<8>(D, beg, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
   beg += p.n_class[2];
-  if ((rc = launch_dense<4>(D, beg, p.n_class[3], st)) != EMR_OK) return rc;
+  if ((rc = launch_dense<6>(D, beg, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
   beg += p.n_class[3];
-  if (mode != kModeFused || p.n_const == 0) return launch_dense<0>(D, beg, p.n_class[4], st);
-  if ((rc = launch_dense<0>(D, beg, p.n_class[4] - p.n_const, st)) != EMR_OK) return rc;
+  if ((rc = launch_dense<4>(D, beg, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
+  beg += p.n_class[4];
+  if (mode != kModeFused || p.n_const == 0) return launch_dense<0>(D, beg, p.n_class[5], st, &overlap);
+  if ((rc = launch_dense<0>(D, beg, p.n_class[5] - p.n_const, st, &overlap)) != EMR_OK) return rc;
   // with tile flags, a constant-output pair has none set and its planes are never read: leave them
   if (tile_flags) return EMR_OK;
-  const int64_t c0 = beg + p.n_class[4] - p.n_const;
+  const int64_t c0 = beg + p.n_class[5] - p.n_const;
   for (int64_t r0 = 0; r0 < p.n_const; r0 += 65535) {  // grid y: pairs, at most 65535 a launch
     D.rank_beg = c0 + r0;
     const int64_t nc = std::min<int64_t>(65535, p.n_const - r0);

@@ -17,6 +17,14 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kBlock = 128;  // threads per evaluation tile CTA
 
+// Programmatic dependent launch: a kernel launched to overlap its predecessor
+// (launch_overlapped) runs pdl_wait() before it reads the predecessor's results,
+// which returns once the predecessor has completed and its writes are visible
+// (at once for a kernel launched the ordinary way); pdl_trigger() lets the next
+// such launch begin.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---- grid arithmetic ---------------------------------------------------------
 
 __host__ __device__ __forceinline__ uint32_t compact1by1(uint32_t x) {
@@ -210,29 +218,19 @@ struct QueryDev {
   int32_t S, per_genome;
 };
 
-// Pair schedule: by kernel class (interpreter, dense-12, dense-8, dense-4), then by
-// estimated cost, heaviest first; a counting sort in one CTA.
+// Pair schedule: by kernel class (heaviest class first), then by estimated
+// cost, heaviest first: order[rank] = pair, by a counting sort over kCostBins
+// bins of the pairs' bins (bins[r]), run by one CTA of nthreads threads (a
+// multiple of 32, at most 1024; each thread scans kCostBins / nthreads bins).
 constexpr int kClassBins = 256;
 constexpr int kCostBins = kClasses * kClassBins;
-// Pair schedule (order[rank] = pair): class-major, heaviest estimated cost first,
-// by a counting sort over kCostBins bins, run by one CTA of nthreads threads
-// (a multiple of 32, at most 1024; each thread scans kCostBins / nthreads bins).
-__device__ void schedule_block(const uint8_t* __restrict__ pack, QueryDev q, int64_t n_pairs,
-                               int32_t* __restrict__ order, int32_t* hist, int32_t* wsum) {
+__device__ void schedule_block(const int32_t* __restrict__ bins, int64_t n_pairs, int32_t* __restrict__ order,
+                               int32_t* hist, int32_t* wsum) {
   const int nthreads = blockDim.x, tid = threadIdx.x;
-  const PackHeader* h = reinterpret_cast<const PackHeader*>(pack);
-  const PackGenome* gt = reinterpret_cast<const PackGenome*>(pack + h->off_genomes);
   for (int k = tid; k < kCostBins; k += nthreads) hist[k] = 0;
   __syncthreads();
-  auto bin_of = [&](int64_t r) {
-    const int g = int(r / q.S), s = int(r % q.S);
-    if (q.per_genome && q.count && s >= q.count[g]) return kCostBins - 1;  // unused: constant 0
-    const int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
-    const int side = q.side[si] ? 1 : 0;
-    const uint32_t c = min(gt[g].cost[side], uint32_t(kClassBins - 1));
-    return pair_class(gt[g].n_varying[side], gt[g].n_joint[side]) * kClassBins + (kClassBins - 1 - int(c));
-  };
-  for (int64_t r = tid; r < n_pairs; r += nthreads) atomicAdd(&hist[bin_of(r)], 1);
+#pragma unroll 4
+  for (int64_t r = tid; r < n_pairs; r += nthreads) atomicAdd(&hist[__ldcg(bins + r)], 1);
   __syncthreads();
   // exclusive scan: thread tid owns bins [tid * per, (tid + 1) * per)
   const int per = kCostBins / nthreads, lane = tid & 31, warp = tid >> 5;
@@ -261,7 +259,8 @@ __device__ void schedule_block(const uint8_t* __restrict__ pack, QueryDev q, int
     run += v;
   }
   __syncthreads();
-  for (int64_t r = tid; r < n_pairs; r += nthreads) order[atomicAdd(&hist[bin_of(r)], 1)] = int32_t(r);
+#pragma unroll 4
+  for (int64_t r = tid; r < n_pairs; r += nthreads) order[atomicAdd(&hist[__ldcg(bins + r)], 1)] = int32_t(r);
 }
 
 // One thread per pair: fold the constant inputs (the slot's node coordinates
@@ -269,22 +268,28 @@ __device__ void schedule_block(const uint8_t* __restrict__ pack, QueryDev q, int
 // constants; list the edges between varying nodes.
 constexpr int kSpecWarps = 4;   // pairs per CTA: a warp per pair
 constexpr int kSpecSmemNodes = 128;  // genomes up to this many kept nodes keep their values in shared memory
+// genomes up to this many kept nodes and edges are staged in shared memory, and
+// their records built there before one coalesced copy out
+constexpr int kSpecStageNodes = 48, kSpecStageEdges = 96;
 
 __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __restrict__ pack, QueryDev q,
                                                                int64_t n_pairs, SpecLayout L,
                                                                uint8_t* __restrict__ spec,
                                                                float* __restrict__ scratch, int32_t scratch_stride,
-                                                               int32_t* __restrict__ order) {
+                                                               int32_t* __restrict__ order, int32_t* __restrict__ bins,
+                                                               unsigned int* __restrict__ done) {
   __shared__ float s_cval[kSpecWarps][kSpecSmemNodes];
   __shared__ int32_t s_hist[kCostBins];
   __shared__ int32_t s_wsum[32];
-  if (blockIdx.x == gridDim.x - 1) {  // the last CTA schedules the pairs while the others build records
-    schedule_block(pack, q, n_pairs, order, s_hist, s_wsum);
-    return;
-  }
+  __shared__ __align__(16) PackNode s_nd[kSpecWarps][kSpecStageNodes];
+  __shared__ __align__(16) PackEdge s_ed[kSpecWarps][kSpecStageEdges];
+  __shared__ float4 s_cf[kSpecWarps][kSpecStageNodes];
+  __shared__ uint2 s_ve[kSpecWarps][kSpecStageEdges];
+  __shared__ __align__(16) float s_W[kSpecWarps][kDenseMax * kDenseMax];
+  __shared__ int s_last;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int64_t r = int64_t(blockIdx.x) * kSpecWarps + wid;
-  if (r >= n_pairs) return;  // whole warps
+  auto pair_record = [&]() {
   const PackHeader* h = reinterpret_cast<const PackHeader*>(pack);
   const PackGenome* gt = reinterpret_cast<const PackGenome*>(pack + h->off_genomes);
   const PackNode* nt = reinterpret_cast<const PackNode*>(pack + h->off_nodes);
@@ -293,10 +298,36 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
   uint8_t* rec = spec + r * L.stride;
   int32_t* hdr = reinterpret_cast<int32_t*>(rec);
   if (q.per_genome && q.count && s >= q.count[g]) {  // unused slot: constant 0, nothing kept
-    if (lane == 0) { hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = pair_class(0, 0); }
+    if (lane == 0) {
+      hdr[0] = 0; hdr[1] = 0; hdr[2] = 0; hdr[3] = pair_class(0, 0);
+      bins[r] = kCostBins - 1;
+    }
     return;
   }
   const PackGenome G = gt[g];
+  if (lane == 0) {  // the pair's schedule bin: its class, then its cost, heaviest first
+    const int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
+    const int side = q.side[si] ? 1 : 0;
+    const int c = int(min(G.cost[side], uint32_t(kClassBins - 1)));
+    bins[r] = pair_class(G.n_varying[side], G.n_joint[side]) * kClassBins + (kClassBins - 1 - c);
+  }
+  // stage a small genome's node and edge records (coalesced, by the warp)
+  const bool staged = G.n_nodes <= kSpecStageNodes && G.n_edges <= kSpecStageEdges;
+  if (staged) {
+    const int4* ns = reinterpret_cast<const int4*>(nt + G.node_beg);
+    int4* nd_s = reinterpret_cast<int4*>(s_nd[wid]);
+    for (int k = lane; k < 2 * int(G.n_nodes); k += 32) nd_s[k] = ns[k];
+    const uint2* es = reinterpret_cast<const uint2*>(et + G.edge_beg);
+    uint2* ed_s = reinterpret_cast<uint2*>(s_ed[wid]);
+    for (int k = lane; k < int(G.n_edges); k += 32) ed_s[k] = es[k];
+    __syncwarp();
+  }
+  const PackNode* NS = staged ? s_nd[wid] : nt + G.node_beg;
+  const PackEdge* ES = staged ? s_ed[wid] : et + G.edge_beg;
+  float4* coef_g = reinterpret_cast<float4*>(rec + L.coef_off());
+  uint2* ve_g = reinterpret_cast<uint2*>(rec + L.edge_off());
+  float4* coef = staged ? s_cf[wid] : coef_g;  // records are built here (staged: copied out below)
+  uint2* ve = staged ? s_ve[wid] : ve_g;
   int nv = 0, nve = 0;
   if (lane == 0) {  // the node loop is sequential (each node folds the constants of its sources)
     int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
@@ -307,14 +338,12 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
     if (side == EMR_SIDE_OUT) { in[EMR_KIND_X1] = a; in[EMR_KIND_Y1] = b; gx = EMR_KIND_X2; gy = EMR_KIND_Y2; }
     else { in[EMR_KIND_X2] = a; in[EMR_KIND_Y2] = b; gx = EMR_KIND_X1; gy = EMR_KIND_Y1; }
     float* cval = G.n_nodes <= kSpecSmemNodes ? s_cval[wid] : scratch + r * scratch_stride;
-    float4* coef = reinterpret_cast<float4*>(rec + L.coef_off());
-    uint2* ve = reinterpret_cast<uint2*>(rec + L.edge_off());
     float out_const = 0.f;
     uint32_t xm = 0, ym = 0;
     int nj = 0;
     for (int t = 0; t < G.n_nodes; t++) {
-      const PackNode nd = nt[G.node_beg + t];
-      const PackEdge* ed = et + G.edge_beg + nd.edge_beg;
+      const PackNode nd = NS[t];
+      const PackEdge* ed = ES + nd.edge_beg;
       if (nd.vary & (1u << side)) {
         const uint32_t ax = (uint32_t(nd.axes) >> (2 * side)) & 3u;
         float c0 = nd.bias;
@@ -322,7 +351,7 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
           if (k != gx && k != gy) c0 = fmaf(nd.w_in[k], in[k], c0);
         int eb = nve;
         for (int e = 0; e < nd.edge_cnt; e++) {
-          const PackNode src = nt[G.node_beg + ed[e].src];
+          const PackNode& src = NS[ed[e].src];
           if (src.vary & (1u << side)) {
             const uint32_t sa = (uint32_t(src.axes) >> (2 * side)) & 3u;
             ve[nve++] = make_uint2(__float_as_uint(cval[ed[e].src]) | (sa << 16), __float_as_uint(ed[e].w));
@@ -357,19 +386,37 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
              (nv <= kDenseMax ? uint32_t(nj) << kHdrJointShift | xm << kHdrXShift | ym << kHdrYShift : 0u);
   }
   nv = __shfl_sync(0xffffffffu, nv, 0);
+  nve = __shfl_sync(0xffffffffu, nve, 0);
   __syncwarp();  // lane 0's coefficient and edge records are visible to the warp
-  if (nv <= kDenseMax) {  // the dense block: zeroed, then the edges added, by the warp's lanes
-    float* W = reinterpret_cast<float*>(rec + L.dense_off());
-    for (int k = lane; k < kDenseMax * kDenseMax; k += 32) W[k] = 0.f;
+  if (staged) {
+    for (int k = lane; k < nv; k += 32) coef_g[k] = coef[k];
+    for (int k = lane; k < nve; k += 32) ve_g[k] = ve[k];
+  }
+  if (nv <= kDenseMax) {  // the dense block: built in shared memory by the warp's lanes, then copied out
+    float* Ws = s_W[wid];
+    for (int k = lane; k < kDenseMax * kDenseMax; k += 32) Ws[k] = 0.f;
     __syncwarp();
-    if (lane < nv) {  // lane k fills row k (its edges in order, duplicates summed as before)
-      const float4* coef = reinterpret_cast<const float4*>(rec + L.coef_off());
-      const uint2* ve = reinterpret_cast<const uint2*>(rec + L.edge_off());
+    if (lane < nv) {  // lane k fills row k (at most one edge per source: parallel connections are merged)
       const uint32_t info = __float_as_uint(coef[lane].w);
       const int eb = int((info >> 8) & 0xfffu), ec = int(info >> 20);
-      for (int e = eb; e < eb + ec; e++) W[lane * kDenseMax + int(ve[e].x & 0xffffu)] += __uint_as_float(ve[e].y);
+      for (int e = eb; e < eb + ec; e++) Ws[lane * kDenseMax + int(ve[e].x & 0xffffu)] += __uint_as_float(ve[e].y);
     }
+    __syncwarp();
+    float4* Wg = reinterpret_cast<float4*>(rec + L.dense_off());
+    for (int k = lane; k < kDenseMax * kDenseMax / 4; k += 32) Wg[k] = reinterpret_cast<const float4*>(Ws)[k];
   }
+  };
+  if (r < n_pairs) pair_record();  // whole warps
+  // the last CTA to finish orders the pairs by their bins (no waiting: the others have
+  // published their bins before counting themselves done)
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  schedule_block(bins, n_pairs, order, s_hist, s_wsum);
+  if (threadIdx.x == 0) *done = 0u;  // ready for the next call
 }
 
 // ---- evaluation tiles ------------------------------------------------------------
@@ -468,7 +515,7 @@ __device__ __forceinline__ void eval4_interp(const float4* __restrict__ coef, co
 
 __global__ void __launch_bounds__(kBlock) tile_kernel(const TileArgs A) {
   extern __shared__ float4 smem4[];
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");  // the dense classes may follow as SMs free up
+  pdl_trigger();  // the dense classes may follow as SMs free up
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t rank = A.rank_beg + blockIdx.x / A.n_tiles;
   const int tile = A.tile_beg + int(blockIdx.x % A.n_tiles);
@@ -905,8 +952,8 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
   // this one frees. When this launch overlaps its predecessor, its last CTA first
   // waits for the predecessor to complete, so that this launch completes only after
   // it (later kernels in the stream read every launch's planes).
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) asm volatile("griddepcontrol.wait;" ::: "memory");
+  pdl_trigger();
+  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) pdl_wait();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid < QPT) {
     const int dx = int(compact1by1(uint32_t(TPB * tid))), dy = int(compact1by1(uint32_t(TPB * tid) >> 1));
@@ -1627,6 +1674,8 @@ __global__ void compact_scan_pair_kernel(const int32_t* __restrict__ bcount, int
 __global__ void compact_scan_pairs_kernel(const int64_t* __restrict__ counts, int64_t n_pairs,
                                           int64_t* __restrict__ offsets) {
   __shared__ long long sh[32];
+  pdl_wait();  // the counts
+  pdl_trigger();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
   long long carry = 0;
   for (int64_t k0 = 0; k0 < n_pairs; k0 += blockDim.x) {
@@ -1841,6 +1890,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_count_kernel(const uint
                                                                       int32_t* __restrict__ tile_base,
                                                                       int64_t* __restrict__ items,
                                                                       unsigned long long* __restrict__ n_items) {
+  pdl_wait();  // the tile launches' planes and flags
+  pdl_trigger();
   const int lane = threadIdx.x & 31;
   const int64_t r = (int64_t(blockIdx.x) * kSelectThreads + threadIdx.x) >> 5;
   if (r >= n_pairs) return;  // whole warps
@@ -1884,6 +1935,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint
                                                                       const int64_t* __restrict__ offsets,
                                                                       int64_t cap, int32_t* __restrict__ idx,
                                                                       float* __restrict__ wv) {
+  pdl_wait();  // the offsets (and, before them, the work items)
+  pdl_trigger();
   const int lane = threadIdx.x & 31;
   const int64_t n = int64_t(*n_items);
   const int64_t warps = int64_t(gridDim.x) * (kSelectThreads / 32);
@@ -1925,6 +1978,7 @@ __global__ void __launch_bounds__(kCompactBlock) select_weights_kernel(RecordSou
                                                                        int64_t n_pairs, int64_t cap,
                                                                        const int32_t* __restrict__ idx,
                                                                        float* __restrict__ wv) {
+  pdl_wait();  // the entries and their pairs
   const int64_t total = offsets[n_pairs] < cap ? offsets[n_pairs] : cap;
   for (int64_t e = int64_t(blockIdx.x) * kCompactBlock + threadIdx.x; e < total;
        e += int64_t(gridDim.x) * kCompactBlock) {
@@ -2044,7 +2098,7 @@ struct EvalPlan {
   int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of class 5
   SpecLayout L;
   int32_t scratch_stride;
-  size_t spec_bytes, scratch_bytes, order_bytes, total;
+  size_t spec_bytes, scratch_bytes, order_bytes, sched_bytes, total;
 };
 
 emr_status eval_plan(const void* pack_host, const emr_query* q, EvalPlan* p) {
@@ -2081,7 +2135,8 @@ emr_status eval_plan(const void* pack_host, const emr_query* q, EvalPlan* p) {
   p->spec_bytes = size_t(p->n_pairs) * size_t(p->L.stride);
   p->scratch_bytes = (size_t(p->n_pairs) * size_t(p->scratch_stride) * 4 + 255) & ~size_t(255);
   p->order_bytes = (size_t(p->n_pairs) * 4 + 255) & ~size_t(255);
-  p->total = ((p->spec_bytes + 255) & ~size_t(255)) + p->scratch_bytes + p->order_bytes;
+  p->sched_bytes = (size_t(p->n_pairs) * 4 + 16 + 255) & ~size_t(255);  // pair bins, then the done counter
+  p->total = ((p->spec_bytes + 255) & ~size_t(255)) + p->scratch_bytes + p->order_bytes + p->sched_bytes;
   return EMR_OK;
 }
 
@@ -2109,10 +2164,13 @@ emr_status prepare(const void* pack_dev, const emr_query* q, const EvalPlan& p, 
                    uint8_t** spec, int32_t** order) {
   float* scratch;
   ws_layout(p, ws, spec, order, &scratch);
+  int32_t* bins = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(*order) + p.order_bytes);
+  auto* done = reinterpret_cast<unsigned int*>(bins + p.n_pairs);
+  if (cudaMemsetAsync(done, 0, sizeof(unsigned int), st) != cudaSuccess) return EMR_ERR_CUDA;
   const QueryDev qd = query_dev(q);
   const uint8_t* pk = static_cast<const uint8_t*>(pack_dev);
-  spec_kernel<<<unsigned((p.n_pairs + kSpecWarps - 1) / kSpecWarps + 1), 32 * kSpecWarps, 0, st>>>(
-      pk, qd, p.n_pairs, p.L, *spec, scratch, p.scratch_stride, *order);
+  spec_kernel<<<unsigned((p.n_pairs + kSpecWarps - 1) / kSpecWarps), 32 * kSpecWarps, 0, st>>>(
+      pk, qd, p.n_pairs, p.L, *spec, scratch, p.scratch_stride, *order, bins, done);
   return cuda_status(cudaGetLastError());
 }
 
@@ -2148,9 +2206,9 @@ constexpr int kDenseMinWaves = 4;
 // (programmatic dependent launch): for tile launches of other pairs, which
 // touch none of the previous launch's outputs. *overlap: whether this launch
 // may overlap its predecessor; set for the next one.
-template <class Kern, class Arg>
-cudaError_t launch_overlapped(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool* overlap,
-                              const Arg& arg) {
+template <class... KArgs, class... Args>
+cudaError_t launch_overlapped(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              bool* overlap, Args... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -2162,7 +2220,7 @@ cudaError_t launch_overlapped(Kern kern, dim3 grid, dim3 block, size_t smem, cud
   cfg.attrs = attr;
   cfg.numAttrs = *overlap ? 1 : 0;
   *overlap = true;
-  return cudaLaunchKernelEx(&cfg, kern, arg);
+  return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
 template <int NJMAX>
@@ -2596,7 +2654,8 @@ emr_status emr_select_workspace_size(const emr_grid* grid, int32_t n_pairs, size
 static emr_status select_launch(const EvalPlan& p, const uint32_t* split, const uint32_t* band_bits,
                                 const uint8_t* tile_flags, const emr_query* q, const void* eval_ws,
                                 const emr_grid* grid, int32_t mode, int32_t types, int32_t* idx, float* w, int64_t cap,
-                                int64_t* counts, int64_t* offsets, void* ws, cudaStream_t st);
+                                int64_t* counts, int64_t* offsets, void* ws, cudaStream_t st,
+                                bool items_zeroed = false);
 
 emr_status emr_select(const uint32_t* split, const uint32_t* band_bits, const uint8_t* tile_flags,
                       const void* pack_host, const emr_query* q, const void* eval_ws, size_t eval_ws_bytes,
@@ -2660,6 +2719,8 @@ emr_status emr_discover(const void* pack_host, const void* pack_dev, const emr_q
   uint8_t* base = static_cast<uint8_t*>(ws);
   uint8_t* spec;
   int32_t* order;
+  // the selection's work-item counter, zeroed ahead so its first kernel can overlap the tile launches
+  if (cudaMemsetAsync(base + L.sel, 0, sizeof(unsigned long long), st) != cudaSuccess) return EMR_ERR_CUDA;
   if ((rc = prepare(pack_dev, q, p, ws, st, &spec, &order)) != EMR_OK) return rc;
   auto* split = reinterpret_cast<uint32_t*>(base + L.split);
   auto* bandb = reinterpret_cast<uint32_t*>(base + L.band);
@@ -2668,13 +2729,18 @@ emr_status emr_discover(const void* pack_host, const void* pack_dev, const emr_q
                          TileRange(), flags)) != EMR_OK)
     return rc;
   return select_launch(p, split, bandb, flags, q, ws, grid, mode, types, idx, w, cap, counts, offsets,
-                       base + L.sel, st);
+                       base + L.sel, st, true);
 }
 
+// Selection over the flagged tiles: count, scan, write, kept weights. Each kernel
+// overlaps its predecessor's end and waits for its results before reading them.
+// items_zeroed: the work-item counter was zeroed earlier in the stream (then the
+// count kernel may overlap the tile launches too).
 static emr_status select_launch(const EvalPlan& p, const uint32_t* split, const uint32_t* band_bits,
                                 const uint8_t* tile_flags, const emr_query* q, const void* eval_ws,
                                 const emr_grid* grid, int32_t mode, int32_t types, int32_t* idx, float* w, int64_t cap,
-                                int64_t* counts, int64_t* offsets, void* ws, cudaStream_t st) {
+                                int64_t* counts, int64_t* offsets, void* ws, cudaStream_t st,
+                                bool items_zeroed) {
   const int64_t n_dense = dense_tiles(grid->D);
   TypeFilter tf = no_type_filter();
   if (types != EMR_CONN_ALL) {
@@ -2686,23 +2752,27 @@ static emr_status select_launch(const EvalPlan& p, const uint32_t* split, const 
   auto* tile_base = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + 256);
   auto* items = reinterpret_cast<int64_t*>(static_cast<uint8_t*>(ws) + 256 +
                                            ((size_t(p.n_pairs) * size_t(n_dense) * 4 + 255) & ~size_t(255)));
-  int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-      cudaMemsetAsync(n_items, 0, sizeof(unsigned long long), st) != cudaSuccess)
+  const int sms = sm_count();
+  if (!items_zeroed && cudaMemsetAsync(n_items, 0, sizeof(unsigned long long), st) != cudaSuccess)
     return EMR_ERR_CUDA;
+  bool overlap = items_zeroed;
   const unsigned blocks = unsigned((p.n_pairs + kSelectThreads / 32 - 1) / (kSelectThreads / 32));
-  select_count_kernel<<<blocks, kSelectThreads, 0, st>>>(split, band_bits, tile_flags, n_dense, G,
-                                                         mode == EMR_GATED, tf, p.n_pairs, counts, tile_base, items,
-                                                         n_items);
-  compact_scan_pairs_kernel<<<1, 1024, 0, st>>>(counts, p.n_pairs, offsets);
-  select_write_kernel<<<unsigned(16 * sms), kSelectThreads, 0, st>>>(split, band_bits, n_dense, G,
-                                                                     mode == EMR_GATED, tf, tile_base, items,
-                                                                     n_items, offsets, cap, idx, w);
-  if (w && cap > 0)
-    select_weights_kernel<<<unsigned(8 * sms), kCompactBlock, 0, st>>>(
-        RecordSource{static_cast<const uint8_t*>(eval_ws), p.L}, G, offsets, p.n_pairs, cap, idx, w);
-  return cuda_status(cudaGetLastError());
+  cudaError_t e = launch_overlapped(select_count_kernel, dim3(blocks), dim3(kSelectThreads), 0, st, &overlap, split,
+                                    band_bits, tile_flags, n_dense, G, int(mode == EMR_GATED), tf, p.n_pairs, counts,
+                                    tile_base, items, n_items);
+  if (e == cudaSuccess)
+    e = launch_overlapped(compact_scan_pairs_kernel, dim3(1), dim3(1024), 0, st, &overlap,
+                          static_cast<const int64_t*>(counts), p.n_pairs, offsets);
+  if (e == cudaSuccess)
+    e = launch_overlapped(select_write_kernel, dim3(unsigned(16 * sms)), dim3(kSelectThreads), 0, st, &overlap, split,
+                          band_bits, n_dense, G, int(mode == EMR_GATED), tf, static_cast<const int32_t*>(tile_base),
+                          static_cast<const int64_t*>(items), static_cast<const unsigned long long*>(n_items),
+                          static_cast<const int64_t*>(offsets), cap, idx, w);
+  if (e == cudaSuccess && w && cap > 0)
+    e = launch_overlapped(select_weights_kernel, dim3(unsigned(8 * sms)), dim3(kCompactBlock), 0, st, &overlap,
+                          RecordSource{static_cast<const uint8_t*>(eval_ws), p.L}, G,
+                          static_cast<const int64_t*>(offsets), p.n_pairs, cap, static_cast<const int32_t*>(idx), w);
+  return cuda_status(e != cudaSuccess ? e : cudaGetLastError());
 }
 
 emr_status emr_compact(const uint32_t* mask, const float* out, const emr_grid* grid, int32_t n_pairs, int32_t* idx,

@@ -525,12 +525,26 @@ def main():
     # before step k's lists are read, and the reads run on a second stream while the GPU computes.
     e2e = None
     if args.e2e_steps > 0:
-        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
         pop = w.pop
-        a_h, b_h, s_h = pin(dsc.query.a), pin(dsc.query.b), pin(dsc.query.side)
-        pack_pinned = [torch.empty(len(dsc.pack) + 4096, dtype=torch.uint8).pin_memory() for _ in range(2)]
+        # one pinned input buffer per step in flight, [a | b | side | packed population], and one
+        # device copy of it: a single host-to-device copy a step of the bytes in use; the packer
+        # writes in place
+        S = dsc.query.S
+        ob = (12 * S + 255) // 256 * 256
+        in_bytes = ob + emr.pack_size(pop)
+        in_pinned = [torch.empty(in_bytes, dtype=torch.uint8).pin_memory() for _ in range(2)]
+        for buf in in_pinned:
+            q_h = buf[:12 * S].numpy()
+            q_h[:4 * S] = np.ascontiguousarray(dsc.query.a, np.float32).view(np.uint8)
+            q_h[4 * S:8 * S] = np.ascontiguousarray(dsc.query.b, np.float32).view(np.uint8)
+            q_h[8 * S:12 * S] = np.ascontiguousarray(dsc.query.side, np.int32).view(np.uint8)
+        in_dev = torch.empty(in_bytes, dtype=torch.uint8, device="cuda")
+        pack_dev = in_dev[ob:]
+        q_e2e = emr.Query(dsc.query.a, dsc.query.b, dsc.query.side, None, in_dev[:4 * S].view(torch.float32),
+                          in_dev[4 * S:8 * S].view(torch.float32), in_dev[8 * S:12 * S].view(torch.int32), None, S,
+                          False)
         dws = torch.zeros(emr.discover_workspace_size(dsc.pack, dsc.query, g), dtype=torch.uint8, device="cuda")
-        qc = dsc.query.c
+        qc = q_e2e.c
         outs = [(dsc.idx, dsc.w, dsc.counts, dsc.offsets),
                 (torch.empty_like(dsc.idx), torch.empty_like(dsc.w), torch.empty_like(dsc.counts),
                  torch.empty_like(dsc.offsets))]
@@ -559,21 +573,19 @@ def main():
             if k == n_warm:
                 t0 = time.perf_counter()
             b = k & 1
-            blob = emr.pack_population(pop)
-            buf = pack_pinned[b]
-            buf[:len(blob)].numpy()[:] = blob
+            buf = in_pinned[b]
+            # this input buffer's last user, step k - 2, has finished (its offsets were synchronised
+            # on in the previous iteration), so the packer may overwrite it
+            blob = emr.pack_population(pop, out=buf[ob:].numpy())
             if k >= 2:
                 stream.wait_event(read[b])  # step k - 2's lists have left this output set
-            dsc.pack_dev[:len(blob)].copy_(buf[:len(blob)], non_blocking=True)
-            dsc.query.a_dev.copy_(a_h, non_blocking=True)
-            dsc.query.b_dev.copy_(b_h, non_blocking=True)
-            dsc.query.side_dev.copy_(s_h, non_blocking=True)
+            h2d = ob + len(blob)
+            in_dev[:h2d].copy_(buf[:h2d], non_blocking=True)
             idx_o, w_o, cnt_o, off_o = outs[b]
-            emr.discover(blob, dsc.pack_dev, dsc.query, g, dsc.theta, dsc.band, dsc.w_min, dsc.mode, dsc.types, dws,
+            emr.discover(blob, pack_dev, q_e2e, g, dsc.theta, dsc.band, dsc.w_min, dsc.mode, dsc.types, dws,
                          idx_o, w_o, dsc.cap, cnt_o, off_o, qc=qc)
             res_off[b].copy_(off_o, non_blocking=True)
             done[b].record(stream)
-            h2d = len(blob) + 4 * (a_h.numel() + b_h.numel() + s_h.numel())
             if k >= 1:
                 d2h = read_lists(k - 1)
         d2h = read_lists(n_warm + n_steps - 1)

@@ -5,6 +5,7 @@
 #include <cmath>
 #include <condition_variable>
 #include <functional>
+#include <memory>
 #include <mutex>
 #include <cstring>
 #include <thread>
@@ -148,6 +149,22 @@ struct Scratch {
   std::vector<PackEdge> in_edges;
   std::vector<int> table;  // id - id_min -> local index (-1: none), when the ids span a small range
   int64_t id_min = 0;
+};
+
+// Packing buffers of the tasks of one call, kept across calls so that a warm
+// packer allocates nothing: scratch, the tasks' node and edge records, the
+// genome table. One caller at a time uses the shared set (never destroyed).
+struct PackBuffers {
+  static constexpr int kTasks = 16;
+  std::mutex mu;
+  Scratch scratch[kTasks];
+  std::vector<PackNode> nodes[kTasks];
+  std::vector<PackEdge> edges[kTasks];
+  std::vector<GenomeOut> gs;
+  static PackBuffers& get() {
+    static PackBuffers* b = new PackBuffers();
+    return *b;
+  }
 };
 
 int local_of(const Scratch& S, int32_t id) {
@@ -402,19 +419,30 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
     return EMR_ERR_ARG;
   const bool has_conns = conn_ptr[P] > conn_ptr[0];
   if (has_conns && (!conn_src || !conn_dst || !conn_w || !conn_enabled)) return EMR_ERR_ARG;
-  std::vector<GenomeOut> gs(P);
+  // per-task buffers kept across calls; a caller that finds them in use packs with its own
+  PackBuffers& shared = PackBuffers::get();
+  std::unique_lock<std::mutex> buf_lock(shared.mu, std::try_to_lock);
+  std::unique_ptr<PackBuffers> own;
+  if (!buf_lock.owns_lock()) own.reset(new PackBuffers());
+  PackBuffers& B = own ? *own : shared;
+  std::vector<GenomeOut>& gs = B.gs;
+  gs.resize(size_t(P));
   // Genomes are independent: pack them on several host threads, each with its
   // own scratch; the lowest failing genome index is reported.
   const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
   // a thread's share costs about as much to hand out as packing a few genomes
-  const int n_threads = std::max(1, std::min({hw, 16, P / 32}));
-  std::vector<emr_status> t_rc(n_threads, EMR_OK);
-  std::vector<int32_t> t_bad(n_threads, -1);
-  std::vector<std::vector<PackNode>> t_nodes(n_threads);
-  std::vector<std::vector<PackEdge>> t_edges(n_threads);
+  const int n_threads = std::max(1, std::min({hw, PackBuffers::kTasks, P / 32}));
+  emr_status t_rc[PackBuffers::kTasks];
+  int32_t t_bad[PackBuffers::kTasks];
+  std::vector<PackNode>* t_nodes = B.nodes;
+  std::vector<PackEdge>* t_edges = B.edges;
   auto g_lo = [&](int t) { return int(int64_t(P) * t / n_threads); };
   auto work = [&](int t) {
-    Scratch scratch;
+    Scratch& scratch = B.scratch[t];
+    t_rc[t] = EMR_OK;
+    t_bad[t] = -1;
+    t_nodes[t].clear();
+    t_edges[t].clear();
     const int64_t n_lo = node_ptr[g_lo(t)], n_hi = node_ptr[g_lo(t + 1)];
     t_nodes[t].reserve(size_t(std::max<int64_t>(0, n_hi - n_lo)));
     for (int g = g_lo(t); g < g_lo(t + 1); g++) {
@@ -459,7 +487,14 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
   *used = size_t(h.total_bytes);
   if (cap < h.total_bytes) return EMR_ERR_CAPACITY;
   auto* base = static_cast<uint8_t*>(buf);
-  std::memset(base, 0, size_t(h.total_bytes));
+  // every record is written in full below; only the alignment gaps between sections are cleared
+  auto clear = [&](uint64_t from, uint64_t to) {
+    if (to > from) std::memset(base + from, 0, size_t(to - from));
+  };
+  clear(sizeof(PackHeader), h.off_genomes);
+  clear(h.off_genomes + sizeof(PackGenome) * uint64_t(P), h.off_nodes);
+  clear(h.off_nodes + sizeof(PackNode) * uint64_t(nn), h.off_edges);
+  clear(h.off_edges + sizeof(PackEdge) * uint64_t(ne), h.total_bytes);
   auto* gt = reinterpret_cast<PackGenome*>(base + h.off_genomes);
   auto* nt = reinterpret_cast<PackNode*>(base + h.off_nodes);
   auto* et = reinterpret_cast<PackEdge*>(base + h.off_edges);

@@ -145,12 +145,25 @@ def index_to_ij(gidx: int):
 
 # ---- a2 -----------------------------------------------------------------------
 
-def pack_population(pop) -> np.ndarray:
-    """Packed blob (numpy uint8) of a workloads.Population."""
+def pack_size(pop) -> int:
+    """Upper bound of the packed blob's bytes for a workloads.Population (emr_pack_size)."""
+    n = C.c_size_t()
+    _check(lib().emr_pack_size(pop.P, _ptr(pop.node_ptr), _ptr(pop.conn_ptr), C.byref(n)), "emr_pack_size")
+    return int(n.value)
+
+
+def pack_population(pop, out=None) -> np.ndarray:
+    """Packed blob (numpy uint8) of a workloads.Population; written into `out` (a
+    contiguous uint8 array, e.g. a view of pinned memory) when given, else into a new array."""
     L = lib()
     n = C.c_size_t()
     _check(L.emr_pack_size(pop.P, _ptr(pop.node_ptr), _ptr(pop.conn_ptr), C.byref(n)), "emr_pack_size")
-    buf = np.empty(n.value + 16, np.uint8)   # the packer clears what it uses
+    if out is not None:
+        if out.dtype != np.uint8 or not out.flags.c_contiguous or len(out) < n.value:
+            raise ValueError("out: contiguous uint8 array of at least %d bytes" % n.value)
+        buf = out
+    else:
+        buf = np.empty(n.value + 16, np.uint8)   # the packer clears what it uses
     used, bad = C.c_size_t(), C.c_int32()
     st = L.emr_pack_population(pop.P, _ptr(pop.node_ptr), _ptr(pop.node_id), _ptr(pop.node_kind),
                                _ptr(pop.node_act), _ptr(pop.node_bias), _ptr(pop.conn_ptr), _ptr(pop.conn_src),

@@ -223,7 +223,7 @@ def profiled_traffic():
     """DRAM bytes per step of the dense tile kernels from the committed ncu summary, if that
     summary was taken on the current kernel source (else None)."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", "tile_kernel_dense_c2_pop100_d7.md")
+    path = os.path.join(ROOT, "profiles", "tile_kernel_dense_c2_pop300_d7.md")
     src = os.path.join(ROOT, "paper_2608_27612_gb300", "csrc", "emr_kernels.cu")
     try:
         fields = dict(l.split(":", 1) for l in open(path).read().splitlines() if l.startswith(("traffic_", "kernel_")))
@@ -509,7 +509,7 @@ def main():
     roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": peak / 1e12, "unit": "Tlane-op/s",
                 "frac": achieved / peak, "traffic": profiled_traffic() if args.pop == 1000 and args.depth == 7 else None,
                 "traffic_note": "DRAM bytes of the dense tile launches per step, from profiles/"
-                                "tile_kernel_dense_c2_pop100_d7.md (100-genome capture scaled x10); null when "
+                                "tile_kernel_dense_c2_pop300_d7.md (300-genome capture scaled by pairs, x10/3); null when "
                                 "the kernel source changed since", "kernel": "tile_kernel_dense (emr_eval_filter)",
                 "kernel_ms": tile_s * 1e3,
                 "fp32_ops_per_query": float(work[..., 0].mean()), "mufu_ops_per_query": float(work[..., 1].mean()),

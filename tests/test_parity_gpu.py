@@ -11,73 +11,11 @@ import torch
 import oracle
 from paper_2608_27612_gb300 import emr
 from paper_2608_27612_gb300 import workloads as W
-from parity_util import check_bits, check_lists, check_outputs, unpack_planes
+from parity_util import check_bits, check_lists, check_outputs, full_parity, run_gpu, run_oracle, unpack_planes
 
 pytestmark = pytest.mark.gpu
 X1, Y1, X2, Y2, BIAS, HID, OUT = range(7)
 IDN, SIG, TNH, GAU, SIN, ABS = range(6)
-
-
-def run_gpu(w, mode=emr.EMR_EAGER, unfused=True, fused=True, cap=None, lists=True):
-    dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, mode, cap=cap, materialise=unfused)
-    g = dsc.grid
-    res = {"dsc": dsc}
-    if unfused:
-        dsc.run_unfused(with_var=True)
-        torch.cuda.synchronize()
-        res["out"] = dsc.out.cpu().numpy()
-        res["halo"] = dsc.out_halo.cpu().numpy()
-        res["var"] = dsc.var_dbg.cpu().numpy()
-        res["mask_u"] = unpack_planes(dsc.mask.cpu().numpy(), g)
-        res["split_u"] = dsc.split.cpu().numpy()
-        res["band_u"] = dsc.band_bits.cpu().numpy()
-        res["lists_u"] = dsc.lists()
-    if fused:
-        dsc.mask.zero_(); dsc.split.zero_(); dsc.band_bits.zero_()
-        dsc.run_fused()
-        torch.cuda.synchronize()
-        res["mask_f"] = unpack_planes(dsc.mask.cpu().numpy(), g)
-        res["split_f"] = dsc.split.cpu().numpy()
-        res["band_f"] = dsc.band_bits.cpu().numpy()
-        res["lists_f"] = dsc.lists() if lists else None
-        if unfused and lists:
-            # the fused kernel's own sparse outputs, read by emr_compact
-            dsc.out.zero_()
-            dsc.run_fused(sparse_out=True)
-            res["lists_s"] = dsc.lists()
-    return res
-
-
-def run_oracle(w, g1=None):
-    r = oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, g1=g1)
-    return {k: v.reshape(-1, v.shape[-1]) for k, v in r.items()}
-
-
-def full_parity(w, mode=emr.EMR_EAGER, n_oracle=None):
-    gpu = run_gpu(w, mode)
-    ora = run_oracle(w, g1=n_oracle)
-    n = ora["w"].shape[0]
-    keep, unc = ("keep_eager", "unc_eager") if mode == emr.EMR_EAGER else ("keep_gated", "unc_gated")
-    rep = {}
-    rep["out"] = check_outputs(gpu["out"][:n], ora["w"], ora["w_err"])
-    rep["halo"] = check_outputs(gpu["halo"][:n], ora["w_halo"], ora["halo_err"], "halo")
-    dv = np.abs(gpu["var"][:n] - ora["var"])
-    assert np.all((dv <= ora["var_err"] + 1e-12) | ~np.isfinite(ora["var_err"]))
-    rep["mask_u"] = check_bits(gpu["mask_u"][:n], ora[keep], ora[unc], "unfused mask")
-    rep["mask_f"] = check_bits(gpu["mask_f"][:n], ora[keep], ora[unc], "fused mask")
-    # fused and unfused paths compute the same fp32 decisions
-    assert np.array_equal(gpu["split_u"], gpu["split_f"])
-    assert np.array_equal(gpu["band_u"], gpu["band_f"])
-    assert np.array_equal(gpu["mask_u"], gpu["mask_f"])
-    rep["kept"] = check_lists(gpu["lists_f"][:n], gpu["mask_f"][:n], ora["w"], ora["w_err"])
-    check_lists(gpu["lists_u"][:n], gpu["mask_u"][:n], ora["w"], ora["w_err"])
-    # weights recomputed from the records at compaction, and those the fused kernel
-    # stores itself, equal the materialised outputs bit for bit
-    for (i_u, w_u), (i_f, w_f), (i_s, w_s) in zip(gpu["lists_u"], gpu["lists_f"], gpu["lists_s"]):
-        assert np.array_equal(i_u, i_f) and np.array_equal(i_u, i_s)
-        assert np.array_equal(w_u.view(np.uint32), w_f.view(np.uint32))
-        assert np.array_equal(w_u.view(np.uint32), w_s.view(np.uint32))
-    return gpu, ora, rep
 
 
 def test_single_genome_depth4_both_modes():

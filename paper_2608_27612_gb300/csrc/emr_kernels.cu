@@ -1321,50 +1321,91 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
     }
     if (!fused) return;
     __syncthreads();
+    // Variance and band test of depths 0..d_hi, one item per quad: depths d_hi .. 3 in whole
+    // warps of 32 quads (their band words are quad-major), then depths 2, 1 and 0 packed into one
+    // warp (lanes 0-15, 16-19 and 20). The band screen of the 64 x 64 tiles applies: a quad with
+    // 16 V <= band^2 has no passing position, and the full test runs only in warps where some
+    // quad fails the screen.
+    int n_big = 0;
+    for (int e = kQuadMajorFrom; e <= d_hi; e++) n_big += 1 << (2 * e);
+    const int n_band_items = n_big + 32;
+    auto depth_of = [&](int u, int* q) {  // an item of the whole-warp depths
+      int e = d_hi;
+      while (u >= (1 << (2 * e))) { u -= 1 << (2 * e); e--; }
+      *q = u;
+      return e;
+    };
     bool any_pass = false;
-    for (int e = 0; e <= d_hi; e++) {
-      const int Te = 1 << (e + 1), nq = Te * Te / 4, pitch = Te + 2 * kPad, sb = wt_seg(e);
-      const int64_t lrow = prow + A.level_off[e];
-      for (int base = 0; base < nq; base += TPB) {
-        const int q = base + tid;
-        const bool valid = q < nq;
-        bool pass[4] = {false, false, false, false}, split = false;
-        float w[4] = {0.f, 0.f, 0.f, 0.f};
-        if (valid) {
-          const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-          const float* t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
-          w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
-          // the four children give the parent's variance (Section 3.2)
-          split = var16(w[0], w[1], w[2], w[3]) > theta16;
-          const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
-          const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
-          const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
+    for (int base = 0; base < n_band_items; base += TPB) {
+      const int u = base + tid;
+      int e = -1, q = 0;
+      if (u < n_big) {
+        e = depth_of(u, &q);
+      } else if (u < n_band_items) {
+        const int v = u - n_big;
+        e = v < 16 ? 2 : v < 20 ? 1 : v == 20 ? 0 : -1;
+        q = v < 16 ? v : v < 20 ? v - 16 : 0;
+        if (e > d_hi) e = -1;
+      }
+      bool pass[4] = {false, false, false, false}, split = false, screened_out = true;
+      float w[4] = {0.f, 0.f, 0.f, 0.f};
+      const float* t = s_wt;
+      int pitch = 0;
+      if (e >= 0) {
+        const int Te = 1 << (e + 1);
+        int sb = 0;
+        for (int k = 0; k < e; k++) sb += ((2 << k) + 2 * kPad) * ((2 << k) + 2 * kPad);
+        pitch = Te + 2 * kPad;
+        const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+        t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+        w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
+        // the four children give the parent's variance (Section 3.2)
+        const float v16 = var16(w[0], w[1], w[2], w[3]);
+        split = v16 > theta16;
+        screened_out = v16 <= band2;
+      }
+      if (__any_sync(kFull, !screened_out) && !screened_out) {
+        const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
+        const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
+        const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
 #pragma unroll
-          for (int c = 0; c < 4; c++) {
-            pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]),
-                                   band2);
-            if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
-          }
+        for (int c = 0; c < 4; c++) {
+          pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]),
+                                 band2);
+          if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
         }
-        const int q0 = base + warp * 32;
-        if (e >= 1) {
-          const unsigned bal = __ballot_sync(kFull, split);
-          if (lane == 0 && q0 < nq) split_row[A.word_off[e - 1] + q0 / 32] = bal;
+      }
+      const uint32_t bs = __ballot_sync(kFull, split);
+      const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+      const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+      any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
+      const int wbase = base + warp * 32;  // this warp's first item
+      if (wbase < n_big) {
+        int q0;
+        const int ew = depth_of(wbase, &q0);
+        if (lane == 0) split_row[A.word_off[ew - 1] + q0 / 32] = bs;
+        if (lane < 4)
+          A.bandb[band_base + A.word_off[ew] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+      } else if (wbase == n_big) {  // depths 2, 1, 0: position-major words
+        if (d_hi >= 2) {
+          if (lane == 0) split_row[A.word_off[1]] = bs & 0xffffu;
+          if (lane < 2) A.bandb[band_base + A.word_off[2] + lane] = band_word(b0, b1, b2, b3, lane);
         }
-        const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
-        const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-        any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
-        if (e >= kQuadMajorFrom) {
-          if (lane < 4 && q0 < nq)
-            A.bandb[band_base + A.word_off[e] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
-        } else if (q0 == 0 && lane * 32 < 4 * nq) {
-          A.bandb[band_base + A.word_off[e] + lane] = band_word(b0, b1, b2, b3, lane);
+        if (d_hi >= 1) {
+          if (lane == 2) split_row[A.word_off[0]] = (bs >> 16) & 0xfu;
+          if (lane == 3)
+            A.bandb[band_base + A.word_off[1]] = band_word((b0 >> 16) & 0xfu, (b1 >> 16) & 0xfu, (b2 >> 16) & 0xfu,
+                                                           (b3 >> 16) & 0xfu, 0);
         }
-        if (A.out && valid && (pass[0] | pass[1] | pass[2] | pass[3])) {
+        if (lane == 4)
+          A.bandb[band_base + A.word_off[0]] = band_word((b0 >> 20) & 1u, (b1 >> 20) & 1u, (b2 >> 20) & 1u,
+                                                         (b3 >> 20) & 1u, 0);
+      }
+      if (A.out && e >= 0 && (pass[0] | pass[1] | pass[2] | pass[3])) {
+        const int64_t lrow = prow + A.level_off[e];
 #pragma unroll
-          for (int c = 0; c < 4; c++)
-            if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
-        }
+        for (int c = 0; c < 4; c++)
+          if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
       }
     }
     if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense] = 1;
@@ -2200,7 +2241,7 @@ int sm_count() {
 }
 
 // Waves of resident CTAs a dense launch keeps at least, when it groups tiles.
-constexpr int kDenseMinWaves = 4;
+constexpr int kDenseMinWaves = 2;
 
 // A launch that may begin while the previous kernel in the stream drains
 // (programmatic dependent launch): for tile launches of other pairs, which

@@ -175,24 +175,39 @@ __device__ __forceinline__ uint32_t band_word(uint32_t b0, uint32_t b1, uint32_t
 //            sy = wy * y and the edges from y-only sources,
 //            a = sx + sy, then the edges from joint sources;
 // each edge adds fma(w, v_source, a); the node's value is act(a).
+// Pairs with at most kDenseMax varying nodes also get, for the tile kernels'
+// node tables, a table program per grid axis, the joint-node block and the
+// joint nodes' activations (the dense block, at dense_off()):
+//   program of axis a: kDenseMax float4 entries {c0, c, info, 0}, in slot order,
+//     one per node with a row on that axis (info: row | kEntMul | kEntJoint |
+//     act << 7 | first source << 10 | source count << 18), and kEntSrcCap
+//     float2 sources {row of the source (int bits), weight}, in slot order;
+//     rows of axis a: the joint nodes first (row m: the axis-a part of joint node
+//     m's input), then the nodes of coordinate a alone (their values);
+//   joint block: kDenseMax x kDenseMax floats, row-major, entry (m, m2) the
+//     weight of the edge from joint node m2 to joint node m (m2 < m), else 0;
+//   joint activations: kDenseMax int32.
+constexpr int kDenseMax = 12;
+constexpr uint32_t kEntMul = 1u << 5, kEntJoint = 1u << 6;
+constexpr int kEntSrcCap = kDenseMax * (kDenseMax - 1) / 2;
 struct SpecLayout {
   int64_t stride;
   int32_t nv_cap, nve_cap;
   __host__ __device__ int64_t coef_off() const { return 16; }
   __host__ __device__ int64_t edge_off() const { return 16 + 16 * int64_t(nv_cap); }
   __host__ __device__ int64_t dense_off() const { return (edge_off() + 8 * int64_t(nve_cap) + 15) & ~int64_t(15); }
+  __host__ __device__ int64_t ent_off() const { return dense_off(); }
+  __host__ __device__ int64_t esrc_off() const { return ent_off() + 2 * 16 * kDenseMax; }
+  __host__ __device__ int64_t wj_off() const { return esrc_off() + 2 * 8 * kEntSrcCap; }
+  __host__ __device__ int64_t jact_off() const { return wj_off() + 4 * kDenseMax * kDenseMax; }
+  __host__ __device__ int64_t end_off() const { return jact_off() + 4 * kDenseMax; }
 };
-
-// Pairs with at most kDenseMax varying nodes also get a dense lower-triangular
-// weight block W[k][j] (row-major, kDenseMax x kDenseMax floats): the weight of
-// the edge from varying slot j to varying slot k, 0 where there is none.
-constexpr int kDenseMax = 12;
 
 inline SpecLayout spec_layout(int nv_cap, int nve_cap) {
   SpecLayout L;
   L.nv_cap = std::max(nv_cap, 1);
   L.nve_cap = std::max(nve_cap, 1);
-  L.stride = (L.dense_off() + 4 * kDenseMax * kDenseMax + 15) & ~int64_t(15);
+  L.stride = (L.end_off() + 15) & ~int64_t(15);
   return L;
 }
 
@@ -329,6 +344,7 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
   float4* coef = staged ? s_cf[wid] : coef_g;  // records are built here (staged: copied out below)
   uint2* ve = staged ? s_ve[wid] : ve_g;
   int nv = 0, nve = 0;
+  int32_t hdr3 = 0;
   if (lane == 0) {  // the node loop is sequential (each node folds the constants of its sources)
     int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
     const int side = q.side[si] ? 1 : 0;
@@ -382,11 +398,13 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
     hdr[0] = nv;
     hdr[1] = nve;
     reinterpret_cast<float*>(hdr)[2] = out_const;
-    hdr[3] = pair_class(nv, nj) |
-             (nv <= kDenseMax ? uint32_t(nj) << kHdrJointShift | xm << kHdrXShift | ym << kHdrYShift : 0u);
+    hdr3 = int32_t(pair_class(nv, nj) |
+                   (nv <= kDenseMax ? uint32_t(nj) << kHdrJointShift | xm << kHdrXShift | ym << kHdrYShift : 0u));
+    hdr[3] = hdr3;
   }
   nv = __shfl_sync(0xffffffffu, nv, 0);
   nve = __shfl_sync(0xffffffffu, nve, 0);
+  const uint32_t h3 = __shfl_sync(0xffffffffu, uint32_t(hdr3), 0);
   __syncwarp();  // lane 0's coefficient and edge records are visible to the warp
   if (staged) {
     for (int k = lane; k < nv; k += 32) coef_g[k] = coef[k];
@@ -402,8 +420,55 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
       for (int e = eb; e < eb + ec; e++) Ws[lane * kDenseMax + int(ve[e].x & 0xffffu)] += __uint_as_float(ve[e].y);
     }
     __syncwarp();
-    float4* Wg = reinterpret_cast<float4*>(rec + L.dense_off());
-    for (int k = lane; k < kDenseMax * kDenseMax / 4; k += 32) Wg[k] = reinterpret_cast<const float4*>(Ws)[k];
+    // the tile kernels' table programs (lane k: slot k), joint block and joint activations
+    const int nj = int((h3 >> kHdrJointShift) & 0xfu);
+    const uint32_t xm = (h3 >> kHdrXShift) & 0xfffu, ym = (h3 >> kHdrYShift) & 0xfffu;
+    const uint32_t jm = ((1u << nv) - 1u) & ~(xm | ym);
+    float4* ent_g = reinterpret_cast<float4*>(rec + L.ent_off());
+    float2* esrc_g = reinterpret_cast<float2*>(rec + L.esrc_off());
+    for (int a = 0; a < 2; a++) {
+      const int k = lane;
+      const uint32_t om = a ? ym : xm, bit = 1u << k, below = bit - 1u;
+      const bool on = k < nv && ((om | jm) & bit) != 0u;
+      const bool joint = (jm & bit) != 0u;
+      uint32_t sm = 0;  // sources: earlier nodes of this coordinate alone with an edge into k
+      if (on)
+        for (uint32_t b = om & below; b; b &= b - 1u)
+          if (Ws[k * kDenseMax + __ffs(b) - 1] != 0.f) sm |= b & (0u - b);
+      const int cnt = __popc(sm);
+      int beg = cnt;  // exclusive prefix over the lanes
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(kFull, beg, o);
+        if (lane >= o) beg += y;
+      }
+      beg -= cnt;
+      if (on) {
+        const float4 cf = coef[k];
+        const int row = joint ? __popc(jm & below) : nj + __popc(om & below);
+        const uint32_t info = uint32_t(row) | (joint && a ? kEntMul : 0u) | (joint ? kEntJoint : 0u) |
+                              ((__float_as_uint(cf.w) & 7u) << 7) | (uint32_t(beg) << 10) | (uint32_t(cnt) << 18);
+        ent_g[a * kDenseMax + __popc((om | jm) & below)] = make_float4(cf.x, a ? cf.z : cf.y, __uint_as_float(info), 0.f);
+        int q = beg;
+        for (uint32_t b = sm; b; b &= b - 1u) {
+          const int j = __ffs(b) - 1;
+          esrc_g[a * kEntSrcCap + q++] =
+              make_float2(__int_as_float(nj + __popc(om & ((1u << j) - 1u))), Ws[k * kDenseMax + j]);
+        }
+      }
+    }
+    auto slot_of = [&](int m) {  // joint node m is the m-th set bit of jm
+      uint32_t b = jm;
+      for (int q = 0; q < m; q++) b &= b - 1u;
+      return b ? __ffs(b) - 1 : 0;
+    };
+    float* wj_g = reinterpret_cast<float*>(rec + L.wj_off());
+    for (int t = lane; t < kDenseMax * kDenseMax; t += 32) {
+      const int m = t / kDenseMax, m2 = t % kDenseMax;
+      wj_g[t] = m < nj && m2 < m ? Ws[slot_of(m) * kDenseMax + slot_of(m2)] : 0.f;
+    }
+    if (lane < kDenseMax)
+      reinterpret_cast<int32_t*>(rec + L.jact_off())[lane] =
+          lane < nj ? int32_t(__float_as_uint(coef[slot_of(lane)].w) & 0xfu) : 0;
   }
   };
   if (r < n_pairs) pair_record();  // whole warps
@@ -729,13 +794,9 @@ constexpr int kTabFull = kTileSide + 4;
 __host__ __device__ constexpr int tab_seg(int d) { return (2 << d) - 2 + 4 * d; }
 constexpr int kTabPyr = tab_seg(kPyramidTop + 1);
 
-// Table program of one axis, built once per CTA: an entry per node with a row
-// on that axis, in slot order: {c0, c, info} with info = row | kEntMul (the
-// input starts as c * coordinate, the y part of a joint node) | kEntJoint (the
-// row holds the input, no activation) | act << 7 | first source << 10 |
-// source count << 18; sources {row of the source, weight}, in slot order.
-constexpr uint32_t kEntMul = 1u << 5, kEntJoint = 1u << 6;
-constexpr int kEntSrcCap = kDenseMax * (kDenseMax - 1) / 2;
+// Table program of one axis (built per pair by spec_kernel, see the record
+// layout): kEntMul: the input starts as c * coordinate (the y part of a joint
+// node); kEntJoint: the row holds the input, no activation.
 
 // One table column: every entry of the axis at coordinate value cv (the common
 // order of the record layout; a node of one coordinate has sources of that
@@ -939,8 +1000,6 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
   constexpr int QPT = kTileSide * kTileSide / 4 / TPB;  // quads per thread in a 64 x 64 tile
   constexpr int P64 = kTileSide + 2 * kPad;
   constexpr int NJ1 = NJMAX > 0 ? NJMAX : 1;
-  __shared__ float4 s_coef[kDenseMax];
-  __shared__ __align__(16) float s_W[kDenseMax * kDenseMax];
   __shared__ __align__(16) float s_WJ[NJ1 * NJ1];
   __shared__ int s_jact[NJ1];
   __shared__ float4 s_ent[2][kDenseMax];  // table programs of the two axes
@@ -978,57 +1037,19 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
     for (int t = t_beg; t < t_end; t++) zero_tile(A, r, t, tid, TPB);
     return;
   }
-  {
-    const float4* gc = reinterpret_cast<const float4*>(rec + A.L.coef_off());
-    const float* gW = reinterpret_cast<const float*>(rec + A.L.dense_off());
-    if (tid < kDenseMax) s_coef[tid] = tid < nv ? gc[tid] : make_float4(0, 0, 0, 0);
-    for (int k = tid; k < kDenseMax * kDenseMax; k += TPB) s_W[k] = gW[k];
+  {  // the pair's table programs, joint block and joint activations (built by spec_kernel)
+    const float4* gent = reinterpret_cast<const float4*>(rec + A.L.ent_off());
+    const float2* gsrc = reinterpret_cast<const float2*>(rec + A.L.esrc_off());
+    for (int k = tid; k < 2 * kDenseMax; k += TPB) s_ent[k / kDenseMax][k % kDenseMax] = gent[k];
+    for (int k = tid; k < 2 * kEntSrcCap; k += TPB) s_esrc[k / kEntSrcCap][k % kEntSrcCap] = gsrc[k];
+    if constexpr (NJMAX > 0) {
+      const float* gwj = reinterpret_cast<const float*>(rec + A.L.wj_off());
+      for (int t = tid; t < NJMAX * NJMAX; t += TPB) s_WJ[t] = gwj[(t / NJMAX) * kDenseMax + t % NJMAX];
+      if (tid < NJMAX) s_jact[tid] = reinterpret_cast<const int32_t*>(rec + A.L.jact_off())[tid];
+    }
   }
-  __syncthreads();
-  // table programs: warp a builds axis a (lane k: slot k); read after the first tile's barrier
   const bool ax_x = (xm | jm) != 0u, ax_y = (ym | jm) != 0u;
-  if (warp < 2) {
-    const int a = warp, k = lane;
-    const uint32_t om = a ? ym : xm, bit = 1u << k, below = bit - 1u;
-    const bool on = k < nv && ((om | jm) & bit) != 0u;
-    const bool joint = (jm & bit) != 0u;
-    uint32_t sm = 0;  // sources: earlier nodes of this coordinate alone with an edge into k
-    if (on)
-      for (uint32_t b = om & below; b; b &= b - 1u)
-        if (s_W[k * kDenseMax + __ffs(b) - 1] != 0.f) sm |= b & (0u - b);
-    const int cnt = __popc(sm);
-    int beg = cnt;  // exclusive prefix over the lanes
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(kFull, beg, o);
-      if (lane >= o) beg += y;
-    }
-    beg -= cnt;
-    if (on) {
-      const float4 cf = s_coef[k];
-      const int row = joint ? __popc(jm & below) : nj + __popc(om & below);
-      const uint32_t info = uint32_t(row) | (joint && a ? kEntMul : 0u) | (joint ? kEntJoint : 0u) |
-                            ((__float_as_uint(cf.w) & 7u) << 7) | (uint32_t(beg) << 10) | (uint32_t(cnt) << 18);
-      s_ent[a][__popc((om | jm) & below)] = make_float4(cf.x, a ? cf.z : cf.y, __uint_as_float(info), 0.f);
-      int q = beg;
-      for (uint32_t b = sm; b; b &= b - 1u) {
-        const int j = __ffs(b) - 1;
-        s_esrc[a][q++] = make_float2(__int_as_float(nj + __popc(om & ((1u << j) - 1u))), s_W[k * kDenseMax + j]);
-      }
-    }
-  }
   const int n_ent_x = __popc((xm | jm) & ((1u << nv) - 1u)), n_ent_y = __popc((ym | jm) & ((1u << nv) - 1u));
-  if constexpr (NJMAX > 0) {  // joint node m is the m-th set bit of jm
-    auto slot_of = [&](int m) {
-      uint32_t b = jm;
-      for (int q = 0; q < m; q++) b &= b - 1u;
-      return b ? __ffs(b) - 1 : 0;
-    };
-    if (tid < NJMAX) s_jact[tid] = int(__float_as_uint(s_coef[slot_of(tid)].w) & 0xfu);
-    for (int t = tid; t < NJMAX * NJMAX; t += TPB) {
-      const int m = t / NJMAX, m2 = t % NJMAX;
-      s_WJ[t] = m < nj && m2 < m ? s_W[slot_of(m) * kDenseMax + slot_of(m2)] : 0.f;
-    }
-  }
   __syncthreads();
   uint32_t* split_row = A.split + int64_t(r) * A.n_words;
   const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;

@@ -965,7 +965,9 @@ constexpr int kPad = 2;
 constexpr int kWtFull = (kTileSide + 2 * kPad) * (kTileSide + 2 * kPad);
 // The pyramid tile's padded grids of depths 0..4, one after the other; its node
 // tables follow them in the same buffer.
-__host__ __device__ constexpr int wt_seg(int d) { return d == 0 ? 0 : wt_seg(d - 1) + ((2 << (d - 1)) + 2 * kPad) * ((2 << (d - 1)) + 2 * kPad); }
+// sum over e < d of (2^(e+1) + 4)^2 = (4^(d+1) - 4) / 3 + 16 (2^d - 1) + 16 d (kPad = 2)
+static_assert(kPad == 2, "wt_seg's closed form");
+__host__ __device__ constexpr int wt_seg(int d) { return ((4 << (2 * d)) - 4) / 3 + 16 * ((1 << d) - 1) + 16 * d; }
 constexpr int kWtPyr = wt_seg(kPyramidTop + 1);
 constexpr int kTileBuf = kWtFull + 2 * kDenseMax * kTabFull;
 static_assert(kWtPyr % 4 == 0 && kWtPyr + 2 * kDenseMax * kTabPyr <= kTileBuf, "pyramid tables fit the tile buffer");
@@ -1374,8 +1376,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
       int pitch = 0;
       if (e >= 0) {
         const int Te = 1 << (e + 1);
-        int sb = 0;
-        for (int k = 0; k < e; k++) sb += ((2 << k) + 2 * kPad) * ((2 << k) + 2 * kPad);
+        const int sb = wt_seg(e);
         pitch = Te + 2 * kPad;
         const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
         t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
@@ -1435,6 +1436,87 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
   for (int t = t_beg; t < t_end; t++) {
     if (t > t_beg) __syncthreads();  // the previous tile's reads of the shared buffer are done
     run_tile(t);
+  }
+}
+
+// The 64 x 64 tiles of pairs whose output depends on one coordinate (no joint
+// node; fused mode, no output buffer): a warp per tile, four tiles at a time per
+// CTA, no block barrier. The warp evaluates the output's axis table at the
+// tile's 64 coordinates (two per lane), then filters per column (row) pair as
+// in tile_kernel_dense; the two ring coordinates are evaluated only where an
+// edge column's band test can pass (its pair's squared difference exceeds
+// band^2: otherwise the smaller difference cannot).
+constexpr int kOneAxisWarps = 4;
+constexpr int kOneAxisBlocks = 12;  // CTAs per SM the kernel is compiled for
+__global__ void __launch_bounds__(32 * kOneAxisWarps, kOneAxisBlocks) tile_kernel_one_axis(const DTileArgs A) {
+  __shared__ float4 s_ent[kDenseMax];
+  __shared__ float2 s_esrc[kEntSrcCap];
+  __shared__ __align__(16) float s_tab[kOneAxisWarps][kDenseMax * kTabFull];
+  pdl_trigger();
+  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) pdl_wait();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int r = A.order[A.rank_beg + blockIdx.y];
+  const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
+  const int nv = reinterpret_cast<const int32_t*>(rec)[0];
+  const uint32_t h3 = reinterpret_cast<const uint32_t*>(rec)[3];
+  const uint32_t xm = (h3 >> kHdrXShift) & 0xfffu, ym = (h3 >> kHdrYShift) & 0xfffu;
+  const bool out_x = nv > 0 && ((xm >> (nv - 1)) & 1u) != 0u;
+  const int a = out_x ? 0 : 1;
+  const uint32_t om = out_x ? xm : ym;
+  const int n_ent = __popc(om & ((1u << nv) - 1u)), orow = __popc(om) - 1;
+  {
+    const float4* gent = reinterpret_cast<const float4*>(rec + A.L.ent_off()) + a * kDenseMax;
+    const float2* gsrc = reinterpret_cast<const float2*>(rec + A.L.esrc_off()) + a * kEntSrcCap;
+    if (tid < kDenseMax) s_ent[tid] = gent[tid];
+    for (int k = tid; k < kEntSrcCap; k += 32 * kOneAxisWarps) s_esrc[k] = gsrc[k];
+  }
+  __syncthreads();
+  if (nv == 0) return;  // (constant pairs are not launched here)
+  uint32_t* split_row = A.split + int64_t(r) * A.n_words;
+  const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;
+  const bool wfilter = A.w_min > 0.f;
+  const float theta16 = 16.f * A.theta, band2 = A.band * A.band;
+  float* tab = s_tab[warp];
+  const float* f = tab + orow * kTabFull;  // coordinate i at i + 2
+  const int t_beg = A.tile_beg + int(blockIdx.x) * A.tiles_per_cta;
+  const int t_end = min(t_beg + A.tiles_per_cta, A.tile_beg + A.n_tiles);
+  for (int tile = t_beg + warp; tile < t_end; tile += kOneAxisWarps) {
+    int u = tile - 1, d = kPyramidTop + 1;
+    while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
+    const uint32_t mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
+    const int c0 = int(compact1by1(out_x ? mb : mb >> 1));  // first column (row) of the tile
+    const float scale = __int_as_float((127 - (d + 1)) << 23);
+    __syncwarp();  // the previous tile's reads of this warp's table are done
+    table_column(grid_coord(c0 + lane, scale), lane + 2, n_ent, s_ent, s_esrc, tab, kTabFull);
+    table_column(grid_coord(c0 + lane + 32, scale), lane + 34, n_ent, s_ent, s_esrc, tab, kTabFull);
+    __syncwarp();
+    const float f0 = f[2 * lane + 2], f1 = f[2 * lane + 3];
+    const float s01 = sqdiff(f0, f1);
+    const bool ring_l = __shfl_sync(kFull, s01 > band2, 0), ring_r = __shfl_sync(kFull, s01 > band2, 31);
+    if (ring_l || ring_r) {
+      if (lane == 0 && ring_l) table_column(grid_coord(c0 - 1, scale), 1, n_ent, s_ent, s_esrc, tab, kTabFull);
+      if (lane == 1 && ring_r) table_column(grid_coord(c0 + 64, scale), 66, n_ent, s_ent, s_esrc, tab, kTabFull);
+      __syncwarp();
+    }
+    // (an edge neighbour not evaluated is only read where the pair's own difference decides)
+    const float fl = f[2 * lane + 1], fr = f[2 * lane + 4];
+    bool g0 = fminf(sqdiff(f0, fl), s01) > band2, g1 = fminf(s01, sqdiff(f1, fr)) > band2;
+    if (wfilter) {
+      g0 = g0 && fabsf(f0) > A.w_min;
+      g1 = g1 && fabsf(f1) > A.w_min;
+    }
+    const uint32_t S = __ballot_sync(kFull, 4.f * s01 > theta16);
+    const uint32_t G0 = __ballot_sync(kFull, g0), G1 = __ballot_sync(kFull, g1);
+    uint32_t* band_t = A.bandb + (band_base + A.word_off[d] + mb / 32);
+#pragma unroll
+    for (int k = 0; k < 4; k++) {  // band word 4 j + c: child c of the quads of split word j
+      const uint32_t wi = uint32_t(4 * lane + k), j = wi >> 2, c = wi & 3u;
+      const uint32_t gsel = (out_x ? (c & 1u) : (c >> 1)) ? G1 : G0;
+      band_t[wi] = out_x ? word_of_columns(gsel, j) : word_of_rows(gsel, j);
+    }
+    split_row[A.word_off[d - 1] + mb / 128 + lane] =
+        out_x ? word_of_columns(S, uint32_t(lane)) : word_of_rows(S, uint32_t(lane));
+    if (A.tile_flags && lane == 0 && (G0 | G1) != 0u) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
   }
 }
 
@@ -2306,6 +2388,23 @@ emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, 
   return cuda_status(cudaGetLastError());
 }
 
+emr_status launch_one_axis(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
+  if (n_ranks <= 0 || A0.n_tiles <= 0) return EMR_OK;
+  DTileArgs A = A0;
+  const int64_t slots = int64_t(sm_count()) * kOneAxisBlocks;
+  int g = 32;  // tiles per CTA, a warp taking every kOneAxisWarps-th
+  while (g > kOneAxisWarps && n_ranks * ((A.n_tiles + g - 1) / g) < kDenseMinWaves * slots) g >>= 1;
+  A.tiles_per_cta = g;
+  const unsigned gx = unsigned((A.n_tiles + g - 1) / g);
+  for (int64_t r0 = 0; r0 < n_ranks; r0 += 65535) {
+    A.rank_beg = rank_beg + r0;
+    const dim3 grid(gx, unsigned(std::min<int64_t>(65535, n_ranks - r0)));
+    const cudaError_t e = launch_overlapped(tile_kernel_one_axis, grid, dim3(32 * kOneAxisWarps), 0, st, overlap, A);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  return cuda_status(cudaGetLastError());
+}
+
 // Tile range (dense numbering: tile 0 = depths 0..4, then the 64 x 64 tiles of
 // depths 5..D in global-index order) and output views of one launch set.
 struct TileRange {
@@ -2416,8 +2515,28 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   beg += p.n_class[3];
   if ((rc = launch_dense<4>(D, beg, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
   beg += p.n_class[4];
-  if (mode != kModeFused || p.n_const == 0) return launch_dense<0>(D, beg, p.n_class[5], st, &overlap);
-  if ((rc = launch_dense<0>(D, beg, p.n_class[5] - p.n_const, st, &overlap)) != EMR_OK) return rc;
+  if (mode == kModeFused && !out && p.n_class[5] > p.n_const) {
+    // one-coordinate outputs: the depths 0..4 tile through the generic kernel, the 64 x 64
+    // tiles a warp each
+    const int64_t n5 = p.n_class[5] - p.n_const;
+    if (tr.beg == 0) {
+      DTileArgs D0 = D;
+      D0.n_tiles = 1;
+      if ((rc = launch_dense<0>(D0, beg, n5, st, &overlap)) != EMR_OK) return rc;
+    }
+    const int32_t t1 = std::max<int32_t>(tr.beg, 1);
+    if (t1 < tr.end) {
+      DTileArgs D1 = D;
+      D1.tile_beg = t1;
+      D1.n_tiles = tr.end - t1;
+      if ((rc = launch_one_axis(D1, beg, n5, st, &overlap)) != EMR_OK) return rc;
+    }
+  } else if (mode != kModeFused || p.n_const == 0) {
+    return launch_dense<0>(D, beg, p.n_class[5], st, &overlap);
+  } else if ((rc = launch_dense<0>(D, beg, p.n_class[5] - p.n_const, st, &overlap)) != EMR_OK) {
+    return rc;
+  }
+  if (mode != kModeFused) return EMR_OK;
   // with tile flags, a constant-output pair has none set and its planes are never read: leave them
   if (tile_flags) return EMR_OK;
   const int64_t c0 = beg + p.n_class[5] - p.n_const;

@@ -376,10 +376,11 @@ def variants_run(emr, torch, W, D=7, P=1000, reps=10):
 
 
 def launches_in_step(emr, dsc):
-    """Kernel launches of one step: prepare (records, with the schedule in one CTA), one tile launch per
-    non-empty kernel class (constant-output pairs need none: their tiles hold no band
-    bit), selection (count, scan, write, kept weights); the tile flags' memset is not a
-    kernel."""
+    """Kernel launches of one step: prepare (records, with the schedule in the last CTA); per
+    non-empty dense kernel class two tile launches (depths 0..5 on the block kernel, the
+    deeper 64 x 64 tiles a warp each), one for the interpreter class (constant-output
+    pairs need none: their tiles hold no band bit); selection (count, scan, write, kept
+    weights). Memsets are not kernels."""
     _, gs, _, _ = emr.pack_records(dsc.pack)
     side = np.asarray(dsc.query.side)
     def per_pair(field):
@@ -388,7 +389,9 @@ def launches_in_step(emr, dsc):
         return f.astype(np.int64)
     nv, nj = per_pair("n_varying"), per_pair("n_joint")
     cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 6, 2, np.where(nj > 4, 3, np.where(nj > 0, 4, 5)))))
-    return 1 + len(np.unique(cls[nv > 0])) + 4
+    present = np.unique(cls[nv > 0])
+    per_class = [1 if c == 0 else (2 if dsc.grid.D >= 6 else 1) for c in present]
+    return 1 + sum(per_class) + 4
 
 
 def oracle_baseline(w, genomes):

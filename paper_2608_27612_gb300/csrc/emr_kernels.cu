@@ -798,22 +798,38 @@ constexpr int kTabPyr = tab_seg(kPyramidTop + 1);
 // layout): kEntMul: the input starts as c * coordinate (the y part of a joint
 // node); kEntJoint: the row holds the input, no activation.
 
-// One table column: every entry of the axis at coordinate value cv (the common
-// order of the record layout; a node of one coordinate has sources of that
-// coordinate only).
-__device__ __forceinline__ void table_column(float cv, int pos, int n_ent, const float4* __restrict__ ent,
-                                             const float2* __restrict__ src, float* __restrict__ tab, int tw) {
+// Table columns: every entry of the axis at the NC coordinate values cv,
+// columns pos (the common order of the record layout; a node of one coordinate
+// has sources of that coordinate only).
+template <int NC>
+__device__ __forceinline__ void table_columns(const float (&cv)[NC], const int (&pos)[NC], int n_ent,
+                                              const float4* __restrict__ ent, const float2* __restrict__ src,
+                                              float* __restrict__ tab, int tw) {
   for (int e = 0; e < n_ent; e++) {
     const float4 E = ent[e];
     const uint32_t info = __float_as_uint(E.z);
-    float z = (info & kEntMul) ? __fmul_rn(E.y, cv) : fmaf(E.y, cv, E.x);
+    float z[NC];
+#pragma unroll
+    for (int c = 0; c < NC; c++) z[c] = (info & kEntMul) ? __fmul_rn(E.y, cv[c]) : fmaf(E.y, cv[c], E.x);
     const int sb = int((info >> 10) & 0xffu), se = sb + int(info >> 18);
     for (int k = sb; k < se; k++) {
       const float2 S = src[k];
-      z = fmaf(S.y, tab[__float_as_int(S.x) * tw + pos], z);
+      const float* col = tab + __float_as_int(S.x) * tw;
+#pragma unroll
+      for (int c = 0; c < NC; c++) z[c] = fmaf(S.y, col[pos[c]], z[c]);
     }
-    tab[int(info & 31u) * tw + pos] = (info & kEntJoint) ? z : act_apply(int((info >> 7) & 7u), z);
+    if (!(info & kEntJoint)) act_applyN<NC>(int((info >> 7) & 7u), z);
+    float* out = tab + int(info & 31u) * tw;
+#pragma unroll
+    for (int c = 0; c < NC; c++) out[pos[c]] = z[c];
   }
+}
+// (NC = 1: one column.)
+__device__ __forceinline__ void table_column(float cv, int pos, int n_ent, const float4* __restrict__ ent,
+                                             const float2* __restrict__ src, float* __restrict__ tab, int tw) {
+  const float c1[1] = {cv};
+  const int p1[1] = {pos};
+  table_columns<1>(c1, p1, n_ent, ent, src, tab, tw);
 }
 
 // The joint nodes of a pair at NP points: init(m, z) gives joint node m's x
@@ -1517,6 +1533,152 @@ __global__ void __launch_bounds__(32 * kOneAxisWarps, kOneAxisBlocks) tile_kerne
     split_row[A.word_off[d - 1] + mb / 128 + lane] =
         out_x ? word_of_columns(S, uint32_t(lane)) : word_of_rows(S, uint32_t(lane));
     if (A.tile_flags && lane == 0 && (G0 | G1) != 0u) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
+  }
+}
+
+// The 64 x 64 tiles of pairs with joint nodes (fused mode, no output buffer): a
+// warp per tile, kWarpTiles tiles at a time per CTA, no block barrier. The warp
+// fills its own node tables (the tile's 64 + 64 coordinates, two per lane and
+// axis), then each lane evaluates 32 sibling quads (quad l + 32 k: the lanes'
+// ballot for k is split word k of the tile) two per pass (one above 6 joint
+// nodes). A tile whose band screen fires (rare) evaluates its ring coordinates
+// and runs the band test with each quad's eight outer neighbours evaluated
+// directly; every other tile stores zero band words.
+constexpr int kWarpTiles = 4;
+constexpr int warp_min_blocks(int njmax) { return njmax <= 4 ? 7 : njmax <= 8 ? 6 : 4; }
+
+// Column (row) offset of quad 32 k of a 64 x 64 tile, in positions: Morton bits
+// 6, 8 of the quad index are x bits 3, 4 (bits 5, 7, 9: y bits 2, 3, 4).
+__device__ __forceinline__ int warp_quad_dx(int k) { return 2 * (8 * ((k >> 1) & 1) + 16 * ((k >> 3) & 1)); }
+__device__ __forceinline__ int warp_quad_dy(int k) { return 2 * (4 * (k & 1) + 8 * ((k >> 2) & 1) + 16 * ((k >> 4) & 1)); }
+
+template <int NJMAX>
+__global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_kernel_warp(const DTileArgs A) {
+  static_assert(NJMAX >= 1 && NJMAX <= kDenseMax, "pairs with joint nodes");
+  constexpr int QPE = NJMAX <= 6 ? 2 : 1;
+  __shared__ __align__(16) float s_WJ[NJMAX * NJMAX];
+  __shared__ int s_jact[NJMAX];
+  __shared__ float4 s_ent[2][kDenseMax];
+  __shared__ float2 s_esrc[2][kEntSrcCap];
+  __shared__ __align__(16) float s_tab[kWarpTiles][2 * kDenseMax * kTabFull];
+  pdl_trigger();
+  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) pdl_wait();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int r = A.order[A.rank_beg + blockIdx.y];
+  const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
+  const int nv = reinterpret_cast<const int32_t*>(rec)[0];
+  const uint32_t h3 = reinterpret_cast<const uint32_t*>(rec)[3];
+  const int nj = int((h3 >> kHdrJointShift) & 0xfu);
+  const uint32_t xm = (h3 >> kHdrXShift) & 0xfffu, ym = (h3 >> kHdrYShift) & 0xfffu;
+  const uint32_t jm = ((1u << nv) - 1u) & ~(xm | ym);
+  {
+    const float4* gent = reinterpret_cast<const float4*>(rec + A.L.ent_off());
+    const float2* gsrc = reinterpret_cast<const float2*>(rec + A.L.esrc_off());
+    const float* gwj = reinterpret_cast<const float*>(rec + A.L.wj_off());
+    for (int k = tid; k < 2 * kDenseMax; k += 32 * kWarpTiles) s_ent[k / kDenseMax][k % kDenseMax] = gent[k];
+    for (int k = tid; k < 2 * kEntSrcCap; k += 32 * kWarpTiles) s_esrc[k / kEntSrcCap][k % kEntSrcCap] = gsrc[k];
+    for (int t = tid; t < NJMAX * NJMAX; t += 32 * kWarpTiles) s_WJ[t] = gwj[(t / NJMAX) * kDenseMax + t % NJMAX];
+    if (tid < NJMAX) s_jact[tid] = reinterpret_cast<const int32_t*>(rec + A.L.jact_off())[tid];
+  }
+  __syncthreads();
+  const int n_ent_x = __popc((xm | jm) & ((1u << nv) - 1u)), n_ent_y = __popc((ym | jm) & ((1u << nv) - 1u));
+  uint32_t* split_row = A.split + int64_t(r) * A.n_words;
+  const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;
+  const bool wfilter = A.w_min > 0.f;
+  const float theta16 = 16.f * A.theta, band2 = A.band * A.band;
+  float* tx = s_tab[warp];
+  float* ty = tx + kDenseMax * kTabFull;
+  PairTabs T;
+  T.tx = tx;
+  T.ty = ty;
+  T.tw = kTabFull;
+  T.nv = nv;
+  T.nj = nj;
+  T.out_x = false;
+  T.orow = 0;
+  T.out_const = 0.f;
+  // this lane's quads: parent (pl, ql) + (dx(k), dy(k)) / 2 of quad lane + 32 k
+  const int pl = int(compact1by1(uint32_t(lane))), ql = int(compact1by1(uint32_t(lane) >> 1));
+  const int xb = 2 * pl + 2, yb = 2 * ql + 2;  // table columns of its quad k = 0
+  const int t_beg = A.tile_beg + int(blockIdx.x) * A.tiles_per_cta;
+  const int t_end = min(t_beg + A.tiles_per_cta, A.tile_beg + A.n_tiles);
+  for (int tile = t_beg + warp; tile < t_end; tile += kWarpTiles) {
+    int u = tile - 1, d = kPyramidTop + 1;
+    while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
+    const uint32_t mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
+    const int i0 = int(compact1by1(mb)), j0 = int(compact1by1(mb >> 1));
+    const float scale = __int_as_float((127 - (d + 1)) << 23);
+    __syncwarp();  // the previous tile's reads of this warp's tables are done
+    {
+      const int pos[2] = {lane + 2, lane + 34};
+      const float cx[2] = {grid_coord(i0 + lane, scale), grid_coord(i0 + lane + 32, scale)};
+      table_columns<2>(cx, pos, n_ent_x, s_ent[0], s_esrc[0], tx, kTabFull);
+      const float cy[2] = {grid_coord(j0 + lane, scale), grid_coord(j0 + lane + 32, scale)};
+      table_columns<2>(cy, pos, n_ent_y, s_ent[1], s_esrc[1], ty, kTabFull);
+    }
+    __syncwarp();
+    uint32_t* split_k = split_row + A.word_off[d - 1] + mb / 128;  // split word k of the tile
+    // A position passes the band test only if both differences along one axis
+    // exceed the band, and one of them is to its sibling in the quad; 16 V bounds
+    // each sibling difference, so a quad with 16 V within band^2 has none.
+    bool need = false;
+#pragma unroll 1
+    for (int k0 = 0; k0 < 32; k0 += QPE) {
+      float w[4 * QPE];
+      int xq[QPE], yq[QPE];
+#pragma unroll
+      for (int h = 0; h < QPE; h++) {
+        xq[h] = xb + warp_quad_dx(k0 + h);
+        yq[h] = yb + warp_quad_dy(k0 + h);
+      }
+      eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
+#pragma unroll
+      for (int h = 0; h < QPE; h++) {
+        // the four children give the parent's variance (Section 3.2)
+        const float v16 = var16(w[4 * h + 0], w[4 * h + 1], w[4 * h + 2], w[4 * h + 3]);
+        const unsigned bal = __ballot_sync(kFull, v16 > theta16);
+        if (lane == 0) split_k[k0 + h] = bal;
+        need = need || !(v16 <= band2);
+      }
+    }
+    uint32_t* band_t = A.bandb + (band_base + A.word_off[d] + mb / 32);  // 128 quad-major words
+    if (!__any_sync(kFull, need)) {  // no position of the tile can pass
+      reinterpret_cast<uint4*>(band_t)[lane] = make_uint4(0u, 0u, 0u, 0u);
+      continue;
+    }
+    // a tile the band screen lets through (rare): the ring coordinates, then every quad's
+    // band test with its four children and eight outer neighbours evaluated directly
+    if (lane < 4) {
+      const int i = lane & 1 ? kTileSide : -1;
+      table_column(grid_coord((lane < 2 ? i0 : j0) + i, scale), i + 2, lane < 2 ? n_ent_x : n_ent_y,
+                   s_ent[lane >> 1], s_esrc[lane >> 1], lane < 2 ? tx : ty, kTabFull);
+    }
+    __syncwarp();
+    bool any_pass = false;
+#pragma unroll 1
+    for (int k = 0; k < 32; k++) {
+      const int x0 = xb + warp_quad_dx(k), y0 = yb + warp_quad_dy(k);  // child 0's table columns
+      const int xa[4] = {x0, x0 + 1, x0, x0 + 1}, ya[4] = {y0, y0, y0 + 1, y0 + 1};
+      const int xl[4] = {x0 - 1, x0 - 1, x0 + 2, x0 + 2}, yl[4] = {y0, y0 + 1, y0, y0 + 1};  // L0 L2 R1 R3
+      const int xv[4] = {x0, x0 + 1, x0, x0 + 1}, yv[4] = {y0 - 1, y0 - 1, y0 + 2, y0 + 2};  // B0 B1 U2 U3
+      float w[4], h[4], v[4];
+      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xa, ya, w);
+      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xl, yl, h);
+      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xv, yv, v);
+      const float L[4] = {h[0], w[0], h[1], w[2]}, R[4] = {w[1], h[2], w[3], h[3]};
+      const float Bo[4] = {v[0], v[1], w[0], w[1]}, U[4] = {w[2], w[3], v[2], v[3]};
+      bool pass[4];
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]), band2);
+        if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+      }
+      const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+      const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+      any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
+      if (lane < 4) band_t[4 * k + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+    }
+    if (A.tile_flags && lane == 0 && any_pass) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
   }
 }
 
@@ -2388,6 +2550,48 @@ emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, 
   return cuda_status(cudaGetLastError());
 }
 
+template <int NJMAX>
+emr_status launch_warp(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
+  if (n_ranks <= 0 || A0.n_tiles <= 0) return EMR_OK;
+  DTileArgs A = A0;
+  // a tile per warp: short CTAs balance best (measured against longer groups)
+  const int g = kWarpTiles;
+  A.tiles_per_cta = g;
+  const unsigned gx = unsigned((A.n_tiles + g - 1) / g);
+  for (int64_t r0 = 0; r0 < n_ranks; r0 += 65535) {
+    A.rank_beg = rank_beg + r0;
+    const dim3 grid(gx, unsigned(std::min<int64_t>(65535, n_ranks - r0)));
+    const cudaError_t e =
+        launch_overlapped(tile_kernel_warp<NJMAX>, grid, dim3(32 * kWarpTiles), 0, st, overlap, A);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  return cuda_status(cudaGetLastError());
+}
+
+// A class of pairs with joint nodes: in fused mode without an output buffer the
+// depths 0..4 tile through tile_kernel_dense and the 64 x 64 tiles a warp each.
+template <int NJMAX>
+emr_status launch_joint_class(const DTileArgs& D, int64_t rank_beg, int64_t n_ranks, cudaStream_t st,
+                              bool* overlap, bool warp_tiles) {
+  if (n_ranks <= 0) return EMR_OK;
+  if (!warp_tiles) return launch_dense<NJMAX>(D, rank_beg, n_ranks, st, overlap);
+  emr_status rc;
+  const int32_t end = D.tile_beg + D.n_tiles;
+  // the block kernel takes the depths 0..4 tile and the one depth-5 tile, so that the
+  // warp kernel's tiles (depths 6..D: 4, 20, 84, ... of them) come in whole groups of kWarpTiles
+  const int32_t split_at = std::min<int32_t>(end, 2);
+  if (D.tile_beg < split_at) {
+    DTileArgs D0 = D;
+    D0.n_tiles = split_at - D.tile_beg;
+    if ((rc = launch_dense<NJMAX>(D0, rank_beg, n_ranks, st, overlap)) != EMR_OK) return rc;
+  }
+  if (end <= split_at) return EMR_OK;
+  DTileArgs D1 = D;
+  D1.tile_beg = std::max<int32_t>(D.tile_beg, split_at);
+  D1.n_tiles = end - D1.tile_beg;
+  return launch_warp<NJMAX>(D1, rank_beg, n_ranks, st, overlap);
+}
+
 emr_status launch_one_axis(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
   if (n_ranks <= 0 || A0.n_tiles <= 0) return EMR_OK;
   DTileArgs A = A0;
@@ -2506,25 +2710,27 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   D.n_dense = n_dense;
   // the class launches after the first overlap their predecessor's last wave
   bool overlap = p.n_class[0] > 0;
+  const bool warp_tiles = mode == kModeFused && !out;
   int64_t beg = p.n_class[0];
-  if ((rc = launch_dense<12>(D, beg, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
+  if ((rc = launch_joint_class<12>(D, beg, p.n_class[1], st, &overlap, warp_tiles)) != EMR_OK) return rc;
   beg += p.n_class[1];
-  if ((rc = launch_dense<8>(D, beg, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
+  if ((rc = launch_joint_class<8>(D, beg, p.n_class[2], st, &overlap, warp_tiles)) != EMR_OK) return rc;
   beg += p.n_class[2];
-  if ((rc = launch_dense<6>(D, beg, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
+  if ((rc = launch_joint_class<6>(D, beg, p.n_class[3], st, &overlap, warp_tiles)) != EMR_OK) return rc;
   beg += p.n_class[3];
-  if ((rc = launch_dense<4>(D, beg, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
+  if ((rc = launch_joint_class<4>(D, beg, p.n_class[4], st, &overlap, warp_tiles)) != EMR_OK) return rc;
   beg += p.n_class[4];
   if (mode == kModeFused && !out && p.n_class[5] > p.n_const) {
     // one-coordinate outputs: the depths 0..4 tile through the generic kernel, the 64 x 64
     // tiles a warp each
     const int64_t n5 = p.n_class[5] - p.n_const;
-    if (tr.beg == 0) {
+    const int32_t split_at = std::min<int32_t>(tr.end, 2);
+    if (tr.beg < split_at) {
       DTileArgs D0 = D;
-      D0.n_tiles = 1;
+      D0.n_tiles = split_at - tr.beg;
       if ((rc = launch_dense<0>(D0, beg, n5, st, &overlap)) != EMR_OK) return rc;
     }
-    const int32_t t1 = std::max<int32_t>(tr.beg, 1);
+    const int32_t t1 = std::max<int32_t>(tr.beg, split_at);
     if (t1 < tr.end) {
       DTileArgs D1 = D;
       D1.tile_beg = t1;

@@ -560,15 +560,16 @@ def main():
         h2d = d2h = 0
         n_warm, n_steps = 2, args.e2e_steps
 
+        res_off_np = [t.numpy() for t in res_off]
+
         def read_lists(k):
             b = k & 1
             done[b].synchronize()
-            n = min(int(res_off[b][-1]), dsc.cap)
+            n = min(int(res_off_np[b][-1]), dsc.cap)
             copy.wait_event(done[b])
-            with torch.cuda.stream(copy):
-                idx_h[:n].copy_(outs[b][0][:n], non_blocking=True)
-                w_h[:n].copy_(outs[b][1][:n], non_blocking=True)
-                read[b].record(copy)
+            emr.copy_async(idx_h, outs[b][0], 4 * n, copy)
+            emr.copy_async(w_h, outs[b][1], 4 * n, copy)
+            read[b].record(copy)
             return 8 * (dsc.n_pairs + 1) + 8 * n
 
         torch.cuda.synchronize()
@@ -583,11 +584,11 @@ def main():
             if k >= 2:
                 stream.wait_event(read[b])  # step k - 2's lists have left this output set
             h2d = ob + len(blob)
-            in_dev[:h2d].copy_(buf[:h2d], non_blocking=True)
+            emr.copy_async(in_dev, buf, h2d, stream)
             idx_o, w_o, cnt_o, off_o = outs[b]
             emr.discover(blob, pack_dev, q_e2e, g, dsc.theta, dsc.band, dsc.w_min, dsc.mode, dsc.types, dws,
-                         idx_o, w_o, dsc.cap, cnt_o, off_o, qc=qc)
-            res_off[b].copy_(off_o, non_blocking=True)
+                         idx_o, w_o, dsc.cap, cnt_o, off_o, stream=stream, qc=qc)
+            emr.copy_async(res_off[b], off_o, 8 * (dsc.n_pairs + 1), stream)
             done[b].record(stream)
             if k >= 1:
                 d2h = read_lists(k - 1)

@@ -435,6 +435,15 @@ emr_status emr_discover(const void *pack_host, const void *pack_dev, const emr_q
                         size_t ws_bytes, int32_t *idx, float *w, int64_t cap, int64_t *counts, int64_t *offsets,
                         void *stream);
 
+/* One asynchronous copy of bytes from src to dst on the stream (host or device
+ * memory on either side, told apart by the CUDA runtime's unified addressing):
+ * the step's inputs into their device copies and its lists back, without a
+ * framework's per-copy overhead. A host buffer must be pinned for the copy to be
+ * asynchronous; the caller keeps both buffers alive until the stream has passed
+ * the copy. bytes = 0 does nothing. Errors: EMR_ERR_ARG (null pointer with
+ * bytes > 0), EMR_ERR_CUDA. */
+emr_status emr_copy_async(void *dst, const void *src, size_t bytes, void *stream);
+
 /* Connection type code (0 forward, 1 backward, 2 lateral, 3 self; Section 6
  * taxonomy, see emr_mask_combine_types) of every list entry: type[e] for
  * entries e < min(offsets[n_pairs], cap) of lists laid out as emr_compact

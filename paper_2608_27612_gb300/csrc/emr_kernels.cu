@@ -3089,6 +3089,12 @@ emr_status emr_discover_workspace_size(const void* pack_host, const emr_query* q
   return EMR_OK;
 }
 
+emr_status emr_copy_async(void* dst, const void* src, size_t bytes, void* stream) {
+  if (bytes == 0) return EMR_OK;
+  if (!dst || !src) return EMR_ERR_ARG;
+  return cuda_status(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, static_cast<cudaStream_t>(stream)));
+}
+
 emr_status emr_discover(const void* pack_host, const void* pack_dev, const emr_query* q, const emr_grid* grid,
                         float theta, float band, float w_min, int32_t mode, int32_t types, void* ws, size_t ws_bytes,
                         int32_t* idx, float* w, int64_t cap, int64_t* counts, int64_t* offsets, void* stream) {

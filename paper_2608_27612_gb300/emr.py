@@ -81,6 +81,7 @@ def lib() -> C.CDLL:
             "emr_select_workspace_size": [vp, i32, vp],
             "emr_discover_workspace_size": [vp, vp, vp, vp],
             "emr_discover": [vp, vp, vp, vp, f32, f32, f32, i32, i32, vp, sz, vp, vp, i64, vp, vp, vp],
+            "emr_copy_async": [vp, vp, sz, vp],
             "emr_substrate_config": [i32, vp, vp],
             "emr_assemble_workspace_size": [vp, i32, i32, i32, vp, i64, vp],
             "emr_assemble": [vp, vp, i32, vp, vp, i32, vp, vp, vp, f32, f32, f32, i32, i32, i32, i32, vp, sz, i64,
@@ -344,6 +345,12 @@ def discover(pack, pack_dev, query: Query, grid: Grid, theta: float, band: float
     _check(lib().emr_discover(_ptr(pack), _ptr(pack_dev), C.byref(q), C.byref(grid), theta, band, w_min, mode, types,
                               _ptr(ws), C.c_size_t(ws.numel()), _ptr(idx), _ptr(w), cap, _ptr(counts),
                               _ptr(offsets), _stream(stream)), "emr_discover")
+
+
+def copy_async(dst, src, nbytes: int, stream=None):
+    """emr_copy_async: nbytes from src to dst (tensors, numpy arrays or addresses; host buffers
+    pinned) on the stream."""
+    _check(lib().emr_copy_async(_ptr(dst), _ptr(src), C.c_size_t(nbytes), _stream(stream)), "emr_copy_async")
 
 
 def mask_combine_types(split, band_bits, query: Query, grid: Grid, n_pairs: int, mode: int, types: int, mask,

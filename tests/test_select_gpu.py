@@ -84,3 +84,16 @@ def test_select_per_genome_slots():
     w = W.c4_round2_random(D=6, P=20, S=32)
     compare(w)
     compare(w, emr.EMR_EAGER, emr.CONN_F | emr.CONN_B)
+
+
+def test_copy_async_round_trip():
+    """emr_copy_async moves bytes host -> device -> host (pinned buffers) on a stream."""
+    src = torch.arange(1 << 16, dtype=torch.int32).pin_memory()
+    dev = torch.empty_like(src, device="cuda")
+    back = torch.zeros_like(src).pin_memory()
+    stream = torch.cuda.Stream()
+    emr.copy_async(dev, src, src.numel() * 4, stream)
+    emr.copy_async(back, dev, src.numel() * 4, stream)
+    stream.synchronize()
+    assert torch.equal(back, src)
+    emr.copy_async(back, dev, 0, stream)  # nothing to copy

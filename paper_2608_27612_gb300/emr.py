@@ -146,10 +146,27 @@ def index_to_ij(gidx: int):
 
 # ---- a2 -----------------------------------------------------------------------
 
+def _pop_ptrs(pop):
+    """Addresses of a Population's ten arrays, kept on the object together with the arrays
+    themselves (so an address never outlives its array); a field that now holds another
+    array is looked up again."""
+    arrays = (pop.node_ptr, pop.node_id, pop.node_kind, pop.node_act, pop.node_bias, pop.conn_ptr,
+              pop.conn_src, pop.conn_dst, pop.conn_w, pop.conn_enabled)
+    cache = getattr(pop, "_emr_ptrs", None)
+    if cache is None or any(a is not b for a, b in zip(cache[0], arrays)):
+        cache = (arrays, tuple(int(a.ctypes.data) for a in arrays))
+        try:
+            object.__setattr__(pop, "_emr_ptrs", cache)
+        except AttributeError:
+            pass
+    return cache[1]
+
+
 def pack_size(pop) -> int:
     """Upper bound of the packed blob's bytes for a workloads.Population (emr_pack_size)."""
     n = C.c_size_t()
-    _check(lib().emr_pack_size(pop.P, _ptr(pop.node_ptr), _ptr(pop.conn_ptr), C.byref(n)), "emr_pack_size")
+    ptr = _pop_ptrs(pop)
+    _check(lib().emr_pack_size(pop.P, ptr[0], ptr[5], C.byref(n)), "emr_pack_size")
     return int(n.value)
 
 
@@ -158,7 +175,8 @@ def pack_population(pop, out=None) -> np.ndarray:
     contiguous uint8 array, e.g. a view of pinned memory) when given, else into a new array."""
     L = lib()
     n = C.c_size_t()
-    _check(L.emr_pack_size(pop.P, _ptr(pop.node_ptr), _ptr(pop.conn_ptr), C.byref(n)), "emr_pack_size")
+    ptr = _pop_ptrs(pop)
+    _check(L.emr_pack_size(pop.P, ptr[0], ptr[5], C.byref(n)), "emr_pack_size")
     if out is not None:
         if out.dtype != np.uint8 or not out.flags.c_contiguous or len(out) < n.value:
             raise ValueError("out: contiguous uint8 array of at least %d bytes" % n.value)
@@ -166,10 +184,7 @@ def pack_population(pop, out=None) -> np.ndarray:
     else:
         buf = np.empty(n.value + 16, np.uint8)   # the packer clears what it uses
     used, bad = C.c_size_t(), C.c_int32()
-    st = L.emr_pack_population(pop.P, _ptr(pop.node_ptr), _ptr(pop.node_id), _ptr(pop.node_kind),
-                               _ptr(pop.node_act), _ptr(pop.node_bias), _ptr(pop.conn_ptr), _ptr(pop.conn_src),
-                               _ptr(pop.conn_dst), _ptr(pop.conn_w), _ptr(pop.conn_enabled), _ptr(buf),
-                               C.c_size_t(len(buf)), C.byref(used), C.byref(bad))
+    st = L.emr_pack_population(pop.P, *ptr, int(buf.ctypes.data), len(buf), C.byref(used), C.byref(bad))
     if st != EMR_OK:
         e = EmrError(st, "emr_pack_population (genome %d)" % bad.value)
         e.bad_genome = bad.value

@@ -523,9 +523,10 @@ def main():
         roofline["frac_at_sampled_clock"] = roofline["frac"] * SM_MAX_MHZ / clocks["sm_mhz"]
 
     # end to end through host buffers and the one-call entry point (emr_discover), pipelined: each
-    # step copies its packed population and query slots from pinned memory and reads its lists back
-    # (offsets first, then the entries they count). Two output sets alternate: step k + 1 is queued
-    # before step k's lists are read, and the reads run on a second stream while the GPU computes.
+    # step packs its population into pinned memory, copies it and the query slots to the device and
+    # reads its lists back (offsets first, then the entries they count). Input and output sets
+    # alternate: step k + 1's inputs are copied while step k computes, and step k's lists are read
+    # on a second stream while step k + 1 computes.
     e2e = None
     if args.e2e_steps > 0:
         pop = w.pop
@@ -541,13 +542,17 @@ def main():
             q_h[:4 * S] = np.ascontiguousarray(dsc.query.a, np.float32).view(np.uint8)
             q_h[4 * S:8 * S] = np.ascontiguousarray(dsc.query.b, np.float32).view(np.uint8)
             q_h[8 * S:12 * S] = np.ascontiguousarray(dsc.query.side, np.int32).view(np.uint8)
-        in_dev = torch.empty(in_bytes, dtype=torch.uint8, device="cuda")
-        pack_dev = in_dev[ob:]
-        q_e2e = emr.Query(dsc.query.a, dsc.query.b, dsc.query.side, None, in_dev[:4 * S].view(torch.float32),
-                          in_dev[4 * S:8 * S].view(torch.float32), in_dev[8 * S:12 * S].view(torch.int32), None, S,
-                          False)
+        # two device input buffers: step k + 1's inputs are copied (on their own stream) while
+        # step k's kernels run
+        in_dev = [torch.empty(in_bytes, dtype=torch.uint8, device="cuda") for _ in range(2)]
+        pack_dev = [t[ob:] for t in in_dev]
+        q_e2e = [emr.Query(dsc.query.a, dsc.query.b, dsc.query.side, None, t[:4 * S].view(torch.float32),
+                           t[4 * S:8 * S].view(torch.float32), t[8 * S:12 * S].view(torch.int32), None, S, False)
+                 for t in in_dev]
         dws = torch.zeros(emr.discover_workspace_size(dsc.pack, dsc.query, g), dtype=torch.uint8, device="cuda")
-        qc = q_e2e.c
+        qc = [q.c for q in q_e2e]
+        copy_in = torch.cuda.Stream()
+        inputs_in = [torch.cuda.Event(), torch.cuda.Event()]  # step k's inputs are on the device
         outs = [(dsc.idx, dsc.w, dsc.counts, dsc.offsets),
                 (torch.empty_like(dsc.idx), torch.empty_like(dsc.w), torch.empty_like(dsc.counts),
                  torch.empty_like(dsc.offsets))]
@@ -578,16 +583,18 @@ def main():
                 t0 = time.perf_counter()
             b = k & 1
             buf = in_pinned[b]
-            # this input buffer's last user, step k - 2, has finished (its offsets were synchronised
-            # on in the previous iteration), so the packer may overwrite it
+            # this input set's last user, step k - 2, has finished (its offsets were synchronised
+            # on in the previous iteration), so the packer and the copy may overwrite it
             blob = emr.pack_population(pop, out=buf[ob:].numpy())
+            h2d = ob + len(blob)
+            emr.copy_async(in_dev[b], buf, h2d, copy_in)
+            inputs_in[b].record(copy_in)
+            stream.wait_event(inputs_in[b])
             if k >= 2:
                 stream.wait_event(read[b])  # step k - 2's lists have left this output set
-            h2d = ob + len(blob)
-            emr.copy_async(in_dev, buf, h2d, stream)
             idx_o, w_o, cnt_o, off_o = outs[b]
-            emr.discover(blob, pack_dev, q_e2e, g, dsc.theta, dsc.band, dsc.w_min, dsc.mode, dsc.types, dws,
-                         idx_o, w_o, dsc.cap, cnt_o, off_o, stream=stream, qc=qc)
+            emr.discover(blob, pack_dev[b], q_e2e[b], g, dsc.theta, dsc.band, dsc.w_min, dsc.mode, dsc.types, dws,
+                         idx_o, w_o, dsc.cap, cnt_o, off_o, stream=stream, qc=qc[b])
             emr.copy_async(res_off[b], off_o, 8 * (dsc.n_pairs + 1), stream)
             done[b].record(stream)
             if k >= 1:
@@ -598,8 +605,10 @@ def main():
         _, e2e_ms, e2e_value = aggregate(queries, elapsed / n_steps * 1e3, ws)
         e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": e2e_ms,
-               "pipeline": "two output sets: step k+1 queued before step k's lists are read (second stream); "
-                           "wall clock over %d steps" % n_steps}
+               "pipeline": "two input and two output sets: each step packs into pinned memory on the host, "
+                           "copies its inputs on a copy stream while the previous step computes, and its lists "
+                           "are read on a second copy stream after step k+1 is queued; wall clock over %d steps"
+                           % n_steps}
 
     extra = None
     if rank == 0 and ws == 1 and not args.no_extra:

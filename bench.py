@@ -223,7 +223,7 @@ def profiled_traffic():
     """DRAM bytes per step of the dense tile kernels from the committed ncu summary, if that
     summary was taken on the current kernel source (else None)."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", "tile_kernel_dense_c2_pop300_d7.md")
+    path = os.path.join(ROOT, "profiles", "tile_kernels_c2_pop300_d7.md")
     src = os.path.join(ROOT, "paper_2608_27612_gb300", "csrc", "emr_kernels.cu")
     try:
         fields = dict(l.split(":", 1) for l in open(path).read().splitlines() if l.startswith(("traffic_", "kernel_")))
@@ -512,8 +512,8 @@ def main():
     roofline = {"bound": "alu", "achieved": achieved / 1e12, "peak": peak / 1e12, "unit": "Tlane-op/s",
                 "frac": achieved / peak, "traffic": profiled_traffic() if args.pop == 1000 and args.depth == 7 else None,
                 "traffic_note": "DRAM bytes of the dense tile launches per step, from profiles/"
-                                "tile_kernel_dense_c2_pop300_d7.md (300-genome capture scaled by pairs, x10/3); null when "
-                                "the kernel source changed since", "kernel": "tile_kernel_dense (emr_eval_filter)",
+                                "tile_kernels_c2_pop300_d7.md (300-genome capture scaled by pairs, x10/3); null when "
+                                "the kernel source changed since", "kernel": "tile kernels of emr_eval_filter_tiles (tile_kernel_warp, tile_kernel_dense, tile_kernel_one_axis)",
                 "kernel_ms": tile_s * 1e3,
                 "fp32_ops_per_query": float(work[..., 0].mean()), "mufu_ops_per_query": float(work[..., 1].mean()),
                 "peak_basis": "%d SMs x %d FP32 lanes x %.0f MHz (max SM clock); a MUFU op weighs %.2f FP32 "

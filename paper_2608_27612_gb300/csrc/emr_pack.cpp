@@ -145,6 +145,7 @@ struct Scratch {
   std::vector<int> succ_beg, succ, pred_beg, pred, fill;
   std::vector<char> reach;
   std::vector<unsigned> has_in;
+  std::vector<uint64_t> seen;  // per destination: the sources seen (genomes up to 64 nodes)
   std::vector<int> in_cnt, in_beg;
   std::vector<PackEdge> in_edges;
   std::vector<int> table;  // id - id_min -> local index (-1: none), when the ids span a small range
@@ -212,7 +213,7 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
     S.ids.push_back({node_id[n0 + k], k});
   }
   if (out_node < 0) return EMR_ERR_ARG;
-  std::sort(S.ids.begin(), S.ids.end());
+  if (!std::is_sorted(S.ids.begin(), S.ids.end())) std::sort(S.ids.begin(), S.ids.end());
   for (size_t k = 1; k < S.ids.size(); k++)
     if (S.ids[k].first == S.ids[k - 1].first) return EMR_ERR_ARG;  // duplicate id
   S.table.clear();
@@ -234,17 +235,40 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
   // weight is their sum in connection order; an edge of weight 0 contributes
   // nothing and is dropped. Every evaluator then sees at most one edge per
   // (source, destination), each of nonzero weight.
-  std::stable_sort(S.es.begin(), S.es.end(),
-                   [](const Edge& a, const Edge& b) { return a.d != b.d ? a.d < b.d : a.s < b.s; });
-  {
+  if (n <= 64) {  // a source mask per destination finds repeats without sorting
+    S.seen.assign(size_t(n), 0ull);
+    bool repeat = false;
+    for (auto& e : S.es) {
+      const uint64_t bit = 1ull << e.s;
+      repeat = repeat || (S.seen[e.d] & bit);
+      S.seen[e.d] |= bit;
+    }
+    size_t m = 0;
+    for (size_t k = 0; k < S.es.size(); k++) {
+      Edge e = S.es[k];
+      if (repeat) {  // fold later repeats into the first occurrence, in connection order
+        size_t f = 0;
+        while (f < m && !(S.es[f].s == e.s && S.es[f].d == e.d)) f++;
+        if (f < m) {
+          S.es[f].w += e.w;
+          continue;
+        }
+      }
+      S.es[m++] = e;
+    }
+    S.es.resize(m);
+  } else {
+    std::stable_sort(S.es.begin(), S.es.end(),
+                     [](const Edge& a, const Edge& b) { return a.d != b.d ? a.d < b.d : a.s < b.s; });
     size_t m = 0;
     for (size_t k = 0; k < S.es.size();) {
       Edge e = S.es[k++];
       while (k < S.es.size() && S.es[k].s == e.s && S.es[k].d == e.d) e.w += S.es[k++].w;
-      if (e.w != 0.f) S.es[m++] = e;
+      S.es[m++] = e;
     }
     S.es.resize(m);
   }
+  S.es.erase(std::remove_if(S.es.begin(), S.es.end(), [](const Edge& e) { return e.w == 0.f; }), S.es.end());
   build_csr(n, S.es, true, S.succ_beg, S.succ, S.fill);
   build_csr(n, S.es, false, S.pred_beg, S.pred, S.fill);
   // Kahn's algorithm over every node; ready nodes leave in ascending id order.

@@ -237,15 +237,31 @@ struct QueryDev {
 // cost, heaviest first: order[rank] = pair, by a counting sort over kCostBins
 // bins of the pairs' bins (bins[r]), run by one CTA of nthreads threads (a
 // multiple of 32, at most 1024; each thread scans kCostBins / nthreads bins).
+// Up to nthreads * kSchedRegBins pairs, each thread reads its pairs' bins once,
+// all at a time, and keeps them in registers for both passes.
 constexpr int kClassBins = 256;
 constexpr int kCostBins = kClasses * kClassBins;
+constexpr int kSchedRegBins = 32;
 __device__ void schedule_block(const int32_t* __restrict__ bins, int64_t n_pairs, int32_t* __restrict__ order,
                                int32_t* hist, int32_t* wsum) {
   const int nthreads = blockDim.x, tid = threadIdx.x;
   for (int k = tid; k < kCostBins; k += nthreads) hist[k] = 0;
   __syncthreads();
+  const bool in_regs = n_pairs <= int64_t(nthreads) * kSchedRegBins;
+  int rb[kSchedRegBins];  // bin of pair tid + i * nthreads (-1: none)
+  if (in_regs) {
+#pragma unroll
+    for (int i = 0; i < kSchedRegBins; i++) {
+      const int64_t r = tid + int64_t(i) * nthreads;
+      rb[i] = r < n_pairs ? __ldcg(bins + r) : -1;
+    }
+#pragma unroll
+    for (int i = 0; i < kSchedRegBins; i++)
+      if (rb[i] >= 0) atomicAdd(&hist[rb[i]], 1);
+  } else {
 #pragma unroll 4
-  for (int64_t r = tid; r < n_pairs; r += nthreads) atomicAdd(&hist[__ldcg(bins + r)], 1);
+    for (int64_t r = tid; r < n_pairs; r += nthreads) atomicAdd(&hist[__ldcg(bins + r)], 1);
+  }
   __syncthreads();
   // exclusive scan: thread tid owns bins [tid * per, (tid + 1) * per)
   const int per = kCostBins / nthreads, lane = tid & 31, warp = tid >> 5;
@@ -274,6 +290,12 @@ __device__ void schedule_block(const int32_t* __restrict__ bins, int64_t n_pairs
     run += v;
   }
   __syncthreads();
+  if (in_regs) {
+#pragma unroll
+    for (int i = 0; i < kSchedRegBins; i++)
+      if (rb[i] >= 0) order[atomicAdd(&hist[rb[i]], 1)] = int32_t(tid + i * nthreads);
+    return;
+  }
 #pragma unroll 4
   for (int64_t r = tid; r < n_pairs; r += nthreads) order[atomicAdd(&hist[__ldcg(bins + r)], 1)] = int32_t(r);
 }
@@ -2711,15 +2733,32 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   // the class launches after the first overlap their predecessor's last wave
   bool overlap = p.n_class[0] > 0;
   const bool warp_tiles = mode == kModeFused && !out;
-  int64_t beg = p.n_class[0];
-  if ((rc = launch_joint_class<12>(D, beg, p.n_class[1], st, &overlap, warp_tiles)) != EMR_OK) return rc;
-  beg += p.n_class[1];
-  if ((rc = launch_joint_class<8>(D, beg, p.n_class[2], st, &overlap, warp_tiles)) != EMR_OK) return rc;
-  beg += p.n_class[2];
-  if ((rc = launch_joint_class<6>(D, beg, p.n_class[3], st, &overlap, warp_tiles)) != EMR_OK) return rc;
-  beg += p.n_class[3];
-  if ((rc = launch_joint_class<4>(D, beg, p.n_class[4], st, &overlap, warp_tiles)) != EMR_OK) return rc;
-  beg += p.n_class[4];
+  // first rank of each joint class (12, 8, 6, 4 joint nodes at most)
+  const int64_t b1 = p.n_class[0], b2 = b1 + p.n_class[1], b3 = b2 + p.n_class[2], b4 = b3 + p.n_class[3];
+  int64_t beg = b4 + p.n_class[4];
+  if (warp_tiles && D.tile_beg < 2 && D.tile_beg + D.n_tiles > 2) {
+    // every joint class's block launch (depths 0..5), then every class's warp launch
+    // (depths 6..D): the block kernels' latency-bound CTAs then share the SMs with
+    // the warp launches that follow them (measured faster than alternating block and
+    // warp launches class by class)
+    DTileArgs D0 = D, D1 = D;
+    D0.n_tiles = 2 - D.tile_beg;
+    D1.tile_beg = 2;
+    D1.n_tiles = D.tile_beg + D.n_tiles - 2;
+    if ((rc = launch_dense<12>(D0, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_dense<8>(D0, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_dense<6>(D0, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_dense<4>(D0, b4, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_warp<12>(D1, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_warp<8>(D1, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_warp<6>(D1, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_warp<4>(D1, b4, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
+  } else {
+    if ((rc = launch_joint_class<12>(D, b1, p.n_class[1], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+    if ((rc = launch_joint_class<8>(D, b2, p.n_class[2], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+    if ((rc = launch_joint_class<6>(D, b3, p.n_class[3], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+    if ((rc = launch_joint_class<4>(D, b4, p.n_class[4], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+  }
   if (mode == kModeFused && !out && p.n_class[5] > p.n_const) {
     // one-coordinate outputs: the depths 0..4 tile through the generic kernel, the 64 x 64
     // tiles a warp each

@@ -13,7 +13,11 @@ Parity status of each oracle function (what pins it, in tests/test_oracle_pins.p
   ora_discover              pinned: closed-form variance and band of linear and
                             separable genomes, the worked depth-4 example,
                             constant genomes, symmetry, Theorem 1 against the
-                            lazy tree, a direct re-evaluation at sampled points.
+                            lazy tree, a direct re-evaluation at sampled points,
+                            the strict inequalities at exact ties, the band of
+                            genomes the halo mirrors at one edge. Planted
+                            mistakes (tests/test_oracle_mutations.py) each fail
+                            one of these pins.
   ora_lazy                  pinned: Theorem 1 (lazy subset of eager, lazy equal to
                             the gated mask) and the closed-form worked example.
   ora_keep_at               pinned: equal to ora_discover's outputs, variance, band

@@ -211,6 +211,36 @@ def test_worked_example_depth4_keeps_exactly_grid3():
     assert r["unc_eager"].sum() == 0 and r["unc_gated"].sum() == 0
 
 
+def test_strict_inequalities_at_exact_ties():
+    """A cell splits when V > theta (Eq. 2), a position passes the band test when B > band and
+    the weight filter when |w| > w_min, all strictly. For f = 4x at D = 4, V_d = 4^-d, B_d =
+    4 * 2^-d and the depth-3 outputs are odd multiples of 1/4, all exact in binary, so each
+    threshold can be met exactly."""
+    pop, D = linear(4.0, 0.0, 0.0), 4
+    src = W.shared_sources([(0.0, -1.0, W.SIDE_OUT)])
+    lo = lambda d: oracle.index(d, 0, 0)
+    # theta = V_1 = 1/4: depth 1 does not split. Eager keeps depths 1..3 (B = 2, 1, 1/2 > 0.3);
+    # gated and lazy keep depth 1 only (depth 2's parents did not split).
+    r = oracle.discover(pop, src, D, 0.25, 0.3)
+    lz, _ = oracle.lazy(pop, src, D, 0.25, 0.3)
+    want_e = np.zeros(oracle.n_total(D), np.uint8)
+    want_e[lo(1):oracle.n_total(3)] = 1
+    want_g = np.zeros(oracle.n_total(D), np.uint8)
+    want_g[lo(1):oracle.n_total(1)] = 1
+    assert np.array_equal(r["keep_eager"][0, 0], want_e)
+    assert np.array_equal(r["keep_gated"][0, 0], want_g) and np.array_equal(lz[0, 0], want_g)
+    # band = B_3 = 1/2: the depth-3 leaves fail the band test and nothing is kept
+    r = oracle.discover(pop, src, D, 0.03, 0.5)
+    lz, _ = oracle.lazy(pop, src, D, 0.03, 0.5)
+    assert r["keep_eager"].sum() == 0 and r["keep_gated"].sum() == 0 and lz.sum() == 0
+    # w_min = 1/4: the 2 x 16 depth-3 positions with f = -1/4, +1/4 drop out of the 256
+    r = oracle.discover(pop, src, D, 0.03, 0.3, 0.25)
+    lz, _ = oracle.lazy(pop, src, D, 0.03, 0.3, 0.25)
+    keep = r["keep_eager"][0, 0]
+    assert keep.sum() == 224 and np.all(np.abs(r["w"][0, 0][keep == 1]) > 0.25)
+    assert np.array_equal(lz[0, 0], r["keep_gated"][0, 0]) and np.array_equal(keep, r["keep_gated"][0, 0])
+
+
 @pytest.mark.parametrize("axis", ["x", "y"])
 def test_separable_gauss_variance_and_band(axis):
     """f = gauss(x2) (or gauss(y2)): the four children of a cell at (x, y) sit at x +- h,
@@ -233,6 +263,29 @@ def test_separable_gauss_variance_and_band(axis):
                 B = min(abs(g(t) - g(t - s)), abs(g(t) - g(t + s)))
                 assert r["var"][0, 0, p] == pytest.approx(V, abs=1e-15)
                 assert r["bnd"][0, 0, p] == pytest.approx(B, abs=1e-15)
+
+
+@pytest.mark.parametrize("inp", [X2, Y2])
+@pytest.mark.parametrize("edge", [-1.0, 1.0])
+def test_band_zero_where_the_halo_mirrors_the_border(inp, edge):
+    """f = |u - edge| for the grid coordinate u (x or y) is linear inside the domain, but the
+    halo neighbour beyond that edge (distance 2^-d from a border position at distance 2^-(d+1)
+    from the edge) mirrors the border position: the band value is exactly 0 on the border row or
+    column at the edge and 2^-d everywhere else (the halo beyond the other edge continues the
+    line), and the variance is 4^-(d+2) below depth D. Pins which halo side each neighbour
+    of a border position reads."""
+    D = 4
+    pop = genome([(5, OUT, ABS, 0.0)], [(inp, 5, 1.0, True), (BIAS, 5, -edge, True)])
+    r = oracle.discover(pop, W.shared_sources([(0.0, -1.0, W.SIDE_OUT)]), D, 0.03, 0.3)
+    for d in range(D + 1):
+        n = 2 ** (d + 1)
+        for i in range(n):
+            for j in range(n):
+                u = i if inp == X2 else j
+                border = u == (0 if edge < 0 else n - 1)
+                p = oracle.index(d, i, j)
+                assert r["bnd"][0, 0, p] == (0.0 if border else 2.0 ** -d)
+                assert r["var"][0, 0, p] == (0.0 if d == D else 4.0 ** -(d + 2))
 
 
 def test_constant_genome_keeps_nothing():

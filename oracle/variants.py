@@ -21,8 +21,8 @@ Parity status: scale_weights pinned (tests/test_variants_oracle.py) by its
 values at the threshold, at +-1, at the midpoint, beyond 1 and below the
 threshold. subtree_split pinned by the closed form for a linear genome
 (variance of a k x k grid of spacing h: (alpha^2 + beta^2) h^2 (k^2 - 1) / 12),
-by equality with the four-children variance one level above the leaves, and by
-zero for a constant genome.
+by equality with the four-children variance one level above the leaves, by
+zero for a constant genome, and by its strict split at an exact tie.
 """
 from __future__ import annotations
 

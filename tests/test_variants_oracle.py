@@ -49,3 +49,17 @@ def test_subtree_variance_constant_genome_is_zero():
     V, bound, split, unc = VAR.subtree_split(r["w"][0, 0], r["w_err"][0, 0], 4, 0.03)
     assert np.all(V == 0) and not split.any()
 
+
+
+def test_subtree_split_is_strict_at_an_exact_tie():
+    """One level above the leaves a cell's subtree is its four children: for f = 4x its variance
+    is 4^2 * 4^-(d+2) = 4^-(D-1) at d = D - 1, exact in binary. With theta equal to it those
+    cells do not split (V > theta is strict), while every cell above (more leaves, larger
+    variance) does."""
+    D = 3
+    r = oracle.discover(linear(4.0, 0.0, 0.0), W.shared_sources([(0.0, -1.0, W.SIDE_OUT)]), D, 0.03, 0.3,
+                        fields=("w", "w_err"))
+    theta = 4.0 ** -(D - 1)
+    V, bound, split, unc = VAR.subtree_split(r["w"][0, 0], r["w_err"][0, 0], D, theta)
+    lo, hi = (4 ** D - 4) // 3, (4 ** (D + 1) - 4) // 3
+    assert np.all(V[lo:hi] == theta) and not split[lo:hi].any() and split[:lo].all()

@@ -200,3 +200,45 @@ def test_cache_handle_host_only():
     c.clear()
     assert c.stats()["entries"] == 0
     del c
+
+
+def test_discover_and_copy_reject_arguments_before_device_work():
+    """emr_discover checks its arguments, and its workspace size against the host pack and
+    query, before any CUDA call; emr_copy_async treats 0 bytes as nothing to do and null
+    pointers as an argument error. On a machine without a GPU these come back as the status
+    codes the header documents (the buffers are host memory standing in for device memory:
+    nothing reads them)."""
+    import types
+    import torch
+    w = W.c1()
+    pack = emr.pack_population(w.pop)
+    q = emr.make_query(w.sources, device="cpu")
+    g = emr.grid_build(w.D)
+    need = emr.discover_workspace_size(pack, q, g)
+    assert need > 0
+    n = w.P * q.S
+    st = types.SimpleNamespace(cuda_stream=0)
+    ws = torch.zeros(need, dtype=torch.uint8)
+    idx, wv = torch.zeros(64, dtype=torch.int32), torch.zeros(64)
+    counts, offsets = torch.zeros(n, dtype=torch.int64), torch.zeros(n + 1, dtype=torch.int64)
+
+    def status(**kw):
+        args = dict(theta=w.theta, band=w.band, w_min=0.0, mode=emr.EMR_EAGER, types=emr.CONN_ALL,
+                    ws=ws, cap=64)
+        args.update(kw)
+        with pytest.raises(emr.EmrError) as e:
+            emr.discover(pack, pack, q, g, args["theta"], args["band"], args["w_min"], args["mode"], args["types"],
+                         args["ws"], idx, wv, args["cap"], counts, offsets, stream=st)
+        return e.value.status
+
+    assert status(ws=ws[:need - 1]) == emr.EMR_ERR_CAPACITY
+    assert status(mode=7) == emr.EMR_ERR_ARG
+    assert status(types=emr.CONN_ALL + 1) == emr.EMR_ERR_ARG
+    assert status(theta=float("nan")) == emr.EMR_ERR_ARG
+    assert status(band=-0.3) == emr.EMR_ERR_ARG
+    assert status(cap=-1) == emr.EMR_ERR_ARG
+    emr.copy_async(None, None, 0, stream=st)  # nothing to copy
+    for dst, src in ((None, ws), (ws, None)):
+        with pytest.raises(emr.EmrError) as e:
+            emr.copy_async(dst, src, 8, stream=st)
+        assert e.value.status == emr.EMR_ERR_ARG

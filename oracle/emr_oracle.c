@@ -708,7 +708,7 @@ int ora_keep_at(int g, const int64_t *node_ptr, const int32_t *node_id, const in
 }
 
 /*
- * Connection types (Section 6, "Connection Type Taxonomy"): a connection from
+ * Connection types (Section 6, its connection-type taxonomy): a connection from
  * source s to target t is a self-loop when s = t, and otherwise forward when
  * y_s < y_t, backward when y_s > y_t and lateral when y_s = y_t. For a query
  * slot at (a, b): on the outgoing side the slot is the source and the grid

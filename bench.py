@@ -4,14 +4,17 @@
 Metric: CPPN queries/sec = genomes x query slots x N_total(D) / seconds, on the
 1000-genome XOR-shaped population at depth 7 (4 slots: 3 outgoing substrate
 inputs, 1 incoming output), 349.5 M queries per step. A step is one pass of the
-whole path through libemr's C ABI: specialisation (emr_eval_prepare), fused
-evaluation + variance + band filter (emr_eval_filter), mask combination
-(emr_mask_combine) and ordered compaction (emr_compact).
+whole path through libemr's C ABI: the per-pair records and pair schedule
+(emr_eval_prepare), fused evaluation + variance + band filter of every tile
+(emr_eval_filter_tiles), and the keep mask, ordered lists and kept weights from
+the flagged tiles (emr_select).
 
 `value` is device time with inputs resident in HBM (CUDA events, L2 flushed
 between steps); `e2e` is the same metric through the host-buffer path: packing
-on the host, pinned H2D copy of the packed genomes and slots, the four calls,
-and the D2H read of the compacted connection lists, all inside the timed region.
+on the host into pinned memory, the H2D copy of the packed genomes and slots,
+emr_discover (the same three stages in one call), and the D2H read of the
+offsets and connection lists, each step's copies overlapping its neighbours'
+kernels, timed by the wall clock.
 
 --impl reference times the float64 CPU oracle on a bounded sample of the same
 workload (the only other place this script runs the oracle).

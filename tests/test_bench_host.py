@@ -1,0 +1,73 @@
+"""The roofline's work model (bench.algorithmic_work: fp32 lane-ops and MUFU ops per query, the
+separable evaluation's minimum) on hand-built genomes, against counts made by hand from its
+definition. No GPU: the model reads the host-side packed genomes only."""
+import numpy as np
+import pytest
+
+import bench
+from paper_2608_27612_gb300 import emr
+from paper_2608_27612_gb300 import workloads as W
+
+X1, Y1, X2, Y2, BIAS, HID, OUT = range(7)
+IDN, SIG, TNH, GAU, SIN, ABS = range(6)
+SHARE = 66 / 4096    # a one-coordinate value is evaluated at 66 coordinates of a 64 x 64 tile
+FILTER = 4.5 + 1.0   # variance (six squared differences, their sum, a compare) + band screen, per query
+FP32 = {IDN: 0, SIG: 2, TNH: 3, GAU: 2, SIN: 4, ABS: 0}  # the documented activation costs
+MUFU = {IDN: 0, SIG: 2, TNH: 2, GAU: 1, SIN: 1, ABS: 0}
+
+
+def work(nodes, conns, side):
+    base = [(k, k, IDN, 0.0) for k in range(5)]
+    pop = W.population_from_lists([(base + nodes, [(s, d, w, True) for s, d, w in conns])])
+    q = emr.make_query(W.shared_sources([(0.25, -1.0, side)]), device="cpu")
+    return bench.algorithmic_work(emr.pack_population(pop), q, emr)[0, 0]
+
+
+def test_cost_table_is_the_documented_one():
+    assert bench.ACT_FP32 == FP32 and bench.ACT_MUFU == MUFU
+    assert (bench.VAR_OPS, bench.BAND_OPS) == (4.5, 1.0) and bench.TILE_SIDE == 64
+
+
+def test_one_coordinate_output():
+    """sin(1.5 x2 + 0.2): one node of x alone (first-layer FMA + sin), once per tile column. A dead
+    hidden node adds nothing; on the incoming side x2 is the slot's coordinate: constant, no work."""
+    nodes = [(5, OUT, SIN, 0.2), (6, HID, TNH, 0.0)]
+    conns = [(X2, 5, 1.5), (Y2, 6, 1.0)]
+    F, M = work(nodes, conns, W.SIDE_OUT)
+    assert F == pytest.approx(SHARE * (1 + FP32[SIN]) + FILTER) and M == pytest.approx(SHARE * MUFU[SIN])
+    assert tuple(work(nodes, conns, W.SIDE_IN)) == (0.0, 0.0)
+
+
+def test_joint_output_of_both_coordinates():
+    """tanh(0.7 x2 - 1.2 y2): per query the x + y add and tanh; per tile column and row the two
+    first-layer products."""
+    F, M = work([(5, OUT, TNH, 0.0)], [(X2, 5, 0.7), (Y2, 5, -1.2)], W.SIDE_OUT)
+    assert F == pytest.approx(1 + FP32[TNH] + SHARE * 2 + FILTER) and M == pytest.approx(MUFU[TNH])
+
+
+def test_joint_node_fed_by_one_coordinate_nodes():
+    """sin(gauss(x2) + sigmoid(y2) + 0.5 x2): the gauss node (x) and the sigmoid node (y) are table
+    work, and so are the output's two first-layer products and its two one-coordinate sources;
+    per query only its add and sin."""
+    nodes = [(5, OUT, SIN, 0.0), (6, HID, GAU, 0.0), (7, HID, SIG, 0.0)]
+    conns = [(X2, 6, 1.0), (Y2, 7, 1.0), (6, 5, 1.0), (7, 5, 1.0), (X2, 5, 0.5)]
+    F, M = work(nodes, conns, W.SIDE_OUT)
+    table = (1 + FP32[GAU]) + (1 + FP32[SIG]) + (2 + 2)
+    assert F == pytest.approx(1 + FP32[SIN] + SHARE * table + FILTER)
+    assert M == pytest.approx(MUFU[SIN] + SHARE * (MUFU[GAU] + MUFU[SIG]))
+
+
+def test_joint_chain():
+    """abs(2 tanh(x2 + y2) + x2): two joint nodes; the output's edge from the joint tanh node is per
+    query work, its own x product table work."""
+    nodes = [(5, OUT, ABS, 0.0), (6, HID, TNH, 0.0)]
+    conns = [(X2, 6, 1.0), (Y2, 6, 1.0), (6, 5, 2.0), (X2, 5, 1.0)]
+    F, M = work(nodes, conns, W.SIDE_OUT)
+    assert F == pytest.approx((1 + FP32[TNH]) + (1 + 1 + FP32[ABS]) + SHARE * (2 + 2) + FILTER)
+    assert M == pytest.approx(MUFU[TNH])
+
+
+def test_constant_output_counts_nothing():
+    nodes = [(5, OUT, SIG, 0.3), (6, HID, SIN, 0.0)]
+    conns = [(X1, 6, 2.0), (6, 5, 1.0), (Y1, 5, -1.0)]
+    assert tuple(work(nodes, conns, W.SIDE_OUT)) == (0.0, 0.0)

@@ -462,13 +462,17 @@ emr_status emr_conn_types(const int32_t *idx, const int64_t *offsets, const emr_
  * clone) and slots, up to max_bytes (least recently used entries go first). A
  * genome is identified by its packed records, so any change to it misses.
  * Reuse does not change results: the device path is deterministic. Not
- * thread-safe: one call at a time per cache. */
+ * thread-safe: one call at a time per cache. Host memory only. create: *cache
+ * receives the new cache (NULL on failure); EMR_ERR_ARG (cache NULL),
+ * EMR_ERR_ALLOC. destroy: frees the cache and its entries (NULL is a no-op).
+ * clear: drops every entry and the counters, keeps max_bytes; EMR_ERR_ARG for
+ * NULL. */
 typedef struct emr_cache emr_cache;
 emr_status emr_cache_create(size_t max_bytes, emr_cache **cache);
 emr_status emr_cache_destroy(emr_cache *cache);
 emr_status emr_cache_clear(emr_cache *cache);
 /* Lookups that hit and missed since creation or the last clear, entries held
- * and their bytes. Any output may be NULL. */
+ * and their bytes. Any output may be NULL. Errors: EMR_ERR_ARG (cache NULL). */
 emr_status emr_cache_stats(const emr_cache *cache, int64_t *hits, int64_t *misses, int64_t *entries,
                            int64_t *bytes);
 

@@ -200,6 +200,12 @@ def test_cache_handle_host_only():
     c.clear()
     assert c.stats()["entries"] == 0
     del c
+    # the raw entry points' documented errors on NULL handles
+    L = emr.lib()
+    assert L.emr_cache_create(C.c_size_t(1 << 20), None) == emr.EMR_ERR_ARG
+    assert L.emr_cache_clear(None) == emr.EMR_ERR_ARG
+    assert L.emr_cache_stats(None, None, None, None, None) == emr.EMR_ERR_ARG
+    assert L.emr_cache_destroy(None) == emr.EMR_OK
 
 
 def test_discover_and_copy_reject_arguments_before_device_work():

@@ -248,3 +248,26 @@ def test_discover_and_copy_reject_arguments_before_device_work():
         with pytest.raises(emr.EmrError) as e:
             emr.copy_async(dst, src, 8, stream=st)
         assert e.value.status == emr.EMR_ERR_ARG
+
+
+def test_every_entry_point_rejects_zero_arguments():
+    """Every status-returning entry point checks its arguments before it reads a pointer or calls
+    CUDA: with every argument zero (null pointers, zero sizes and counts) it returns an argument or
+    range error, except where zero arguments are a valid call (index 0, destroying a null cache,
+    copying 0 bytes, the feedforward substrate configuration), which returns EMR_OK."""
+    L = emr.lib()
+    zero_ok = {"emr_index_to_ij", "emr_cache_destroy", "emr_copy_async", "emr_substrate_config"}
+    pointer_types = (C.c_void_p, C.c_char_p)
+    tested = 0
+    for name in sorted(declared_symbols()):
+        f = getattr(L, name)
+        if f.restype is not C.c_int32 or not f.argtypes:  # emr_strerror, emr_version
+            continue
+        args = [None if (t in pointer_types or issubclass(t, C._Pointer)) else t(0) for t in f.argtypes]
+        rc = f(*args)
+        if name in zero_ok:
+            assert rc == emr.EMR_OK, name
+        else:
+            assert rc in (emr.EMR_ERR_ARG, emr.EMR_ERR_RANGE), (name, rc)
+        tested += 1
+    assert tested >= 35

@@ -271,3 +271,17 @@ def test_every_entry_point_rejects_zero_arguments():
             assert rc in (emr.EMR_ERR_ARG, emr.EMR_ERR_RANGE), (name, rc)
         tested += 1
     assert tested >= 35
+
+
+def test_stream_workspace_holds_the_split_plane_and_two_chunks():
+    """emr_stream_workspace_size (host only): the resident split plane of every pair plus the
+    records and two chunk buffers, growing with the chunk and with the device list capacity; 5.3 GB
+    for the depth-13 configuration with the benchmark's chunk (2^26) and list capacity (2^24)."""
+    w = W.c5()
+    pack = emr.pack_population(w.pop)
+    q = emr.make_query(w.sources, device="cpu")
+    size = lambda chunk, cap: emr.stream_workspace_size(pack, q, emr.grid_build(w.D, chunk), cap)
+    split_plane = w.P * q.S * emr.grid_build(w.D).n_words * 4
+    big = size(1 << 26, 1 << 24)
+    assert split_plane < size(1 << 20, 1 << 20) < size(1 << 26, 1 << 20) < big
+    assert size(1 << 26, 1 << 20) < big and round(big / 1e9, 1) == 5.3

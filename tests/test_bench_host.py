@@ -71,3 +71,17 @@ def test_constant_output_counts_nothing():
     nodes = [(5, OUT, SIG, 0.3), (6, HID, SIN, 0.0)]
     conns = [(X1, 6, 2.0), (6, 5, 1.0), (Y1, 5, -1.0)]
     assert tuple(work(nodes, conns, W.SIDE_OUT)) == (0.0, 0.0)
+
+
+def test_launch_count_matches_the_profiled_launch_list():
+    """bench.py's gpu_launches claim for the 1000-genome depth-7 step equals the kernels per step
+    in the committed ncu launch list (profiles/launches_c2_pop1000_d7.md: launches over 8 steps)."""
+    import os
+    import types
+    path = os.path.join(os.path.dirname(bench.__file__), "profiles", "launches_c2_pop1000_d7.md")
+    rows = [l.split("|") for l in open(path) if l.startswith("| ") and not l.startswith("| kernel")]
+    per_step = sum(int(r[2]) for r in rows) / 8
+    w = W.c2(D=7, P=1000)
+    dsc = types.SimpleNamespace(pack=emr.pack_population(w.pop), grid=emr.grid_build(7),
+                                query=emr.make_query(w.sources, device="cpu"))
+    assert bench.launches_in_step(emr, dsc) == per_step == 13

@@ -85,3 +85,25 @@ def test_launch_count_matches_the_profiled_launch_list():
     dsc = types.SimpleNamespace(pack=emr.pack_population(w.pop), grid=emr.grid_build(7),
                                 query=emr.make_query(w.sources, device="cpu"))
     assert bench.launches_in_step(emr, dsc) == per_step == 13
+
+
+def test_reference_arm_prints_the_contract_line():
+    """bench.py --impl reference (the oracle on the host cores, a bounded sample of the same
+    workload) prints one JSON line with the benchmark's metric and the reference arm's keys."""
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(bench.__file__)
+    p = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--steps", "1",
+                        "--warmup", "1"], capture_output=True, text=True, timeout=600, cwd=root)
+    assert p.returncode == 0, p.stderr[-2000:]
+    lines = [l for l in p.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    j = json.loads(lines[0])
+    assert j["impl"] == "reference" and j["metric"] == bench.METRIC and j["unit"] == bench.UNIT
+    assert j["value"] > 0 and j["higher_is_better"] is True and j["steps"] == 1 and j["warmup"] == 1
+    assert j["cpu_baseline"]["kind"] == "oracle" and j["cpu_baseline"]["value"] == j["value"]
+    assert j["cpu_baseline"]["cores"] >= 1 and j["cpu_baseline"]["sample"]
+    assert j["e2e"] == {"value": j["value"], "unit": j["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    assert j["config"]["workload"] == "c2_xor_pop1000_d7"

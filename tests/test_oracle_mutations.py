@@ -37,6 +37,7 @@ C_PINS = [  # the quick pins of test_oracle_pins.py (parametrized pins over all 
         "test_constant_genome_keeps_nothing",
         "test_reflection_symmetry_of_x_only_genome",
         "test_in_side_equals_out_side_of_swapped_genome",
+        "test_per_genome_slots_address_like_shared_slots",
         "test_eq2_active_mask_by_recursion",
         "test_theorem1_single_genome",
     )]
@@ -87,6 +88,14 @@ MUTATIONS = {
                                 "if (side == 0) { in[0] = a; in[1] = b; in[2] = y; in[3] = x; }", C_PINS),
     "in_side_as_out_side": (C, "else { in[0] = x; in[1] = y; in[2] = a; in[3] = b; }",
                             "else { in[0] = a; in[1] = b; in[2] = x; in[3] = y; }", C_PINS),
+    # per-genome query slots (the hidden-to-hidden round)
+    "per_genome_slot_relative_to_range": (C, "            int64_t si = per_genome ? (int64_t)g * S + s : s;\n            double a",
+                                          "            int64_t si = per_genome ? (int64_t)gl * S + s : s;\n            double a",
+                                          C_PINS),
+    "unused_slots_evaluated": (C, "            if (per_genome && src_count && s >= src_count[g]) continue;\n            int64_t si",
+                               "            int64_t si", C_PINS),
+    "lazy_unused_slots_evaluated": (C, "        if (per_genome && src_count && s >= src_count[g]) continue;\n        int64_t si",
+                                    "        int64_t si", C_PINS),
     # CPPN evaluation
     "bias_dropped": (C, "double z = (double)G->bias[v];", "double z = 0.0;", C_PINS),
     "edge_weight_dropped": (C, "z += G->w[e] * val[s];", "z += val[s];", C_PINS),

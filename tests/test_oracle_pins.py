@@ -329,6 +329,36 @@ def test_in_side_equals_out_side_of_swapped_genome():
     assert np.array_equal(o["w"], i["w"]) and np.array_equal(o["keep_eager"], i["keep_eager"])
 
 
+def test_per_genome_slots_address_like_shared_slots():
+    """Per-genome query slots (a [P, S] slot table with a count per genome, as the hidden-to-hidden
+    round uses): over the genome range [1, 5), genome g's slot s is evaluated exactly like the same
+    point given as a shared slot, and a slot at or past the genome's count keeps nothing and holds
+    zeros; the lazy tree reads the same slots."""
+    pop = W.random_population(5, seed=31)
+    rng = np.random.default_rng(7)
+    P, S, D = 5, 3, 4
+    a = rng.uniform(-1, 1, (P, S)).astype(np.float32)
+    b = rng.uniform(-1, 1, (P, S)).astype(np.float32)
+    side = rng.integers(0, 2, (P, S)).astype(np.int32)
+    count = np.array([3, 1, 0, 2, 3], np.int32)
+    per = W.Sources(a=a, b=b, side=side, count=count)
+    r = oracle.discover(pop, per, D, 0.03, 0.3, g0=1, g1=5)
+    lz, _ = oracle.lazy(pop, per, D, 0.03, 0.3, g0=1, g1=5)
+    assert np.array_equal(lz, r["keep_gated"])
+    used = 0
+    for gl, g in enumerate(range(1, 5)):
+        for k in range(S):
+            if k < count[g]:
+                ref = oracle.discover(pop, W.shared_sources([(float(a[g, k]), float(b[g, k]), int(side[g, k]))]),
+                                      D, 0.03, 0.3, g0=g, g1=g + 1)
+                for f in ("w", "w_halo", "var", "bnd", "keep_eager", "keep_gated"):
+                    assert np.array_equal(r[f][gl, k], ref[f][0, 0]), (g, k, f)
+                used += 1
+            else:
+                assert not r["w"][gl, k].any() and not r["keep_eager"][gl, k].any() and not lz[gl, k].any()
+    assert used == 6
+
+
 # ---- brute force: re-evaluation at Eq. 1 coordinates ------------------------
 
 def test_discover_matches_direct_evaluation_at_grid_and_halo_points():

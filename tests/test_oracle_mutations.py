@@ -42,6 +42,7 @@ C_PINS = [  # the quick pins of test_oracle_pins.py (parametrized pins over all 
         "test_theorem1_single_genome",
     )]
 KEEP_AT_PINS = ["test_oracle_pins.test_keep_at_matches_whole_grid_decisions"]
+TYPE_PINS = ["test_types_oracle.*"]
 VARIANT_PINS = ["test_variants_oracle.*"]
 ASSEMBLY_PINS = ["test_assembly_oracle.*"]
 
@@ -112,6 +113,12 @@ MUTATIONS = {
     # decisions at individual positions (checked against the whole-grid definition)
     "keep_at_band_axes_mixed": (C, "double B = fmax(fmin(dt, db), fmin(dl, dr)), Be = 0.0,",
                                 "double B = fmax(fmin(dt, dl), fmin(db, dr)), Be = 0.0,", KEEP_AT_PINS),
+    # connection types (Section 6's taxonomy)
+    "types_ignore_the_query_side": (C, "    double xs = side == 0 ? a : x, ys = side == 0 ? b : y;   /* source */\n"
+                                       "    double xt = side == 0 ? x : a, yt = side == 0 ? y : b;   /* target */",
+                                    "    double xs = a, ys = b;\n    double xt = x, yt = y;", TYPE_PINS),
+    "lateral_typed_forward_in_types": (C, "if (ys < yt) return 0;", "if (ys <= yt) return 0;", TYPE_PINS),
+    "self_loop_typed_lateral": (C, "    if (xs == xt && ys == yt) return 3;\n", "", TYPE_PINS),
     # method variants (HyperNEAT weight scaling, subtree-leaf variance)
     "scaling_without_clamp": ("variants.py", "(np.minimum(a, 1.0) - thr) / (1.0 - thr)", "(a - thr) / (1.0 - thr)",
                               VARIANT_PINS),
@@ -206,7 +213,7 @@ def tmpdir_mut():
 def test_unmutated_oracle_passes_every_pin(tmpdir_mut):
     """The harness itself: an unchanged copy of the package fails no pin."""
     pkg = _package(tmpdir_mut, "unmutated")
-    assert _caught(pkg, C_PINS + KEEP_AT_PINS + VARIANT_PINS + ASSEMBLY_PINS) == []
+    assert _caught(pkg, C_PINS + KEEP_AT_PINS + TYPE_PINS + VARIANT_PINS + ASSEMBLY_PINS) == []
 
 
 @pytest.mark.parametrize("name", sorted(MUTATIONS))

@@ -15,7 +15,8 @@ Parity status of each oracle function (what pins it, in tests/test_oracle_pins.p
                             constant genomes, symmetry, Theorem 1 against the
                             lazy tree, a direct re-evaluation at sampled points,
                             the strict inequalities at exact ties, the band of
-                            genomes the halo mirrors at one edge. Planted
+                            genomes the halo mirrors at one edge, per-genome
+                            slots against the same points as shared slots. Planted
                             mistakes (tests/test_oracle_mutations.py) each fail
                             one of these pins.
   ora_lazy                  pinned: Theorem 1 (lazy subset of eager, lazy equal to

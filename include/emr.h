@@ -323,12 +323,16 @@ emr_status emr_stream_mode(const void *pack_host, const void *pack_dev, const em
  *    emr_eval_workspace_size reports must be <= EMR_STATIC_SCRATCH_BYTES);
  *    nothing is launched then.
  *  - The first call on a device looks up the array's device address
- *    (cudaGetSymbolAddress, with that device current) and caches it; make that
- *    first call before any stream capture.
+ *    (cudaGetSymbolAddress, with that device current) and caches it. With the
+ *    CUDA runtime's lazy module loading, that lookup may also be what loads
+ *    libemr's device code (and so the array) onto the device; make that first
+ *    call before any stream capture.
  *  - All calls on a device share the one array and it keeps the previous
- *    call's contents. Nothing in it needs to start at zero (every call writes
- *    each entry it reads), but calls whose work overlaps on the GPU (other
- *    streams, other host threads) race on it: serialise them.
+ *    call's contents. The one entry that must start at zero (the pair
+ *    schedule's completion counter) is cleared by each call on its stream;
+ *    every other entry is written before it is read. Calls whose work overlaps
+ *    on the GPU (other streams, other host threads) race on the array:
+ *    serialise them.
  * Errors: EMR_ERR_ARG, EMR_ERR_RANGE, EMR_ERR_CUDA. */
 #define EMR_STATIC_SCRATCH_BYTES (16u << 20)
 emr_status emr_eval_filter_noalloc(const void *pack_host, const void *pack_dev, const emr_query *q,

@@ -1,3 +1,4 @@
+import json
 import os
 import sys
 
@@ -21,3 +22,17 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+def pytest_terminal_summary(terminalreporter):
+    """The parity tests' exclusion counts per workload (ill-conditioned outputs, uncertain
+    decisions, kept entries); also written as JSON to $EMR_PARITY_REPORT when set."""
+    pu = sys.modules.get("parity_util")
+    if pu is None or not pu.REPORT:
+        return
+    for line in pu.report_lines():
+        terminalreporter.write_line(line)
+    path = os.environ.get("EMR_PARITY_REPORT")
+    if path:
+        with open(path, "w") as f:
+            json.dump(pu.REPORT, f, indent=1, sort_keys=True)

@@ -130,3 +130,77 @@ def test_reference_arm_under_torchrun_prints_from_rank_0_only():
     assert len(lines) == 1
     j = json.loads(lines[0])
     assert j["impl"] == "reference" and j["n_gpus"] == 2 and j["value"] > 0
+
+
+def survey(nodes, conns, side):
+    base = [(k, k, IDN, 0.0) for k in range(5)]
+    pop = W.population_from_lists([(base + nodes, [(s, d, w, True) for s, d, w in conns])])
+    q = emr.make_query(W.shared_sources([(0.25, -1.0, side)]), device="cpu")
+    return bench.survey_work(emr.pack_population(pop), q, emr)[0, 0]
+
+
+def test_survey_model_counts_every_node_at_every_position():
+    """The survey model (every varying node evaluated per query): tanh(2 x2 - y2 + h), h = sin(x2 + 0.3)
+    on the outgoing side: h has 1 varying in-connection + sin (4 FP32, 1 sin); the output 3 (x2, y2,
+    h) + tanh (3 FP32, ex2 + rcp); plus 3.25 + 8 of filter. On the incoming side nothing varies."""
+    nodes = [(5, OUT, TNH, 0.0), (6, HID, SIN, 0.0)]
+    conns = [(X2, 6, 1.0), (BIAS, 6, 0.3), (X2, 5, 2.0), (Y2, 5, -1.0), (6, 5, 1.0)]
+    F, ex2, rcp, sn = survey(nodes, conns, W.SIDE_OUT)
+    assert F == pytest.approx(1 + 4 + 3 + 3 + 3.25 + 8) and (ex2, rcp, sn) == (1, 1, 1)
+    assert tuple(survey(nodes, conns, W.SIDE_IN)) == (11.25, 0, 0, 0)
+
+
+def test_survey_roofline_takes_the_slower_pipe():
+    work = np.array([[[20.0, 1.0, 1.0, 0.0]]])
+    probe = {"ex2_Gops": 1e3, "rcp_Gops": 5e2, "sin_Gops": 5e2}
+    r = bench.survey_roofline(work, 1000, 152, probe, 1e-6)
+    t_fp32 = 20.0 * 1000 / (152 * 128 * 2070e6)
+    t_mufu = 1000 * (1 / 1e12 + 1 / 5e11)
+    assert r["t_fp32_ms"] == pytest.approx(t_fp32 * 1e3) and r["t_mufu_ms"] == pytest.approx(t_mufu * 1e3)
+    assert r["frac"] == pytest.approx(max(t_fp32, t_mufu) / 1e-6)
+
+
+def test_level_ij_inverts_the_oracle_numbering():
+    import oracle
+    rng = np.random.default_rng(3)
+    d = rng.integers(0, 10, 500)
+    i = np.array([rng.integers(0, 2 ** (k + 1)) for k in d])
+    j = np.array([rng.integers(0, 2 ** (k + 1)) for k in d])
+    p = [oracle.index(int(a), int(b), int(c)) for a, b, c in zip(d, i, j)]
+    dd, ii, jj = bench.level_ij(p)
+    assert np.array_equal(dd, d) and np.array_equal(ii, i) and np.array_equal(jj, j)
+
+
+class _FakeDiscovery:
+    """Lists held like emr.Discovery's (host tensors), filled from the oracle."""
+
+    def __init__(self, w, keep, ws):
+        import torch
+        from types import SimpleNamespace
+        rows = keep.reshape(-1, keep.shape[-1])
+        idx = [np.flatnonzero(r) for r in rows]
+        off = np.concatenate([[0], np.cumsum([len(x) for x in idx])])
+        self.grid = SimpleNamespace(n_total=keep.shape[-1])
+        self.offsets = torch.from_numpy(off.astype(np.int64))
+        self.idx = torch.from_numpy(np.concatenate(idx).astype(np.int32))
+        self.w = torch.from_numpy(np.concatenate([ws.reshape(len(rows), -1)[r][x] for r, x in enumerate(idx)])
+                                  .astype(np.float32))
+
+
+def test_lists_parity_counts_agreement_and_planted_errors():
+    """bench.lists_parity on oracle-made lists: no mismatch; a dropped entry and a wrong weight are
+    each counted."""
+    import oracle
+    w = W.c2(D=4, P=6)
+    r = oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, fields=("keep_eager", "unc_eager", "w"))
+    ora = {"keep_eager": r["keep_eager"], "unc_eager": r["unc_eager"]}
+    fake = _FakeDiscovery(w, r["keep_eager"], r["w"])
+    rep = bench.lists_parity(w, fake, ora, w.P)
+    assert rep["mismatches"] == 0 and rep["weight_mismatches"] == 0 and rep["kept"] > 0
+    fake.w[0] += 0.01
+    assert bench.lists_parity(w, fake, ora, w.P)["weight_mismatches"] == 1
+    keep = r["keep_eager"].copy()
+    k = np.flatnonzero(keep.reshape(-1))[0]
+    keep.reshape(-1)[k] = 0
+    fake = _FakeDiscovery(w, keep, r["w"])
+    assert bench.lists_parity(w, fake, ora, w.P)["mismatches"] == 1

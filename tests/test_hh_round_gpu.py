@@ -7,9 +7,10 @@ import pytest
 import torch
 
 import oracle
+from hh_sources import round2_workload
 from paper_2608_27612_gb300 import emr
 from paper_2608_27612_gb300 import workloads as W
-from parity_util import check_bits, check_lists, unpack_planes
+from parity_util import assert_stored, check_bits, check_lists, oracle_blocks, record, unpack_planes
 
 pytestmark = pytest.mark.gpu
 
@@ -21,63 +22,40 @@ def fused(w):
     return dsc, dsc.lists()
 
 
-def dij(p, D):
-    """Depth and grid indices of a global index (depth-major, Morton within a depth)."""
-    d = 0
-    while (4 ** (d + 2) - 4) // 3 <= p:
-        d += 1
-    m = p - (4 ** (d + 1) - 4) // 3
-    i = sum(((m >> (2 * k)) & 1) << k for k in range(d + 1))
-    j = sum(((m >> (2 * k + 1)) & 1) << k for k in range(d + 1))
-    return d, i, j
-
-
-def hidden_sources(w1, keep, S=256):
-    """Per genome: the distinct positions its outgoing round-1 slots keep, ascending, first S,
-    each queried outgoing from its grid coordinates (Eq. 1)."""
-    P, S1 = w1.P, w1.S
-    a = np.zeros((P, S), np.float32); b = np.zeros((P, S), np.float32)
-    side = np.zeros((P, S), np.int32); count = np.zeros(P, np.int32)
-    for g in range(P):
-        rows = [keep[g, s] for s in range(S1) if int(w1.sources.side[s]) == W.SIDE_OUT]
-        idx = np.flatnonzero(np.any(rows, axis=0))[:S]
-        count[g] = len(idx)
-        for k, p in enumerate(idx):
-            d, i, j = dij(int(p), w1.D)
-            a[g, k] = (2 * i + 1) / 2.0 ** (d + 1) - 1.0
-            b[g, k] = (2 * j + 1) / 2.0 ** (d + 1) - 1.0
-    return W.Sources(a=a, b=b, side=side, count=count)
-
-
-def test_round1_depth8_against_oracle():
+def test_round1_depth8_all_genomes_against_oracle():
+    """All 150 genomes x 12 slots at depth 8 (629 M decisions)."""
     w = W.c4_round1()
     dsc, lists = fused(w)
-    mask = unpack_planes(dsc.mask.cpu().numpy(), dsc.grid)
-    n_gen = 6
-    ora = oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, g1=n_gen,
-                          fields=("w", "w_err", "keep_eager", "unc_eager"))
-    ora = {k: v.reshape(-1, v.shape[-1]) for k, v in ora.items()}
-    n = n_gen * w.S
-    check_bits(mask[:n], ora["keep_eager"], ora["unc_eager"])
-    check_lists(lists[:n], mask[:n], ora["w"], ora["w_err"])
+    planes = dsc.mask.cpu().numpy()
+    S = w.S
+    for g0, g1, ora in oracle_blocks(w, 10):
+        rows = slice(g0 * S, g1 * S)
+        mask = unpack_planes(planes[rows], dsc.grid)
+        b = check_bits(mask, ora["keep_eager"], ora["unc_eager"])
+        l = check_lists(lists[rows], mask, ora["w"], ora["w_err"])
+        record("c4_r1_d8", b, l)
+    assert_stored("c4_r1_d8")
 
 
 def test_round2_hidden_sources_against_oracle_and_stream():
-    w1 = W.c4_round1(P=8)
+    """Round 2 of the first 8 genomes (of 40) whose round 1, by the oracle, found hidden nodes: those
+    nodes as per-genome slots (up to 256 per genome), every genome compared; then the same round
+    streamed in chunks."""
+    w1 = W.c4_round1(P=40)
     r1 = oracle.discover(w1.pop, w1.sources, w1.D, w1.theta, w1.band, fields=("keep_eager",))
-    src2 = hidden_sources(w1, r1["keep_eager"], S=256)
-    assert src2.count.max() > 0
-    w2 = W.Workload("c4_round2", w1.pop, src2, w1.D, w1.theta, w1.band)
+    w2 = round2_workload(w1, r1["keep_eager"], 8)
+    src2 = w2.sources
+    assert w2.P == 8 and src2.count.min() > 0 and src2.count.max() == 256
     dsc, lists2 = fused(w2)
-    mask = unpack_planes(dsc.mask.cpu().numpy(), dsc.grid)
+    planes = dsc.mask.cpu().numpy()
     S = src2.S
-    g = int(np.argmax(src2.count > 0))
-    ora = oracle.discover(w2.pop, src2, w2.D, w2.theta, w2.band, g0=g, g1=g + 1,
-                          fields=("w", "w_err", "keep_eager", "unc_eager"))
-    ora = {k: v.reshape(-1, v.shape[-1]) for k, v in ora.items()}
-    rows = slice(g * S, (g + 1) * S)
-    check_bits(mask[rows], ora["keep_eager"], ora["unc_eager"])
-    check_lists(lists2[rows], mask[rows], ora["w"], ora["w_err"])
+    for g0, g1, ora in oracle_blocks(w2, 1):
+        rows = slice(g0 * S, g1 * S)
+        mask = unpack_planes(planes[rows], dsc.grid)
+        b = check_bits(mask, ora["keep_eager"], ora["unc_eager"])
+        l = check_lists(lists2[rows], mask, ora["w"], ora["w_err"])
+        record("c4_r2_d8_g8", b, l)
+    assert_stored("c4_r2_d8_g8")
     for r in range(w2.P * S):
         if r % S >= src2.count[r // S]:
             assert len(lists2[r][0]) == 0

@@ -1,17 +1,22 @@
 """GPU parity: libemr's kernels (through the C ABI) against the float64 oracle.
 
-Bars: CPPN outputs within 1e-5 + 1e-4 |oracle| (positions whose fp32 error
-bound exceeds that are counted as ill-conditioned); masks and compacted indices
-bit-exact wherever the oracle's decision is certain (uncertain ones counted).
+Bars: CPPN outputs within max(1e-5 + 1e-4 |oracle|, the oracle's fp32 error bound)
+(outputs whose bound exceeds the plain tolerance are counted as ill-conditioned);
+masks and compacted indices bit-exact wherever the oracle's decision is certain
+(uncertain ones counted). The single-genome, 1000-genome (depths 5 and 7) and
+wide-input workloads are compared over every genome; their counts must stay within
+the oracle's stored counts.
 """
 import numpy as np
 import pytest
 import torch
 
 import oracle
+import special_genomes as SG
 from paper_2608_27612_gb300 import emr
 from paper_2608_27612_gb300 import workloads as W
-from parity_util import check_bits, check_lists, check_outputs, full_parity, run_gpu, run_oracle, unpack_planes
+from parity_util import (assert_stored, check_bits, check_lists, check_outputs, full_parity, mask_from_lists,
+                         oracle_blocks, record, run_gpu, run_oracle, unpack_planes)
 
 pytestmark = pytest.mark.gpu
 X1, Y1, X2, Y2, BIAS, HID, OUT = range(7)
@@ -19,16 +24,17 @@ IDN, SIG, TNH, GAU, SIN, ABS = range(6)
 
 
 def test_single_genome_depth4_both_modes():
-    for mode in (emr.EMR_EAGER, emr.EMR_GATED):
-        _, _, rep = full_parity(W.c1(), mode)
+    for mode, name in ((emr.EMR_EAGER, "c1_d4_eager"), (emr.EMR_GATED, "c1_d4_gated")):
+        _, _, rep = full_parity(W.c1(), mode, name=name)
         assert rep["out"]["ill_conditioned"] == 0
+        assert_stored(name)
 
 
 def test_population_depth5_all_genomes():
     w = W.c2(D=5)
-    _, ora, rep = full_parity(w)
+    _, ora, rep = full_parity(w, name="c2_d5")
     assert rep["kept"] > 0
-    print("c2 d5:", rep)
+    assert_stored("c2_d5")
 
 
 def test_population_depth5_gated_matches_lazy_tree():
@@ -40,69 +46,47 @@ def test_population_depth5_gated_matches_lazy_tree():
     check_bits(gpu["mask_f"], lz, ora["unc_gated"], "gated vs lazy")
 
 
-def test_wide_input_depth6_subset():
+def test_wide_input_depth6_all_genomes():
+    """All 256 genomes x 33 slots: materialised outputs, fused and unfused masks, lists."""
     w = W.c3(D=6)
     gpu = run_gpu(w, unfused=True, fused=True)
-    n_gen = 12
-    ora = run_oracle(w, g1=n_gen)
-    n = ora["w"].shape[0]
-    check_outputs(gpu["out"][:n], ora["w"], ora["w_err"])
-    check_bits(gpu["mask_f"][:n], ora["keep_eager"], ora["unc_eager"])
-    check_lists(gpu["lists_f"][:n], gpu["mask_f"][:n], ora["w"], ora["w_err"])
     assert np.array_equal(gpu["mask_u"], gpu["mask_f"])
+    S = w.S
+    for g0, g1, ora in oracle_blocks(w, 32):
+        rows = slice(g0 * S, g1 * S)
+        o = check_outputs(gpu["out"][rows], ora["w"], ora["w_err"])
+        b = check_bits(gpu["mask_f"][rows], ora["keep_eager"], ora["unc_eager"])
+        l = check_lists(gpu["lists_f"][rows], gpu["mask_f"][rows], ora["w"], ora["w_err"])
+        record("c3_d6", o, b, l)
+    assert_stored("c3_d6")
 
 
-def test_bench_configuration_depth7_sampled():
-    """The benchmark's workload (1000 genomes, 4 slots, depth 7) in its launch
-    configuration: full masks and lists for 16 genomes, outputs at sampled
-    positions of every genome."""
+def test_bench_configuration_depth7_all_genomes():
+    """The benchmark's workload (1000 genomes, 4 slots, depth 7) over every genome: the
+    materialised outputs (emr_eval), and the keep decisions and lists of the benchmark
+    step's own launch path (emr_eval_prepare + emr_eval_filter_tiles + emr_select)."""
     w = W.c2(D=7)
-    gpu = run_gpu(w, unfused=True, fused=True)
-    ora = run_oracle(w, g1=16)
-    n = ora["w"].shape[0]
-    check_outputs(gpu["out"][:n], ora["w"], ora["w_err"])
-    check_bits(gpu["mask_f"][:n], ora["keep_eager"], ora["unc_eager"])
-    check_lists(gpu["lists_f"][:n], gpu["mask_f"][:n], ora["w"], ora["w_err"])
-    assert np.array_equal(gpu["mask_u"], gpu["mask_f"])
-    rng = np.random.default_rng(7)
-    g = emr.grid_build(7)
-    for gi in rng.choice(w.P, 40, replace=False):
-        for s in range(w.S):
-            pos = rng.integers(0, g.n_total, 64)
-            ins = []
-            for p in pos:
-                d, i, j = emr.index_to_ij(int(p))
-                x, y = (2 * i + 1) / 2 ** (d + 1) - 1, (2 * j + 1) / 2 ** (d + 1) - 1
-                a, b = float(w.sources.a[s]), float(w.sources.b[s])
-                ins.append([a, b, x, y, 1.0] if w.sources.side[s] == W.SIDE_OUT else [x, y, a, b, 1.0])
-            ref, err = oracle.cppn(w.pop, int(gi), np.array(ins))
-            check_outputs(gpu["out"][gi * w.S + s, pos], ref, err)
-    # the benchmark step's own path (emr_eval_filter_tiles + emr_select): the same lists for every pair,
-    # and its keep decisions at sampled positions of every genome against the oracle's
-    dsc = gpu["dsc"]
-    dsc.idx.zero_(); dsc.w.zero_()
+    dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, emr.EMR_EAGER, materialise=True)
+    g = dsc.grid
+    dsc.run_unfused()
+    torch.cuda.synchronize()
+    out = dsc.out.cpu().numpy()
+    mask_u = unpack_planes(dsc.mask.cpu().numpy(), g)
+    dsc.idx.zero_(); dsc.w.zero_(); dsc.counts.zero_(); dsc.offsets.zero_()
     dsc.run_select()
     torch.cuda.synchronize()
     sel = dsc.lists()
-    for (ri, rw), (si, sw) in zip(gpu["lists_f"], sel):
-        assert np.array_equal(ri, si) and np.array_equal(rw.view(np.uint32), sw.view(np.uint32))
-    n_checked = 0
-    for gi in rng.choice(w.P, 60, replace=False):
-        for s in range(w.S):
-            r = gi * w.S + s
-            kept = sel[r][0]
-            # every kept position, plus random others
-            pos = np.unique(np.concatenate([kept[:32], rng.integers(0, g.n_total, 32)])).astype(np.int64)
-            d = np.zeros(len(pos), np.int32); ii = np.zeros(len(pos), np.int64); jj = np.zeros(len(pos), np.int64)
-            for k, p in enumerate(pos):
-                d[k], ii[k], jj[k] = emr.index_to_ij(int(p))
-            ko = oracle.keep_at(w.pop, int(gi), float(w.sources.a[s]), float(w.sources.b[s]),
-                                int(w.sources.side[s]), w.D, w.theta, w.band, w.w_min, d, ii, jj)
-            ok = ko["unc"] == 0
-            got = np.isin(pos, kept)
-            assert np.array_equal(got[ok], ko["keep"][ok].astype(bool)), "pair %d" % r
-            n_checked += int(ok.sum())
-    assert n_checked > 8000
+    S = w.S
+    for g0, g1, ora in oracle_blocks(w, 100):
+        rows = slice(g0 * S, g1 * S)
+        o = check_outputs(out[rows], ora["w"], ora["w_err"])
+        mask = mask_from_lists(sel[rows], g.n_total)
+        assert np.array_equal(mask, mask_u[rows]), "genomes %d..%d: step lists differ from the unfused mask" % (g0, g1)
+        b = check_bits(mask, ora["keep_eager"], ora["unc_eager"])
+        l = check_lists(sel[rows], mask, ora["w"], ora["w_err"])
+        record("c2_d7", o, b, l)
+    tot = assert_stored("c2_d7")
+    assert tot["entries"] == int(dsc.offsets[-1]) > 0
 
 
 def test_linear_worked_example_keeps_grid3():
@@ -118,48 +102,36 @@ def test_linear_worked_example_keeps_grid3():
 
 
 def test_edge_cases_small_depths_constant_and_hidden_free_genomes():
-    const = ([(k, k, IDN, 0.0) for k in range(5)] + [(5, OUT, SIG, 0.3)], [(X1, 5, 1.0, True)])
-    nohid = ([(k, k, IDN, 0.0) for k in range(5)] + [(5, OUT, SIN, 0.0)],
-             [(X2, 5, 3.0, True), (Y2, 5, -2.0, True), (BIAS, 5, 0.5, True)])
-    rnd = W.random_population(6, seed=9)
-    pop = W.population_from_lists([const, nohid] + [rnd.genome(k) for k in range(6)])
-    src = W.shared_sources([(0.0, -1.0, W.SIDE_OUT), (0.5, 1.0, W.SIDE_IN)])
     for D in (0, 1, 2, 3):
-        w = W.Workload("edge", pop, src, D, 0.03, 0.3)
-        full_parity(w)
+        w = SG.edge_cases(D)
+        full_parity(w, name=w.name)
+        assert_stored(w.name)
 
 
 def test_every_kernel_class_including_interpreter():
     """Genomes with 0..30 varying nodes: the constant, dense-4, dense-8, dense-12
     and interpreter (more than 12 varying nodes) classes in one population."""
-    big = W.random_population(24, seed=31, h_lo=14, h_hi=30, e_max=120)
-    small = W.random_population(40, seed=32, h_lo=0, h_hi=12, e_max=40)
-    pop = W.population_from_lists([big.genome(k) for k in range(24)] + [small.genome(k) for k in range(40)])
-    h, gs, _, _ = emr.pack_records(emr.pack_population(pop))
-    assert gs["n_varying"][:, 0].max() > 12 and (gs["n_varying"][:, 0] == 0).any()
-    src = W.shared_sources([(-1.0, -1.0, W.SIDE_OUT), (0.0, 1.0, W.SIDE_IN)])
     for D in (4, 6):
-        w = W.Workload("classes", pop, src, D, 0.03, 0.3)
-        full_parity(w)
+        w = SG.kernel_classes(D)
+        if D == 4:
+            h, gs, _, _ = emr.pack_records(emr.pack_population(w.pop))
+            assert gs["n_varying"][:, 0].max() > 12 and (gs["n_varying"][:, 0] == 0).any()
+        full_parity(w, name=w.name)
+        assert_stored(w.name)
 
 
 def test_weight_filter_and_gated_mode():
-    w = W.c2(D=5, P=100)
-    w.w_min = 0.1
-    full_parity(w, emr.EMR_EAGER)
-    full_parity(w, emr.EMR_GATED)
+    w = SG.weight_filter()
+    for mode, name in ((emr.EMR_EAGER, w.name + "_eager"), (emr.EMR_GATED, w.name + "_gated")):
+        full_parity(w, mode, name=name)
+        assert_stored(name)
 
 
 def test_per_genome_slots_with_counts():
-    pop = W.random_population(5, seed=12)
-    rng = np.random.default_rng(4)
-    S = 6
-    a = rng.uniform(-1, 1, (5, S)).astype(np.float32)
-    b = rng.uniform(-1, 1, (5, S)).astype(np.float32)
-    side = rng.integers(0, 2, (5, S)).astype(np.int32)
-    cnt = np.array([6, 0, 3, 1, 6], np.int32)
-    w = W.Workload("pergenome", pop, W.Sources(a=a, b=b, side=side, count=cnt), 4, 0.03, 0.3)
-    gpu, ora, _ = full_parity(w)
+    w = SG.per_genome_slots()
+    cnt, S = w.sources.count, w.S
+    gpu, ora, _ = full_parity(w, name=w.name)
+    assert_stored(w.name)
     for g in range(5):
         for s in range(cnt[g], S):
             assert gpu["mask_f"][g * S + s].sum() == 0 and len(gpu["lists_f"][g * S + s][0]) == 0

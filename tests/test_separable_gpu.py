@@ -17,66 +17,8 @@ import torch
 
 from paper_2608_27612_gb300 import emr
 from paper_2608_27612_gb300 import workloads as W
-from parity_util import full_parity
-
-X1, Y1, X2, Y2, BIAS, HID, OUT = range(7)
-IDN, SIG, TNH, GAU, SIN, ABS = range(6)
-
-
-def _genome(hidden, out_act, conns):
-    """hidden: [(id, act)], output id 5; conns: [(src, dst, w)] (all enabled)."""
-    nodes = [(k, k, IDN, 0.0) for k in range(5)] + [(5, OUT, out_act, 0.1)]
-    nodes += [(i, HID, a, 0.05 * i) for i, a in hidden]
-    return nodes, [(s, d, w, True) for s, d, w in conns]
-
-
-def _chain(n_joint):
-    """n_joint joint nodes in a chain (the output last), each fed by x2, y2 and earlier nodes."""
-    acts = [SIN, TNH, GAU, SIG, ABS, IDN, SIN, TNH]
-    ids = list(range(6, 6 + n_joint - 1)) + [5]
-    conns = []
-    for k, v in enumerate(ids):
-        conns += [(X2, v, 0.7 + 0.1 * k), (Y2, v, -0.5 + 0.2 * k)]
-        if k >= 1:
-            conns.append((ids[k - 1], v, 0.9))
-        if k >= 3:
-            conns.append((ids[k - 3], v, -0.6))
-    hidden = [(v, acts[k % len(acts)]) for k, v in enumerate(ids[:-1])]
-    return _genome(hidden, acts[(n_joint - 1) % len(acts)], conns)
-
-
-def separable_population():
-    g = []
-    # x only: a chain of nodes of x2 alone (one table row each), filtered per column
-    g.append(_genome([(6, SIN), (7, TNH)], SIG, [(X2, 6, 3.0), (BIAS, 6, 0.2), (6, 7, 2.0), (X2, 7, -0.5),
-                                                (7, 5, 1.5)]))
-    # y only
-    g.append(_genome([(6, GAU)], TNH, [(Y2, 6, 2.0), (6, 5, 1.0), (Y2, 5, 0.7)]))
-    # joint output fed by an x node, a y node and x directly
-    g.append(_genome([(6, SIN), (7, SIG)], TNH, [(X2, 6, 5.0), (Y2, 7, 4.0), (6, 5, 1.0), (7, 5, 1.0),
-                                                 (X2, 5, 0.5)]))
-    # joint only through its sources (no grid input of its own)
-    g.append(_genome([(6, SIN), (7, GAU)], ABS, [(X2, 6, 3.0), (Y2, 7, 2.0), (6, 5, 1.0), (7, 5, -1.0)]))
-    # joint on the incoming side (x1, y1), x only on the outgoing side (x2)
-    g.append(_genome([(6, SIN), (7, GAU), (8, SIG)], IDN,
-                     [(X1, 6, 3.0), (Y1, 6, 2.0), (X2, 6, 1.0), (6, 7, 1.0), (X1, 7, 1.0), (Y1, 8, 1.0),
-                      (7, 5, 1.0), (8, 5, -1.0), (6, 5, 1.0)]))
-    # steep joint and steep x-only outputs: their tiles pass the band screen at depths 5 and 6
-    g.append(_genome([], SIN, [(X2, 5, 40.0), (Y2, 5, 30.0)]))
-    g.append(_genome([], SIN, [(X2, 5, 50.0)]))
-    g.append(_genome([(6, SIN)], GAU, [(Y2, 6, 45.0), (6, 5, 1.5)]))
-    # parallel connections (0.5 + 0.25 into the output; x2 twice into 6) and a cancelling pair (7 drops out)
-    g.append(_genome([(6, SIG), (7, SIN)], TNH, [(X2, 6, 1.0), (X2, 6, 0.5), (6, 5, 0.5), (Y2, 7, 1.0),
-                                                 (7, 5, 1.0), (6, 5, 0.25), (7, 5, -1.0)]))
-    # 6 and 8 joint nodes (their own kernel classes) and 14 (above the dense limit: the interpreter)
-    g += [_chain(6), _chain(8), _chain(14)]
-    return W.population_from_lists(g)
-
-
-def _workload(D=6):
-    src = W.shared_sources([(0.0, -1.0, W.SIDE_OUT), (0.3, 1.0, W.SIDE_IN), (-0.5, -1.0, W.SIDE_OUT)])
-    return W.Workload("separable_d%d" % D, separable_population(), src, D, 0.03, 0.3)
-
+from parity_util import assert_stored, full_parity
+from special_genomes import separable as _workload
 
 def test_classes_cover_every_case():
     """The population reaches the one-coordinate, joint, 6-, 8-joint and interpreter classes (host
@@ -95,7 +37,9 @@ def test_classes_cover_every_case():
 @pytest.mark.parametrize("mode", [emr.EMR_EAGER, emr.EMR_GATED])
 def test_separable_population_parity(mode):
     w = _workload()
-    gpu, ora, rep = full_parity(w, mode)
+    name = "separable_d6_" + ("eager" if mode == emr.EMR_EAGER else "gated")
+    gpu, ora, rep = full_parity(w, mode, name=name)
+    assert_stored(name)
     # the steep genomes keep positions at depths 5 and 6 through the band test
     g = gpu["dsc"].grid
     wo = list(g.word_off)
@@ -120,7 +64,8 @@ def test_separable_population_depth7():
     """Depth 7 (22 tiles per pair, the pyramid tile included): outputs, halo, planes and lists against
     the oracle, and the selection path's lists equal to the fused lists bit for bit."""
     w = _workload(D=7)
-    gpu, ora, rep = full_parity(w, emr.EMR_EAGER)
+    gpu, ora, rep = full_parity(w, emr.EMR_EAGER, name="separable_d7_eager")
+    assert_stored("separable_d7_eager")
     assert rep["kept"] > 0
     dsc = gpu["dsc"]
     dsc.idx.zero_(); dsc.w.zero_()

@@ -1,14 +1,15 @@
 """emr_eval_filter_noalloc: the fused evaluation for callers that cannot
 allocate device memory (its scratch is a static array inside libemr). Checked
 through the C ABI against emr_eval_prepare + emr_eval_filter on two calls in a
-row; collected last so that a failure here never hides another test."""
+row. Both run the same specialisation and tile kernels on the same inputs, so the
+check is exact equality (planes and every output word), not a tolerance. The
+file is collected last so that a failure here never hides another test."""
 import numpy as np
 import pytest
 import torch
 
 from paper_2608_27612_gb300 import emr
 from paper_2608_27612_gb300 import workloads as W
-from parity_util import check_outputs
 
 pytestmark = pytest.mark.gpu
 
@@ -34,8 +35,7 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls():
         torch.cuda.synchronize()
         assert torch.equal(split, split_ref), "call %d: split plane differs" % call
         assert torch.equal(band_bits, band_ref), "call %d: band plane differs" % call
-        ref = out_ref.cpu().numpy().astype(np.float64)
-        check_outputs(out.cpu().numpy(), ref, np.zeros_like(ref), "call %d outputs" % call)
+        assert torch.equal(out.view(torch.int32), out_ref.view(torch.int32)), "call %d: outputs differ" % call
         assert torch.equal(out != 0, passed)
 
 

@@ -11,7 +11,7 @@ import oracle
 from paper_2608_27612_gb300 import emr
 from paper_2608_27612_gb300 import workloads as W
 from parity_util import check_bits, unpack_planes
-from test_hh_round_gpu import hidden_sources
+from hh_sources import hidden_sources
 
 pytestmark = pytest.mark.gpu
 

@@ -162,6 +162,26 @@ emr_status emr_pack_population(int32_t P, const int64_t *node_ptr, const int32_t
                                const float *conn_w, const uint8_t *conn_enabled, void *buf, size_t cap,
                                size_t *used, int32_t *bad_genome);
 
+/* Genome ranges. The packer reads genome g through node_ptr[g] and conn_ptr[g]
+ * as absolute offsets into the node and connection arrays, so genomes
+ * [g0, g1) of a population are packed on their own by passing P = g1 - g0,
+ * node_ptr + g0 and conn_ptr + g0 (the other arrays unchanged): the blob then
+ * holds those genomes as genomes 0 .. g1 - g0 - 1. With per-genome query slots,
+ * the query of such a range is rows g0 .. g1 - 1 of the slot arrays. */
+
+/* Population-parallel split (Section 3, Table 1: the CPPN query, variance and
+ * mask stages are O(4^D / P) work over the population): n_parts contiguous
+ * genome ranges of balanced estimated cost for this pack and query. A pair's
+ * cost is the packer's per-query work estimate of its genome on the slot's
+ * query side plus the filter's per-query work; constant-output pairs and unused
+ * per-genome slots count 1. Writes g_begin[0 .. n_parts] (host int32):
+ * part k is genomes [g_begin[k], g_begin[k+1]), g_begin[0] = 0,
+ * g_begin[n_parts] = P, non-decreasing (a part may be empty when n_parts > P).
+ * Concatenating the parts' connection lists in part order gives the lists of
+ * the whole population (pair r = g * S + s). Host only.
+ * Errors: EMR_ERR_ARG (null pointer, n_parts <= 0, bad side, not a pack). */
+emr_status emr_partition_genomes(const void *pack_host, const emr_query *q, int32_t n_parts, int32_t *g_begin);
+
 /* Summary of a packed blob: population size and, per query side, the largest
  * number of varying nodes. Any output pointer may be NULL. */
 emr_status emr_pack_info(const void *pack_host, int32_t *P, int32_t *max_varying_out,

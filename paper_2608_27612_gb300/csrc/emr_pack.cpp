@@ -555,6 +555,44 @@ emr_status emr_pack_info(const void* pack_host, int32_t* P, int32_t* max_varying
   return EMR_OK;
 }
 
+// Contiguous genome ranges of balanced cost for population-parallel work
+// (Table 1: the CPPN query, variance and mask stages split over the
+// population). A pair's weight is its packed per-query work estimate plus the
+// filter's per-query work; a pair whose output is constant over the grid, or an
+// unused per-genome slot, weighs 1 (its tiles are only cleared).
+emr_status emr_partition_genomes(const void* pack_host, const emr_query* q, int32_t n_parts, int32_t* g_begin) {
+  if (!pack_host || !q || q->S <= 0 || !q->side_host || n_parts <= 0 || !g_begin) return EMR_ERR_ARG;
+  const PackHeader* h = pack_header(pack_host);
+  if (h->magic != kPackMagic || h->version != kPackVersion || h->P <= 0) return EMR_ERR_ARG;
+  const PackGenome* gt =
+      reinterpret_cast<const PackGenome*>(static_cast<const uint8_t*>(pack_host) + h->off_genomes);
+  constexpr uint64_t kFilterWork = 6;  // variance and band screen per query, in the cost estimate's units
+  const int32_t P = h->P, S = q->S;
+  std::vector<uint64_t> prefix(size_t(P) + 1, 0);
+  for (int32_t g = 0; g < P; g++) {
+    uint64_t w = 0;
+    for (int32_t s = 0; s < S; s++) {
+      const int64_t si = q->per_genome ? int64_t(g) * S + s : s;
+      const int32_t side = q->side_host[si];
+      if (side != EMR_SIDE_OUT && side != EMR_SIDE_IN) return EMR_ERR_ARG;
+      const bool unused = q->per_genome && q->count_host && s >= q->count_host[g];
+      w += (unused || gt[g].n_varying[side] == 0) ? 1 : uint64_t(gt[g].cost[side]) + kFilterWork;
+    }
+    prefix[size_t(g) + 1] = prefix[size_t(g)] + w;
+  }
+  const uint64_t total = prefix[size_t(P)];
+  g_begin[0] = 0;
+  for (int32_t k = 1; k < n_parts; k++) {
+    // the boundary nearest to k / n_parts of the total, never before the previous one
+    const uint64_t target = total / uint64_t(n_parts) * uint64_t(k) + total % uint64_t(n_parts) * uint64_t(k) / uint64_t(n_parts);
+    int32_t g = int32_t(std::lower_bound(prefix.begin(), prefix.end(), target) - prefix.begin());
+    if (g > 0 && target - prefix[size_t(g) - 1] < prefix[size_t(g)] - target) g--;
+    g_begin[k] = std::max(std::min(g, P), g_begin[k - 1]);
+  }
+  g_begin[n_parts] = P;
+  return EMR_OK;
+}
+
 const char* emr_strerror(emr_status s) {
   switch (s) {
     case EMR_OK: return "ok";

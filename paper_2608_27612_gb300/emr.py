@@ -61,6 +61,7 @@ def lib() -> C.CDLL:
             "emr_pack_size": [i32, vp, vp, vp],
             "emr_pack_population": [i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp, vp],
             "emr_pack_info": [vp, vp, vp, vp],
+            "emr_partition_genomes": [vp, vp, i32, vp],
             "emr_eval_workspace_size": [vp, vp, vp],
             "emr_eval_prepare": [vp, vp, vp, vp, sz, vp],
             "emr_eval": [vp, vp, vp, vp, vp, vp, sz, vp],
@@ -162,21 +163,34 @@ def _pop_ptrs(pop):
     return cache[1]
 
 
-def pack_size(pop) -> int:
+def _range_ptrs(pop, genomes):
+    """P and the ten array addresses for genomes [g0, g1) of pop (the whole population when
+    genomes is None): node_ptr and conn_ptr offset to g0, the other arrays unchanged."""
+    ptr = _pop_ptrs(pop)
+    if genomes is None:
+        return pop.P, ptr
+    g0, g1 = int(genomes[0]), int(genomes[1])
+    if not 0 <= g0 < g1 <= pop.P:
+        raise ValueError("genome range [%d, %d) outside [0, %d)" % (g0, g1, pop.P))
+    return g1 - g0, (ptr[0] + 8 * g0,) + ptr[1:5] + (ptr[5] + 8 * g0,) + ptr[6:]
+
+
+def pack_size(pop, genomes=None) -> int:
     """Upper bound of the packed blob's bytes for a workloads.Population (emr_pack_size)."""
     n = C.c_size_t()
-    ptr = _pop_ptrs(pop)
-    _check(lib().emr_pack_size(pop.P, ptr[0], ptr[5], C.byref(n)), "emr_pack_size")
+    P, ptr = _range_ptrs(pop, genomes)
+    _check(lib().emr_pack_size(P, ptr[0], ptr[5], C.byref(n)), "emr_pack_size")
     return int(n.value)
 
 
-def pack_population(pop, out=None) -> np.ndarray:
-    """Packed blob (numpy uint8) of a workloads.Population; written into `out` (a
-    contiguous uint8 array, e.g. a view of pinned memory) when given, else into a new array."""
+def pack_population(pop, out=None, genomes=None) -> np.ndarray:
+    """Packed blob (numpy uint8) of a workloads.Population, or of its genomes [g0, g1) when
+    genomes = (g0, g1); written into `out` (a contiguous uint8 array, e.g. a view of pinned
+    memory) when given, else into a new array."""
     L = lib()
     n = C.c_size_t()
-    ptr = _pop_ptrs(pop)
-    _check(L.emr_pack_size(pop.P, ptr[0], ptr[5], C.byref(n)), "emr_pack_size")
+    P, ptr = _range_ptrs(pop, genomes)
+    _check(L.emr_pack_size(P, ptr[0], ptr[5], C.byref(n)), "emr_pack_size")
     if out is not None:
         if out.dtype != np.uint8 or not out.flags.c_contiguous or len(out) < n.value:
             raise ValueError("out: contiguous uint8 array of at least %d bytes" % n.value)
@@ -184,12 +198,21 @@ def pack_population(pop, out=None) -> np.ndarray:
     else:
         buf = np.empty(n.value + 16, np.uint8)   # the packer clears what it uses
     used, bad = C.c_size_t(), C.c_int32()
-    st = L.emr_pack_population(pop.P, *ptr, int(buf.ctypes.data), len(buf), C.byref(used), C.byref(bad))
+    st = L.emr_pack_population(P, *ptr, int(buf.ctypes.data), len(buf), C.byref(used), C.byref(bad))
     if st != EMR_OK:
         e = EmrError(st, "emr_pack_population (genome %d)" % bad.value)
         e.bad_genome = bad.value
         raise e
     return buf[:used.value]
+
+
+def partition_genomes(pack: np.ndarray, query, n_parts: int) -> np.ndarray:
+    """Contiguous genome ranges of balanced cost (emr_partition_genomes): int32 [n_parts + 1],
+    part k = genomes [g[k], g[k+1])."""
+    g = np.zeros(n_parts + 1, np.int32)
+    q = query.c
+    _check(lib().emr_partition_genomes(_ptr(pack), C.byref(q), n_parts, _ptr(g)), "emr_partition_genomes")
+    return g
 
 
 def pack_info(pack: np.ndarray):

@@ -237,9 +237,10 @@ def c1(D: int = 4) -> Workload:
 
 def c2(D: int = 7, P: int = 1000) -> Workload:
     """XOR-shaped population: 1000 genomes with 0-12 hidden nodes and <=40 connections;
-    substrate inputs (-1,-1), (1,-1), bias (0,-1) queried outgoing, output (0,1) incoming."""
-    pop = random_population(1000, seed=2, h_lo=0, h_hi=12, e_max=40)
-    if P != 1000:
+    substrate inputs (-1,-1), (1,-1), bias (0,-1) queried outgoing, output (0,1) incoming.
+    P > 1000 continues the same generator (the first 1000 genomes are unchanged)."""
+    pop = random_population(max(P, 1000), seed=2, h_lo=0, h_hi=12, e_max=40)
+    if P != pop.P:
         pop = pop.subset(range(P))
     src = shared_sources([(-1.0, -1.0, SIDE_OUT), (1.0, -1.0, SIDE_OUT), (0.0, -1.0, SIDE_OUT),
                           (0.0, 1.0, SIDE_IN)])

@@ -94,14 +94,22 @@ def allreduce_max(x, ws):
     return allreduce(x, ws, "max")
 
 
-def rank_workload(W, rank, depth, pop):
-    """Each rank runs its own population (independent problems, no data exchange): rank 0 the
-    paper-shaped seed, rank r > 0 an equally drawn population from a rank-specific seed."""
-    w = W.c2(D=depth, P=pop)
-    if rank > 0:
-        w.pop = W.random_population(pop, seed=2 + 7919 * rank)
-        w.name = w.name + "_rank%d" % rank
-    return w
+def rank_workload(W, emr, rank, ws, depth, pop):
+    """This rank's share of one population: pop x ws genomes of the 1000-genome recipe (same
+    generator, so at one rank it is that population), split by packed cost into ws contiguous
+    genome ranges (emr_partition_genomes); about pop genomes per rank, so the work per GPU stays
+    fixed as ranks are added (weak scaling). Returns the rank's workload and its genome range."""
+    w = W.c2(D=depth, P=pop * ws)
+    if ws == 1:
+        return w, (0, w.P)
+    from paper_2608_27612_gb300 import dist as pdist
+    g = pdist.genome_ranges(emr.pack_population(w.pop), emr.make_query(w.sources, device="cpu"), ws)
+    g0, g1 = int(g[rank]), int(g[rank + 1])
+    full = w.pop
+    w.pop = full.subset(range(g0, g1))
+    w.name = "%s_genomes%d-%d" % (w.name, g0, g1)
+    w.extra["full_population"] = full
+    return w, (g0, g1)
 
 
 def aggregate(local_queries, local_ms, ws):
@@ -465,6 +473,151 @@ def variants_run(emr, torch, W, D=7, P=1000, reps=10):
             "timing": "CUDA events, mean of %d" % reps}
 
 
+def _events_mean(torch, fn, reps, flush):
+    """Mean CUDA-event time (s) of fn() over reps runs, L2 flushed before each."""
+    t = 0.0
+    for _ in range(reps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        torch.cuda.synchronize()
+        t += e0.elapsed_time(e1) / 1e3
+    return t / reps
+
+
+def config_table(emr, torch, W, sms, probe, flush, reps=10, oracle_seconds=2.0):
+    """Per workload: the step's device throughput (prepare + tiles + select, L2 flushed, CUDA
+    events), the tile kernels' ALU roofline under both work models, and the float64 oracle's
+    throughput on a sample of about oracle_seconds (cores stated); the lazy ES-HyperNEAT tree
+    timed on the single-genome and 1000-genome workloads."""
+    import oracle
+    oracle.build()
+    rows = []
+    specs = [("c1_single_d4", W.c1(), True), ("c2_xor_pop1000_d5", W.c2(D=5), True),
+             ("c2_xor_pop1000_d6", W.c2(D=6), True), ("c2_xor_pop1000_d7", W.c2(D=7), True),
+             ("c3_wide_pop256_d6", W.c3(D=6), False), ("c4_recurrent_r1_pop150_d8", W.c4_round1(), False)]
+    for name, w, lazy in specs:
+        dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, emr.EMR_EAGER)
+        g = dsc.grid
+        q = dsc.n_pairs * g.n_total
+        dsc.run_select()
+        torch.cuda.synchronize()
+        tile = {}
+
+        def step():
+            dsc.prepare()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            emr.eval_filter_tiles(dsc.pack, dsc.query, g, dsc.theta, dsc.band, dsc.w_min, dsc.split,
+                                  dsc.band_bits, dsc.tile_flags, dsc.ws)
+            b.record()
+            emr.select(dsc.split, dsc.band_bits, dsc.tile_flags, dsc.pack, dsc.query, dsc.ws, g, dsc.mode,
+                       dsc.types, dsc.idx, dsc.w, dsc.cap, dsc.counts, dsc.offsets, dsc.sws)
+            tile.setdefault("ev", []).append((a, b))
+
+        t_step = _events_mean(torch, step, reps, flush)
+        t_tile = statistics.mean(a.elapsed_time(b) for a, b in tile["ev"]) / 1e3
+        roof = roofline_entry(emr, dsc, g, sms, probe, t_tile)
+        row = {"workload": name, "queries": q, "gpu_step_ms": t_step * 1e3, "gpu_value": q / t_step,
+               "tile_kernels_ms": t_tile * 1e3, "frac_survey_model": roof["frac_survey_model"],
+               "frac_executed": roof["frac_executed"], "kept": int(dsc.offsets[-1])}
+        # oracle: whole genomes until about oracle_seconds have passed
+        n_g, t_o = 0, 0.0
+        while n_g < w.P and t_o < oracle_seconds:
+            k = max(1, min(w.P - n_g, 8))
+            t0 = time.perf_counter()
+            oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, g0=n_g, g1=n_g + k,
+                            fields=("keep_eager",))
+            t_o += time.perf_counter() - t0
+            n_g += k
+        qo = n_g * w.S * g.n_total
+        row["oracle"] = {"value": qo / t_o, "cores": oracle.threads(),
+                         "sample": "%d of %d genomes x %d slots (%.3g queries + halo), %.2f s"
+                                   % (n_g, w.P, w.S, qo, t_o)}
+        if lazy:
+            n_l = min(w.P, n_g)
+            t0 = time.perf_counter()
+            _, evals = oracle.lazy(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, g0=0, g1=n_l)
+            t_l = time.perf_counter() - t0
+            ql = n_l * w.S * g.n_total
+            row["lazy"] = {"seconds": t_l, "cppn_evaluations": int(evals.sum()),
+                           "evaluations_per_s": float(evals.sum()) / t_l,
+                           "grid_equivalent_value": ql / t_l, "cores": oracle.threads(),
+                           "sample": "%d genomes x %d slots, the lazy float64 quadtree (the ES-HyperNEAT order): "
+                                     "grid_equivalent_value = the grid's queries of the sample / its time"
+                                     % (n_l, w.S)}
+        rows.append(row)
+        del dsc
+        torch.cuda.empty_cache()
+    return rows
+
+
+def hbm_rates(emr, torch, W, flush, reps=10):
+    """Achieved bandwidth of the materialised evaluation (emr_eval: 4 B written per position and
+    halo point) and of the compaction of a materialised mask (emr_compact: the mask plane read,
+    8 B per kept entry and 16 B per pair written), 1000 genomes x 4 slots at depth 7, against the
+    measured copy bandwidth."""
+    w = W.c2(D=7)
+    dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, emr.EMR_EAGER, materialise=True)
+    g = dsc.grid
+    peak, basis = hbm_peak()
+    dsc.prepare()
+    t_eval = _events_mean(torch, lambda: emr.eval(dsc.pack, dsc.query, g, dsc.out, dsc.out_halo, dsc.ws), reps,
+                          flush)
+    b_eval = 4 * dsc.n_pairs * (g.n_total + g.n_halo)
+    dsc.run_unfused()
+    torch.cuda.synchronize()
+    kept = int(dsc.offsets[-1])
+    t_cmp = _events_mean(torch, lambda: emr.compact(dsc.mask, dsc.out, g, dsc.n_pairs, dsc.idx, dsc.w, dsc.cap,
+                                                    dsc.counts, dsc.offsets, dsc.cws), reps, flush)
+    b_cmp = 4 * dsc.n_pairs * g.n_words + 8 * kept + 16 * dsc.n_pairs
+    del dsc
+    torch.cuda.empty_cache()
+    ent = lambda b, t, what: {"bytes": b, "ms": t * 1e3, "achieved_gbs": b / t / 1e9, "peak_gbs": peak,
+                              "frac": b / t / 1e9 / peak, "peak_basis": basis, "bytes_counted": what}
+    return {"emr_eval_materialised": ent(b_eval, t_eval, "4 B per position and halo point written"),
+            "emr_compact": ent(b_cmp, t_cmp, "mask plane read, 8 B per kept entry and 16 B per pair written"),
+            "workload": "c2_xor_pop1000_d7", "timing": "CUDA events, L2 flushed, mean of %d" % reps}
+
+
+def oracle_samples(W):
+    """The float64 oracle on stated samples of the two workloads too large to run whole: the
+    hidden-to-hidden round (2 genomes x 256 slots at depth 8) and the streamed depth-13 grid
+    (the oracle's per-position keep decision, by direct CPPN queries, at 2^18 sampled positions
+    of each of the 64 pairs)."""
+    import oracle
+    oracle.build()
+    out = {}
+    w = W.c4_round2_random()
+    t0 = time.perf_counter()
+    oracle.discover(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, g0=0, g1=2, fields=("keep_eager",))
+    t = time.perf_counter() - t0
+    q = 2 * w.S * oracle.n_total(w.D)
+    out["c4_round2_hh_d8"] = {"value": q / t, "cores": oracle.threads(),
+                              "sample": "2 of %d genomes x %d slots at depth %d (%.3g queries + halo), %.2f s"
+                                        % (w.P, w.S, w.D, q, t)}
+    w = W.c5()
+    rng = np.random.default_rng(13)
+    n = 1 << 14
+    N = oracle.n_total(w.D)
+    t = 0.0
+    for gen in range(w.P):
+        for s in range(w.S):
+            d, i, j = level_ij(rng.integers(0, N, n))
+            t0 = time.perf_counter()
+            oracle.keep_at(w.pop, gen, float(w.sources.a[s]), float(w.sources.b[s]), int(w.sources.side[s]), w.D,
+                           w.theta, w.band, w.w_min, d, i, j)
+            t += time.perf_counter() - t0
+    q = w.P * w.S * n
+    out["c5_streamed_d13"] = {"value": q / t, "cores": oracle.threads(),
+                              "sample": "%d positions of each of the %d pairs at depth %d, each position's keep "
+                                        "decision from direct CPPN queries (itself, its 4 children, its 4 band "
+                                        "neighbours), %.2f s" % (n, w.P * w.S, w.D, t)}
+    return out
+
+
 def launches_in_step(emr, dsc):
     """Kernel launches of one step: prepare (records, with the schedule in the last CTA); per
     non-empty dense kernel class two tile launches (depths 0..5 on the block kernel, the
@@ -592,8 +745,9 @@ def main():
     from paper_2608_27612_gb300 import emr
     from paper_2608_27612_gb300 import workloads as W
 
-    # Each rank runs its own population (independent problems, no collective on the data path).
-    w = rank_workload(W, rank, args.depth, args.pop)
+    # One population split by cost over the ranks (no collective on the data path; the lists are
+    # gathered to rank 0 after the timed region).
+    w, g_range = rank_workload(W, emr, rank, ws, args.depth, args.pop)
     dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, emr.EMR_EAGER)
     g = dsc.grid
     queries = dsc.n_pairs * g.n_total
@@ -639,6 +793,11 @@ def main():
     clocks = sampler.stop()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     tile_ms = [a.elapsed_time(b) for a, b in tiles]
+    phases = {"prepare_ms": statistics.mean(s.elapsed_time(t[0]) for s, t in zip(starts, tiles)),
+              "tiles_ms": statistics.mean(tile_ms),
+              "select_ms": statistics.mean(t[1].elapsed_time(e) for t, e in zip(tiles, ends)),
+              "note": "CUDA events between the three calls of a step (emr_eval_prepare, emr_eval_filter_tiles, "
+                      "emr_select); the events keep the selection from overlapping the last tile launch"}
     _, ms, value = aggregate(queries, statistics.mean(step_ms), ws)
 
     # roofline of the dominant kernel (fused eval + variance + band)
@@ -663,13 +822,15 @@ def main():
     # on a second stream while step k + 1 computes.
     e2e = None
     if args.e2e_steps > 0:
-        pop = w.pop
+        # each rank packs its genome range of the whole population through the range hook
+        full_pop = w.extra.get("full_population", w.pop)
+        pack_range = g_range if full_pop is not w.pop else None
         # one pinned input buffer per step in flight, [a | b | side | packed population], and one
         # device copy of it: a single host-to-device copy a step of the bytes in use; the packer
         # writes in place
         S = dsc.query.S
         ob = (12 * S + 255) // 256 * 256
-        in_bytes = ob + emr.pack_size(pop)
+        in_bytes = ob + emr.pack_size(full_pop, genomes=pack_range)
         in_pinned = [torch.empty(in_bytes, dtype=torch.uint8).pin_memory() for _ in range(2)]
         for buf in in_pinned:
             q_h = buf[:12 * S].numpy()
@@ -719,7 +880,7 @@ def main():
             buf = in_pinned[b]
             # this input set's last user, step k - 2, has finished (its offsets were synchronised
             # on in the previous iteration), so the packer and the copy may overwrite it
-            blob = emr.pack_population(pop, out=buf[ob:].numpy())
+            blob = emr.pack_population(full_pop, out=buf[ob:].numpy(), genomes=pack_range)
             h2d = ob + len(blob)
             emr.copy_async(in_dev[b], buf, h2d, copy_in)
             inputs_in[b].record(copy_in)
@@ -744,6 +905,23 @@ def main():
                            "are read on a second copy stream after step k+1 is queued; wall clock over %d steps"
                            % n_steps}
 
+    gather = None
+    if ws > 1:
+        # the lists of every rank's genome range to rank 0 (the rank that assembles networks)
+        from paper_2608_27612_gb300 import dist as pdist
+        n_loc = min(int(dsc.offsets[-1]), dsc.cap)
+        torch.cuda.synchronize()
+        barrier(ws)
+        t0 = time.perf_counter()
+        got = pdist.gather_lists(dsc.counts, dsc.idx[:n_loc], dsc.w[:n_loc])
+        torch.cuda.synchronize()
+        g_ms = allreduce((time.perf_counter() - t0) * 1e3, ws, "max")
+        gather = {"ms": g_ms, "entries_local": n_loc,
+                  "entries_total": int(got[1][-1]) if got is not None else None,
+                  "pairs_total": int(got[0].numel()) if got is not None else None,
+                  "how": "torch.distributed all_gather of sizes, then gather of padded counts, indices and "
+                         "weights to rank 0 (NCCL); wall clock, max over ranks; outside the timed steps"}
+
     extra = None
     if rank == 0 and ws == 1 and not args.no_extra:
         c4r2 = W.c4_round2_random()
@@ -755,7 +933,11 @@ def main():
                      emr, torch, c4r2, 1 << 16, 1 << 24, 1 << 26, 3,
                      types=emr.substrate_config(emr.SUBSTRATE_BACKWARD)[0], label=c4r2.name + "_backward"),
                  "xor_networks_hh_d5": networks_run(emr, torch, W),
-                 "variants_c2_d7": variants_run(emr, torch, W)}
+                 "variants_c2_d7": variants_run(emr, torch, W),
+                 "configs": config_table(emr, torch, W, sms, probe, flush),
+                 "hbm": hbm_rates(emr, torch, W, flush)}
+        if not args.no_cpu_baseline:
+            extra["oracle_samples"] = oracle_samples(W)
 
     cpu = parity = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -772,8 +954,12 @@ def main():
             "config": {"workload": w.name, "genomes": w.P, "slots": w.S, "depth": w.D, "n_total": g.n_total,
                        "queries_per_step": queries, "theta": w.theta, "band": w.band, "mode": "eager",
                        "l2": "flushed between steps (256 MB write)", "kept_connections": kept,
-                       "parallelism": "independent populations per GPU" if ws > 1 else "single GPU"},
-            "roofline": roofline, "cpu_baseline": cpu, "parity": parity, "e2e": e2e, "extra": extra,
+                       "parallelism": ("one population of %d x %d genomes split by cost into contiguous genome "
+                                       "ranges, one per GPU" % (args.pop, ws)) if ws > 1 else "single GPU",
+                       "genome_range": list(g_range)},
+            "phases": phases, "roofline": roofline, "cpu_baseline": cpu, "parity": parity, "e2e": e2e,
+            "gather": gather,
+            "extra": extra,
             "gpu_launches": launches_per_step * args.steps, "clocks": clocks,
             "wall_s_timed_region": wall, "gpu": props.name,
         }))

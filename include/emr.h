@@ -182,6 +182,17 @@ emr_status emr_pack_population(int32_t P, const int64_t *node_ptr, const int32_t
  * Errors: EMR_ERR_ARG (null pointer, n_parts <= 0, bad side, not a pack). */
 emr_status emr_partition_genomes(const void *pack_host, const emr_query *q, int32_t n_parts, int32_t *g_begin);
 
+/* The packer's state kept between calls: up to 15 host worker threads (started
+ * on first use; starting them costs as much as packing a few dozen genomes) and
+ * its per-thread packing buffers (grown to the largest population packed). This
+ * is libemr's one process-wide state besides emr_eval_filter_noalloc's static
+ * device array; it holds no results, only scratch. emr_pack_release joins the
+ * worker threads and frees the buffers; the next emr_pack_population (or
+ * emr_assemble, which shares the workers) recreates them. Libemr also joins
+ * the workers when it is unloaded or the process exits. Must not be called
+ * while another thread is inside emr_pack_population or emr_assemble. */
+void emr_pack_release(void);
+
 /* Summary of a packed blob: population size and, per query side, the largest
  * number of varying nodes. Any output pointer may be NULL. */
 emr_status emr_pack_info(const void *pack_host, int32_t *P, int32_t *max_varying_out,
@@ -302,7 +313,10 @@ emr_status emr_stream_workspace_size(const void *pack_host, const emr_query *q, 
  * limit): queued work is still running then and writes into ws and the host
  * arrays, so synchronise the device before reusing them; EMR_ERR_CUDA.
  * Allocates per call a copy stream, four events and 16 (n_pairs + 1) bytes of
- * pinned host staging. */
+ * pinned host staging. On EMR_ERR_TIMEOUT the pinned staging is not freed
+ * (copies still queued may write into it, and freeing pinned memory would wait
+ * for them): each timed-out call leaks those 16 (n_pairs + 1) bytes of pinned
+ * host memory until the process exits; the stream and events are released. */
 emr_status emr_stream(const void *pack_host, const void *pack_dev, const emr_query *q, const emr_grid *grid,
                       float theta, float band, float w_min, void *ws, size_t ws_bytes, int64_t chunk_cap,
                       int32_t *h_idx, float *h_w, int64_t cap, int64_t *counts, int64_t *offsets,

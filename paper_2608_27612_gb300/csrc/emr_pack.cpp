@@ -23,8 +23,9 @@ inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 // Host worker threads kept across calls (starting threads costs as much as
 // packing a few dozen genomes). run() executes fn(0 .. n-1) on the workers and
 // the caller and returns when all are done; one job at a time (a caller that
-// finds the pool busy runs its job alone). The pool lives until exit and is
-// never destroyed; a process forked from this one starts a fresh pool.
+// finds the pool busy runs its job alone). shutdown() (emr_pack_release, and
+// the library's unload) stops and joins the workers; the next run() starts a
+// fresh pool. A process forked from this one starts a fresh pool too.
 class WorkerPool {
  public:
   static WorkerPool& get() {
@@ -33,6 +34,26 @@ class WorkerPool {
     std::lock_guard<std::mutex> lk(create_mu());
     if (!instance()) instance() = new WorkerPool();
     return *instance();
+  }
+
+  // Stop and join the workers and free the pool (never while a job runs on it).
+  static void shutdown() {
+    WorkerPool* p;
+    {
+      std::lock_guard<std::mutex> lk(create_mu());
+      p = instance();
+      instance() = nullptr;
+    }
+    if (!p) return;
+    {
+      std::lock_guard<std::mutex> job(p->job_mu_);  // a job in progress finishes first
+      std::lock_guard<std::mutex> lk(p->mu_);
+      p->stop_ = true;
+    }
+    p->cv_.notify_all();
+    for (std::thread& t : p->threads_)
+      if (t.joinable()) t.join();
+    delete p;
   }
 
   void run(int n, const std::function<void(int)>& fn) {
@@ -79,17 +100,15 @@ class WorkerPool {
   }
 
   void ensure(int workers) {
-    while (int(n_workers_) < workers) {
-      std::thread([this] { loop(); }).detach();
-      n_workers_++;
-    }
+    while (int(threads_.size()) < workers) threads_.emplace_back([this] { loop(); });
   }
 
   void loop() {
     uint64_t seen = 0;
     for (;;) {
       std::unique_lock<std::mutex> lk(mu_);
-      cv_.wait(lk, [&] { return gen_ != seen && job_ && next_ < n_; });
+      cv_.wait(lk, [&] { return stop_ || (gen_ != seen && job_ && next_ < n_); });
+      if (stop_) return;
       seen = gen_;
       while (job_ && next_ < n_) {
         const int t = next_++;
@@ -107,7 +126,8 @@ class WorkerPool {
   const std::function<void(int)>* job_ = nullptr;
   int n_ = 0, next_ = 0, left_ = 0;
   uint64_t gen_ = 0;
-  unsigned n_workers_ = 0;
+  bool stop_ = false;
+  std::vector<std::thread> threads_;
 };
 
 uint32_t compact_bits(uint64_t m) {  // even bits of m, packed
@@ -154,7 +174,8 @@ struct Scratch {
 
 // Packing buffers of the tasks of one call, kept across calls so that a warm
 // packer allocates nothing: scratch, the tasks' node and edge records, the
-// genome table. One caller at a time uses the shared set (never destroyed).
+// genome table. One caller at a time uses the shared set; release() (from
+// emr_pack_release) frees their memory, and the next call grows them again.
 struct PackBuffers {
   static constexpr int kTasks = 16;
   std::mutex mu;
@@ -165,6 +186,15 @@ struct PackBuffers {
   static PackBuffers& get() {
     static PackBuffers* b = new PackBuffers();
     return *b;
+  }
+  void release() {
+    std::lock_guard<std::mutex> lk(mu);
+    for (int t = 0; t < kTasks; t++) {
+      scratch[t] = Scratch();
+      std::vector<PackNode>().swap(nodes[t]);
+      std::vector<PackEdge>().swap(edges[t]);
+    }
+    std::vector<GenomeOut>().swap(gs);
   }
 };
 
@@ -554,6 +584,15 @@ emr_status emr_pack_info(const void* pack_host, int32_t* P, int32_t* max_varying
   if (max_varying_in) *max_varying_in = h->max_varying[EMR_SIDE_IN];
   return EMR_OK;
 }
+
+void emr_pack_release(void) {
+  WorkerPool::shutdown();
+  PackBuffers::get().release();
+}
+
+// The worker threads are joined when libemr is unloaded (or the process exits),
+// so no thread outlives the library's code.
+__attribute__((destructor)) static void emr_pack_unload() { WorkerPool::shutdown(); }
 
 // Contiguous genome ranges of balanced cost for population-parallel work
 // (Table 1: the CPPN query, variance and mask stages split over the

@@ -102,6 +102,8 @@ def lib() -> C.CDLL:
             f = getattr(_lib, name)
             f.argtypes = args
             f.restype = C.c_int32
+        _lib.emr_pack_release.argtypes = []
+        _lib.emr_pack_release.restype = None
         _lib.emr_strerror.argtypes = [C.c_int32]
         _lib.emr_strerror.restype = C.c_char_p
     return _lib
@@ -204,6 +206,11 @@ def pack_population(pop, out=None, genomes=None) -> np.ndarray:
         e.bad_genome = bad.value
         raise e
     return buf[:used.value]
+
+
+def pack_release() -> None:
+    """Join the packer's worker threads and free its kept buffers (emr_pack_release)."""
+    lib().emr_pack_release()
 
 
 def partition_genomes(pack: np.ndarray, query, n_parts: int) -> np.ndarray:

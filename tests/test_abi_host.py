@@ -285,3 +285,20 @@ def test_stream_workspace_holds_the_split_plane_and_two_chunks():
     big = size(1 << 26, 1 << 24)
     assert split_plane < size(1 << 20, 1 << 20) < size(1 << 26, 1 << 20) < big
     assert size(1 << 26, 1 << 20) < big and round(big / 1e9, 1) == 5.3
+
+
+def test_pack_release_joins_workers_and_the_next_pack_is_identical():
+    """emr_pack_release joins the packer's worker threads (the process's native thread count drops)
+    and frees its buffers; packing again starts them afresh and gives the same blob (host only)."""
+    tasks = lambda: len(os.listdir("/proc/self/task"))
+    w = W.c2(D=5)
+    first = emr.pack_population(w.pop)
+    with_pool = tasks()
+    emr.pack_release()
+    without = tasks()
+    emr.pack_release()  # idempotent
+    assert tasks() == without
+    if (os.cpu_count() or 1) > 1:
+        assert without < with_pool
+    again = emr.pack_population(w.pop)
+    assert np.array_equal(first, again) and tasks() == with_pool

@@ -2212,12 +2212,16 @@ __device__ __forceinline__ int warp_exclusive_scan(int v, int* total) {
 __global__ void __launch_bounds__(kSelectThreads) select_count_kernel(const uint32_t* __restrict__ split,
                                                                       const uint32_t* __restrict__ bandb,
                                                                       const uint8_t* __restrict__ flags,
-                                                                      int64_t n_dense, GridDev G, int gated,
+                                                                      int64_t n_dense, GridDev G_arg, int gated,
                                                                       TypeFilter tf, int64_t n_pairs,
                                                                       int64_t* __restrict__ counts,
                                                                       int32_t* __restrict__ tile_base,
                                                                       int64_t* __restrict__ items,
                                                                       unsigned long long* __restrict__ n_items) {
+  __shared__ GridDev G;  // dynamically indexed below: a shared copy instead of a local one
+  for (int k = threadIdx.x; k < int(sizeof(GridDev) / 4); k += blockDim.x)
+    reinterpret_cast<int*>(&G)[k] = reinterpret_cast<const int*>(&G_arg)[k];
+  __syncthreads();
   pdl_wait();  // the tile launches' planes and flags
   pdl_trigger();
   const int lane = threadIdx.x & 31;
@@ -2255,7 +2259,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_count_kernel(const uint
 // entries go to offsets[pair] + tile_base, in ascending global index.
 __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint32_t* __restrict__ split,
                                                                       const uint32_t* __restrict__ bandb,
-                                                                      int64_t n_dense, GridDev G, int gated,
+                                                                      int64_t n_dense, GridDev G_arg, int gated,
                                                                       TypeFilter tf,
                                                                       const int32_t* __restrict__ tile_base,
                                                                       const int64_t* __restrict__ items,
@@ -2263,6 +2267,10 @@ __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint
                                                                       const int64_t* __restrict__ offsets,
                                                                       int64_t cap, int32_t* __restrict__ idx,
                                                                       float* __restrict__ wv) {
+  __shared__ GridDev G;  // dynamically indexed below: a shared copy instead of a local one
+  for (int k = threadIdx.x; k < int(sizeof(GridDev) / 4); k += blockDim.x)
+    reinterpret_cast<int*>(&G)[k] = reinterpret_cast<const int*>(&G_arg)[k];
+  __syncthreads();
   pdl_wait();  // the offsets (and, before them, the work items)
   pdl_trigger();
   const int lane = threadIdx.x & 31;
@@ -2282,16 +2290,30 @@ __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(const uint
       int total;
       const int ex = warp_exclusive_scan(__popc(m[0]) + __popc(m[1]) + __popc(m[2]) + __popc(m[3]), &total);
       int64_t dst = base + ex;
+      // one non-empty word at a time across the warp, lane l its bit l: consecutive set
+      // bits go to consecutive entries, so the stores coalesce
+#pragma unroll
       for (int c = 0; c < 4; c++) {
-        if (!m[c]) continue;
-        int d = 0;
-        while (G.word_off[d + 1] <= wi + c) d++;
-        const int64_t gbase = G.level_off[d] + (wi + c - G.word_off[d]) * 32;
-        for (uint32_t v = m[c]; v; v &= v - 1, dst++)
-          if (dst < cap) {
-            idx[dst] = int32_t(gbase + __ffs(v) - 1);
-            if (wv) wv[dst] = __int_as_float(int32_t(r));  // the pair, for select_weights_kernel
+        int64_t gb = 0;
+        if (m[c]) {
+          int d = 0;
+          while (G.word_off[d + 1] <= wi + c) d++;
+          gb = G.level_off[d] + (wi + c - G.word_off[d]) * 32;
+        }
+        for (uint32_t nz = __ballot_sync(kFull, m[c] != 0u); nz; nz &= nz - 1) {
+          const int src = __ffs(nz) - 1;
+          const uint32_t word = __shfl_sync(kFull, m[c], src);
+          const int64_t wd = __shfl_sync(kFull, dst, src);
+          const int64_t wg = __shfl_sync(kFull, gb, src);
+          if ((word >> lane) & 1u) {
+            const int64_t e = wd + __popc(word & ((1u << lane) - 1u));
+            if (e < cap) {
+              idx[e] = int32_t(wg + lane);
+              if (wv) wv[e] = __int_as_float(int32_t(r));  // the pair, for select_weights_kernel
+            }
           }
+        }
+        dst += __popc(m[c]);
       }
       base += total;
     }

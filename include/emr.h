@@ -227,6 +227,29 @@ emr_status emr_eval_prepare(const void *pack_host, const void *pack_dev, const e
 emr_status emr_eval(const void *pack_host, const emr_query *q, const emr_grid *grid, float *out, float *out_halo,
                     void *ws, size_t ws_bytes, void *stream);
 
+/* Chunks of a grid (the chunking emr_stream uses; Section 5.2 and Section 6
+ * stream depths 8..13 because W no longer fits): grid->chunk positions per
+ * chunk in whole 64 x 64 tiles (0 = one chunk), the tile of depths 0..4 in the
+ * lowest chunk, chunks numbered 0 .. *n_chunks - 1 in ascending global index.
+ * Chunk chunk_idx covers global indices [*pos_beg, *pos_end). n_chunks, pos_beg,
+ * pos_end may each be NULL (with both position pointers NULL only *n_chunks is
+ * written and chunk_idx is not checked). Host only. Errors: EMR_ERR_ARG (bad
+ * grid, chunk not a multiple of 4096), EMR_ERR_RANGE (chunk_idx outside). */
+emr_status emr_grid_chunk(const emr_grid *grid, int64_t chunk_idx, int64_t *n_chunks, int64_t *pos_beg,
+                          int64_t *pos_end);
+
+/* emr_eval over one chunk of the grid (emr_grid_chunk), for materialising W one
+ * chunk at a time when the whole grid does not fit (Section 5.2: the paper
+ * streams W through host memory at depth 7 and beyond). out: device float
+ * [P * S][pos_end - pos_beg], pair r's output at global index g in
+ * out[r][g - pos_beg] (16-byte aligned); out_halo: NULL or the whole-grid halo
+ * buffer of emr_eval (only the halo points next to the chunk's tiles are
+ * written). ws: prepared by emr_eval_prepare. Every chunk's values equal
+ * emr_eval's at the same positions. Errors: EMR_ERR_ARG, EMR_ERR_RANGE
+ * (chunk_idx outside), EMR_ERR_CAPACITY, EMR_ERR_CUDA. */
+emr_status emr_eval_chunk(const void *pack_host, const emr_query *q, const emr_grid *grid, int64_t chunk_idx,
+                          float *out, float *out_halo, void *ws, size_t ws_bytes, void *stream);
+
 /* ---- a4, a5: variance and band/threshold filter --------------------------- */
 
 /* Filter a materialised evaluation (Section 3.2, Eq. 2; Theorem 1's band

@@ -3336,21 +3336,30 @@ inline int64_t tile_word(const emr_grid* g, int32_t t, int32_t n_dense) {
   return t == 0 ? 0 : g->word_off[kPyramidTop + 1] + int64_t(t - 1) * (kTileSide * kTileSide / 32);
 }
 
+// The grid's chunks as dense tile ranges, from the highest global index down:
+// grid->chunk positions each (whole 64 x 64 tiles; 0 = one chunk), the tile of
+// depths 0..4 joining the lowest chunk.
+std::vector<std::pair<int32_t, int32_t>> grid_chunks(const emr_grid* g) {
+  const int32_t n_dense = int32_t(dense_tiles(g->D));
+  const int64_t tile_positions = int64_t(kTileSide) * kTileSide;
+  const int32_t tpc = g->chunk > 0 ? int32_t(std::max<int64_t>(1, g->chunk / tile_positions)) : n_dense;
+  std::vector<std::pair<int32_t, int32_t>> chunks;
+  for (int32_t hi = n_dense; hi > 0;) {
+    int32_t lo = std::max(hi - tpc, 1);
+    if (lo == 1) lo = 0;  // the tile of depths 0..4 joins the last chunk
+    chunks.push_back({lo, hi});
+    hi = lo;
+  }
+  return chunks;
+}
+
 emr_status stream_plan(const void* pack_host, const emr_query* q, const emr_grid* g, int64_t chunk_cap,
                        StreamPlan* sp) {
   if (!grid_ok(g) || chunk_cap <= 0) return EMR_ERR_ARG;
   emr_status rc = eval_plan(pack_host, q, &sp->ev);
   if (rc != EMR_OK) return rc;
   const int32_t n_dense = int32_t(dense_tiles(g->D));
-  const int64_t tile_positions = int64_t(kTileSide) * kTileSide;
-  const int32_t tpc = g->chunk > 0 ? int32_t(std::max<int64_t>(1, g->chunk / tile_positions)) : n_dense;
-  sp->chunks.clear();
-  for (int32_t hi = n_dense; hi > 0;) {
-    int32_t lo = std::max(hi - tpc, 1);
-    if (lo == 1) lo = 0;  // the tile of depths 0..4 joins the last chunk
-    sp->chunks.push_back({lo, hi});
-    hi = lo;
-  }
+  sp->chunks = grid_chunks(g);
   sp->wpc = sp->ppc = 0;
   for (auto& c : sp->chunks) {
     sp->wpc = std::max(sp->wpc, tile_word(g, c.second, n_dense) - tile_word(g, c.first, n_dense));
@@ -3377,6 +3386,51 @@ emr_status stream_plan(const void* pack_host, const emr_query* q, const emr_grid
   sp->total = o;
   return EMR_OK;
 }
+
+}  // namespace
+
+extern "C" emr_status emr_grid_chunk(const emr_grid* grid, int64_t chunk_idx, int64_t* n_chunks, int64_t* pos_beg,
+                                     int64_t* pos_end) {
+  if (!grid_ok(grid)) return EMR_ERR_ARG;
+  if (grid->chunk < 0 || (grid->chunk > 0 && grid->chunk % (int64_t(kTileSide) * kTileSide) != 0))
+    return EMR_ERR_ARG;
+  const auto chunks = grid_chunks(grid);
+  const int64_t n = int64_t(chunks.size());
+  if (n_chunks) *n_chunks = n;
+  if (!pos_beg && !pos_end) return EMR_OK;
+  if (chunk_idx < 0 || chunk_idx >= n) return EMR_ERR_RANGE;
+  const auto& c = chunks[size_t(n - 1 - chunk_idx)];  // ascending global index
+  const int32_t n_dense = int32_t(dense_tiles(grid->D));
+  if (pos_beg) *pos_beg = tile_pos(grid, c.first, n_dense);
+  if (pos_end) *pos_end = tile_pos(grid, c.second, n_dense);
+  return EMR_OK;
+}
+
+extern "C" emr_status emr_eval_chunk(const void* pack_host, const emr_query* q, const emr_grid* grid,
+                                     int64_t chunk_idx, float* out, float* out_halo, void* ws, size_t ws_bytes,
+                                     void* stream) {
+  if (!grid_ok(grid) || !out || !ws) return EMR_ERR_ARG;
+  int64_t n_chunks = 0, p_lo = 0, p_hi = 0;
+  emr_status rc = emr_grid_chunk(grid, chunk_idx, &n_chunks, &p_lo, &p_hi);
+  if (rc != EMR_OK) return rc;
+  EvalPlan p;
+  if ((rc = eval_plan(pack_host, q, &p)) != EMR_OK) return rc;
+  if (ws_bytes < p.total) return EMR_ERR_CAPACITY;
+  uint8_t* spec;
+  int32_t* order;
+  ws_layout(p, ws, &spec, &order);
+  const auto chunks = grid_chunks(grid);
+  const auto& c = chunks[size_t(n_chunks - 1 - chunk_idx)];
+  TileRange tr;
+  tr.beg = c.first;
+  tr.end = c.second;
+  tr.out_stride = p_hi - p_lo;
+  tr.out_shift = p_lo;
+  return launch_tiles(p, grid, spec, order, kModeMaterialise, 0.f, 0.f, 0.f, out, out_halo, nullptr, nullptr,
+                      static_cast<cudaStream_t>(stream), tr);
+}
+
+namespace {
 
 // Wait for an event with a host-side deadline (timeout_ms <= 0: no limit).
 emr_status wait_event(cudaEvent_t ev, std::chrono::steady_clock::time_point deadline, bool limited) {

@@ -65,6 +65,8 @@ def lib() -> C.CDLL:
             "emr_eval_workspace_size": [vp, vp, vp],
             "emr_eval_prepare": [vp, vp, vp, vp, sz, vp],
             "emr_eval": [vp, vp, vp, vp, vp, vp, sz, vp],
+            "emr_grid_chunk": [vp, i64, vp, vp, vp],
+            "emr_eval_chunk": [vp, vp, vp, i64, vp, vp, vp, sz, vp],
             "emr_variance_filter": [vp, vp, vp, i32, i32, f32, f32, f32, i32, vp, vp, vp, vp, vp],
             "emr_mask_combine": [vp, vp, vp, i32, i32, vp, vp],
             "emr_eval_filter": [vp, vp, vp, f32, f32, f32, vp, vp, vp, vp, sz, vp],
@@ -290,6 +292,19 @@ def eval(pack, query: Query, grid: Grid, out, out_halo, ws, stream=None):
     _check(lib().emr_eval(_ptr(pack), C.byref(q), C.byref(grid), _ptr(out), _ptr(out_halo), _ptr(ws),
                           C.c_size_t(ws.numel()), _stream(stream)), "emr_eval")
 
+
+def grid_chunk(grid: Grid, chunk_idx: int = 0):
+    """(number of chunks, first global index, end global index) of chunk chunk_idx (emr_grid_chunk)."""
+    n, lo, hi = C.c_int64(), C.c_int64(), C.c_int64()
+    _check(lib().emr_grid_chunk(C.byref(grid), chunk_idx, C.byref(n), C.byref(lo), C.byref(hi)), "emr_grid_chunk")
+    return n.value, lo.value, hi.value
+
+
+def eval_chunk(pack, query: Query, grid: Grid, chunk_idx: int, out, out_halo, ws, stream=None):
+    """emr_eval_chunk: CPPN outputs of one chunk, out [pairs, chunk positions]."""
+    q = query.c
+    _check(lib().emr_eval_chunk(_ptr(pack), C.byref(q), C.byref(grid), chunk_idx, _ptr(out), _ptr(out_halo),
+                                _ptr(ws), ws.numel(), _stream(stream)), "emr_eval_chunk")
 
 def variance_filter(out, out_halo, grid: Grid, P: int, S: int, theta: float, band: float, w_min: float, mode: int,
                     mask, split, band_bits, var_dbg=None, stream=None):

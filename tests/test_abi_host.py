@@ -302,3 +302,23 @@ def test_pack_release_joins_workers_and_the_next_pack_is_identical():
         assert without < with_pool
     again = emr.pack_population(w.pop)
     assert np.array_equal(first, again) and tasks() == with_pool
+
+
+def test_grid_chunks_cover_the_grid_in_whole_tiles():
+    """emr_grid_chunk: chunks in ascending global index, contiguous, covering [0, N_total), every
+    boundary but the first a 64 x 64 tile boundary past depth 4, the same count emr_stream uses."""
+    for D, chunk in ((0, 0), (5, 4096), (7, 0), (7, 1 << 14), (10, 1 << 16), (13, 1 << 26)):
+        g = emr.grid_build(D, chunk)
+        n = emr.grid_chunk(g)[0]
+        r = [emr.grid_chunk(g, k)[1:] for k in range(n)]
+        assert r[0][0] == 0 and r[-1][1] == g.n_total
+        assert all(a[1] == b[0] for a, b in zip(r, r[1:]))
+        lo5 = oracle.n_total(4) if D >= 5 else g.n_total
+        assert all(b[0] >= lo5 and (b[0] - lo5) % 4096 == 0 for b in r[1:])
+        if chunk:
+            assert all(hi - lo <= max(chunk, lo5 + chunk) for lo, hi in r)
+        with pytest.raises(emr.EmrError) as e:
+            emr.grid_chunk(g, n)
+        assert e.value.status == emr.EMR_ERR_RANGE
+    g = emr.grid_build(13, 1 << 26)
+    assert emr.grid_chunk(g)[0] == 6  # depth 13 in chunks of 2^26: 5.33 chunks, the remainder in the lowest

@@ -115,3 +115,49 @@ def test_stream_host_wait_times_out_and_device_stays_usable():
     torch.cuda.synchronize()
     x = torch.ones(16, device="cuda")
     assert float(x.sum()) == 16.0
+
+
+def test_eval_chunks_equal_the_whole_grid_evaluation():
+    """emr_eval_chunk over every chunk of a depth-7 grid (chunks of 2^14 positions) gives emr_eval's
+    outputs and halo bit for bit."""
+    w = W.c2(D=7, P=60)
+    dsc = emr.Discovery(w.pop, w.sources, w.D, w.theta, w.band, w.w_min, materialise=True)
+    dsc.prepare()
+    emr.eval(dsc.pack, dsc.query, dsc.grid, dsc.out, dsc.out_halo, dsc.ws)
+    gc = emr.grid_build(7, 1 << 14)
+    n = emr.grid_chunk(gc)[0]
+    assert n == 6
+    halo = torch.full_like(dsc.out_halo, float("nan"))
+    for k in range(n):
+        _, lo, hi = emr.grid_chunk(gc, k)
+        out = torch.full((dsc.n_pairs, hi - lo), float("nan"), device="cuda")
+        emr.eval_chunk(dsc.pack, dsc.query, gc, k, out, halo, dsc.ws)
+        torch.cuda.synchronize()
+        assert torch.equal(out.view(torch.int32), dsc.out[:, lo:hi].view(torch.int32)), "chunk %d" % k
+    assert torch.equal(halo.view(torch.int32), dsc.out_halo.view(torch.int32))
+
+
+def test_eval_chunk_at_depth_13_against_the_oracle():
+    """One depth-13 chunk (2^26 positions) of one deep-grid genome's four slots, materialised, against the
+    oracle's CPPN at sampled positions of the chunk."""
+    w = W.c5(P=1)
+    pack = emr.pack_population(w.pop)
+    pack_dev = torch.from_numpy(pack).cuda()
+    q = emr.make_query(w.sources)
+    g = emr.grid_build(13, 1 << 26)
+    ws = torch.zeros(emr.eval_workspace_size(pack, q), dtype=torch.uint8, device="cuda")
+    emr.eval_prepare(pack, pack_dev, q, ws)
+    n, lo, hi = emr.grid_chunk(g, 3)
+    out = torch.empty(q.S, hi - lo, device="cuda")
+    emr.eval_chunk(pack, q, g, 3, out, None, ws)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(11)
+    pos = np.sort(rng.integers(lo, hi, 300))
+    for s in range(q.S):
+        ins = []
+        for p in pos:
+            d, i, j = emr.index_to_ij(int(p))
+            x, y = (2 * i + 1) / 2 ** (d + 1) - 1, (2 * j + 1) / 2 ** (d + 1) - 1
+            ins.append([float(w.sources.a[s]), float(w.sources.b[s]), x, y, 1.0])
+        ref, err = oracle.cppn(w.pop, 0, np.array(ins))
+        check_outputs(out[s, torch.from_numpy(pos - lo).cuda()].cpu().numpy(), ref, err, "slot %d" % s)

@@ -14,7 +14,10 @@ between steps); `e2e` is the same metric through the host-buffer path: packing
 on the host into pinned memory, the H2D copy of the packed genomes and slots,
 emr_discover (the same three stages in one call), and the D2H read of the
 offsets and connection lists, each step's copies overlapping its neighbours'
-kernels, timed by the wall clock.
+kernels, timed by the wall clock. Steps alternate between two compute streams
+(each with its own workspace), so one step's latency-bound preparation and
+selection overlap the next step's tile kernels; the figure with every step on
+one stream is reported beside it (`e2e.one_stream`).
 
 --impl reference times the float64 CPU oracle on a bounded sample of the same
 workload (the only other place this script runs the oracle).
@@ -819,7 +822,8 @@ def main():
     # step packs its population into pinned memory, copies it and the query slots to the device and
     # reads its lists back (offsets first, then the entries they count). Input and output sets
     # alternate: step k + 1's inputs are copied while step k computes, and step k's lists are read
-    # on a second stream while step k + 1 computes.
+    # on a second stream while step k + 1 computes. Measured with every step on one compute stream,
+    # and with steps alternating between two compute streams (the reported figure).
     e2e = None
     if args.e2e_steps > 0:
         # each rank packs its genome range of the whole population through the range hook
@@ -844,66 +848,81 @@ def main():
         q_e2e = [emr.Query(dsc.query.a, dsc.query.b, dsc.query.side, None, t[:4 * S].view(torch.float32),
                            t[4 * S:8 * S].view(torch.float32), t[8 * S:12 * S].view(torch.int32), None, S, False)
                  for t in in_dev]
-        dws = torch.zeros(emr.discover_workspace_size(dsc.pack, dsc.query, g), dtype=torch.uint8, device="cuda")
         qc = [q.c for q in q_e2e]
-        copy_in = torch.cuda.Stream()
-        inputs_in = [torch.cuda.Event(), torch.cuda.Event()]  # step k's inputs are on the device
         outs = [(dsc.idx, dsc.w, dsc.counts, dsc.offsets),
                 (torch.empty_like(dsc.idx), torch.empty_like(dsc.w), torch.empty_like(dsc.counts),
                  torch.empty_like(dsc.offsets))]
         res_off = [torch.empty(dsc.n_pairs + 1, dtype=torch.int64).pin_memory() for _ in range(2)]
         idx_h = torch.empty(dsc.cap, dtype=torch.int32).pin_memory()
         w_h = torch.empty(dsc.cap, dtype=torch.float32).pin_memory()
-        done = [torch.cuda.Event(), torch.cuda.Event()]     # step k's offsets are on the host
-        read = [torch.cuda.Event(), torch.cuda.Event()]     # step k's lists are on the host
-        copy = torch.cuda.Stream()
-        h2d = d2h = 0
-        n_warm, n_steps = 2, args.e2e_steps
-
         res_off_np = [t.numpy() for t in res_off]
+        ws_bytes = emr.discover_workspace_size(dsc.pack, dsc.query, g)
 
-        def read_lists(k):
-            b = k & 1
-            done[b].synchronize()
-            n = min(int(res_off_np[b][-1]), dsc.cap)
-            copy.wait_event(done[b])
-            emr.copy_async(idx_h, outs[b][0], 4 * n, copy)
-            emr.copy_async(w_h, outs[b][1], 4 * n, copy)
-            read[b].record(copy)
-            return 8 * (dsc.n_pairs + 1) + 8 * n
+        def e2e_run(n_compute):
+            """Wall-clock steps through emr_discover with n_compute compute streams (1: every step on
+            the benchmark's stream; 2: steps alternate between two streams and workspaces, so that
+            one step's latency-bound preparation and selection overlap the other's tile kernels)."""
+            cstreams = [stream] if n_compute == 1 else [torch.cuda.Stream() for _ in range(2)]
+            dws = [torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda") for _ in range(len(cstreams))]
+            copy_in = torch.cuda.Stream()
+            inputs_in = [torch.cuda.Event(), torch.cuda.Event()]  # step k's inputs are on the device
+            done = [torch.cuda.Event(), torch.cuda.Event()]       # step k's offsets are on the host
+            read = [torch.cuda.Event(), torch.cuda.Event()]       # step k's lists are on the host
+            copy = torch.cuda.Stream()
+            h2d = d2h = 0
+            n_warm, n_steps = 2, args.e2e_steps
 
-        torch.cuda.synchronize()
-        for k in range(n_warm + n_steps):
-            if k == n_warm:
-                t0 = time.perf_counter()
-            b = k & 1
-            buf = in_pinned[b]
-            # this input set's last user, step k - 2, has finished (its offsets were synchronised
-            # on in the previous iteration), so the packer and the copy may overwrite it
-            blob = emr.pack_population(full_pop, out=buf[ob:].numpy(), genomes=pack_range)
-            h2d = ob + len(blob)
-            emr.copy_async(in_dev[b], buf, h2d, copy_in)
-            inputs_in[b].record(copy_in)
-            stream.wait_event(inputs_in[b])
-            if k >= 2:
-                stream.wait_event(read[b])  # step k - 2's lists have left this output set
-            idx_o, w_o, cnt_o, off_o = outs[b]
-            emr.discover(blob, pack_dev[b], q_e2e[b], g, dsc.theta, dsc.band, dsc.w_min, dsc.mode, dsc.types, dws,
-                         idx_o, w_o, dsc.cap, cnt_o, off_o, stream=stream, qc=qc[b])
-            emr.copy_async(res_off[b], off_o, 8 * (dsc.n_pairs + 1), stream)
-            done[b].record(stream)
-            if k >= 1:
-                d2h = read_lists(k - 1)
-        d2h = read_lists(n_warm + n_steps - 1)
-        torch.cuda.synchronize()
-        elapsed = time.perf_counter() - t0
-        _, e2e_ms, e2e_value = aggregate(queries, elapsed / n_steps * 1e3, ws)
-        e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-               "ms_per_step": e2e_ms,
-               "pipeline": "two input and two output sets: each step packs into pinned memory on the host, "
-                           "copies its inputs on a copy stream while the previous step computes, and its lists "
-                           "are read on a second copy stream after step k+1 is queued; wall clock over %d steps"
-                           % n_steps}
+            def read_lists(k):
+                b = k & 1
+                done[b].synchronize()
+                n = min(int(res_off_np[b][-1]), dsc.cap)
+                copy.wait_event(done[b])
+                emr.copy_async(idx_h, outs[b][0], 4 * n, copy)
+                emr.copy_async(w_h, outs[b][1], 4 * n, copy)
+                read[b].record(copy)
+                return 8 * (dsc.n_pairs + 1) + 8 * n
+
+            torch.cuda.synchronize()
+            for k in range(n_warm + n_steps):
+                if k == n_warm:
+                    t0 = time.perf_counter()
+                b = k & 1
+                cs, wsp = cstreams[k % len(cstreams)], dws[k % len(cstreams)]
+                buf = in_pinned[b]
+                # this input set's last user, step k - 2, has finished (its offsets were synchronised
+                # on in the previous iteration), so the packer and the copy may overwrite it
+                blob = emr.pack_population(full_pop, out=buf[ob:].numpy(), genomes=pack_range)
+                h2d = ob + len(blob)
+                emr.copy_async(in_dev[b], buf, h2d, copy_in)
+                inputs_in[b].record(copy_in)
+                cs.wait_event(inputs_in[b])
+                if k >= 2:
+                    cs.wait_event(read[b])  # step k - 2's lists have left this output set
+                idx_o, w_o, cnt_o, off_o = outs[b]
+                emr.discover(blob, pack_dev[b], q_e2e[b], g, dsc.theta, dsc.band, dsc.w_min, dsc.mode, dsc.types,
+                             wsp, idx_o, w_o, dsc.cap, cnt_o, off_o, stream=cs, qc=qc[b])
+                emr.copy_async(res_off[b], off_o, 8 * (dsc.n_pairs + 1), cs)
+                done[b].record(cs)
+                if k >= 1:
+                    d2h = read_lists(k - 1)
+            d2h = read_lists(n_warm + n_steps - 1)
+            torch.cuda.synchronize()
+            elapsed = time.perf_counter() - t0
+            _, e2e_ms, e2e_value = aggregate(queries, elapsed / n_steps * 1e3, ws)
+            return {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "ms_per_step": e2e_ms, "compute_streams": n_compute,
+                    "pipeline": "two input and two output sets: each step packs into pinned memory on the host, "
+                                "copies its inputs on a copy stream while the previous step computes, and its "
+                                "lists are read on a second copy stream after step k+1 is queued; %s; wall "
+                                "clock over %d steps"
+                                % ("every step on one compute stream" if n_compute == 1 else
+                                   "steps alternate between two compute streams, each with its own workspace",
+                                   n_steps)}
+
+        # output set 0 is dsc's own buffers: the parity check below reads the lists an even step left there
+        one = e2e_run(1)
+        e2e = e2e_run(2)
+        e2e["one_stream"] = {"value": one["value"], "ms_per_step": one["ms_per_step"]}
 
     gather = None
     if ws > 1:

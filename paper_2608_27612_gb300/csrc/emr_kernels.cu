@@ -1559,13 +1559,14 @@ __global__ void __launch_bounds__(32 * kOneAxisWarps, kOneAxisBlocks) tile_kerne
 }
 
 // The 64 x 64 tiles of pairs with joint nodes (fused mode, no output buffer): a
-// warp per tile, kWarpTiles tiles at a time per CTA, no block barrier. The warp
-// fills its own node tables (the tile's 64 + 64 coordinates, two per lane and
-// axis), then each lane evaluates 32 sibling quads (quad l + 32 k: the lanes'
-// ballot for k is split word k of the tile) two per pass (one above 6 joint
-// nodes). A tile whose band screen fires (rare) evaluates its ring coordinates
-// and runs the band test with each quad's eight outer neighbours evaluated
-// directly; every other tile stores zero band words.
+// warp per tile, kWarpTiles tiles of one pair at a time per CTA. The warp fills
+// its own node tables (the tile's 64 + 64 coordinates, two per lane and axis),
+// then each lane evaluates 32 sibling quads (quad l + 32 k: the lanes' ballot
+// for k is split word k of the tile) two per pass (one above 6 joint nodes). A
+// tile whose band screen fires (rare) is left to the whole CTA after the warps'
+// tiles: its tables and ring again, its outputs into a shared tile (which takes
+// the place of the other warps' tables), and the band test from shared memory,
+// 128 threads at a time; every other tile stores zero band words.
 constexpr int kWarpTiles = 4;
 constexpr int warp_min_blocks(int njmax) { return njmax <= 4 ? 7 : njmax <= 8 ? 6 : 4; }
 
@@ -1583,9 +1584,14 @@ __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_
   __shared__ float4 s_ent[2][kDenseMax];
   __shared__ float2 s_esrc[2][kEntSrcCap];
   __shared__ __align__(16) float s_tab[kWarpTiles][2 * kDenseMax * kTabFull];
+  __shared__ int s_defer[kWarpTiles];  // the CTA's tiles whose band screen fired
+  __shared__ int s_ndefer;
+  static_assert(kWarpTiles >= 4 && (kWarpTiles - 1) * 2 * kDenseMax * kTabFull >= kWtFull,
+                "the shared output tile fits in the tables of warps 1..kWarpTiles-1");
   pdl_trigger();
   if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) pdl_wait();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) s_ndefer = 0;
   const int r = A.order[A.rank_beg + blockIdx.y];
   const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
   const int nv = reinterpret_cast<const int32_t*>(rec)[0];
@@ -1668,27 +1674,80 @@ __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_
       reinterpret_cast<uint4*>(band_t)[lane] = make_uint4(0u, 0u, 0u, 0u);
       continue;
     }
-    // a tile the band screen lets through (rare): the ring coordinates, then every quad's
-    // band test with its four children and eight outer neighbours evaluated directly
-    if (lane < 4) {
-      const int i = lane & 1 ? kTileSide : -1;
-      table_column(grid_coord((lane < 2 ? i0 : j0) + i, scale), i + 2, lane < 2 ? n_ent_x : n_ent_y,
-                   s_ent[lane >> 1], s_esrc[lane >> 1], lane < 2 ? tx : ty, kTabFull);
+    if (lane == 0) s_defer[atomicAdd(&s_ndefer, 1)] = tile;  // the CTA's band test, below
+  }
+  __syncthreads();  // every warp's tiles are done: the tables are free
+  const int n_defer = s_ndefer;
+  // A tile whose band screen fired: its band test by the whole CTA. Its tables (ring
+  // coordinates included) go to warp 0's slot, its outputs and ring into a shared tile
+  // over the other slots (position (i, j) at row j + kPad, column i + kPad), then each
+  // thread tests quads tid + 128 k from shared memory.
+  constexpr int P64 = kTileSide + 2 * kPad;
+  constexpr int NT = 32 * kWarpTiles;
+  float* s_wt = s_tab[1];
+  T.tx = s_tab[0];
+  T.ty = s_tab[0] + kDenseMax * kTabFull;
+  for (int q = 0; q < n_defer; q++) {
+    const int tile = s_defer[q];
+    int u = tile - 1, d = kPyramidTop + 1;
+    while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
+    const uint32_t mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
+    const int i0 = int(compact1by1(mb)), j0 = int(compact1by1(mb >> 1));
+    const float scale = __int_as_float((127 - (d + 1)) << 23);
+    if (q > 0) __syncthreads();  // the previous tile's reads of the tables and the shared tile are done
+    for (int v = tid; v < 2 * (kTileSide + 2); v += NT) {  // coordinates -1 .. 64 of each axis
+      const int ax = v / (kTileSide + 2), i = v % (kTileSide + 2) - 1;
+      table_column(grid_coord((ax ? j0 : i0) + i, scale), i + 2, ax ? n_ent_y : n_ent_x, s_ent[ax], s_esrc[ax],
+                   ax ? const_cast<float*>(T.ty) : const_cast<float*>(T.tx), kTabFull);
     }
-    __syncwarp();
+    __syncthreads();
+#pragma unroll 1
+    for (int k0 = 0; k0 < kTileSide * kTileSide / 4 / NT; k0 += QPE) {  // the tile's quads into the shared tile
+      float w[4 * QPE];
+      int xq[QPE], yq[QPE], so[QPE];
+#pragma unroll
+      for (int h = 0; h < QPE; h++) {
+        const uint32_t qi = uint32_t(tid + NT * (k0 + h));
+        const int px = int(compact1by1(qi)), py = int(compact1by1(qi >> 1));
+        xq[h] = 2 * px + 2;
+        yq[h] = 2 * py + 2;
+        so[h] = (2 * py + kPad) * P64 + 2 * px + kPad;
+      }
+      eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
+#pragma unroll
+      for (int h = 0; h < QPE; h++) {
+        *reinterpret_cast<float2*>(s_wt + so[h]) = make_float2(w[4 * h + 0], w[4 * h + 1]);
+        *reinterpret_cast<float2*>(s_wt + so[h] + P64) = make_float2(w[4 * h + 2], w[4 * h + 3]);
+      }
+    }
+    if (tid < kTileSide) {  // the ring: 4 sides x 64 points, four at a time
+      const int sd = tid >> 4, u0 = 4 * (tid & 15);
+      int li[4], lj[4], xp[4], yp[4];
+      float w[4];
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        li[c] = sd == 0 ? -1 : sd == 1 ? kTileSide : u0 + c;
+        lj[c] = sd == 2 ? -1 : sd == 3 ? kTileSide : u0 + c;
+        xp[c] = li[c] + 2;
+        yp[c] = lj[c] + 2;
+      }
+      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xp, yp, w);
+#pragma unroll
+      for (int c = 0; c < 4; c++) s_wt[(lj[c] + kPad) * P64 + li[c] + kPad] = w[c];
+    }
+    __syncthreads();
+    uint32_t* band_t = A.bandb + (band_base + A.word_off[d] + mb / 32);
     bool any_pass = false;
 #pragma unroll 1
-    for (int k = 0; k < 32; k++) {
-      const int x0 = xb + warp_quad_dx(k), y0 = yb + warp_quad_dy(k);  // child 0's table columns
-      const int xa[4] = {x0, x0 + 1, x0, x0 + 1}, ya[4] = {y0, y0, y0 + 1, y0 + 1};
-      const int xl[4] = {x0 - 1, x0 - 1, x0 + 2, x0 + 2}, yl[4] = {y0, y0 + 1, y0, y0 + 1};  // L0 L2 R1 R3
-      const int xv[4] = {x0, x0 + 1, x0, x0 + 1}, yv[4] = {y0 - 1, y0 - 1, y0 + 2, y0 + 2};  // B0 B1 U2 U3
-      float w[4], h[4], v[4];
-      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xa, ya, w);
-      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xl, yl, h);
-      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xv, yv, v);
-      const float L[4] = {h[0], w[0], h[1], w[2]}, R[4] = {w[1], h[2], w[3], h[3]};
-      const float Bo[4] = {v[0], v[1], w[0], w[1]}, U[4] = {w[2], w[3], v[2], v[3]};
+    for (int k = 0; k < kTileSide * kTileSide / 4 / NT; k++) {
+      const uint32_t qi = uint32_t(tid + NT * k);  // quad lane + 32 (warp + kWarpTiles k)
+      const int px = int(compact1by1(qi)), py = int(compact1by1(qi >> 1));
+      const float* t = s_wt + (2 * py + kPad) * P64 + 2 * px + kPad;  // child 0
+      const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
+      const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
+      const float w[4] = {w01.x, w01.y, w23.x, w23.y};
+      const float L[4] = {t[-1], w[0], t[P64 - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[P64 + 2]};
+      const float Bo[4] = {bel.x, bel.y, w[0], w[1]}, U[4] = {w[2], w[3], abv.x, abv.y};
       bool pass[4];
 #pragma unroll
       for (int c = 0; c < 4; c++) {
@@ -1698,9 +1757,10 @@ __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_
       const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
       const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
       any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
-      if (lane < 4) band_t[4 * k + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+      if (lane < 4)  // quad-major words of quads 32 kk .. 32 kk + 31, kk = warp + kWarpTiles k
+        band_t[4 * (warp + kWarpTiles * k) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
     }
-    if (A.tile_flags && lane == 0 && any_pass) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
+    if (__syncthreads_or(any_pass) && A.tile_flags && tid == 0) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
   }
 }
 
@@ -2598,7 +2658,8 @@ template <int NJMAX>
 emr_status launch_warp(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
   if (n_ranks <= 0 || A0.n_tiles <= 0) return EMR_OK;
   DTileArgs A = A0;
-  // a tile per warp: short CTAs balance best (measured against longer groups)
+  // a tile per warp: short CTAs balance best (measured against longer groups); the kernel
+  // keeps at most one deferred band test per warp
   const int g = kWarpTiles;
   A.tiles_per_cta = g;
   const unsigned gx = unsigned((A.n_tiles + g - 1) / g);
@@ -2621,9 +2682,8 @@ emr_status launch_joint_class(const DTileArgs& D, int64_t rank_beg, int64_t n_ra
   if (!warp_tiles) return launch_dense<NJMAX>(D, rank_beg, n_ranks, st, overlap);
   emr_status rc;
   const int32_t end = D.tile_beg + D.n_tiles;
-  // the block kernel takes the depths 0..4 tile and the one depth-5 tile, so that the
-  // warp kernel's tiles (depths 6..D: 4, 20, 84, ... of them) come in whole groups of kWarpTiles
-  const int32_t split_at = std::min<int32_t>(end, 2);
+  // the block kernel takes the depths 0..4 tile, the warp kernel the 64 x 64 tiles
+  const int32_t split_at = std::min<int32_t>(end, 1);
   if (D.tile_beg < split_at) {
     DTileArgs D0 = D;
     D0.n_tiles = split_at - D.tile_beg;
@@ -2758,15 +2818,15 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   // first rank of each joint class (12, 8, 6, 4 joint nodes at most)
   const int64_t b1 = p.n_class[0], b2 = b1 + p.n_class[1], b3 = b2 + p.n_class[2], b4 = b3 + p.n_class[3];
   int64_t beg = b4 + p.n_class[4];
-  if (warp_tiles && D.tile_beg < 2 && D.tile_beg + D.n_tiles > 2) {
-    // every joint class's block launch (depths 0..5), then every class's warp launch
-    // (depths 6..D): the block kernels' latency-bound CTAs then share the SMs with
+  if (warp_tiles && D.tile_beg < 1 && D.tile_beg + D.n_tiles > 1) {
+    // every joint class's block launch (the depths 0..4 tile), then every class's warp
+    // launch (depths 5..D): the block kernels' latency-bound CTAs then share the SMs with
     // the warp launches that follow them (measured faster than alternating block and
     // warp launches class by class)
     DTileArgs D0 = D, D1 = D;
-    D0.n_tiles = 2 - D.tile_beg;
-    D1.tile_beg = 2;
-    D1.n_tiles = D.tile_beg + D.n_tiles - 2;
+    D0.n_tiles = 1 - D.tile_beg;
+    D1.tile_beg = 1;
+    D1.n_tiles = D.tile_beg + D.n_tiles - 1;
     if ((rc = launch_dense<12>(D0, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_dense<8>(D0, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_dense<6>(D0, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;

@@ -2843,9 +2843,9 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   }
   if (mode == kModeFused && !out && p.n_class[5] > p.n_const) {
     // one-coordinate outputs: the depths 0..4 tile through the generic kernel, the 64 x 64
-    // tiles a warp each
+    // tiles (depths 5..D) a warp each
     const int64_t n5 = p.n_class[5] - p.n_const;
-    const int32_t split_at = std::min<int32_t>(tr.end, 2);
+    const int32_t split_at = std::min<int32_t>(tr.end, 1);
     if (tr.beg < split_at) {
       DTileArgs D0 = D;
       D0.n_tiles = split_at - tr.beg;

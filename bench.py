@@ -623,8 +623,8 @@ def oracle_samples(W):
 
 def launches_in_step(emr, dsc):
     """Kernel launches of one step: prepare (records, with the schedule in the last CTA); per
-    non-empty dense kernel class two tile launches (depths 0..5 on the block kernel, the
-    deeper 64 x 64 tiles a warp each), one for the interpreter class (constant-output
+    non-empty dense kernel class two tile launches (depths 0..4 on the block kernel, the
+    64 x 64 tiles of depths 5..D a warp each), one for the interpreter class (constant-output
     pairs need none: their tiles hold no band bit); selection (count, scan, write, kept
     weights). Memsets are not kernels."""
     _, gs, _, _ = emr.pack_records(dsc.pack)
@@ -634,9 +634,10 @@ def launches_in_step(emr, dsc):
             np.take_along_axis(gs[field], side.reshape(gs.shape[0], -1), axis=1)
         return f.astype(np.int64)
     nv, nj = per_pair("n_varying"), per_pair("n_joint")
-    cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 6, 2, np.where(nj > 4, 3, np.where(nj > 0, 4, 5)))))
+    cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 6, 2, np.where(nj > 4, 3, np.where(
+        nj > 2, 4, np.where(nj > 0, 5, 6))))))
     present = np.unique(cls[nv > 0])
-    per_class = [1 if c == 0 else (2 if dsc.grid.D >= 6 else 1) for c in present]
+    per_class = [1 if c == 0 else (2 if dsc.grid.D >= 5 else 1) for c in present]
     return 1 + sum(per_class) + 4
 
 

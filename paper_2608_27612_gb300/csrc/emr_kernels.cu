@@ -214,12 +214,13 @@ inline SpecLayout spec_layout(int nv_cap, int nve_cap) {
 // Kernel class of a pair by its varying-node count nv and its joint-node count
 // nj: 0 = interpreter (nv above kDenseMax); otherwise by the joint nodes, the
 // only ones evaluated per position: 1 = up to 12, 2 = up to 8, 3 = up to 6,
-// 4 = up to 4, 5 = none (the output depends on one coordinate, or on none:
-// constant outputs are the last pairs of class 5). Classes run in this order,
-// heaviest first.
-constexpr int kClasses = 6;
+// 4 = up to 4, 5 = up to 2, 6 = none (the output depends on one coordinate, or
+// on none: constant outputs are the last pairs of class 6). Classes run in this
+// order, heaviest first.
+constexpr int kClasses = 7;
+constexpr int kClassNone = kClasses - 1;
 __host__ __device__ __forceinline__ int pair_class(int nv, int nj) {
-  return nv > kDenseMax ? 0 : nj > 8 ? 1 : nj > 6 ? 2 : nj > 4 ? 3 : nj > 0 ? 4 : 5;
+  return nv > kDenseMax ? 0 : nj > 8 ? 1 : nj > 6 ? 2 : nj > 4 ? 3 : nj > 2 ? 4 : nj > 0 ? 5 : kClassNone;
 }
 
 // Header word 3 of a record: its kernel class (bits 0..3) and, when nv <=
@@ -2505,7 +2506,7 @@ GridDev grid_dev(const emr_grid* g) {
 struct EvalPlan {
   int64_t n_pairs;
   int64_t n_class[kClasses];  // pairs per kernel class (schedule order)
-  int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of class 5
+  int64_t n_const;            // pairs whose output is constant over the grid: the last ranks of kClassNone
   SpecLayout L;
   int32_t scratch_stride;
   size_t spec_bytes, scratch_bytes, order_bytes, sched_bytes, total;
@@ -2817,7 +2818,8 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   const bool warp_tiles = mode == kModeFused && !out;
   // first rank of each joint class (12, 8, 6, 4 joint nodes at most)
   const int64_t b1 = p.n_class[0], b2 = b1 + p.n_class[1], b3 = b2 + p.n_class[2], b4 = b3 + p.n_class[3];
-  int64_t beg = b4 + p.n_class[4];
+  const int64_t b5 = b4 + p.n_class[4];
+  int64_t beg = b5 + p.n_class[5];
   if (warp_tiles && D.tile_beg < 1 && D.tile_beg + D.n_tiles > 1) {
     // every joint class's block launch (the depths 0..4 tile), then every class's warp
     // launch (depths 5..D): the block kernels' latency-bound CTAs then share the SMs with
@@ -2831,20 +2833,23 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
     if ((rc = launch_dense<8>(D0, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_dense<6>(D0, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_dense<4>(D0, b4, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_dense<2>(D0, b5, p.n_class[5], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_warp<12>(D1, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_warp<8>(D1, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_warp<6>(D1, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_warp<4>(D1, b4, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_warp<2>(D1, b5, p.n_class[5], st, &overlap)) != EMR_OK) return rc;
   } else {
     if ((rc = launch_joint_class<12>(D, b1, p.n_class[1], st, &overlap, warp_tiles)) != EMR_OK) return rc;
     if ((rc = launch_joint_class<8>(D, b2, p.n_class[2], st, &overlap, warp_tiles)) != EMR_OK) return rc;
     if ((rc = launch_joint_class<6>(D, b3, p.n_class[3], st, &overlap, warp_tiles)) != EMR_OK) return rc;
     if ((rc = launch_joint_class<4>(D, b4, p.n_class[4], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+    if ((rc = launch_joint_class<2>(D, b5, p.n_class[5], st, &overlap, warp_tiles)) != EMR_OK) return rc;
   }
-  if (mode == kModeFused && !out && p.n_class[5] > p.n_const) {
+  if (mode == kModeFused && !out && p.n_class[kClassNone] > p.n_const) {
     // one-coordinate outputs: the depths 0..4 tile through the generic kernel, the 64 x 64
     // tiles (depths 5..D) a warp each
-    const int64_t n5 = p.n_class[5] - p.n_const;
+    const int64_t n5 = p.n_class[kClassNone] - p.n_const;
     const int32_t split_at = std::min<int32_t>(tr.end, 1);
     if (tr.beg < split_at) {
       DTileArgs D0 = D;
@@ -2859,14 +2864,14 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
       if ((rc = launch_one_axis(D1, beg, n5, st, &overlap)) != EMR_OK) return rc;
     }
   } else if (mode != kModeFused || p.n_const == 0) {
-    return launch_dense<0>(D, beg, p.n_class[5], st, &overlap);
-  } else if ((rc = launch_dense<0>(D, beg, p.n_class[5] - p.n_const, st, &overlap)) != EMR_OK) {
+    return launch_dense<0>(D, beg, p.n_class[kClassNone], st, &overlap);
+  } else if ((rc = launch_dense<0>(D, beg, p.n_class[kClassNone] - p.n_const, st, &overlap)) != EMR_OK) {
     return rc;
   }
   if (mode != kModeFused) return EMR_OK;
   // with tile flags, a constant-output pair has none set and its planes are never read: leave them
   if (tile_flags) return EMR_OK;
-  const int64_t c0 = beg + p.n_class[5] - p.n_const;
+  const int64_t c0 = beg + p.n_class[kClassNone] - p.n_const;
   for (int64_t r0 = 0; r0 < p.n_const; r0 += 65535) {  // grid y: pairs, at most 65535 a launch
     D.rank_beg = c0 + r0;
     const int64_t nc = std::min<int64_t>(65535, p.n_const - r0);

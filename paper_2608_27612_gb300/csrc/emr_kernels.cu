@@ -1034,6 +1034,213 @@ __device__ __forceinline__ uint32_t word_of_rows(uint32_t bits32, uint32_t w) {
 // CTAs resident per SM that each class is compiled for (bounds its registers).
 constexpr int dense_min_blocks(int njmax, int tpb) { return (njmax <= 4 ? 2048 : njmax <= 8 ? 1536 : 1024) / tpb / 2; }
 
+// The tile of depths 0..min(D, 4) of pair r (dense tile 0), by all TPB threads of the CTA:
+// in fused mode its split and band words and its tile flag, in materialise mode its outputs
+// and halo points. The pair's table programs, joint block and joint activations are in
+// shared memory (s_ent, s_esrc, s_WJ, s_jact); s_buf holds kWtPyr floats of padded
+// per-depth outputs, then the two axes' node tables (2 kDenseMax rows of kTabPyr).
+template <int NJMAX, int TPB>
+__device__ __forceinline__ void pyramid_tile(const DTileArgs& A, const int r, const int nv, const int nj,
+                                             const uint32_t xm, const uint32_t ym, const float out_const,
+                                             const float4 (*s_ent)[kDenseMax], const float2 (*s_esrc)[kEntSrcCap],
+                                             const float* s_WJ, const int* s_jact, float* s_buf) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t jm = ((1u << nv) - 1u) & ~(xm | ym);
+  const bool ax_x = (xm | jm) != 0u, ax_y = (ym | jm) != 0u;
+  const int n_ent_x = __popc((xm | jm) & ((1u << nv) - 1u)), n_ent_y = __popc((ym | jm) & ((1u << nv) - 1u));
+  const bool fused = A.mode == kModeFused;
+  const bool wfilter = A.w_min > 0.f;
+  const float theta16 = 16.f * A.theta, band2 = A.band * A.band;
+  uint32_t* split_row = A.split + int64_t(r) * A.n_words;
+  const int64_t band_base = int64_t(r) * A.band_stride - A.band_shift;
+  const int64_t prow = int64_t(r) * A.out_stride - A.out_shift;
+  const int d_hi = min(A.D, kPyramidTop);
+  float* s_wt = s_buf;
+  float* tab = s_buf + kWtPyr;
+  // node tables: depth e's coordinates -1 .. 2^(e+1) at columns tab_seg(e) + 1 ..
+  {
+    const int P = (4 << d_hi) - 2 + 2 * (d_hi + 1);  // sum over depths of 2^(d+1) + 2
+    const int n_items = (ax_x ? P : 0) + (ax_y ? P : 0);
+    for (int u = tid; u < n_items; u += TPB) {
+      const int a = ax_x && u < P ? 0 : 1;
+      int e = 0, v = a == 1 && ax_x ? u - P : u;
+      while (v >= (2 << e) + 2) { v -= (2 << e) + 2; e++; }
+      table_column(grid_coord(v - 1, __int_as_float((127 - (e + 1)) << 23)), tab_seg(e) + v + 1,
+                   a ? n_ent_y : n_ent_x, s_ent[a], s_esrc[a], tab + a * kDenseMax * kTabPyr, kTabPyr);
+    }
+  }
+  __syncthreads();
+  PairTabs T;
+  T.tx = tab;
+  T.ty = tab + kDenseMax * kTabPyr;
+  T.tw = kTabPyr;
+  T.nv = nv;
+  T.nj = nj;
+  T.out_x = nv > 0 && ((xm >> (nv - 1)) & 1u) != 0u;
+  T.orow = __popc(T.out_x ? xm : ym) - 1;  // an output of one coordinate (no joint node): its axis' last row
+  T.out_const = out_const;
+
+  // ---- tile 0: depths 0..min(D, 4). One pass evaluates the quads and ring points
+  // of every depth (work items: the quads of depth 0, 1, ..., then four ring
+  // points at a time), one barrier, then each depth is filtered from shared memory.
+  const bool ring = fused || A.out_halo != nullptr;
+  const int n_quads = ((4 << (2 * d_hi)) - 1) / 3;       // quads of depths 0..d_hi
+  const int n_items = n_quads + (ring ? (4 << d_hi) - 2 : 0);  // + ring groups (side / 4 ... of each depth)
+  // work item u's depth, its four points (li, lj) in that depth's grid (ring points
+  // outside [0, 2^(e+1))), and whether it is a quad
+  auto item_points = [&](int u, int& e, int (&li)[4], int (&lj)[4]) {
+    e = 0;
+    const bool quad = u < n_quads;
+    if (quad) {
+      while (((4 << (2 * e)) - 1) / 3 <= u) e++;
+      const uint32_t q = uint32_t(u - ((1 << (2 * e)) - 1) / 3);
+      const int pi = int(compact1by1(q)), pj = int(compact1by1(q >> 1));
+#pragma unroll
+      for (int c = 0; c < 4; c++) { li[c] = 2 * pi + (c & 1); lj[c] = 2 * pj + (c >> 1); }
+    } else {
+      const int g = u - n_quads;
+      while ((2 << (e + 1)) - 2 <= g) e++;
+      const int Te = 1 << (e + 1);
+#pragma unroll
+      for (int c = 0; c < 4; c++) {  // ring point t lies on side t / Te
+        const int t = 4 * (g - ((2 << e) - 2)) + c, sd = t >> (e + 1), uu = t & (Te - 1);
+        li[c] = sd == 0 ? -1 : sd == 1 ? Te : uu;
+        lj[c] = sd == 2 ? -1 : sd == 3 ? Te : uu;
+      }
+    }
+    return quad;
+  };
+  auto store_item = [&](int u, bool quad, int e, const int (&li)[4], const int (&lj)[4], const float* w) {
+    const int Te = 1 << (e + 1), pitch = Te + 2 * kPad;
+    if (fused) {
+      const int sb = wt_seg(e);  // this depth's padded grid in shared memory
+#pragma unroll
+      for (int c = 0; c < 4; c++) s_wt[sb + (lj[c] + kPad) * pitch + li[c] + kPad] = w[c];
+    } else if (quad) {
+      const uint32_t q = uint32_t(u - ((1 << (2 * e)) - 1) / 3);
+      *reinterpret_cast<float4*>(A.out + prow + A.level_off[e] + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
+    } else {
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        const int hs = li[c] < 0 ? 0 : li[c] >= Te ? 1 : lj[c] < 0 ? 2 : 3;
+        A.out_halo[int64_t(r) * A.n_halo + A.halo_off[e] + hs * Te + (hs < 2 ? lj[c] : li[c])] = w[c];
+      }
+    }
+  };
+  // IPT items a pass (their points evaluated together). Two measured slower than one (more
+  // registers and spills in the block kernel than the extra work in flight gains).
+  constexpr int IPT = 1;
+  for (int u0 = tid; u0 < n_items; u0 += IPT * TPB) {
+    int e[IPT], li[IPT][4], lj[IPT][4], xp[4 * IPT], yp[4 * IPT];
+    bool quad[IPT], valid[IPT];
+#pragma unroll
+    for (int k = 0; k < IPT; k++) {
+      const int u = u0 + k * TPB;
+      valid[k] = u < n_items;
+      quad[k] = item_points(valid[k] ? u : u0, e[k], li[k], lj[k]);  // past the end: item u0 again
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        xp[4 * k + c] = tab_seg(e[k]) + li[k][c] + 2;
+        yp[4 * k + c] = tab_seg(e[k]) + lj[k][c] + 2;
+      }
+    }
+    float w[4 * IPT];
+    eval_points<NJMAX, 4 * IPT>(T, s_WJ, s_jact, xp, yp, w);
+#pragma unroll
+    for (int k = 0; k < IPT; k++)
+      if (valid[k]) store_item(u0 + k * TPB, quad[k], e[k], li[k], lj[k], w + 4 * k);
+  }
+  if (!fused) return;
+  __syncthreads();
+  // Variance and band test of depths 0..d_hi, one item per quad: depths d_hi .. 3 in whole
+  // warps of 32 quads (their band words are quad-major), then depths 2, 1 and 0 packed into one
+  // warp (lanes 0-15, 16-19 and 20). The band screen of the 64 x 64 tiles applies: a quad with
+  // 16 V <= band^2 has no passing position, and the full test runs only in warps where some
+  // quad fails the screen.
+  int n_big = 0;
+  for (int e = kQuadMajorFrom; e <= d_hi; e++) n_big += 1 << (2 * e);
+  const int n_band_items = n_big + 32;
+  auto depth_of = [&](int u, int* q) {  // an item of the whole-warp depths
+    int e = d_hi;
+    while (u >= (1 << (2 * e))) { u -= 1 << (2 * e); e--; }
+    *q = u;
+    return e;
+  };
+  bool any_pass = false;
+  for (int base = 0; base < n_band_items; base += TPB) {
+    const int u = base + tid;
+    int e = -1, q = 0;
+    if (u < n_big) {
+      e = depth_of(u, &q);
+    } else if (u < n_band_items) {
+      const int v = u - n_big;
+      e = v < 16 ? 2 : v < 20 ? 1 : v == 20 ? 0 : -1;
+      q = v < 16 ? v : v < 20 ? v - 16 : 0;
+      if (e > d_hi) e = -1;
+    }
+    bool pass[4] = {false, false, false, false}, split = false, screened_out = true;
+    float w[4] = {0.f, 0.f, 0.f, 0.f};
+    const float* t = s_wt;
+    int pitch = 0;
+    if (e >= 0) {
+      const int Te = 1 << (e + 1);
+      const int sb = wt_seg(e);
+      pitch = Te + 2 * kPad;
+      const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
+      t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
+      w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
+      // the four children give the parent's variance (Section 3.2)
+      const float v16 = var16(w[0], w[1], w[2], w[3]);
+      split = v16 > theta16;
+      screened_out = v16 <= band2;
+    }
+    if (__any_sync(kFull, !screened_out) && !screened_out) {
+      const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
+      const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
+      const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]),
+                               band2);
+        if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+      }
+    }
+    const uint32_t bs = __ballot_sync(kFull, split);
+    const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+    const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+    any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
+    const int wbase = base + warp * 32;  // this warp's first item
+    if (wbase < n_big) {
+      int q0;
+      const int ew = depth_of(wbase, &q0);
+      if (lane == 0) split_row[A.word_off[ew - 1] + q0 / 32] = bs;
+      if (lane < 4)
+        A.bandb[band_base + A.word_off[ew] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
+    } else if (wbase == n_big) {  // depths 2, 1, 0: position-major words
+      if (d_hi >= 2) {
+        if (lane == 0) split_row[A.word_off[1]] = bs & 0xffffu;
+        if (lane < 2) A.bandb[band_base + A.word_off[2] + lane] = band_word(b0, b1, b2, b3, lane);
+      }
+      if (d_hi >= 1) {
+        if (lane == 2) split_row[A.word_off[0]] = (bs >> 16) & 0xfu;
+        if (lane == 3)
+          A.bandb[band_base + A.word_off[1]] = band_word((b0 >> 16) & 0xfu, (b1 >> 16) & 0xfu, (b2 >> 16) & 0xfu,
+                                                         (b3 >> 16) & 0xfu, 0);
+      }
+      if (lane == 4)
+        A.bandb[band_base + A.word_off[0]] = band_word((b0 >> 20) & 1u, (b1 >> 20) & 1u, (b2 >> 20) & 1u,
+                                                       (b3 >> 20) & 1u, 0);
+    }
+    if (A.out && e >= 0 && (pass[0] | pass[1] | pass[2] | pass[3])) {
+      const int64_t lrow = prow + A.level_off[e];
+#pragma unroll
+      for (int c = 0; c < 4; c++)
+        if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
+    }
+  }
+  if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense] = 1;
+}
+
 template <int NJMAX, int TPB>
 __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel_dense(const DTileArgs A) {
   static_assert(NJMAX <= kDenseMax, "joint block holds at most kDenseMax rows");
@@ -1100,10 +1307,14 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
 
   // ---- one tile of the pair
   auto run_tile = [&](const int tile) {
-    // geometry: a 64 x 64 tile of depth d >= 5 at Morton block mb; tile 0: depths 0..d_hi
+    if (tile == 0) {
+      pyramid_tile<NJMAX, TPB>(A, r, nv, nj, xm, ym, out_const, s_ent, s_esrc, s_WJ, s_jact, s_buf);
+      return;
+    }
+    // geometry: a 64 x 64 tile of depth d >= 5 at Morton block mb
     int d = 0, i0 = 0, j0 = 0;
     uint32_t mb = 0;
-    if (tile > 0) {
+    {
       int u = tile - 1;
       d = kPyramidTop + 1;
       while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
@@ -1111,30 +1322,21 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
       i0 = int(compact1by1(mb));
       j0 = int(compact1by1(mb >> 1));
     }
-    const int tw = tile > 0 ? kTabFull : kTabPyr;
-    float* tab = s_buf + (tile > 0 ? kWtFull : kWtPyr);
+    const int tw = kTabFull;
+    float* tab = s_buf + kWtFull;
     // node tables, one coordinate per thread. A 64 x 64 tile with nodes on one axis
     // takes its 66 coordinates (ring included); with both, the 64 + 64 inside the
     // tile, and the four ring coordinates only where a ring is evaluated.
     auto column = [&](int a, float cv, int pos) {
       table_column(cv, pos, a ? n_ent_y : n_ent_x, s_ent[a], s_esrc[a], tab + a * kDenseMax * tw, tw);
     };
-    if (tile > 0) {
+    {
       const float scale = __int_as_float((127 - (d + 1)) << 23);
       const int n_items = ax_x && ax_y ? 2 * kTileSide : (ax_x || ax_y) ? kTileSide + 2 : 0;
       for (int u = tid; u < n_items; u += TPB) {
         const int a = ax_x && ax_y ? u / kTileSide : ax_x ? 0 : 1;
         const int i = ax_x && ax_y ? u % kTileSide : u - 1;
         column(a, grid_coord((a ? j0 : i0) + i, scale), i + 2);
-      }
-    } else {
-      const int P = (4 << d_hi) - 2 + 2 * (d_hi + 1);  // sum over depths of 2^(d+1) + 2
-      const int n_items = (ax_x ? P : 0) + (ax_y ? P : 0);
-      for (int u = tid; u < n_items; u += TPB) {
-        const int a = ax_x && u < P ? 0 : 1;
-        int e = 0, v = a == 1 && ax_x ? u - P : u;
-        while (v >= (2 << e) + 2) { v -= (2 << e) + 2; e++; }
-        column(a, grid_coord(v - 1, __int_as_float((127 - (e + 1)) << 23)), tab_seg(e) + v + 1);
       }
     }
     __syncthreads();
@@ -1188,7 +1390,7 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
         return;
       }
     }
-    if (tile > 0) {
+    {
       // ---- a full 64 x 64 tile of one depth >= 5: 4 quads and 1 ring point per thread
       const int n = 1 << (d + 1);
       const int64_t lrow = prow + A.level_off[d];
@@ -1334,142 +1536,6 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
       return;
     }
 
-    // ---- tile 0: depths 0..min(D, 4). One pass evaluates the quads and ring points
-    // of every depth (work items: the quads of depth 0, 1, ..., then four ring
-    // points at a time), one barrier, then each depth is filtered from shared memory.
-    const bool ring = fused || A.out_halo != nullptr;
-    const int n_quads = ((4 << (2 * d_hi)) - 1) / 3;       // quads of depths 0..d_hi
-    const int n_items = n_quads + (ring ? (4 << d_hi) - 2 : 0);  // + ring groups (side / 4 ... of each depth)
-    for (int u = tid; u < n_items; u += TPB) {
-      int e = 0, li[4], lj[4];
-      bool quad = u < n_quads;
-      if (quad) {
-        while (((4 << (2 * e)) - 1) / 3 <= u) e++;
-        const uint32_t q = uint32_t(u - ((1 << (2 * e)) - 1) / 3);
-        const int pi = int(compact1by1(q)), pj = int(compact1by1(q >> 1));
-#pragma unroll
-        for (int c = 0; c < 4; c++) { li[c] = 2 * pi + (c & 1); lj[c] = 2 * pj + (c >> 1); }
-      } else {
-        const int g = u - n_quads;
-        while ((2 << (e + 1)) - 2 <= g) e++;
-        const int Te = 1 << (e + 1);
-#pragma unroll
-        for (int c = 0; c < 4; c++) {  // ring point t lies on side t / Te
-          const int t = 4 * (g - ((2 << e) - 2)) + c, sd = t >> (e + 1), uu = t & (Te - 1);
-          li[c] = sd == 0 ? -1 : sd == 1 ? Te : uu;
-          lj[c] = sd == 2 ? -1 : sd == 3 ? Te : uu;
-        }
-      }
-      const int Te = 1 << (e + 1), pitch = Te + 2 * kPad;
-      int xp[4], yp[4];
-#pragma unroll
-      for (int c = 0; c < 4; c++) { xp[c] = tab_seg(e) + li[c] + 2; yp[c] = tab_seg(e) + lj[c] + 2; }
-      float w[4];
-      eval_points<NJMAX, 4>(T, s_WJ, s_jact, xp, yp, w);
-      if (fused) {
-        const int sb = wt_seg(e);  // this depth's padded grid in shared memory
-#pragma unroll
-        for (int c = 0; c < 4; c++) s_wt[sb + (lj[c] + kPad) * pitch + li[c] + kPad] = w[c];
-      } else if (quad) {
-        const uint32_t q = uint32_t(u - ((1 << (2 * e)) - 1) / 3);
-        *reinterpret_cast<float4*>(A.out + prow + A.level_off[e] + 4 * q) = make_float4(w[0], w[1], w[2], w[3]);
-      } else {
-#pragma unroll
-        for (int c = 0; c < 4; c++) {
-          const int hs = li[c] < 0 ? 0 : li[c] >= Te ? 1 : lj[c] < 0 ? 2 : 3;
-          A.out_halo[int64_t(r) * A.n_halo + A.halo_off[e] + hs * Te + (hs < 2 ? lj[c] : li[c])] = w[c];
-        }
-      }
-    }
-    if (!fused) return;
-    __syncthreads();
-    // Variance and band test of depths 0..d_hi, one item per quad: depths d_hi .. 3 in whole
-    // warps of 32 quads (their band words are quad-major), then depths 2, 1 and 0 packed into one
-    // warp (lanes 0-15, 16-19 and 20). The band screen of the 64 x 64 tiles applies: a quad with
-    // 16 V <= band^2 has no passing position, and the full test runs only in warps where some
-    // quad fails the screen.
-    int n_big = 0;
-    for (int e = kQuadMajorFrom; e <= d_hi; e++) n_big += 1 << (2 * e);
-    const int n_band_items = n_big + 32;
-    auto depth_of = [&](int u, int* q) {  // an item of the whole-warp depths
-      int e = d_hi;
-      while (u >= (1 << (2 * e))) { u -= 1 << (2 * e); e--; }
-      *q = u;
-      return e;
-    };
-    bool any_pass = false;
-    for (int base = 0; base < n_band_items; base += TPB) {
-      const int u = base + tid;
-      int e = -1, q = 0;
-      if (u < n_big) {
-        e = depth_of(u, &q);
-      } else if (u < n_band_items) {
-        const int v = u - n_big;
-        e = v < 16 ? 2 : v < 20 ? 1 : v == 20 ? 0 : -1;
-        q = v < 16 ? v : v < 20 ? v - 16 : 0;
-        if (e > d_hi) e = -1;
-      }
-      bool pass[4] = {false, false, false, false}, split = false, screened_out = true;
-      float w[4] = {0.f, 0.f, 0.f, 0.f};
-      const float* t = s_wt;
-      int pitch = 0;
-      if (e >= 0) {
-        const int Te = 1 << (e + 1);
-        const int sb = wt_seg(e);
-        pitch = Te + 2 * kPad;
-        const int pi = int(compact1by1(uint32_t(q))), pj = int(compact1by1(uint32_t(q) >> 1));
-        t = s_wt + sb + (2 * pj + kPad) * pitch + 2 * pi + kPad;
-        w[0] = t[0]; w[1] = t[1]; w[2] = t[pitch]; w[3] = t[pitch + 1];
-        // the four children give the parent's variance (Section 3.2)
-        const float v16 = var16(w[0], w[1], w[2], w[3]);
-        split = v16 > theta16;
-        screened_out = v16 <= band2;
-      }
-      if (__any_sync(kFull, !screened_out) && !screened_out) {
-        const float L[4] = {t[-1], w[0], t[pitch - 1], w[2]}, R[4] = {w[1], t[2], w[3], t[pitch + 2]};
-        const float Bo[4] = {t[-pitch], t[-pitch + 1], w[0], w[1]};
-        const float U[4] = {w[2], w[3], t[2 * pitch], t[2 * pitch + 1]};
-#pragma unroll
-        for (int c = 0; c < 4; c++) {
-          pass[c] = band_pass_sq(sqdiff(w[c], L[c]), sqdiff(w[c], R[c]), sqdiff(w[c], Bo[c]), sqdiff(w[c], U[c]),
-                                 band2);
-          if (wfilter) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
-        }
-      }
-      const uint32_t bs = __ballot_sync(kFull, split);
-      const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
-      const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-      any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
-      const int wbase = base + warp * 32;  // this warp's first item
-      if (wbase < n_big) {
-        int q0;
-        const int ew = depth_of(wbase, &q0);
-        if (lane == 0) split_row[A.word_off[ew - 1] + q0 / 32] = bs;
-        if (lane < 4)
-          A.bandb[band_base + A.word_off[ew] + 4 * (q0 / 32) + lane] = lane == 0 ? b0 : lane == 1 ? b1 : lane == 2 ? b2 : b3;
-      } else if (wbase == n_big) {  // depths 2, 1, 0: position-major words
-        if (d_hi >= 2) {
-          if (lane == 0) split_row[A.word_off[1]] = bs & 0xffffu;
-          if (lane < 2) A.bandb[band_base + A.word_off[2] + lane] = band_word(b0, b1, b2, b3, lane);
-        }
-        if (d_hi >= 1) {
-          if (lane == 2) split_row[A.word_off[0]] = (bs >> 16) & 0xfu;
-          if (lane == 3)
-            A.bandb[band_base + A.word_off[1]] = band_word((b0 >> 16) & 0xfu, (b1 >> 16) & 0xfu, (b2 >> 16) & 0xfu,
-                                                           (b3 >> 16) & 0xfu, 0);
-        }
-        if (lane == 4)
-          A.bandb[band_base + A.word_off[0]] = band_word((b0 >> 20) & 1u, (b1 >> 20) & 1u, (b2 >> 20) & 1u,
-                                                         (b3 >> 20) & 1u, 0);
-      }
-      if (A.out && e >= 0 && (pass[0] | pass[1] | pass[2] | pass[3])) {
-        const int64_t lrow = prow + A.level_off[e];
-#pragma unroll
-        for (int c = 0; c < 4; c++)
-          if (pass[c]) A.out[lrow + 4 * q + c] = w[c];
-      }
-    }
-    if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense] = 1;
   };
 
   for (int t = t_beg; t < t_end; t++) {

@@ -637,7 +637,7 @@ def launches_in_step(emr, dsc):
     cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 6, 2, np.where(nj > 4, 3, np.where(
         nj > 2, 4, np.where(nj > 0, 5, 6))))))
     present = np.unique(cls[nv > 0])
-    per_class = [1 if c == 0 else (2 if dsc.grid.D >= 5 else 1) for c in present]
+    per_class = [1 if c == 0 else (2 if dsc.grid.D >= 6 else 1) for c in present]
     return 1 + sum(per_class) + 4
 
 

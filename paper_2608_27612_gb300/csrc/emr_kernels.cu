@@ -1307,235 +1307,233 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
 
   // ---- one tile of the pair
   auto run_tile = [&](const int tile) {
-    if (tile == 0) {
-      pyramid_tile<NJMAX, TPB>(A, r, nv, nj, xm, ym, out_const, s_ent, s_esrc, s_WJ, s_jact, s_buf);
-      return;
-    }
-    // geometry: a 64 x 64 tile of depth d >= 5 at Morton block mb
-    int d = 0, i0 = 0, j0 = 0;
-    uint32_t mb = 0;
-    {
-      int u = tile - 1;
-      d = kPyramidTop + 1;
-      while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
-      mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
-      i0 = int(compact1by1(mb));
-      j0 = int(compact1by1(mb >> 1));
-    }
-    const int tw = kTabFull;
-    float* tab = s_buf + kWtFull;
-    // node tables, one coordinate per thread. A 64 x 64 tile with nodes on one axis
-    // takes its 66 coordinates (ring included); with both, the 64 + 64 inside the
-    // tile, and the four ring coordinates only where a ring is evaluated.
-    auto column = [&](int a, float cv, int pos) {
-      table_column(cv, pos, a ? n_ent_y : n_ent_x, s_ent[a], s_esrc[a], tab + a * kDenseMax * tw, tw);
-    };
-    {
-      const float scale = __int_as_float((127 - (d + 1)) << 23);
-      const int n_items = ax_x && ax_y ? 2 * kTileSide : (ax_x || ax_y) ? kTileSide + 2 : 0;
-      for (int u = tid; u < n_items; u += TPB) {
-        const int a = ax_x && ax_y ? u / kTileSide : ax_x ? 0 : 1;
-        const int i = ax_x && ax_y ? u % kTileSide : u - 1;
-        column(a, grid_coord((a ? j0 : i0) + i, scale), i + 2);
+    if (tile > 0) {  // a 64 x 64 tile; tile 0 (depths 0..4) below
+      // geometry: a 64 x 64 tile of depth d >= 5 at Morton block mb
+      int d = 0, i0 = 0, j0 = 0;
+      uint32_t mb = 0;
+      {
+        int u = tile - 1;
+        d = kPyramidTop + 1;
+        while (u >= (1 << (2 * (d - kPyramidTop - 1)))) { u -= 1 << (2 * (d - kPyramidTop - 1)); d++; }
+        mb = uint32_t(u) * uint32_t(kTileSide * kTileSide);
+        i0 = int(compact1by1(mb));
+        j0 = int(compact1by1(mb >> 1));
       }
-    }
-    __syncthreads();
-    // the ring coordinates of a 64 x 64 tile with nodes on both axes (CTA-uniform call)
-    auto ring_columns = [&]() {
-      if (ax_x && ax_y) {
-        if (tid < 4) {
-          const int a = tid >> 1, i = tid & 1 ? kTileSide : -1;
-          column(a, grid_coord((a ? j0 : i0) + i, __int_as_float((127 - (d + 1)) << 23)), i + 2);
+      const int tw = kTabFull;
+      float* tab = s_buf + kWtFull;
+      // node tables, one coordinate per thread. A 64 x 64 tile with nodes on one axis
+      // takes its 66 coordinates (ring included); with both, the 64 + 64 inside the
+      // tile, and the four ring coordinates only where a ring is evaluated.
+      auto column = [&](int a, float cv, int pos) {
+        table_column(cv, pos, a ? n_ent_y : n_ent_x, s_ent[a], s_esrc[a], tab + a * kDenseMax * tw, tw);
+      };
+      {
+        const float scale = __int_as_float((127 - (d + 1)) << 23);
+        const int n_items = ax_x && ax_y ? 2 * kTileSide : (ax_x || ax_y) ? kTileSide + 2 : 0;
+        for (int u = tid; u < n_items; u += TPB) {
+          const int a = ax_x && ax_y ? u / kTileSide : ax_x ? 0 : 1;
+          const int i = ax_x && ax_y ? u % kTileSide : u - 1;
+          column(a, grid_coord((a ? j0 : i0) + i, scale), i + 2);
         }
-        __syncthreads();
       }
-    };
-    PairTabs T;
-    T.tx = tab;
-    T.ty = tab + kDenseMax * tw;
-    T.tw = tw;
-    T.nv = nv;
-    T.nj = nj;
-    T.out_x = nv > 0 && ((xm >> (nv - 1)) & 1u) != 0u;
-    T.orow = __popc(T.out_x ? xm : ym) - 1;  // an output of one coordinate (no joint node): its axis' last row
-    T.out_const = out_const;
-
-    if constexpr (NJMAX == 0) {
-      if (tile > 0 && fused && !A.out && nv > 0) {
-        // ---- a 64 x 64 tile whose output f depends on one coordinate: every quad of a
-        // column pair (x) or row pair (y) has the children f0, f1 (twice), so its
-        // variance is 16 V = 4 (f0 - f1)^2 (the six-difference sum, exactly), and a
-        // position's band value is the smaller squared difference to its two
-        // neighbours along that coordinate (the other axis gives 0). Each warp takes
-        // the 32 pairs (one per lane) and writes a quarter of the tile's words.
-        const float* f = (T.out_x ? T.tx : T.ty) + T.orow * kTabFull;  // coordinate i at i + 2
-        const float fl = f[2 * lane + 1], f0 = f[2 * lane + 2], f1 = f[2 * lane + 3], fr = f[2 * lane + 4];
-        const float s01 = sqdiff(f0, f1);
-        bool g0 = fminf(sqdiff(f0, fl), s01) > band2, g1 = fminf(s01, sqdiff(f1, fr)) > band2;
-        if (wfilter) {
-          g0 = g0 && fabsf(f0) > A.w_min;
-          g1 = g1 && fabsf(f1) > A.w_min;
-        }
-        const uint32_t S = __ballot_sync(kFull, 4.f * s01 > theta16);
-        const uint32_t G0 = __ballot_sync(kFull, g0), G1 = __ballot_sync(kFull, g1);
-        // band word 4 j + c holds child c of the quads of split word j: child c lies in the
-        // pair's first or second column (c & 1) or row (c >> 1)
-        const uint32_t j = uint32_t(tid) >> 2, c = uint32_t(tid) & 3u;
-        const uint32_t gsel = (T.out_x ? (c & 1u) : (c >> 1)) ? G1 : G0;
-        A.bandb[band_base + A.word_off[d] + mb / 32 + tid] = T.out_x ? word_of_columns(gsel, j) : word_of_rows(gsel, j);
-        if (tid < 32)
-          split_row[A.word_off[d - 1] + mb / 128 + tid] =
-              T.out_x ? word_of_columns(S, uint32_t(tid)) : word_of_rows(S, uint32_t(tid));
-        if (A.tile_flags && tid == 0 && (G0 | G1) != 0u) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
-        return;
-      }
-    }
-    {
-      // ---- a full 64 x 64 tile of one depth >= 5: 4 quads and 1 ring point per thread
-      const int n = 1 << (d + 1);
-      const int64_t lrow = prow + A.level_off[d];
-      // quad q = tid + TPB k of the tile has parent (pl + dx(k), ql + dy(k)), where
-      // (dx, dy) are the Morton coordinates of TPB k (its bits lie above tid's)
-      const int pl = int(compact1by1(uint32_t(tid))), ql = int(compact1by1(uint32_t(tid) >> 1));
-      const int xb = 2 * pl + 2, yb = 2 * ql + 2;  // table columns of this thread's quad k = 0
-      const int sbase = (2 * ql + kPad) * P64 + 2 * pl + kPad;
-      uint32_t* split_k = split_row + A.word_off[d - 1] + mb / 128 + warp;  // this warp's parents, k = 0
-      uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
-      // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the joint nodes
-      constexpr int QPE = NJMAX <= 6 ? 2 : 1;
-      // A position passes the band test only if both differences along one axis
-      // exceed the band, and one of them is to its sibling in the quad. The sum of the
-      // six squared sibling differences (16 V, rounded upward monotonically) bounds
-      // each of them, so a quad with 16 V within band^2 has no passing position,
-      // whatever its neighbours; need: some quad of this thread may have one.
-      bool need = false;
-#pragma unroll 1
-      for (int k0 = 0; k0 < QPT; k0 += QPE) {
-        float w[4 * QPE];
-        int4 kq[QPE];
-        int xq[QPE], yq[QPE];
-#pragma unroll
-        for (int h = 0; h < QPE; h++) {
-          kq[h] = s_kq[k0 + h];
-          xq[h] = xb + kq[h].x;
-          yq[h] = yb + kq[h].y;
-        }
-        eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
-#pragma unroll
-        for (int h = 0; h < QPE; h++) {
-          const int k = k0 + h;
-          const float* wq = w + 4 * h;
-          if (fused) {
-            // the four children give the parent's variance (Section 3.2)
-            const float v16 = var16(wq[0], wq[1], wq[2], wq[3]);
-            const unsigned bal = __ballot_sync(kFull, v16 > theta16);
-            if (lane == 0) split_k[(TPB / 32) * k] = bal;
-            need = need || !(v16 <= band2);
-          } else {
-            *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
-                make_float4(wq[0], wq[1], wq[2], wq[3]);
+      __syncthreads();
+      // the ring coordinates of a 64 x 64 tile with nodes on both axes (CTA-uniform call)
+      auto ring_columns = [&]() {
+        if (ax_x && ax_y) {
+          if (tid < 4) {
+            const int a = tid >> 1, i = tid & 1 ? kTileSide : -1;
+            column(a, grid_coord((a ? j0 : i0) + i, __int_as_float((127 - (d + 1)) << 23)), i + 2);
           }
+          __syncthreads();
+        }
+      };
+      PairTabs T;
+      T.tx = tab;
+      T.ty = tab + kDenseMax * tw;
+      T.tw = tw;
+      T.nv = nv;
+      T.nj = nj;
+      T.out_x = nv > 0 && ((xm >> (nv - 1)) & 1u) != 0u;
+      T.orow = __popc(T.out_x ? xm : ym) - 1;  // an output of one coordinate (no joint node): its axis' last row
+      T.out_const = out_const;
+
+      if constexpr (NJMAX == 0) {
+        if (tile > 0 && fused && !A.out && nv > 0) {
+          // ---- a 64 x 64 tile whose output f depends on one coordinate: every quad of a
+          // column pair (x) or row pair (y) has the children f0, f1 (twice), so its
+          // variance is 16 V = 4 (f0 - f1)^2 (the six-difference sum, exactly), and a
+          // position's band value is the smaller squared difference to its two
+          // neighbours along that coordinate (the other axis gives 0). Each warp takes
+          // the 32 pairs (one per lane) and writes a quarter of the tile's words.
+          const float* f = (T.out_x ? T.tx : T.ty) + T.orow * kTabFull;  // coordinate i at i + 2
+          const float fl = f[2 * lane + 1], f0 = f[2 * lane + 2], f1 = f[2 * lane + 3], fr = f[2 * lane + 4];
+          const float s01 = sqdiff(f0, f1);
+          bool g0 = fminf(sqdiff(f0, fl), s01) > band2, g1 = fminf(s01, sqdiff(f1, fr)) > band2;
+          if (wfilter) {
+            g0 = g0 && fabsf(f0) > A.w_min;
+            g1 = g1 && fabsf(f1) > A.w_min;
+          }
+          const uint32_t S = __ballot_sync(kFull, 4.f * s01 > theta16);
+          const uint32_t G0 = __ballot_sync(kFull, g0), G1 = __ballot_sync(kFull, g1);
+          // band word 4 j + c holds child c of the quads of split word j: child c lies in the
+          // pair's first or second column (c & 1) or row (c >> 1)
+          const uint32_t j = uint32_t(tid) >> 2, c = uint32_t(tid) & 3u;
+          const uint32_t gsel = (T.out_x ? (c & 1u) : (c >> 1)) ? G1 : G0;
+          A.bandb[band_base + A.word_off[d] + mb / 32 + tid] = T.out_x ? word_of_columns(gsel, j) : word_of_rows(gsel, j);
+          if (tid < 32)
+            split_row[A.word_off[d - 1] + mb / 128 + tid] =
+                T.out_x ? word_of_columns(S, uint32_t(tid)) : word_of_rows(S, uint32_t(tid));
+          if (A.tile_flags && tid == 0 && (G0 | G1) != 0u) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
+          return;
         }
       }
-      if (fused && !__syncthreads_or(need)) {  // no position of the tile can pass
-        if (lane == 0)
-          for (int k = 0; k < QPT; k++) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
-        return;
-      }
-      if (fused || A.out_halo) ring_columns();
-      if (fused) {  // a tile the band screen lets through (rare): its outputs again, into the shared tile
-#pragma unroll 1
+      {
+        // ---- a full 64 x 64 tile of one depth >= 5: 4 quads and 1 ring point per thread
+        const int n = 1 << (d + 1);
+        const int64_t lrow = prow + A.level_off[d];
+        // quad q = tid + TPB k of the tile has parent (pl + dx(k), ql + dy(k)), where
+        // (dx, dy) are the Morton coordinates of TPB k (its bits lie above tid's)
+        const int pl = int(compact1by1(uint32_t(tid))), ql = int(compact1by1(uint32_t(tid) >> 1));
+        const int xb = 2 * pl + 2, yb = 2 * ql + 2;  // table columns of this thread's quad k = 0
+        const int sbase = (2 * ql + kPad) * P64 + 2 * pl + kPad;
+        uint32_t* split_k = split_row + A.word_off[d - 1] + mb / 128 + warp;  // this warp's parents, k = 0
+        uint32_t* band_k = A.bandb + (band_base + A.word_off[d] + 4 * (mb / 128 + warp));
+        // QPE quads per evaluation: quads k .. k + QPE - 1 share one pass over the joint nodes
+        constexpr int QPE = NJMAX <= 6 ? 2 : 1;
+        // A position passes the band test only if both differences along one axis
+        // exceed the band, and one of them is to its sibling in the quad. The sum of the
+        // six squared sibling differences (16 V, rounded upward monotonically) bounds
+        // each of them, so a quad with 16 V within band^2 has no passing position,
+        // whatever its neighbours; need: some quad of this thread may have one.
+        bool need = false;
+  #pragma unroll 1
         for (int k0 = 0; k0 < QPT; k0 += QPE) {
           float w[4 * QPE];
           int4 kq[QPE];
           int xq[QPE], yq[QPE];
-#pragma unroll
+  #pragma unroll
           for (int h = 0; h < QPE; h++) {
             kq[h] = s_kq[k0 + h];
             xq[h] = xb + kq[h].x;
             yq[h] = yb + kq[h].y;
           }
           eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
-#pragma unroll
+  #pragma unroll
           for (int h = 0; h < QPE; h++) {
-            float* t = s_wt + sbase + kq[h].z;
-            *reinterpret_cast<float2*>(t) = make_float2(w[4 * h + 0], w[4 * h + 1]);
-            *reinterpret_cast<float2*>(t + P64) = make_float2(w[4 * h + 2], w[4 * h + 3]);
-          }
-        }
-      }
-      // ring: 4 sides x 64 points, evaluated four at a time by threads 0..63
-      // (point t = 4 tid + c lies on side t / 64, the same for all four)
-      if (tid < kTileSide && (fused || A.out_halo)) {
-        const int sd = tid >> 4, u0 = 4 * (tid & 15);
-        int li[4], lj[4], xp[4], yp[4];
-        float w[4];
-#pragma unroll
-        for (int c = 0; c < 4; c++) {
-          li[c] = sd == 0 ? -1 : sd == 1 ? kTileSide : u0 + c;
-          lj[c] = sd == 2 ? -1 : sd == 3 ? kTileSide : u0 + c;
-          xp[c] = li[c] + 2;
-          yp[c] = lj[c] + 2;
-        }
-        const int gi = i0 + li[0], gj = j0 + lj[0];  // a side lies wholly inside or outside the domain
-        const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
-        if (fused || outside) {  // materialised: only points outside the domain are written
-          eval_points<NJMAX, 4>(T, s_WJ, s_jact, xp, yp, w);
-#pragma unroll
-          for (int c = 0; c < 4; c++) {
+            const int k = k0 + h;
+            const float* wq = w + 4 * h;
             if (fused) {
-              s_wt[(lj[c] + kPad) * P64 + li[c] + kPad] = w[c];
+              // the four children give the parent's variance (Section 3.2)
+              const float v16 = var16(wq[0], wq[1], wq[2], wq[3]);
+              const unsigned bal = __ballot_sync(kFull, v16 > theta16);
+              if (lane == 0) split_k[(TPB / 32) * k] = bal;
+              need = need || !(v16 <= band2);
             } else {
-              const int pi_ = i0 + li[c], pj_ = j0 + lj[c];
-              const int hs = pi_ < 0 ? 0 : pi_ >= n ? 1 : pj_ < 0 ? 2 : 3;
-              A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? pj_ : pi_)] = w[c];
+              *reinterpret_cast<float4*>(A.out + lrow + mb + 4 * (tid + TPB * k)) =
+                  make_float4(wq[0], wq[1], wq[2], wq[3]);
             }
           }
         }
-      }
-      if (!fused) return;
-      __syncthreads();
-      // band value of each position from its four neighbours at distance 2^-d
-      bool any_pass = false;
-#pragma unroll 2
-      for (int k = 0; k < QPT; k++) {
-        const float* t = s_wt + sbase + s_kq[k].z;  // (2pi, 2pj)
-        const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
-        const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
-        const float l0 = t[-1], l2 = t[P64 - 1], r1 = t[2], r3 = t[P64 + 2];
-        const float w[4] = {w01.x, w01.y, w23.x, w23.y};
-        const float L[4] = {l0, w[0], l2, w[2]}, R[4] = {w[1], r1, w[3], r3};
-        const float Bo[4] = {bel.x, bel.y, w[0], w[1]}, U[4] = {w[2], w[3], abv.x, abv.y};
-        bool pass[4];
-        // squared differences between siblings are shared by both
-        const float h01 = sqdiff(w[0], w[1]), h23 = sqdiff(w[2], w[3]);
-        const float v02 = sqdiff(w[0], w[2]), v13 = sqdiff(w[1], w[3]);
-        const float DL[4] = {sqdiff(w[0], L[0]), h01, sqdiff(w[2], L[2]), h23};
-        const float DR[4] = {h01, sqdiff(w[1], R[1]), h23, sqdiff(w[3], R[3])};
-        const float DB[4] = {sqdiff(w[0], Bo[0]), sqdiff(w[1], Bo[1]), v02, v13};
-        const float DT[4] = {v02, v13, sqdiff(w[2], U[2]), sqdiff(w[3], U[3])};
-#pragma unroll
-        for (int c = 0; c < 4; c++) pass[c] = band_pass_sq(DL[c], DR[c], DB[c], DT[c], band2);
-        if (wfilter) {
-#pragma unroll
-          for (int c = 0; c < 4; c++) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+        if (fused && !__syncthreads_or(need)) {  // no position of the tile can pass
+          if (lane == 0)
+            for (int k = 0; k < QPT; k++) *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(0, 0, 0, 0);
+          return;
         }
-        const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
-        const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
-        any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
-        if (lane == 0)  // the four quad-major words of this warp's 32 quads
-          *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(b0, b1, b2, b3);
-        if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
-          float* o = A.out + lrow + mb + 4 * (tid + TPB * k);
-#pragma unroll
-          for (int c = 0; c < 4; c++)
-            if (pass[c]) o[c] = w[c];
+        if (fused || A.out_halo) ring_columns();
+        if (fused) {  // a tile the band screen lets through (rare): its outputs again, into the shared tile
+  #pragma unroll 1
+          for (int k0 = 0; k0 < QPT; k0 += QPE) {
+            float w[4 * QPE];
+            int4 kq[QPE];
+            int xq[QPE], yq[QPE];
+  #pragma unroll
+            for (int h = 0; h < QPE; h++) {
+              kq[h] = s_kq[k0 + h];
+              xq[h] = xb + kq[h].x;
+              yq[h] = yb + kq[h].y;
+            }
+            eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
+  #pragma unroll
+            for (int h = 0; h < QPE; h++) {
+              float* t = s_wt + sbase + kq[h].z;
+              *reinterpret_cast<float2*>(t) = make_float2(w[4 * h + 0], w[4 * h + 1]);
+              *reinterpret_cast<float2*>(t + P64) = make_float2(w[4 * h + 2], w[4 * h + 3]);
+            }
+          }
         }
+        // ring: 4 sides x 64 points, evaluated four at a time by threads 0..63
+        // (point t = 4 tid + c lies on side t / 64, the same for all four)
+        if (tid < kTileSide && (fused || A.out_halo)) {
+          const int sd = tid >> 4, u0 = 4 * (tid & 15);
+          int li[4], lj[4], xp[4], yp[4];
+          float w[4];
+  #pragma unroll
+          for (int c = 0; c < 4; c++) {
+            li[c] = sd == 0 ? -1 : sd == 1 ? kTileSide : u0 + c;
+            lj[c] = sd == 2 ? -1 : sd == 3 ? kTileSide : u0 + c;
+            xp[c] = li[c] + 2;
+            yp[c] = lj[c] + 2;
+          }
+          const int gi = i0 + li[0], gj = j0 + lj[0];  // a side lies wholly inside or outside the domain
+          const bool outside = gi < 0 || gi >= n || gj < 0 || gj >= n;
+          if (fused || outside) {  // materialised: only points outside the domain are written
+            eval_points<NJMAX, 4>(T, s_WJ, s_jact, xp, yp, w);
+  #pragma unroll
+            for (int c = 0; c < 4; c++) {
+              if (fused) {
+                s_wt[(lj[c] + kPad) * P64 + li[c] + kPad] = w[c];
+              } else {
+                const int pi_ = i0 + li[c], pj_ = j0 + lj[c];
+                const int hs = pi_ < 0 ? 0 : pi_ >= n ? 1 : pj_ < 0 ? 2 : 3;
+                A.out_halo[int64_t(r) * A.n_halo + A.halo_off[d] + hs * n + (hs < 2 ? pj_ : pi_)] = w[c];
+              }
+            }
+          }
+        }
+        if (!fused) return;
+        __syncthreads();
+        // band value of each position from its four neighbours at distance 2^-d
+        bool any_pass = false;
+  #pragma unroll 2
+        for (int k = 0; k < QPT; k++) {
+          const float* t = s_wt + sbase + s_kq[k].z;  // (2pi, 2pj)
+          const float2 w01 = *reinterpret_cast<const float2*>(t), w23 = *reinterpret_cast<const float2*>(t + P64);
+          const float2 bel = *reinterpret_cast<const float2*>(t - P64), abv = *reinterpret_cast<const float2*>(t + 2 * P64);
+          const float l0 = t[-1], l2 = t[P64 - 1], r1 = t[2], r3 = t[P64 + 2];
+          const float w[4] = {w01.x, w01.y, w23.x, w23.y};
+          const float L[4] = {l0, w[0], l2, w[2]}, R[4] = {w[1], r1, w[3], r3};
+          const float Bo[4] = {bel.x, bel.y, w[0], w[1]}, U[4] = {w[2], w[3], abv.x, abv.y};
+          bool pass[4];
+          // squared differences between siblings are shared by both
+          const float h01 = sqdiff(w[0], w[1]), h23 = sqdiff(w[2], w[3]);
+          const float v02 = sqdiff(w[0], w[2]), v13 = sqdiff(w[1], w[3]);
+          const float DL[4] = {sqdiff(w[0], L[0]), h01, sqdiff(w[2], L[2]), h23};
+          const float DR[4] = {h01, sqdiff(w[1], R[1]), h23, sqdiff(w[3], R[3])};
+          const float DB[4] = {sqdiff(w[0], Bo[0]), sqdiff(w[1], Bo[1]), v02, v13};
+          const float DT[4] = {v02, v13, sqdiff(w[2], U[2]), sqdiff(w[3], U[3])};
+  #pragma unroll
+          for (int c = 0; c < 4; c++) pass[c] = band_pass_sq(DL[c], DR[c], DB[c], DT[c], band2);
+          if (wfilter) {
+  #pragma unroll
+            for (int c = 0; c < 4; c++) pass[c] = pass[c] && fabsf(w[c]) > A.w_min;
+          }
+          const uint32_t b0 = __ballot_sync(kFull, pass[0]), b1 = __ballot_sync(kFull, pass[1]);
+          const uint32_t b2 = __ballot_sync(kFull, pass[2]), b3 = __ballot_sync(kFull, pass[3]);
+          any_pass = any_pass || (b0 | b1 | b2 | b3) != 0u;
+          if (lane == 0)  // the four quad-major words of this warp's 32 quads
+            *reinterpret_cast<uint4*>(band_k + 4 * (TPB / 32) * k) = make_uint4(b0, b1, b2, b3);
+          if (A.out && (pass[0] | pass[1] | pass[2] | pass[3])) {
+            float* o = A.out + lrow + mb + 4 * (tid + TPB * k);
+  #pragma unroll
+            for (int c = 0; c < 4; c++)
+              if (pass[c]) o[c] = w[c];
+          }
+        }
+        if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
+        return;
       }
-      if (A.tile_flags && __syncthreads_or(any_pass) && tid == 0) A.tile_flags[int64_t(r) * A.n_dense + tile] = 1;
-      return;
     }
-
+    pyramid_tile<NJMAX, TPB>(A, r, nv, nj, xm, ym, out_const, s_ent, s_esrc, s_WJ, s_jact, s_buf);
   };
 
   for (int t = t_beg; t < t_end; t++) {
@@ -2700,6 +2698,11 @@ cudaError_t launch_overlapped(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+// Dense tiles the block kernel takes in fused mode (the rest run a warp per tile): the
+// depths 0..4 tile, and at depth 5 also the grid's one 64 x 64 tile (a warp launch of one
+// tile per pair would leave three of a CTA's four warps idle).
+inline int32_t block_tiles(int64_t n_dense) { return n_dense == 2 ? 2 : 1; }
+
 template <int NJMAX>
 emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
   if (n_ranks <= 0) return EMR_OK;
@@ -2749,8 +2752,9 @@ emr_status launch_joint_class(const DTileArgs& D, int64_t rank_beg, int64_t n_ra
   if (!warp_tiles) return launch_dense<NJMAX>(D, rank_beg, n_ranks, st, overlap);
   emr_status rc;
   const int32_t end = D.tile_beg + D.n_tiles;
-  // the block kernel takes the depths 0..4 tile, the warp kernel the 64 x 64 tiles
-  const int32_t split_at = std::min<int32_t>(end, 1);
+  // the block kernel takes the depths 0..4 tile, the warp kernel the 64 x 64 tiles (with a
+  // single 64 x 64 tile, D = 5, the block kernel takes it too)
+  const int32_t split_at = std::min<int32_t>(end, block_tiles(D.n_dense));
   if (D.tile_beg < split_at) {
     DTileArgs D0 = D;
     D0.n_tiles = split_at - D.tile_beg;
@@ -2886,15 +2890,16 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   const int64_t b1 = p.n_class[0], b2 = b1 + p.n_class[1], b3 = b2 + p.n_class[2], b4 = b3 + p.n_class[3];
   const int64_t b5 = b4 + p.n_class[4];
   int64_t beg = b5 + p.n_class[5];
-  if (warp_tiles && D.tile_beg < 1 && D.tile_beg + D.n_tiles > 1) {
+  const int32_t bt = block_tiles(n_dense);
+  if (warp_tiles && D.tile_beg < bt && D.tile_beg + D.n_tiles > bt) {
     // every joint class's block launch (the depths 0..4 tile), then every class's warp
     // launch (depths 5..D): the block kernels' latency-bound CTAs then share the SMs with
     // the warp launches that follow them (measured faster than alternating block and
     // warp launches class by class)
     DTileArgs D0 = D, D1 = D;
-    D0.n_tiles = 1 - D.tile_beg;
-    D1.tile_beg = 1;
-    D1.n_tiles = D.tile_beg + D.n_tiles - 1;
+    D0.n_tiles = bt - D.tile_beg;
+    D1.tile_beg = bt;
+    D1.n_tiles = D.tile_beg + D.n_tiles - bt;
     if ((rc = launch_dense<12>(D0, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_dense<8>(D0, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_dense<6>(D0, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
@@ -2909,14 +2914,21 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
     if ((rc = launch_joint_class<12>(D, b1, p.n_class[1], st, &overlap, warp_tiles)) != EMR_OK) return rc;
     if ((rc = launch_joint_class<8>(D, b2, p.n_class[2], st, &overlap, warp_tiles)) != EMR_OK) return rc;
     if ((rc = launch_joint_class<6>(D, b3, p.n_class[3], st, &overlap, warp_tiles)) != EMR_OK) return rc;
-    if ((rc = launch_joint_class<4>(D, b4, p.n_class[4], st, &overlap, warp_tiles)) != EMR_OK) return rc;
-    if ((rc = launch_joint_class<2>(D, b5, p.n_class[5], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+    if (warp_tiles && D.tile_beg + D.n_tiles > bt) {
+      if ((rc = launch_joint_class<4>(D, b4, p.n_class[4], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+      if ((rc = launch_joint_class<2>(D, b5, p.n_class[5], st, &overlap, warp_tiles)) != EMR_OK) return rc;
+    } else {
+      // block tiles only: the 1..2-joint pairs (the ranks after the 3..4-joint ones) with them in one
+      // launch (a launch of its own pays more than the smaller kernel saves)
+      if ((rc = launch_joint_class<4>(D, b4, p.n_class[4] + p.n_class[5], st, &overlap, warp_tiles)) != EMR_OK)
+        return rc;
+    }
   }
   if (mode == kModeFused && !out && p.n_class[kClassNone] > p.n_const) {
     // one-coordinate outputs: the depths 0..4 tile through the generic kernel, the 64 x 64
     // tiles (depths 5..D) a warp each
     const int64_t n5 = p.n_class[kClassNone] - p.n_const;
-    const int32_t split_at = std::min<int32_t>(tr.end, 1);
+    const int32_t split_at = std::min<int32_t>(tr.end, block_tiles(n_dense));
     if (tr.beg < split_at) {
       DTileArgs D0 = D;
       D0.n_tiles = split_at - tr.beg;

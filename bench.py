@@ -622,11 +622,13 @@ def oracle_samples(W):
 
 
 def launches_in_step(emr, dsc):
-    """Kernel launches of one step: prepare (records, with the schedule in the last CTA); per
-    non-empty dense kernel class two tile launches (depths 0..4 on the block kernel, the
-    64 x 64 tiles of depths 5..D a warp each), one for the interpreter class (constant-output
-    pairs need none: their tiles hold no band bit); selection (count, scan, write, kept
-    weights). Memsets are not kernels."""
+    """Kernel launches of one step: prepare (records, with the schedule in the last CTA); the
+    tiles; selection (count, scan, write, kept weights). From depth 6 on, the tiles take one
+    block launch for the depths 0..4 tile of every pair up to 8 joint nodes and of the
+    one-coordinate pairs (one more for 9..12 joint nodes), then a warp-per-tile launch for the
+    64 x 64 tiles of each non-empty class; up to depth 5, a block launch per class, the 1..2
+    and 3..4 joint classes sharing one. The interpreter class takes one launch; constant-output
+    pairs none (their tiles hold no band bit). Memsets are not kernels."""
     _, gs, _, _ = emr.pack_records(dsc.pack)
     side = np.asarray(dsc.query.side)
     def per_pair(field):
@@ -636,9 +638,12 @@ def launches_in_step(emr, dsc):
     nv, nj = per_pair("n_varying"), per_pair("n_joint")
     cls = np.where(nv > 12, 0, np.where(nj > 8, 1, np.where(nj > 6, 2, np.where(nj > 4, 3, np.where(
         nj > 2, 4, np.where(nj > 0, 5, 6))))))
-    present = np.unique(cls[nv > 0])
-    per_class = [1 if c == 0 else (2 if dsc.grid.D >= 6 else 1) for c in present]
-    return 1 + sum(per_class) + 4
+    present = set(np.unique(cls[nv > 0]).tolist())
+    if dsc.grid.D >= 6:
+        tiles = len(present) + (1 if 1 in present else 0) + (1 if present & {2, 3, 4, 5, 6} else 0)
+    else:
+        tiles = len(present) - (1 if {4, 5} <= present else 0)
+    return 1 + tiles + 4
 
 
 def oracle_baseline(w, genomes):

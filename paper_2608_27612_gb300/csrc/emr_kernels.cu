@@ -24,6 +24,19 @@ constexpr int kBlock = 128;  // threads per evaluation tile CTA
 // such launch begin.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+// A launch that overlaps its predecessor without reading its results still has to
+// complete after it (later kernels in the stream read every launch's output): its
+// last CTA waits for the predecessor as it exits, after its own work, so that a
+// chain of such launches adds no CTA lifetime per launch to the stream's timeline.
+struct PdlWaitAtExit {
+  bool on;
+  __device__ __forceinline__ ~PdlWaitAtExit() {
+    if (on) pdl_wait();
+  }
+};
+__device__ __forceinline__ bool last_cta() {
+  return blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1 && blockIdx.z == gridDim.z - 1;
+}
 
 // ---- grid arithmetic ---------------------------------------------------------
 
@@ -1256,11 +1269,11 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
   // quad TPB k of a tile: its column and row offsets (in positions) and its shared-tile offset
   __shared__ int4 s_kq[QPT];
   // The next class's launch (other pairs, other outputs) may start filling the SMs
-  // this one frees. When this launch overlaps its predecessor, its last CTA first
-  // waits for the predecessor to complete, so that this launch completes only after
-  // it (later kernels in the stream read every launch's planes).
+  // this one frees. When this launch overlaps its predecessor, its last CTA waits,
+  // as it exits, for the predecessor to complete, so that this launch completes only
+  // after it (later kernels in the stream read every launch's planes).
   pdl_trigger();
-  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) pdl_wait();
+  const PdlWaitAtExit pdl_exit{last_cta()};
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid < QPT) {
     const int dx = int(compact1by1(uint32_t(TPB * tid))), dy = int(compact1by1(uint32_t(TPB * tid) >> 1));
@@ -1556,7 +1569,7 @@ __global__ void __launch_bounds__(32 * kOneAxisWarps, kOneAxisBlocks) tile_kerne
   __shared__ float2 s_esrc[kEntSrcCap];
   __shared__ __align__(16) float s_tab[kOneAxisWarps][kDenseMax * kTabFull];
   pdl_trigger();
-  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) pdl_wait();
+  const PdlWaitAtExit pdl_exit{last_cta()};
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int r = A.order[A.rank_beg + blockIdx.y];
   const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
@@ -1654,7 +1667,7 @@ __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_
   static_assert(kWarpTiles >= 4 && (kWarpTiles - 1) * 2 * kDenseMax * kTabFull >= kWtFull,
                 "the shared output tile fits in the tables of warps 1..kWarpTiles-1");
   pdl_trigger();
-  if (blockIdx.x == gridDim.x - 1 && blockIdx.y == gridDim.y - 1) pdl_wait();
+  const PdlWaitAtExit pdl_exit{last_cta()};
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) s_ndefer = 0;
   const int r = A.order[A.rank_beg + blockIdx.y];
@@ -2891,20 +2904,23 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   const int64_t b5 = b4 + p.n_class[4];
   int64_t beg = b5 + p.n_class[5];
   const int32_t bt = block_tiles(n_dense);
+  // non-constant one-coordinate pairs: ranks beg .. beg + n_one - 1 (the constant ones follow)
+  const int64_t n_one = p.n_class[kClassNone] - p.n_const;
+  const bool one_fused = mode == kModeFused && !out && n_one > 0;
+  bool one_tile0_done = false;
   if (warp_tiles && D.tile_beg < bt && D.tile_beg + D.n_tiles > bt) {
-    // every joint class's block launch (the depths 0..4 tile), then every class's warp
-    // launch (depths 5..D): the block kernels' latency-bound CTAs then share the SMs with
-    // the warp launches that follow them (measured faster than alternating block and
-    // warp launches class by class)
+    // the depths 0..4 tile of every pair in one block launch (the 12-joint class in one of
+    // its own), then every class's warp launch (depths 5..D): the block kernel's
+    // latency-bound CTAs share the SMs with the warp launches that follow. The pairs of up
+    // to 8 joint nodes and the one-coordinate pairs are consecutive ranks; one launch of
+    // the 8-joint kernel for all of them measured faster than a launch per class.
     DTileArgs D0 = D, D1 = D;
     D0.n_tiles = bt - D.tile_beg;
     D1.tile_beg = bt;
     D1.n_tiles = D.tile_beg + D.n_tiles - bt;
     if ((rc = launch_dense<12>(D0, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
-    if ((rc = launch_dense<8>(D0, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
-    if ((rc = launch_dense<6>(D0, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
-    if ((rc = launch_dense<4>(D0, b4, p.n_class[4], st, &overlap)) != EMR_OK) return rc;
-    if ((rc = launch_dense<2>(D0, b5, p.n_class[5], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_dense<8>(D0, b2, beg + (one_fused ? n_one : 0) - b2, st, &overlap)) != EMR_OK) return rc;
+    one_tile0_done = one_fused;
     if ((rc = launch_warp<12>(D1, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_warp<8>(D1, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_warp<6>(D1, b3, p.n_class[3], st, &overlap)) != EMR_OK) return rc;
@@ -2924,12 +2940,12 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
         return rc;
     }
   }
-  if (mode == kModeFused && !out && p.n_class[kClassNone] > p.n_const) {
-    // one-coordinate outputs: the depths 0..4 tile through the generic kernel, the 64 x 64
-    // tiles (depths 5..D) a warp each
-    const int64_t n5 = p.n_class[kClassNone] - p.n_const;
+  if (one_fused) {
+    // one-coordinate outputs: the depths 0..4 tile through the generic kernel (unless the
+    // joint classes' block launch took it), the 64 x 64 tiles (depths 5..D) a warp each
+    const int64_t n5 = n_one;
     const int32_t split_at = std::min<int32_t>(tr.end, block_tiles(n_dense));
-    if (tr.beg < split_at) {
+    if (tr.beg < split_at && !one_tile0_done) {
       DTileArgs D0 = D;
       D0.n_tiles = split_at - tr.beg;
       if ((rc = launch_dense<0>(D0, beg, n5, st, &overlap)) != EMR_OK) return rc;

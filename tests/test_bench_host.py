@@ -84,7 +84,7 @@ def test_launch_count_matches_the_profiled_launch_list():
     w = W.c2(D=7, P=1000)
     dsc = types.SimpleNamespace(pack=emr.pack_population(w.pop), grid=emr.grid_build(7),
                                 query=emr.make_query(w.sources, device="cpu"))
-    assert bench.launches_in_step(emr, dsc) == per_step == 15
+    assert bench.launches_in_step(emr, dsc) == per_step == 11
 
 
 def test_reference_arm_prints_the_contract_line():

@@ -125,6 +125,101 @@ __device__ __forceinline__ void act_apply4(int a, float& z0, float& z1, float& z
   }
 }
 
+// ---- packed pairs of fp32 -----------------------------------------------------------
+// Two fp32 values in one 64-bit register pair, for the f32x2 add / mul / fma
+// instructions: one issue slot for two lanes' worth of arithmetic, each half
+// rounded exactly as the scalar instruction rounds it (so a packed evaluation
+// gives the scalar one's bits). MUFU operations stay scalar, on the halves.
+typedef unsigned long long f2;
+__device__ __forceinline__ f2 f2_pack(float lo, float hi) {
+  f2 r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(f2 v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ float f2_lo(f2 v) {
+  float lo, hi;
+  f2_unpack(v, lo, hi);
+  return lo;
+}
+__device__ __forceinline__ f2 f2_add(f2 a, f2 b) {
+  f2 r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ f2 f2_mul(f2 a, f2 b) {
+  f2 r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ f2 f2_fma(f2 a, f2 b, f2 c) {
+  f2 r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ f2 f2_splat(float c) { return f2_pack(c, c); }
+__device__ __forceinline__ f2 f2_ex2(f2 v) {
+  float a, b;
+  f2_unpack(v, a, b);
+  return f2_pack(mufu_ex2(a), mufu_ex2(b));
+}
+__device__ __forceinline__ f2 f2_rcp(f2 v) {
+  float a, b;
+  f2_unpack(v, a, b);
+  return f2_pack(mufu_rcp(a), mufu_rcp(b));
+}
+// The activations above, on pairs, operation for operation: sigmoid and tanh
+// add 1 to the power of two, sin's reduction computes fma(k, -c, r) for
+// fma(-k, c, r) (the same exact product) and adds -shift for "- shift".
+template <int NPP>
+__device__ __forceinline__ void act_apply_pairs(int a, f2 (&z)[NPP]) {
+  switch (a) {
+    case EMR_ACT_SIGMOID: {
+      const f2 c = f2_splat(-kLog2e), one = f2_splat(1.0f);
+#pragma unroll
+      for (int p = 0; p < NPP; p++) z[p] = f2_rcp(f2_add(one, f2_ex2(f2_mul(z[p], c))));
+      break;
+    }
+    case EMR_ACT_TANH: {
+      const f2 c = f2_splat(2.0f * kLog2e), one = f2_splat(1.0f), m2 = f2_splat(-2.0f);
+#pragma unroll
+      for (int p = 0; p < NPP; p++) z[p] = f2_fma(m2, f2_rcp(f2_add(one, f2_ex2(f2_mul(z[p], c)))), one);
+      break;
+    }
+    case EMR_ACT_GAUSS: {
+      const f2 c = f2_splat(-kLog2e);
+#pragma unroll
+      for (int p = 0; p < NPP; p++) z[p] = f2_ex2(f2_mul(z[p], f2_mul(z[p], c)));
+      break;
+    }
+    case EMR_ACT_SIN: {
+      const f2 inv = f2_splat(kInvTwoPi), sh = f2_splat(kRoundShift), nsh = f2_splat(-kRoundShift);
+      const f2 nhi = f2_splat(-kTwoPiHi), nlo = f2_splat(-kTwoPiLo);
+#pragma unroll
+      for (int p = 0; p < NPP; p++) {
+        const f2 k = f2_add(f2_fma(z[p], inv, sh), nsh);
+        const f2 r = f2_fma(k, nlo, f2_fma(k, nhi, z[p]));
+        float a0, a1;
+        f2_unpack(r, a0, a1);
+        z[p] = f2_pack(mufu_sin(a0), mufu_sin(a1));
+      }
+      break;
+    }
+    case EMR_ACT_ABS:
+#pragma unroll
+      for (int p = 0; p < NPP; p++) {
+        float a0, a1;
+        f2_unpack(z[p], a0, a1);
+        z[p] = f2_pack(fabsf(a0), fabsf(a1));
+      }
+      break;
+    default:
+      break;
+  }
+}
+
 // ---- filter arithmetic shared by every kernel ------------------------------------
 // All kernels take the same fp32 decisions, operation for operation:
 //   variance: S = sum_c (w_c - m)^2 with m = (w0 + w1 + w2 + w3) / 4; V = S / 4 and
@@ -935,6 +1030,32 @@ __device__ __forceinline__ void eval_points(const PairTabs& T, const float* __re
   for (int p = 0; p < NP; p++) w[p] = t[T.out_x ? xp[p] : yp[p]];
 }
 
+// The joint nodes of a pair at 2 NPP points held as NPP packed pairs (eval_joint
+// on pairs): WJ2 holds each joint weight twice (both halves of a pair).
+template <int NJMAX, int NPP, class Init>
+__device__ __forceinline__ void eval_joint_pairs(int nj, const f2* __restrict__ WJ2, const int* __restrict__ jact,
+                                                 Init init, f2 (&w)[NPP]) {
+  f2 v[NJMAX > 1 ? NJMAX - 1 : 1][NPP];
+#pragma unroll
+  for (int m = 0; m < NJMAX; m++) {
+    if (m >= nj) break;
+    if (m > 0) {
+#pragma unroll
+      for (int p = 0; p < NPP; p++) v[m - 1][p] = w[p];
+    }
+    init(m, w);
+#pragma unroll
+    for (int m2 = 0; m2 < m; m2++) {
+      const f2 wk = WJ2[m * NJMAX + m2];
+      if (f2_lo(wk) != 0.f) {
+#pragma unroll
+        for (int p = 0; p < NPP; p++) w[p] = f2_fma(wk, v[m2][p], w[p]);
+      }
+    }
+    act_apply_pairs<NPP>(jact[m], w);
+  }
+}
+
 // Output at QPE sibling quads of a 64 x 64 tile: quad h has its children at
 // table columns xq[h], xq[h] + 1 and rows yq[h], yq[h] + 1 (both even), read as
 // pairs; w[4 h + c] is child c (x fastest). Joint node m's parts are row m.
@@ -958,6 +1079,52 @@ __device__ __forceinline__ void eval_quads(const PairTabs& T, const float* __res
         }
       };
       eval_joint<NJMAX, 4 * QPE>(T.nj, WJ, jact, init, w);
+      return;
+    }
+  }
+  if (T.nv == 0) {
+#pragma unroll
+    for (int p = 0; p < 4 * QPE; p++) w[p] = T.out_const;
+    return;
+  }
+  const float* t = (T.out_x ? T.tx : T.ty) + T.orow * kTabFull;
+#pragma unroll
+  for (int h = 0; h < QPE; h++) {
+    const float2 a = *reinterpret_cast<const float2*>(t + (T.out_x ? xq[h] : yq[h]));
+    w[4 * h + 0] = a.x;
+    w[4 * h + 1] = T.out_x ? a.y : a.x;
+    w[4 * h + 2] = T.out_x ? a.x : a.y;
+    w[4 * h + 3] = a.y;
+  }
+}
+
+// eval_quads with the joint nodes on packed pairs (children 0, 1 and 2, 3 of
+// each quad), the joint weights twice each in WJ2: the same bits in about half
+// the issue slots of the fp32 work, for kernels whose registers hold the pairs.
+template <int NJMAX, int QPE>
+__device__ __forceinline__ void eval_quads_packed(const PairTabs& T, const f2* __restrict__ WJ2,
+                                                  const int* __restrict__ jact, const int (&xq)[QPE],
+                                                  const int (&yq)[QPE], float (&w)[4 * QPE]) {
+  if constexpr (NJMAX > 0) {
+    if (T.nj > 0) {
+      auto init = [&](int m, f2 (&z)[2 * QPE]) {
+        const float* sx = T.tx + m * kTabFull;
+        const float* sy = T.ty + m * kTabFull;
+#pragma unroll
+        for (int h = 0; h < QPE; h++) {
+          const f2 a = *reinterpret_cast<const f2*>(sx + xq[h]);  // the x parts of columns xq, xq + 1
+          const float2 b = *reinterpret_cast<const float2*>(sy + yq[h]);
+          z[2 * h + 0] = f2_add(a, f2_splat(b.x));
+          z[2 * h + 1] = f2_add(a, f2_splat(b.y));
+        }
+      };
+      f2 z[2 * QPE];
+      eval_joint_pairs<NJMAX, 2 * QPE>(T.nj, WJ2, jact, init, z);
+#pragma unroll
+      for (int h = 0; h < QPE; h++) {
+        f2_unpack(z[2 * h + 0], w[4 * h + 0], w[4 * h + 1]);
+        f2_unpack(z[2 * h + 1], w[4 * h + 2], w[4 * h + 3]);
+      }
       return;
     }
   }
@@ -1555,6 +1722,48 @@ __global__ void __launch_bounds__(TPB, dense_min_blocks(NJMAX, TPB)) tile_kernel
   }
 }
 
+// The depths 0..4 tile (dense tile 0) of the pairs in one launch, fused mode: a CTA
+// per pair, the record's table programs, joint block and activations staged in
+// shared memory, then pyramid_tile. The block kernel does the same among its other
+// paths; this kernel holds only this one, so its CTAs fetch less code.
+constexpr int kPyrTPB = 128;  // threads per pyramid CTA
+template <int NJMAX>
+__global__ void __launch_bounds__(kPyrTPB, dense_min_blocks(NJMAX, kPyrTPB)) tile_kernel_pyramid(const DTileArgs A) {
+  constexpr int NJ1 = NJMAX > 0 ? NJMAX : 1;
+  __shared__ __align__(16) float s_WJ[NJ1 * NJ1];
+  __shared__ int s_jact[NJ1];
+  __shared__ float4 s_ent[2][kDenseMax];
+  __shared__ float2 s_esrc[2][kEntSrcCap];
+  __shared__ __align__(16) float s_buf[kWtPyr + 2 * kDenseMax * kTabPyr];
+  pdl_trigger();
+  const PdlWaitAtExit pdl_exit{last_cta()};
+  const int tid = threadIdx.x;
+  const int r = A.order[A.rank_beg + blockIdx.y];
+  const uint8_t* rec = A.spec + int64_t(r) * A.L.stride;
+  const int nv = reinterpret_cast<const int32_t*>(rec)[0];
+  const float out_const = reinterpret_cast<const float*>(rec)[2];
+  const uint32_t h3 = reinterpret_cast<const uint32_t*>(rec)[3];
+  const int nj = int((h3 >> kHdrJointShift) & 0xfu);
+  const uint32_t xm = (h3 >> kHdrXShift) & 0xfffu, ym = (h3 >> kHdrYShift) & 0xfffu;
+  if (nv == 0) {  // constant output: every variance and band value is exactly 0
+    zero_tile(A, r, 0, tid, kPyrTPB);
+    return;
+  }
+  {
+    const float4* gent = reinterpret_cast<const float4*>(rec + A.L.ent_off());
+    const float2* gsrc = reinterpret_cast<const float2*>(rec + A.L.esrc_off());
+    for (int k = tid; k < 2 * kDenseMax; k += kPyrTPB) s_ent[k / kDenseMax][k % kDenseMax] = gent[k];
+    for (int k = tid; k < 2 * kEntSrcCap; k += kPyrTPB) s_esrc[k / kEntSrcCap][k % kEntSrcCap] = gsrc[k];
+    if constexpr (NJMAX > 0) {
+      const float* gwj = reinterpret_cast<const float*>(rec + A.L.wj_off());
+      for (int t = tid; t < NJMAX * NJMAX; t += kPyrTPB) s_WJ[t] = gwj[(t / NJMAX) * kDenseMax + t % NJMAX];
+      if (tid < NJMAX) s_jact[tid] = reinterpret_cast<const int32_t*>(rec + A.L.jact_off())[tid];
+    }
+  }
+  __syncthreads();
+  pyramid_tile<NJMAX, kPyrTPB>(A, r, nv, nj, xm, ym, out_const, s_ent, s_esrc, s_WJ, s_jact, s_buf);
+}
+
 // The 64 x 64 tiles of pairs whose output depends on one coordinate (no joint
 // node; fused mode, no output buffer): a warp per tile, four tiles at a time per
 // CTA, no block barrier. The warp evaluates the output's axis table at the
@@ -1653,11 +1862,28 @@ constexpr int warp_min_blocks(int njmax) { return njmax <= 4 ? 7 : njmax <= 8 ? 
 __device__ __forceinline__ int warp_quad_dx(int k) { return 2 * (8 * ((k >> 1) & 1) + 16 * ((k >> 3) & 1)); }
 __device__ __forceinline__ int warp_quad_dy(int k) { return 2 * (4 * (k & 1) + 8 * ((k >> 2) & 1) + 16 * ((k >> 4) & 1)); }
 
+// The warp kernel's quads on packed pairs for the 5..6-joint class only (measured): its
+// register budget (six CTAs per SM) takes the pairs, and its edges and activations give
+// the packed arithmetic the most to do. Under the 1..4-joint classes' tighter budget the
+// moves that form the pairs took as many issue slots as the packed arithmetic saved; the
+// 7..8-joint class gained nothing.
+__host__ __device__ constexpr bool warp_packed(int njmax) { return njmax > 4 && njmax <= 6; }
+template <int NJMAX, int QPE>
+__device__ __forceinline__ void warp_quads(const PairTabs& T, const float* __restrict__ WJ, const f2* __restrict__ WJ2,
+                                           const int* __restrict__ jact, const int (&xq)[QPE], const int (&yq)[QPE],
+                                           float (&w)[4 * QPE]) {
+  if constexpr (warp_packed(NJMAX))
+    eval_quads_packed<NJMAX, QPE>(T, WJ2, jact, xq, yq, w);
+  else
+    eval_quads<NJMAX, QPE>(T, WJ, jact, xq, yq, w);
+}
+
 template <int NJMAX>
 __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_kernel_warp(const DTileArgs A) {
   static_assert(NJMAX >= 1 && NJMAX <= kDenseMax, "pairs with joint nodes");
   constexpr int QPE = NJMAX <= 6 ? 2 : 1;
   __shared__ __align__(16) float s_WJ[NJMAX * NJMAX];
+  __shared__ f2 s_WJ2[NJMAX * NJMAX];  // the same weights twice each, for the packed quads
   __shared__ int s_jact[NJMAX];
   __shared__ float4 s_ent[2][kDenseMax];
   __shared__ float2 s_esrc[2][kEntSrcCap];
@@ -1683,7 +1909,11 @@ __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_
     const float* gwj = reinterpret_cast<const float*>(rec + A.L.wj_off());
     for (int k = tid; k < 2 * kDenseMax; k += 32 * kWarpTiles) s_ent[k / kDenseMax][k % kDenseMax] = gent[k];
     for (int k = tid; k < 2 * kEntSrcCap; k += 32 * kWarpTiles) s_esrc[k / kEntSrcCap][k % kEntSrcCap] = gsrc[k];
-    for (int t = tid; t < NJMAX * NJMAX; t += 32 * kWarpTiles) s_WJ[t] = gwj[(t / NJMAX) * kDenseMax + t % NJMAX];
+    for (int t = tid; t < NJMAX * NJMAX; t += 32 * kWarpTiles) {
+      const float wk = gwj[(t / NJMAX) * kDenseMax + t % NJMAX];
+      s_WJ[t] = wk;
+      s_WJ2[t] = f2_splat(wk);
+    }
     if (tid < NJMAX) s_jact[tid] = reinterpret_cast<const int32_t*>(rec + A.L.jact_off())[tid];
   }
   __syncthreads();
@@ -1737,7 +1967,7 @@ __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_
         xq[h] = xb + warp_quad_dx(k0 + h);
         yq[h] = yb + warp_quad_dy(k0 + h);
       }
-      eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
+      warp_quads<NJMAX, QPE>(T, s_WJ, s_WJ2, s_jact, xq, yq, w);
 #pragma unroll
       for (int h = 0; h < QPE; h++) {
         // the four children give the parent's variance (Section 3.2)
@@ -1791,7 +2021,7 @@ __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_
         yq[h] = 2 * py + 2;
         so[h] = (2 * py + kPad) * P64 + 2 * px + kPad;
       }
-      eval_quads<NJMAX, QPE>(T, s_WJ, s_jact, xq, yq, w);
+      warp_quads<NJMAX, QPE>(T, s_WJ, s_WJ2, s_jact, xq, yq, w);
 #pragma unroll
       for (int h = 0; h < QPE; h++) {
         *reinterpret_cast<float2*>(s_wt + so[h]) = make_float2(w[4 * h + 0], w[4 * h + 1]);
@@ -2737,6 +2967,20 @@ emr_status launch_dense(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, 
   return cuda_status(cudaGetLastError());
 }
 
+// Dense tile 0 of n_ranks pairs through tile_kernel_pyramid (fused mode, no output buffer).
+template <int NJMAX>
+emr_status launch_pyramid(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
+  if (n_ranks <= 0) return EMR_OK;
+  DTileArgs A = A0;
+  for (int64_t r0 = 0; r0 < n_ranks; r0 += 65535) {  // grid y: ranks, at most 65535 a launch
+    A.rank_beg = rank_beg + r0;
+    const dim3 grid(1, unsigned(std::min<int64_t>(65535, n_ranks - r0)));
+    const cudaError_t e = launch_overlapped(tile_kernel_pyramid<NJMAX>, grid, dim3(kPyrTPB), 0, st, overlap, A);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  return cuda_status(cudaGetLastError());
+}
+
 template <int NJMAX>
 emr_status launch_warp(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, cudaStream_t st, bool* overlap) {
   if (n_ranks <= 0 || A0.n_tiles <= 0) return EMR_OK;
@@ -2918,8 +3162,8 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
     D0.n_tiles = bt - D.tile_beg;
     D1.tile_beg = bt;
     D1.n_tiles = D.tile_beg + D.n_tiles - bt;
-    if ((rc = launch_dense<12>(D0, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
-    if ((rc = launch_dense<8>(D0, b2, beg + (one_fused ? n_one : 0) - b2, st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_pyramid<12>(D0, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
+    if ((rc = launch_pyramid<8>(D0, b2, beg + (one_fused ? n_one : 0) - b2, st, &overlap)) != EMR_OK) return rc;
     one_tile0_done = one_fused;
     if ((rc = launch_warp<12>(D1, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_warp<8>(D1, b2, p.n_class[2], st, &overlap)) != EMR_OK) return rc;

@@ -424,6 +424,7 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
                                                                float* __restrict__ scratch, int32_t scratch_stride,
                                                                int32_t* __restrict__ order, int32_t* __restrict__ bins,
                                                                unsigned int* __restrict__ done) {
+  pdl_trigger();  // a tile launch set to overlap this kernel waits for its completion in every CTA
   __shared__ float s_cval[kSpecWarps][kSpecSmemNodes];
   __shared__ int32_t s_hist[kCostBins];
   __shared__ int32_t s_wsum[32];
@@ -884,6 +885,7 @@ struct DTileArgs {
   uint32_t* bandb;
   uint8_t* tile_flags;  // fused, optional: [pair][dense tile] set to 1 where a band bit is set
   int64_t n_dense;
+  int32_t wait_at_start;  // pyramid kernel: the launch overlaps the record kernel, whose records it reads
 };
 
 template <int NP>
@@ -1735,6 +1737,9 @@ __global__ void __launch_bounds__(kPyrTPB, dense_min_blocks(NJMAX, kPyrTPB)) til
   __shared__ float4 s_ent[2][kDenseMax];
   __shared__ float2 s_esrc[2][kEntSrcCap];
   __shared__ __align__(16) float s_buf[kWtPyr + 2 * kDenseMax * kTabPyr];
+  // Launched to overlap the record kernel, every CTA waits for its records first; the
+  // launches after this one may start only then (they read the records unwaited).
+  if (A.wait_at_start) pdl_wait();
   pdl_trigger();
   const PdlWaitAtExit pdl_exit{last_cta()};
   const int tid = threadIdx.x;
@@ -3051,10 +3056,13 @@ struct TileRange {
 emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spec, const int32_t* order, int mode,
                         float theta, float band, float w_min, float* out, float* out_halo, uint32_t* split,
                         uint32_t* bandb, cudaStream_t st, TileRange tr = TileRange(),
-                        uint8_t* tile_flags = nullptr) {
+                        uint8_t* tile_flags = nullptr, bool after_records = false) {
+  // after_records: the record kernel is this stream's last launch and the tile flags are
+  // already zeroed, so the first tile launch may overlap it (when that launch waits for it)
   emr_status rc = EMR_OK;
   const int32_t n_dense = int32_t(dense_tiles(g->D));
-  if (tile_flags && cudaMemsetAsync(tile_flags, 0, size_t(p.n_pairs) * size_t(n_dense), st) != cudaSuccess)
+  if (tile_flags && !after_records &&
+      cudaMemsetAsync(tile_flags, 0, size_t(p.n_pairs) * size_t(n_dense), st) != cudaSuccess)
     return EMR_ERR_CUDA;
   if (tr.end < 0) tr.end = n_dense;
   if (tr.band_stride < 0) tr.band_stride = g->n_words;
@@ -3162,6 +3170,10 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
     D0.n_tiles = bt - D.tile_beg;
     D1.tile_beg = bt;
     D1.n_tiles = D.tile_beg + D.n_tiles - bt;
+    if (after_records && !overlap) {  // the depths 0..4 launches overlap the record kernel
+      overlap = true;
+      D0.wait_at_start = 1;
+    }
     if ((rc = launch_pyramid<12>(D0, b1, p.n_class[1], st, &overlap)) != EMR_OK) return rc;
     if ((rc = launch_pyramid<8>(D0, b2, beg + (one_fused ? n_one : 0) - b2, st, &overlap)) != EMR_OK) return rc;
     one_tile0_done = one_fused;
@@ -3576,14 +3588,17 @@ emr_status emr_discover(const void* pack_host, const void* pack_dev, const emr_q
   uint8_t* base = static_cast<uint8_t*>(ws);
   uint8_t* spec;
   int32_t* order;
-  // the selection's work-item counter, zeroed ahead so its first kernel can overlap the tile launches
-  if (cudaMemsetAsync(base + L.sel, 0, sizeof(unsigned long long), st) != cudaSuccess) return EMR_ERR_CUDA;
+  uint8_t* flags = base + L.flags;
+  // the selection's work-item counter and the tile flags, zeroed ahead: the first tile launch
+  // may then overlap the record kernel and the selection's first kernel the tile launches
+  // (adjacent in the workspace: one memset)
+  if (cudaMemsetAsync(flags, 0, L.sel - L.flags + sizeof(unsigned long long), st) != cudaSuccess)
+    return EMR_ERR_CUDA;
   if ((rc = prepare(pack_dev, q, p, ws, st, &spec, &order)) != EMR_OK) return rc;
   auto* split = reinterpret_cast<uint32_t*>(base + L.split);
   auto* bandb = reinterpret_cast<uint32_t*>(base + L.band);
-  uint8_t* flags = base + L.flags;
   if ((rc = launch_tiles(p, grid, spec, order, kModeFused, theta, band, w_min, nullptr, nullptr, split, bandb, st,
-                         TileRange(), flags)) != EMR_OK)
+                         TileRange(), flags, true)) != EMR_OK)
     return rc;
   return select_launch(p, split, bandb, flags, q, ws, grid, mode, types, idx, w, cap, counts, offsets,
                        base + L.sel, st, true);

@@ -75,12 +75,12 @@ def test_constant_output_counts_nothing():
 
 def test_launch_count_matches_the_profiled_launch_list():
     """bench.py's gpu_launches claim for the 1000-genome depth-7 step equals the kernels per step
-    in the committed ncu launch list (profiles/launches_c2_pop1000_d7.md: launches over 8 steps)."""
+    in the committed ncu launch list (profiles/launches_c2_pop1000_d7.md: launches over 16 steps)."""
     import os
     import types
     path = os.path.join(os.path.dirname(bench.__file__), "profiles", "launches_c2_pop1000_d7.md")
     rows = [l.split("|") for l in open(path) if l.startswith("| ") and not l.startswith("| kernel")]
-    per_step = sum(int(r[2]) for r in rows) / 8
+    per_step = sum(int(r[2]) for r in rows) / 16
     w = W.c2(D=7, P=1000)
     dsc = types.SimpleNamespace(pack=emr.pack_population(w.pop), grid=emr.grid_build(7),
                                 query=emr.make_query(w.sources, device="cpu"))

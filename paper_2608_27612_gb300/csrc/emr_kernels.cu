@@ -1860,19 +1860,18 @@ __global__ void __launch_bounds__(32 * kOneAxisWarps, kOneAxisBlocks) tile_kerne
 // the place of the other warps' tables), and the band test from shared memory,
 // 128 threads at a time; every other tile stores zero band words.
 constexpr int kWarpTiles = 4;
-constexpr int warp_min_blocks(int njmax) { return njmax <= 4 ? 7 : njmax <= 8 ? 6 : 4; }
+constexpr int warp_min_blocks(int njmax) { return njmax <= 2 ? 7 : njmax <= 8 ? 6 : 4; }
 
 // Column (row) offset of quad 32 k of a 64 x 64 tile, in positions: Morton bits
 // 6, 8 of the quad index are x bits 3, 4 (bits 5, 7, 9: y bits 2, 3, 4).
 __device__ __forceinline__ int warp_quad_dx(int k) { return 2 * (8 * ((k >> 1) & 1) + 16 * ((k >> 3) & 1)); }
 __device__ __forceinline__ int warp_quad_dy(int k) { return 2 * (4 * (k & 1) + 8 * ((k >> 2) & 1) + 16 * ((k >> 4) & 1)); }
 
-// The warp kernel's quads on packed pairs for the 5..6-joint class only (measured): its
-// register budget (six CTAs per SM) takes the pairs, and its edges and activations give
-// the packed arithmetic the most to do. Under the 1..4-joint classes' tighter budget the
-// moves that form the pairs took as many issue slots as the packed arithmetic saved; the
-// 7..8-joint class gained nothing.
-__host__ __device__ constexpr bool warp_packed(int njmax) { return njmax > 4 && njmax <= 6; }
+// The warp kernel's quads on packed pairs up to 8 joint nodes (measured). The 3..4-joint class
+// needs its six-CTA budget for them: under seven CTAs' registers the moves that form the pairs
+// took as many issue slots as the packed arithmetic saved. The 9..12-joint class (128 registers
+// at four CTAs per SM) stays scalar.
+__host__ __device__ constexpr bool warp_packed(int njmax) { return njmax <= 8; }
 template <int NJMAX, int QPE>
 __device__ __forceinline__ void warp_quads(const PairTabs& T, const float* __restrict__ WJ, const f2* __restrict__ WJ2,
                                            const int* __restrict__ jact, const int (&xq)[QPE], const int (&yq)[QPE],
@@ -1886,7 +1885,8 @@ __device__ __forceinline__ void warp_quads(const PairTabs& T, const float* __res
 template <int NJMAX>
 __global__ void __launch_bounds__(32 * kWarpTiles, warp_min_blocks(NJMAX)) tile_kernel_warp(const DTileArgs A) {
   static_assert(NJMAX >= 1 && NJMAX <= kDenseMax, "pairs with joint nodes");
-  constexpr int QPE = NJMAX <= 6 ? 2 : 1;
+  // quads per pass (measured): four up to 4 joint nodes, two above
+  constexpr int QPE = NJMAX <= 4 ? 4 : 2;
   __shared__ __align__(16) float s_WJ[NJMAX * NJMAX];
   __shared__ f2 s_WJ2[NJMAX * NJMAX];  // the same weights twice each, for the packed quads
   __shared__ int s_jact[NJMAX];

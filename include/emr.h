@@ -132,7 +132,9 @@ emr_status emr_index_to_ij(int64_t gidx, int32_t *d, int32_t *i, int32_t *j);
 
 /* ---- a2: population packing (host) -------------------------------------- */
 
-/* Bytes emr_pack_population needs for this population (an upper bound). */
+/* Bytes emr_pack_population writes for this population: each genome's records
+ * take the room of its input nodes and connections, so that genomes pack
+ * independently (on several host threads) straight into the blob. */
 emr_status emr_pack_size(int32_t P, const int64_t *node_ptr, const int64_t *conn_ptr, size_t *bytes);
 
 /* Pack P NEAT genomes (Section 2; the TensorNEAT genomes of Section 5.1) into
@@ -183,8 +185,9 @@ emr_status emr_pack_population(int32_t P, const int64_t *node_ptr, const int32_t
 emr_status emr_partition_genomes(const void *pack_host, const emr_query *q, int32_t n_parts, int32_t *g_begin);
 
 /* The packer's state kept between calls: up to 15 host worker threads (started
- * on first use; starting them costs as much as packing a few dozen genomes) and
- * its per-thread packing buffers (grown to the largest population packed). This
+ * on first use; starting them costs as much as packing a few dozen genomes;
+ * after a call they watch for the next one for 0.4 ms before they sleep) and
+ * its per-thread scratch (grown to the largest genome packed). This
  * is libemr's one process-wide state besides emr_eval_filter_noalloc's static
  * device array; it holds no results, only scratch. emr_pack_release joins the
  * worker threads and frees the buffers; the next emr_pack_population (or

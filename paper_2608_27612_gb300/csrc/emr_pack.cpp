@@ -2,6 +2,8 @@
 #include <pthread.h>
 
 #include <algorithm>
+#include <atomic>
+#include <chrono>
 #include <cmath>
 #include <condition_variable>
 #include <functional>
@@ -23,11 +25,16 @@ inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 // Host worker threads kept across calls (starting threads costs as much as
 // packing a few dozen genomes). run() executes fn(0 .. n-1) on the workers and
 // the caller and returns when all are done; one job at a time (a caller that
-// finds the pool busy runs its job alone). shutdown() (emr_pack_release, and
-// the library's unload) stops and joins the workers; the next run() starts a
-// fresh pool. A process forked from this one starts a fresh pool too.
+// finds the pool busy runs its job alone). A worker that finishes a job watches
+// for the next one for kSpinMicros before it sleeps, so that calls in quick
+// succession (a packing pipeline) hand out their tasks without waking threads.
+// shutdown() (emr_pack_release, and the library's unload) stops and joins the
+// workers; the next run() starts a fresh pool. A process forked from this one
+// starts a fresh pool too.
 class WorkerPool {
  public:
+  static constexpr int kSpinMicros = 400;
+
   static WorkerPool& get() {
     static std::once_flag once;
     std::call_once(once, [] { pthread_atfork(nullptr, nullptr, [] { instance() = nullptr; }); });
@@ -48,7 +55,7 @@ class WorkerPool {
     {
       std::lock_guard<std::mutex> job(p->job_mu_);  // a job in progress finishes first
       std::lock_guard<std::mutex> lk(p->mu_);
-      p->stop_ = true;
+      p->stop_.store(true);
     }
     p->cv_.notify_all();
     for (std::thread& t : p->threads_)
@@ -63,29 +70,30 @@ class WorkerPool {
       return;
     }
     ensure(n - 1);
+    uint64_t g;
     {
       std::lock_guard<std::mutex> lk(mu_);
       job_ = &fn;
       n_ = n;
-      next_ = 1;  // task 0 is the caller's
-      left_ = n - 1;
-      gen_++;
+      left_.store(n - 1);
+      g = gen_.load() + 1;
+      claim_.store((g << 32) | 1u, std::memory_order_release);  // task 0 is the caller's
+      gen_.store(g, std::memory_order_release);
     }
-    cv_.notify_all();
+    cv_.notify_all();  // the workers asleep; the spinning ones have seen gen_
     fn(0);
-    for (;;) {  // help with the remaining tasks, then wait for the workers' last ones
-      int t;
-      {
-        std::lock_guard<std::mutex> lk(mu_);
-        if (next_ >= n_) break;
-        t = next_++;
-      }
+    for (int t; (t = claim(g, n)) >= 0;) {  // help with the tasks not yet taken
       fn(t);
-      std::lock_guard<std::mutex> lk(mu_);
-      if (--left_ == 0) break;
+      left_.fetch_sub(1, std::memory_order_acq_rel);
     }
-    std::unique_lock<std::mutex> lk(mu_);
-    done_cv_.wait(lk, [&] { return left_ == 0 || (next_ >= n_ && left_ == 0); });
+    // the workers' last tasks: short, so wait by spinning, then on the condition variable
+    for (int k = 0; left_.load(std::memory_order_acquire) != 0 && k < 4096; k++) {
+    }
+    if (left_.load(std::memory_order_acquire) != 0) {
+      std::unique_lock<std::mutex> lk(mu_);
+      done_cv_.wait(lk, [&] { return left_.load(std::memory_order_acquire) == 0; });
+    }
+    std::lock_guard<std::mutex> lk(mu_);
     job_ = nullptr;
   }
 
@@ -103,20 +111,45 @@ class WorkerPool {
     while (int(threads_.size()) < workers) threads_.emplace_back([this] { loop(); });
   }
 
-  void loop() {
-    uint64_t seen = 0;
+  // The next task of job generation g (of n tasks), or -1 when it has none left or a newer
+  // job was posted: a task is claimed together with its job's generation, so a thread late
+  // to a finished job never runs the next job's tasks with the old function.
+  int claim(uint64_t g, int n) {
+    uint64_t c = claim_.load(std::memory_order_acquire);
     for (;;) {
-      std::unique_lock<std::mutex> lk(mu_);
-      cv_.wait(lk, [&] { return stop_ || (gen_ != seen && job_ && next_ < n_); });
-      if (stop_) return;
-      seen = gen_;
-      while (job_ && next_ < n_) {
-        const int t = next_++;
-        const std::function<void(int)>* fn = job_;
-        lk.unlock();
+      if ((c >> 32) != (g & 0xffffffffu) || int(c & 0xffffffffu) >= n) return -1;
+      if (claim_.compare_exchange_weak(c, c + 1, std::memory_order_acq_rel)) return int(c & 0xffffffffu);
+    }
+  }
+
+  void loop() {
+    uint64_t seen = gen_.load(std::memory_order_acquire);
+    for (;;) {
+      // watch for a new job for a while, then sleep until one is posted
+      const auto t0 = std::chrono::steady_clock::now();
+      for (int k = 1; gen_.load(std::memory_order_acquire) == seen && !stop_.load(); k++) {
+        if ((k & 255) == 0 && std::chrono::steady_clock::now() - t0 > std::chrono::microseconds(kSpinMicros)) {
+          std::unique_lock<std::mutex> lk(mu_);
+          cv_.wait(lk, [&] { return stop_.load() || gen_.load(std::memory_order_acquire) != seen; });
+          break;
+        }
+      }
+      if (stop_.load()) return;
+      const std::function<void(int)>* fn;
+      int n;
+      {
+        std::lock_guard<std::mutex> lk(mu_);
+        seen = gen_.load(std::memory_order_acquire);
+        fn = job_;
+        n = n_;
+      }
+      if (!fn) continue;
+      for (int t; (t = claim(seen, n)) >= 0;) {
         (*fn)(t);
-        lk.lock();
-        if (--left_ == 0) done_cv_.notify_all();
+        if (left_.fetch_sub(1, std::memory_order_acq_rel) == 1) {
+          std::lock_guard<std::mutex> lk(mu_);
+          done_cv_.notify_all();
+        }
       }
     }
   }
@@ -124,9 +157,10 @@ class WorkerPool {
   std::mutex job_mu_, mu_;
   std::condition_variable cv_, done_cv_;
   const std::function<void(int)>* job_ = nullptr;
-  int n_ = 0, next_ = 0, left_ = 0;
-  uint64_t gen_ = 0;
-  bool stop_ = false;
+  int n_ = 0;
+  std::atomic<int> left_{0};
+  std::atomic<uint64_t> gen_{0}, claim_{0};  // claim_: generation (high 32 bits) and next task
+  std::atomic<bool> stop_{false};
   std::vector<std::thread> threads_;
 };
 
@@ -145,12 +179,6 @@ int act_cost(int a) {
   static const int c[6] = {0, 5, 6, 3, 7, 1};
   return (a >= 0 && a < 6) ? c[a] : 8;
 }
-
-// A genome's packed record; its nodes and edges are appended to its thread's
-// arrays (node_beg / edge_beg are positions there until the blob is assembled).
-struct GenomeOut {
-  PackGenome g{};
-};
 
 struct Edge {
   int s, d;
@@ -172,29 +200,21 @@ struct Scratch {
   int64_t id_min = 0;
 };
 
-// Packing buffers of the tasks of one call, kept across calls so that a warm
-// packer allocates nothing: scratch, the tasks' node and edge records, the
-// genome table. One caller at a time uses the shared set; release() (from
-// emr_pack_release) frees their memory, and the next call grows them again.
+// Scratch of the packing tasks of one call, kept across calls so that a warm
+// packer allocates nothing. One caller at a time uses the shared set (a caller
+// that finds it in use packs with its own); release() (from emr_pack_release)
+// frees the memory, and the next call grows it again.
 struct PackBuffers {
   static constexpr int kTasks = 16;
   std::mutex mu;
   Scratch scratch[kTasks];
-  std::vector<PackNode> nodes[kTasks];
-  std::vector<PackEdge> edges[kTasks];
-  std::vector<GenomeOut> gs;
   static PackBuffers& get() {
     static PackBuffers* b = new PackBuffers();
     return *b;
   }
   void release() {
     std::lock_guard<std::mutex> lk(mu);
-    for (int t = 0; t < kTasks; t++) {
-      scratch[t] = Scratch();
-      std::vector<PackNode>().swap(nodes[t]);
-      std::vector<PackEdge>().swap(edges[t]);
-    }
-    std::vector<GenomeOut>().swap(gs);
+    for (int t = 0; t < kTasks; t++) scratch[t] = Scratch();
   }
 };
 
@@ -222,12 +242,13 @@ void build_csr(int n, const std::vector<Edge>& es, bool by_src, std::vector<int>
 }
 
 // Topological order (Kahn, ties by id), dead-node removal, input folding and
-// per-side variation flags for one genome.
+// per-side variation flags for one genome. Its records go to on[] (room for
+// n1 - n0 nodes) and oe[] (room for c1 - c0 edges), the unused rest zeroed;
+// *out is its genome record, node_beg and edge_beg left to the caller.
 emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_t* node_id,
                     const int32_t* node_kind, const int32_t* node_act, const float* node_bias,
                     const int32_t* conn_src, const int32_t* conn_dst, const float* conn_w,
-                    const uint8_t* conn_en, Scratch& S, std::vector<PackNode>& nodes,
-                    std::vector<PackEdge>& edges, GenomeOut* out) {
+                    const uint8_t* conn_en, Scratch& S, PackNode* on, PackEdge* oe, PackGenome* out) {
   const int n = int(n1 - n0);
   if (n <= 0 || n > 1 << 20) return EMR_ERR_ARG;
   S.ids.clear();
@@ -299,38 +320,84 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
     S.es.resize(m);
   }
   S.es.erase(std::remove_if(S.es.begin(), S.es.end(), [](const Edge& e) { return e.w == 0.f; }), S.es.end());
-  build_csr(n, S.es, true, S.succ_beg, S.succ, S.fill);
-  build_csr(n, S.es, false, S.pred_beg, S.pred, S.fill);
-  // Kahn's algorithm over every node; ready nodes leave in ascending id order.
-  S.indeg.assign(n, 0);
-  for (auto& e : S.es) S.indeg[e.d]++;
-  S.order.clear();
-  S.ready.clear();
-  auto by_id = [&](int a, int b) { return node_id[n0 + a] > node_id[n0 + b]; };  // min-heap on id
-  for (int v = 0; v < n; v++)
-    if (S.indeg[v] == 0) S.ready.push_back(v);
-  std::make_heap(S.ready.begin(), S.ready.end(), by_id);
-  while (!S.ready.empty()) {
-    std::pop_heap(S.ready.begin(), S.ready.end(), by_id);
-    const int v = S.ready.back();
-    S.ready.pop_back();
-    S.order.push_back(v);
-    for (int k = S.succ_beg[v]; k < S.succ_beg[v + 1]; k++)
-      if (--S.indeg[S.succ[k]] == 0) {
-        S.ready.push_back(S.succ[k]);
-        std::push_heap(S.ready.begin(), S.ready.end(), by_id);
-      }
-  }
-  if (int(S.order.size()) != n) return EMR_ERR_CYCLE;
-  // Keep the non-input nodes from which the output is reachable.
   S.reach.assign(n, 0);
-  S.stack.assign(1, out_node);
-  S.reach[out_node] = 1;
-  while (!S.stack.empty()) {
-    const int v = S.stack.back();
-    S.stack.pop_back();
-    for (int k = S.pred_beg[v]; k < S.pred_beg[v + 1]; k++)
-      if (!S.reach[S.pred[k]]) { S.reach[S.pred[k]] = 1; S.stack.push_back(S.pred[k]); }
+  if (n <= 64) {
+    // Kahn's algorithm and the reachability on bit masks: bit k of succ[v] / pred[v] is local
+    // node k; the ready set holds nodes by rank in id order, so its lowest bit is the ready
+    // node of smallest id.
+    uint64_t succ[64], pred[64];
+    int indeg[64];
+    uint8_t rank_of[64], node_at[64];
+    for (int k = 0; k < n; k++) {
+      succ[k] = pred[k] = 0;
+      indeg[k] = 0;
+    }
+    for (auto& e : S.es) {  // parallel edges are merged: one per source
+      succ[e.s] |= 1ull << e.d;
+      pred[e.d] |= 1ull << e.s;
+      indeg[e.d]++;
+    }
+    for (int r = 0; r < n; r++) {
+      node_at[r] = uint8_t(S.ids[size_t(r)].second);
+      rank_of[S.ids[size_t(r)].second] = uint8_t(r);
+    }
+    uint64_t ready = 0;
+    for (int k = 0; k < n; k++)
+      if (indeg[k] == 0) ready |= 1ull << rank_of[k];
+    S.order.clear();
+    while (ready) {
+      const int v = node_at[__builtin_ctzll(ready)];
+      ready &= ready - 1;
+      S.order.push_back(v);
+      for (uint64_t m = succ[v]; m; m &= m - 1) {
+        const int u = __builtin_ctzll(m);
+        if (--indeg[u] == 0) ready |= 1ull << rank_of[u];
+      }
+    }
+    if (int(S.order.size()) != n) return EMR_ERR_CYCLE;
+    // the nodes from which the output is reachable
+    uint64_t reach = 1ull << out_node, todo = reach;
+    while (todo) {
+      const int v = __builtin_ctzll(todo);
+      todo &= todo - 1;
+      const uint64_t fresh = pred[v] & ~reach;
+      reach |= fresh;
+      todo |= fresh;
+    }
+    for (int k = 0; k < n; k++) S.reach[size_t(k)] = char((reach >> k) & 1u);
+  } else {
+    build_csr(n, S.es, true, S.succ_beg, S.succ, S.fill);
+    build_csr(n, S.es, false, S.pred_beg, S.pred, S.fill);
+    // Kahn's algorithm over every node; ready nodes leave in ascending id order.
+    S.indeg.assign(n, 0);
+    for (auto& e : S.es) S.indeg[e.d]++;
+    S.order.clear();
+    S.ready.clear();
+    auto by_id = [&](int a, int b) { return node_id[n0 + a] > node_id[n0 + b]; };  // min-heap on id
+    for (int v = 0; v < n; v++)
+      if (S.indeg[v] == 0) S.ready.push_back(v);
+    std::make_heap(S.ready.begin(), S.ready.end(), by_id);
+    while (!S.ready.empty()) {
+      std::pop_heap(S.ready.begin(), S.ready.end(), by_id);
+      const int v = S.ready.back();
+      S.ready.pop_back();
+      S.order.push_back(v);
+      for (int k = S.succ_beg[v]; k < S.succ_beg[v + 1]; k++)
+        if (--S.indeg[S.succ[k]] == 0) {
+          S.ready.push_back(S.succ[k]);
+          std::push_heap(S.ready.begin(), S.ready.end(), by_id);
+        }
+    }
+    if (int(S.order.size()) != n) return EMR_ERR_CYCLE;
+    // Keep the non-input nodes from which the output is reachable.
+    S.stack.assign(1, out_node);
+    S.reach[out_node] = 1;
+    while (!S.stack.empty()) {
+      const int v = S.stack.back();
+      S.stack.pop_back();
+      for (int k = S.pred_beg[v]; k < S.pred_beg[v + 1]; k++)
+        if (!S.reach[S.pred[k]]) { S.reach[S.pred[k]] = 1; S.stack.push_back(S.pred[k]); }
+    }
   }
   S.slot.assign(n, -1);
   S.kept.clear();
@@ -339,9 +406,7 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
   if (S.kept.empty() || S.kept.back() != out_node) return EMR_ERR_ARG;  // output must be last
   if (S.kept.size() > 65535) return EMR_ERR_RANGE;
   const int nk = int(S.kept.size());
-  const size_t nb = nodes.size();
-  nodes.resize(nb + size_t(nk));  // value-initialised records
-  PackNode* on = nodes.data() + nb;
+  std::memset(on, 0, sizeof(PackNode) * size_t(n));  // the kept nodes' records, then zeros
   S.has_in.assign(nk, 0);  // bit k: has an enabled in-connection from input kind k
   S.in_cnt.assign(nk, 0);
   for (int t = 0; t < nk; t++) {
@@ -365,19 +430,16 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
   S.in_beg.assign(nk + 1, 0);
   for (int t = 0; t < nk; t++) S.in_beg[t + 1] = S.in_beg[t] + S.in_cnt[t];
   if (S.in_beg[nk] > 65535) return EMR_ERR_RANGE;
-  const size_t eb = edges.size();
-  edges.resize(eb + size_t(S.in_beg[nk]));
-  PackEdge* oe = edges.data() + eb;
+  if (S.in_beg[nk] > c1 - c0) return EMR_ERR_ARG;  // cannot happen: an edge per kept connection at most
+  std::memset(oe, 0, sizeof(PackEdge) * size_t(c1 - c0));
   S.fill.assign(nk, 0);
   for (auto& e : S.es) {
     const int t = S.slot[e.d];
     if (t < 0 || node_kind[n0 + e.s] < EMR_KIND_HIDDEN) continue;
     oe[S.in_beg[t] + S.fill[t]++] = PackEdge{uint16_t(S.slot[e.s]), 0, e.w};
   }
-  PackGenome& g = out->g;
+  PackGenome& g = *out;
   g = PackGenome{};
-  g.node_beg = uint32_t(nb);
-  g.edge_beg = uint32_t(eb);
   g.n_nodes = uint16_t(nk);
   for (int t = 0; t < nk; t++) {
     on[t].edge_beg = uint16_t(S.in_beg[t]);
@@ -473,103 +535,109 @@ emr_status emr_pack_population(int32_t P, const int64_t* node_ptr, const int32_t
     return EMR_ERR_ARG;
   const bool has_conns = conn_ptr[P] > conn_ptr[0];
   if (has_conns && (!conn_src || !conn_dst || !conn_w || !conn_enabled)) return EMR_ERR_ARG;
-  // per-task buffers kept across calls; a caller that finds them in use packs with its own
-  PackBuffers& shared = PackBuffers::get();
-  std::unique_lock<std::mutex> buf_lock(shared.mu, std::try_to_lock);
-  std::unique_ptr<PackBuffers> own;
-  if (!buf_lock.owns_lock()) own.reset(new PackBuffers());
-  PackBuffers& B = own ? *own : shared;
-  std::vector<GenomeOut>& gs = B.gs;
-  gs.resize(size_t(P));
-  // Genomes are independent: pack them on several host threads, each with its
-  // own scratch; the lowest failing genome index is reported.
-  const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
-  // a thread's share costs about as much to hand out as packing a few genomes
-  const int n_threads = std::max(1, std::min({hw, PackBuffers::kTasks, P / 32}));
-  emr_status t_rc[PackBuffers::kTasks];
-  int32_t t_bad[PackBuffers::kTasks];
-  std::vector<PackNode>* t_nodes = B.nodes;
-  std::vector<PackEdge>* t_edges = B.edges;
-  auto g_lo = [&](int t) { return int(int64_t(P) * t / n_threads); };
-  auto work = [&](int t) {
-    Scratch& scratch = B.scratch[t];
-    t_rc[t] = EMR_OK;
-    t_bad[t] = -1;
-    t_nodes[t].clear();
-    t_edges[t].clear();
-    const int64_t n_lo = node_ptr[g_lo(t)], n_hi = node_ptr[g_lo(t + 1)];
-    t_nodes[t].reserve(size_t(std::max<int64_t>(0, n_hi - n_lo)));
-    for (int g = g_lo(t); g < g_lo(t + 1); g++) {
-      emr_status rc = EMR_OK;
-      if (node_ptr[g + 1] < node_ptr[g] || conn_ptr[g + 1] < conn_ptr[g]) rc = EMR_ERR_ARG;
-      if (rc == EMR_OK)
-        rc = pack_one(node_ptr[g], node_ptr[g + 1], conn_ptr[g], conn_ptr[g + 1], node_id, node_kind, node_act,
-                      node_bias, conn_src, conn_dst, conn_w, conn_enabled, scratch, t_nodes[t], t_edges[t], &gs[g]);
-      if (rc != EMR_OK) {
-        t_rc[t] = rc;
-        t_bad[t] = g;
-        return;
-      }
-    }
-  };
-  if (n_threads == 1) {
-    work(0);
-  } else {
-    WorkerPool::get().run(n_threads, work);
-  }
-  for (int t = 0; t < n_threads; t++)
-    if (t_rc[t] != EMR_OK) {
-      if (bad_genome) *bad_genome = t_bad[t];
-      return t_rc[t];
-    }
-  size_t nn = 0, ne = 0;
-  std::vector<size_t> t_nb(n_threads), t_eb(n_threads);  // each thread's first node / edge in the blob
-  for (int t = 0; t < n_threads; t++) {
-    t_nb[t] = nn;
-    t_eb[t] = ne;
-    nn += t_nodes[t].size();
-    ne += t_edges[t].size();
-  }
+  // Layout: genome g's node records start at node index node_ptr[g] - node_ptr[0] and its edge
+  // records at conn_ptr[g] - conn_ptr[0] (room for all its input nodes and connections; the
+  // unused rest is zeroed), so every genome packs straight into the blob, independently.
+  const int64_t nn = node_ptr[P] - node_ptr[0], nc = conn_ptr[P] - conn_ptr[0];
+  if (nn < 0 || nc < 0) return EMR_ERR_ARG;
+  if (nn > int64_t(UINT32_MAX) || nc > int64_t(UINT32_MAX)) return EMR_ERR_RANGE;
   PackHeader h{};
   h.magic = kPackMagic;
   h.version = kPackVersion;
   h.P = P;
   h.off_genomes = align16(sizeof(PackHeader));
   h.off_nodes = h.off_genomes + align16(sizeof(PackGenome) * size_t(P));
-  h.off_edges = h.off_nodes + align16(sizeof(PackNode) * nn);
-  h.total_bytes = h.off_edges + align16(sizeof(PackEdge) * ne);
+  h.off_edges = h.off_nodes + align16(sizeof(PackNode) * size_t(nn));
+  h.total_bytes = h.off_edges + align16(sizeof(PackEdge) * size_t(nc));
   *used = size_t(h.total_bytes);
   if (cap < h.total_bytes) return EMR_ERR_CAPACITY;
   auto* base = static_cast<uint8_t*>(buf);
-  // every record is written in full below; only the alignment gaps between sections are cleared
+  // the genome records, nodes and edges are written below; clear the alignment gaps between sections
   auto clear = [&](uint64_t from, uint64_t to) {
     if (to > from) std::memset(base + from, 0, size_t(to - from));
   };
   clear(sizeof(PackHeader), h.off_genomes);
   clear(h.off_genomes + sizeof(PackGenome) * uint64_t(P), h.off_nodes);
   clear(h.off_nodes + sizeof(PackNode) * uint64_t(nn), h.off_edges);
-  clear(h.off_edges + sizeof(PackEdge) * uint64_t(ne), h.total_bytes);
+  clear(h.off_edges + sizeof(PackEdge) * uint64_t(nc), h.total_bytes);
   auto* gt = reinterpret_cast<PackGenome*>(base + h.off_genomes);
   auto* nt = reinterpret_cast<PackNode*>(base + h.off_nodes);
   auto* et = reinterpret_cast<PackEdge*>(base + h.off_edges);
-  for (int t = 0; t < n_threads; t++) {
-    if (!t_nodes[t].empty()) std::memcpy(nt + t_nb[t], t_nodes[t].data(), t_nodes[t].size() * sizeof(PackNode));
-    if (!t_edges[t].empty()) std::memcpy(et + t_eb[t], t_edges[t].data(), t_edges[t].size() * sizeof(PackEdge));
+  // per-task scratch kept across calls; a caller that finds it in use packs with its own
+  PackBuffers& shared = PackBuffers::get();
+  std::unique_lock<std::mutex> buf_lock(shared.mu, std::try_to_lock);
+  std::unique_ptr<PackBuffers> own;
+  if (!buf_lock.owns_lock()) own.reset(new PackBuffers());
+  PackBuffers& B = own ? *own : shared;
+  // Genomes are independent: host tasks take chunks of kChunk genomes from a shared counter,
+  // each with its own scratch; the lowest failing genome index is reported.
+  constexpr int kChunk = 8;
+  const int n_chunks = (P + kChunk - 1) / kChunk;
+  const int hw = int(std::max(1u, std::thread::hardware_concurrency()));
+  // a task's share costs about as much to hand out as packing a few genomes
+  const int n_tasks = std::max(1, std::min({hw, PackBuffers::kTasks, P / 32}));
+  struct TaskOut {
+    int32_t bad = -1;
+    emr_status rc = EMR_OK;
+    int32_t max_nodes = 0, max_edges = 0, max_varying[2] = {0, 0}, max_vedges[2] = {0, 0};
+  };
+  TaskOut outs[PackBuffers::kTasks];
+  std::atomic<int> next_chunk{0};
+  auto work = [&](int t) {
+    Scratch& scratch = B.scratch[t];
+    TaskOut& o = outs[t];
+    o = TaskOut();
+    for (int c; (c = next_chunk.fetch_add(1, std::memory_order_relaxed)) < n_chunks;) {
+      const int g_end = std::min(P, (c + 1) * kChunk);
+      for (int g = c * kChunk; g < g_end; g++) {
+        emr_status rc = EMR_OK;
+        if (node_ptr[g + 1] < node_ptr[g] || conn_ptr[g + 1] < conn_ptr[g]) rc = EMR_ERR_ARG;
+        const int64_t nb = node_ptr[g] - node_ptr[0], eb = conn_ptr[g] - conn_ptr[0];
+        PackGenome& pg = gt[g];
+        if (rc == EMR_OK)
+          rc = pack_one(node_ptr[g], node_ptr[g + 1], conn_ptr[g], conn_ptr[g + 1], node_id, node_kind, node_act,
+                        node_bias, conn_src, conn_dst, conn_w, conn_enabled, scratch, nt + nb, et + eb, &pg);
+        if (rc != EMR_OK) {
+          if (o.bad < 0 || g < o.bad) {
+            o.bad = g;
+            o.rc = rc;
+          }
+          continue;
+        }
+        pg.node_beg = uint32_t(nb);
+        pg.edge_beg = uint32_t(eb);
+        o.max_nodes = std::max<int32_t>(o.max_nodes, pg.n_nodes);
+        o.max_edges = std::max<int32_t>(o.max_edges, pg.n_edges);
+        for (int sd = 0; sd < 2; sd++) {
+          o.max_varying[sd] = std::max<int32_t>(o.max_varying[sd], pg.n_varying[sd]);
+          o.max_vedges[sd] = std::max<int32_t>(o.max_vedges[sd], pg.n_vedges[sd]);
+        }
+      }
+    }
+  };
+  if (n_tasks == 1) {
+    work(0);
+  } else {
+    WorkerPool::get().run(n_tasks, work);
   }
-  for (int t = 0; t < n_threads; t++)
-    for (int g = g_lo(t); g < g_lo(t + 1); g++) {
-      gs[g].g.node_beg += uint32_t(t_nb[t]);
-      gs[g].g.edge_beg += uint32_t(t_eb[t]);
+  int32_t bad = -1;
+  emr_status bad_rc = EMR_OK;
+  for (int t = 0; t < n_tasks; t++) {
+    const TaskOut& o = outs[t];
+    if (o.bad >= 0 && (bad < 0 || o.bad < bad)) {
+      bad = o.bad;
+      bad_rc = o.rc;
     }
-  for (int g = 0; g < P; g++) {
-    const PackGenome pg = gs[g].g;
-    gt[g] = pg;
-    h.max_nodes = std::max<int32_t>(h.max_nodes, pg.n_nodes);
-    h.max_edges = std::max<int32_t>(h.max_edges, pg.n_edges);
-    for (int s = 0; s < 2; s++) {
-      h.max_varying[s] = std::max<int32_t>(h.max_varying[s], pg.n_varying[s]);
-      h.max_vedges[s] = std::max<int32_t>(h.max_vedges[s], pg.n_vedges[s]);
+    h.max_nodes = std::max(h.max_nodes, o.max_nodes);
+    h.max_edges = std::max(h.max_edges, o.max_edges);
+    for (int sd = 0; sd < 2; sd++) {
+      h.max_varying[sd] = std::max(h.max_varying[sd], o.max_varying[sd]);
+      h.max_vedges[sd] = std::max(h.max_vedges[sd], o.max_vedges[sd]);
     }
+  }
+  if (bad >= 0) {
+    if (bad_genome) *bad_genome = bad;
+    return bad_rc;
   }
   std::memcpy(base, &h, sizeof h);
   return EMR_OK;

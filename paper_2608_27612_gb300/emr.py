@@ -720,12 +720,14 @@ _EDGE = np.dtype([("src", "<u2"), ("reserved", "<u2"), ("w", "<f4")])
 
 
 def pack_records(pack: np.ndarray):
-    """(header, genome table, node records, edge records) of a packed blob, as numpy views."""
+    """(header, genome table, node records, edge records) of a packed blob, as numpy views. The node
+    and edge arrays are the blob's whole sections: genome g's records start at its node_beg and
+    edge_beg (the slots past its n_nodes and n_edges are zero)."""
     raw = np.ascontiguousarray(pack).tobytes()
     h = np.frombuffer(raw[:_HDR.itemsize], _HDR)[0]
     P = int(h["P"])
     gs = np.frombuffer(raw, _GEN, P, int(h["off_genomes"]))
-    nn = int(gs["n_nodes"].astype(np.int64).sum())
-    ne = int(gs["n_edges"].astype(np.int64).sum())
+    nn = (int(h["off_edges"]) - int(h["off_nodes"])) // _NODE.itemsize
+    ne = (int(h["total"]) - int(h["off_edges"])) // _EDGE.itemsize
     return h, gs, np.frombuffer(raw, _NODE, nn, int(h["off_nodes"])), np.frombuffer(raw, _EDGE, ne,
                                                                                     int(h["off_edges"]))

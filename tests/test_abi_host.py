@@ -136,6 +136,7 @@ def test_pack_merges_parallel_connections_and_drops_zero_weights():
     g = gs[0]
     assert g["n_nodes"] == 3 and g["n_edges"] == 2  # 6, 8, out; edges 6 -> out, 8 -> out
     _, _, _, ed = emr.pack_records(blob)
+    ed = ed[int(g["edge_beg"]):int(g["edge_beg"]) + int(g["n_edges"])]
     assert sorted(float(e["w"]) for e in ed) == [0.75, 1.0]
     # OUT side: 6 joint (x2, y2), 8 y only (its x2 inputs cancel), the output joint
     assert [int(a) & 3 for a in nd["axes"]] == [3, 2, 3]

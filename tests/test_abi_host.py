@@ -305,6 +305,26 @@ def test_pack_release_joins_workers_and_the_next_pack_is_identical():
     assert np.array_equal(first, again) and tasks() == with_pool
 
 
+def test_pack_writes_every_byte_and_each_genome_in_its_own_slot():
+    """The blob's bytes do not depend on what the buffer held before (every byte written: records,
+    zeroed slot tails, section gaps), and each genome's records start at its input's offsets
+    (node_ptr[g] - node_ptr[0], conn_ptr[g] - conn_ptr[0]) with room for its input (host only)."""
+    w = W.c2(D=5)
+    n = emr.pack_size(w.pop)
+    a = emr.pack_population(w.pop, out=np.zeros(n, np.uint8)).copy()
+    b = emr.pack_population(w.pop, out=np.full(n, 0xA5, np.uint8)).copy()
+    assert len(a) <= n and np.array_equal(a, b)
+    h, gs, nodes, edges = emr.pack_records(a)
+    nptr, cptr = np.asarray(w.pop.node_ptr), np.asarray(w.pop.conn_ptr)
+    assert np.array_equal(gs["node_beg"], nptr[:-1] - nptr[0])
+    assert np.array_equal(gs["edge_beg"], cptr[:-1] - cptr[0])
+    assert np.all(gs["n_nodes"] <= np.diff(nptr)) and np.all(gs["n_edges"] <= np.diff(cptr))
+    used_n = np.zeros(len(nodes), bool)
+    for g in range(int(h["P"])):
+        used_n[int(gs["node_beg"][g]):int(gs["node_beg"][g]) + int(gs["n_nodes"][g])] = True
+    assert not nodes[~used_n].view(np.uint8).any()  # the slots' unused records are zero
+
+
 def test_grid_chunks_cover_the_grid_in_whole_tiles():
     """emr_grid_chunk: chunks in ascending global index, contiguous, covering [0, N_total), every
     boundary but the first a 64 x 64 tile boundary past depth 4, the same count emr_stream uses."""

@@ -477,8 +477,8 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
   uint2* ve = staged ? s_ve[wid] : ve_g;
   int nv = 0, nve = 0;
   int32_t hdr3 = 0;
-  if (lane == 0) {  // the node loop is sequential (each node folds the constants of its sources)
-    int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
+  {
+    const int64_t si = q.per_genome ? int64_t(g) * q.S + s : s;
     const int side = q.side[si] ? 1 : 0;
     const float a = q.a[si], b = q.b[si];
     float in[5] = {0.f, 0.f, 0.f, 0.f, 1.f};
@@ -486,40 +486,16 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
     if (side == EMR_SIDE_OUT) { in[EMR_KIND_X1] = a; in[EMR_KIND_Y1] = b; gx = EMR_KIND_X2; gy = EMR_KIND_Y2; }
     else { in[EMR_KIND_X2] = a; in[EMR_KIND_Y2] = b; gx = EMR_KIND_X1; gy = EMR_KIND_Y1; }
     float* cval = G.n_nodes <= kSpecSmemNodes ? s_cval[wid] : scratch + r * scratch_stride;
+    const int n = G.n_nodes;
+    const uint32_t vbit = 1u << side;
+    // The constants: the nodes that do not vary, in topological order (each folds its sources'
+    // values), by lane 0. A node that does not vary has no varying source.
     float out_const = 0.f;
-    uint32_t xm = 0, ym = 0;
-    int nj = 0;
-    for (int t = 0; t < G.n_nodes; t++) {
-      const PackNode nd = NS[t];
-      const PackEdge* ed = ES + nd.edge_beg;
-      if (nd.vary & (1u << side)) {
-        const uint32_t ax = (uint32_t(nd.axes) >> (2 * side)) & 3u;
-        float c0 = nd.bias;
-        for (int k = 0; k < 5; k++)
-          if (k != gx && k != gy) c0 = fmaf(nd.w_in[k], in[k], c0);
-        int eb = nve;
-        for (int e = 0; e < nd.edge_cnt; e++) {
-          const PackNode& src = NS[ed[e].src];
-          if (src.vary & (1u << side)) {
-            const uint32_t sa = (uint32_t(src.axes) >> (2 * side)) & 3u;
-            ve[nve++] = make_uint2(__float_as_uint(cval[ed[e].src]) | (sa << 16), __float_as_uint(ed[e].w));
-          } else {
-            c0 = fmaf(ed[e].w, cval[ed[e].src], c0);
-          }
-        }
-        for (int e = eb + 1; e < nve; e++) {  // ascending (source axes, slot) (insertion sort, a few edges)
-          const uint2 key = ve[e];
-          int f = e - 1;
-          while (f >= eb && ve[f].x > key.x) { ve[f + 1] = ve[f]; f--; }
-          ve[f + 1] = key;
-        }
-        uint32_t info = uint32_t(nd.act) | (ax << 4) | (uint32_t(eb) << 8) | (uint32_t(nve - eb) << 20);
-        coef[nv] = make_float4(c0, nd.w_in[gx], nd.w_in[gy], __uint_as_float(info));
-        cval[t] = __uint_as_float(uint32_t(nv));
-        if (ax == kAxisXY) nj++;
-        else if (nv < kDenseMax) (ax == kAxisX ? xm : ym) |= 1u << nv;
-        nv++;
-      } else {
+    if (lane == 0) {
+      for (int t = 0; t < n; t++) {
+        const PackNode nd = NS[t];
+        if (nd.vary & vbit) continue;
+        const PackEdge* ed = ES + nd.edge_beg;
         float z = nd.bias;
         for (int k = 0; k < 5; k++) z = fmaf(nd.w_in[k], in[k], z);
         for (int e = 0; e < nd.edge_cnt; e++) z = fmaf(ed[e].w, cval[ed[e].src], z);
@@ -527,17 +503,85 @@ __global__ void __launch_bounds__(32 * kSpecWarps) spec_kernel(const uint8_t* __
         out_const = cval[t];
       }
     }
-    hdr[0] = nv;
-    hdr[1] = nve;
-    reinterpret_cast<float*>(hdr)[2] = out_const;
+    // the varying nodes' record indices (their order among the varying nodes), in their value
+    // slots, by the warp
+    for (int t0 = 0; t0 < n; t0 += 32) {
+      const int t = t0 + lane;
+      const bool v = t < n && (NS[t].vary & vbit);
+      const uint32_t bal = __ballot_sync(kFull, v);
+      if (v) cval[t] = __uint_as_float(uint32_t(nv + __popc(bal & ((1u << lane) - 1u))));
+      nv += __popc(bal);
+    }
+    __syncwarp();  // lane 0's constants and every record index are visible to the warp
+    // Each varying node's record, by its lane: the constant part of its input (the inputs of
+    // fixed value, then its sources that do not vary, in edge order) and its edges from varying
+    // sources, ascending (source axes, source index); edge offsets by a warp scan.
+    uint32_t xm = 0, ym = 0;
+    int nj = 0, k0 = 0;
+    for (int t0 = 0; t0 < n; t0 += 32) {
+      const int t = t0 + lane;
+      const bool v = t < n && (NS[t].vary & vbit);
+      PackNode nd{};
+      int cnt = 0;
+      if (v) {
+        nd = NS[t];
+        const PackEdge* ed = ES + nd.edge_beg;
+        for (int e = 0; e < nd.edge_cnt; e++) cnt += (NS[ed[e].src].vary & vbit) ? 1 : 0;
+      }
+      int incl = cnt;  // inclusive warp scan of the edge counts
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += u;
+      }
+      const int total = __shfl_sync(kFull, incl, 31);
+      const int eb = nve + incl - cnt;
+      const uint32_t bal = __ballot_sync(kFull, v);
+      const int slot = k0 + __popc(bal & ((1u << lane) - 1u));
+      const uint32_t ax = v ? (uint32_t(nd.axes) >> (2 * side)) & 3u : 0u;
+      if (v) {
+        float c0 = nd.bias;
+        for (int k = 0; k < 5; k++)
+          if (k != gx && k != gy) c0 = fmaf(nd.w_in[k], in[k], c0);
+        const PackEdge* ed = ES + nd.edge_beg;
+        int ne = eb;
+        for (int e = 0; e < nd.edge_cnt; e++) {
+          const PackNode& src = NS[ed[e].src];
+          if (src.vary & vbit) {
+            const uint32_t sa = (uint32_t(src.axes) >> (2 * side)) & 3u;
+            ve[ne++] = make_uint2(__float_as_uint(cval[ed[e].src]) | (sa << 16), __float_as_uint(ed[e].w));
+          } else {
+            c0 = fmaf(ed[e].w, cval[ed[e].src], c0);
+          }
+        }
+        for (int e = eb + 1; e < ne; e++) {  // (insertion sort, a few edges)
+          const uint2 key = ve[e];
+          int f = e - 1;
+          while (f >= eb && ve[f].x > key.x) { ve[f + 1] = ve[f]; f--; }
+          ve[f + 1] = key;
+        }
+        const uint32_t info = uint32_t(nd.act) | (ax << 4) | (uint32_t(eb) << 8) | (uint32_t(cnt) << 20);
+        coef[slot] = make_float4(c0, nd.w_in[gx], nd.w_in[gy], __uint_as_float(info));
+      }
+      nj += __popc(__ballot_sync(kFull, ax == kAxisXY));
+      const bool dense_slot = slot < kDenseMax;
+      xm |= __reduce_or_sync(kFull, ax == kAxisX && dense_slot ? 1u << slot : 0u);
+      ym |= __reduce_or_sync(kFull, ax == kAxisY && dense_slot ? 1u << slot : 0u);
+      nve += total;
+      k0 += __popc(bal);
+    }
+    out_const = __shfl_sync(kFull, out_const, 0);
     hdr3 = int32_t(pair_class(nv, nj) |
                    (nv <= kDenseMax ? uint32_t(nj) << kHdrJointShift | xm << kHdrXShift | ym << kHdrYShift : 0u));
-    hdr[3] = hdr3;
+    if (lane == 0) {
+      hdr[0] = nv;
+      hdr[1] = nve;
+      reinterpret_cast<float*>(hdr)[2] = out_const;
+      hdr[3] = hdr3;
+    }
   }
-  nv = __shfl_sync(0xffffffffu, nv, 0);
-  nve = __shfl_sync(0xffffffffu, nve, 0);
-  const uint32_t h3 = __shfl_sync(0xffffffffu, uint32_t(hdr3), 0);
-  __syncwarp();  // lane 0's coefficient and edge records are visible to the warp
+  const uint32_t h3 = uint32_t(hdr3);
+  __syncwarp();  // the lanes' coefficient and edge records are visible to the warp
   if (staged) {
     for (int k = lane; k < nv; k += 32) coef_g[k] = coef[k];
     for (int k = lane; k < nve; k += 32) ve_g[k] = ve[k];

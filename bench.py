@@ -300,8 +300,8 @@ def roofline_entry(emr, dsc, g, sms, probe, tile_s):
                                          "measured FFMA:MUFU ratio %.2f" % ratio,
             "fp32_ops_per_query_executed": float(work[..., 0].mean()),
             "mufu_ops_per_query_executed": float(work[..., 1].mean()),
-            "kernel": "tile kernels of emr_eval_filter_tiles (tile_kernel_warp, tile_kernel_dense, "
-                      "tile_kernel_one_axis)", "kernel_ms": tile_s * 1e3,
+            "kernel": "tile kernels of emr_eval_filter_tiles (tile_kernel_pyramid, tile_kernel_warp, "
+                      "tile_kernel_one_axis; tile_kernel_dense up to depth 5)", "kernel_ms": tile_s * 1e3,
             "peak_basis": "%d SMs x %d FP32 lanes x %.0f MHz (max SM clock, nominal unit counts)"
                           % (sms, FP32_PER_SM_CLK, SM_MAX_MHZ)}
 
@@ -850,9 +850,11 @@ def main():
     tile_s = statistics.mean(tile_ms) / 1e3
     roofline = roofline_entry(emr, dsc, g, sms, probe, tile_s)
     roofline["traffic"] = profiled_traffic() if args.pop == 1000 and args.depth == 7 else None
-    roofline["traffic_note"] = ("DRAM bytes of the dense tile launches per step, from profiles/"
+    roofline["traffic_note"] = ("DRAM bytes of the tile launches per step, from profiles/"
                                 "tile_kernels_c2_pop300_d7.md (300-genome capture scaled by pairs, x10/3); null "
                                 "when the kernel source changed since")
+    roofline["kernel_ms_source"] = ("CUDA events around emr_eval_filter_tiles in the phase pass right after the "
+                                    "timed region (same inputs, L2 flushed before each step, same clocks sampled)")
     roofline["alu_probe"] = probe
     if clocks:
         roofline["frac_at_sampled_clock"] = roofline["frac"] * SM_MAX_MHZ / clocks["sm_mhz"]

@@ -2990,9 +2990,10 @@ cudaError_t launch_overlapped(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
-// Dense tiles the block kernel takes in fused mode (the rest run a warp per tile): the
-// depths 0..4 tile, and at depth 5 also the grid's one 64 x 64 tile (a warp launch of one
-// tile per pair would leave three of a CTA's four warps idle).
+// Dense tiles a CTA-wide launch takes in fused mode (tile_kernel_pyramid, or the block kernel
+// tile_kernel_dense; the rest run a warp per tile): the depths 0..4 tile, and at depth 5 also
+// the grid's one 64 x 64 tile, on the block kernel (a warp launch of one tile per pair would
+// leave three of a CTA's four warps idle).
 inline int32_t block_tiles(int64_t n_dense) { return n_dense == 2 ? 2 : 1; }
 
 template <int NJMAX>
@@ -3049,8 +3050,10 @@ emr_status launch_warp(const DTileArgs& A0, int64_t rank_beg, int64_t n_ranks, c
   return cuda_status(cudaGetLastError());
 }
 
-// A class of pairs with joint nodes: in fused mode without an output buffer the
-// depths 0..4 tile through tile_kernel_dense and the 64 x 64 tiles a warp each.
+// A class of pairs with joint nodes, tiles [D.tile_beg, D.tile_beg + D.n_tiles): in fused
+// mode without an output buffer the depths 0..4 tile through tile_kernel_dense and the
+// 64 x 64 tiles a warp each (launch_tiles itself gives a full range's depths 0..4 tiles to
+// one tile_kernel_pyramid launch); otherwise all through tile_kernel_dense.
 template <int NJMAX>
 emr_status launch_joint_class(const DTileArgs& D, int64_t rank_beg, int64_t n_ranks, cudaStream_t st,
                               bool* overlap, bool warp_tiles) {
@@ -3205,11 +3208,11 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
   const bool one_fused = mode == kModeFused && !out && n_one > 0;
   bool one_tile0_done = false;
   if (warp_tiles && D.tile_beg < bt && D.tile_beg + D.n_tiles > bt) {
-    // the depths 0..4 tile of every pair in one block launch (the 12-joint class in one of
-    // its own), then every class's warp launch (depths 5..D): the block kernel's
-    // latency-bound CTAs share the SMs with the warp launches that follow. The pairs of up
-    // to 8 joint nodes and the one-coordinate pairs are consecutive ranks; one launch of
-    // the 8-joint kernel for all of them measured faster than a launch per class.
+    // the depths 0..4 tile of every pair in one tile_kernel_pyramid launch (the 12-joint
+    // class in one of its own), then every class's warp launch (depths 5..D): the pyramid
+    // kernel's latency-bound CTAs share the SMs with the warp launches that follow. The
+    // pairs of up to 8 joint nodes and the one-coordinate pairs are consecutive ranks; one
+    // launch of the 8-joint kernel for all of them measured faster than a launch per class.
     DTileArgs D0 = D, D1 = D;
     D0.n_tiles = bt - D.tile_beg;
     D1.tile_beg = bt;
@@ -3241,8 +3244,8 @@ emr_status launch_tiles(const EvalPlan& p, const emr_grid* g, const uint8_t* spe
     }
   }
   if (one_fused) {
-    // one-coordinate outputs: the depths 0..4 tile through the generic kernel (unless the
-    // joint classes' block launch took it), the 64 x 64 tiles (depths 5..D) a warp each
+    // one-coordinate outputs: the depths 0..4 tile through the block kernel (unless the
+    // pyramid launch took it), the 64 x 64 tiles (depths 5..D) a warp each
     const int64_t n5 = n_one;
     const int32_t split_at = std::min<int32_t>(tr.end, block_tiles(n_dense));
     if (tr.beg < split_at && !one_tile0_done) {

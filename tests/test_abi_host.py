@@ -325,6 +325,33 @@ def test_pack_writes_every_byte_and_each_genome_in_its_own_slot():
     assert not nodes[~used_n].view(np.uint8).any()  # the slots' unused records are zero
 
 
+def test_pack_from_several_threads_at_once_gives_the_sequential_blobs():
+    """emr_pack_population called from several host threads at once (ctypes releases the GIL):
+    one call gets the worker pool and the shared scratch, the others pack on their own; every
+    result equals the blob of a call made alone, back-to-back calls included (host only)."""
+    import threading
+    pops = [W.c2(D=5).pop, W.c3(D=6).pop, W.c4_round1().pop, W.random_population(300, seed=4)]
+    ref = [emr.pack_population(p).copy() for p in pops]
+    out = [[None] * 6 for _ in pops]
+    errs = []
+
+    def run(i):
+        try:
+            for k in range(6):
+                out[i][k] = emr.pack_population(pops[i]).copy()
+        except Exception as e:  # noqa: BLE001 - reported below
+            errs.append(e)
+
+    ts = [threading.Thread(target=run, args=(i,)) for i in range(len(pops))]
+    for t in ts:
+        t.start()
+    for t in ts:
+        t.join()
+    assert not errs
+    for i in range(len(pops)):
+        assert all(np.array_equal(o, ref[i]) for o in out[i])
+
+
 def test_grid_chunks_cover_the_grid_in_whole_tiles():
     """emr_grid_chunk: chunks in ascending global index, contiguous, covering [0, N_total), every
     boundary but the first a 64 x 64 tile boundary past depth 4, the same count emr_stream uses."""

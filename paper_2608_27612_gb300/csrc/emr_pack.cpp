@@ -183,6 +183,7 @@ int act_cost(int a) {
 struct Edge {
   int s, d;
   float w;
+  int ord;  // position among the genome's enabled connections (the large-genome merge restores it)
 };
 
 // Buffers reused across genomes (capacity kept; no allocation per genome once warm).
@@ -309,15 +310,18 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
     }
     S.es.resize(m);
   } else {
+    for (size_t k = 0; k < S.es.size(); k++) S.es[k].ord = int(k);
     std::stable_sort(S.es.begin(), S.es.end(),
                      [](const Edge& a, const Edge& b) { return a.d != b.d ? a.d < b.d : a.s < b.s; });
     size_t m = 0;
     for (size_t k = 0; k < S.es.size();) {
-      Edge e = S.es[k++];
+      Edge e = S.es[k++];  // the first occurrence: the sort is stable
       while (k < S.es.size() && S.es[k].s == e.s && S.es[k].d == e.d) e.w += S.es[k++].w;
       S.es[m++] = e;
     }
     S.es.resize(m);
+    // back to the order of first occurrence, the order the path above keeps
+    std::sort(S.es.begin(), S.es.end(), [](const Edge& a, const Edge& b) { return a.ord < b.ord; });
   }
   S.es.erase(std::remove_if(S.es.begin(), S.es.end(), [](const Edge& e) { return e.w == 0.f; }), S.es.end());
   S.reach.assign(n, 0);
@@ -426,7 +430,8 @@ emr_status pack_one(int64_t n0, int64_t n1, int64_t c0, int64_t c1, const int32_
       S.in_cnt[t]++;
     }
   }
-  // in-edges from kept non-input nodes, grouped by destination (ascending source)
+  // in-edges from kept non-input nodes, grouped by destination (each group in the order of
+  // the edges' first connections)
   S.in_beg.assign(nk + 1, 0);
   for (int t = 0; t < nk; t++) S.in_beg[t + 1] = S.in_beg[t] + S.in_cnt[t];
   if (S.in_beg[nk] > 65535) return EMR_ERR_RANGE;

@@ -352,6 +352,34 @@ def test_pack_from_several_threads_at_once_gives_the_sequential_blobs():
         assert all(np.array_equal(o, ref[i]) for o in out[i])
 
 
+def test_pack_large_and_small_genome_paths_agree():
+    """Genomes of up to 64 nodes take the packer's bit-mask Kahn order and reachability, larger ones
+    the adjacency-list path. The same genomes with 60 isolated hidden nodes added (interleaved ids;
+    isolated nodes never reach the output, and Kahn's smallest-id order of the other nodes is
+    unchanged by them) go through the large path and must give the same records (host only)."""
+    base = W.random_population(200, seed=11)
+    padded = []
+    for g in range(base.P):
+        nodes, conns = base.genome(g)
+        top = max(i for i, _, _, _ in nodes)
+        extra = [(top + 1 + 2 * k if k % 2 else -(k + 1), W.KIND_HIDDEN, W.ACT_SIGMOID, 0.5) for k in range(60)]
+        padded.append((nodes + extra, conns))
+    pop_pad = W.population_from_lists(padded)
+    a, b = emr.pack_population(base), emr.pack_population(pop_pad)
+    ha, ga, na, ea = emr.pack_records(a)
+    hb, gb, nb, eb = emr.pack_records(b)
+    assert int(W.np.diff(pop_pad.node_ptr).min()) > 64
+    for f in ("max_nodes", "max_varying", "max_vedges", "max_edges"):
+        assert W.np.array_equal(ha[f], hb[f])
+    for g in range(base.P):
+        for f in ("n_nodes", "n_edges", "n_varying", "n_vedges", "cost", "n_joint"):
+            assert W.np.array_equal(ga[g][f], gb[g][f]), (g, f)
+        x0, x1, n = int(ga[g]["node_beg"]), int(gb[g]["node_beg"]), int(ga[g]["n_nodes"])
+        assert na[x0:x0 + n].tobytes() == nb[x1:x1 + n].tobytes()
+        y0, y1, m = int(ga[g]["edge_beg"]), int(gb[g]["edge_beg"]), int(ga[g]["n_edges"])
+        assert ea[y0:y0 + m].tobytes() == eb[y1:y1 + m].tobytes()
+
+
 def test_grid_chunks_cover_the_grid_in_whole_tiles():
     """emr_grid_chunk: chunks in ascending global index, contiguous, covering [0, N_total), every
     boundary but the first a 64 x 64 tile boundary past depth 4, the same count emr_stream uses."""
